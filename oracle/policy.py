@@ -1,0 +1,140 @@
+"""Next-use estimate, eviction eligibility and victim order (Section 5.1).
+
+Victim order, two formulations that must agree exactly:
+  A (``order_global``): every eligible HBM-resident block, sorted by
+    (T_next descending, session id ascending, block id descending).
+  B (``order_scan``): the paper's procedure -- order eligible sessions by
+    decreasing T_next, take blocks from the farthest session, suffix blocks
+    first, then continue with the next session.
+
+Readings:
+  * Ties in T_next are broken by session id ascending; within a session the
+    suffix-first rule (Section 5.1, last paragraph) orders blocks by
+    decreasing block id.  ``ASCENDING`` orders them by increasing block id
+    instead (the literal "(session id, block id) ascending" tie-break).
+  * T_next is clamped to [0, 2^32 - 1] microseconds; the estimate "need not
+    be an exact wall-clock prediction" (Section 5.1).
+  * T_play in the progress-counter mode is the current reply's length in
+    units times ``unit_us`` while the reply is unfinished, else 0 ("longer
+    unfinished responses" mean later reuse, Section 5.1).
+  * Protection holds against *normal* eviction only (Section 5.1), and warmed
+    KV may be "evicted before reuse" (Section 5.2).  With ``fallback`` set (a
+    foreground turn that cannot otherwise run), protected sessions that are
+    not running form a second tier, ordered by the same rule after every
+    normally eligible block.  Pinned running KV is never a candidate.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+from .sessions import (SessionState, RUNNING, IMMEDIATE, RESP_OPEN, MODE_PLAYBACK,
+                       MODE_COUNTERS)
+
+KEY_MAX = 2**32 - 1
+SUFFIX_FIRST = 0
+ASCENDING = 1
+
+
+def t_next(st: SessionState, mode: int, reply_prior_us: int, unit_us: int) -> int:
+    """Eq. 4: T_next = T_play + T_reply for one session (clamped to 32 bits)."""
+    if mode == MODE_PLAYBACK:
+        t_play = max(0, st.gen_us - st.play_us)            # remaining playback horizon
+    elif mode == MODE_COUNTERS:
+        t_play = st.reply_tokens * unit_us if (st.flags & RESP_OPEN) else 0
+    else:
+        raise ValueError(f"unknown T_play mode {mode}")
+    # per-session moving average when available, workload-level prior otherwise
+    t_reply = st.reply_ema_us if st.reply_n > 0 else reply_prior_us
+    return min(KEY_MAX, max(0, t_play + t_reply))
+
+
+next_use_key = t_next
+
+
+def is_eligible(st: SessionState, now_us: int) -> bool:
+    """Only idle-resident multi-turn KV may be evicted (Section 5.1, Eviction policy):
+    pinned running KV, immediate-reuse sessions (speech start / barge-in) and
+    preload-protected sessions (Section 5.2) are excluded."""
+    if st.flags & (RUNNING | IMMEDIATE):
+        return False
+    if now_us < st.protect_until_us:
+        return False
+    return True
+
+
+def tier(st: SessionState, now_us: int, fallback: bool):
+    """0: normally eligible; 1: protected, a candidate only with ``fallback``; None: never."""
+    if is_eligible(st, now_us):
+        return 0
+    if fallback and not (st.flags & RUNNING):
+        return 1
+    return None
+
+
+def _resident_blocks(table_row: np.ndarray, nblocks: int) -> np.ndarray:
+    row = table_row[:nblocks]
+    return np.nonzero(row >= 0)[0]
+
+
+def order_global(tables, nblocks, sessions, now_us, mode, reply_prior_us, unit_us,
+                 within=SUFFIX_FIRST, fallback=False):
+    """Formulation A. Returns int64 arrays (sid, blk, page) of the full victim order."""
+    sids, blks, keys, tiers = [], [], [], []
+    for s, st in enumerate(sessions):
+        tr = tier(st, now_us, fallback)
+        if tr is None:
+            continue
+        b = _resident_blocks(tables[s], int(nblocks[s]))
+        if b.size == 0:
+            continue
+        sids.append(np.full(b.size, s, dtype=np.int64))
+        blks.append(b.astype(np.int64))
+        keys.append(np.full(b.size, t_next(st, mode, reply_prior_us, unit_us), dtype=np.int64))
+        tiers.append(np.full(b.size, tr, dtype=np.int64))
+    if not sids:
+        z = np.zeros(0, dtype=np.int64)
+        return z, z.copy(), z.copy()
+    sid = np.concatenate(sids)
+    blk = np.concatenate(blks)
+    key = np.concatenate(keys)
+    tr = np.concatenate(tiers)
+    blk_key = -blk if within == SUFFIX_FIRST else blk
+    # np.lexsort sorts by the LAST key first: tier, then -T_next, then sid, then block
+    order = np.lexsort((blk_key, sid, -key, tr))
+    sid, blk = sid[order], blk[order]
+    page = np.asarray(tables)[sid, blk].astype(np.int64)
+    return sid, blk, page
+
+
+def order_scan(tables, nblocks, sessions, now_us, mode, reply_prior_us, unit_us,
+               within=SUFFIX_FIRST, k=None, fallback=False):
+    """Formulation B (the paper's session scan). Returns (sid, blk, page) lists."""
+    elig = []
+    for s, st in enumerate(sessions):
+        tr = tier(st, now_us, fallback)
+        if tr is not None:
+            elig.append((tr, t_next(st, mode, reply_prior_us, unit_us), s))
+    # normal tier first; decreasing T_next; equal T_next by increasing session id
+    elig.sort(key=lambda e: (e[0], -e[1], e[2]))
+    out_s, out_b, out_p = [], [], []
+    for _, _, s in elig:
+        n = int(nblocks[s])
+        rng = range(n - 1, -1, -1) if within == SUFFIX_FIRST else range(n)
+        for b in rng:
+            if k is not None and len(out_s) >= k:
+                return out_s, out_b, out_p
+            e = int(tables[s][b])
+            if e >= 0:
+                out_s.append(s)
+                out_b.append(b)
+                out_p.append(e)
+    return out_s, out_b, out_p
+
+
+def select_victims(tables, nblocks, sessions, now_us, k, mode, reply_prior_us, unit_us,
+                   within=SUFFIX_FIRST, fallback=False):
+    """The first min(k, #candidates) blocks of the victim order."""
+    sid, blk, page = order_global(tables, nblocks, sessions, now_us, mode,
+                                  reply_prior_us, unit_us, within, fallback)
+    k = min(int(k), sid.size)
+    return sid[:k], blk[:k], page[:k]
