@@ -1,0 +1,448 @@
+#!/usr/bin/env python
+"""KV reload/offload throughput of the interaction-aware swap path on GB300.
+
+One step = one turn of the thinker-shaped workload (48 layers, 4 KV heads x
+128, 16-token pages of 1.5 MiB, 64 sessions with log-uniform 2k-16k token
+contexts, 40 GB HBM budget): playback reports for every session, then the
+turn's session is made fully resident -- next-use ranking (census, sort,
+top-k), host-slot allocation, swap-out, commit, HBM-page allocation, swap-in,
+commit.  ``value`` is the payload moved over the host link in both
+directions per second (GB/s, 1e9 B) with every input resident before timing;
+``e2e`` is the same through the C ABI with host buffers (event batches copied
+in, victim / slot / page lists read back every step).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+N > 1 runs N independent replicas (one pool per GPU, one process per GPU, no
+collective on the data path); ``value`` is then the sum over replicas divided
+by the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "KV reload+offload payload GB/s on 1 GB300 (thinker-shaped pages, 40 GB HBM budget)"
+UNIT = "GB/s"
+WORKLOAD = "thinker"
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def aggregate(per_rank_bytes, per_rank_seconds):
+    """Whole-job throughput: all ranks' bytes over the slowest rank's time."""
+    t = max(per_rank_seconds)
+    return (sum(per_rank_bytes) / t) if t > 0 else 0.0
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------- our arm
+class KernelTimer:
+    """CUDA-event brackets around the swap calls, on the launching stream."""
+
+    def __init__(self, torch):
+        self.torch = torch
+        self.pending = {}
+        self.done = {}
+        self.enabled = False
+
+    def start(self, name):
+        if not self.enabled:
+            return
+        e = self.torch.cuda.Event(enable_timing=True)
+        e.record()
+        self.pending[name] = e
+
+    def stop(self, name, nbytes):
+        if not self.enabled:
+            return
+        e = self.torch.cuda.Event(enable_timing=True)
+        e.record()
+        self.done.setdefault(name, []).append((self.pending.pop(name), e, nbytes))
+
+    def summary(self):
+        self.torch.cuda.synchronize()
+        out = {}
+        for name, lst in self.done.items():
+            ms = [a.elapsed_time(b) for a, b, _ in lst]
+            nb = [n for _, _, n in lst]
+            out[name] = {"launches": len(lst), "total_ms": sum(ms), "avg_ms": sum(ms) / len(ms),
+                         "bytes_per_launch": sum(nb) / len(nb),
+                         "gbs": (sum(nb) / 1e9) / (sum(ms) / 1e3) if sum(ms) > 0 else 0.0}
+        return out
+
+
+def link_peaks(torch, pool, nbytes, reps=5):
+    """Contiguous page-locked cudaMemcpyAsync of nbytes each way, and both at once."""
+    src = pool.kv.view(-1)[:nbytes]
+    host = torch.from_numpy(pool.host.reshape(-1)[:nbytes])
+    dev2 = torch.empty(nbytes, dtype=torch.uint8, device=pool.device)
+    host2 = torch.from_numpy(pool.host.reshape(-1)[nbytes:2 * nbytes]) \
+        if pool.host.size >= 2 * nbytes else None
+    res = {}
+    for name, fn in (("d2h", lambda: host.copy_(src, non_blocking=True)),
+                     ("h2d", lambda: dev2.copy_(host, non_blocking=True))):
+        best = 1e30
+        for _ in range(reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            b.synchronize()
+            best = min(best, a.elapsed_time(b))
+        res[name] = nbytes / (best / 1e3) / 1e9
+    if host2 is not None:
+        s2 = torch.cuda.Stream()
+        best = 1e30
+        for _ in range(reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            s2.wait_event(a)
+            host.copy_(src, non_blocking=True)
+            with torch.cuda.stream(s2):
+                dev2.copy_(host2, non_blocking=True)
+            torch.cuda.current_stream().wait_stream(s2)
+            b.record()
+            b.synchronize()
+            best = min(best, a.elapsed_time(b))
+        res["bidir"] = 2 * nbytes / (best / 1e3) / 1e9
+    del dev2
+    return res
+
+
+def run_turns(torch, gm, wl, lo, hi, dev_events=None, timer=None):
+    """Turns lo..hi of a turn-driven script; returns payload bytes moved."""
+    from paper_2606_22983_gb300 import lv
+    S = wl.spec.n_sessions
+    moved0 = gm.bytes_moved
+    per_turn = S + 1
+    for i in range(lo, hi):
+        base = i * per_turn
+        t = int(wl.t_us[base])
+        if dev_events is not None:
+            lv.lv_session_events(gm.pool.handle, dev_events[i], S, gm.pool.stream)
+            gm.pool.launches += 1
+        else:
+            ev = np.zeros(S, dtype=lv.EVENT_DTYPE)
+            ev["kind"], ev["sid"], ev["t_us"], ev["a"] = (lv.LV_EV_PLAYBACK, wl.sid[base:base + S],
+                                                          t, wl.a[base:base + S])
+            gm.pool.events(ev)
+        gm.timer = timer
+        gm.step(wl.event(base + S), base + S)
+    return gm.bytes_moved - moved0
+
+
+def ours(args, torch):
+    from paper_2606_22983_gb300 import build, lv
+    build()
+    from paper_2606_22983_gb300.harness import fill_random, pool_for
+    from paper_2606_22983_gb300.manager import KVManager
+    from workloads import make_workload
+
+    ws, rank, local = _dist()
+    torch.cuda.set_device(local)
+    dist = None
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    K, W = args.steps, args.warmup
+    over = {}
+    if args.sessions or args.budget_pages:
+        from workloads import pool_spec
+        sp = pool_spec(WORKLOAD)
+        b = args.budget_pages or sp.hbm_budget_pages
+        over["spec"] = sp.with_(n_sessions=args.sessions or sp.n_sessions, hbm_pages=b,
+                                hbm_budget_pages=b)
+    wl = make_workload(WORKLOAD, args.seed + rank, n_turns=W + 2 * K, **over)
+    pool = pool_for(wl)
+    fill_random(pool, args.seed + rank)
+    page_bytes = pool.J * pool.P
+    gm = KVManager(pool, perms=wl.perms, rank_on="none", mode=args.mode, record=False)
+    timer = KernelTimer(torch)
+    gm.timer = timer
+    S = wl.spec.n_sessions
+    # the PLAYBACK batches of the device-timed pass, resident before timing
+    dev_events = []
+    for i in range(W + K):
+        base = i * (S + 1)
+        ev = np.zeros(S, dtype=lv.EVENT_DTYPE)
+        ev["kind"], ev["sid"], ev["t_us"], ev["a"] = (lv.LV_EV_PLAYBACK, wl.sid[base:base + S],
+                                                      int(wl.t_us[base]), wl.a[base:base + S])
+        dev_events.append(torch.from_numpy(ev.view(np.uint8).copy()).to(pool.device))
+    torch.cuda.synchronize()
+
+    run_turns(torch, gm, wl, 0, W, dev_events)                  # warm-up
+    pool.sync()
+    clocks = ClockSampler(local)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    timer.enabled = True
+    l0 = pool.launches
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    moved = run_turns(torch, gm, wl, W, W + K, dev_events, timer)
+    t1.record()
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    launches = pool.launches - l0
+    clk = clocks.stop()
+    timer.enabled = False
+    dev_s = t0.elapsed_time(t1) / 1e3
+    assert pool.sync(raise_on_error=False) == 0, "device error during the timed turns"
+    kern = timer.summary()
+
+    # e2e: the next K turns through the C ABI with host buffers
+    gm.record = True
+    h2d = d2h = 0
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    moved_e2e = 0
+    for i in range(W + K, W + 2 * K):
+        moved_e2e += run_turns(torch, gm, wl, i, i + 1, None, None)
+        h2d += (S + 2) * lv.EVENT_DTYPE.itemsize
+        d2h += gm.last_readback_bytes
+    e1.record()
+    torch.cuda.synchronize()
+    e2e_s = e0.elapsed_time(e1) / 1e3
+    if dist:
+        tt = torch.tensor([dev_s, e2e_s, moved, moved_e2e], dtype=torch.float64, device="cuda")
+        gathered = [torch.zeros_like(tt) for _ in range(ws)]
+        dist.all_gather(gathered, tt)
+        g = torch.stack(gathered).cpu().numpy()
+        value = aggregate(g[:, 2], g[:, 0]) / 1e9
+        e2e_value = aggregate(g[:, 3], g[:, 1]) / 1e9
+        t_max = float(g[:, 0].max())
+    else:
+        value = moved / dev_s / 1e9
+        e2e_value = moved_e2e / e2e_s / 1e9
+        t_max = dev_s
+
+    line = None
+    if rank == 0:
+        mean_turn = moved / K / 2
+        peaks = link_peaks(torch, pool, int(min(mean_turn, 1 << 30)) // 4096 * 4096)
+        # roofline of the dominant kernel (longest total time)
+        dom = max(kern, key=lambda n: kern[n]["total_ms"])
+        dk = kern[dom]
+        peak = peaks["d2h"] if dom == "swap_out" else peaks["h2d"]
+        traffic = _profiled_traffic(dom, dk["bytes_per_launch"])
+        line = {
+            "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": ws,
+            "steps": K, "warmup": W, "ms_per_step": round(t_max * 1e3 / K, 4),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "u8", "data": "synthetic",
+            "config": {"workload": "thinker: 48 layers, 4 KV heads x 128, bf16, 16-token pages "
+                                   "(1.5 MiB), 64 sessions log-uniform 2k-16k tokens, 40 GB HBM "
+                                   "budget, one turn = evict + reload",
+                       "hbm_budget_pages": wl.spec.hbm_budget_pages, "host_pages": wl.spec.host_pages,
+                       "mode": {0: "auto", 1: "zero_copy", 2: "staged"}[args.mode],
+                       "l2": "inputs larger than L2 (mean turn moves "
+                             f"{mean_turn / 1e6:.0f} MB each way from a 40 GB pool)",
+                       "parallelism": f"replicas x{ws}"},
+            "blocks_per_s": round(moved / page_bytes / t_max, 1),
+            "link_peak_gbs": {k: round(v, 1) for k, v in peaks.items()},
+            "link_frac": round(value / peaks["bidir"], 3) if "bidir" in peaks else None,
+            "roofline": {"kernel": dom, "bound": "host_link", "achieved": round(dk["gbs"], 1),
+                         "peak": round(peak, 1), "unit": "GB/s", "frac": round(dk["gbs"] / peak, 3),
+                         "traffic": traffic,
+                         "peak_source": "same-run contiguous page-locked cudaMemcpyAsync "
+                                        f"({'D2H' if dom == 'swap_out' else 'H2D'}, "
+                                        "mean-turn byte count)"},
+            "kernels": {n: {k: round(v, 3) for k, v in d.items()} for n, d in kern.items()},
+            "e2e": {"value": round(e2e_value, 3), "unit": UNIT,
+                    "h2d_bytes_per_step": int(h2d / K), "d2h_bytes_per_step": int(d2h / K)},
+            "gpu_launches": int(launches),
+            "clocks": clk,
+        }
+    pool.close()
+    if line is not None and args.cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(args.cpu_seconds, args.seed)
+    if dist:
+        dist.destroy_process_group()
+    return line
+
+
+def _profiled_traffic(kernel, bytes_per_launch):
+    """DRAM bytes per launch from the committed ncu summary, when it covers this kernel."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        e = d[kernel]
+        return round(e["dram_bytes_per_payload_byte"] * bytes_per_launch)
+    except (OSError, KeyError, ValueError):
+        return None
+
+
+# ----------------------------------------------------------- the oracle arm
+def _oracle_sample(seed):
+    from workloads import make_workload, pool_spec
+    spec = pool_spec(WORKLOAD).with_(n_sessions=8, hbm_pages=1500, hbm_budget_pages=1500)
+    return make_workload(WORKLOAD, seed, spec=spec, n_turns=400)
+
+
+def cpu_baseline(seconds, seed, steps=None):
+    """The oracle (single thread, numpy memcpy per sub-page) on a bounded sample:
+    thinker-shaped pages, 8 sessions, a 1500-page HBM image, turns until about
+    ``seconds`` of CPU time (or ``steps`` turns)."""
+    from oracle import OracleManager
+    wl = _oracle_sample(seed)
+    om = OracleManager(wl, with_bytes=True, content=None, rank_on="none")
+    om.pool.hbm.fill(1)        # touch the images so that timing excludes first-touch faults
+    om.pool.host.fill(1)
+    S = wl.spec.n_sessions
+    moved, turns = 0, 0
+    t0 = time.perf_counter()
+    i = 0
+    per_turn = S + 1
+    while i + per_turn <= wl.n_events:
+        b0 = om.pool.bytes_out + om.pool.bytes_in
+        for j in range(i, i + per_turn):
+            om.step(j)
+        moved += om.pool.bytes_out + om.pool.bytes_in - b0
+        turns += 1
+        i += per_turn
+        el = time.perf_counter() - t0
+        if (steps is not None and turns >= steps) or (steps is None and el >= seconds):
+            break
+    el = time.perf_counter() - t0
+    return {"value": round(moved / el / 1e9, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{turns} turns of a thinker-shaped pool (8 sessions, 1500-page HBM image, "
+                      f"{wl.spec.host_pages} host slots), {moved / 1e9:.2f} GB moved in {el:.1f} s",
+            "seconds": round(el, 2)}
+
+
+def reference(args):
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return None
+    K, W = args.steps, args.warmup
+    from oracle import OracleManager
+    wl = _oracle_sample(args.seed)
+    om = OracleManager(wl, with_bytes=True, content=None, rank_on="none")
+    om.pool.hbm.fill(1)
+    om.pool.host.fill(1)
+    S = wl.spec.n_sessions
+    per_turn = S + 1
+
+    def turn(i):
+        b0 = om.pool.bytes_out + om.pool.bytes_in
+        for j in range(i * per_turn, (i + 1) * per_turn):
+            om.step(j)
+        return om.pool.bytes_out + om.pool.bytes_in - b0
+
+    for i in range(W):
+        turn(i)
+    t0 = time.perf_counter()
+    moved = sum(turn(i) for i in range(W, W + K))
+    el = time.perf_counter() - t0
+    v = moved / el / 1e9
+    return {"impl": "reference", "metric": METRIC, "value": round(v, 4), "unit": UNIT,
+            "n_gpus": ws, "steps": K, "warmup": W, "ms_per_step": round(el * 1e3 / K, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
+            "data": "synthetic",
+            "config": {"workload": "thinker-shaped pages; the oracle's bounded sample "
+                                   "(8 sessions, 1500-page HBM image)"},
+            "cpu_baseline": {"value": round(v, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": f"{K} turns after {W} warm-up, {moved / 1e9:.2f} GB moved"},
+            "e2e": {"value": round(v, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=40)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--mode", type=int, default=0, help="0 auto, 1 zero-copy, 2 staged")
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
+    ap.add_argument("--sessions", type=int, default=0,
+                    help="smaller case for profiling: number of sessions")
+    ap.add_argument("--budget-pages", type=int, default=0,
+                    help="smaller case for profiling: HBM budget in pages")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    if args.impl == "reference":
+        line = reference(args)
+    else:
+        import torch
+        line = ours(args, torch)
+    if line is not None:
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,314 @@
+/*
+ * lv.h -- C ABI of the interaction-aware KV swap path (liblv.so).
+ *
+ * A pool holds one engine stage's paged KV cache in two tiers: HBM (the
+ * caller's per-layer K and V page arrays) and a page-locked host pool.  The
+ * calls below rank resident blocks by predicted next use (Section 5.1, Eq. 4),
+ * move blocks between the tiers (Section 5, Fig. 6: eviction to DRAM and
+ * loading back, Section 5.2: speech-triggered preload) and commit the moves in
+ * the block tables (Section 6, "Hierarchical KV cache manager": side tables on
+ * sessions and blocks).
+ *
+ * Terms.  T tokens form a page (the paper's KV block); a page of one layer's K
+ * or V is a sub-page of P = T*H*D*elem bytes laid out [T][H][D].  A page is
+ * the allocation and eviction unit: all 2L sub-pages of T tokens share one
+ * page id.  HBM sub-page j = 2*layer + kv (kv 0 = K, 1 = V) of page p lives at
+ * hbm_kv[j] + p*P.  Host slot h holds a page as one contiguous run
+ * [2L][P] at host_kv + h*2L*P.
+ *
+ * Block-table entries: e >= 0 is an HBM page id, e == -1 means "no block",
+ * e <= -2 is host slot -(e + 2).
+ *
+ * Execution model.  Every call is asynchronous and ordered on the stream it
+ * is given; argument checks that need no device data run at once and are the
+ * return value.  Conditions found on the device (a bounds violation, a double
+ * mapping, an exhausted tier) are recorded in a sticky per-pool error word that
+ * lv_sync / lv_get_stats report; the kernels skip the offending item instead of
+ * faulting, and no call traps, aborts or falls back to the CPU.  Nothing in the
+ * library waits on the device except lv_sync, lv_get_stats and the readers
+ * named as synchronous below.
+ *
+ * Pointers.  Array arguments may point to device memory or to host memory.  A
+ * host input is copied to the device in stream order before use (pageable host
+ * memory: before the call returns; page-locked host memory: the caller keeps
+ * it unchanged until the stream reaches the call).  A host output is written
+ * by a copy queued on the stream: read it after the stream has completed.
+ * Calls that allocate from the same tier (swap-out: host slots; swap-in and
+ * append: HBM pages) must be ordered with respect to each other.
+ */
+#ifndef LV_H
+#define LV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef void* lv_stream;            /* a cudaStream_t; NULL = the legacy default stream */
+typedef struct lv_pool lv_pool;     /* opaque */
+
+typedef enum lv_status {
+  LV_OK = 0,
+  LV_ERR_INVALID = 1,     /* bad argument (size, alignment, pointer kind, range) */
+  LV_ERR_OOM = 2,         /* a device or host allocation failed */
+  LV_ERR_CUDA = 3,        /* a CUDA runtime call failed */
+  LV_ERR_NO_HBM = 4,      /* HBM budget exhausted (device-detected) */
+  LV_ERR_NO_HOST = 5,     /* host pool exhausted (device-detected) */
+  LV_ERR_BOUNDS = 6,      /* an index outside the pool (device-detected) */
+  LV_ERR_DOUBLE_MAP = 7,  /* a location or block committed twice (device-detected) */
+  LV_ERR_BUDGET = 8,      /* more HBM pages allocated than the budget (device-detected) */
+  LV_ERR_TIMEOUT = 9,     /* a bounded device wait ran out */
+  LV_ERR_STATE = 10       /* a block is not where the call says it is (device-detected) */
+} lv_status;
+
+#define LV_ALL INT64_MAX             /* lv_select_victims: the whole victim order */
+
+enum { LV_SUFFIX_FIRST = 0, LV_ASCENDING = 1 };        /* lv_pool_desc.within_order */
+enum { LV_PLAY_PLAYBACK = 0, LV_PLAY_COUNTERS = 1 };   /* lv_pool_desc.t_play_mode */
+enum { LV_MODE_AUTO = 0, LV_MODE_ZERO_COPY = 1, LV_MODE_STAGED = 2 };   /* swap modes */
+enum { LV_SELECT_FALLBACK = 1 };                       /* lv_select_victims flags */
+
+/* session flag bits (lv_session_state.flags) */
+enum {
+  LV_RUNNING = 1,      /* the session's request executes: pinned running KV */
+  LV_IMMEDIATE = 2,    /* speech start or barge-in seen: immediate reuse */
+  LV_RESP_OPEN = 4,    /* the current reply is unfinished */
+  LV_DONE_VALID = 8    /* t_done_us holds the completion time of the current reply */
+};
+
+/* monitor events (lv_event.kind) */
+enum {
+  LV_EV_TURN_BEGIN = 1,    /* the turn's request starts running */
+  LV_EV_TURN_END = 2,      /* a = reply audio us, b = reply length in progress units */
+  LV_EV_PLAYBACK = 3,      /* a = further us of the reply reported as played */
+  LV_EV_SPEECH_START = 4,
+  LV_EV_BARGE_IN = 5,      /* speech while the reply plays: unplayed audio discarded */
+  LV_EV_SPEECH_STOP = 6,   /* the user input is complete */
+  LV_EV_PRELOADED = 7      /* a preload completed at t_us: protect the warmed KV */
+};
+
+typedef struct lv_pool_desc {
+  int32_t num_layers;          /* L */
+  int32_t num_kv_heads;        /* H */
+  int32_t head_dim;            /* D */
+  int32_t page_tokens;         /* T */
+  int32_t elem_bytes;          /* bytes per K/V element (2 for bf16) */
+  int32_t max_sessions;        /* S, 1..4096 */
+  int32_t max_blocks;          /* block-table capacity per session, 1..65536 */
+  int32_t within_order;        /* LV_SUFFIX_FIRST (default) or LV_ASCENDING */
+  int64_t hbm_pages;           /* pages in each HBM sub-page array */
+  int64_t hbm_budget_pages;    /* 0 < budget <= hbm_pages: allocated HBM pages at most */
+  int64_t host_pages;          /* host pool slots */
+  void* const* hbm_kv;         /* host array of 2L device pointers, each [hbm_pages][P],
+                                  16-byte aligned; caller-owned, kept alive by the caller */
+  void* host_kv;               /* page-locked host pool [host_pages][2L][P], or NULL: the
+                                  library allocates (and frees) a mapped page-locked pool */
+  int64_t reply_prior_us;      /* workload-level T_reply prior (>= 0) */
+  int64_t protect_us;          /* preload protection window (>= 0) */
+  int64_t unit_us;             /* progress-counter unit, 1..2^31 */
+  int32_t t_play_mode;         /* LV_PLAY_PLAYBACK or LV_PLAY_COUNTERS */
+  int32_t reserved;            /* must be 0 */
+} lv_pool_desc;
+
+/* Per-session interaction state (64 bytes).  ctx_tokens is maintained by
+   lv_pool_import and lv_session_append and ignored by lv_session_set. */
+typedef struct lv_session_state {
+  int32_t ctx_tokens;
+  int32_t flags;               /* LV_RUNNING | LV_IMMEDIATE | LV_RESP_OPEN | LV_DONE_VALID */
+  int64_t gen_us;              /* audio generated for the current reply */
+  int64_t play_us;             /* audio of it reported as played */
+  int64_t t_done_us;           /* completion time of the current reply (if LV_DONE_VALID) */
+  int64_t reply_ema_us;        /* moving average of the reply interval */
+  int32_t reply_n;             /* samples in it (0: the prior applies) */
+  int32_t pad;
+  int64_t reply_tokens;        /* current reply length in progress units */
+  int64_t protect_until_us;    /* preload protection ends at this time */
+} lv_session_state;
+
+typedef struct lv_event {      /* 32 bytes */
+  int32_t kind;                /* LV_EV_* */
+  int32_t sid;
+  int64_t t_us;
+  int64_t a;
+  int64_t b;
+} lv_event;
+
+typedef struct lv_victim {     /* one block chosen for eviction */
+  int32_t sid;
+  int32_t blk;
+  int32_t page;                /* its HBM page */
+} lv_victim;
+
+typedef struct lv_remap_entry {  /* commit block (sid, blk) to location loc (encoded) */
+  int32_t sid;
+  int32_t blk;
+  int32_t loc;
+} lv_remap_entry;
+
+typedef struct lv_stats {
+  int64_t hbm_allocated;       /* HBM pages reserved or owned */
+  int64_t host_allocated;      /* host slots reserved or owned */
+  int64_t hbm_budget_pages;
+  int64_t host_pages;
+  int64_t error;               /* sticky lv_status of the first device-detected error */
+  int64_t error_detail;        /* index of the offending item */
+  int64_t last_select_count;   /* victims written by the last lv_select_victims */
+  int64_t last_select_total;   /* candidates it saw */
+  /* counters ("counters for policy fallbacks and preload outcomes", Section 6) */
+  int64_t selects, victims, shortfalls, pages_out, pages_in, bytes_out, bytes_in;
+  int64_t remap_entries, appended_pages, cancels, events, fallback_selects;
+} lv_stats;
+
+/* ---------------------------------------------------------------- pool */
+
+/* Section 6 ("Hierarchical KV cache manager"): the paged block pool with side
+   tables.  Validates the descriptor, allocates the device metadata (session
+   table, block tables, owner tables, allocation bitmaps, error word and
+   counters) and, when desc->host_kv is NULL, a mapped page-locked host pool.
+   All tables start empty.  Returns LV_ERR_INVALID for a bad descriptor (sizes
+   out of range, P not a multiple of 16, a misaligned or non-device KV pointer,
+   a host_kv that is not page-locked), LV_ERR_OOM or LV_ERR_CUDA. */
+lv_status lv_pool_create(const lv_pool_desc* desc, lv_stream stream, lv_pool** out);
+
+/* Waits for the pool's outstanding work on `stream`, then frees everything the
+   library allocated.  The caller's KV arrays and host pool are not touched. */
+lv_status lv_pool_destroy(lv_pool* pool, lv_stream stream);
+
+/* Host-visible address of the host pool ([host_pages][2L][P]). */
+void* lv_pool_host_ptr(lv_pool* pool);
+
+/* Loads a placement: placement is int32 [max_sessions][max_blocks] of encoded
+   entries, ctx_tokens is int32 [max_sessions].  Block b of session s must be
+   placed (entry != -1) exactly when b < ceil(ctx_tokens[s] / T).  Rebuilds the
+   owner tables, bitmaps and counts.  Device-detected: LV_ERR_DOUBLE_MAP (two
+   blocks on one location), LV_ERR_BOUNDS, LV_ERR_BUDGET. */
+lv_status lv_pool_import(lv_pool* pool, const int32_t* placement, const int32_t* ctx_tokens,
+                         lv_stream stream);
+
+/* ------------------------------------------------------------ sessions */
+
+/* Writes states[0..n) to sessions first..first+n (ctx_tokens is ignored). */
+lv_status lv_session_set(lv_pool* pool, const lv_session_state* states, int32_t first,
+                         int32_t n, lv_stream stream);
+
+/* Reads sessions first..first+n into out (host or device). */
+lv_status lv_session_get(lv_pool* pool, lv_session_state* out, int32_t first, int32_t n,
+                         lv_stream stream);
+
+/* Section 3 (runtime monitor: playback progress, speech activity, barge-in)
+   and Sections 5.1-5.2: applies n events in order to the session table.
+   TURN_BEGIN sets RUNNING, clears IMMEDIATE and the preload protection.
+   TURN_END(a, b) clears RUNNING, starts a reply of a us and b units (LV_RESP_OPEN).
+   PLAYBACK(a) advances play_us by a, at most to gen_us; reaching it ends the
+   reply and records t_done_us.  SPEECH_START sets IMMEDIATE.  BARGE_IN sets
+   gen_us = play_us (unplayed audio discarded), ends the reply without a
+   completion time, sets IMMEDIATE.  SPEECH_STOP clears IMMEDIATE and, when the
+   reply had completed, folds x = t - t_done_us into the reply-interval average
+   (first sample: ema = x; later: ema = floor((3*ema + x) / 4)).  PRELOADED
+   sets protect_until_us = t + protect_us.  Device-detected: LV_ERR_BOUNDS for an
+   unknown kind or session id (that event is skipped). */
+lv_status lv_session_events(lv_pool* pool, const lv_event* events, int64_t n, lv_stream stream);
+
+/* Section 5.1 / Eq. 4 and "Eviction policy": ranks every HBM-resident block of
+   every candidate session by (T_next descending, session id ascending, block
+   id descending -- suffix first; ascending under LV_ASCENDING) and writes the
+   first min(k, capacity, #candidates) to out (lv_victim [capacity]).
+   T_next = T_play + T_reply, clamped to [0, 2^32-1]: T_play = max(0, gen - play)
+   (or reply_tokens * unit_us while the reply is open, in LV_PLAY_COUNTERS mode),
+   T_reply = reply_ema_us if reply_n > 0 else reply_prior_us.  Candidates are
+   sessions that are neither RUNNING nor IMMEDIATE nor protected
+   (now_us < protect_until_us).  With LV_SELECT_FALLBACK, protected sessions
+   that are not RUNNING follow as a second tier, in the same order.  The count
+   written goes to *count_out (int64, host or device; may be NULL); fewer than k
+   candidates is not an error (the count says so) and is counted as a shortfall. */
+lv_status lv_select_victims(lv_pool* pool, int64_t now_us, int64_t k, uint32_t flags,
+                            lv_victim* out, int64_t capacity, int64_t* count_out,
+                            lv_stream stream);
+
+/* ------------------------------------------------------------ movement */
+
+/* Section 5 (Fig. 6, eviction to DRAM) / Section 6 (offload connector):
+   reserves the n lowest-numbered free host slots (ascending, in victim order)
+   and copies every sub-page of each victim's HBM page into its slot.  Does not
+   change the block tables: the victims stay valid until lv_remap commits.
+   slots_out (int32 [n], may be NULL) receives the slots, commit_out
+   (lv_remap_entry [n], may be NULL) ready-to-commit entries.  mode:
+   LV_MODE_ZERO_COPY (SM copies straight into the mapped host pool),
+   LV_MODE_STAGED (pack into HBM staging, then copy-engine transfer) or
+   LV_MODE_AUTO.  Device-detected: LV_ERR_NO_HOST (nothing reserved or copied),
+   LV_ERR_BOUNDS, LV_ERR_STATE (a victim is not resident where it says). */
+lv_status lv_swap_out(lv_pool* pool, const lv_victim* victims, int64_t n, int32_t* slots_out,
+                      lv_remap_entry* commit_out, int32_t mode, lv_stream stream);
+
+/* Section 5.2 (speech-triggered preload) and the synchronous load of Section 6:
+   reserves the n lowest-free HBM pages (ascending, in list order) and copies
+   each listed host-resident block of session sid into its page.  Does not
+   change the block tables.  pages_out (int32 [n]) and commit_out
+   (lv_remap_entry [n]) may be NULL.  A preload is this call on a side stream.
+   Device-detected: LV_ERR_NO_HBM (budget short: nothing reserved or copied),
+   LV_ERR_BOUNDS, LV_ERR_STATE (a block is not in the host tier). */
+lv_status lv_swap_in(lv_pool* pool, int32_t sid, const int32_t* blks, int64_t n,
+                     int32_t* pages_out, lv_remap_entry* commit_out, int32_t mode,
+                     lv_stream stream);
+
+/* Section 6 (side tables) and Section 5.2 ("preloading affects latency but not
+   correctness"): commits n entries.  For each, the new location must be a
+   reservation not yet owned; it becomes owned by (sid, blk), the block table
+   points to it and the old location is freed.  Entries are independent;
+   a bad one is skipped.  Device-detected: LV_ERR_DOUBLE_MAP (location not a
+   free reservation, or the same block twice in one call), LV_ERR_BOUNDS,
+   LV_ERR_BUDGET. */
+lv_status lv_remap(lv_pool* pool, const lv_remap_entry* entries, int64_t n, lv_stream stream);
+
+/* Releases reservations that will never be committed (a cancelled or failed
+   transfer, Section 5.2).  locs are encoded locations.  Device-detected:
+   LV_ERR_STATE when a location is owned or not reserved. */
+lv_status lv_cancel(lv_pool* pool, const int32_t* locs, int64_t n, lv_stream stream);
+
+/* Block-level allocation kept (Section 5.1): grows session sid's context by
+   n_tokens; each new block takes the lowest free HBM page, in block order, and
+   is committed at once.  pages_out (int32, capacity ceil(n_tokens/T)+1, may be
+   NULL) receives the new pages; *count_out (int32, may be NULL) their number.
+   Device-detected: LV_ERR_NO_HBM (nothing changes), LV_ERR_BOUNDS (the block
+   table would overflow). */
+lv_status lv_session_append(lv_pool* pool, int32_t sid, int32_t n_tokens, int32_t* pages_out,
+                            int32_t* count_out, lv_stream stream);
+
+/* --------------------------------------------------------------- views */
+
+/* Per-session counts of blocks in HBM and in the host tier (int32 [S] each,
+   either may be NULL). */
+lv_status lv_session_counts(lv_pool* pool, int32_t* hbm_blocks, int32_t* host_blocks,
+                            lv_stream stream);
+
+/* The blocks of session sid in one tier (where 0: HBM, 1: host), ascending,
+   into blks_out (int32, capacity max_blocks); *count_out (int64) their number. */
+lv_status lv_session_blocks(lv_pool* pool, int32_t sid, int32_t where, int32_t* blks_out,
+                            int64_t* count_out, lv_stream stream);
+
+/* Copies the block tables (int32 [S][max_blocks]) and, if not NULL, the owner
+   tables (int64 [hbm_pages] and [host_pages]: sid << 32 | blk, or -1). */
+lv_status lv_read_tables(lv_pool* pool, int32_t* tables, int64_t* hbm_owner,
+                         int64_t* host_owner, lv_stream stream);
+
+/* ------------------------------------------------------------- status */
+
+/* Synchronous: waits for `stream`, returns the sticky device error (LV_OK if
+   none) or LV_ERR_CUDA. */
+lv_status lv_sync(lv_pool* pool, lv_stream stream);
+
+/* Synchronous: waits for `stream` and fills *out. */
+lv_status lv_get_stats(lv_pool* pool, lv_stats* out, lv_stream stream);
+
+/* Clears the sticky device error (stream-ordered). */
+lv_status lv_clear_error(lv_pool* pool, lv_stream stream);
+
+const char* lv_status_str(lv_status s);
+int32_t lv_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* LV_H */

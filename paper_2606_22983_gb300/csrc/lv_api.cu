@@ -1,0 +1,626 @@
+// C-ABI entry points of liblv (see include/lv.h): argument checks, device
+// metadata, staging of host-pointer arguments, and kernel launches.
+#include <cstdint>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "lv_internal.cuh"
+
+struct lv_pool {
+  lv::DevPool d{};
+  int device = 0;
+  int num_sms = 0;
+  int32_t epoch = 0;
+  bool own_host = false;
+  void* host_base = nullptr;       // host-visible address of the host pool
+  std::vector<void*> dev_allocs;
+  cudaMemPool_t mp = nullptr;      // stream-ordered staging memory
+};
+
+namespace {
+
+using lv::DevPool;
+
+#define LV_TRY(expr)                              \
+  do {                                            \
+    cudaError_t _e = (expr);                      \
+    if (_e != cudaSuccess) return lv_cuda_fail(_e); \
+  } while (0)
+
+lv_status lv_cuda_fail(cudaError_t e) {
+  if (e == cudaErrorMemoryAllocation) {
+    cudaGetLastError();
+    return LV_ERR_OOM;
+  }
+  return LV_ERR_CUDA;
+}
+
+class DeviceGuard {
+ public:
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev_) == cudaSuccess && prev_ != dev) {
+      cudaSetDevice(dev);
+      restore_ = true;
+    }
+  }
+  ~DeviceGuard() {
+    if (restore_) cudaSetDevice(prev_);
+  }
+
+ private:
+  int prev_ = 0;
+  bool restore_ = false;
+};
+
+bool is_device_ptr(const void* p) {
+  cudaPointerAttributes a{};
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+// Per-call staging: host-pointer inputs are copied in, host-pointer (or absent)
+// outputs get stream-ordered device buffers that are copied back at the end.
+class Staging {
+ public:
+  Staging(lv_pool* pool, cudaStream_t s) : pool_(pool), s_(s) {}
+  ~Staging() {
+    for (void* t : temps_) cudaFreeAsync(t, s_);
+  }
+
+  lv_status in(const void* user, size_t bytes, const void** dev) {
+    *dev = nullptr;
+    if (bytes == 0) return LV_OK;
+    if (user == nullptr) return LV_ERR_INVALID;
+    if (is_device_ptr(user)) {
+      *dev = user;
+      return LV_OK;
+    }
+    void* t = nullptr;
+    lv_status st = temp(bytes, &t);
+    if (st != LV_OK) return st;
+    LV_TRY(cudaMemcpyAsync(t, user, bytes, cudaMemcpyHostToDevice, s_));
+    *dev = t;
+    return LV_OK;
+  }
+
+  // required: a device buffer is needed even when the caller passes NULL
+  lv_status out(void* user, size_t bytes, void** dev, bool required) {
+    *dev = nullptr;
+    if (bytes == 0) return LV_OK;
+    if (user != nullptr && is_device_ptr(user)) {
+      *dev = user;
+      return LV_OK;
+    }
+    if (user == nullptr && !required) return LV_OK;
+    void* t = nullptr;
+    lv_status st = temp(bytes, &t);
+    if (st != LV_OK) return st;
+    *dev = t;
+    if (user != nullptr) backs_.push_back({user, t, bytes});
+    return LV_OK;
+  }
+
+  lv_status finish() {
+    for (const Back& b : backs_) LV_TRY(cudaMemcpyAsync(b.user, b.dev, b.bytes, cudaMemcpyDeviceToHost, s_));
+    backs_.clear();
+    return LV_OK;
+  }
+
+ private:
+  struct Back {
+    void* user;
+    void* dev;
+    size_t bytes;
+  };
+  lv_status temp(size_t bytes, void** t) {
+    cudaError_t e = cudaMallocFromPoolAsync(t, bytes, pool_->mp, s_);
+    if (e != cudaSuccess) return lv_cuda_fail(e);
+    temps_.push_back(*t);
+    return LV_OK;
+  }
+  lv_pool* pool_;
+  cudaStream_t s_;
+  std::vector<void*> temps_;
+  std::vector<Back> backs_;
+};
+
+template <typename T>
+lv_status dev_alloc(lv_pool* pool, T** ptr, size_t count) {
+  void* p = nullptr;
+  if (count == 0) count = 1;
+  cudaError_t e = cudaMalloc(&p, count * sizeof(T));
+  if (e != cudaSuccess) return lv_cuda_fail(e);
+  pool->dev_allocs.push_back(p);
+  *ptr = static_cast<T*>(p);
+  return LV_OK;
+}
+
+void free_pool(lv_pool* pool) {
+  for (void* p : pool->dev_allocs) cudaFree(p);
+  pool->dev_allocs.clear();
+  if (pool->own_host && pool->host_base) cudaFreeHost(pool->host_base);
+  if (pool->mp) cudaMemPoolDestroy(pool->mp);
+  delete pool;
+}
+
+inline cudaStream_t as_stream(lv_stream s) { return static_cast<cudaStream_t>(s); }
+
+lv_status validate_desc(const lv_pool_desc* d) {
+  if (!d) return LV_ERR_INVALID;
+  if (d->num_layers < 1 || d->num_kv_heads < 1 || d->head_dim < 1 || d->page_tokens < 1 ||
+      d->elem_bytes < 1)
+    return LV_ERR_INVALID;
+  const long long P = (long long)d->page_tokens * d->num_kv_heads * d->head_dim * d->elem_bytes;
+  if (P % 16 != 0 || P > (1ll << 30)) return LV_ERR_INVALID;
+  if (d->num_layers > 4096) return LV_ERR_INVALID;
+  if (d->max_sessions < 1 || d->max_sessions > 4096) return LV_ERR_INVALID;
+  if (d->max_blocks < 1 || d->max_blocks > 65536) return LV_ERR_INVALID;
+  if (d->hbm_pages < 1 || d->hbm_pages > 0x7fffffffll) return LV_ERR_INVALID;
+  if (d->hbm_budget_pages < 1 || d->hbm_budget_pages > d->hbm_pages) return LV_ERR_INVALID;
+  if (d->host_pages < 0 || d->host_pages > 0x7ffffffdll) return LV_ERR_INVALID;
+  if (d->reply_prior_us < 0 || d->protect_us < 0) return LV_ERR_INVALID;
+  if (d->unit_us < 1 || d->unit_us > (1ll << 31)) return LV_ERR_INVALID;
+  if (d->t_play_mode != LV_PLAY_PLAYBACK && d->t_play_mode != LV_PLAY_COUNTERS) return LV_ERR_INVALID;
+  if (d->within_order != LV_SUFFIX_FIRST && d->within_order != LV_ASCENDING) return LV_ERR_INVALID;
+  if (d->reserved != 0 || d->hbm_kv == nullptr) return LV_ERR_INVALID;
+  return LV_OK;
+}
+
+lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
+  lv_status st = validate_desc(desc);
+  if (st != LV_OK) return st;
+  lv_pool* pool = new (std::nothrow) lv_pool();
+  if (!pool) return LV_ERR_OOM;
+  auto fail = [&](lv_status code) {
+    free_pool(pool);
+    return code;
+  };
+  DevPool& d = pool->d;
+  if (cudaGetDevice(&pool->device) != cudaSuccess) return fail(LV_ERR_CUDA);
+  if (cudaDeviceGetAttribute(&pool->num_sms, cudaDevAttrMultiProcessorCount, pool->device) != cudaSuccess)
+    return fail(LV_ERR_CUDA);
+  d.S = desc->max_sessions;
+  d.maxB = desc->max_blocks;
+  d.T = desc->page_tokens;
+  d.J = 2 * desc->num_layers;
+  d.P = (int64_t)desc->page_tokens * desc->num_kv_heads * desc->head_dim * desc->elem_bytes;
+  d.hbm_pages = desc->hbm_pages;
+  d.budget = desc->hbm_budget_pages;
+  d.host_pages = desc->host_pages;
+  d.reply_prior_us = desc->reply_prior_us;
+  d.protect_us = desc->protect_us;
+  d.unit_us = desc->unit_us;
+  d.within = desc->within_order;
+  d.tplay = desc->t_play_mode;
+
+  // the caller's HBM sub-page arrays
+  std::vector<uint8_t*> kv(d.J);
+  for (int j = 0; j < d.J; ++j) {
+    void* p = desc->hbm_kv[j];
+    if (!p || (reinterpret_cast<uintptr_t>(p) & 15) || !is_device_ptr(p)) return fail(LV_ERR_INVALID);
+    kv[j] = static_cast<uint8_t*>(p);
+  }
+  // the host pool
+  const size_t host_bytes = (size_t)d.host_pages * d.J * d.P;
+  if (desc->host_kv) {
+    cudaPointerAttributes a{};
+    if (cudaPointerGetAttributes(&a, desc->host_kv) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(LV_ERR_INVALID);
+    }
+    if (a.type != cudaMemoryTypeHost || a.devicePointer == nullptr ||
+        (reinterpret_cast<uintptr_t>(a.devicePointer) & 15))
+      return fail(LV_ERR_INVALID);
+    pool->host_base = desc->host_kv;
+    d.host = static_cast<uint8_t*>(a.devicePointer);
+  } else if (host_bytes > 0) {
+    void* h = nullptr;
+    cudaError_t e = cudaHostAlloc(&h, host_bytes, cudaHostAllocMapped | cudaHostAllocPortable);
+    if (e != cudaSuccess) {
+      cudaGetLastError();
+      return fail(LV_ERR_OOM);
+    }
+    pool->own_host = true;
+    pool->host_base = h;
+    void* hd = nullptr;
+    if (cudaHostGetDevicePointer(&hd, h, 0) != cudaSuccess) return fail(LV_ERR_CUDA);
+    d.host = static_cast<uint8_t*>(hd);
+  }
+
+  uint8_t** kv_dev = nullptr;
+  const size_t tb = (size_t)d.S * d.maxB;
+  const size_t wh = (size_t)((d.hbm_pages + 31) / 32), wo = (size_t)((d.host_pages + 31) / 32);
+  if ((st = dev_alloc(pool, &kv_dev, d.J)) != LV_OK ||
+      (st = dev_alloc(pool, &d.sess, d.S)) != LV_OK ||
+      (st = dev_alloc(pool, &d.table, tb)) != LV_OK ||
+      (st = dev_alloc(pool, &d.mark, tb)) != LV_OK ||
+      (st = dev_alloc(pool, &d.own_hbm, (size_t)d.hbm_pages)) != LV_OK ||
+      (st = dev_alloc(pool, &d.own_host, (size_t)d.host_pages)) != LV_OK ||
+      (st = dev_alloc(pool, &d.bits_hbm, wh)) != LV_OK ||
+      (st = dev_alloc(pool, &d.bits_host, wo)) != LV_OK ||
+      (st = dev_alloc(pool, &d.ctl, (size_t)lv::C_N)) != LV_OK ||
+      (st = dev_alloc(pool, &d.skey, d.S)) != LV_OK ||
+      (st = dev_alloc(pool, &d.scount, d.S)) != LV_OK ||
+      (st = dev_alloc(pool, &d.sorder, d.S)) != LV_OK ||
+      (st = dev_alloc(pool, &d.soff, d.S)) != LV_OK)
+    return fail(st);
+  d.kv = kv_dev;
+  if (cudaMemcpyAsync(kv_dev, kv.data(), d.J * sizeof(uint8_t*), cudaMemcpyHostToDevice, s) != cudaSuccess ||
+      cudaMemsetAsync(d.sess, 0, d.S * sizeof(lv_session_state), s) != cudaSuccess ||
+      cudaMemsetAsync(d.table, 0xff, tb * sizeof(int32_t), s) != cudaSuccess ||
+      cudaMemsetAsync(d.mark, 0, tb * sizeof(int32_t), s) != cudaSuccess ||
+      cudaMemsetAsync(d.own_hbm, 0xff, (size_t)d.hbm_pages * 8, s) != cudaSuccess ||
+      cudaMemsetAsync(d.own_host, 0xff, (size_t)(d.host_pages ? d.host_pages : 1) * 8, s) != cudaSuccess ||
+      cudaMemsetAsync(d.bits_hbm, 0, wh * 4, s) != cudaSuccess ||
+      cudaMemsetAsync(d.bits_host, 0, (wo ? wo : 1) * 4, s) != cudaSuccess ||
+      cudaMemsetAsync(d.ctl, 0, lv::C_N * sizeof(long long), s) != cudaSuccess)
+    return fail(LV_ERR_CUDA);
+
+  if (lv::configure_kernels() != cudaSuccess) return fail(LV_ERR_CUDA);
+  cudaMemPoolProps props{};
+  props.allocType = cudaMemAllocationTypePinned;
+  props.location.type = cudaMemLocationTypeDevice;
+  props.location.id = pool->device;
+  if (cudaMemPoolCreate(&pool->mp, &props) != cudaSuccess) {
+    pool->mp = nullptr;
+    return fail(LV_ERR_CUDA);
+  }
+  uint64_t threshold = UINT64_MAX;
+  cudaMemPoolSetAttribute(pool->mp, cudaMemPoolAttrReleaseThreshold, &threshold);
+  if (cudaStreamSynchronize(s) != cudaSuccess) return fail(LV_ERR_CUDA);
+  *out = pool;
+  return LV_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+lv_status lv_pool_create(const lv_pool_desc* desc, lv_stream stream, lv_pool** out) {
+  if (!out) return LV_ERR_INVALID;
+  *out = nullptr;
+  try {
+    return create_impl(desc, as_stream(stream), out);
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_pool_destroy(lv_pool* pool, lv_stream stream) {
+  if (!pool) return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  cudaError_t e = cudaStreamSynchronize(as_stream(stream));
+  free_pool(pool);
+  return e == cudaSuccess ? LV_OK : LV_ERR_CUDA;
+}
+
+void* lv_pool_host_ptr(lv_pool* pool) { return pool ? pool->host_base : nullptr; }
+
+lv_status lv_pool_import(lv_pool* pool, const int32_t* placement, const int32_t* ctx_tokens,
+                         lv_stream stream) {
+  if (!pool || !placement || !ctx_tokens) return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  DevPool& d = pool->d;
+  try {
+    Staging st(pool, s);
+    const void *pl = nullptr, *cx = nullptr;
+    lv_status r;
+    if ((r = st.in(placement, (size_t)d.S * d.maxB * 4, &pl)) != LV_OK) return r;
+    if ((r = st.in(ctx_tokens, (size_t)d.S * 4, &cx)) != LV_OK) return r;
+    LV_TRY(cudaMemsetAsync(d.own_hbm, 0xff, (size_t)d.hbm_pages * 8, s));
+    if (d.host_pages) LV_TRY(cudaMemsetAsync(d.own_host, 0xff, (size_t)d.host_pages * 8, s));
+    LV_TRY(cudaMemsetAsync(d.bits_hbm, 0, (size_t)((d.hbm_pages + 31) / 32) * 4, s));
+    if (d.host_pages) LV_TRY(cudaMemsetAsync(d.bits_host, 0, (size_t)((d.host_pages + 31) / 32) * 4, s));
+    LV_TRY(cudaMemsetAsync(d.ctl, 0, 2 * sizeof(long long), s));   // allocation counts
+    LV_TRY(lv::launch_import(d, static_cast<const int32_t*>(pl), static_cast<const int32_t*>(cx), s));
+    LV_TRY(lv::launch_check_budget(d, s));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_session_set(lv_pool* pool, const lv_session_state* states, int32_t first, int32_t n,
+                         lv_stream stream) {
+  if (!pool || first < 0 || n < 0 || (long long)first + n > pool->d.S) return LV_ERR_INVALID;
+  if (n == 0) return LV_OK;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  try {
+    Staging st(pool, s);
+    const void* in = nullptr;
+    lv_status r = st.in(states, (size_t)n * sizeof(lv_session_state), &in);
+    if (r != LV_OK) return r;
+    LV_TRY(lv::launch_session_set(pool->d, static_cast<const lv_session_state*>(in), first, n, s));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_session_get(lv_pool* pool, lv_session_state* out, int32_t first, int32_t n,
+                         lv_stream stream) {
+  if (!pool || !out || first < 0 || n < 0 || (long long)first + n > pool->d.S) return LV_ERR_INVALID;
+  if (n == 0) return LV_OK;
+  DeviceGuard g(pool->device);
+  LV_TRY(cudaMemcpyAsync(out, pool->d.sess + first, (size_t)n * sizeof(lv_session_state),
+                         cudaMemcpyDefault, as_stream(stream)));
+  return LV_OK;
+}
+
+lv_status lv_session_events(lv_pool* pool, const lv_event* events, int64_t n, lv_stream stream) {
+  if (!pool || n < 0 || (n > 0 && !events)) return LV_ERR_INVALID;
+  if (n == 0) return LV_OK;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  try {
+    Staging st(pool, s);
+    const void* in = nullptr;
+    lv_status r = st.in(events, (size_t)n * sizeof(lv_event), &in);
+    if (r != LV_OK) return r;
+    LV_TRY(lv::launch_events(pool->d, static_cast<const lv_event*>(in), n, s));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_select_victims(lv_pool* pool, int64_t now_us, int64_t k, uint32_t flags,
+                            lv_victim* out, int64_t capacity, int64_t* count_out,
+                            lv_stream stream) {
+  if (!pool || k < 0 || capacity < 0 || (flags & ~(uint32_t)LV_SELECT_FALLBACK)) return LV_ERR_INVALID;
+  const int64_t keff = k < capacity ? k : capacity;
+  if (keff > 0 && !out) return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  try {
+    Staging st(pool, s);
+    void *vdev = nullptr, *cdev = nullptr;
+    lv_status r;
+    if ((r = st.out(out, (size_t)keff * sizeof(lv_victim), &vdev, false)) != LV_OK) return r;
+    if ((r = st.out(count_out, sizeof(int64_t), &cdev, false)) != LV_OK) return r;
+    LV_TRY(lv::launch_select(pool->d, now_us, keff, (flags & LV_SELECT_FALLBACK) != 0,
+                             static_cast<lv_victim*>(vdev), static_cast<long long*>(cdev), s,
+                             pool->num_sms));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_swap_out(lv_pool* pool, const lv_victim* victims, int64_t n, int32_t* slots_out,
+                      lv_remap_entry* commit_out, int32_t mode, lv_stream stream) {
+  if (!pool || n < 0 || n > 0x7fffffffll || (n > 0 && !victims)) return LV_ERR_INVALID;
+  if (mode != LV_MODE_AUTO && mode != LV_MODE_ZERO_COPY) return LV_ERR_INVALID;
+  if (n == 0) return LV_OK;
+  if (pool->d.host_pages == 0) return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  try {
+    Staging st(pool, s);
+    const void* vin = nullptr;
+    void *sdev = nullptr, *cdev = nullptr;
+    lv_status r;
+    if ((r = st.in(victims, (size_t)n * sizeof(lv_victim), &vin)) != LV_OK) return r;
+    if ((r = st.out(slots_out, (size_t)n * 4, &sdev, true)) != LV_OK) return r;
+    if ((r = st.out(commit_out, (size_t)n * sizeof(lv_remap_entry), &cdev, false)) != LV_OK) return r;
+    int32_t* slots = static_cast<int32_t*>(sdev);
+    LV_TRY(lv::launch_alloc(pool->d, false, n, slots, s));
+    LV_TRY(lv::launch_swap_out(pool->d, static_cast<const lv_victim*>(vin), slots, n,
+                               static_cast<lv_remap_entry*>(cdev), s, pool->num_sms));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_swap_in(lv_pool* pool, int32_t sid, const int32_t* blks, int64_t n, int32_t* pages_out,
+                     lv_remap_entry* commit_out, int32_t mode, lv_stream stream) {
+  if (!pool || n < 0 || n > 0x7fffffffll || (n > 0 && !blks)) return LV_ERR_INVALID;
+  if (mode != LV_MODE_AUTO && mode != LV_MODE_ZERO_COPY) return LV_ERR_INVALID;
+  if (sid < 0 || sid >= pool->d.S) return LV_ERR_INVALID;
+  if (n == 0) return LV_OK;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  try {
+    Staging st(pool, s);
+    const void* bin = nullptr;
+    void *pdev = nullptr, *cdev = nullptr;
+    lv_status r;
+    if ((r = st.in(blks, (size_t)n * 4, &bin)) != LV_OK) return r;
+    if ((r = st.out(pages_out, (size_t)n * 4, &pdev, true)) != LV_OK) return r;
+    if ((r = st.out(commit_out, (size_t)n * sizeof(lv_remap_entry), &cdev, false)) != LV_OK) return r;
+    int32_t* pages = static_cast<int32_t*>(pdev);
+    LV_TRY(lv::launch_alloc(pool->d, true, n, pages, s));
+    LV_TRY(lv::launch_swap_in(pool->d, sid, static_cast<const int32_t*>(bin), pages, n,
+                              static_cast<lv_remap_entry*>(cdev), s, pool->num_sms));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_remap(lv_pool* pool, const lv_remap_entry* entries, int64_t n, lv_stream stream) {
+  if (!pool || n < 0 || (n > 0 && !entries)) return LV_ERR_INVALID;
+  if (n == 0) return LV_OK;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  try {
+    Staging st(pool, s);
+    const void* in = nullptr;
+    lv_status r = st.in(entries, (size_t)n * sizeof(lv_remap_entry), &in);
+    if (r != LV_OK) return r;
+    if (++pool->epoch <= 0) pool->epoch = 1;
+    LV_TRY(lv::launch_remap(pool->d, static_cast<const lv_remap_entry*>(in), n, pool->epoch, s));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_cancel(lv_pool* pool, const int32_t* locs, int64_t n, lv_stream stream) {
+  if (!pool || n < 0 || (n > 0 && !locs)) return LV_ERR_INVALID;
+  if (n == 0) return LV_OK;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  try {
+    Staging st(pool, s);
+    const void* in = nullptr;
+    lv_status r = st.in(locs, (size_t)n * 4, &in);
+    if (r != LV_OK) return r;
+    LV_TRY(lv::launch_cancel(pool->d, static_cast<const int32_t*>(in), n, s));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_session_append(lv_pool* pool, int32_t sid, int32_t n_tokens, int32_t* pages_out,
+                            int32_t* count_out, lv_stream stream) {
+  if (!pool || sid < 0 || sid >= pool->d.S || n_tokens < 0) return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  const size_t cap = (size_t)(n_tokens / pool->d.T) + 2;
+  try {
+    Staging st(pool, s);
+    void *pdev = nullptr, *cdev = nullptr;
+    lv_status r;
+    if ((r = st.out(pages_out, cap * 4, &pdev, true)) != LV_OK) return r;
+    if ((r = st.out(count_out, 4, &cdev, false)) != LV_OK) return r;
+    LV_TRY(lv::launch_append(pool->d, sid, n_tokens, static_cast<int32_t*>(pdev),
+                             static_cast<int32_t*>(cdev), s));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_session_counts(lv_pool* pool, int32_t* hbm_blocks, int32_t* host_blocks, lv_stream stream) {
+  if (!pool) return LV_ERR_INVALID;
+  if (!hbm_blocks && !host_blocks) return LV_OK;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  try {
+    Staging st(pool, s);
+    void *a = nullptr, *b = nullptr;
+    lv_status r;
+    if ((r = st.out(hbm_blocks, (size_t)pool->d.S * 4, &a, false)) != LV_OK) return r;
+    if ((r = st.out(host_blocks, (size_t)pool->d.S * 4, &b, false)) != LV_OK) return r;
+    LV_TRY(lv::launch_counts(pool->d, static_cast<int32_t*>(a), static_cast<int32_t*>(b), s));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_session_blocks(lv_pool* pool, int32_t sid, int32_t where, int32_t* blks_out,
+                            int64_t* count_out, lv_stream stream) {
+  if (!pool || sid < 0 || sid >= pool->d.S || (where != 0 && where != 1) || !blks_out)
+    return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  try {
+    Staging st(pool, s);
+    void *bdev = nullptr, *cdev = nullptr;
+    lv_status r;
+    if ((r = st.out(blks_out, (size_t)pool->d.maxB * 4, &bdev, true)) != LV_OK) return r;
+    if ((r = st.out(count_out, 8, &cdev, false)) != LV_OK) return r;
+    LV_TRY(lv::launch_blocks(pool->d, sid, where, static_cast<int32_t*>(bdev),
+                             static_cast<long long*>(cdev), s));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_read_tables(lv_pool* pool, int32_t* tables, int64_t* hbm_owner, int64_t* host_owner,
+                         lv_stream stream) {
+  if (!pool) return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  const DevPool& d = pool->d;
+  if (tables)
+    LV_TRY(cudaMemcpyAsync(tables, d.table, (size_t)d.S * d.maxB * 4, cudaMemcpyDefault, s));
+  if (hbm_owner)
+    LV_TRY(cudaMemcpyAsync(hbm_owner, d.own_hbm, (size_t)d.hbm_pages * 8, cudaMemcpyDefault, s));
+  if (host_owner && d.host_pages)
+    LV_TRY(cudaMemcpyAsync(host_owner, d.own_host, (size_t)d.host_pages * 8, cudaMemcpyDefault, s));
+  return LV_OK;
+}
+
+lv_status lv_sync(lv_pool* pool, lv_stream stream) {
+  if (!pool) return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  long long ctl[2] = {0, 0};
+  cudaStream_t s = as_stream(stream);
+  if (cudaMemcpyAsync(ctl, pool->d.ctl + lv::C_ERR, sizeof(ctl), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return LV_ERR_CUDA;
+  return static_cast<lv_status>(ctl[0]);
+}
+
+lv_status lv_get_stats(lv_pool* pool, lv_stats* out, lv_stream stream) {
+  if (!pool || !out) return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  long long c[lv::C_N];
+  cudaStream_t s = as_stream(stream);
+  if (cudaMemcpyAsync(c, pool->d.ctl, sizeof(c), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return LV_ERR_CUDA;
+  const long long page_bytes = (long long)pool->d.J * pool->d.P;
+  std::memset(out, 0, sizeof(*out));
+  out->hbm_allocated = c[lv::C_HBM_ALLOC];
+  out->host_allocated = c[lv::C_HOST_ALLOC];
+  out->hbm_budget_pages = pool->d.budget;
+  out->host_pages = pool->d.host_pages;
+  out->error = c[lv::C_ERR];
+  out->error_detail = c[lv::C_ERR_DETAIL];
+  out->last_select_count = c[lv::C_SEL_COUNT];
+  out->last_select_total = c[lv::C_SEL_TOTAL];
+  out->selects = c[lv::C_SELECTS];
+  out->victims = c[lv::C_VICTIMS];
+  out->shortfalls = c[lv::C_SHORTFALLS];
+  out->pages_out = c[lv::C_PAGES_OUT];
+  out->pages_in = c[lv::C_PAGES_IN];
+  out->bytes_out = c[lv::C_PAGES_OUT] * page_bytes;
+  out->bytes_in = c[lv::C_PAGES_IN] * page_bytes;
+  out->remap_entries = c[lv::C_REMAP];
+  out->appended_pages = c[lv::C_APPENDED];
+  out->cancels = c[lv::C_CANCELS];
+  out->events = c[lv::C_EVENTS];
+  out->fallback_selects = c[lv::C_FALLBACK];
+  return LV_OK;
+}
+
+lv_status lv_clear_error(lv_pool* pool, lv_stream stream) {
+  if (!pool) return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  LV_TRY(cudaMemsetAsync(pool->d.ctl + lv::C_ERR, 0, 2 * sizeof(long long), as_stream(stream)));
+  return LV_OK;
+}
+
+const char* lv_status_str(lv_status s) {
+  switch (s) {
+    case LV_OK: return "LV_OK";
+    case LV_ERR_INVALID: return "LV_ERR_INVALID";
+    case LV_ERR_OOM: return "LV_ERR_OOM";
+    case LV_ERR_CUDA: return "LV_ERR_CUDA";
+    case LV_ERR_NO_HBM: return "LV_ERR_NO_HBM";
+    case LV_ERR_NO_HOST: return "LV_ERR_NO_HOST";
+    case LV_ERR_BOUNDS: return "LV_ERR_BOUNDS";
+    case LV_ERR_DOUBLE_MAP: return "LV_ERR_DOUBLE_MAP";
+    case LV_ERR_BUDGET: return "LV_ERR_BUDGET";
+    case LV_ERR_TIMEOUT: return "LV_ERR_TIMEOUT";
+    case LV_ERR_STATE: return "LV_ERR_STATE";
+  }
+  return "LV_ERR_UNKNOWN";
+}
+
+int32_t lv_version(void) { return 1; }
+
+}  // extern "C"

@@ -1,0 +1,92 @@
+// Internal declarations shared by the kernels and the C-ABI layer of liblv.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "lv.h"
+
+namespace lv {
+
+constexpr unsigned long long kOwnerNone = ~0ull;
+constexpr long long kKeyMax = 0xFFFFFFFFll;   // T_next is clamped to 32 bits (microseconds)
+
+// Layout of the per-pool int64 control block in device memory.
+enum Ctl : int {
+  C_HBM_ALLOC = 0,     // HBM pages reserved or owned
+  C_HOST_ALLOC = 1,    // host slots reserved or owned
+  C_ERR = 2,           // sticky lv_status (first device-detected error)
+  C_ERR_DETAIL = 3,
+  C_SEL_COUNT = 4,     // victims written by the last select
+  C_SEL_TOTAL = 5,     // candidates seen by the last select
+  C_SELECTS = 8,
+  C_VICTIMS,
+  C_SHORTFALLS,
+  C_PAGES_OUT,
+  C_PAGES_IN,
+  C_REMAP,
+  C_APPENDED,
+  C_CANCELS,
+  C_EVENTS,
+  C_FALLBACK,
+  C_N = 32
+};
+
+// Everything a kernel needs to know about a pool, passed by value.
+struct DevPool {
+  int32_t S;              // sessions
+  int32_t maxB;           // block-table capacity per session
+  int32_t T;              // tokens per page
+  int32_t J;              // sub-pages per page (2L)
+  int64_t P;              // bytes per sub-page (multiple of 16)
+  int64_t hbm_pages, budget, host_pages;
+  int64_t reply_prior_us, protect_us, unit_us;
+  int32_t within;         // LV_SUFFIX_FIRST / LV_ASCENDING
+  int32_t tplay;          // LV_PLAY_PLAYBACK / LV_PLAY_COUNTERS
+  uint8_t* const* kv;     // [J] device pointers, sub-page j of page p at kv[j] + p*P
+  uint8_t* host;          // device view of the host pool [host_pages][J][P]
+  lv_session_state* sess; // [S]
+  int32_t* table;         // [S][maxB]
+  int32_t* mark;          // [S][maxB] epoch of the last remap that touched the block
+  unsigned long long* own_hbm;   // [hbm_pages] sid << 32 | blk, or kOwnerNone
+  unsigned long long* own_host;  // [host_pages]
+  uint32_t* bits_hbm;     // allocation bitmap, 1 = reserved or owned
+  uint32_t* bits_host;
+  long long* ctl;         // [C_N]
+  // ranking scratch
+  unsigned long long* skey;  // [S] session sort key (0 = not a candidate)
+  int32_t* scount;           // [S] resident blocks of the session
+  int32_t* sorder;           // [S] session id at rank r
+  long long* soff;           // [S] first victim position of rank r
+};
+
+__host__ __device__ inline unsigned long long owner_key(int32_t sid, int32_t blk) {
+  return ((unsigned long long)(uint32_t)sid << 32) | (uint32_t)blk;
+}
+
+// ---- launch wrappers (lv_kernels.cu); each returns cudaGetLastError() ----
+cudaError_t launch_import(const DevPool& p, const int32_t* placement, const int32_t* ctx,
+                          cudaStream_t s);
+cudaError_t launch_session_set(const DevPool& p, const lv_session_state* in, int32_t first,
+                               int32_t n, cudaStream_t s);
+cudaError_t launch_events(const DevPool& p, const lv_event* ev, int64_t n, cudaStream_t s);
+cudaError_t launch_select(const DevPool& p, int64_t now_us, int64_t k, bool fallback,
+                          lv_victim* out, long long* count_dev, cudaStream_t s, int num_sms);
+cudaError_t launch_alloc(const DevPool& p, bool hbm, int64_t n, int32_t* out, cudaStream_t s);
+cudaError_t launch_swap_out(const DevPool& p, const lv_victim* v, const int32_t* slots,
+                            int64_t n, lv_remap_entry* commit, cudaStream_t s, int num_sms);
+cudaError_t launch_swap_in(const DevPool& p, int32_t sid, const int32_t* blks,
+                           const int32_t* pages, int64_t n, lv_remap_entry* commit,
+                           cudaStream_t s, int num_sms);
+cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, int32_t epoch,
+                         cudaStream_t s);
+cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cudaStream_t s);
+cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32_t* pages,
+                          int32_t* count, cudaStream_t s);
+cudaError_t launch_counts(const DevPool& p, int32_t* hbm, int32_t* host, cudaStream_t s);
+cudaError_t launch_blocks(const DevPool& p, int32_t sid, int32_t where, int32_t* out,
+                          long long* count, cudaStream_t s);
+cudaError_t launch_check_budget(const DevPool& p, cudaStream_t s);
+cudaError_t configure_kernels();   // once per device, before the first launch
+
+}  // namespace lv

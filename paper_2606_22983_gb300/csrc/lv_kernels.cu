@@ -1,0 +1,749 @@
+// CUDA kernels of the KV swap path (sm_103a).
+//
+//   ranking   k_rank_census -> k_rank_sort -> k_rank_emit   (Section 5.1, Eq. 4)
+//   allocate  k_alloc                                        (lowest free, Section 5.1)
+//   move      k_swap_out / k_swap_in                         (Section 5, Fig. 6; Section 5.2)
+//   commit    k_remap, k_cancel, k_append                    (Section 6 side tables)
+//   monitor   k_events                                       (Section 3, Sections 5.1-5.2)
+//
+// No kernel waits on another agent, so none can hang; every index read from
+// memory is range-checked and a bad item is skipped with the sticky error set.
+#include <cstdint>
+
+#include "lv_internal.cuh"
+
+namespace lv {
+
+namespace {
+
+__device__ __forceinline__ void set_error(long long* ctl, int code, long long detail) {
+  if (atomicCAS(reinterpret_cast<unsigned long long*>(&ctl[C_ERR]), 0ull,
+                (unsigned long long)code) == 0ull) {
+    ctl[C_ERR_DETAIL] = detail;
+  }
+}
+
+__device__ __forceinline__ int32_t nblocks_of(const DevPool& p, int32_t sid) {
+  long long c = p.sess[sid].ctx_tokens;
+  long long nb = (c + p.T - 1) / p.T;
+  if (nb < 0) nb = 0;
+  if (nb > p.maxB) nb = p.maxB;
+  return (int32_t)nb;
+}
+
+// Exclusive scan over the block of NT threads; *total receives the sum.
+template <int NT>
+__device__ long long block_excl_scan(long long v, long long* total) {
+  static_assert(NT % 32 == 0 && NT <= 1024, "block size");
+  __shared__ long long warp_sums[NT / 32];
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  long long x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    long long y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_sums[wid] = x;
+  __syncthreads();
+  if (wid == 0) {
+    long long w = lane < NT / 32 ? warp_sums[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      long long y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    if (lane < NT / 32) warp_sums[lane] = w;
+  }
+  __syncthreads();
+  long long before = wid > 0 ? warp_sums[wid - 1] : 0;
+  *total = warp_sums[NT / 32 - 1];
+  __syncthreads();
+  return before + x - v;
+}
+
+__device__ __forceinline__ uint32_t free_bits(const uint32_t* bits, long long w, long long W,
+                                              long long nbits) {
+  uint32_t valid = 0xffffffffu;
+  if (w == W - 1 && (nbits & 31)) valid = (1u << (nbits & 31)) - 1u;
+  return ~bits[w] & valid;
+}
+
+// The n lowest free bits of a bitmap, ascending, into out[0..n); sets them.
+// Each thread owns a contiguous run of words and writes only the ranks it
+// counted, so a concurrent free elsewhere cannot make two threads write one rank.
+template <int NT>
+__device__ void block_alloc_lowest(uint32_t* bits, long long nbits, long long n, int32_t* out) {
+  const long long W = (nbits + 31) >> 5;
+  const long long per = (W + NT - 1) / NT;
+  const long long w0 = min(W, (long long)threadIdx.x * per);
+  const long long w1 = min(W, w0 + per);
+  long long cnt = 0;
+  for (long long w = w0; w < w1; ++w) cnt += __popc(free_bits(bits, w, W, nbits));
+  long long total;
+  const long long base = block_excl_scan<NT>(cnt, &total);
+  long long r = base;
+  const long long r_end = min(n, base + cnt);
+  for (long long w = w0; w < w1 && r < r_end; ++w) {
+    uint32_t f = free_bits(bits, w, W, nbits);
+    uint32_t take = 0;
+    while (f && r < r_end) {
+      int b = __ffs(f) - 1;
+      f &= f - 1;
+      out[r++] = (int32_t)(w * 32 + b);
+      take |= 1u << b;
+    }
+    if (take) atomicOr(&bits[w], take);
+  }
+}
+
+// ---------------------------------------------------------------- import
+__global__ void k_import(DevPool p, const int32_t* __restrict__ placement,
+                         const int32_t* __restrict__ ctx) {
+  const long long total = (long long)p.S * p.maxB;
+  for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
+       idx += (long long)gridDim.x * blockDim.x) {
+    const int32_t s = (int32_t)(idx / p.maxB), b = (int32_t)(idx % p.maxB);
+    const long long c = ctx[s];
+    long long nb = (c + p.T - 1) / p.T;
+    if (b == 0) {
+      if (c < 0 || nb > p.maxB) {
+        set_error(p.ctl, LV_ERR_BOUNDS, s);
+      }
+      p.sess[s].ctx_tokens = (c < 0 || nb > p.maxB) ? 0 : (int32_t)c;
+    }
+    if (c < 0 || nb > p.maxB) nb = 0;
+    const int32_t e = placement[idx];
+    p.table[idx] = -1;
+    p.mark[idx] = 0;
+    if (b >= nb) {
+      if (e != -1) set_error(p.ctl, LV_ERR_BOUNDS, idx);
+      continue;
+    }
+    const unsigned long long key = owner_key(s, b);
+    if (e >= 0) {
+      if (e >= p.hbm_pages) { set_error(p.ctl, LV_ERR_BOUNDS, idx); continue; }
+      if (atomicCAS(&p.own_hbm[e], kOwnerNone, key) != kOwnerNone) {
+        set_error(p.ctl, LV_ERR_DOUBLE_MAP, idx);
+        continue;
+      }
+      atomicOr(&p.bits_hbm[e >> 5], 1u << (e & 31));
+      atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HBM_ALLOC]), 1ull);
+    } else if (e <= -2) {
+      const long long h = -(long long)e - 2;
+      if (h >= p.host_pages) { set_error(p.ctl, LV_ERR_BOUNDS, idx); continue; }
+      if (atomicCAS(&p.own_host[h], kOwnerNone, key) != kOwnerNone) {
+        set_error(p.ctl, LV_ERR_DOUBLE_MAP, idx);
+        continue;
+      }
+      atomicOr(&p.bits_host[h >> 5], 1u << (h & 31));
+      atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HOST_ALLOC]), 1ull);
+    } else {
+      set_error(p.ctl, LV_ERR_BOUNDS, idx);   // a block inside the context with no location
+      continue;
+    }
+    p.table[idx] = e;
+  }
+}
+
+__global__ void k_check_budget(DevPool p) {
+  if (p.ctl[C_HBM_ALLOC] > p.budget) set_error(p.ctl, LV_ERR_BUDGET, p.ctl[C_HBM_ALLOC]);
+}
+
+// -------------------------------------------------------------- sessions
+__global__ void k_session_set(DevPool p, const lv_session_state* __restrict__ in, int32_t first,
+                              int32_t n) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  lv_session_state st = in[i];
+  st.ctx_tokens = p.sess[first + i].ctx_tokens;   // owned by import / append
+  p.sess[first + i] = st;
+}
+
+// One thread per session applies, in order, the events addressed to it.
+__global__ void k_events(DevPool p, const lv_event* __restrict__ ev, long long n) {
+  const int s = blockIdx.x * blockDim.x + threadIdx.x;
+  if (s == 0) {
+    for (long long e = 0; e < n; ++e) {
+      if (ev[e].kind < LV_EV_TURN_BEGIN || ev[e].kind > LV_EV_PRELOADED || ev[e].sid < 0 ||
+          ev[e].sid >= p.S) {
+        set_error(p.ctl, LV_ERR_BOUNDS, e);
+      }
+    }
+    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_EVENTS]), (unsigned long long)n);
+  }
+  if (s >= p.S) return;
+  lv_session_state st = p.sess[s];
+  bool touched = false;
+  for (long long e = 0; e < n; ++e) {
+    if (ev[e].sid != s) continue;
+    const lv_event x = ev[e];
+    touched = true;
+    switch (x.kind) {
+      case LV_EV_TURN_BEGIN:
+        st.flags = (st.flags | LV_RUNNING) & ~LV_IMMEDIATE;
+        st.protect_until_us = 0;
+        break;
+      case LV_EV_TURN_END:
+        st.flags &= ~(LV_RUNNING | LV_DONE_VALID);
+        st.gen_us = x.a;
+        st.play_us = 0;
+        st.reply_tokens = x.b;
+        if (st.gen_us > 0) {
+          st.flags |= LV_RESP_OPEN;
+        } else {
+          st.flags = (st.flags & ~LV_RESP_OPEN) | LV_DONE_VALID;
+          st.t_done_us = x.t_us;
+        }
+        break;
+      case LV_EV_PLAYBACK:
+        if (st.flags & LV_RESP_OPEN) {
+          const long long np = st.play_us + x.a;
+          st.play_us = np < st.gen_us ? np : st.gen_us;
+          if (st.play_us >= st.gen_us) {
+            st.flags = (st.flags & ~LV_RESP_OPEN) | LV_DONE_VALID;
+            st.t_done_us = x.t_us;
+          }
+        }
+        break;
+      case LV_EV_SPEECH_START:
+        st.flags |= LV_IMMEDIATE;
+        break;
+      case LV_EV_BARGE_IN:
+        st.gen_us = st.play_us;
+        st.flags = (st.flags | LV_IMMEDIATE) & ~(LV_RESP_OPEN | LV_DONE_VALID);
+        break;
+      case LV_EV_SPEECH_STOP:
+        if (st.flags & LV_DONE_VALID) {
+          long long xs = x.t_us - st.t_done_us;
+          if (xs < 0) xs = 0;
+          st.reply_ema_us = st.reply_n == 0 ? xs : (3 * st.reply_ema_us + xs) / 4;
+          if (st.reply_n < 0x7fffffff) st.reply_n += 1;
+        }
+        st.flags &= ~(LV_IMMEDIATE | LV_DONE_VALID);
+        break;
+      case LV_EV_PRELOADED:
+        st.protect_until_us = x.t_us + p.protect_us;
+        break;
+      default:
+        break;   // reported above
+    }
+  }
+  if (touched) p.sess[s] = st;
+}
+
+// --------------------------------------------------------------- ranking
+// Sort key of a session, 0 when it is not a candidate.  Larger keys are
+// evicted first: bit 63 = normal tier, bits 31..62 = T_next (Eq. 4), bits
+// 0..30 = 2^31-1-sid so that equal T_next rank by ascending session id.
+__device__ __forceinline__ unsigned long long session_key(const DevPool& p, int32_t s,
+                                                          long long now_us, bool fallback) {
+  const lv_session_state st = p.sess[s];
+  const bool normal = !(st.flags & (LV_RUNNING | LV_IMMEDIATE)) && !(now_us < st.protect_until_us);
+  if (!normal && !(fallback && !(st.flags & LV_RUNNING))) return 0ull;
+  long long t_play;
+  if (p.tplay == LV_PLAY_PLAYBACK) {
+    const long long d = st.gen_us - st.play_us;            // remaining playback horizon
+    t_play = d > 0 ? d : 0;
+  } else {
+    // progress counters: a longer unfinished reply means later reuse
+    if (!(st.flags & LV_RESP_OPEN) || st.reply_tokens <= 0) t_play = 0;
+    else if (st.reply_tokens > kKeyMax / p.unit_us) t_play = kKeyMax;
+    else t_play = st.reply_tokens * p.unit_us;
+  }
+  long long t_reply = st.reply_n > 0 ? st.reply_ema_us : p.reply_prior_us;
+  if (t_reply < 0) t_reply = 0;
+  if (t_play > kKeyMax) t_play = kKeyMax;
+  if (t_reply > kKeyMax) t_reply = kKeyMax;
+  long long t_next = t_play + t_reply;
+  if (t_next > kKeyMax) t_next = kKeyMax;
+  return ((normal ? 1ull : 0ull) << 63) | ((unsigned long long)t_next << 31) |
+         (unsigned long long)(0x7fffffff - s);
+}
+
+constexpr int kCensusThreads = 256;
+
+// One CTA per session: its key and its count of HBM-resident blocks.
+__global__ void __launch_bounds__(kCensusThreads)
+k_rank_census(DevPool p, long long now_us, bool fallback) {
+  const int32_t s = blockIdx.x;
+  __shared__ unsigned long long key;
+  if (threadIdx.x == 0) key = session_key(p, s, now_us, fallback);
+  __syncthreads();
+  if (key == 0ull) {
+    if (threadIdx.x == 0) { p.skey[s] = 0ull; p.scount[s] = 0; }
+    return;
+  }
+  const int32_t nb = nblocks_of(p, s);
+  const int32_t* row = p.table + (size_t)s * p.maxB;
+  long long c = 0;
+  for (int32_t b = threadIdx.x; b < nb; b += kCensusThreads) c += row[b] >= 0 ? 1 : 0;
+  long long total;
+  block_excl_scan<kCensusThreads>(c, &total);
+  if (threadIdx.x == 0) {
+    p.skey[s] = key;
+    p.scount[s] = (int32_t)total;
+  }
+}
+
+constexpr int kSortThreads = 1024;
+
+// One CTA: bitonic sort of the session keys (descending), scan of the counts
+// in rank order, and the number of victims to emit.
+__global__ void __launch_bounds__(kSortThreads)
+k_rank_sort(DevPool p, long long k, bool fallback, long long* count_dev, int N) {
+  extern __shared__ unsigned char smem_raw[];
+  unsigned long long* keys = reinterpret_cast<unsigned long long*>(smem_raw);
+  int32_t* vals = reinterpret_cast<int32_t*>(keys + N);
+  for (int i = threadIdx.x; i < N; i += kSortThreads) {
+    keys[i] = i < p.S ? p.skey[i] : 0ull;
+    vals[i] = i;
+  }
+  __syncthreads();
+  for (int kk = 2; kk <= N; kk <<= 1) {
+    for (int j = kk >> 1; j > 0; j >>= 1) {
+      for (int i = threadIdx.x; i < N; i += kSortThreads) {
+        const int ixj = i ^ j;
+        if (ixj > i) {
+          const unsigned long long a = keys[i], b = keys[ixj];
+          const bool swap = ((i & kk) == 0) ? (a < b) : (a > b);
+          if (swap) {
+            keys[i] = b; keys[ixj] = a;
+            const int32_t t = vals[i]; vals[i] = vals[ixj]; vals[ixj] = t;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+  // counts in rank order, each thread a contiguous run of ranks
+  const int per = (N + kSortThreads - 1) / kSortThreads;
+  const int r0 = min(N, (int)threadIdx.x * per), r1 = min(N, r0 + per);
+  long long local = 0;
+  for (int r = r0; r < r1; ++r) local += keys[r] ? p.scount[vals[r]] : 0;
+  long long total;
+  long long run = block_excl_scan<kSortThreads>(local, &total);
+  for (int r = r0; r < r1; ++r) {
+    if (r < p.S) {
+      p.sorder[r] = vals[r];
+      p.soff[r] = run;
+    }
+    run += keys[r] ? p.scount[vals[r]] : 0;
+  }
+  if (threadIdx.x == 0) {
+    const long long n_out = k < total ? k : total;
+    p.ctl[C_SEL_COUNT] = n_out;
+    p.ctl[C_SEL_TOTAL] = total;
+    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_SELECTS]), 1ull);
+    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_VICTIMS]), (unsigned long long)n_out);
+    if (k != INT64_MAX && total < k)
+      atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_SHORTFALLS]), 1ull);
+    if (fallback) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_FALLBACK]), 1ull);
+    if (count_dev) *count_dev = n_out;
+  }
+}
+
+constexpr int kEmitThreads = 256;
+
+// One CTA per rank: writes the session's resident blocks, suffix first (or
+// ascending), to its slice of the victim list, up to the global count.
+__global__ void __launch_bounds__(kEmitThreads)
+k_rank_emit(DevPool p, lv_victim* __restrict__ out) {
+  const int r = blockIdx.x;
+  const long long n_out = p.ctl[C_SEL_COUNT];
+  const long long off = p.soff[r];
+  if (off >= n_out) return;
+  const int32_t sid = p.sorder[r];
+  if (sid < 0 || sid >= p.S || p.skey[sid] == 0ull) return;
+  const int32_t nb = nblocks_of(p, sid);
+  const int32_t* row = p.table + (size_t)sid * p.maxB;
+  const bool suffix = p.within == LV_SUFFIX_FIRST;
+  long long run = 0;
+  for (int32_t q0 = 0; q0 < nb && off + run < n_out; q0 += kEmitThreads) {
+    const int32_t q = q0 + threadIdx.x;
+    const int32_t b = suffix ? nb - 1 - q : q;
+    int32_t e = -1;
+    if (q < nb) e = row[b];
+    const long long flag = e >= 0 ? 1 : 0;
+    long long chunk;
+    const long long pos = off + run + block_excl_scan<kEmitThreads>(flag, &chunk);
+    if (flag && pos < n_out) out[pos] = lv_victim{sid, b, e};
+    run += chunk;
+  }
+}
+
+// ------------------------------------------------------------ allocation
+constexpr int kAllocThreads = 1024;
+
+__global__ void __launch_bounds__(kAllocThreads)
+k_alloc(DevPool p, bool hbm, long long n, int32_t* __restrict__ out) {
+  __shared__ int ok;
+  uint32_t* bits = hbm ? p.bits_hbm : p.bits_host;
+  const long long nbits = hbm ? p.hbm_pages : p.host_pages;
+  const long long cap = hbm ? p.budget : p.host_pages;
+  long long* counter = &p.ctl[hbm ? C_HBM_ALLOC : C_HOST_ALLOC];
+  if (threadIdx.x == 0) {
+    const long long before = (long long)atomicAdd(reinterpret_cast<unsigned long long*>(counter),
+                                                  (unsigned long long)n);
+    ok = before + n <= cap;
+    if (!ok) {
+      atomicAdd(reinterpret_cast<unsigned long long*>(counter), (unsigned long long)(-n));
+      set_error(p.ctl, hbm ? LV_ERR_NO_HBM : LV_ERR_NO_HOST, n);
+    }
+  }
+  __syncthreads();
+  if (!ok) {
+    for (long long i = threadIdx.x; i < n; i += kAllocThreads) out[i] = -1;
+    return;
+  }
+  block_alloc_lowest<kAllocThreads>(bits, nbits, n, out);
+}
+
+// ------------------------------------------------------------------ copy
+constexpr int kCopyThreads = 256;
+constexpr int kCopyUnroll = 4;
+
+// Copies one sub-page: 16-byte vectors, kCopyUnroll loads in flight per thread.
+__device__ __forceinline__ void copy_subpage(const int4* __restrict__ src, int4* __restrict__ dst,
+                                             int nvec) {
+  for (int base = threadIdx.x; base < nvec; base += kCopyThreads * kCopyUnroll) {
+    int4 r[kCopyUnroll];
+#pragma unroll
+    for (int u = 0; u < kCopyUnroll; ++u) {
+      const int q = base + u * kCopyThreads;
+      if (q < nvec) r[u] = src[q];
+    }
+#pragma unroll
+    for (int u = 0; u < kCopyUnroll; ++u) {
+      const int q = base + u * kCopyThreads;
+      if (q < nvec) dst[q] = r[u];
+    }
+  }
+}
+
+// Unit u = (victim i, sub-page j): hbm_kv[j][page_i] -> host[slot_i][j].
+__global__ void __launch_bounds__(kCopyThreads)
+k_swap_out(DevPool p, const lv_victim* __restrict__ v, const int32_t* __restrict__ slots,
+           long long n, lv_remap_entry* __restrict__ commit) {
+  const long long units = n * p.J;
+  const int nvec = (int)(p.P >> 4);
+  for (long long u = blockIdx.x; u < units; u += gridDim.x) {
+    const long long i = u / p.J;
+    const int j = (int)(u % p.J);
+    const lv_victim x = v[i];
+    const int32_t slot = slots[i];
+    if (slot < 0) continue;                          // reservation failed (error already set)
+    bool ok = x.sid >= 0 && x.sid < p.S && x.blk >= 0 && x.page >= 0 && x.page < p.hbm_pages &&
+              slot < p.host_pages;
+    ok = ok && x.blk < nblocks_of(p, x.sid);
+    ok = ok && p.table[(size_t)x.sid * p.maxB + x.blk] == x.page &&
+         p.own_hbm[x.page] == owner_key(x.sid, x.blk);
+    if (j == 0 && threadIdx.x == 0) {
+      if (!ok) set_error(p.ctl, LV_ERR_STATE, i);
+      else atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PAGES_OUT]), 1ull);
+      if (commit) commit[i] = lv_remap_entry{x.sid, x.blk, ok ? -(slot + 2) : -1};
+    }
+    if (!ok) continue;
+    const int4* src = reinterpret_cast<const int4*>(p.kv[j] + (size_t)x.page * p.P);
+    int4* dst = reinterpret_cast<int4*>(p.host + ((size_t)slot * p.J + j) * p.P);
+    copy_subpage(src, dst, nvec);
+  }
+}
+
+// Unit u = (block i, sub-page j): host[slot(blk_i)][j] -> hbm_kv[j][page_i].
+__global__ void __launch_bounds__(kCopyThreads)
+k_swap_in(DevPool p, int32_t sid, const int32_t* __restrict__ blks,
+          const int32_t* __restrict__ pages, long long n, lv_remap_entry* __restrict__ commit) {
+  const long long units = n * p.J;
+  const int nvec = (int)(p.P >> 4);
+  const bool sid_ok = sid >= 0 && sid < p.S;
+  const int32_t nb = sid_ok ? nblocks_of(p, sid) : 0;
+  for (long long u = blockIdx.x; u < units; u += gridDim.x) {
+    const long long i = u / p.J;
+    const int j = (int)(u % p.J);
+    const int32_t blk = blks[i];
+    const int32_t page = pages[i];
+    if (page < 0) continue;                          // reservation failed (error already set)
+    bool ok = sid_ok && blk >= 0 && blk < nb && page < p.hbm_pages;
+    long long slot = -1;
+    if (ok) {
+      const int32_t e = p.table[(size_t)sid * p.maxB + blk];
+      slot = -(long long)e - 2;
+      ok = e <= -2 && slot < p.host_pages && p.own_host[slot] == owner_key(sid, blk);
+    }
+    if (j == 0 && threadIdx.x == 0) {
+      if (!ok) set_error(p.ctl, sid_ok ? LV_ERR_STATE : LV_ERR_BOUNDS, i);
+      else atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PAGES_IN]), 1ull);
+      if (commit) commit[i] = lv_remap_entry{sid, blk, ok ? page : -1};
+    }
+    if (!ok) continue;
+    const int4* src = reinterpret_cast<const int4*>(p.host + ((size_t)slot * p.J + j) * p.P);
+    int4* dst = reinterpret_cast<int4*>(p.kv[j] + (size_t)page * p.P);
+    copy_subpage(src, dst, nvec);
+  }
+}
+
+// ---------------------------------------------------------------- commit
+__device__ __forceinline__ bool bit_is_set(const uint32_t* bits, long long i) {
+  return (bits[i >> 5] >> (i & 31)) & 1u;
+}
+
+__global__ void k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t epoch) {
+  const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const lv_remap_entry x = e[i];
+  if (x.sid < 0 || x.sid >= p.S || x.blk < 0 || x.blk >= nblocks_of(p, x.sid)) {
+    set_error(p.ctl, LV_ERR_BOUNDS, i);
+    return;
+  }
+  const size_t ti = (size_t)x.sid * p.maxB + x.blk;
+  if (atomicExch(&p.mark[ti], epoch) == epoch) {      // the same block twice in one call
+    set_error(p.ctl, LV_ERR_DOUBLE_MAP, i);
+    return;
+  }
+  const unsigned long long key = owner_key(x.sid, x.blk);
+  if (x.loc >= 0) {
+    if (x.loc >= p.hbm_pages) { set_error(p.ctl, LV_ERR_BOUNDS, i); return; }
+    if (!bit_is_set(p.bits_hbm, x.loc) || atomicCAS(&p.own_hbm[x.loc], kOwnerNone, key) != kOwnerNone) {
+      set_error(p.ctl, LV_ERR_DOUBLE_MAP, i);
+      return;
+    }
+  } else if (x.loc <= -2) {
+    const long long h = -(long long)x.loc - 2;
+    if (h >= p.host_pages) { set_error(p.ctl, LV_ERR_BOUNDS, i); return; }
+    if (!bit_is_set(p.bits_host, h) || atomicCAS(&p.own_host[h], kOwnerNone, key) != kOwnerNone) {
+      set_error(p.ctl, LV_ERR_DOUBLE_MAP, i);
+      return;
+    }
+  } else {
+    set_error(p.ctl, LV_ERR_BOUNDS, i);
+    return;
+  }
+  const int32_t old = p.table[ti];
+  p.table[ti] = x.loc;
+  if (old >= 0 && old < p.hbm_pages) {
+    if (atomicCAS(&p.own_hbm[old], key, kOwnerNone) != key) set_error(p.ctl, LV_ERR_STATE, i);
+    atomicAnd(&p.bits_hbm[old >> 5], ~(1u << (old & 31)));
+    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HBM_ALLOC]), (unsigned long long)-1ll);
+  } else if (old <= -2 && (-(long long)old - 2) < p.host_pages) {
+    const long long h = -(long long)old - 2;
+    if (atomicCAS(&p.own_host[h], key, kOwnerNone) != key) set_error(p.ctl, LV_ERR_STATE, i);
+    atomicAnd(&p.bits_host[h >> 5], ~(1u << (h & 31)));
+    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HOST_ALLOC]), (unsigned long long)-1ll);
+  }
+  atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_REMAP]), 1ull);
+}
+
+__global__ void k_cancel(DevPool p, const int32_t* __restrict__ locs, long long n) {
+  const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const int32_t loc = locs[i];
+  uint32_t* bits;
+  unsigned long long* own;
+  long long idx;
+  int which;
+  if (loc >= 0 && loc < p.hbm_pages) {
+    bits = p.bits_hbm; own = p.own_hbm; idx = loc; which = C_HBM_ALLOC;
+  } else if (loc <= -2 && (-(long long)loc - 2) < p.host_pages) {
+    bits = p.bits_host; own = p.own_host; idx = -(long long)loc - 2; which = C_HOST_ALLOC;
+  } else {
+    set_error(p.ctl, LV_ERR_BOUNDS, i);
+    return;
+  }
+  if (own[idx] != kOwnerNone) { set_error(p.ctl, LV_ERR_STATE, i); return; }
+  const uint32_t m = 1u << (idx & 31);
+  const uint32_t before = atomicAnd(&bits[idx >> 5], ~m);
+  if (!(before & m)) { set_error(p.ctl, LV_ERR_STATE, i); return; }
+  atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[which]), (unsigned long long)-1ll);
+  atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_CANCELS]), 1ull);
+}
+
+__global__ void __launch_bounds__(kAllocThreads)
+k_append(DevPool p, int32_t sid, int32_t n_tokens, int32_t* __restrict__ pages,
+         int32_t* __restrict__ count) {
+  __shared__ long long m_s, nb_s, ctx_s;
+  if (threadIdx.x == 0) {
+    long long m = -1;
+    if (sid >= 0 && sid < p.S && n_tokens >= 0) {
+      const long long ctx = p.sess[sid].ctx_tokens;
+      const long long nb = (ctx + p.T - 1) / p.T;
+      const long long nctx = ctx + n_tokens;
+      const long long nnb = (nctx + p.T - 1) / p.T;
+      if (nnb > p.maxB || nctx > 0x7fffffffll) {
+        set_error(p.ctl, LV_ERR_BOUNDS, sid);
+      } else {
+        m = nnb - nb;
+        if (m > 0) {
+          const long long before = (long long)atomicAdd(
+              reinterpret_cast<unsigned long long*>(&p.ctl[C_HBM_ALLOC]), (unsigned long long)m);
+          if (before + m > p.budget) {
+            atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HBM_ALLOC]),
+                      (unsigned long long)(-m));
+            set_error(p.ctl, LV_ERR_NO_HBM, sid);
+            m = -1;
+          }
+        }
+      }
+      nb_s = nb;
+      ctx_s = nctx;
+    } else {
+      set_error(p.ctl, LV_ERR_BOUNDS, sid);
+    }
+    m_s = m;
+  }
+  __syncthreads();
+  const long long m = m_s;
+  if (m < 0) {
+    if (threadIdx.x == 0 && count) *count = 0;
+    return;
+  }
+  if (m > 0) block_alloc_lowest<kAllocThreads>(p.bits_hbm, p.hbm_pages, m, pages);
+  __syncthreads();
+  for (long long i = threadIdx.x; i < m; i += kAllocThreads) {
+    const int32_t pg = pages[i];
+    const int32_t b = (int32_t)(nb_s + i);
+    p.table[(size_t)sid * p.maxB + b] = pg;
+    p.own_hbm[pg] = owner_key(sid, b);
+  }
+  if (threadIdx.x == 0) {
+    p.sess[sid].ctx_tokens = (int32_t)ctx_s;
+    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_APPENDED]), (unsigned long long)m);
+    if (count) *count = (int32_t)m;
+  }
+}
+
+// ----------------------------------------------------------------- views
+__global__ void __launch_bounds__(kCensusThreads)
+k_counts(DevPool p, int32_t* __restrict__ hbm, int32_t* __restrict__ host) {
+  const int32_t s = blockIdx.x;
+  const int32_t nb = nblocks_of(p, s);
+  const int32_t* row = p.table + (size_t)s * p.maxB;
+  long long a = 0, h = 0;
+  for (int32_t b = threadIdx.x; b < nb; b += kCensusThreads) {
+    const int32_t e = row[b];
+    a += e >= 0;
+    h += e <= -2;
+  }
+  long long ta, th;
+  block_excl_scan<kCensusThreads>(a, &ta);
+  block_excl_scan<kCensusThreads>(h, &th);
+  if (threadIdx.x == 0) {
+    if (hbm) hbm[s] = (int32_t)ta;
+    if (host) host[s] = (int32_t)th;
+  }
+}
+
+__global__ void __launch_bounds__(kCensusThreads)
+k_blocks(DevPool p, int32_t sid, int32_t where, int32_t* __restrict__ out, long long* count) {
+  const int32_t nb = nblocks_of(p, sid);
+  const int32_t* row = p.table + (size_t)sid * p.maxB;
+  long long run = 0;
+  for (int32_t q0 = 0; q0 < nb; q0 += kCensusThreads) {
+    const int32_t b = q0 + threadIdx.x;
+    long long flag = 0;
+    if (b < nb) flag = where == 0 ? row[b] >= 0 : row[b] <= -2;
+    long long chunk;
+    const long long pos = run + block_excl_scan<kCensusThreads>(flag, &chunk);
+    if (flag) out[pos] = b;
+    run += chunk;
+  }
+  if (threadIdx.x == 0 && count) *count = run;
+}
+
+inline unsigned blocks_for(long long n, int threads, long long cap) {
+  long long b = (n + threads - 1) / threads;
+  if (b < 1) b = 1;
+  if (b > cap) b = cap;
+  return (unsigned)b;
+}
+
+}  // namespace
+
+// ======================================================== launch wrappers
+cudaError_t launch_import(const DevPool& p, const int32_t* placement, const int32_t* ctx,
+                          cudaStream_t s) {
+  k_import<<<blocks_for((long long)p.S * p.maxB, 256, 4096), 256, 0, s>>>(p, placement, ctx);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_check_budget(const DevPool& p, cudaStream_t s) {
+  k_check_budget<<<1, 1, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_session_set(const DevPool& p, const lv_session_state* in, int32_t first,
+                               int32_t n, cudaStream_t s) {
+  k_session_set<<<blocks_for(n, 256, 1 << 20), 256, 0, s>>>(p, in, first, n);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_events(const DevPool& p, const lv_event* ev, int64_t n, cudaStream_t s) {
+  k_events<<<blocks_for(p.S, 128, 1 << 20), 128, 0, s>>>(p, ev, n);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_select(const DevPool& p, int64_t now_us, int64_t k, bool fallback,
+                          lv_victim* out, long long* count_dev, cudaStream_t s, int /*num_sms*/) {
+  int N = 1;
+  while (N < p.S) N <<= 1;
+  const size_t smem = (size_t)N * (sizeof(unsigned long long) + sizeof(int32_t));
+  k_rank_census<<<p.S, kCensusThreads, 0, s>>>(p, now_us, fallback);
+  k_rank_sort<<<1, kSortThreads, smem, s>>>(p, k, fallback, count_dev, N);
+  k_rank_emit<<<p.S, kEmitThreads, 0, s>>>(p, out);
+  return cudaGetLastError();
+}
+
+cudaError_t configure_kernels() {
+  // the session sort keeps up to 4096 keys and ids in dynamic shared memory (48 KiB)
+  return cudaFuncSetAttribute(k_rank_sort, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * 1024);
+}
+
+cudaError_t launch_alloc(const DevPool& p, bool hbm, int64_t n, int32_t* out, cudaStream_t s) {
+  k_alloc<<<1, kAllocThreads, 0, s>>>(p, hbm, n, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_swap_out(const DevPool& p, const lv_victim* v, const int32_t* slots, int64_t n,
+                            lv_remap_entry* commit, cudaStream_t s, int num_sms) {
+  const long long units = (long long)n * p.J;
+  k_swap_out<<<blocks_for(units, 1, (long long)num_sms * 8), kCopyThreads, 0, s>>>(
+      p, v, slots, n, commit);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_swap_in(const DevPool& p, int32_t sid, const int32_t* blks, const int32_t* pages,
+                           int64_t n, lv_remap_entry* commit, cudaStream_t s, int num_sms) {
+  const long long units = (long long)n * p.J;
+  k_swap_in<<<blocks_for(units, 1, (long long)num_sms * 8), kCopyThreads, 0, s>>>(
+      p, sid, blks, pages, n, commit);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, int32_t epoch,
+                         cudaStream_t s) {
+  k_remap<<<blocks_for(n, 256, 1ll << 30), 256, 0, s>>>(p, e, n, epoch);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cudaStream_t s) {
+  k_cancel<<<blocks_for(n, 256, 1ll << 30), 256, 0, s>>>(p, locs, n);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32_t* pages,
+                          int32_t* count, cudaStream_t s) {
+  k_append<<<1, kAllocThreads, 0, s>>>(p, sid, n_tokens, pages, count);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_counts(const DevPool& p, int32_t* hbm, int32_t* host, cudaStream_t s) {
+  k_counts<<<p.S, kCensusThreads, 0, s>>>(p, hbm, host);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_blocks(const DevPool& p, int32_t sid, int32_t where, int32_t* out,
+                          long long* count, cudaStream_t s) {
+  k_blocks<<<1, kCensusThreads, 0, s>>>(p, sid, where, out, count);
+  return cudaGetLastError();
+}
+
+}  // namespace lv

@@ -1,0 +1,259 @@
+"""ctypes binding of liblv.so (include/lv.h), with the same function names.
+
+This module only marshals arguments: every step of the KV swap path runs in the
+library's CUDA kernels.  Array arguments may be torch tensors, numpy arrays or
+raw integer addresses (device or host memory, as the C ABI allows).  A
+non-``LV_OK`` status raises :class:`LvError`.  If liblv.so is missing the import
+fails loudly; there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "liblv.so")
+
+LV_OK = 0
+STATUS_NAMES = {0: "LV_OK", 1: "LV_ERR_INVALID", 2: "LV_ERR_OOM", 3: "LV_ERR_CUDA",
+                4: "LV_ERR_NO_HBM", 5: "LV_ERR_NO_HOST", 6: "LV_ERR_BOUNDS",
+                7: "LV_ERR_DOUBLE_MAP", 8: "LV_ERR_BUDGET", 9: "LV_ERR_TIMEOUT",
+                10: "LV_ERR_STATE"}
+LV_ERR_INVALID, LV_ERR_OOM, LV_ERR_CUDA, LV_ERR_NO_HBM, LV_ERR_NO_HOST = 1, 2, 3, 4, 5
+LV_ERR_BOUNDS, LV_ERR_DOUBLE_MAP, LV_ERR_BUDGET, LV_ERR_TIMEOUT, LV_ERR_STATE = 6, 7, 8, 9, 10
+LV_ALL = 2**63 - 1
+LV_SUFFIX_FIRST, LV_ASCENDING = 0, 1
+LV_PLAY_PLAYBACK, LV_PLAY_COUNTERS = 0, 1
+LV_MODE_AUTO, LV_MODE_ZERO_COPY, LV_MODE_STAGED = 0, 1, 2
+LV_SELECT_FALLBACK = 1
+LV_RUNNING, LV_IMMEDIATE, LV_RESP_OPEN, LV_DONE_VALID = 1, 2, 4, 8
+(LV_EV_TURN_BEGIN, LV_EV_TURN_END, LV_EV_PLAYBACK, LV_EV_SPEECH_START, LV_EV_BARGE_IN,
+ LV_EV_SPEECH_STOP, LV_EV_PRELOADED) = 1, 2, 3, 4, 5, 6, 7
+
+
+class LvError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = int(status)
+        super().__init__(f"{where}: {STATUS_NAMES.get(self.status, self.status)}")
+
+
+class lv_pool_desc(ctypes.Structure):
+    _fields_ = [("num_layers", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("page_tokens", ctypes.c_int32),
+                ("elem_bytes", ctypes.c_int32), ("max_sessions", ctypes.c_int32),
+                ("max_blocks", ctypes.c_int32), ("within_order", ctypes.c_int32),
+                ("hbm_pages", ctypes.c_int64), ("hbm_budget_pages", ctypes.c_int64),
+                ("host_pages", ctypes.c_int64), ("hbm_kv", ctypes.POINTER(ctypes.c_void_p)),
+                ("host_kv", ctypes.c_void_p), ("reply_prior_us", ctypes.c_int64),
+                ("protect_us", ctypes.c_int64), ("unit_us", ctypes.c_int64),
+                ("t_play_mode", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+class lv_stats(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int64) for n in (
+        "hbm_allocated", "host_allocated", "hbm_budget_pages", "host_pages", "error",
+        "error_detail", "last_select_count", "last_select_total", "selects", "victims",
+        "shortfalls", "pages_out", "pages_in", "bytes_out", "bytes_in", "remap_entries",
+        "appended_pages", "cancels", "events", "fallback_selects")]
+
+    def as_dict(self):
+        return {n: int(getattr(self, n)) for n, _ in self._fields_}
+
+
+# numpy views of the ABI's array element types
+SESSION_DTYPE = np.dtype([("ctx_tokens", "<i4"), ("flags", "<i4"), ("gen_us", "<i8"),
+                          ("play_us", "<i8"), ("t_done_us", "<i8"), ("reply_ema_us", "<i8"),
+                          ("reply_n", "<i4"), ("pad", "<i4"), ("reply_tokens", "<i8"),
+                          ("protect_until_us", "<i8")])
+EVENT_DTYPE = np.dtype([("kind", "<i4"), ("sid", "<i4"), ("t_us", "<i8"), ("a", "<i8"), ("b", "<i8")])
+VICTIM_DTYPE = np.dtype([("sid", "<i4"), ("blk", "<i4"), ("page", "<i4")])
+REMAP_DTYPE = np.dtype([("sid", "<i4"), ("blk", "<i4"), ("loc", "<i4")])
+assert SESSION_DTYPE.itemsize == 64 and EVENT_DTYPE.itemsize == 32
+assert VICTIM_DTYPE.itemsize == 12 and REMAP_DTYPE.itemsize == 12
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is missing: build it with "
+                          "paper_2606_22983_gb300._build.build() (nvcc, sm_103a)")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, i32, i64, u32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32
+    sigs = {
+        "lv_pool_create": [ctypes.POINTER(lv_pool_desc), vp, ctypes.POINTER(vp)],
+        "lv_pool_destroy": [vp, vp],
+        "lv_pool_import": [vp, vp, vp, vp],
+        "lv_session_set": [vp, vp, i32, i32, vp],
+        "lv_session_get": [vp, vp, i32, i32, vp],
+        "lv_session_events": [vp, vp, i64, vp],
+        "lv_select_victims": [vp, i64, i64, u32, vp, i64, vp, vp],
+        "lv_swap_out": [vp, vp, i64, vp, vp, i32, vp],
+        "lv_swap_in": [vp, i32, vp, i64, vp, vp, i32, vp],
+        "lv_remap": [vp, vp, i64, vp],
+        "lv_cancel": [vp, vp, i64, vp],
+        "lv_session_append": [vp, i32, i32, vp, vp, vp],
+        "lv_session_counts": [vp, vp, vp, vp],
+        "lv_session_blocks": [vp, i32, i32, vp, vp, vp],
+        "lv_read_tables": [vp, vp, vp, vp, vp],
+        "lv_sync": [vp, vp],
+        "lv_get_stats": [vp, ctypes.POINTER(lv_stats), vp],
+        "lv_clear_error": [vp, vp],
+    }
+    for name, args in sigs.items():
+        f = getattr(lib, name)
+        f.argtypes = args
+        f.restype = ctypes.c_int
+    lib.lv_pool_host_ptr.argtypes = [vp]
+    lib.lv_pool_host_ptr.restype = vp
+    lib.lv_status_str.argtypes = [ctypes.c_int]
+    lib.lv_status_str.restype = ctypes.c_char_p
+    lib.lv_version.argtypes = []
+    lib.lv_version.restype = i32
+    return lib
+
+
+_lib = _load()
+
+EXPORTED = ("lv_pool_create", "lv_pool_destroy", "lv_pool_host_ptr", "lv_pool_import",
+            "lv_session_set", "lv_session_get", "lv_session_events", "lv_select_victims",
+            "lv_swap_out", "lv_swap_in", "lv_remap", "lv_cancel", "lv_session_append",
+            "lv_session_counts", "lv_session_blocks", "lv_read_tables", "lv_sync",
+            "lv_get_stats", "lv_clear_error", "lv_status_str", "lv_version")
+
+
+def lib():
+    return _lib
+
+
+def ptr(x):
+    """Address of a tensor / array / integer, or None."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "data_ptr"):
+        return x.data_ptr()
+    if isinstance(x, np.ndarray):
+        if not x.flags["C_CONTIGUOUS"]:
+            raise ValueError("array arguments must be C-contiguous")
+        return x.ctypes.data
+    if isinstance(x, ctypes.Array):
+        return ctypes.addressof(x)
+    raise TypeError(f"cannot pass {type(x).__name__} as an array argument")
+
+
+def stream_handle(stream):
+    """cudaStream_t of a torch stream (None: the current stream of the current device)."""
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream()
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(status, where):
+    if status != LV_OK:
+        raise LvError(status, where)
+
+
+# ----------------------------------------------------------------- entry points
+def lv_pool_create(desc: lv_pool_desc, stream=None):
+    h = ctypes.c_void_p()
+    _check(_lib.lv_pool_create(ctypes.byref(desc), stream_handle(stream), ctypes.byref(h)),
+           "lv_pool_create")
+    return h.value
+
+
+def lv_pool_destroy(pool, stream=None):
+    _check(_lib.lv_pool_destroy(pool, stream_handle(stream)), "lv_pool_destroy")
+
+
+def lv_pool_host_ptr(pool) -> int:
+    return _lib.lv_pool_host_ptr(pool)
+
+
+def lv_pool_import(pool, placement, ctx_tokens, stream=None):
+    _check(_lib.lv_pool_import(pool, ptr(placement), ptr(ctx_tokens), stream_handle(stream)),
+           "lv_pool_import")
+
+
+def lv_session_set(pool, states, first, n, stream=None):
+    _check(_lib.lv_session_set(pool, ptr(states), first, n, stream_handle(stream)), "lv_session_set")
+
+
+def lv_session_get(pool, out, first, n, stream=None):
+    _check(_lib.lv_session_get(pool, ptr(out), first, n, stream_handle(stream)), "lv_session_get")
+
+
+def lv_session_events(pool, events, n, stream=None):
+    _check(_lib.lv_session_events(pool, ptr(events), n, stream_handle(stream)), "lv_session_events")
+
+
+def lv_select_victims(pool, now_us, k, flags, out, capacity, count_out, stream=None):
+    _check(_lib.lv_select_victims(pool, now_us, k, flags, ptr(out), capacity, ptr(count_out),
+                                  stream_handle(stream)), "lv_select_victims")
+
+
+def lv_swap_out(pool, victims, n, slots_out, commit_out, mode=LV_MODE_AUTO, stream=None):
+    _check(_lib.lv_swap_out(pool, ptr(victims), n, ptr(slots_out), ptr(commit_out), mode,
+                            stream_handle(stream)), "lv_swap_out")
+
+
+def lv_swap_in(pool, sid, blks, n, pages_out, commit_out, mode=LV_MODE_AUTO, stream=None):
+    _check(_lib.lv_swap_in(pool, sid, ptr(blks), n, ptr(pages_out), ptr(commit_out), mode,
+                           stream_handle(stream)), "lv_swap_in")
+
+
+def lv_remap(pool, entries, n, stream=None):
+    _check(_lib.lv_remap(pool, ptr(entries), n, stream_handle(stream)), "lv_remap")
+
+
+def lv_cancel(pool, locs, n, stream=None):
+    _check(_lib.lv_cancel(pool, ptr(locs), n, stream_handle(stream)), "lv_cancel")
+
+
+def lv_session_append(pool, sid, n_tokens, pages_out, count_out, stream=None):
+    _check(_lib.lv_session_append(pool, sid, n_tokens, ptr(pages_out), ptr(count_out),
+                                  stream_handle(stream)), "lv_session_append")
+
+
+def lv_session_counts(pool, hbm_blocks, host_blocks, stream=None):
+    _check(_lib.lv_session_counts(pool, ptr(hbm_blocks), ptr(host_blocks), stream_handle(stream)),
+           "lv_session_counts")
+
+
+def lv_session_blocks(pool, sid, where, blks_out, count_out, stream=None):
+    _check(_lib.lv_session_blocks(pool, sid, where, ptr(blks_out), ptr(count_out),
+                                  stream_handle(stream)), "lv_session_blocks")
+
+
+def lv_read_tables(pool, tables, hbm_owner, host_owner, stream=None):
+    _check(_lib.lv_read_tables(pool, ptr(tables), ptr(hbm_owner), ptr(host_owner),
+                               stream_handle(stream)), "lv_read_tables")
+
+
+def lv_sync(pool, stream=None, raise_on_error=True) -> int:
+    st = _lib.lv_sync(pool, stream_handle(stream))
+    if raise_on_error:
+        _check(st, "lv_sync")
+    return st
+
+
+def lv_get_stats(pool, stream=None) -> dict:
+    s = lv_stats()
+    _check(_lib.lv_get_stats(pool, ctypes.byref(s), stream_handle(stream)), "lv_get_stats")
+    return s.as_dict()
+
+
+def lv_clear_error(pool, stream=None):
+    _check(_lib.lv_clear_error(pool, stream_handle(stream)), "lv_clear_error")
+
+
+def lv_status_str(status: int) -> str:
+    return _lib.lv_status_str(status).decode()
+
+
+def lv_version() -> int:
+    return _lib.lv_version()

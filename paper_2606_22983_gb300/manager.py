@@ -1,0 +1,185 @@
+"""The KV manager's turn and preload procedure over liblv (Sections 5.1 and 5.2).
+
+Consumes monitor event scripts (records ``(t_us, kind, sid, a, b, c, d)``):
+
+  kind 1 TURN(sid, a=append_tokens, b=reply_audio_us, c=reply_tokens)
+  kind 2 TURN_ANY(d=row of perms): the first session in perms[d] with blocks in
+         the host tier takes the turn (perms[d][0] when none has)
+  kind 3 PLAYBACK(sid, a=delta_us)    kind 4 SPEECH_START(sid)
+  kind 5 BARGE_IN(sid)                kind 6 SPEECH_STOP(sid)
+
+A turn makes the session fully resident (a synchronous foreground load),
+grows its context, then records the reply.  Speech start and barge-in trigger a
+best-effort preload of the session's host blocks.  Making a session resident
+with ``need`` missing pages first evicts exactly ``k = need - free`` pages in
+the next-use order (foreground turns may also take protected, non-running KV
+after every normally eligible block; a preload may not), swaps them out, commits,
+then swaps the host blocks in (ascending block order) and commits.  A preload
+that finds fewer than k victims is skipped; a completed one protects the
+warmed KV for the pool's protection window.
+
+Every step runs in liblv's kernels; this class only decides which calls to
+make, reading back the few counts it needs to decide (free pages, host
+blocks, victims found).
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import lv
+from .pool import KVPool
+
+EV_TURN, EV_TURN_ANY, EV_PLAYBACK, EV_SPEECH_START, EV_BARGE_IN, EV_SPEECH_STOP = 1, 2, 3, 4, 5, 6
+
+_STATE_EVENT = {EV_PLAYBACK: lv.LV_EV_PLAYBACK, EV_SPEECH_START: lv.LV_EV_SPEECH_START,
+                EV_BARGE_IN: lv.LV_EV_BARGE_IN, EV_SPEECH_STOP: lv.LV_EV_SPEECH_STOP}
+
+
+def _event(kind, sid, t, a=0, b=0):
+    e = np.zeros(1, dtype=lv.EVENT_DTYPE)
+    e["kind"], e["sid"], e["t_us"], e["a"], e["b"] = kind, sid, t, a, b
+    return e
+
+
+class KVManager:
+    def __init__(self, pool: KVPool, perms=None, on_append=None, rank_on="none", admit=None,
+                 mode=lv.LV_MODE_AUTO, record=True):
+        self.pool = pool
+        self.perms = perms
+        self.on_append = on_append      # callback(sid, old_ctx, new_ctx, pages) after growth
+        self.rank_on = rank_on          # 'all' events, 'turns' only, or 'none'
+        self.admit = admit              # callback(manager, sid, now, n_host_blocks) -> bool
+        self.mode = mode
+        self.record = record
+        self.counters = dict(victims=0, pages_out=0, pages_in=0, preloads=0,
+                             preload_skipped=0, turns=0, sync_loads=0, appended=0)
+        self.bytes_moved = 0
+        self.timer = None               # optional start(name) / stop(name, bytes) hooks
+        self.last_readback_bytes = 0    # bytes of lists read back to the host by the last step
+
+    # ------------------------------------------------------------- queries
+    def free_budget(self) -> int:
+        st = self.pool.stats()
+        if st["error"]:
+            raise lv.LvError(st["error"], "device error")
+        return st["hbm_budget_pages"] - st["hbm_allocated"]
+
+    def host_blocks(self, sid):
+        return self.pool.blocks(sid, 1)
+
+    def ctx_tokens(self, sid) -> int:
+        return int(self.pool.get_sessions()["ctx_tokens"][sid])
+
+    # ------------------------------------------------------------ movement
+    def make_resident(self, sid, now_us, append_tokens, foreground, rec):
+        pool = self.pool
+        hblk, nh = self.host_blocks(sid)
+        new_blocks = 0
+        if append_tokens:
+            ctx = self.ctx_tokens(sid)
+            T = pool.T
+            new_blocks = -(-(ctx + append_tokens) // T) - (-(-ctx // T))
+        need = nh + new_blocks
+        k = max(0, need - self.free_budget())
+        rec["k"] = k
+        if k > 0:
+            flags = lv.LV_SELECT_FALLBACK if foreground else 0
+            victims, n = pool.select(now_us, k, flags)
+            if self.record:
+                rec["victims"] = victims.cpu().numpy().astype(np.int64)
+                self.last_readback_bytes += n * 12
+            if n < k:
+                if foreground:
+                    raise lv.LvError(lv.LV_ERR_NO_HBM, f"turn of session {sid} needs {k} victims, {n} found")
+                return False
+            if self.timer:
+                self.timer.start("swap_out")
+            slots, commit = pool.swap_out(victims, n, self.mode)
+            if self.timer:
+                self.timer.stop("swap_out", n * pool.J * pool.P)
+            pool.remap(commit, n)
+            if self.record:
+                rec["slots"] = slots.cpu().numpy().astype(np.int64)
+                self.last_readback_bytes += n * 4
+            self.counters["victims"] += n
+            self.counters["pages_out"] += n
+            self.bytes_moved += n * pool.J * pool.P
+        if nh:
+            if self.timer:
+                self.timer.start("swap_in")
+            pages, commit = pool.swap_in(sid, hblk, nh, self.mode)
+            if self.timer:
+                self.timer.stop("swap_in", nh * pool.J * pool.P)
+            pool.remap(commit, nh)
+            if self.record:
+                rec["in_blocks"] = hblk.cpu().numpy().astype(np.int64)
+                rec["in_pages"] = pages.cpu().numpy().astype(np.int64)
+                self.last_readback_bytes += nh * 8
+            self.counters["pages_in"] += nh
+            self.bytes_moved += nh * pool.J * pool.P
+        if append_tokens:
+            old_ctx = self.ctx_tokens(sid)
+            pages = pool.append(sid, append_tokens)
+            if self.record:
+                rec["append_pages"] = pages.cpu().numpy().astype(np.int64)
+            self.counters["appended"] += int(pages.numel())
+            if self.on_append is not None:
+                self.on_append(sid, old_ctx, old_ctx + append_tokens)
+        return True
+
+    def preload(self, sid, now_us, rec):
+        _, nh = self.host_blocks(sid)
+        if nh == 0:
+            return
+        if self.admit is not None and not self.admit(self, sid, now_us, nh):
+            self.counters["preload_skipped"] += 1
+            rec["preload"] = "skipped"
+            return
+        if self.make_resident(sid, now_us, 0, foreground=False, rec=rec):
+            self.pool.events(_event(lv.LV_EV_PRELOADED, sid, now_us))
+            self.counters["preloads"] += 1
+            rec["preload"] = "done"
+        else:
+            self.counters["preload_skipped"] += 1
+            rec["preload"] = "skipped"
+
+    def turn_target(self, row):
+        _, host = self.pool.counts()
+        for s in self.perms[row]:
+            if host[int(s)] > 0:
+                return int(s)
+        return int(self.perms[row][0])
+
+    # --------------------------------------------------------------- events
+    def step(self, ev, index=None):
+        t, kind, sid, a, b, c, d = (int(x) for x in ev)
+        self.last_readback_bytes = 0
+        rec = {"i": index, "t": t, "kind": kind}
+        pool = self.pool
+        if kind in _STATE_EVENT:
+            pool.events(_event(_STATE_EVENT[kind], sid, t, a))
+            if kind in (EV_SPEECH_START, EV_BARGE_IN):
+                self.preload(sid, t, rec)
+        elif kind in (EV_TURN, EV_TURN_ANY):
+            if kind == EV_TURN_ANY:
+                sid = self.turn_target(d)
+            pool.events(_event(lv.LV_EV_TURN_BEGIN, sid, t))
+            if self.host_blocks(sid)[1]:
+                self.counters["sync_loads"] += 1
+            self.make_resident(sid, t, a, foreground=True, rec=rec)
+            pool.events(_event(lv.LV_EV_TURN_END, sid, t, b, c))
+            self.counters["turns"] += 1
+        else:
+            raise ValueError(f"unknown script event kind {kind}")
+        rec["sid"] = sid
+        if self.rank_on == "all" or (self.rank_on == "turns" and kind in (EV_TURN, EV_TURN_ANY)):
+            order, n = pool.select(t, lv.LV_ALL, 0)
+            rec["order"] = order.cpu().numpy().astype(np.int64)
+        return rec
+
+    def playback_batch(self, t_us, sids, deltas):
+        """Many PLAYBACK reports at once (one kernel launch)."""
+        ev = np.zeros(len(sids), dtype=lv.EVENT_DTYPE)
+        ev["kind"], ev["sid"], ev["t_us"], ev["a"] = lv.LV_EV_PLAYBACK, sids, t_us, deltas
+        self.pool.events(ev)

@@ -1,0 +1,120 @@
+"""The C ABI without a GPU: the library builds, loads and exports every function
+include/lv.h declares, and the binding's struct layouts match the header's."""
+import ctypes
+import os
+import re
+import subprocess
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "lv.h")
+
+
+def _declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(lv_[a-z_]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2606_22983_gb300 import build
+    path = build()
+    return ctypes.CDLL(path)
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = _declared_functions()
+    assert len(names) >= 20
+    for n in names:
+        assert hasattr(lib, n), n
+    out = subprocess.run(["nm", "-D", "--defined-only", os.path.join(ROOT, "paper_2606_22983_gb300", "liblv.so")],
+                         capture_output=True, text=True).stdout
+    exported = set(re.findall(r" T (lv_[a-z_]+)", out))
+    assert set(names) <= exported
+
+
+def test_binding_names_match_header():
+    from paper_2606_22983_gb300 import lv
+    assert sorted(lv.EXPORTED) == _declared_functions()
+    for n in lv.EXPORTED:
+        assert callable(getattr(lv, n)), n
+
+
+def test_struct_layouts_match_header(tmp_path):
+    from paper_2606_22983_gb300 import lv
+    src = tmp_path / "layout.c"
+    src.write_text(r'''
+#include <stdio.h>
+#include <stddef.h>
+#include "lv.h"
+#define F(T, m) printf(#T "." #m " %zu %zu\n", offsetof(T, m), sizeof(((T*)0)->m))
+int main(void) {
+  printf("sizeof lv_pool_desc %zu\n", sizeof(lv_pool_desc));
+  printf("sizeof lv_session_state %zu\n", sizeof(lv_session_state));
+  printf("sizeof lv_event %zu\n", sizeof(lv_event));
+  printf("sizeof lv_victim %zu\n", sizeof(lv_victim));
+  printf("sizeof lv_remap_entry %zu\n", sizeof(lv_remap_entry));
+  printf("sizeof lv_stats %zu\n", sizeof(lv_stats));
+  F(lv_session_state, ctx_tokens); F(lv_session_state, flags); F(lv_session_state, gen_us);
+  F(lv_session_state, play_us); F(lv_session_state, t_done_us); F(lv_session_state, reply_ema_us);
+  F(lv_session_state, reply_n); F(lv_session_state, reply_tokens); F(lv_session_state, protect_until_us);
+  F(lv_event, kind); F(lv_event, sid); F(lv_event, t_us); F(lv_event, a); F(lv_event, b);
+  F(lv_pool_desc, hbm_pages); F(lv_pool_desc, hbm_kv); F(lv_pool_desc, host_kv);
+  F(lv_pool_desc, reply_prior_us); F(lv_pool_desc, t_play_mode); F(lv_pool_desc, reserved);
+  return 0;
+}
+''')
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-std=c99", "-Wall", "-Werror", "-I", os.path.dirname(HEADER), str(src),
+                    "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout
+    got = {}
+    for line in out.splitlines():
+        parts = line.split()
+        if parts[0] == "sizeof":
+            got[parts[1]] = int(parts[2])
+        else:
+            got[parts[0]] = (int(parts[1]), int(parts[2]))
+    assert got["lv_session_state"] == lv.SESSION_DTYPE.itemsize
+    assert got["lv_event"] == lv.EVENT_DTYPE.itemsize
+    assert got["lv_victim"] == lv.VICTIM_DTYPE.itemsize
+    assert got["lv_remap_entry"] == lv.REMAP_DTYPE.itemsize
+    assert got["lv_pool_desc"] == ctypes.sizeof(lv.lv_pool_desc)
+    assert got["lv_stats"] == ctypes.sizeof(lv.lv_stats)
+    for name in lv.SESSION_DTYPE.names:
+        if name == "pad":
+            continue
+        off, size = got[f"lv_session_state.{name}"]
+        assert lv.SESSION_DTYPE.fields[name][1] == off and lv.SESSION_DTYPE.fields[name][0].itemsize == size
+    for name in lv.EVENT_DTYPE.names:
+        off, size = got[f"lv_event.{name}"]
+        assert lv.EVENT_DTYPE.fields[name][1] == off
+    for name in ("hbm_pages", "hbm_kv", "host_kv", "reply_prior_us", "t_play_mode", "reserved"):
+        assert getattr(lv.lv_pool_desc, name).offset == got[f"lv_pool_desc.{name}"][0], name
+
+
+def test_status_strings_and_argument_checks(lib):
+    from paper_2606_22983_gb300 import lv
+    for code, name in lv.STATUS_NAMES.items():
+        assert lv.lv_status_str(code) == name
+    assert lv.lv_version() >= 1
+    # argument checks that need no device: a NULL descriptor / NULL out pointer
+    L = lv.lib()
+    h = ctypes.c_void_p()
+    assert L.lv_pool_create(None, None, ctypes.byref(h)) == lv.LV_ERR_INVALID
+    assert L.lv_pool_create(None, None, None) == lv.LV_ERR_INVALID
+    assert L.lv_sync(None, None) == lv.LV_ERR_INVALID
+    assert L.lv_remap(None, None, 0, None) == lv.LV_ERR_INVALID
+
+
+def test_no_oracle_in_product_package():
+    pkg = os.path.join(ROOT, "paper_2606_22983_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h", ".cpp")):
+                text = open(os.path.join(dirpath, f)).read()
+                assert not re.search(r"^\s*(from|import)\s+oracle\b", text, re.M), f
+                assert "oracle/" not in text, f
