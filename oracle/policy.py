@@ -16,7 +16,8 @@ Readings:
     be an exact wall-clock prediction" (Section 5.1).
   * T_play in the progress-counter mode is the current reply's length in
     units times ``unit_us`` while the reply is unfinished, else 0 ("longer
-    unfinished responses" mean later reuse, Section 5.1).
+    unfinished responses" mean later reuse, Section 5.1); like the playback
+    horizon it is never negative.
   * Protection holds against *normal* eviction only (Section 5.1), and warmed
     KV may be "evicted before reuse" (Section 5.2).  With ``fallback`` set (a
     foreground turn that cannot otherwise run), protected sessions that are
@@ -40,7 +41,7 @@ def t_next(st: SessionState, mode: int, reply_prior_us: int, unit_us: int) -> in
     if mode == MODE_PLAYBACK:
         t_play = max(0, st.gen_us - st.play_us)            # remaining playback horizon
     elif mode == MODE_COUNTERS:
-        t_play = st.reply_tokens * unit_us if (st.flags & RESP_OPEN) else 0
+        t_play = max(0, st.reply_tokens * unit_us) if (st.flags & RESP_OPEN) else 0
     else:
         raise ValueError(f"unknown T_play mode {mode}")
     # per-session moving average when available, workload-level prior otherwise
