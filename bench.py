@@ -332,13 +332,17 @@ def ours(args, torch):
 
 
 def _profiled_traffic(kernel, bytes_per_launch):
-    """DRAM bytes per launch from the committed ncu summary, when it covers this kernel."""
-    path = os.path.join(ROOT, "profiles", "traffic.json")
+    """DRAM bytes per launch from the committed ncu summary, or None when that
+    summary does not cover this kernel or the kernel source changed since."""
+    import hashlib
     try:
-        with open(path) as f:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
             d = json.load(f)
-        e = d[kernel]
-        return round(e["dram_bytes_per_payload_byte"] * bytes_per_launch)
+        src = os.path.join(ROOT, "paper_2606_22983_gb300", "csrc", "lv_kernels.cu")
+        with open(src, "rb") as f:
+            if hashlib.sha256(f.read()).hexdigest() != d["kernel_source_sha256"]:
+                return None
+        return round(d[kernel]["dram_bytes_per_payload_byte"] * bytes_per_launch)
     except (OSError, KeyError, ValueError):
         return None
 
