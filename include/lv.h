@@ -293,6 +293,54 @@ lv_status lv_session_blocks(lv_pool* pool, int32_t sid, int32_t where, int32_t* 
 lv_status lv_read_tables(lv_pool* pool, int32_t* tables, int64_t* hbm_owner,
                          int64_t* host_owner, lv_stream stream);
 
+/* ------------------------------------------- ranking without allocation */
+
+/* The paper has no counterpart to this entry point; it exists for callers of
+   this library that must not allocate GPU memory while they rank victims -- an
+   engine that has already given nearly all free HBM to its KV pages, where a
+   further cudaMalloc can fail or fragment that reservation, or a
+   latency-critical scheduler thread, where cudaMalloc / cudaFree can
+   synchronise the device.
+
+   lv_select_victims_noalloc computes exactly what lv_select_victims computes
+   (same order, same count, same fallback tier), but from a session table and
+   block tables that the caller passes in, without a pool: sessions is
+   lv_session_state [num_sessions] (ctx_tokens gives each session's block
+   count), tables is int32 [num_sessions][max_blocks] in the block-table
+   encoding above.  Both, and out (lv_victim [capacity]) and count_out (int64,
+   may be NULL), must be device memory or mapped page-locked host memory;
+   pageable host pointers are rejected with LV_ERR_INVALID because staging them
+   would need an allocation.
+
+   Its working memory is one array of LV_NOALLOC_MAX_SESSIONS x 24 bytes plus
+   256 bytes (96.25 KiB) compiled into liblv as device memory: every GPU that
+   loads the library holds it until the process exits.  num_sessions above
+   LV_NOALLOC_MAX_SESSIONS is rejected with LV_ERR_INVALID.  The call allocates
+   nothing (no cudaMalloc, cudaFree or allocating library routine).  The first
+   call on a device looks up that array's device address (cudaGetSymbolAddress)
+   and sets a kernel attribute, so make the first call on each device before
+   any stream capture.  All calls on a device share the one array and each call
+   starts by clearing its counters: calls whose execution overlaps on the GPU
+   (two streams, or two host threads) race and may return wrong victims, so
+   order them, for example on one stream. */
+#define LV_NOALLOC_MAX_SESSIONS 4096
+
+typedef struct lv_rank_params {
+  int32_t num_sessions;        /* 1..LV_NOALLOC_MAX_SESSIONS */
+  int32_t max_blocks;          /* row length of the block tables, 1..65536 */
+  int32_t page_tokens;         /* T */
+  int32_t within_order;        /* LV_SUFFIX_FIRST or LV_ASCENDING */
+  int32_t t_play_mode;         /* LV_PLAY_PLAYBACK or LV_PLAY_COUNTERS */
+  uint32_t flags;              /* 0 or LV_SELECT_FALLBACK */
+  int64_t reply_prior_us;      /* >= 0 */
+  int64_t unit_us;             /* 1..2^31 */
+} lv_rank_params;
+
+lv_status lv_select_victims_noalloc(const lv_rank_params* params, const lv_session_state* sessions,
+                                    const int32_t* tables, int64_t now_us, int64_t k,
+                                    lv_victim* out, int64_t capacity, int64_t* count_out,
+                                    lv_stream stream);
+
 /* ------------------------------------------------------------- status */
 
 /* Synchronous: waits for `stream`, returns the sticky device error (LV_OK if

@@ -62,6 +62,15 @@ class lv_stats(ctypes.Structure):
         return {n: int(getattr(self, n)) for n, _ in self._fields_}
 
 
+class lv_rank_params(ctypes.Structure):
+    _fields_ = [("num_sessions", ctypes.c_int32), ("max_blocks", ctypes.c_int32),
+                ("page_tokens", ctypes.c_int32), ("within_order", ctypes.c_int32),
+                ("t_play_mode", ctypes.c_int32), ("flags", ctypes.c_uint32),
+                ("reply_prior_us", ctypes.c_int64), ("unit_us", ctypes.c_int64)]
+
+
+LV_NOALLOC_MAX_SESSIONS = 4096
+
 # numpy views of the ABI's array element types
 SESSION_DTYPE = np.dtype([("ctx_tokens", "<i4"), ("flags", "<i4"), ("gen_us", "<i8"),
                           ("play_us", "<i8"), ("t_done_us", "<i8"), ("reply_ema_us", "<i8"),
@@ -99,6 +108,8 @@ def _load():
         "lv_sync": [vp, vp],
         "lv_get_stats": [vp, ctypes.POINTER(lv_stats), vp],
         "lv_clear_error": [vp, vp],
+        "lv_select_victims_noalloc": [ctypes.POINTER(lv_rank_params), vp, vp, i64, i64, vp, i64,
+                                      vp, vp],
     }
     for name, args in sigs.items():
         f = getattr(lib, name)
@@ -119,7 +130,8 @@ EXPORTED = ("lv_pool_create", "lv_pool_destroy", "lv_pool_host_ptr", "lv_pool_im
             "lv_session_set", "lv_session_get", "lv_session_events", "lv_select_victims",
             "lv_swap_out", "lv_swap_in", "lv_remap", "lv_cancel", "lv_session_append",
             "lv_session_counts", "lv_session_blocks", "lv_read_tables", "lv_sync",
-            "lv_get_stats", "lv_clear_error", "lv_status_str", "lv_version")
+            "lv_get_stats", "lv_clear_error", "lv_status_str", "lv_version",
+            "lv_select_victims_noalloc")
 
 
 def lib():
@@ -249,6 +261,13 @@ def lv_get_stats(pool, stream=None) -> dict:
 
 def lv_clear_error(pool, stream=None):
     _check(_lib.lv_clear_error(pool, stream_handle(stream)), "lv_clear_error")
+
+
+def lv_select_victims_noalloc(params: lv_rank_params, sessions, tables, now_us, k, out, capacity,
+                              count_out, stream=None):
+    _check(_lib.lv_select_victims_noalloc(ctypes.byref(params), ptr(sessions), ptr(tables), now_us,
+                                          k, ptr(out), capacity, ptr(count_out),
+                                          stream_handle(stream)), "lv_select_victims_noalloc")
 
 
 def lv_status_str(status: int) -> str:
