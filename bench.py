@@ -220,7 +220,8 @@ def ours(args, torch):
     pool = pool_for(wl)
     fill_random(pool, args.seed + rank)
     page_bytes = pool.J * pool.P
-    gm = KVManager(pool, perms=wl.perms, rank_on="none", mode=args.mode, record=False)
+    gm = KVManager(pool, perms=wl.perms, rank_on="none", mode=args.mode, record=False,
+                   exchange=not args.sequential)
     timer = KernelTimer(torch)
     gm.timer = timer
     S = wl.spec.n_sessions
@@ -293,7 +294,8 @@ def ours(args, torch):
         # roofline of the dominant kernel (longest total time)
         dom = max(kern, key=lambda n: kern[n]["total_ms"])
         dk = kern[dom]
-        peak = peaks["d2h"] if dom == "swap_out" else peaks["h2d"]
+        peak = {"swap_out": peaks["d2h"], "swap_in": peaks["h2d"]}.get(dom, peaks.get("bidir"))
+        peak_dir = {"swap_out": "D2H", "swap_in": "H2D"}.get(dom, "D2H and H2D concurrently")
         traffic = _profiled_traffic(dom, dk["bytes_per_launch"])
         line = {
             "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": ws,
@@ -305,6 +307,7 @@ def ours(args, torch):
                                    "budget, one turn = evict + reload",
                        "hbm_budget_pages": wl.spec.hbm_budget_pages, "host_pages": wl.spec.host_pages,
                        "mode": {0: "auto", 1: "zero_copy", 2: "staged"}[args.mode],
+                       "path": "sequential" if args.sequential else "exchange",
                        "l2": "inputs larger than L2 (mean turn moves "
                              f"{mean_turn / 1e6:.0f} MB each way from a 40 GB pool)",
                        "parallelism": f"replicas x{ws}"},
@@ -315,8 +318,7 @@ def ours(args, torch):
                          "peak": round(peak, 1), "unit": "GB/s", "frac": round(dk["gbs"] / peak, 3),
                          "traffic": traffic,
                          "peak_source": "same-run contiguous page-locked cudaMemcpyAsync "
-                                        f"({'D2H' if dom == 'swap_out' else 'H2D'}, "
-                                        "mean-turn byte count)"},
+                                        f"({peak_dir}, mean-turn byte count)"},
             "kernels": {n: {k: round(v, 3) for k, v in d.items()} for n, d in kern.items()},
             "e2e": {"value": round(e2e_value, 3), "unit": UNIT,
                     "h2d_bytes_per_step": int(h2d / K), "d2h_bytes_per_step": int(d2h / K)},
@@ -429,6 +431,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--mode", type=int, default=0, help="0 auto, 1 zero-copy, 2 staged")
+    ap.add_argument("--sequential", action="store_true",
+                    help="swap-out, commit, swap-in, commit one after the other (no exchange)")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")

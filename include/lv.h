@@ -253,6 +253,27 @@ lv_status lv_swap_in(lv_pool* pool, int32_t sid, const int32_t* blks, int64_t n,
                      int32_t* pages_out, lv_remap_entry* commit_out, int32_t mode,
                      lv_stream stream);
 
+/* Section 5.1 (evict "until enough HBM is released") followed by the load of
+   Section 5.2 / Section 6, as one step: evicts n_out victims to the host tier
+   and loads n_in host-resident blocks of session sid, committing both.  The
+   result -- slots_out (int32 [n_out], victim order), pages_out (int32 [n_in],
+   list order), block and owner tables, bitmaps, counters, bytes -- is exactly
+   that of lv_swap_out, lv_remap (its commits), lv_swap_in, lv_remap (its
+   commits) issued one after the other: victims take the lowest free host
+   slots before any slot is freed, incoming blocks take the lowest free HBM
+   pages after the victims' pages are freed.  All metadata is decided first by
+   one small kernel; then one copy kernel moves both directions together (an
+   incoming block that lands on a victim's old page is copied by the same
+   thread right after it read the old bytes), so the host link carries data
+   both ways at once.  Either list may be empty.  The whole call is validated
+   before anything changes: on LV_ERR_STATE / LV_ERR_BOUNDS (a victim not
+   resident where it says, a block not in the host tier, a block listed twice),
+   LV_ERR_NO_HOST or LV_ERR_NO_HBM (device-detected) nothing is reserved,
+   committed or copied, and the outputs are -1. */
+lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_out, int32_t sid,
+                           const int32_t* blks, int64_t n_in, int32_t* slots_out,
+                           int32_t* pages_out, int32_t mode, lv_stream stream);
+
 /* Section 6 (side tables) and Section 5.2 ("preloading affects latency but not
    correctness"): commits n entries.  For each, the new location must be a
    reservation not yet owned; it becomes owned by (sid, blk), the block table

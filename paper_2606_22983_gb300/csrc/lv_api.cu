@@ -1,6 +1,7 @@
 // C-ABI entry points of liblv (see include/lv.h): argument checks, device
 // metadata, staging of host-pointer arguments, and kernel launches.
 #include <cstdint>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 #include <vector>
@@ -12,6 +13,7 @@ struct lv_pool {
   int device = 0;
   int num_sms = 0;
   int32_t epoch = 0;
+  int exchange_ctas = 0;           // grid of the exchange copy kernel
   bool own_host = false;
   void* host_base = nullptr;       // host-visible address of the host pool
   std::vector<void*> dev_allocs;
@@ -246,7 +248,8 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       (st = dev_alloc(pool, &d.skey, d.S)) != LV_OK ||
       (st = dev_alloc(pool, &d.scount, d.S)) != LV_OK ||
       (st = dev_alloc(pool, &d.sorder, d.S)) != LV_OK ||
-      (st = dev_alloc(pool, &d.soff, d.S)) != LV_OK)
+      (st = dev_alloc(pool, &d.soff, d.S)) != LV_OK ||
+      (st = dev_alloc(pool, &d.page_tag, (size_t)d.hbm_pages)) != LV_OK)
     return fail(st);
   d.kv = kv_dev;
   if (cudaMemcpyAsync(kv_dev, kv.data(), d.J * sizeof(uint8_t*), cudaMemcpyHostToDevice, s) != cudaSuccess ||
@@ -257,8 +260,14 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       cudaMemsetAsync(d.own_host, 0xff, (size_t)(d.host_pages ? d.host_pages : 1) * 8, s) != cudaSuccess ||
       cudaMemsetAsync(d.bits_hbm, 0, wh * 4, s) != cudaSuccess ||
       cudaMemsetAsync(d.bits_host, 0, (wo ? wo : 1) * 4, s) != cudaSuccess ||
-      cudaMemsetAsync(d.ctl, 0, lv::C_N * sizeof(long long), s) != cudaSuccess)
+      cudaMemsetAsync(d.ctl, 0, lv::C_N * sizeof(long long), s) != cudaSuccess ||
+      cudaMemsetAsync(d.page_tag, 0, (size_t)d.hbm_pages * 8, s) != cudaSuccess)
     return fail(LV_ERR_CUDA);
+  pool->exchange_ctas = pool->num_sms;   // one CTA per SM measured best for both directions at once
+  if (const char* env = std::getenv("LV_EXCHANGE_CTAS_PER_SM")) {
+    const int per = std::atoi(env);
+    if (per >= 1 && per <= 16) pool->exchange_ctas = pool->num_sms * per;
+  }
 
   if (lv::configure_kernels() != cudaSuccess) return fail(LV_ERR_CUDA);
   cudaMemPoolProps props{};
@@ -439,6 +448,41 @@ lv_status lv_swap_in(lv_pool* pool, int32_t sid, const int32_t* blks, int64_t n,
     LV_TRY(lv::launch_alloc(pool->d, true, n, pages, s));
     LV_TRY(lv::launch_swap_in(pool->d, sid, static_cast<const int32_t*>(bin), pages, n,
                               static_cast<lv_remap_entry*>(cdev), s, pool->num_sms));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_out, int32_t sid,
+                           const int32_t* blks, int64_t n_in, int32_t* slots_out, int32_t* pages_out,
+                           int32_t mode, lv_stream stream) {
+  if (!pool || n_out < 0 || n_in < 0 || n_out > 0x7fffffffll || n_in > 0x7fffffffll ||
+      (n_out > 0 && !victims) || (n_in > 0 && !blks))
+    return LV_ERR_INVALID;
+  if (mode != LV_MODE_AUTO && mode != LV_MODE_ZERO_COPY) return LV_ERR_INVALID;
+  if (n_in > 0 && (sid < 0 || sid >= pool->d.S)) return LV_ERR_INVALID;
+  if (n_out > 0 && pool->d.host_pages == 0) return LV_ERR_INVALID;
+  if (n_out == 0 && n_in == 0) return LV_OK;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  try {
+    Staging st(pool, s);
+    const void *vin = nullptr, *bin = nullptr;
+    void *sdev = nullptr, *pdev = nullptr, *tdev = nullptr, *ndev = nullptr;
+    lv_status r;
+    if ((r = st.in(victims, (size_t)n_out * sizeof(lv_victim), &vin)) != LV_OK) return r;
+    if ((r = st.in(blks, (size_t)n_in * 4, &bin)) != LV_OK) return r;
+    if ((r = st.out(slots_out, (size_t)n_out * 4, &sdev, true)) != LV_OK) return r;
+    if ((r = st.out(pages_out, (size_t)n_in * 4, &pdev, true)) != LV_OK) return r;
+    if ((r = st.out(nullptr, (size_t)(n_out + n_in) * sizeof(int4), &tdev, true)) != LV_OK) return r;
+    if ((r = st.out(nullptr, sizeof(long long), &ndev, true)) != LV_OK) return r;
+    if (++pool->epoch <= 0) pool->epoch = 1;
+    LV_TRY(lv::launch_exchange(pool->d, static_cast<const lv_victim*>(vin), n_out, sid,
+                               static_cast<const int32_t*>(bin), n_in, static_cast<int32_t*>(sdev),
+                               static_cast<int32_t*>(pdev), static_cast<int4*>(tdev),
+                               static_cast<long long*>(ndev), pool->epoch, pool->d.page_tag, s,
+                               pool->exchange_ctas));
     return st.finish();
   } catch (const std::bad_alloc&) {
     return LV_ERR_OOM;

@@ -58,6 +58,8 @@ struct DevPool {
   int32_t* scount;           // [S] resident blocks of the session
   int32_t* sorder;           // [S] session id at rank r
   long long* soff;           // [S] first victim position of rank r
+  // exchange scratch
+  unsigned long long* page_tag;  // [hbm_pages] epoch << 32 | victim index (| paired bit)
 };
 
 __host__ __device__ inline unsigned long long owner_key(int32_t sid, int32_t blk) {
@@ -78,6 +80,10 @@ cudaError_t launch_swap_out(const DevPool& p, const lv_victim* v, const int32_t*
 cudaError_t launch_swap_in(const DevPool& p, int32_t sid, const int32_t* blks,
                            const int32_t* pages, int64_t n, lv_remap_entry* commit,
                            cudaStream_t s, int num_sms);
+cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out, int32_t sid,
+                            const int32_t* blks, int64_t n_in, int32_t* slots, int32_t* pages,
+                            int4* tasks, long long* n_tasks, int32_t epoch,
+                            unsigned long long* page_tag, cudaStream_t s, int copy_ctas);
 cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, int32_t epoch,
                          cudaStream_t s);
 cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cudaStream_t s);

@@ -482,6 +482,171 @@ k_swap_in(DevPool p, int32_t sid, const int32_t* __restrict__ blks,
   }
 }
 
+// -------------------------------------------------------------- exchange
+// Evict n_out victims and load n_in host blocks of one session in a single
+// stream-ordered step whose result equals swap-out, commit, swap-in, commit
+// done one after the other.  k_exchange_plan (one CTA) takes every metadata
+// decision in that order -- validation, host slots (lowest free, victim
+// order), out-commit, HBM pages (lowest free after the frees, list order),
+// in-commit -- and emits copy tasks {out page, out slot, in slot, in page}.
+// An incoming block that lands on a victim's old page shares that victim's
+// task, so one thread reads the old bytes before it writes the new ones and
+// both directions of the host link carry data at the same time.
+constexpr int kPlanThreads = 1024;
+constexpr unsigned long long kPairedBit = 1ull << 31;
+
+__global__ void __launch_bounds__(kPlanThreads)
+k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int32_t sid,
+                const int32_t* __restrict__ blks, long long n_in, int32_t* __restrict__ slots,
+                int32_t* __restrict__ pages, int4* __restrict__ tasks, long long* n_tasks,
+                int32_t epoch, unsigned long long* __restrict__ page_tag) {
+  __shared__ int bad;
+  if (threadIdx.x == 0) bad = 0;
+  __syncthreads();
+  const bool sid_ok = sid >= 0 && sid < p.S;
+  const int32_t nb_in = sid_ok ? nblocks_of(p, sid) : 0;
+  // validation: every victim is resident where it says, every incoming block is in
+  // the host tier, and no block appears twice
+  for (long long i = threadIdx.x; i < n_out; i += kPlanThreads) {
+    const lv_victim x = v[i];
+    bool ok = x.sid >= 0 && x.sid < p.S && x.blk >= 0 && x.page >= 0 && x.page < p.hbm_pages;
+    ok = ok && x.blk < nblocks_of(p, x.sid);
+    ok = ok && p.table[(size_t)x.sid * p.maxB + x.blk] == x.page &&
+         p.own_hbm[x.page] == owner_key(x.sid, x.blk);
+    ok = ok && atomicExch(&p.mark[(size_t)x.sid * p.maxB + x.blk], epoch) != epoch;
+    if (!ok) { set_error(p.ctl, LV_ERR_STATE, i); bad = 1; }
+  }
+  for (long long i = threadIdx.x; i < n_in; i += kPlanThreads) {
+    const int32_t b = blks[i];
+    bool ok = sid_ok && b >= 0 && b < nb_in;
+    if (ok) {
+      const int32_t e = p.table[(size_t)sid * p.maxB + b];
+      const long long h = -(long long)e - 2;
+      ok = e <= -2 && h < p.host_pages && p.own_host[h] == owner_key(sid, b);
+      ok = ok && atomicExch(&p.mark[(size_t)sid * p.maxB + b], epoch) != epoch;
+    }
+    if (!ok) { set_error(p.ctl, sid_ok ? LV_ERR_STATE : LV_ERR_BOUNDS, n_out + i); bad = 1; }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && !bad) {
+    // capacity, as the sequential calls see it: host slots before any is freed,
+    // HBM pages after the victims' pages are freed
+    if (p.ctl[C_HOST_ALLOC] + n_out > p.host_pages) {
+      set_error(p.ctl, LV_ERR_NO_HOST, n_out);
+      bad = 1;
+    } else if (p.ctl[C_HBM_ALLOC] - n_out + n_in > p.budget) {
+      set_error(p.ctl, LV_ERR_NO_HBM, n_in);
+      bad = 1;
+    }
+  }
+  __syncthreads();
+  if (bad) {
+    for (long long i = threadIdx.x; i < n_out; i += kPlanThreads) slots[i] = -1;
+    for (long long i = threadIdx.x; i < n_in; i += kPlanThreads) pages[i] = -1;
+    if (threadIdx.x == 0) *n_tasks = 0;
+    return;
+  }
+  // host slots for the victims
+  if (n_out > 0) block_alloc_lowest<kPlanThreads>(p.bits_host, p.host_pages, n_out, slots);
+  __syncthreads();
+  // out-commit: victims now live in their slots, their pages are free
+  const unsigned long long tag = (unsigned long long)(uint32_t)epoch << 32;
+  for (long long i = threadIdx.x; i < n_out; i += kPlanThreads) {
+    const lv_victim x = v[i];
+    const unsigned long long key = owner_key(x.sid, x.blk);
+    p.table[(size_t)x.sid * p.maxB + x.blk] = -(slots[i] + 2);
+    p.own_host[slots[i]] = key;
+    p.own_hbm[x.page] = kOwnerNone;
+    atomicAnd(&p.bits_hbm[x.page >> 5], ~(1u << (x.page & 31)));
+    page_tag[x.page] = tag | (unsigned long long)i;
+  }
+  __syncthreads();
+  // HBM pages for the incoming blocks
+  if (n_in > 0) block_alloc_lowest<kPlanThreads>(p.bits_hbm, p.hbm_pages, n_in, pages);
+  __syncthreads();
+  // in-commit, and one task per incoming block (paired with the victim whose page it takes)
+  for (long long i = threadIdx.x; i < n_in; i += kPlanThreads) {
+    const int32_t b = blks[i];
+    const size_t ti = (size_t)sid * p.maxB + b;
+    const long long g = -(long long)p.table[ti] - 2;
+    const int32_t pg = pages[i];
+    p.table[ti] = pg;
+    p.own_hbm[pg] = owner_key(sid, b);
+    p.own_host[g] = kOwnerNone;
+    atomicAnd(&p.bits_host[g >> 5], ~(1u << (g & 31)));
+    int4 t = make_int4(-1, -1, (int32_t)g, pg);
+    const unsigned long long pt = page_tag[pg];
+    if ((pt >> 32) == (unsigned long long)(uint32_t)epoch && !(pt & kPairedBit)) {
+      const long long vi = (long long)(pt & 0x7fffffffull);
+      t.x = pg;
+      t.y = slots[vi];
+      page_tag[pg] = pt | kPairedBit;
+    }
+    tasks[i] = t;
+  }
+  __syncthreads();
+  // victims whose page no incoming block takes: out-only tasks, in victim order
+  long long run = 0;
+  for (long long i0 = 0; i0 < n_out; i0 += kPlanThreads) {
+    const long long i = i0 + threadIdx.x;
+    long long flag = 0;
+    int32_t pg = -1;
+    if (i < n_out) {
+      pg = v[i].page;
+      flag = (page_tag[pg] & kPairedBit) ? 0 : 1;
+    }
+    long long chunk;
+    const long long pos = run + block_excl_scan<kPlanThreads>(flag, &chunk);
+    if (flag) tasks[n_in + pos] = make_int4(pg, slots[i], -1, -1);
+    run += chunk;
+  }
+  if (threadIdx.x == 0) {
+    *n_tasks = n_in + run;
+    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HOST_ALLOC]), (unsigned long long)(n_out - n_in));
+    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HBM_ALLOC]), (unsigned long long)(n_in - n_out));
+    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PAGES_OUT]), (unsigned long long)n_out);
+    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PAGES_IN]), (unsigned long long)n_in);
+    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_REMAP]), (unsigned long long)(n_out + n_in));
+  }
+}
+
+// Unit u = (task t, sub-page j): the out half copies hbm_kv[j][page] to host[slot][j],
+// the in half host[slot'][j] to hbm_kv[j][page']; each thread loads both before it
+// stores either, so a paired task reads the old page before overwriting it.
+__global__ void __launch_bounds__(kCopyThreads)
+k_exchange_copy(DevPool p, const int4* __restrict__ tasks, const long long* __restrict__ n_tasks) {
+  const long long units = *n_tasks * p.J;
+  const int nvec = (int)(p.P >> 4);
+  for (long long u = blockIdx.x; u < units; u += gridDim.x) {
+    const int4 t = tasks[u / p.J];
+    const int j = (int)(u % p.J);
+    const bool has_out = t.x >= 0, has_in = t.z >= 0;
+    const int4* so = has_out ? reinterpret_cast<const int4*>(p.kv[j] + (size_t)t.x * p.P) : nullptr;
+    int4* dout = has_out ? reinterpret_cast<int4*>(p.host + ((size_t)t.y * p.J + j) * p.P) : nullptr;
+    const int4* si = has_in ? reinterpret_cast<const int4*>(p.host + ((size_t)t.z * p.J + j) * p.P) : nullptr;
+    int4* din = has_in ? reinterpret_cast<int4*>(p.kv[j] + (size_t)t.w * p.P) : nullptr;
+    for (int base = threadIdx.x; base < nvec; base += kCopyThreads * kCopyUnroll) {
+      int4 ro[kCopyUnroll], ri[kCopyUnroll];
+#pragma unroll
+      for (int k = 0; k < kCopyUnroll; ++k) {
+        const int q = base + k * kCopyThreads;
+        if (q < nvec) {
+          if (has_in) ri[k] = si[q];
+          if (has_out) ro[k] = so[q];
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < kCopyUnroll; ++k) {
+        const int q = base + k * kCopyThreads;
+        if (q < nvec) {
+          if (has_out) dout[q] = ro[k];
+          if (has_in) din[q] = ri[k];
+        }
+      }
+    }
+  }
+}
+
 // ---------------------------------------------------------------- commit
 __device__ __forceinline__ bool bit_is_set(const uint32_t* bits, long long i) {
   return (bits[i >> 5] >> (i & 31)) & 1u;
@@ -715,6 +880,17 @@ cudaError_t launch_swap_in(const DevPool& p, int32_t sid, const int32_t* blks, c
   const long long units = (long long)n * p.J;
   k_swap_in<<<blocks_for(units, 1, (long long)num_sms * 8), kCopyThreads, 0, s>>>(
       p, sid, blks, pages, n, commit);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out, int32_t sid,
+                            const int32_t* blks, int64_t n_in, int32_t* slots, int32_t* pages,
+                            int4* tasks, long long* n_tasks, int32_t epoch,
+                            unsigned long long* page_tag, cudaStream_t s, int copy_ctas) {
+  k_exchange_plan<<<1, kPlanThreads, 0, s>>>(p, v, n_out, sid, blks, n_in, slots, pages, tasks,
+                                             n_tasks, epoch, page_tag);
+  const long long units = (n_out + n_in) * (long long)p.J;
+  k_exchange_copy<<<blocks_for(units, 1, copy_ctas), kCopyThreads, 0, s>>>(p, tasks, n_tasks);
   return cudaGetLastError();
 }
 

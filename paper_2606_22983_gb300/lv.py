@@ -99,6 +99,7 @@ def _load():
         "lv_select_victims": [vp, i64, i64, u32, vp, i64, vp, vp],
         "lv_swap_out": [vp, vp, i64, vp, vp, i32, vp],
         "lv_swap_in": [vp, i32, vp, i64, vp, vp, i32, vp],
+        "lv_swap_exchange": [vp, vp, i64, i32, vp, i64, vp, vp, i32, vp],
         "lv_remap": [vp, vp, i64, vp],
         "lv_cancel": [vp, vp, i64, vp],
         "lv_session_append": [vp, i32, i32, vp, vp, vp],
@@ -128,7 +129,7 @@ _lib = _load()
 
 EXPORTED = ("lv_pool_create", "lv_pool_destroy", "lv_pool_host_ptr", "lv_pool_import",
             "lv_session_set", "lv_session_get", "lv_session_events", "lv_select_victims",
-            "lv_swap_out", "lv_swap_in", "lv_remap", "lv_cancel", "lv_session_append",
+            "lv_swap_out", "lv_swap_in", "lv_swap_exchange", "lv_remap", "lv_cancel", "lv_session_append",
             "lv_session_counts", "lv_session_blocks", "lv_read_tables", "lv_sync",
             "lv_get_stats", "lv_clear_error", "lv_status_str", "lv_version",
             "lv_select_victims_noalloc")
@@ -216,6 +217,12 @@ def lv_swap_out(pool, victims, n, slots_out, commit_out, mode=LV_MODE_AUTO, stre
 def lv_swap_in(pool, sid, blks, n, pages_out, commit_out, mode=LV_MODE_AUTO, stream=None):
     _check(_lib.lv_swap_in(pool, sid, ptr(blks), n, ptr(pages_out), ptr(commit_out), mode,
                            stream_handle(stream)), "lv_swap_in")
+
+
+def lv_swap_exchange(pool, victims, n_out, sid, blks, n_in, slots_out, pages_out,
+                     mode=LV_MODE_AUTO, stream=None):
+    _check(_lib.lv_swap_exchange(pool, ptr(victims), n_out, sid, ptr(blks), n_in, ptr(slots_out),
+                                 ptr(pages_out), mode, stream_handle(stream)), "lv_swap_exchange")
 
 
 def lv_remap(pool, entries, n, stream=None):

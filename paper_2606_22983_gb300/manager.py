@@ -9,7 +9,10 @@ Consumes monitor event scripts (records ``(t_us, kind, sid, a, b, c, d)``):
   kind 5 BARGE_IN(sid)                kind 6 SPEECH_STOP(sid)
 
 A turn makes the session fully resident (a synchronous foreground load),
-grows its context, then records the reply.  Speech start and barge-in trigger a
+grows its context, then records the reply.  By default the evictions and loads
+of one step go through lv_swap_exchange (both link directions at once);
+``exchange=False`` issues swap-out, commit, swap-in, commit one after the other,
+with the same result.  Speech start and barge-in trigger a
 best-effort preload of the session's host blocks.  Making a session resident
 with ``need`` missing pages first evicts exactly ``k = need - free`` pages in
 the next-use order (foreground turns may also take protected, non-running KV
@@ -44,7 +47,7 @@ def _event(kind, sid, t, a=0, b=0):
 
 class KVManager:
     def __init__(self, pool: KVPool, perms=None, on_append=None, rank_on="none", admit=None,
-                 mode=lv.LV_MODE_AUTO, record=True):
+                 mode=lv.LV_MODE_AUTO, record=True, exchange=True):
         self.pool = pool
         self.perms = perms
         self.on_append = on_append      # callback(sid, old_ctx, new_ctx, pages) after growth
@@ -52,6 +55,7 @@ class KVManager:
         self.admit = admit              # callback(manager, sid, now, n_host_blocks) -> bool
         self.mode = mode
         self.record = record
+        self.exchange = exchange        # one lv_swap_exchange instead of four sequential calls
         self.counters = dict(victims=0, pages_out=0, pages_in=0, preloads=0,
                              preload_skipped=0, turns=0, sync_loads=0, appended=0)
         self.bytes_moved = 0
@@ -83,15 +87,68 @@ class KVManager:
         need = nh + new_blocks
         k = max(0, need - self.free_budget())
         rec["k"] = k
-        if k > 0:
-            flags = lv.LV_SELECT_FALLBACK if foreground else 0
-            victims, n = pool.select(now_us, k, flags)
+        if self.exchange:
+            if not self._exchange(sid, now_us, k, hblk, nh, foreground, rec):
+                return False
+        else:
+            if not self._sequential(sid, now_us, k, hblk, nh, foreground, rec):
+                return False
+        if append_tokens:
+            old_ctx = self.ctx_tokens(sid)
+            pages = pool.append(sid, append_tokens)
             if self.record:
-                rec["victims"] = victims.cpu().numpy().astype(np.int64)
-                self.last_readback_bytes += n * 12
-            if n < k:
-                if foreground:
-                    raise lv.LvError(lv.LV_ERR_NO_HBM, f"turn of session {sid} needs {k} victims, {n} found")
+                rec["append_pages"] = pages.cpu().numpy().astype(np.int64)
+            self.counters["appended"] += int(pages.numel())
+            if self.on_append is not None:
+                self.on_append(sid, old_ctx, old_ctx + append_tokens)
+        return True
+
+    def _victims(self, sid, now_us, k, foreground, rec):
+        flags = lv.LV_SELECT_FALLBACK if foreground else 0
+        victims, n = self.pool.select(now_us, k, flags)
+        if self.record:
+            rec["victims"] = victims.cpu().numpy().astype(np.int64)
+            self.last_readback_bytes += n * 12
+        if n < k:
+            if foreground:
+                raise lv.LvError(lv.LV_ERR_NO_HBM, f"turn of session {sid} needs {k} victims, {n} found")
+            return None, n
+        return victims, n
+
+    def _exchange(self, sid, now_us, k, hblk, nh, foreground, rec):
+        pool = self.pool
+        victims, n = None, 0
+        if k > 0:
+            victims, n = self._victims(sid, now_us, k, foreground, rec)
+            if victims is None:
+                return False
+        if n == 0 and nh == 0:
+            return True
+        nbytes = (n + nh) * pool.J * pool.P
+        if self.timer:
+            self.timer.start("exchange")
+        slots, pages = pool.exchange(victims, n, sid, hblk, nh, self.mode)
+        if self.timer:
+            self.timer.stop("exchange", nbytes)
+        if self.record:
+            if n:
+                rec["slots"] = slots.cpu().numpy().astype(np.int64)
+                self.last_readback_bytes += n * 4
+            if nh:
+                rec["in_blocks"] = hblk.cpu().numpy().astype(np.int64)
+                rec["in_pages"] = pages.cpu().numpy().astype(np.int64)
+                self.last_readback_bytes += nh * 8
+        self.counters["victims"] += n
+        self.counters["pages_out"] += n
+        self.counters["pages_in"] += nh
+        self.bytes_moved += nbytes
+        return True
+
+    def _sequential(self, sid, now_us, k, hblk, nh, foreground, rec):
+        pool = self.pool
+        if k > 0:
+            victims, n = self._victims(sid, now_us, k, foreground, rec)
+            if victims is None:
                 return False
             if self.timer:
                 self.timer.start("swap_out")
@@ -118,14 +175,6 @@ class KVManager:
                 self.last_readback_bytes += nh * 8
             self.counters["pages_in"] += nh
             self.bytes_moved += nh * pool.J * pool.P
-        if append_tokens:
-            old_ctx = self.ctx_tokens(sid)
-            pages = pool.append(sid, append_tokens)
-            if self.record:
-                rec["append_pages"] = pages.cpu().numpy().astype(np.int64)
-            self.counters["appended"] += int(pages.numel())
-            if self.on_append is not None:
-                self.on_append(sid, old_ctx, old_ctx + append_tokens)
         return True
 
     def preload(self, sid, now_us, rec):

@@ -121,6 +121,13 @@ class KVPool:
         self.launches += 2
         return self.pages[:n], self.commit[:n]
 
+    def exchange(self, victims, n_out: int, sid: int, blks, n_in: int, mode=lv.LV_MODE_AUTO):
+        """Evict n_out victims and load n_in host blocks of sid, committed, in one step."""
+        lv.lv_swap_exchange(self.handle, victims, n_out, sid, blks, n_in, self.slots, self.pages,
+                            mode, self.stream)
+        self.launches += 2
+        return self.slots[:n_out], self.pages[:n_in]
+
     def remap(self, entries, n: int):
         lv.lv_remap(self.handle, entries, n, self.stream)
         self.launches += 1

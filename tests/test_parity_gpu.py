@@ -10,13 +10,14 @@ from ._lockstep import run_lockstep
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("seed", [0, 1])
-def test_tiny_workload_full_images(seed):
+@pytest.mark.parametrize("seed,exchange", [(0, True), (1, True), (0, False)])
+def test_tiny_workload_full_images(seed, exchange):
     """1000 scripted events of the tiny pool: every ranking (full order after
     each event), eviction, preload, reload and growth, with full HBM and host
-    byte images compared every 50 events."""
+    byte images compared every 50 events -- through lv_swap_exchange and
+    through the four sequential calls."""
     wl = make_workload("tiny", seed)
-    om, gm = run_lockstep(wl, with_bytes=True, check_every=50)
+    om, gm = run_lockstep(wl, with_bytes=True, check_every=50, exchange=exchange)
     assert om.counters == gm.counters
     assert gm.counters["pages_out"] > 500 and gm.counters["preloads"] > 10
 
