@@ -100,41 +100,6 @@ class ClockSampler:
 
 
 # --------------------------------------------------------------- our arm
-class KernelTimer:
-    """CUDA-event brackets around the swap calls, on the launching stream."""
-
-    def __init__(self, torch):
-        self.torch = torch
-        self.pending = {}
-        self.done = {}
-        self.enabled = False
-
-    def start(self, name):
-        if not self.enabled:
-            return
-        e = self.torch.cuda.Event(enable_timing=True)
-        e.record()
-        self.pending[name] = e
-
-    def stop(self, name, nbytes):
-        if not self.enabled:
-            return
-        e = self.torch.cuda.Event(enable_timing=True)
-        e.record()
-        self.done.setdefault(name, []).append((self.pending.pop(name), e, nbytes))
-
-    def summary(self):
-        self.torch.cuda.synchronize()
-        out = {}
-        for name, lst in self.done.items():
-            ms = [a.elapsed_time(b) for a, b, _ in lst]
-            nb = [n for _, _, n in lst]
-            out[name] = {"launches": len(lst), "total_ms": sum(ms), "avg_ms": sum(ms) / len(ms),
-                         "bytes_per_launch": sum(nb) / len(nb),
-                         "gbs": (sum(nb) / 1e9) / (sum(ms) / 1e3) if sum(ms) > 0 else 0.0}
-        return out
-
-
 def link_peaks(torch, pool, nbytes, reps=5):
     """Contiguous page-locked cudaMemcpyAsync of nbytes each way, and both at once."""
     src = pool.kv.view(-1)[:nbytes]
@@ -173,26 +138,27 @@ def link_peaks(torch, pool, nbytes, reps=5):
     return res
 
 
-def run_turns(torch, gm, wl, lo, hi, dev_events=None, timer=None):
-    """Turns lo..hi of a turn-driven script; returns payload bytes moved."""
+def run_turns(gm, wl, lo, hi, dev_events=None):
+    """Turns lo..hi of a turn-driven script (playback batch, then the turn)."""
     from paper_2606_22983_gb300 import lv
     S = wl.spec.n_sessions
-    moved0 = gm.bytes_moved
     per_turn = S + 1
     for i in range(lo, hi):
         base = i * per_turn
-        t = int(wl.t_us[base])
         if dev_events is not None:
             lv.lv_session_events(gm.pool.handle, dev_events[i], S, gm.pool.stream)
             gm.pool.launches += 1
         else:
             ev = np.zeros(S, dtype=lv.EVENT_DTYPE)
             ev["kind"], ev["sid"], ev["t_us"], ev["a"] = (lv.LV_EV_PLAYBACK, wl.sid[base:base + S],
-                                                          t, wl.a[base:base + S])
+                                                          int(wl.t_us[base]), wl.a[base:base + S])
             gm.pool.events(ev)
-        gm.timer = timer
         gm.step(wl.event(base + S), base + S)
-    return gm.bytes_moved - moved0
+
+
+def _moved_pages(pool):
+    st = pool.stats()
+    return st["pages_out"] + st["pages_in"], st["pages_out"], st["pages_in"]
 
 
 def ours(args, torch):
@@ -221,9 +187,7 @@ def ours(args, torch):
     fill_random(pool, args.seed + rank)
     page_bytes = pool.J * pool.P
     gm = KVManager(pool, perms=wl.perms, rank_on="none", mode=args.mode, record=False,
-                   exchange=not args.sequential)
-    timer = KernelTimer(torch)
-    gm.timer = timer
+                   driver=args.driver)
     S = wl.spec.n_sessions
     # the PLAYBACK batches of the device-timed pass, resident before timing
     dev_events = []
@@ -235,29 +199,42 @@ def ours(args, torch):
         dev_events.append(torch.from_numpy(ev.view(np.uint8).copy()).to(pool.device))
     torch.cuda.synchronize()
 
-    run_turns(torch, gm, wl, 0, W, dev_events)                  # warm-up
+    run_turns(gm, wl, 0, W, dev_events)                         # warm-up
     pool.sync()
+    p0, o0, i0 = _moved_pages(pool)
+    lv.lv_timing_read(pool.handle, reset=True)
+    lv.lv_timing_enable(pool.handle, True)
     clocks = ClockSampler(local)
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
     clocks.start()
-    timer.enabled = True
     l0 = pool.launches
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
     t0.record()
-    moved = run_turns(torch, gm, wl, W, W + K, dev_events, timer)
+    run_turns(gm, wl, W, W + K, dev_events)
     t1.record()
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
     launches = pool.launches - l0
     clk = clocks.stop()
-    timer.enabled = False
+    lv.lv_timing_enable(pool.handle, False)
+    timing = lv.lv_timing_read(pool.handle, reset=True)
     dev_s = t0.elapsed_time(t1) / 1e3
     assert pool.sync(raise_on_error=False) == 0, "device error during the timed turns"
-    kern = timer.summary()
+    p1, o1, i1 = _moved_pages(pool)
+    moved = (p1 - p0) * page_bytes
+    kern = {}
+    for name, t in timing.items():
+        if t["launches"]:
+            pages = {"swap_out": o1 - o0, "swap_in": i1 - i0}.get(name, p1 - p0)
+            nb = pages * page_bytes
+            kern[name] = {"launches": t["launches"], "total_ms": t["total_ms"],
+                          "avg_ms": t["total_ms"] / t["launches"],
+                          "bytes_per_launch": nb / t["launches"],
+                          "gbs": nb / 1e9 / (t["total_ms"] / 1e3)}
 
     # e2e: the next K turns through the C ABI with host buffers
     gm.record = True
@@ -265,15 +242,16 @@ def ours(args, torch):
     torch.cuda.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
+    q0 = _moved_pages(pool)[0]
     e0.record()
-    moved_e2e = 0
     for i in range(W + K, W + 2 * K):
-        moved_e2e += run_turns(torch, gm, wl, i, i + 1, None, None)
+        run_turns(gm, wl, i, i + 1, None)
         h2d += (S + 2) * lv.EVENT_DTYPE.itemsize
-        d2h += gm.last_readback_bytes
+        d2h += gm.last_readback_bytes + lv.RESIDENT_DTYPE.itemsize
     e1.record()
     torch.cuda.synchronize()
     e2e_s = e0.elapsed_time(e1) / 1e3
+    moved_e2e = (_moved_pages(pool)[0] - q0) * page_bytes
     if dist:
         tt = torch.tensor([dev_s, e2e_s, moved, moved_e2e], dtype=torch.float64, device="cuda")
         gathered = [torch.zeros_like(tt) for _ in range(ws)]
@@ -307,7 +285,7 @@ def ours(args, torch):
                                    "budget, one turn = evict + reload",
                        "hbm_budget_pages": wl.spec.hbm_budget_pages, "host_pages": wl.spec.host_pages,
                        "mode": {0: "auto", 1: "zero_copy", 2: "staged"}[args.mode],
-                       "path": "sequential" if args.sequential else "exchange",
+                       "driver": args.driver,
                        "l2": "inputs larger than L2 (mean turn moves "
                              f"{mean_turn / 1e6:.0f} MB each way from a 40 GB pool)",
                        "parallelism": f"replicas x{ws}"},
@@ -427,12 +405,13 @@ def reference(args):
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=40)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--mode", type=int, default=0, help="0 auto, 1 zero-copy, 2 staged")
-    ap.add_argument("--sequential", action="store_true",
-                    help="swap-out, commit, swap-in, commit one after the other (no exchange)")
+    ap.add_argument("--driver", choices=("device", "exchange", "sequential"), default="device",
+                    help="device: one lv_make_resident per turn; exchange: select + "
+                         "lv_swap_exchange; sequential: swap-out, commit, swap-in, commit")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")

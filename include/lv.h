@@ -159,6 +159,7 @@ typedef struct lv_stats {
   /* counters ("counters for policy fallbacks and preload outcomes", Section 6) */
   int64_t selects, victims, shortfalls, pages_out, pages_in, bytes_out, bytes_in;
   int64_t remap_entries, appended_pages, cancels, events, fallback_selects;
+  int64_t preloads, preloads_skipped;   /* lv_make_resident with LV_RESIDENT_PRELOAD */
 } lv_stats;
 
 /* ---------------------------------------------------------------- pool */
@@ -274,6 +275,45 @@ lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_ou
                            const int32_t* blks, int64_t n_in, int32_t* slots_out,
                            int32_t* pages_out, int32_t mode, lv_stream stream);
 
+/* lv_make_resident flags and result */
+enum { LV_RESIDENT_PRELOAD = 1 };
+enum { LV_RESIDENT_DONE = 0, LV_RESIDENT_SKIPPED = 1, LV_RESIDENT_NOTHING = 2,
+       LV_RESIDENT_FAILED = 3 /* a device-detected error stopped it (see lv_sync) */ };
+
+typedef struct lv_resident_result {
+  int64_t k;              /* pages the HBM budget was short (victims asked for) */
+  int64_t n_found;        /* victims the ranking found (min(k, candidates)) */
+  int64_t n_victims;      /* victims evicted */
+  int64_t n_loaded;       /* host blocks loaded */
+  int64_t n_appended;     /* new pages for appended tokens */
+  int32_t status;         /* LV_RESIDENT_DONE / _SKIPPED / _NOTHING */
+  int32_t pad;
+} lv_resident_result;
+
+/* Sections 5.1 and 5.2, one step with no host round trip: makes session sid
+   fully resident and grows its context by append_tokens.  On the device, in
+   stream order: list sid's host-tier blocks (ascending); k = max(0, host
+   blocks + new blocks - free budget); rank with lv_select_victims' order and
+   take the first k (with LV_SELECT_FALLBACK unless LV_RESIDENT_PRELOAD);
+   then evict and load exactly as lv_swap_exchange does; then append as
+   lv_session_append does.  The results equal those of the host-driven
+   sequence select -> exchange -> append.
+   Foreground (flags 0): fewer than k victims is LV_ERR_NO_HBM (device-
+   detected) and nothing moves.  Preload (LV_RESIDENT_PRELOAD, Section 5.2):
+   no host blocks gives LV_RESIDENT_NOTHING; more than max_load_pages host
+   blocks (admission; < 0 means no limit) or fewer than k victims gives
+   LV_RESIDENT_SKIPPED and nothing moves; a completed preload protects the
+   session until now_us + protect_us.  append_tokens must be 0 for a preload.
+   Optional outputs (host or device, NULL to skip): victims_out
+   (lv_victim [hbm_budget_pages]), slots_out (int32 [hbm_budget_pages]),
+   blocks_out and pages_out (int32 [max_blocks]: blocks loaded and their
+   pages), append_out (int32 [append_tokens / T + 2]), result_out. */
+lv_status lv_make_resident(lv_pool* pool, int32_t sid, int64_t now_us, int32_t append_tokens,
+                           uint32_t flags, int64_t max_load_pages, lv_victim* victims_out,
+                           int32_t* slots_out, int32_t* blocks_out, int32_t* pages_out,
+                           int32_t* append_out, lv_resident_result* result_out,
+                           lv_stream stream);
+
 /* Section 6 (side tables) and Section 5.2 ("preloading affects latency but not
    correctness"): commits n entries.  For each, the new location must be a
    reservation not yet owned; it becomes owned by (sid, blk), the block table
@@ -373,6 +413,23 @@ lv_status lv_get_stats(lv_pool* pool, lv_stats* out, lv_stream stream);
 
 /* Clears the sticky device error (stream-ordered). */
 lv_status lv_clear_error(lv_pool* pool, lv_stream stream);
+
+/* Instrumentation (Section 6: counters that validate which paths run).  While
+   enabled, every launch of a copy kernel -- swap-out, swap-in, exchange -- is
+   bracketed by two CUDA events recorded on its own stream.  lv_timing_read
+   waits for them and reports, per kernel kind (index LV_TIMING_SWAP_OUT,
+   _SWAP_IN, _EXCHANGE), the launches and their summed, shortest and longest
+   durations; reset != 0 starts a new record.  Enabling it adds two event
+   records per launch and nothing else. */
+enum { LV_TIMING_SWAP_OUT = 0, LV_TIMING_SWAP_IN = 1, LV_TIMING_EXCHANGE = 2, LV_TIMING_KINDS = 3 };
+typedef struct lv_kernel_timing {
+  int64_t launches;
+  double total_ms;
+  double min_ms;
+  double max_ms;
+} lv_kernel_timing;
+lv_status lv_timing_enable(lv_pool* pool, int32_t enable);
+lv_status lv_timing_read(lv_pool* pool, lv_kernel_timing* out /* [LV_TIMING_KINDS] */, int32_t reset);
 
 const char* lv_status_str(lv_status s);
 int32_t lv_version(void);

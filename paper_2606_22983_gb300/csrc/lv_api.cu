@@ -14,6 +14,11 @@ struct lv_pool {
   int num_sms = 0;
   int32_t epoch = 0;
   int exchange_ctas = 0;           // grid of the exchange copy kernel
+  lv::ResidentScratch rs{};        // lv_make_resident buffers
+  // copy-kernel timing (lv_timing_enable): event pairs recorded per kind, reused
+  bool timing = false;
+  std::vector<lv::EventPair> ev_free;
+  std::vector<lv::EventPair> ev_used[LV_TIMING_KINDS];
   bool own_host = false;
   void* host_base = nullptr;       // host-visible address of the host pool
   std::vector<void*> dev_allocs;
@@ -141,7 +146,28 @@ lv_status dev_alloc(lv_pool* pool, T** ptr, size_t count) {
   return LV_OK;
 }
 
+// The event pair for the next launch of kind `kind`, or nullptr when timing is off.
+const lv::EventPair* timing_pair(lv_pool* pool, int kind) {
+  if (!pool->timing) return nullptr;
+  lv::EventPair ev{};
+  if (!pool->ev_free.empty()) {
+    ev = pool->ev_free.back();
+    pool->ev_free.pop_back();
+  } else if (cudaEventCreate(&ev.start) != cudaSuccess || cudaEventCreate(&ev.end) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  pool->ev_used[kind].push_back(ev);
+  return &pool->ev_used[kind].back();
+}
+
 void free_pool(lv_pool* pool) {
+  for (auto& v : pool->ev_used)
+    for (auto& e : v) pool->ev_free.push_back(e);
+  for (auto& e : pool->ev_free) {
+    cudaEventDestroy(e.start);
+    cudaEventDestroy(e.end);
+  }
   for (void* p : pool->dev_allocs) cudaFree(p);
   pool->dev_allocs.clear();
   if (pool->own_host && pool->host_base) cudaFreeHost(pool->host_base);
@@ -250,6 +276,15 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       (st = dev_alloc(pool, &d.sorder, d.S)) != LV_OK ||
       (st = dev_alloc(pool, &d.soff, d.S)) != LV_OK ||
       (st = dev_alloc(pool, &d.page_tag, (size_t)d.hbm_pages)) != LV_OK)
+    return fail(st);
+  lv::ResidentScratch& rs = pool->rs;
+  if ((st = dev_alloc(pool, &rs.victims, (size_t)d.budget)) != LV_OK ||
+      (st = dev_alloc(pool, &rs.slots, (size_t)d.budget)) != LV_OK ||
+      (st = dev_alloc(pool, &rs.blocks, (size_t)d.maxB)) != LV_OK ||
+      (st = dev_alloc(pool, &rs.pages, (size_t)d.maxB)) != LV_OK ||
+      (st = dev_alloc(pool, &rs.append, (size_t)d.maxB + 2)) != LV_OK ||
+      (st = dev_alloc(pool, &rs.tasks, (size_t)d.budget + d.maxB)) != LV_OK ||
+      (st = dev_alloc(pool, &rs.words, 16)) != LV_OK)
     return fail(st);
   d.kv = kv_dev;
   if (cudaMemcpyAsync(kv_dev, kv.data(), d.J * sizeof(uint8_t*), cudaMemcpyHostToDevice, s) != cudaSuccess ||
@@ -421,7 +456,8 @@ lv_status lv_swap_out(lv_pool* pool, const lv_victim* victims, int64_t n, int32_
     int32_t* slots = static_cast<int32_t*>(sdev);
     LV_TRY(lv::launch_alloc(pool->d, false, n, slots, s));
     LV_TRY(lv::launch_swap_out(pool->d, static_cast<const lv_victim*>(vin), slots, n,
-                               static_cast<lv_remap_entry*>(cdev), s, pool->num_sms));
+                               static_cast<lv_remap_entry*>(cdev), s, pool->num_sms,
+                               timing_pair(pool, LV_TIMING_SWAP_OUT)));
     return st.finish();
   } catch (const std::bad_alloc&) {
     return LV_ERR_OOM;
@@ -447,7 +483,8 @@ lv_status lv_swap_in(lv_pool* pool, int32_t sid, const int32_t* blks, int64_t n,
     int32_t* pages = static_cast<int32_t*>(pdev);
     LV_TRY(lv::launch_alloc(pool->d, true, n, pages, s));
     LV_TRY(lv::launch_swap_in(pool->d, sid, static_cast<const int32_t*>(bin), pages, n,
-                              static_cast<lv_remap_entry*>(cdev), s, pool->num_sms));
+                              static_cast<lv_remap_entry*>(cdev), s, pool->num_sms,
+                              timing_pair(pool, LV_TIMING_SWAP_IN)));
     return st.finish();
   } catch (const std::bad_alloc&) {
     return LV_ERR_OOM;
@@ -482,7 +519,46 @@ lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_ou
                                static_cast<const int32_t*>(bin), n_in, static_cast<int32_t*>(sdev),
                                static_cast<int32_t*>(pdev), static_cast<int4*>(tdev),
                                static_cast<long long*>(ndev), pool->epoch, pool->d.page_tag, s,
-                               pool->exchange_ctas));
+                               pool->exchange_ctas, nullptr, 0, timing_pair(pool, LV_TIMING_EXCHANGE)));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_make_resident(lv_pool* pool, int32_t sid, int64_t now_us, int32_t append_tokens,
+                           uint32_t flags, int64_t max_load_pages, lv_victim* victims_out,
+                           int32_t* slots_out, int32_t* blocks_out, int32_t* pages_out,
+                           int32_t* append_out, lv_resident_result* result_out, lv_stream stream) {
+  if (!pool || sid < 0 || sid >= pool->d.S || append_tokens < 0) return LV_ERR_INVALID;
+  if (flags & ~(uint32_t)LV_RESIDENT_PRELOAD) return LV_ERR_INVALID;
+  const bool preload = (flags & LV_RESIDENT_PRELOAD) != 0;
+  if (preload && append_tokens != 0) return LV_ERR_INVALID;
+  if (pool->d.host_pages == 0) return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  const DevPool& d = pool->d;
+  const lv::ResidentScratch& rs = pool->rs;
+  try {
+    Staging st(pool, s);
+    void* rdev = nullptr;
+    lv_status r;
+    if ((r = st.out(result_out, sizeof(lv_resident_result), &rdev, false)) != LV_OK) return r;
+    if (++pool->epoch <= 0) pool->epoch = 1;
+    LV_TRY(lv::launch_make_resident(d, rs, sid, now_us, append_tokens, preload, max_load_pages,
+                                    pool->epoch, s, pool->exchange_ctas,
+                                    static_cast<lv_resident_result*>(rdev),
+                                    timing_pair(pool, LV_TIMING_EXCHANGE)));
+    // optional copies of the decisions (whole buffers: the counts live on the device)
+    const struct { void* user; const void* dev; size_t bytes; } outs[] = {
+        {victims_out, rs.victims, (size_t)d.budget * sizeof(lv_victim)},
+        {slots_out, rs.slots, (size_t)d.budget * 4},
+        {blocks_out, rs.blocks, (size_t)d.maxB * 4},
+        {pages_out, rs.pages, (size_t)d.maxB * 4},
+        {append_out, rs.append,
+         (size_t)(append_tokens / d.T + 2 < d.maxB + 2 ? append_tokens / d.T + 2 : d.maxB + 2) * 4}};
+    for (const auto& o : outs)
+      if (o.user) LV_TRY(cudaMemcpyAsync(o.user, o.dev, o.bytes, cudaMemcpyDefault, s));
     return st.finish();
   } catch (const std::bad_alloc&) {
     return LV_ERR_OOM;
@@ -638,6 +714,8 @@ lv_status lv_get_stats(lv_pool* pool, lv_stats* out, lv_stream stream) {
   out->cancels = c[lv::C_CANCELS];
   out->events = c[lv::C_EVENTS];
   out->fallback_selects = c[lv::C_FALLBACK];
+  out->preloads = c[lv::C_PRELOADS];
+  out->preloads_skipped = c[lv::C_PRELOADS_SKIPPED];
   return LV_OK;
 }
 
@@ -645,6 +723,35 @@ lv_status lv_clear_error(lv_pool* pool, lv_stream stream) {
   if (!pool) return LV_ERR_INVALID;
   DeviceGuard g(pool->device);
   LV_TRY(cudaMemsetAsync(pool->d.ctl + lv::C_ERR, 0, 2 * sizeof(long long), as_stream(stream)));
+  return LV_OK;
+}
+
+lv_status lv_timing_enable(lv_pool* pool, int32_t enable) {
+  if (!pool) return LV_ERR_INVALID;
+  pool->timing = enable != 0;
+  return LV_OK;
+}
+
+lv_status lv_timing_read(lv_pool* pool, lv_kernel_timing* out, int32_t reset) {
+  if (!pool || !out) return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  for (int kind = 0; kind < LV_TIMING_KINDS; ++kind) {
+    lv_kernel_timing t{0, 0.0, 0.0, 0.0};
+    for (const lv::EventPair& e : pool->ev_used[kind]) {
+      if (cudaEventSynchronize(e.end) != cudaSuccess) return LV_ERR_CUDA;
+      float ms = 0.f;
+      if (cudaEventElapsedTime(&ms, e.start, e.end) != cudaSuccess) return LV_ERR_CUDA;
+      t.total_ms += ms;
+      t.min_ms = t.launches == 0 || ms < t.min_ms ? ms : t.min_ms;
+      t.max_ms = ms > t.max_ms ? ms : t.max_ms;
+      t.launches += 1;
+    }
+    out[kind] = t;
+    if (reset) {
+      for (const lv::EventPair& e : pool->ev_used[kind]) pool->ev_free.push_back(e);
+      pool->ev_used[kind].clear();
+    }
+  }
   return LV_OK;
 }
 

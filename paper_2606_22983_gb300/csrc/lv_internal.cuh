@@ -29,6 +29,8 @@ enum Ctl : int {
   C_CANCELS,
   C_EVENTS,
   C_FALLBACK,
+  C_PRELOADS,
+  C_PRELOADS_SKIPPED,
   C_N = 32
 };
 
@@ -66,6 +68,12 @@ __host__ __device__ inline unsigned long long owner_key(int32_t sid, int32_t blk
   return ((unsigned long long)(uint32_t)sid << 32) | (uint32_t)blk;
 }
 
+// Optional CUDA events recorded around a copy kernel launch.
+struct EventPair {
+  cudaEvent_t start;
+  cudaEvent_t end;
+};
+
 // ---- launch wrappers (lv_kernels.cu); each returns cudaGetLastError() ----
 cudaError_t launch_import(const DevPool& p, const int32_t* placement, const int32_t* ctx,
                           cudaStream_t s);
@@ -73,22 +81,41 @@ cudaError_t launch_session_set(const DevPool& p, const lv_session_state* in, int
                                int32_t n, cudaStream_t s);
 cudaError_t launch_events(const DevPool& p, const lv_event* ev, int64_t n, cudaStream_t s);
 cudaError_t launch_select(const DevPool& p, int64_t now_us, int64_t k, bool fallback,
-                          lv_victim* out, long long* count_dev, cudaStream_t s, int num_sms);
+                          lv_victim* out, long long* count_dev, cudaStream_t s, int num_sms,
+                          const long long* k_dev = nullptr);
 cudaError_t launch_alloc(const DevPool& p, bool hbm, int64_t n, int32_t* out, cudaStream_t s);
 cudaError_t launch_swap_out(const DevPool& p, const lv_victim* v, const int32_t* slots,
-                            int64_t n, lv_remap_entry* commit, cudaStream_t s, int num_sms);
+                            int64_t n, lv_remap_entry* commit, cudaStream_t s, int num_sms,
+                            const EventPair* ev = nullptr);
 cudaError_t launch_swap_in(const DevPool& p, int32_t sid, const int32_t* blks,
                            const int32_t* pages, int64_t n, lv_remap_entry* commit,
-                           cudaStream_t s, int num_sms);
+                           cudaStream_t s, int num_sms, const EventPair* ev = nullptr);
 cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out, int32_t sid,
                             const int32_t* blks, int64_t n_in, int32_t* slots, int32_t* pages,
                             int4* tasks, long long* n_tasks, int32_t epoch,
-                            unsigned long long* page_tag, cudaStream_t s, int copy_ctas);
+                            unsigned long long* page_tag, cudaStream_t s, int copy_ctas,
+                            const long long* counts_dev = nullptr, long long max_units = 0,
+                            const EventPair* ev = nullptr);
 cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, int32_t epoch,
                          cudaStream_t s);
 cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cudaStream_t s);
 cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32_t* pages,
-                          int32_t* count, cudaStream_t s);
+                          int32_t* count, cudaStream_t s, const long long* gate = nullptr);
+
+// Device buffers of lv_make_resident, owned by the pool.
+struct ResidentScratch {
+  lv_victim* victims;   // [budget]
+  int32_t* slots;       // [budget]
+  int32_t* blocks;      // [maxB]
+  int32_t* pages;       // [maxB]
+  int32_t* append;      // [maxB + 2]
+  int4* tasks;          // [budget + maxB]
+  long long* words;     // [16]
+};
+cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, int32_t sid,
+                                 int64_t now_us, int32_t append_tokens, bool preload,
+                                 int64_t max_load, int32_t epoch, cudaStream_t s, int copy_ctas,
+                                 lv_resident_result* result, const EventPair* ev = nullptr);
 cudaError_t launch_counts(const DevPool& p, int32_t* hbm, int32_t* host, cudaStream_t s);
 cudaError_t launch_blocks(const DevPool& p, int32_t sid, int32_t where, int32_t* out,
                           long long* count, cudaStream_t s);

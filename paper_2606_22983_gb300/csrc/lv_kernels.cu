@@ -290,7 +290,9 @@ constexpr int kSortThreads = 1024;
 // One CTA: bitonic sort of the session keys (descending), scan of the counts
 // in rank order, and the number of victims to emit.
 __global__ void __launch_bounds__(kSortThreads)
-k_rank_sort(DevPool p, long long k, bool fallback, long long* count_dev, int N) {
+k_rank_sort(DevPool p, long long k, const long long* k_dev, bool fallback, long long* count_dev,
+            int N) {
+  if (k_dev) k = *k_dev;   // k decided on the device (lv_make_resident)
   extern __shared__ unsigned char smem_raw[];
   unsigned long long* keys = reinterpret_cast<unsigned long long*>(smem_raw);
   int32_t* vals = reinterpret_cast<int32_t*>(keys + N);
@@ -499,7 +501,12 @@ __global__ void __launch_bounds__(kPlanThreads)
 k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int32_t sid,
                 const int32_t* __restrict__ blks, long long n_in, int32_t* __restrict__ slots,
                 int32_t* __restrict__ pages, int4* __restrict__ tasks, long long* n_tasks,
-                int32_t epoch, unsigned long long* __restrict__ page_tag) {
+                int32_t epoch, unsigned long long* __restrict__ page_tag,
+                const long long* __restrict__ counts_dev) {
+  if (counts_dev) {          // counts decided on the device (lv_make_resident)
+    n_out = counts_dev[0];
+    n_in = counts_dev[1];
+  }
   __shared__ int bad;
   if (threadIdx.x == 0) bad = 0;
   __syncthreads();
@@ -724,8 +731,12 @@ __global__ void k_cancel(DevPool p, const int32_t* __restrict__ locs, long long 
 
 __global__ void __launch_bounds__(kAllocThreads)
 k_append(DevPool p, int32_t sid, int32_t n_tokens, int32_t* __restrict__ pages,
-         int32_t* __restrict__ count) {
+         int32_t* __restrict__ count, const long long* __restrict__ gate) {
   __shared__ long long m_s, nb_s, ctx_s;
+  if (gate && *gate != 0) {   // an earlier step of lv_make_resident did not complete
+    if (threadIdx.x == 0 && count) *count = 0;
+    return;
+  }
   if (threadIdx.x == 0) {
     long long m = -1;
     if (sid >= 0 && sid < p.S && n_tokens >= 0) {
@@ -773,6 +784,109 @@ k_append(DevPool p, int32_t sid, int32_t n_tokens, int32_t* __restrict__ pages,
     p.sess[sid].ctx_tokens = (int32_t)ctx_s;
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_APPENDED]), (unsigned long long)m);
     if (count) *count = (int32_t)m;
+  }
+}
+
+// -------------------------------------------------------- make_resident
+// Words shared by the steps of one lv_make_resident call.
+enum ResWord : int {
+  R_K_SELECT = 0,   // k handed to the ranker (0 when nothing is to be evicted)
+  R_N_OUT = 1,      // victims the exchange evicts
+  R_N_IN = 2,       // host blocks the exchange loads
+  R_STATUS = 3,     // LV_RESIDENT_*
+  R_K = 4,          // pages the budget was short
+  R_GATE = 5,       // 0: the append may run
+  R_N_TASKS = 6,
+  R_APPENDED = 7,   // int32 count of appended pages, in the low half
+  R_FOUND = 8       // victims the ranking found
+};
+
+// One CTA: sid's host-tier blocks (ascending), the deficit k and the admission.
+__global__ void __launch_bounds__(kCensusThreads)
+k_resident_prepare(DevPool p, int32_t sid, int32_t append_tokens, bool preload,
+                   long long max_load, int32_t* __restrict__ blocks, long long* __restrict__ R) {
+  const int32_t nb = nblocks_of(p, sid);
+  const int32_t* row = p.table + (size_t)sid * p.maxB;
+  long long run = 0;
+  for (int32_t q0 = 0; q0 < nb; q0 += kCensusThreads) {
+    const int32_t b = q0 + threadIdx.x;
+    const long long flag = (b < nb && row[b] <= -2) ? 1 : 0;
+    long long chunk;
+    const long long pos = run + block_excl_scan<kCensusThreads>(flag, &chunk);
+    if (flag) blocks[pos] = b;
+    run += chunk;
+  }
+  if (threadIdx.x == 0) {
+    const long long nh = run;
+    const long long ctx = p.sess[sid].ctx_tokens;
+    const long long nctx = ctx + append_tokens;
+    const long long nnb = (nctx + p.T - 1) / p.T;
+    int status = LV_RESIDENT_DONE;
+    long long k = 0;
+    if (nnb > p.maxB || nctx > 0x7fffffffll) {
+      set_error(p.ctl, LV_ERR_BOUNDS, sid);
+      status = LV_RESIDENT_FAILED;
+    } else {
+      const long long need = nh + (nnb - nb);
+      const long long free_pages = p.budget - p.ctl[C_HBM_ALLOC];
+      k = need - free_pages > 0 ? need - free_pages : 0;
+      if (preload && nh == 0) status = LV_RESIDENT_NOTHING;
+      else if (preload && max_load >= 0 && nh > max_load) status = LV_RESIDENT_SKIPPED;
+    }
+    const bool go = status == LV_RESIDENT_DONE;
+    R[R_K_SELECT] = go ? k : 0;
+    R[R_N_OUT] = 0;
+    R[R_N_IN] = go ? nh : 0;
+    R[R_STATUS] = status;
+    R[R_K] = k;
+    R[R_GATE] = go ? 0 : 1;
+    R[R_APPENDED] = 0;
+    R[R_FOUND] = 0;
+    if (preload && status == LV_RESIDENT_SKIPPED)
+      atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PRELOADS_SKIPPED]), 1ull);
+  }
+}
+
+// After the ranking: a shortfall stops the step (a preload is skipped, a
+// foreground turn fails), otherwise the exchange evicts exactly k victims.
+__global__ void k_resident_gate(DevPool p, bool preload, long long* __restrict__ R) {
+  if (threadIdx.x != 0 || R[R_STATUS] != LV_RESIDENT_DONE) return;
+  const long long found = p.ctl[C_SEL_COUNT], k = R[R_K];
+  R[R_FOUND] = found;
+  if (found < k) {
+    if (preload) {
+      R[R_STATUS] = LV_RESIDENT_SKIPPED;
+      atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PRELOADS_SKIPPED]), 1ull);
+    } else {
+      set_error(p.ctl, LV_ERR_NO_HBM, k);
+      R[R_STATUS] = LV_RESIDENT_FAILED;
+    }
+    R[R_N_OUT] = 0;
+    R[R_N_IN] = 0;
+    R[R_GATE] = 1;
+  } else {
+    R[R_N_OUT] = k;
+  }
+}
+
+__global__ void k_resident_finish(DevPool p, int32_t sid, long long now_us, bool preload,
+                                  long long* __restrict__ R, lv_resident_result* __restrict__ out) {
+  if (threadIdx.x != 0) return;
+  const int status = (int)R[R_STATUS];
+  if (preload && status == LV_RESIDENT_DONE) {
+    p.sess[sid].protect_until_us = now_us + p.protect_us;   // warmed KV (Section 5.2)
+    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PRELOADS]), 1ull);
+  }
+  if (out) {
+    lv_resident_result r;
+    r.k = R[R_K];
+    r.n_found = R[R_FOUND];
+    r.n_victims = R[R_N_OUT];
+    r.n_loaded = R[R_N_IN];
+    r.n_appended = (int32_t)R[R_APPENDED];
+    r.status = status;
+    r.pad = 0;
+    *out = r;
   }
 }
 
@@ -847,12 +961,13 @@ cudaError_t launch_events(const DevPool& p, const lv_event* ev, int64_t n, cudaS
 }
 
 cudaError_t launch_select(const DevPool& p, int64_t now_us, int64_t k, bool fallback,
-                          lv_victim* out, long long* count_dev, cudaStream_t s, int /*num_sms*/) {
+                          lv_victim* out, long long* count_dev, cudaStream_t s, int /*num_sms*/,
+                          const long long* k_dev) {
   int N = 1;
   while (N < p.S) N <<= 1;
   const size_t smem = (size_t)N * (sizeof(unsigned long long) + sizeof(int32_t));
   k_rank_census<<<p.S, kCensusThreads, 0, s>>>(p, now_us, fallback);
-  k_rank_sort<<<1, kSortThreads, smem, s>>>(p, k, fallback, count_dev, N);
+  k_rank_sort<<<1, kSortThreads, smem, s>>>(p, k, k_dev, fallback, count_dev, N);
   k_rank_emit<<<p.S, kEmitThreads, 0, s>>>(p, out);
   return cudaGetLastError();
 }
@@ -868,29 +983,60 @@ cudaError_t launch_alloc(const DevPool& p, bool hbm, int64_t n, int32_t* out, cu
 }
 
 cudaError_t launch_swap_out(const DevPool& p, const lv_victim* v, const int32_t* slots, int64_t n,
-                            lv_remap_entry* commit, cudaStream_t s, int num_sms) {
+                            lv_remap_entry* commit, cudaStream_t s, int num_sms, const EventPair* ev) {
   const long long units = (long long)n * p.J;
+  if (ev) cudaEventRecord(ev->start, s);
   k_swap_out<<<blocks_for(units, 1, (long long)num_sms * 8), kCopyThreads, 0, s>>>(
       p, v, slots, n, commit);
+  if (ev) cudaEventRecord(ev->end, s);
   return cudaGetLastError();
 }
 
 cudaError_t launch_swap_in(const DevPool& p, int32_t sid, const int32_t* blks, const int32_t* pages,
-                           int64_t n, lv_remap_entry* commit, cudaStream_t s, int num_sms) {
+                           int64_t n, lv_remap_entry* commit, cudaStream_t s, int num_sms,
+                           const EventPair* ev) {
   const long long units = (long long)n * p.J;
+  if (ev) cudaEventRecord(ev->start, s);
   k_swap_in<<<blocks_for(units, 1, (long long)num_sms * 8), kCopyThreads, 0, s>>>(
       p, sid, blks, pages, n, commit);
+  if (ev) cudaEventRecord(ev->end, s);
   return cudaGetLastError();
 }
 
 cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out, int32_t sid,
                             const int32_t* blks, int64_t n_in, int32_t* slots, int32_t* pages,
                             int4* tasks, long long* n_tasks, int32_t epoch,
-                            unsigned long long* page_tag, cudaStream_t s, int copy_ctas) {
+                            unsigned long long* page_tag, cudaStream_t s, int copy_ctas,
+                            const long long* counts_dev, long long max_units, const EventPair* ev) {
   k_exchange_plan<<<1, kPlanThreads, 0, s>>>(p, v, n_out, sid, blks, n_in, slots, pages, tasks,
-                                             n_tasks, epoch, page_tag);
-  const long long units = (n_out + n_in) * (long long)p.J;
+                                             n_tasks, epoch, page_tag, counts_dev);
+  const long long units = counts_dev ? max_units : (n_out + n_in) * (long long)p.J;
+  if (ev) cudaEventRecord(ev->start, s);
   k_exchange_copy<<<blocks_for(units, 1, copy_ctas), kCopyThreads, 0, s>>>(p, tasks, n_tasks);
+  if (ev) cudaEventRecord(ev->end, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, int32_t sid,
+                                 int64_t now_us, int32_t append_tokens, bool preload,
+                                 int64_t max_load, int32_t epoch, cudaStream_t s, int copy_ctas,
+                                 lv_resident_result* result, const EventPair* ev) {
+  long long* R = rs.words;
+  k_resident_prepare<<<1, kCensusThreads, 0, s>>>(p, sid, append_tokens, preload, max_load,
+                                                  rs.blocks, R);
+  cudaError_t e = launch_select(p, now_us, 0, !preload, rs.victims, nullptr, s, 0, R + R_K_SELECT);
+  if (e != cudaSuccess) return e;
+  k_resident_gate<<<1, 32, 0, s>>>(p, preload, R);
+  const long long max_units = ((long long)p.budget + p.maxB) * p.J;
+  e = launch_exchange(p, rs.victims, 0, sid, rs.blocks, 0, rs.slots, rs.pages, rs.tasks,
+                      R + R_N_TASKS, epoch, p.page_tag, s, copy_ctas, R + R_N_OUT, max_units, ev);
+  if (e != cudaSuccess) return e;
+  if (append_tokens > 0) {
+    e = launch_append(p, sid, append_tokens, rs.append, reinterpret_cast<int32_t*>(R + R_APPENDED), s,
+                      R + R_GATE);
+    if (e != cudaSuccess) return e;
+  }
+  k_resident_finish<<<1, 32, 0, s>>>(p, sid, now_us, preload, R, result);
   return cudaGetLastError();
 }
 
@@ -906,8 +1052,8 @@ cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cuda
 }
 
 cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32_t* pages,
-                          int32_t* count, cudaStream_t s) {
-  k_append<<<1, kAllocThreads, 0, s>>>(p, sid, n_tokens, pages, count);
+                          int32_t* count, cudaStream_t s, const long long* gate) {
+  k_append<<<1, kAllocThreads, 0, s>>>(p, sid, n_tokens, pages, count, gate);
   return cudaGetLastError();
 }
 

@@ -56,10 +56,20 @@ class lv_stats(ctypes.Structure):
         "hbm_allocated", "host_allocated", "hbm_budget_pages", "host_pages", "error",
         "error_detail", "last_select_count", "last_select_total", "selects", "victims",
         "shortfalls", "pages_out", "pages_in", "bytes_out", "bytes_in", "remap_entries",
-        "appended_pages", "cancels", "events", "fallback_selects")]
+        "appended_pages", "cancels", "events", "fallback_selects", "preloads",
+        "preloads_skipped")]
 
     def as_dict(self):
         return {n: int(getattr(self, n)) for n, _ in self._fields_}
+
+
+class lv_kernel_timing(ctypes.Structure):
+    _fields_ = [("launches", ctypes.c_int64), ("total_ms", ctypes.c_double),
+                ("min_ms", ctypes.c_double), ("max_ms", ctypes.c_double)]
+
+
+LV_TIMING_SWAP_OUT, LV_TIMING_SWAP_IN, LV_TIMING_EXCHANGE, LV_TIMING_KINDS = 0, 1, 2, 3
+TIMING_NAMES = ("swap_out", "swap_in", "exchange")
 
 
 class lv_rank_params(ctypes.Structure):
@@ -70,6 +80,8 @@ class lv_rank_params(ctypes.Structure):
 
 
 LV_NOALLOC_MAX_SESSIONS = 4096
+LV_RESIDENT_PRELOAD = 1
+LV_RESIDENT_DONE, LV_RESIDENT_SKIPPED, LV_RESIDENT_NOTHING, LV_RESIDENT_FAILED = 0, 1, 2, 3
 
 # numpy views of the ABI's array element types
 SESSION_DTYPE = np.dtype([("ctx_tokens", "<i4"), ("flags", "<i4"), ("gen_us", "<i8"),
@@ -78,6 +90,8 @@ SESSION_DTYPE = np.dtype([("ctx_tokens", "<i4"), ("flags", "<i4"), ("gen_us", "<
                           ("protect_until_us", "<i8")])
 EVENT_DTYPE = np.dtype([("kind", "<i4"), ("sid", "<i4"), ("t_us", "<i8"), ("a", "<i8"), ("b", "<i8")])
 VICTIM_DTYPE = np.dtype([("sid", "<i4"), ("blk", "<i4"), ("page", "<i4")])
+RESIDENT_DTYPE = np.dtype([("k", "<i8"), ("n_found", "<i8"), ("n_victims", "<i8"), ("n_loaded", "<i8"),
+                           ("n_appended", "<i8"), ("status", "<i4"), ("pad", "<i4")])
 REMAP_DTYPE = np.dtype([("sid", "<i4"), ("blk", "<i4"), ("loc", "<i4")])
 assert SESSION_DTYPE.itemsize == 64 and EVENT_DTYPE.itemsize == 32
 assert VICTIM_DTYPE.itemsize == 12 and REMAP_DTYPE.itemsize == 12
@@ -100,6 +114,9 @@ def _load():
         "lv_swap_out": [vp, vp, i64, vp, vp, i32, vp],
         "lv_swap_in": [vp, i32, vp, i64, vp, vp, i32, vp],
         "lv_swap_exchange": [vp, vp, i64, i32, vp, i64, vp, vp, i32, vp],
+        "lv_make_resident": [vp, i32, i64, i32, u32, i64, vp, vp, vp, vp, vp, vp, vp],
+        "lv_timing_enable": [vp, i32],
+        "lv_timing_read": [vp, ctypes.POINTER(lv_kernel_timing), i32],
         "lv_remap": [vp, vp, i64, vp],
         "lv_cancel": [vp, vp, i64, vp],
         "lv_session_append": [vp, i32, i32, vp, vp, vp],
@@ -129,10 +146,10 @@ _lib = _load()
 
 EXPORTED = ("lv_pool_create", "lv_pool_destroy", "lv_pool_host_ptr", "lv_pool_import",
             "lv_session_set", "lv_session_get", "lv_session_events", "lv_select_victims",
-            "lv_swap_out", "lv_swap_in", "lv_swap_exchange", "lv_remap", "lv_cancel", "lv_session_append",
+            "lv_swap_out", "lv_swap_in", "lv_swap_exchange", "lv_make_resident", "lv_remap", "lv_cancel", "lv_session_append",
             "lv_session_counts", "lv_session_blocks", "lv_read_tables", "lv_sync",
             "lv_get_stats", "lv_clear_error", "lv_status_str", "lv_version",
-            "lv_select_victims_noalloc")
+            "lv_select_victims_noalloc", "lv_timing_enable", "lv_timing_read")
 
 
 def lib():
@@ -225,6 +242,14 @@ def lv_swap_exchange(pool, victims, n_out, sid, blks, n_in, slots_out, pages_out
                                  ptr(pages_out), mode, stream_handle(stream)), "lv_swap_exchange")
 
 
+def lv_make_resident(pool, sid, now_us, append_tokens, flags, max_load_pages, victims_out,
+                     slots_out, blocks_out, pages_out, append_out, result_out, stream=None):
+    _check(_lib.lv_make_resident(pool, sid, now_us, append_tokens, flags, max_load_pages,
+                                 ptr(victims_out), ptr(slots_out), ptr(blocks_out), ptr(pages_out),
+                                 ptr(append_out), ptr(result_out), stream_handle(stream)),
+           "lv_make_resident")
+
+
 def lv_remap(pool, entries, n, stream=None):
     _check(_lib.lv_remap(pool, ptr(entries), n, stream_handle(stream)), "lv_remap")
 
@@ -275,6 +300,18 @@ def lv_select_victims_noalloc(params: lv_rank_params, sessions, tables, now_us, 
     _check(_lib.lv_select_victims_noalloc(ctypes.byref(params), ptr(sessions), ptr(tables), now_us,
                                           k, ptr(out), capacity, ptr(count_out),
                                           stream_handle(stream)), "lv_select_victims_noalloc")
+
+
+def lv_timing_enable(pool, enable=True):
+    _check(_lib.lv_timing_enable(pool, 1 if enable else 0), "lv_timing_enable")
+
+
+def lv_timing_read(pool, reset=False) -> dict:
+    arr = (lv_kernel_timing * LV_TIMING_KINDS)()
+    _check(_lib.lv_timing_read(pool, arr, 1 if reset else 0), "lv_timing_read")
+    return {TIMING_NAMES[i]: {"launches": int(arr[i].launches), "total_ms": arr[i].total_ms,
+                              "min_ms": arr[i].min_ms, "max_ms": arr[i].max_ms}
+            for i in range(LV_TIMING_KINDS)}
 
 
 def lv_status_str(status: int) -> str:

@@ -9,10 +9,11 @@ Consumes monitor event scripts (records ``(t_us, kind, sid, a, b, c, d)``):
   kind 5 BARGE_IN(sid)                kind 6 SPEECH_STOP(sid)
 
 A turn makes the session fully resident (a synchronous foreground load),
-grows its context, then records the reply.  By default the evictions and loads
-of one step go through lv_swap_exchange (both link directions at once);
-``exchange=False`` issues swap-out, commit, swap-in, commit one after the other,
-with the same result.  Speech start and barge-in trigger a
+grows its context, then records the reply.  By default (``driver="device"``)
+each step is one lv_make_resident call that decides and moves everything on the
+GPU without a host round trip; ``driver="exchange"`` ranks, reads the count back
+and calls lv_swap_exchange; ``driver="sequential"`` issues swap-out, commit,
+swap-in, commit one after the other.  All three give the same result.  Speech start and barge-in trigger a
 best-effort preload of the session's host blocks.  Making a session resident
 with ``need`` missing pages first evicts exactly ``k = need - free`` pages in
 the next-use order (foreground turns may also take protected, non-running KV
@@ -22,8 +23,7 @@ that finds fewer than k victims is skipped; a completed one protects the
 warmed KV for the pool's protection window.
 
 Every step runs in liblv's kernels; this class only decides which calls to
-make, reading back the few counts it needs to decide (free pages, host
-blocks, victims found).
+make (and, on the host-driven paths, reads back the few counts it needs).
 """
 from __future__ import annotations
 
@@ -47,7 +47,7 @@ def _event(kind, sid, t, a=0, b=0):
 
 class KVManager:
     def __init__(self, pool: KVPool, perms=None, on_append=None, rank_on="none", admit=None,
-                 mode=lv.LV_MODE_AUTO, record=True, exchange=True):
+                 mode=lv.LV_MODE_AUTO, record=True, driver="device"):
         self.pool = pool
         self.perms = perms
         self.on_append = on_append      # callback(sid, old_ctx, new_ctx, pages) after growth
@@ -55,7 +55,12 @@ class KVManager:
         self.admit = admit              # callback(manager, sid, now, n_host_blocks) -> bool
         self.mode = mode
         self.record = record
-        self.exchange = exchange        # one lv_swap_exchange instead of four sequential calls
+        if driver not in ("device", "exchange", "sequential"):
+            raise ValueError(f"unknown driver {driver!r}")
+        # device: one lv_make_resident per step, no host round trip;
+        # exchange: select, then one lv_swap_exchange; sequential: the four calls
+        self.driver = driver
+        self.res_h = torch.zeros(lv.RESIDENT_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
         self.counters = dict(victims=0, pages_out=0, pages_in=0, preloads=0,
                              preload_skipped=0, turns=0, sync_loads=0, appended=0)
         self.bytes_moved = 0
@@ -76,7 +81,59 @@ class KVManager:
         return int(self.pool.get_sessions()["ctx_tokens"][sid])
 
     # ------------------------------------------------------------ movement
+    def _device(self, sid, now_us, append_tokens, foreground, rec):
+        pool = self.pool
+        flags = 0 if foreground else lv.LV_RESIDENT_PRELOAD
+        rec_bufs = self.record or self.on_append is not None
+        old_ctx = self.ctx_tokens(sid) if (append_tokens and self.on_append is not None) else 0
+        outs = (pool.victims, pool.slots, pool.blks, pool.pages, pool.app) if rec_bufs else (None,) * 5
+        if self.timer:
+            self.timer.start("resident")
+        lv.lv_make_resident(pool.handle, sid, now_us, append_tokens, flags, -1, *outs,
+                            self.res_h, pool.stream)
+        pool.launches += 8 + (1 if append_tokens else 0)
+        if self.timer:
+            self.timer.stop("resident", None)
+        if not rec_bufs:
+            return None
+        pool.sync()
+        r = self.res_h.numpy().view(lv.RESIDENT_DTYPE)[0]
+        k, found, nv, nl, na, status = (int(r["k"]), int(r["n_found"]), int(r["n_victims"]),
+                                        int(r["n_loaded"]), int(r["n_appended"]), int(r["status"]))
+        if status == lv.LV_RESIDENT_NOTHING:
+            return status
+        rec["k"] = k
+        if self.record:
+            if k > 0:
+                rec["victims"] = pool.victims[:found].cpu().numpy().astype(np.int64)
+                self.last_readback_bytes += found * 12
+            if nv:
+                rec["slots"] = pool.slots[:nv].cpu().numpy().astype(np.int64)
+                self.last_readback_bytes += nv * 4
+            if nl:
+                rec["in_blocks"] = pool.blks[:nl].cpu().numpy().astype(np.int64)
+                rec["in_pages"] = pool.pages[:nl].cpu().numpy().astype(np.int64)
+                self.last_readback_bytes += nl * 8
+            if append_tokens:
+                rec["append_pages"] = pool.app[:na].cpu().numpy().astype(np.int64)
+        self.counters["victims"] += nv
+        self.counters["pages_out"] += nv
+        self.counters["pages_in"] += nl
+        self.counters["appended"] += na
+        self.bytes_moved += (nv + nl) * pool.J * pool.P
+        if foreground and nl:
+            self.counters["sync_loads"] += 1
+        if status == lv.LV_RESIDENT_DONE and append_tokens and self.on_append is not None:
+            self.on_append(sid, old_ctx, old_ctx + append_tokens)
+        return status
+
     def make_resident(self, sid, now_us, append_tokens, foreground, rec):
+        if self.driver == "device":
+            status = self._device(sid, now_us, append_tokens, foreground, rec)
+            if status == lv.LV_RESIDENT_FAILED:
+                raise lv.LvError(self.pool.sync(raise_on_error=False) or lv.LV_ERR_NO_HBM,
+                                 f"turn of session {sid}")
+            return status
         pool = self.pool
         hblk, nh = self.host_blocks(sid)
         new_blocks = 0
@@ -87,7 +144,7 @@ class KVManager:
         need = nh + new_blocks
         k = max(0, need - self.free_budget())
         rec["k"] = k
-        if self.exchange:
+        if self.driver == "exchange":
             if not self._exchange(sid, now_us, k, hblk, nh, foreground, rec):
                 return False
         else:
@@ -178,6 +235,15 @@ class KVManager:
         return True
 
     def preload(self, sid, now_us, rec):
+        if self.driver == "device" and self.admit is None:
+            status = self._device(sid, now_us, 0, False, rec)
+            if status == lv.LV_RESIDENT_DONE:
+                self.counters["preloads"] += 1
+                rec["preload"] = "done"
+            elif status == lv.LV_RESIDENT_SKIPPED:
+                self.counters["preload_skipped"] += 1
+                rec["preload"] = "skipped"
+            return
         _, nh = self.host_blocks(sid)
         if nh == 0:
             return
@@ -214,7 +280,7 @@ class KVManager:
             if kind == EV_TURN_ANY:
                 sid = self.turn_target(d)
             pool.events(_event(lv.LV_EV_TURN_BEGIN, sid, t))
-            if self.host_blocks(sid)[1]:
+            if self.driver != "device" and self.host_blocks(sid)[1]:
                 self.counters["sync_loads"] += 1
             self.make_resident(sid, t, a, foreground=True, rec=rec)
             pool.events(_event(lv.LV_EV_TURN_END, sid, t, b, c))

@@ -55,6 +55,7 @@ class KVPool:
             self.slots = torch.empty(cap, dtype=torch.int32, device=dev)
             self.pages = torch.empty(cap, dtype=torch.int32, device=dev)
             self.blks = torch.empty(max_blocks, dtype=torch.int32, device=dev)
+            self.app = torch.empty(max_blocks + 2, dtype=torch.int32, device=dev)
             self.count_h = torch.zeros(4, dtype=torch.int64).pin_memory()
         hp = lv.lv_pool_host_ptr(self.handle)
         self.host = None

@@ -54,7 +54,7 @@ def compare_state(om: OracleManager, pool, where, with_bytes):
         assert np.array_equal(pool.host, om.pool.host), (where, "host bytes")
 
 
-def make_pair(workload, with_bytes, rank_on="all", mode=lv.LV_MODE_AUTO, exchange=True):
+def make_pair(workload, with_bytes, rank_on="all", mode=lv.LV_MODE_AUTO, driver="device"):
     seed = workload.seed
     table = value_table(seed)
     om = OracleManager(workload, with_bytes=with_bytes, content=(seed, table) if with_bytes else None,
@@ -67,13 +67,13 @@ def make_pair(workload, with_bytes, rank_on="all", mode=lv.LV_MODE_AUTO, exchang
         writer.write_initial(workload)
     gm = KVManager(pool, perms=workload.perms,
                    on_append=writer.write_appended if writer else None,
-                   rank_on=rank_on, mode=mode, exchange=exchange)
+                   rank_on=rank_on, mode=mode, driver=driver)
     return om, pool, gm
 
 
 def run_lockstep(workload, with_bytes=True, check_every=50, n_events=None, rank_on="all",
-                 mode=lv.LV_MODE_AUTO, exchange=True):
-    om, pool, gm = make_pair(workload, with_bytes, rank_on, mode, exchange)
+                 mode=lv.LV_MODE_AUTO, driver="device"):
+    om, pool, gm = make_pair(workload, with_bytes, rank_on, mode, driver)
     n = workload.n_events if n_events is None else n_events
     try:
         compare_state(om, pool, "initial", with_bytes)

@@ -58,6 +58,9 @@ int main(void) {
   printf("sizeof lv_victim %zu\n", sizeof(lv_victim));
   printf("sizeof lv_remap_entry %zu\n", sizeof(lv_remap_entry));
   printf("sizeof lv_stats %zu\n", sizeof(lv_stats));
+  printf("sizeof lv_resident_result %zu\n", sizeof(lv_resident_result));
+  F(lv_resident_result, k); F(lv_resident_result, n_found); F(lv_resident_result, n_victims);
+  F(lv_resident_result, n_loaded); F(lv_resident_result, n_appended); F(lv_resident_result, status);
   F(lv_session_state, ctx_tokens); F(lv_session_state, flags); F(lv_session_state, gen_us);
   F(lv_session_state, play_us); F(lv_session_state, t_done_us); F(lv_session_state, reply_ema_us);
   F(lv_session_state, reply_n); F(lv_session_state, reply_tokens); F(lv_session_state, protect_until_us);
@@ -84,6 +87,10 @@ int main(void) {
     assert got["lv_remap_entry"] == lv.REMAP_DTYPE.itemsize
     assert got["lv_pool_desc"] == ctypes.sizeof(lv.lv_pool_desc)
     assert got["lv_stats"] == ctypes.sizeof(lv.lv_stats)
+    assert got["lv_resident_result"] == lv.RESIDENT_DTYPE.itemsize
+    for name in lv.RESIDENT_DTYPE.names:
+        if name != "pad":
+            assert lv.RESIDENT_DTYPE.fields[name][1] == got[f"lv_resident_result.{name}"][0], name
     for name in lv.SESSION_DTYPE.names:
         if name == "pad":
             continue

@@ -10,14 +10,15 @@ from ._lockstep import run_lockstep
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("seed,exchange", [(0, True), (1, True), (0, False)])
-def test_tiny_workload_full_images(seed, exchange):
+@pytest.mark.parametrize("seed,driver", [(0, "device"), (1, "device"), (0, "exchange"),
+                                         (1, "sequential")])
+def test_tiny_workload_full_images(seed, driver):
     """1000 scripted events of the tiny pool: every ranking (full order after
     each event), eviction, preload, reload and growth, with full HBM and host
-    byte images compared every 50 events -- through lv_swap_exchange and
-    through the four sequential calls."""
+    byte images compared every 50 events -- through lv_make_resident, through
+    select + lv_swap_exchange, and through the four sequential calls."""
     wl = make_workload("tiny", seed)
-    om, gm = run_lockstep(wl, with_bytes=True, check_every=50, exchange=exchange)
+    om, gm = run_lockstep(wl, with_bytes=True, check_every=50, driver=driver)
     assert om.counters == gm.counters
     assert gm.counters["pages_out"] > 500 and gm.counters["preloads"] > 10
 
@@ -39,7 +40,8 @@ def _expected_block(seed, table, shape, sid, blk, ctx):
     return subpage_values_np(table, off, rows, shape).view(np.uint8).reshape(J, -1)
 
 
-def test_thinker_full_size_sampled_bytes():
+@pytest.mark.parametrize("driver", ["device", "exchange"])
+def test_thinker_full_size_sampled_bytes(driver):
     """The thinker pool at full size (40 GB HBM budget, 1.5 MiB pages), in the
     launch configuration the benchmark times: every turn's victims, host slots
     and pages match the oracle; afterwards the tables and owners match, and
@@ -58,7 +60,7 @@ def test_thinker_full_size_sampled_bytes():
     try:
         writer = ContentWriter(pool, wl)
         writer.write_initial(wl)
-        gm = KVManager(pool, perms=wl.perms, rank_on="turns")
+        gm = KVManager(pool, perms=wl.perms, rank_on="turns", driver=driver)
         last = None
         for i in range(wl.n_events):
             ro, rg = om.step(i), gm.step(wl.event(i), i)
