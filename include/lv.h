@@ -238,7 +238,9 @@ lv_status lv_select_victims(lv_pool* pool, int64_t now_us, int64_t k, uint32_t f
    (lv_remap_entry [n], may be NULL) ready-to-commit entries.  mode:
    LV_MODE_ZERO_COPY (SM copies straight into the mapped host pool),
    LV_MODE_STAGED (pack into HBM staging, then copy-engine transfer) or
-   LV_MODE_AUTO.  Device-detected: LV_ERR_NO_HOST (nothing reserved or copied),
+   LV_MODE_AUTO (zero-copy).  LV_MODE_STAGED reads the reserved slots back
+   to build one copy per contiguous slot run, so it waits on the host for the
+   work queued before it on `stream` (and for the reservation).  Device-detected: LV_ERR_NO_HOST (nothing reserved or copied),
    LV_ERR_BOUNDS, LV_ERR_STATE (a victim is not resident where it says). */
 lv_status lv_swap_out(lv_pool* pool, const lv_victim* victims, int64_t n, int32_t* slots_out,
                       lv_remap_entry* commit_out, int32_t mode, lv_stream stream);
@@ -248,6 +250,9 @@ lv_status lv_swap_out(lv_pool* pool, const lv_victim* victims, int64_t n, int32_
    each listed host-resident block of session sid into its page.  Does not
    change the block tables.  pages_out (int32 [n]) and commit_out
    (lv_remap_entry [n]) may be NULL.  A preload is this call on a side stream.
+   mode as for lv_swap_out (LV_MODE_STAGED: copy-engine transfer of each
+   contiguous slot run into HBM staging, then an unpack kernel; it waits on
+   the host for the work queued before it).
    Device-detected: LV_ERR_NO_HBM (budget short: nothing reserved or copied),
    LV_ERR_BOUNDS, LV_ERR_STATE (a block is not in the host tier). */
 lv_status lv_swap_in(lv_pool* pool, int32_t sid, const int32_t* blks, int64_t n,
@@ -266,7 +271,10 @@ lv_status lv_swap_in(lv_pool* pool, int32_t sid, const int32_t* blks, int64_t n,
    one small kernel; then one copy kernel moves both directions together (an
    incoming block that lands on a victim's old page is copied by the same
    thread right after it read the old bytes), so the host link carries data
-   both ways at once.  Either list may be empty.  The whole call is validated
+   both ways at once.  LV_MODE_STAGED instead packs the evicted pages into HBM
+   staging and unpacks the loaded ones, with the copy engines carrying one
+   transfer per contiguous slot run in each direction on two side streams (it
+   waits on the host for the plan).  Either list may be empty.  The whole call is validated
    before anything changes: on LV_ERR_STATE / LV_ERR_BOUNDS (a victim not
    resident where it says, a block not in the host tier, a block listed twice),
    LV_ERR_NO_HOST or LV_ERR_NO_HBM (device-detected) nothing is reserved,
@@ -415,13 +423,14 @@ lv_status lv_get_stats(lv_pool* pool, lv_stats* out, lv_stream stream);
 lv_status lv_clear_error(lv_pool* pool, lv_stream stream);
 
 /* Instrumentation (Section 6: counters that validate which paths run).  While
-   enabled, every launch of a copy kernel -- swap-out, swap-in, exchange -- is
-   bracketed by two CUDA events recorded on its own stream.  lv_timing_read
-   waits for them and reports, per kernel kind (index LV_TIMING_SWAP_OUT,
-   _SWAP_IN, _EXCHANGE), the launches and their summed, shortest and longest
+   enabled, every launch of a copy kernel -- swap-out, swap-in, exchange, and the
+   staged path's pack and unpack -- is bracketed by two CUDA events recorded on
+   its own stream.  lv_timing_read waits for them and reports, per kernel kind
+   (index LV_TIMING_*), the launches and their summed, shortest and longest
    durations; reset != 0 starts a new record.  Enabling it adds two event
    records per launch and nothing else. */
-enum { LV_TIMING_SWAP_OUT = 0, LV_TIMING_SWAP_IN = 1, LV_TIMING_EXCHANGE = 2, LV_TIMING_KINDS = 3 };
+enum { LV_TIMING_SWAP_OUT = 0, LV_TIMING_SWAP_IN = 1, LV_TIMING_EXCHANGE = 2, LV_TIMING_PACK = 3,
+       LV_TIMING_UNPACK = 4, LV_TIMING_KINDS = 5 };
 typedef struct lv_kernel_timing {
   int64_t launches;
   double total_ms;

@@ -1,5 +1,6 @@
 // C-ABI entry points of liblv (see include/lv.h): argument checks, device
 // metadata, staging of host-pointer arguments, and kernel launches.
+#include <algorithm>
 #include <cstdint>
 #include <cstdlib>
 #include <cstring>
@@ -15,6 +16,12 @@ struct lv_pool {
   int32_t epoch = 0;
   int exchange_ctas = 0;           // grid of the exchange copy kernel
   lv::ResidentScratch rs{};        // lv_make_resident buffers
+  // staged path: side streams for the copy engines, a host copy of the tasks, sync events
+  cudaStream_t s_d2h = nullptr, s_h2d = nullptr;
+  int4* tasks_host = nullptr;
+  size_t tasks_host_cap = 0;
+  std::vector<cudaEvent_t> sync_events;
+  int stage_ctas = 0;
   // copy-kernel timing (lv_timing_enable): event pairs recorded per kind, reused
   bool timing = false;
   std::vector<lv::EventPair> ev_free;
@@ -161,7 +168,102 @@ const lv::EventPair* timing_pair(lv_pool* pool, int kind) {
   return &pool->ev_used[kind].back();
 }
 
+// At least n timing-free events, created on first use and reused.
+lv_status sync_events(lv_pool* pool, size_t n) {
+  while (pool->sync_events.size() < n) {
+    cudaEvent_t e;
+    if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return LV_ERR_CUDA;
+    pool->sync_events.push_back(e);
+  }
+  return LV_OK;
+}
+
+// The staged data movement of n validated tasks {out page, out slot, in slot, in page}
+// on `s`: pack out pages into staging, copy-engine runs of consecutive slots in each
+// direction on the side streams, unpack into the in pages; joined back into `s`.
+lv_status staged_move(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStream_t s) {
+  const lv::DevPool& d = pool->d;
+  if (n <= 0) return LV_OK;
+  if ((size_t)n > pool->tasks_host_cap) return LV_ERR_INVALID;
+  LV_TRY(cudaMemcpyAsync(pool->tasks_host, tasks_dev, (size_t)n * sizeof(int4), cudaMemcpyDeviceToHost, s));
+  LV_TRY(cudaStreamSynchronize(s));
+  const int4* t = pool->tasks_host;
+  const size_t pb = (size_t)d.J * d.P;
+  const int64_t chunk = std::max<int64_t>(1, (int64_t)((96u << 20) / pb));
+  const int64_t nchunks = (n + chunk - 1) / chunk;
+  lv_status st = sync_events(pool, (size_t)(2 * nchunks + 3));
+  if (st != LV_OK) return st;
+  cudaEvent_t* ev = pool->sync_events.data();
+  cudaEvent_t ev_start = ev[0], ev_d2h_done = ev[1], ev_h2d_done = ev[2];
+  cudaEvent_t* ev_pack = ev + 3;            // [nchunks]
+  cudaEvent_t* ev_h2d = ev + 3 + nchunks;   // [nchunks]
+  bool any_out = false, any_in = false;
+  for (int64_t i = 0; i < n; ++i) {
+    any_out |= t[i].x >= 0;
+    any_in |= t[i].z >= 0;
+  }
+  // staging[t] per direction: out pages are packed into one run, in pages land in another
+  void* staging = nullptr;
+  {
+    const size_t bytes = (size_t)n * pb * ((any_out ? 1 : 0) + (any_in ? 1 : 0));
+    cudaError_t e = cudaMallocFromPoolAsync(&staging, bytes, pool->mp, s);
+    if (e != cudaSuccess) return lv_cuda_fail(e);
+  }
+  uint8_t* stg_out = static_cast<uint8_t*>(staging);
+  uint8_t* stg_in = stg_out + (any_out ? (size_t)n * pb : 0);
+  uint8_t* host = static_cast<uint8_t*>(pool->host_base);
+  LV_TRY(cudaEventRecord(ev_start, s));
+  LV_TRY(cudaStreamWaitEvent(pool->s_d2h, ev_start, 0));
+  LV_TRY(cudaStreamWaitEvent(pool->s_h2d, ev_start, 0));
+  // H2D first so that the inbound copies start at once
+  for (int64_t c = 0; c < nchunks && any_in; ++c) {
+    const int64_t a = c * chunk, b = std::min(n, a + chunk);
+    for (int64_t i = a; i < b;) {
+      if (t[i].z < 0) { ++i; continue; }
+      int64_t j = i + 1;
+      while (j < b && t[j].z == t[j - 1].z + 1) ++j;
+      LV_TRY(cudaMemcpyAsync(stg_in + (size_t)i * pb, host + (size_t)t[i].z * pb, (size_t)(j - i) * pb,
+                             cudaMemcpyHostToDevice, pool->s_h2d));
+      i = j;
+    }
+    LV_TRY(cudaEventRecord(ev_h2d[c], pool->s_h2d));
+  }
+  // pack every chunk on s; the D2H runs of chunk c follow its pack
+  for (int64_t c = 0; c < nchunks && any_out; ++c) {
+    const int64_t a = c * chunk, b = std::min(n, a + chunk);
+    LV_TRY(lv::launch_stage(d, true, tasks_dev, a, b, stg_out, s, pool->stage_ctas,
+                            timing_pair(pool, LV_TIMING_PACK)));
+    LV_TRY(cudaEventRecord(ev_pack[c], s));
+    LV_TRY(cudaStreamWaitEvent(pool->s_d2h, ev_pack[c], 0));
+    for (int64_t i = a; i < b;) {
+      if (t[i].x < 0) { ++i; continue; }
+      int64_t j = i + 1;
+      while (j < b && t[j].x >= 0 && t[j].y == t[j - 1].y + 1) ++j;
+      LV_TRY(cudaMemcpyAsync(host + (size_t)t[i].y * pb, stg_out + (size_t)i * pb, (size_t)(j - i) * pb,
+                             cudaMemcpyDeviceToHost, pool->s_d2h));
+      i = j;
+    }
+  }
+  // unpack each chunk once it has arrived (every pack precedes it on s)
+  for (int64_t c = 0; c < nchunks && any_in; ++c) {
+    const int64_t a = c * chunk, b = std::min(n, a + chunk);
+    LV_TRY(cudaStreamWaitEvent(s, ev_h2d[c], 0));
+    LV_TRY(lv::launch_stage(d, false, tasks_dev, a, b, stg_in, s, pool->stage_ctas,
+                            timing_pair(pool, LV_TIMING_UNPACK)));
+  }
+  LV_TRY(cudaEventRecord(ev_d2h_done, pool->s_d2h));
+  LV_TRY(cudaEventRecord(ev_h2d_done, pool->s_h2d));
+  LV_TRY(cudaStreamWaitEvent(s, ev_d2h_done, 0));
+  LV_TRY(cudaStreamWaitEvent(s, ev_h2d_done, 0));
+  LV_TRY(cudaFreeAsync(staging, s));
+  return LV_OK;
+}
+
 void free_pool(lv_pool* pool) {
+  for (cudaEvent_t e : pool->sync_events) cudaEventDestroy(e);
+  if (pool->s_d2h) cudaStreamDestroy(pool->s_d2h);
+  if (pool->s_h2d) cudaStreamDestroy(pool->s_h2d);
+  if (pool->tasks_host) cudaFreeHost(pool->tasks_host);
   for (auto& v : pool->ev_used)
     for (auto& e : v) pool->ev_free.push_back(e);
   for (auto& e : pool->ev_free) {
@@ -305,6 +407,17 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
   }
 
   if (lv::configure_kernels() != cudaSuccess) return fail(LV_ERR_CUDA);
+  if (lv::configure_stage_kernels(d) != cudaSuccess) return fail(LV_ERR_CUDA);
+  if (cudaStreamCreateWithFlags(&pool->s_d2h, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&pool->s_h2d, cudaStreamNonBlocking) != cudaSuccess)
+    return fail(LV_ERR_CUDA);
+  pool->tasks_host_cap = (size_t)d.budget + d.maxB + (size_t)d.host_pages;
+  if (cudaHostAlloc((void**)&pool->tasks_host, pool->tasks_host_cap * sizeof(int4), cudaHostAllocDefault) !=
+      cudaSuccess) {
+    pool->tasks_host = nullptr;
+    return fail(LV_ERR_OOM);
+  }
+  pool->stage_ctas = pool->num_sms;
   cudaMemPoolProps props{};
   props.allocType = cudaMemAllocationTypePinned;
   props.location.type = cudaMemLocationTypeDevice;
@@ -440,9 +553,10 @@ lv_status lv_select_victims(lv_pool* pool, int64_t now_us, int64_t k, uint32_t f
 lv_status lv_swap_out(lv_pool* pool, const lv_victim* victims, int64_t n, int32_t* slots_out,
                       lv_remap_entry* commit_out, int32_t mode, lv_stream stream) {
   if (!pool || n < 0 || n > 0x7fffffffll || (n > 0 && !victims)) return LV_ERR_INVALID;
-  if (mode != LV_MODE_AUTO && mode != LV_MODE_ZERO_COPY) return LV_ERR_INVALID;
+  if (mode != LV_MODE_AUTO && mode != LV_MODE_ZERO_COPY && mode != LV_MODE_STAGED) return LV_ERR_INVALID;
   if (n == 0) return LV_OK;
   if (pool->d.host_pages == 0) return LV_ERR_INVALID;
+  if (mode == LV_MODE_STAGED && (size_t)n > pool->tasks_host_cap) return LV_ERR_INVALID;
   DeviceGuard g(pool->device);
   cudaStream_t s = as_stream(stream);
   try {
@@ -455,6 +569,14 @@ lv_status lv_swap_out(lv_pool* pool, const lv_victim* victims, int64_t n, int32_
     if ((r = st.out(commit_out, (size_t)n * sizeof(lv_remap_entry), &cdev, false)) != LV_OK) return r;
     int32_t* slots = static_cast<int32_t*>(sdev);
     LV_TRY(lv::launch_alloc(pool->d, false, n, slots, s));
+    if (mode == LV_MODE_STAGED) {
+      void* tdev = nullptr;
+      if ((r = st.out(nullptr, (size_t)n * sizeof(int4), &tdev, true)) != LV_OK) return r;
+      LV_TRY(lv::launch_tasks_out(pool->d, static_cast<const lv_victim*>(vin), slots, n,
+                                  static_cast<int4*>(tdev), static_cast<lv_remap_entry*>(cdev), s));
+      if ((r = staged_move(pool, static_cast<int4*>(tdev), n, s)) != LV_OK) return r;
+      return st.finish();
+    }
     LV_TRY(lv::launch_swap_out(pool->d, static_cast<const lv_victim*>(vin), slots, n,
                                static_cast<lv_remap_entry*>(cdev), s, pool->num_sms,
                                timing_pair(pool, LV_TIMING_SWAP_OUT)));
@@ -467,8 +589,9 @@ lv_status lv_swap_out(lv_pool* pool, const lv_victim* victims, int64_t n, int32_
 lv_status lv_swap_in(lv_pool* pool, int32_t sid, const int32_t* blks, int64_t n, int32_t* pages_out,
                      lv_remap_entry* commit_out, int32_t mode, lv_stream stream) {
   if (!pool || n < 0 || n > 0x7fffffffll || (n > 0 && !blks)) return LV_ERR_INVALID;
-  if (mode != LV_MODE_AUTO && mode != LV_MODE_ZERO_COPY) return LV_ERR_INVALID;
+  if (mode != LV_MODE_AUTO && mode != LV_MODE_ZERO_COPY && mode != LV_MODE_STAGED) return LV_ERR_INVALID;
   if (sid < 0 || sid >= pool->d.S) return LV_ERR_INVALID;
+  if (mode == LV_MODE_STAGED && (size_t)n > pool->tasks_host_cap) return LV_ERR_INVALID;
   if (n == 0) return LV_OK;
   DeviceGuard g(pool->device);
   cudaStream_t s = as_stream(stream);
@@ -482,6 +605,14 @@ lv_status lv_swap_in(lv_pool* pool, int32_t sid, const int32_t* blks, int64_t n,
     if ((r = st.out(commit_out, (size_t)n * sizeof(lv_remap_entry), &cdev, false)) != LV_OK) return r;
     int32_t* pages = static_cast<int32_t*>(pdev);
     LV_TRY(lv::launch_alloc(pool->d, true, n, pages, s));
+    if (mode == LV_MODE_STAGED) {
+      void* tdev = nullptr;
+      if ((r = st.out(nullptr, (size_t)n * sizeof(int4), &tdev, true)) != LV_OK) return r;
+      LV_TRY(lv::launch_tasks_in(pool->d, sid, static_cast<const int32_t*>(bin), pages, n,
+                                 static_cast<int4*>(tdev), static_cast<lv_remap_entry*>(cdev), s));
+      if ((r = staged_move(pool, static_cast<int4*>(tdev), n, s)) != LV_OK) return r;
+      return st.finish();
+    }
     LV_TRY(lv::launch_swap_in(pool->d, sid, static_cast<const int32_t*>(bin), pages, n,
                               static_cast<lv_remap_entry*>(cdev), s, pool->num_sms,
                               timing_pair(pool, LV_TIMING_SWAP_IN)));
@@ -497,8 +628,9 @@ lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_ou
   if (!pool || n_out < 0 || n_in < 0 || n_out > 0x7fffffffll || n_in > 0x7fffffffll ||
       (n_out > 0 && !victims) || (n_in > 0 && !blks))
     return LV_ERR_INVALID;
-  if (mode != LV_MODE_AUTO && mode != LV_MODE_ZERO_COPY) return LV_ERR_INVALID;
+  if (mode != LV_MODE_AUTO && mode != LV_MODE_ZERO_COPY && mode != LV_MODE_STAGED) return LV_ERR_INVALID;
   if (n_in > 0 && (sid < 0 || sid >= pool->d.S)) return LV_ERR_INVALID;
+  if (mode == LV_MODE_STAGED && (size_t)(n_out + n_in) > pool->tasks_host_cap) return LV_ERR_INVALID;
   if (n_out > 0 && pool->d.host_pages == 0) return LV_ERR_INVALID;
   if (n_out == 0 && n_in == 0) return LV_OK;
   DeviceGuard g(pool->device);
@@ -515,6 +647,17 @@ lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_ou
     if ((r = st.out(nullptr, (size_t)(n_out + n_in) * sizeof(int4), &tdev, true)) != LV_OK) return r;
     if ((r = st.out(nullptr, sizeof(long long), &ndev, true)) != LV_OK) return r;
     if (++pool->epoch <= 0) pool->epoch = 1;
+    if (mode == LV_MODE_STAGED) {
+      LV_TRY(lv::launch_exchange_plan(pool->d, static_cast<const lv_victim*>(vin), n_out, sid,
+                                      static_cast<const int32_t*>(bin), n_in, static_cast<int32_t*>(sdev),
+                                      static_cast<int32_t*>(pdev), static_cast<int4*>(tdev),
+                                      static_cast<long long*>(ndev), pool->epoch, pool->d.page_tag, s));
+      long long nt = 0;
+      LV_TRY(cudaMemcpyAsync(&nt, ndev, sizeof(nt), cudaMemcpyDeviceToHost, s));
+      LV_TRY(cudaStreamSynchronize(s));
+      if ((r = staged_move(pool, static_cast<int4*>(tdev), nt, s)) != LV_OK) return r;
+      return st.finish();
+    }
     LV_TRY(lv::launch_exchange(pool->d, static_cast<const lv_victim*>(vin), n_out, sid,
                                static_cast<const int32_t*>(bin), n_in, static_cast<int32_t*>(sdev),
                                static_cast<int32_t*>(pdev), static_cast<int4*>(tdev),

@@ -120,6 +120,20 @@ cudaError_t launch_counts(const DevPool& p, int32_t* hbm, int32_t* host, cudaStr
 cudaError_t launch_blocks(const DevPool& p, int32_t sid, int32_t where, int32_t* out,
                           long long* count, cudaStream_t s);
 cudaError_t launch_check_budget(const DevPool& p, cudaStream_t s);
+// staged path
+cudaError_t launch_tasks_out(const DevPool& p, const lv_victim* v, const int32_t* slots, int64_t n,
+                             int4* tasks, lv_remap_entry* commit, cudaStream_t s);
+cudaError_t launch_tasks_in(const DevPool& p, int32_t sid, const int32_t* blks, const int32_t* pages,
+                            int64_t n, int4* tasks, lv_remap_entry* commit, cudaStream_t s);
+cudaError_t launch_exchange_plan(const DevPool& p, const lv_victim* v, int64_t n_out, int32_t sid,
+                                 const int32_t* blks, int64_t n_in, int32_t* slots, int32_t* pages,
+                                 int4* tasks, long long* n_tasks, int32_t epoch,
+                                 unsigned long long* page_tag, cudaStream_t s);
+// pack (staging[t] <- out pages) or unpack (in pages <- staging[t]) for tasks [t_begin, t_end)
+cudaError_t launch_stage(const DevPool& p, bool pack, const int4* tasks, int64_t t_begin,
+                         int64_t t_end, uint8_t* staging, cudaStream_t s, int ctas,
+                         const EventPair* ev);
+cudaError_t configure_stage_kernels(const DevPool& p);
 cudaError_t configure_kernels();   // once per device, before the first launch
 
 }  // namespace lv

@@ -654,6 +654,215 @@ k_exchange_copy(DevPool p, const int4* __restrict__ tasks, const long long* __re
   }
 }
 
+// ---------------------------------------------------------------- staged
+// The staged path moves pages through a contiguous HBM staging run so that the
+// copy engines can carry them over the host link: tasks (the exchange's
+// {out page, out slot, in slot, in page}) are built and validated first, then
+// k_pack_tasks gathers every out page's 2L sub-pages into staging[t] and
+// k_unpack_tasks scatters staging[t] into every in page.  Both kernels move
+// whole sub-pages with TMA bulk copies (global -> shared -> global), issued by
+// one thread per CTA through a ring of shared-memory stages.
+
+// Validated out-tasks of a swap-out: {page, slot, -1, -1} (all -1 when invalid).
+__global__ void k_tasks_out(DevPool p, const lv_victim* __restrict__ v, const int32_t* __restrict__ slots,
+                            long long n, int4* __restrict__ tasks, lv_remap_entry* __restrict__ commit) {
+  const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const lv_victim x = v[i];
+  const int32_t slot = slots[i];
+  int4 t = make_int4(-1, -1, -1, -1);
+  if (slot >= 0) {
+    bool ok = x.sid >= 0 && x.sid < p.S && x.blk >= 0 && x.page >= 0 && x.page < p.hbm_pages &&
+              slot < p.host_pages;
+    ok = ok && x.blk < nblocks_of(p, x.sid);
+    ok = ok && p.table[(size_t)x.sid * p.maxB + x.blk] == x.page &&
+         p.own_hbm[x.page] == owner_key(x.sid, x.blk);
+    if (!ok) set_error(p.ctl, LV_ERR_STATE, i);
+    else {
+      t = make_int4(x.page, slot, -1, -1);
+      atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PAGES_OUT]), 1ull);
+    }
+    if (commit) commit[i] = lv_remap_entry{x.sid, x.blk, ok ? -(slot + 2) : -1};
+  } else if (commit) {
+    commit[i] = lv_remap_entry{x.sid, x.blk, -1};
+  }
+  tasks[i] = t;
+}
+
+// Validated in-tasks of a swap-in: {-1, -1, slot, page} (all -1 when invalid).
+__global__ void k_tasks_in(DevPool p, int32_t sid, const int32_t* __restrict__ blks,
+                           const int32_t* __restrict__ pages, long long n, int4* __restrict__ tasks,
+                           lv_remap_entry* __restrict__ commit) {
+  const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const int32_t blk = blks[i], page = pages[i];
+  int4 t = make_int4(-1, -1, -1, -1);
+  const bool sid_ok = sid >= 0 && sid < p.S;
+  if (page >= 0) {
+    bool ok = sid_ok && blk >= 0 && blk < nblocks_of(p, sid) && page < p.hbm_pages;
+    long long slot = -1;
+    if (ok) {
+      const int32_t e = p.table[(size_t)sid * p.maxB + blk];
+      slot = -(long long)e - 2;
+      ok = e <= -2 && slot < p.host_pages && p.own_host[slot] == owner_key(sid, blk);
+    }
+    if (!ok) set_error(p.ctl, sid_ok ? LV_ERR_STATE : LV_ERR_BOUNDS, i);
+    else {
+      t = make_int4(-1, -1, (int32_t)slot, page);
+      atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PAGES_IN]), 1ull);
+    }
+    if (commit) commit[i] = lv_remap_entry{sid, blk, ok ? page : -1};
+  } else if (commit) {
+    commit[i] = lv_remap_entry{sid, blk, -1};
+  }
+  tasks[i] = t;
+}
+
+__device__ __forceinline__ uint32_t smem_addr(const void* ptr) {
+  return (uint32_t)__cvta_generic_to_shared(ptr);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(done)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+
+// 1-D bulk copy global -> this CTA's shared memory, completing on `bar`.
+__device__ __forceinline__ void bulk_load(void* dst_smem, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_addr(dst_smem)),
+      "l"(src), "r"(bytes), "r"(smem_addr(bar))
+      : "memory");
+}
+
+// 1-D bulk copy shared -> global, tracked by the bulk async-group.
+__device__ __forceinline__ void bulk_store(void* dst, const void* src_smem, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst),
+               "r"(smem_addr(src_smem)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_all() {
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+// Bounded wait on a stage barrier: false after `limit` polls (the data never came).
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, long long limit) {
+  for (long long it = 0; it < limit; ++it)
+    if (mbar_try_wait(bar, parity)) return true;
+  return false;
+}
+
+constexpr int kStageThreads = 32;     // one warp per CTA; lane 0 issues the bulk copies
+constexpr int kMaxStages = 8;
+constexpr long long kWaitPolls = 1ll << 22;   // each poll may also suspend briefly in hardware
+
+// Moves units u = (task t, sub-page j) of P bytes through `stages` shared-memory
+// buffers: unit i's load is issued `stages` units ahead of its store.
+// pack:   staging[t][j] <- hbm_kv[j][task.x]   for tasks with task.x >= 0
+// unpack: hbm_kv[j][task.w] <- staging[t][j]   for tasks with task.z >= 0
+template <bool kPack>
+__global__ void __launch_bounds__(kStageThreads)
+k_stage_tasks(DevPool p, const int4* __restrict__ tasks, long long t_begin, long long t_end,
+              uint8_t* __restrict__ staging, int stages) {
+  extern __shared__ __align__(128) unsigned char stage_mem[];
+  __shared__ __align__(8) uint64_t bars[kMaxStages];
+  if (threadIdx.x != 0) return;
+  const uint32_t P = (uint32_t)p.P;
+  for (int s = 0; s < stages; ++s) mbar_init(&bars[s], 1);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  const long long units = (t_end - t_begin) * p.J;
+  // the units of this CTA, in order: u = blockIdx.x + k * gridDim.x
+  auto unit_ptrs = [&](long long k, const uint8_t** src, uint8_t** dst) -> bool {
+    const long long u = blockIdx.x + k * (long long)gridDim.x;
+    const long long t = t_begin + u / p.J;
+    const int j = (int)(u % p.J);
+    const int4 tk = tasks[t];
+    uint8_t* st = staging + ((size_t)t * p.J + j) * P;
+    if (kPack) {
+      if (tk.x < 0) return false;
+      *src = p.kv[j] + (size_t)tk.x * P;
+      *dst = st;
+    } else {
+      if (tk.z < 0) return false;
+      *src = st;
+      *dst = p.kv[j] + (size_t)tk.w * P;
+    }
+    return true;
+  };
+  const long long mine = units > blockIdx.x ? (units - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
+  uint8_t* dsts[kMaxStages];
+  bool live[kMaxStages];
+  uint32_t phase[kMaxStages];
+  for (int s = 0; s < stages; ++s) { live[s] = false; phase[s] = 0; }
+  bool failed = false;
+  // prologue: fill the ring
+  long long issued = 0;
+  for (; issued < mine && issued < stages; ++issued) {
+    const int s = (int)(issued % stages);
+    const uint8_t* src;
+    if (unit_ptrs(issued, &src, &dsts[s])) {
+      mbar_expect_tx(&bars[s], P);
+      bulk_load(stage_mem + (size_t)s * P, src, P, &bars[s]);
+      live[s] = true;
+    } else {
+      live[s] = false;
+    }
+  }
+  for (long long k = 0; k < mine; ++k) {
+    const int s = (int)(k % stages);
+    if (live[s]) {
+      if (!mbar_wait_bounded(&bars[s], phase[s], kWaitPolls)) {
+        failed = true;
+        break;
+      }
+      phase[s] ^= 1u;
+      bulk_store(dsts[s], stage_mem + (size_t)s * P, P);
+      bulk_commit();
+      bulk_wait_read_all();          // stage s may be refilled once the store has read it
+    }
+    if (issued < mine) {
+      const uint8_t* src;
+      if (unit_ptrs(issued, &src, &dsts[s])) {
+        mbar_expect_tx(&bars[s], P);
+        bulk_load(stage_mem + (size_t)s * P, src, P, &bars[s]);
+        live[s] = true;
+      } else {
+        live[s] = false;
+      }
+      ++issued;
+    } else {
+      live[s] = false;
+    }
+  }
+  if (failed) {
+    set_error(p.ctl, LV_ERR_TIMEOUT, blockIdx.x);
+    // let every load still in flight land before the shared memory is released
+    for (int s = 0; s < stages; ++s)
+      if (live[s]) mbar_wait_bounded(&bars[s], phase[s], kWaitPolls);
+  }
+  bulk_wait_all();
+}
+
 // ---------------------------------------------------------------- commit
 __device__ __forceinline__ bool bit_is_set(const uint32_t* bits, long long i) {
   return (bits[i >> 5] >> (i & 31)) & 1u;
@@ -1037,6 +1246,55 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
     if (e != cudaSuccess) return e;
   }
   k_resident_finish<<<1, 32, 0, s>>>(p, sid, now_us, preload, R, result);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_tasks_out(const DevPool& p, const lv_victim* v, const int32_t* slots, int64_t n,
+                             int4* tasks, lv_remap_entry* commit, cudaStream_t s) {
+  k_tasks_out<<<blocks_for(n, 256, 1ll << 30), 256, 0, s>>>(p, v, slots, n, tasks, commit);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_tasks_in(const DevPool& p, int32_t sid, const int32_t* blks, const int32_t* pages,
+                            int64_t n, int4* tasks, lv_remap_entry* commit, cudaStream_t s) {
+  k_tasks_in<<<blocks_for(n, 256, 1ll << 30), 256, 0, s>>>(p, sid, blks, pages, n, tasks, commit);
+  return cudaGetLastError();
+}
+
+int stage_count(const DevPool& p) {
+  int st = (int)((160 * 1024) / p.P);
+  return st < 2 ? 2 : (st > kMaxStages ? kMaxStages : st);
+}
+
+cudaError_t configure_stage_kernels(const DevPool& p) {
+  const int smem = stage_count(p) * (int)p.P;
+  cudaError_t e = cudaFuncSetAttribute(k_stage_tasks<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(k_stage_tasks<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+}
+
+cudaError_t launch_stage(const DevPool& p, bool pack, const int4* tasks, int64_t t_begin, int64_t t_end,
+                         uint8_t* staging, cudaStream_t s, int ctas, const EventPair* ev) {
+  if (t_end <= t_begin) return cudaSuccess;
+  const int stages = stage_count(p);
+  const size_t smem = (size_t)stages * p.P;
+  const long long units = (t_end - t_begin) * (long long)p.J;
+  const unsigned grid = blocks_for(units, 1, ctas);
+  if (ev) cudaEventRecord(ev->start, s);
+  if (pack)
+    k_stage_tasks<true><<<grid, kStageThreads, smem, s>>>(p, tasks, t_begin, t_end, staging, stages);
+  else
+    k_stage_tasks<false><<<grid, kStageThreads, smem, s>>>(p, tasks, t_begin, t_end, staging, stages);
+  if (ev) cudaEventRecord(ev->end, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_exchange_plan(const DevPool& p, const lv_victim* v, int64_t n_out, int32_t sid,
+                                 const int32_t* blks, int64_t n_in, int32_t* slots, int32_t* pages,
+                                 int4* tasks, long long* n_tasks, int32_t epoch,
+                                 unsigned long long* page_tag, cudaStream_t s) {
+  k_exchange_plan<<<1, kPlanThreads, 0, s>>>(p, v, n_out, sid, blks, n_in, slots, pages, tasks,
+                                             n_tasks, epoch, page_tag, nullptr);
   return cudaGetLastError();
 }
 

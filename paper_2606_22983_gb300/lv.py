@@ -68,8 +68,9 @@ class lv_kernel_timing(ctypes.Structure):
                 ("min_ms", ctypes.c_double), ("max_ms", ctypes.c_double)]
 
 
-LV_TIMING_SWAP_OUT, LV_TIMING_SWAP_IN, LV_TIMING_EXCHANGE, LV_TIMING_KINDS = 0, 1, 2, 3
-TIMING_NAMES = ("swap_out", "swap_in", "exchange")
+LV_TIMING_SWAP_OUT, LV_TIMING_SWAP_IN, LV_TIMING_EXCHANGE, LV_TIMING_PACK, LV_TIMING_UNPACK = 0, 1, 2, 3, 4
+LV_TIMING_KINDS = 5
+TIMING_NAMES = ("swap_out", "swap_in", "exchange", "pack", "unpack")
 
 
 class lv_rank_params(ctypes.Structure):

@@ -10,15 +10,17 @@ from ._lockstep import run_lockstep
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("seed,driver", [(0, "device"), (1, "device"), (0, "exchange"),
-                                         (1, "sequential")])
-def test_tiny_workload_full_images(seed, driver):
+@pytest.mark.parametrize("seed,driver,mode", [(0, "device", 0), (1, "device", 0), (0, "exchange", 0),
+                                              (1, "sequential", 0), (0, "exchange", 2),
+                                              (1, "sequential", 2)])
+def test_tiny_workload_full_images(seed, driver, mode):
     """1000 scripted events of the tiny pool: every ranking (full order after
     each event), eviction, preload, reload and growth, with full HBM and host
     byte images compared every 50 events -- through lv_make_resident, through
-    select + lv_swap_exchange, and through the four sequential calls."""
+    select + lv_swap_exchange, and through the four sequential calls, with
+    zero-copy kernels (mode 0) and with the staged copy-engine path (mode 2)."""
     wl = make_workload("tiny", seed)
-    om, gm = run_lockstep(wl, with_bytes=True, check_every=50, driver=driver)
+    om, gm = run_lockstep(wl, with_bytes=True, check_every=50, driver=driver, mode=mode)
     assert om.counters == gm.counters
     assert gm.counters["pages_out"] > 500 and gm.counters["preloads"] > 10
 
@@ -40,8 +42,8 @@ def _expected_block(seed, table, shape, sid, blk, ctx):
     return subpage_values_np(table, off, rows, shape).view(np.uint8).reshape(J, -1)
 
 
-@pytest.mark.parametrize("driver", ["device", "exchange"])
-def test_thinker_full_size_sampled_bytes(driver):
+@pytest.mark.parametrize("driver,mode", [("device", 0), ("exchange", 0), ("exchange", 2)])
+def test_thinker_full_size_sampled_bytes(driver, mode):
     """The thinker pool at full size (40 GB HBM budget, 1.5 MiB pages), in the
     launch configuration the benchmark times: every turn's victims, host slots
     and pages match the oracle; afterwards the tables and owners match, and
@@ -60,7 +62,7 @@ def test_thinker_full_size_sampled_bytes(driver):
     try:
         writer = ContentWriter(pool, wl)
         writer.write_initial(wl)
-        gm = KVManager(pool, perms=wl.perms, rank_on="turns", driver=driver)
+        gm = KVManager(pool, perms=wl.perms, rank_on="turns", driver=driver, mode=mode)
         last = None
         for i in range(wl.n_events):
             ro, rg = om.step(i), gm.step(wl.event(i), i)
