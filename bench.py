@@ -327,18 +327,103 @@ def ours(args, torch):
             "link_frac": round(value / peaks["bidir"], 3) if "bidir" in peaks else None,
             "roofline": roof,
             "kernels": {n: {k: round(v, 3) for k, v in d.items()} for n, d in kern.items()},
-            "hbm_kernels": hbm_kern or None,
+            "in_turn_hbm_kernels": hbm_kern or None,
             "e2e": {"value": round(e2e_value, 3), "unit": UNIT,
                     "h2d_bytes_per_step": int(h2d / K), "d2h_bytes_per_step": int(d2h / K)},
             "gpu_launches": int(launches),
             "clocks": clk,
         }
+    if line is not None and args.micro:
+        micro = kernel_micro(torch, pool, args.seed)
+        line["ranker"] = micro.pop("ranker")
+        line["hbm_kernels"] = micro
     pool.close()
     if line is not None and args.cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(args.cpu_seconds, args.seed)
     if dist:
         dist.destroy_process_group()
     return line
+
+
+REMAP_BYTES_PER_ENTRY = 72   # entry 12, table 4+4, epoch 4+4, bitmap 4, new owner 8+8, old owner 8+8, old bitmap 4+4
+
+
+def kernel_micro(torch, pool, seed=0):
+    """Standalone timings of the HBM-bound kernels and the ranker (rank 0, after the turns).
+
+    pack/unpack: 4096 scattered pages of the bench pool to / from one contiguous 6.4 GB
+    run (each payload byte is read once and written once in HBM); ranker and remap:
+    a metadata-sized pool (16-token pages of 256 B) with 2^20 resident pages in 1024
+    sessions -- one top-256 decision, and one commit of all 2^20 pages to the host tier."""
+    from paper_2606_22983_gb300 import lv
+    from paper_2606_22983_gb300.pool import KVPool
+    out = {}
+    g = torch.Generator(device=pool.device).manual_seed(seed)
+    n = min(4096, pool.hbm_pages)
+    pages = torch.randperm(pool.hbm_pages, generator=g, device=pool.device)[:n].to(torch.int32)
+    payload = n * pool.J * pool.P
+    run = torch.empty(payload, dtype=torch.uint8, device=pool.device)
+    for _ in range(2):
+        lv.lv_pack_pages(pool.handle, pages, n, run, pool.stream)
+        lv.lv_unpack_pages(pool.handle, run, pages, n, pool.stream)   # writes back the same bytes
+    pool.sync()
+    lv.lv_timing_read(pool.handle, reset=True)
+    lv.lv_timing_enable(pool.handle, True)
+    for _ in range(5):
+        lv.lv_pack_pages(pool.handle, pages, n, run, pool.stream)
+        lv.lv_unpack_pages(pool.handle, run, pages, n, pool.stream)
+    t = lv.lv_timing_read(pool.handle, reset=True)
+    lv.lv_timing_enable(pool.handle, False)
+    assert pool.sync(raise_on_error=False) == 0
+    for name in ("pack", "unpack"):
+        ms = t[name]["total_ms"] / t[name]["launches"]
+        gbs = 2 * payload / (ms / 1e3) / 1e9
+        out[name] = {"pages": n, "bytes_per_launch": 2 * payload, "avg_ms": round(ms, 4),
+                     "achieved_gbs": round(gbs, 1), "peak_gbs": HBM_PEAK, "frac": round(gbs / HBM_PEAK, 3)}
+    del run
+    # a metadata-sized pool: 1024 sessions x 1024 resident blocks = 2^20 pages
+    S = B = 1024
+    N = S * B
+    mp = KVPool(layers=1, kv_heads=1, head_dim=8, max_sessions=S, max_blocks=B, hbm_pages=N,
+                hbm_budget_pages=N, host_pages=N, device=pool.device, stream=pool.stream)
+    try:
+        rng = np.random.default_rng(seed)
+        mp.import_placement(rng.permutation(N).astype(np.int32).reshape(S, B),
+                            np.full(S, B * 16, np.int32))
+        st = np.zeros(S, dtype=lv.SESSION_DTYPE)
+        st["gen_us"] = rng.integers(0, 10_000_000, S)
+        mp.set_sessions(st)
+        mp.sync()
+        o = torch.empty((256, 3), dtype=torch.int32, device=pool.device)
+        c = torch.zeros(1, dtype=torch.int64, device=pool.device)
+        for _ in range(5):
+            lv.lv_select_victims(mp.handle, 0, 256, 0, o, 256, c, mp.stream)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(50):
+            lv.lv_select_victims(mp.handle, 0, 256, 0, o, 256, c, mp.stream)
+        b.record()
+        torch.cuda.synchronize()
+        out["ranker"] = {"resident_pages": N, "sessions": S, "k": 256,
+                         "us_per_decision": round(a.elapsed_time(b) * 1e3 / 50, 2)}
+        victims, nv = mp.select(0, lv.LV_ALL, 0)
+        assert nv == N
+        slots, commit = mp.swap_out(victims, nv)
+        mp.sync()
+        a.record()
+        mp.remap(commit, nv)
+        b.record()
+        torch.cuda.synchronize()
+        assert mp.sync(raise_on_error=False) == 0 and mp.stats()["host_allocated"] == N
+        ms = a.elapsed_time(b)
+        gbs = REMAP_BYTES_PER_ENTRY * N / (ms / 1e3) / 1e9
+        out["remap_1m"] = {"entries": N, "bytes_per_entry": REMAP_BYTES_PER_ENTRY, "ms": round(ms, 4),
+                           "entries_per_s": round(N / (ms / 1e3)), "achieved_gbs": round(gbs, 1),
+                           "peak_gbs": HBM_PEAK, "frac": round(gbs / HBM_PEAK, 3)}
+    finally:
+        mp.close()
+    return out
 
 
 def _profiled_traffic(kernel, bytes_per_launch):
@@ -445,6 +530,8 @@ def main():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
+    ap.add_argument("--no-micro", dest="micro", action="store_false",
+                    help="skip the standalone pack/unpack/remap/ranker timings")
     ap.add_argument("--sessions", type=int, default=0,
                     help="smaller case for profiling: number of sessions")
     ap.add_argument("--budget-pages", type=int, default=0,

@@ -69,6 +69,12 @@ enum { LV_SUFFIX_FIRST = 0, LV_ASCENDING = 1 };        /* lv_pool_desc.within_or
 enum { LV_PLAY_PLAYBACK = 0, LV_PLAY_COUNTERS = 1 };   /* lv_pool_desc.t_play_mode */
 enum { LV_MODE_AUTO = 0, LV_MODE_ZERO_COPY = 1, LV_MODE_STAGED = 2 };   /* swap modes */
 enum { LV_SELECT_FALLBACK = 1 };                       /* lv_select_victims flags */
+/* Victim order.  LV_POLICY_NEXT_USE: the paper's order (Section 5.1).
+   LV_POLICY_LRU: the substrate's least-recently-used order that the paper
+   compares against (Sections 2.3 and 5): candidates are all sessions that are
+   not running, ranked by last use ascending (then session id ascending, suffix
+   blocks first); speech, barge-in and preload protection are ignored. */
+enum { LV_POLICY_NEXT_USE = 0, LV_POLICY_LRU = 1 };
 
 /* session flag bits (lv_session_state.flags) */
 enum {
@@ -109,10 +115,10 @@ typedef struct lv_pool_desc {
   int64_t protect_us;          /* preload protection window (>= 0) */
   int64_t unit_us;             /* progress-counter unit, 1..2^31 */
   int32_t t_play_mode;         /* LV_PLAY_PLAYBACK or LV_PLAY_COUNTERS */
-  int32_t reserved;            /* must be 0 */
+  int32_t policy;              /* LV_POLICY_NEXT_USE (Section 5.1) or LV_POLICY_LRU */
 } lv_pool_desc;
 
-/* Per-session interaction state (64 bytes).  ctx_tokens is maintained by
+/* Per-session interaction state (72 bytes).  ctx_tokens is maintained by
    lv_pool_import and lv_session_append and ignored by lv_session_set. */
 typedef struct lv_session_state {
   int32_t ctx_tokens;
@@ -125,6 +131,7 @@ typedef struct lv_session_state {
   int32_t pad;
   int64_t reply_tokens;        /* current reply length in progress units */
   int64_t protect_until_us;    /* preload protection ends at this time */
+  int64_t last_use_us;         /* time of the last turn begin or end (LRU order) */
 } lv_session_state;
 
 typedef struct lv_event {      /* 32 bytes */
@@ -180,6 +187,10 @@ lv_status lv_pool_destroy(lv_pool* pool, lv_stream stream);
 /* Host-visible address of the host pool ([host_pages][2L][P]). */
 void* lv_pool_host_ptr(lv_pool* pool);
 
+/* Device-visible address of the same host pool (kernels may read and write it
+   over the host link; on GB300 it equals the host address). */
+void* lv_pool_host_device_ptr(lv_pool* pool);
+
 /* Loads a placement: placement is int32 [max_sessions][max_blocks] of encoded
    entries, ctx_tokens is int32 [max_sessions].  Block b of session s must be
    placed (entry != -1) exactly when b < ceil(ctx_tokens[s] / T).  Rebuilds the
@@ -202,6 +213,7 @@ lv_status lv_session_get(lv_pool* pool, lv_session_state* out, int32_t first, in
    and Sections 5.1-5.2: applies n events in order to the session table.
    TURN_BEGIN sets RUNNING, clears IMMEDIATE and the preload protection.
    TURN_END(a, b) clears RUNNING, starts a reply of a us and b units (LV_RESP_OPEN).
+   Both set last_use_us = t.
    PLAYBACK(a) advances play_us by a, at most to gen_us; reaching it ends the
    reply and records t_done_us.  SPEECH_START sets IMMEDIATE.  BARGE_IN sets
    gen_us = play_us (unplayed audio discarded), ends the reply without a
@@ -335,6 +347,18 @@ lv_status lv_remap(lv_pool* pool, const lv_remap_entry* entries, int64_t n, lv_s
    transfer, Section 5.2).  locs are encoded locations.  Device-detected:
    LV_ERR_STATE when a location is owned or not reserved. */
 lv_status lv_cancel(lv_pool* pool, const int32_t* locs, int64_t n, lv_stream stream);
+
+/* The staged path's building blocks (Section 6, offload connector), usable on
+   their own: lv_pack_pages gathers the 2L sub-pages of each listed HBM page into
+   one contiguous run, dst[i][j] = hbm_kv[j][pages[i]] (dst [n][2L][P]);
+   lv_unpack_pages scatters such a run back, hbm_kv[j][pages[i]] = src[i][j].
+   The run must be device memory or mapped page-locked host memory, 16-byte
+   aligned.  They move raw bytes and touch no table: the caller decides which
+   pages may be read or written.  Device-detected: LV_ERR_BOUNDS for a page id
+   outside the pool (that page is skipped). */
+lv_status lv_pack_pages(lv_pool* pool, const int32_t* pages, int64_t n, void* dst, lv_stream stream);
+lv_status lv_unpack_pages(lv_pool* pool, const void* src, const int32_t* pages, int64_t n,
+                          lv_stream stream);
 
 /* Block-level allocation kept (Section 5.1): grows session sid's context by
    n_tokens; each new block takes the lowest free HBM page, in block order, and

@@ -9,6 +9,8 @@ For each script event (see ``workloads.scripts`` for the kinds):
   TURN          the request runs: the session's KV is made fully resident
                 (a synchronous, foreground load of any host blocks), its
                 context grows, then the reply is recorded.
+  TURN_SCATTER  a turn whose host blocks are reloaded in a given scattered order.
+  EVICT         k pages are freed now, in the victim order of Section 5.1.
 
 Making a session resident with ``need`` missing pages (host blocks plus new
 blocks) first evicts ``k = need - free`` pages when the HBM budget is short,
@@ -30,11 +32,12 @@ from __future__ import annotations
 import numpy as np
 
 from . import sessions as se
-from .policy import order_global, select_victims
+from .policy import LRU, order_global, order_lru, select_victims
 from .pool import OraclePool, OracleError, _enc_host
 
 # script event kinds (the published script format)
 EV_TURN, EV_TURN_ANY, EV_PLAYBACK, EV_SPEECH_START, EV_BARGE_IN, EV_SPEECH_STOP = 1, 2, 3, 4, 5, 6
+EV_TURN_SCATTER, EV_EVICT = 7, 8
 
 
 class OracleManager:
@@ -105,19 +108,28 @@ class OracleManager:
     # ------------------------------------------------------------- ranking
     def full_order(self, now_us):
         sp = self.spec
+        if sp.policy == LRU:
+            return order_lru(self.pool.tables, self.pool.nblocks, self.sessions, sp.within_order)
         return order_global(self.pool.tables, self.pool.nblocks, self.sessions, now_us,
                             sp.t_play_mode, sp.reply_prior_us, sp.unit_us, sp.within_order)
 
     def select(self, now_us, k, fallback=False):
         sp = self.spec
+        if sp.policy == LRU:
+            s_, b_, p_ = order_lru(self.pool.tables, self.pool.nblocks, self.sessions, sp.within_order)
+            k = min(int(k), s_.size)
+            return s_[:k], b_[:k], p_[:k]
         return select_victims(self.pool.tables, self.pool.nblocks, self.sessions, now_us, k,
                               sp.t_play_mode, sp.reply_prior_us, sp.unit_us, sp.within_order,
                               fallback)
 
     # ------------------------------------------------------------ movement
-    def make_resident(self, sid, now_us, append_tokens, foreground, rec):
+    def make_resident(self, sid, now_us, append_tokens, foreground, rec, order_key=None):
         pool = self.pool
         host_blks = pool.host_blocks(sid)
+        if order_key is not None:
+            from workloads.scripts import scatter_order
+            host_blks = scatter_order(order_key, host_blks)
         new_ctx = int(pool.ctx[sid]) + int(append_tokens)
         new_blocks = -(-new_ctx // pool.T) - int(pool.nblocks[sid])
         need = int(host_blks.size) + new_blocks
@@ -155,6 +167,8 @@ class OracleManager:
         return True
 
     def preload(self, sid, now_us, rec):
+        if self.spec.policy == LRU:
+            return              # the baseline loads at turn start only
         host_blks = self.pool.host_blocks(sid)
         if host_blks.size == 0:
             return
@@ -170,6 +184,20 @@ class OracleManager:
         else:
             self.counters["preload_skipped"] += 1
             rec["preload"] = "skipped"
+
+    def evict(self, now_us, k, rec):
+        """Free k pages now (memory pressure from elsewhere): the first k of the victim
+        order, or all candidates when there are fewer."""
+        pool = self.pool
+        vs, vb, vp = self.select(now_us, k)
+        rec["k"] = int(k)
+        rec["victims"] = np.stack([vs, vb, vp], axis=1) if vs.size else np.zeros((0, 3), np.int64)
+        if vs.size:
+            slots = pool.swap_out(vs, vb, vp)
+            rec["slots"] = slots
+            pool.remap(vs, vb, _enc_host(slots))
+            self.counters["victims"] += int(vs.size)
+            self.counters["pages_out"] += int(vs.size)
 
     def turn_target(self, perm_row):
         perm = self.wl.perms[perm_row]
@@ -194,19 +222,26 @@ class OracleManager:
             self.preload(sid, t, rec)
         elif kind == EV_SPEECH_STOP:
             se.apply_event(sts[sid], se.SE_SPEECH_STOP, t)
-        elif kind in (EV_TURN, EV_TURN_ANY):
-            if kind == EV_TURN_ANY:
+        elif kind in (EV_TURN, EV_TURN_ANY, EV_TURN_SCATTER):
+            order_key = None
+            if kind == EV_TURN_SCATTER:
+                sid = self.turn_target(d)
+                order_key, a = a, 0
+            elif kind == EV_TURN_ANY:
                 sid = self.turn_target(d)
             se.apply_event(sts[sid], se.SE_TURN_BEGIN, t)
             if self.pool.host_blocks(sid).size:
                 self.counters["sync_loads"] += 1
-            self.make_resident(sid, t, a, foreground=True, rec=rec)
+            self.make_resident(sid, t, a, foreground=True, rec=rec, order_key=order_key)
             se.apply_event(sts[sid], se.SE_TURN_END, t, b, c)
             self.counters["turns"] += 1
+        elif kind == EV_EVICT:
+            self.evict(t, a, rec)
         else:
             raise ValueError(f"unknown script event kind {kind}")
         rec["sid"] = sid
-        if self.rank_on == "all" or (self.rank_on == "turns" and kind in (EV_TURN, EV_TURN_ANY)):
+        if self.rank_on == "all" or (self.rank_on == "turns" and kind in (EV_TURN, EV_TURN_ANY,
+                                                                           EV_TURN_SCATTER)):
             rec["order"] = np.stack(self.full_order(t), axis=1)
         return rec
 
@@ -217,5 +252,5 @@ class OracleManager:
     # ------------------------------------------------------------- snapshot
     def session_arrays(self):
         keys = ("ctx_tokens", "flags", "gen_us", "play_us", "t_done_us", "reply_ema_us",
-                "reply_n", "reply_tokens", "protect_until_us")
+                "reply_n", "reply_tokens", "protect_until_us", "last_use_us")
         return {k: np.array([getattr(s, k) for s in self.sessions], dtype=np.int64) for k in keys}

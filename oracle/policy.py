@@ -34,6 +34,8 @@ from .sessions import (SessionState, RUNNING, IMMEDIATE, RESP_OPEN, MODE_PLAYBAC
 KEY_MAX = 2**32 - 1
 SUFFIX_FIRST = 0
 ASCENDING = 1
+NEXT_USE = 0        # the paper's order (Section 5.1)
+LRU = 1             # the substrate's least-recently-used baseline (Sections 2.3, 5)
 
 
 def t_next(st: SessionState, mode: int, reply_prior_us: int, unit_us: int) -> int:
@@ -70,6 +72,27 @@ def tier(st: SessionState, now_us: int, fallback: bool):
     if fallback and not (st.flags & RUNNING):
         return 1
     return None
+
+
+def order_lru(tables, nblocks, sessions, within=SUFFIX_FIRST):
+    """The LRU baseline: every HBM-resident block of a session that is not running,
+    least recently used session first (last turn time ascending, then session id
+    ascending), suffix blocks first within a session.  Immediate reuse and preload
+    protection do not exist for it."""
+    cands = [(s, st.last_use_us) for s, st in enumerate(sessions) if not (st.flags & RUNNING)]
+    cands.sort(key=lambda c: (min(max(c[1], 0), KEY_MAX), c[0]))
+    out_s, out_b, out_p = [], [], []
+    for s, _ in cands:
+        n = int(nblocks[s])
+        rng = range(n - 1, -1, -1) if within == SUFFIX_FIRST else range(n)
+        for b in rng:
+            e = int(tables[s][b])
+            if e >= 0:
+                out_s.append(s)
+                out_b.append(b)
+                out_p.append(e)
+    return (np.array(out_s, dtype=np.int64), np.array(out_b, dtype=np.int64),
+            np.array(out_p, dtype=np.int64))
 
 
 def _resident_blocks(table_row: np.ndarray, nblocks: int) -> np.ndarray:

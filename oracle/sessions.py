@@ -58,6 +58,7 @@ class SessionState:
     reply_n: int = 0           # samples in the moving average
     reply_tokens: int = 0      # length of the current reply in progress units
     protect_until_us: int = 0  # preload protection ends at this time
+    last_use_us: int = 0       # last turn begin or end (the LRU baseline's recency)
 
     def copy(self) -> "SessionState":
         return SessionState(**self.__dict__)
@@ -71,8 +72,10 @@ def apply_event(st: SessionState, kind: int, t_us: int, a: int = 0, b: int = 0,
         # immediate-reuse ends, warmed KV has been reused (Section 5.2).
         st.flags = (st.flags | RUNNING) & ~IMMEDIATE
         st.protect_until_us = 0
+        st.last_use_us = t_us
     elif kind == SE_TURN_END:
         # The LLM stage produced a reply of a = audio us, b = units; playback restarts.
+        st.last_use_us = t_us
         st.flags &= ~(RUNNING | DONE_VALID)
         st.gen_us, st.play_us, st.reply_tokens = int(a), 0, int(b)
         if st.gen_us > 0:

@@ -22,6 +22,7 @@ struct lv_pool {
   size_t tasks_host_cap = 0;
   std::vector<cudaEvent_t> sync_events;
   int stage_ctas = 0;
+  bool stage_tma = true;           // pack/unpack with TMA bulk copies (else 16-byte LSU copies)
   // copy-kernel timing (lv_timing_enable): event pairs recorded per kind, reused
   bool timing = false;
   std::vector<lv::EventPair> ev_free;
@@ -232,7 +233,7 @@ lv_status staged_move(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStrea
   for (int64_t c = 0; c < nchunks && any_out; ++c) {
     const int64_t a = c * chunk, b = std::min(n, a + chunk);
     LV_TRY(lv::launch_stage(d, true, tasks_dev, a, b, stg_out, s, pool->stage_ctas,
-                            timing_pair(pool, LV_TIMING_PACK)));
+                            timing_pair(pool, LV_TIMING_PACK), pool->stage_tma));
     LV_TRY(cudaEventRecord(ev_pack[c], s));
     LV_TRY(cudaStreamWaitEvent(pool->s_d2h, ev_pack[c], 0));
     for (int64_t i = a; i < b;) {
@@ -249,7 +250,7 @@ lv_status staged_move(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStrea
     const int64_t a = c * chunk, b = std::min(n, a + chunk);
     LV_TRY(cudaStreamWaitEvent(s, ev_h2d[c], 0));
     LV_TRY(lv::launch_stage(d, false, tasks_dev, a, b, stg_in, s, pool->stage_ctas,
-                            timing_pair(pool, LV_TIMING_UNPACK)));
+                            timing_pair(pool, LV_TIMING_UNPACK), pool->stage_tma));
   }
   LV_TRY(cudaEventRecord(ev_d2h_done, pool->s_d2h));
   LV_TRY(cudaEventRecord(ev_h2d_done, pool->s_h2d));
@@ -296,7 +297,8 @@ lv_status validate_desc(const lv_pool_desc* d) {
   if (d->unit_us < 1 || d->unit_us > (1ll << 31)) return LV_ERR_INVALID;
   if (d->t_play_mode != LV_PLAY_PLAYBACK && d->t_play_mode != LV_PLAY_COUNTERS) return LV_ERR_INVALID;
   if (d->within_order != LV_SUFFIX_FIRST && d->within_order != LV_ASCENDING) return LV_ERR_INVALID;
-  if (d->reserved != 0 || d->hbm_kv == nullptr) return LV_ERR_INVALID;
+  if (d->policy != LV_POLICY_NEXT_USE && d->policy != LV_POLICY_LRU) return LV_ERR_INVALID;
+  if (d->hbm_kv == nullptr) return LV_ERR_INVALID;
   return LV_OK;
 }
 
@@ -326,6 +328,7 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
   d.unit_us = desc->unit_us;
   d.within = desc->within_order;
   d.tplay = desc->t_play_mode;
+  d.policy = desc->policy;
 
   // the caller's HBM sub-page arrays
   std::vector<uint8_t*> kv(d.J);
@@ -418,6 +421,7 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
     return fail(LV_ERR_OOM);
   }
   pool->stage_ctas = pool->num_sms;
+  if (const char* env = std::getenv("LV_STAGE_KERNEL")) pool->stage_tma = std::strcmp(env, "lsu") != 0;
   cudaMemPoolProps props{};
   props.allocType = cudaMemAllocationTypePinned;
   props.location.type = cudaMemLocationTypeDevice;
@@ -707,6 +711,62 @@ lv_status lv_make_resident(lv_pool* pool, int32_t sid, int64_t now_us, int32_t a
     return LV_ERR_OOM;
   }
 }
+
+namespace {
+// A device address for p (device memory, or mapped page-locked host memory), else nullptr.
+void* device_alias(const void* p) {
+  cudaPointerAttributes a{};
+  if (p == nullptr || cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return const_cast<void*>(p);
+  if (a.type == cudaMemoryTypeHost) return a.devicePointer;
+  return nullptr;
+}
+
+lv_status pack_impl(lv_pool* pool, const int32_t* pages, int64_t n, void* run, bool pack, cudaStream_t s) {
+  void* rdev = device_alias(run);
+  if (!rdev || (reinterpret_cast<uintptr_t>(rdev) & 15)) return LV_ERR_INVALID;
+  Staging st(pool, s);
+  const void* pin = nullptr;
+  void* tdev = nullptr;
+  lv_status r;
+  if ((r = st.in(pages, (size_t)n * 4, &pin)) != LV_OK) return r;
+  if ((r = st.out(nullptr, (size_t)n * sizeof(int4), &tdev, true)) != LV_OK) return r;
+  LV_TRY(lv::launch_tasks_pages(pool->d, static_cast<const int32_t*>(pin), n, pack,
+                                static_cast<int4*>(tdev), s));
+  LV_TRY(lv::launch_stage(pool->d, pack, static_cast<int4*>(tdev), 0, n, static_cast<uint8_t*>(rdev), s,
+                          pool->stage_ctas, timing_pair(pool, pack ? LV_TIMING_PACK : LV_TIMING_UNPACK),
+                          pool->stage_tma));
+  return st.finish();
+}
+}  // namespace
+
+lv_status lv_pack_pages(lv_pool* pool, const int32_t* pages, int64_t n, void* dst, lv_stream stream) {
+  if (!pool || n < 0 || n > 0x7fffffffll || (n > 0 && (!pages || !dst))) return LV_ERR_INVALID;
+  if (n == 0) return LV_OK;
+  DeviceGuard g(pool->device);
+  try {
+    return pack_impl(pool, pages, n, dst, true, as_stream(stream));
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_unpack_pages(lv_pool* pool, const void* src, const int32_t* pages, int64_t n,
+                          lv_stream stream) {
+  if (!pool || n < 0 || n > 0x7fffffffll || (n > 0 && (!pages || !src))) return LV_ERR_INVALID;
+  if (n == 0) return LV_OK;
+  DeviceGuard g(pool->device);
+  try {
+    return pack_impl(pool, pages, n, const_cast<void*>(src), false, as_stream(stream));
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+void* lv_pool_host_device_ptr(lv_pool* pool) { return pool ? pool->d.host : nullptr; }
 
 lv_status lv_remap(lv_pool* pool, const lv_remap_entry* entries, int64_t n, lv_stream stream) {
   if (!pool || n < 0 || (n > 0 && !entries)) return LV_ERR_INVALID;

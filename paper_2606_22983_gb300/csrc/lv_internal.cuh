@@ -45,6 +45,7 @@ struct DevPool {
   int64_t reply_prior_us, protect_us, unit_us;
   int32_t within;         // LV_SUFFIX_FIRST / LV_ASCENDING
   int32_t tplay;          // LV_PLAY_PLAYBACK / LV_PLAY_COUNTERS
+  int32_t policy;         // LV_POLICY_NEXT_USE / LV_POLICY_LRU
   uint8_t* const* kv;     // [J] device pointers, sub-page j of page p at kv[j] + p*P
   uint8_t* host;          // device view of the host pool [host_pages][J][P]
   lv_session_state* sess; // [S]
@@ -132,7 +133,9 @@ cudaError_t launch_exchange_plan(const DevPool& p, const lv_victim* v, int64_t n
 // pack (staging[t] <- out pages) or unpack (in pages <- staging[t]) for tasks [t_begin, t_end)
 cudaError_t launch_stage(const DevPool& p, bool pack, const int4* tasks, int64_t t_begin,
                          int64_t t_end, uint8_t* staging, cudaStream_t s, int ctas,
-                         const EventPair* ev);
+                         const EventPair* ev, bool tma);
+cudaError_t launch_tasks_pages(const DevPool& p, const int32_t* pages, int64_t n, bool pack,
+                               int4* tasks, cudaStream_t s);
 cudaError_t configure_stage_kernels(const DevPool& p);
 cudaError_t configure_kernels();   // once per device, before the first launch
 

@@ -182,8 +182,10 @@ __global__ void k_events(DevPool p, const lv_event* __restrict__ ev, long long n
       case LV_EV_TURN_BEGIN:
         st.flags = (st.flags | LV_RUNNING) & ~LV_IMMEDIATE;
         st.protect_until_us = 0;
+        st.last_use_us = x.t_us;
         break;
       case LV_EV_TURN_END:
+        st.last_use_us = x.t_us;
         st.flags &= ~(LV_RUNNING | LV_DONE_VALID);
         st.gen_us = x.a;
         st.play_us = 0;
@@ -238,6 +240,15 @@ __global__ void k_events(DevPool p, const lv_event* __restrict__ ev, long long n
 __device__ __forceinline__ unsigned long long session_key(const DevPool& p, int32_t s,
                                                           long long now_us, bool fallback) {
   const lv_session_state st = p.sess[s];
+  if (p.policy == LV_POLICY_LRU) {
+    // least recently used first: every non-running session is a candidate
+    if (st.flags & LV_RUNNING) return 0ull;
+    long long t = st.last_use_us;
+    if (t < 0) t = 0;
+    if (t > kKeyMax) t = kKeyMax;
+    return (1ull << 63) | ((unsigned long long)(kKeyMax - t) << 31) |
+           (unsigned long long)(0x7fffffff - s);
+  }
   const bool normal = !(st.flags & (LV_RUNNING | LV_IMMEDIATE)) && !(now_us < st.protect_until_us);
   if (!normal && !(fallback && !(st.flags & LV_RUNNING))) return 0ull;
   long long t_play;
@@ -763,6 +774,9 @@ __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.comm
 __device__ __forceinline__ void bulk_wait_read_all() {
   asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
+__device__ __forceinline__ void bulk_wait_read_1() {
+  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 // Bounded wait on a stage barrier: false after `limit` polls (the data never came).
@@ -815,21 +829,20 @@ k_stage_tasks(DevPool p, const int4* __restrict__ tasks, long long t_begin, long
   uint32_t phase[kMaxStages];
   for (int s = 0; s < stages; ++s) { live[s] = false; phase[s] = 0; }
   bool failed = false;
-  // prologue: fill the ring
-  long long issued = 0;
-  for (; issued < mine && issued < stages; ++issued) {
-    const int s = (int)(issued % stages);
+  auto issue = [&](long long k) {
+    const int s = (int)(k % stages);
     const uint8_t* src;
-    if (unit_ptrs(issued, &src, &dsts[s])) {
+    live[s] = unit_ptrs(k, &src, &dsts[s]);
+    if (live[s]) {
       mbar_expect_tx(&bars[s], P);
       bulk_load(stage_mem + (size_t)s * P, src, P, &bars[s]);
-      live[s] = true;
-    } else {
-      live[s] = false;
     }
-  }
+  };
+  // prologue: one load in flight per stage
+  for (long long k = 0; k < mine && k < stages; ++k) issue(k);
   for (long long k = 0; k < mine; ++k) {
     const int s = (int)(k % stages);
+    bool stored = false;
     if (live[s]) {
       if (!mbar_wait_bounded(&bars[s], phase[s], kWaitPolls)) {
         failed = true;
@@ -838,20 +851,13 @@ k_stage_tasks(DevPool p, const int4* __restrict__ tasks, long long t_begin, long
       phase[s] ^= 1u;
       bulk_store(dsts[s], stage_mem + (size_t)s * P, P);
       bulk_commit();
-      bulk_wait_read_all();          // stage s may be refilled once the store has read it
+      stored = true;
     }
-    if (issued < mine) {
-      const uint8_t* src;
-      if (unit_ptrs(issued, &src, &dsts[s])) {
-        mbar_expect_tx(&bars[s], P);
-        bulk_load(stage_mem + (size_t)s * P, src, P, &bars[s]);
-        live[s] = true;
-      } else {
-        live[s] = false;
-      }
-      ++issued;
-    } else {
-      live[s] = false;
+    // refill the stage of unit k-1 once its store has read it; unit k's store may still run
+    if (k >= 1 && k - 1 + stages < mine) {
+      if (stored) bulk_wait_read_1();
+      else bulk_wait_read_all();
+      issue(k - 1 + stages);
     }
   }
   if (failed) {
@@ -863,55 +869,108 @@ k_stage_tasks(DevPool p, const int4* __restrict__ tasks, long long t_begin, long
   bulk_wait_all();
 }
 
+// The same moves with plain 16-byte loads and stores (256 threads per CTA).
+template <bool kPack>
+__global__ void __launch_bounds__(kCopyThreads)
+k_stage_tasks_lsu(DevPool p, const int4* __restrict__ tasks, long long t_begin, long long t_end,
+                  uint8_t* __restrict__ staging) {
+  const long long units = (t_end - t_begin) * p.J;
+  const int nvec = (int)(p.P >> 4);
+  for (long long u = blockIdx.x; u < units; u += gridDim.x) {
+    const long long t = t_begin + u / p.J;
+    const int j = (int)(u % p.J);
+    const int4 tk = tasks[t];
+    uint8_t* st = staging + ((size_t)t * p.J + j) * p.P;
+    if (kPack) {
+      if (tk.x < 0) continue;
+      copy_subpage(reinterpret_cast<const int4*>(p.kv[j] + (size_t)tk.x * p.P), reinterpret_cast<int4*>(st), nvec);
+    } else {
+      if (tk.z < 0) continue;
+      copy_subpage(reinterpret_cast<const int4*>(st), reinterpret_cast<int4*>(p.kv[j] + (size_t)tk.w * p.P), nvec);
+    }
+  }
+}
+
+// Tasks for a plain list of pages: pack reads them ({page, -1, -1, -1}), unpack
+// writes them ({-1, -1, 0, page}); an out-of-range page gives an empty task.
+__global__ void k_tasks_pages(DevPool p, const int32_t* __restrict__ pages, long long n, bool pack,
+                              int4* __restrict__ tasks) {
+  const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const int32_t pg = pages[i];
+  if (pg < 0 || pg >= p.hbm_pages) {
+    set_error(p.ctl, LV_ERR_BOUNDS, i);
+    tasks[i] = make_int4(-1, -1, -1, -1);
+    return;
+  }
+  tasks[i] = pack ? make_int4(pg, -1, -1, -1) : make_int4(-1, -1, 0, pg);
+}
+
 // ---------------------------------------------------------------- commit
 __device__ __forceinline__ bool bit_is_set(const uint32_t* bits, long long i) {
   return (bits[i >> 5] >> (i & 31)) & 1u;
 }
 
-__global__ void k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t epoch) {
+constexpr int kRemapThreads = 256;
+
+// One thread per entry.  The allocation counts and the commit counter change
+// by block totals (one atomic per block and counter, not one per entry).
+__global__ void __launch_bounds__(kRemapThreads)
+k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t epoch) {
   const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
-  if (i >= n) return;
-  const lv_remap_entry x = e[i];
-  if (x.sid < 0 || x.sid >= p.S || x.blk < 0 || x.blk >= nblocks_of(p, x.sid)) {
-    set_error(p.ctl, LV_ERR_BOUNDS, i);
-    return;
-  }
-  const size_t ti = (size_t)x.sid * p.maxB + x.blk;
-  if (atomicExch(&p.mark[ti], epoch) == epoch) {      // the same block twice in one call
-    set_error(p.ctl, LV_ERR_DOUBLE_MAP, i);
-    return;
-  }
-  const unsigned long long key = owner_key(x.sid, x.blk);
-  if (x.loc >= 0) {
-    if (x.loc >= p.hbm_pages) { set_error(p.ctl, LV_ERR_BOUNDS, i); return; }
-    if (!bit_is_set(p.bits_hbm, x.loc) || atomicCAS(&p.own_hbm[x.loc], kOwnerNone, key) != kOwnerNone) {
-      set_error(p.ctl, LV_ERR_DOUBLE_MAP, i);
-      return;
+  bool ok = false, freed_hbm = false, freed_host = false;
+  if (i < n) {
+    const lv_remap_entry x = e[i];
+    int err = 0;
+    size_t ti = 0;
+    if (x.sid < 0 || x.sid >= p.S || x.blk < 0 || x.blk >= nblocks_of(p, x.sid)) {
+      err = LV_ERR_BOUNDS;
+    } else {
+      ti = (size_t)x.sid * p.maxB + x.blk;
+      if (atomicExch(&p.mark[ti], epoch) == epoch) err = LV_ERR_DOUBLE_MAP;   // same block twice
     }
-  } else if (x.loc <= -2) {
-    const long long h = -(long long)x.loc - 2;
-    if (h >= p.host_pages) { set_error(p.ctl, LV_ERR_BOUNDS, i); return; }
-    if (!bit_is_set(p.bits_host, h) || atomicCAS(&p.own_host[h], kOwnerNone, key) != kOwnerNone) {
-      set_error(p.ctl, LV_ERR_DOUBLE_MAP, i);
-      return;
+    const unsigned long long key = err ? 0ull : owner_key(x.sid, x.blk);
+    if (!err) {
+      if (x.loc >= 0) {
+        if (x.loc >= p.hbm_pages) err = LV_ERR_BOUNDS;
+        else if (!bit_is_set(p.bits_hbm, x.loc) ||
+                 atomicCAS(&p.own_hbm[x.loc], kOwnerNone, key) != kOwnerNone)
+          err = LV_ERR_DOUBLE_MAP;
+      } else if (x.loc <= -2) {
+        const long long h = -(long long)x.loc - 2;
+        if (h >= p.host_pages) err = LV_ERR_BOUNDS;
+        else if (!bit_is_set(p.bits_host, h) || atomicCAS(&p.own_host[h], kOwnerNone, key) != kOwnerNone)
+          err = LV_ERR_DOUBLE_MAP;
+      } else {
+        err = LV_ERR_BOUNDS;
+      }
     }
-  } else {
-    set_error(p.ctl, LV_ERR_BOUNDS, i);
-    return;
+    if (err) {
+      set_error(p.ctl, err, i);
+    } else {
+      const int32_t old = p.table[ti];
+      p.table[ti] = x.loc;
+      if (old >= 0 && old < p.hbm_pages) {
+        if (atomicCAS(&p.own_hbm[old], key, kOwnerNone) != key) set_error(p.ctl, LV_ERR_STATE, i);
+        atomicAnd(&p.bits_hbm[old >> 5], ~(1u << (old & 31)));
+        freed_hbm = true;
+      } else if (old <= -2 && (-(long long)old - 2) < p.host_pages) {
+        const long long h = -(long long)old - 2;
+        if (atomicCAS(&p.own_host[h], key, kOwnerNone) != key) set_error(p.ctl, LV_ERR_STATE, i);
+        atomicAnd(&p.bits_host[h >> 5], ~(1u << (h & 31)));
+        freed_host = true;
+      }
+      ok = true;
+    }
   }
-  const int32_t old = p.table[ti];
-  p.table[ti] = x.loc;
-  if (old >= 0 && old < p.hbm_pages) {
-    if (atomicCAS(&p.own_hbm[old], key, kOwnerNone) != key) set_error(p.ctl, LV_ERR_STATE, i);
-    atomicAnd(&p.bits_hbm[old >> 5], ~(1u << (old & 31)));
-    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HBM_ALLOC]), (unsigned long long)-1ll);
-  } else if (old <= -2 && (-(long long)old - 2) < p.host_pages) {
-    const long long h = -(long long)old - 2;
-    if (atomicCAS(&p.own_host[h], key, kOwnerNone) != key) set_error(p.ctl, LV_ERR_STATE, i);
-    atomicAnd(&p.bits_host[h >> 5], ~(1u << (h & 31)));
-    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HOST_ALLOC]), (unsigned long long)-1ll);
+  const int n_ok = __syncthreads_count(ok);
+  const int n_hbm = __syncthreads_count(freed_hbm);
+  const int n_host = __syncthreads_count(freed_host);
+  if (threadIdx.x == 0) {
+    if (n_hbm) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HBM_ALLOC]), (unsigned long long)-(long long)n_hbm);
+    if (n_host) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HOST_ALLOC]), (unsigned long long)-(long long)n_host);
+    if (n_ok) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_REMAP]), (unsigned long long)n_ok);
   }
-  atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_REMAP]), 1ull);
 }
 
 __global__ void k_cancel(DevPool p, const int32_t* __restrict__ locs, long long n) {
@@ -1274,18 +1333,32 @@ cudaError_t configure_stage_kernels(const DevPool& p) {
 }
 
 cudaError_t launch_stage(const DevPool& p, bool pack, const int4* tasks, int64_t t_begin, int64_t t_end,
-                         uint8_t* staging, cudaStream_t s, int ctas, const EventPair* ev) {
+                         uint8_t* staging, cudaStream_t s, int ctas, const EventPair* ev, bool tma) {
   if (t_end <= t_begin) return cudaSuccess;
-  const int stages = stage_count(p);
-  const size_t smem = (size_t)stages * p.P;
   const long long units = (t_end - t_begin) * (long long)p.J;
-  const unsigned grid = blocks_for(units, 1, ctas);
   if (ev) cudaEventRecord(ev->start, s);
-  if (pack)
-    k_stage_tasks<true><<<grid, kStageThreads, smem, s>>>(p, tasks, t_begin, t_end, staging, stages);
-  else
-    k_stage_tasks<false><<<grid, kStageThreads, smem, s>>>(p, tasks, t_begin, t_end, staging, stages);
+  if (tma) {
+    const int stages = stage_count(p);
+    const size_t smem = (size_t)stages * p.P;
+    const unsigned grid = blocks_for(units, 1, ctas);
+    if (pack)
+      k_stage_tasks<true><<<grid, kStageThreads, smem, s>>>(p, tasks, t_begin, t_end, staging, stages);
+    else
+      k_stage_tasks<false><<<grid, kStageThreads, smem, s>>>(p, tasks, t_begin, t_end, staging, stages);
+  } else {
+    const unsigned grid = blocks_for(units, 1, 4ll * ctas);
+    if (pack)
+      k_stage_tasks_lsu<true><<<grid, kCopyThreads, 0, s>>>(p, tasks, t_begin, t_end, staging);
+    else
+      k_stage_tasks_lsu<false><<<grid, kCopyThreads, 0, s>>>(p, tasks, t_begin, t_end, staging);
+  }
   if (ev) cudaEventRecord(ev->end, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_tasks_pages(const DevPool& p, const int32_t* pages, int64_t n, bool pack, int4* tasks,
+                               cudaStream_t s) {
+  k_tasks_pages<<<blocks_for(n, 256, 1ll << 30), 256, 0, s>>>(p, pages, n, pack, tasks);
   return cudaGetLastError();
 }
 
@@ -1300,7 +1373,7 @@ cudaError_t launch_exchange_plan(const DevPool& p, const lv_victim* v, int64_t n
 
 cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, int32_t epoch,
                          cudaStream_t s) {
-  k_remap<<<blocks_for(n, 256, 1ll << 30), 256, 0, s>>>(p, e, n, epoch);
+  k_remap<<<blocks_for(n, kRemapThreads, 1ll << 30), kRemapThreads, 0, s>>>(p, e, n, epoch);
   return cudaGetLastError();
 }
 

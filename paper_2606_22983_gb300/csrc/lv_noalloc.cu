@@ -93,6 +93,7 @@ extern "C" lv_status lv_select_victims_noalloc(const lv_rank_params* prm,
   p.T = prm->page_tokens;
   p.within = prm->within_order;
   p.tplay = prm->t_play_mode;
+  p.policy = LV_POLICY_NEXT_USE;
   p.reply_prior_us = prm->reply_prior_us;
   p.unit_us = prm->unit_us;
   p.sess = const_cast<lv_session_state*>(static_cast<const lv_session_state*>(sess));

@@ -15,6 +15,12 @@ from . import lv
 from .pool import KVPool
 
 
+def zero_host(pool: KVPool):
+    if pool.host_dev is not None:
+        pool.host_dev.zero_()
+        torch.cuda.synchronize(pool.device)
+
+
 def pool_for(workload, device=None, stream=None, kv=None) -> KVPool:
     spec = workload.spec
     sh = spec.shape
@@ -25,7 +31,7 @@ def pool_for(workload, device=None, stream=None, kv=None) -> KVPool:
                   host_pages=spec.host_pages, reply_prior_us=spec.reply_prior_us,
                   protect_us=spec.protect_us, unit_us=spec.unit_us,
                   within_order=spec.within_order, t_play_mode=spec.t_play_mode,
-                  device=device, stream=stream, kv=kv)
+                  device=device, stream=stream, kv=kv, policy=spec.policy)
     init = workload.init
     pool.import_placement(init.placement, init.ctx_tokens)
     st = np.zeros(spec.n_sessions, dtype=lv.SESSION_DTYPE)
@@ -74,9 +80,9 @@ class ContentWriter:
                     idx = torch.from_numpy(locs[sl][m]).to(pool.device)
                     pool.kv[j].index_copy_(0, idx, vals[torch.from_numpy(m).to(pool.device)].view(torch.uint8))
                 if (~m).any():
-                    slots = -(locs[sl][~m] + 2)
-                    host_vals = vals[torch.from_numpy(~m).to(pool.device)].view(torch.uint8).cpu().numpy()
-                    pool.host[slots, j, :] = host_vals
+                    slots = torch.from_numpy(-(locs[sl][~m] + 2)).to(pool.device)
+                    host_vals = vals[torch.from_numpy(~m).to(pool.device)].view(torch.uint8)
+                    pool.host_dev[:, j, :].index_copy_(0, slots, host_vals)   # GPU writes over the link
         torch.cuda.synchronize(pool.device)
 
     def write_initial(self, workload):
@@ -116,5 +122,5 @@ def fill_random(pool: KVPool, seed: int = 0):
             n = min(step, pool.host_pages - lo)
             v = torch.randn((n, pool.J * pool.P // 2), generator=g, device=pool.device,
                             dtype=torch.float32).to(torch.bfloat16)
-            pool.host[lo:lo + n] = v.view(torch.uint8).cpu().numpy().reshape(n, pool.J, pool.P)
+            pool.host_dev[lo:lo + n].copy_(v.view(torch.uint8).view(n, pool.J, pool.P))
     torch.cuda.synchronize(pool.device)

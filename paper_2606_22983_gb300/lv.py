@@ -28,6 +28,7 @@ LV_SUFFIX_FIRST, LV_ASCENDING = 0, 1
 LV_PLAY_PLAYBACK, LV_PLAY_COUNTERS = 0, 1
 LV_MODE_AUTO, LV_MODE_ZERO_COPY, LV_MODE_STAGED = 0, 1, 2
 LV_SELECT_FALLBACK = 1
+LV_POLICY_NEXT_USE, LV_POLICY_LRU = 0, 1
 LV_RUNNING, LV_IMMEDIATE, LV_RESP_OPEN, LV_DONE_VALID = 1, 2, 4, 8
 (LV_EV_TURN_BEGIN, LV_EV_TURN_END, LV_EV_PLAYBACK, LV_EV_SPEECH_START, LV_EV_BARGE_IN,
  LV_EV_SPEECH_STOP, LV_EV_PRELOADED) = 1, 2, 3, 4, 5, 6, 7
@@ -48,7 +49,7 @@ class lv_pool_desc(ctypes.Structure):
                 ("host_pages", ctypes.c_int64), ("hbm_kv", ctypes.POINTER(ctypes.c_void_p)),
                 ("host_kv", ctypes.c_void_p), ("reply_prior_us", ctypes.c_int64),
                 ("protect_us", ctypes.c_int64), ("unit_us", ctypes.c_int64),
-                ("t_play_mode", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+                ("t_play_mode", ctypes.c_int32), ("policy", ctypes.c_int32)]
 
 
 class lv_stats(ctypes.Structure):
@@ -88,13 +89,13 @@ LV_RESIDENT_DONE, LV_RESIDENT_SKIPPED, LV_RESIDENT_NOTHING, LV_RESIDENT_FAILED =
 SESSION_DTYPE = np.dtype([("ctx_tokens", "<i4"), ("flags", "<i4"), ("gen_us", "<i8"),
                           ("play_us", "<i8"), ("t_done_us", "<i8"), ("reply_ema_us", "<i8"),
                           ("reply_n", "<i4"), ("pad", "<i4"), ("reply_tokens", "<i8"),
-                          ("protect_until_us", "<i8")])
+                          ("protect_until_us", "<i8"), ("last_use_us", "<i8")])
 EVENT_DTYPE = np.dtype([("kind", "<i4"), ("sid", "<i4"), ("t_us", "<i8"), ("a", "<i8"), ("b", "<i8")])
 VICTIM_DTYPE = np.dtype([("sid", "<i4"), ("blk", "<i4"), ("page", "<i4")])
 RESIDENT_DTYPE = np.dtype([("k", "<i8"), ("n_found", "<i8"), ("n_victims", "<i8"), ("n_loaded", "<i8"),
                            ("n_appended", "<i8"), ("status", "<i4"), ("pad", "<i4")])
 REMAP_DTYPE = np.dtype([("sid", "<i4"), ("blk", "<i4"), ("loc", "<i4")])
-assert SESSION_DTYPE.itemsize == 64 and EVENT_DTYPE.itemsize == 32
+assert SESSION_DTYPE.itemsize == 72 and EVENT_DTYPE.itemsize == 32
 assert VICTIM_DTYPE.itemsize == 12 and REMAP_DTYPE.itemsize == 12
 
 
@@ -117,6 +118,8 @@ def _load():
         "lv_swap_exchange": [vp, vp, i64, i32, vp, i64, vp, vp, i32, vp],
         "lv_make_resident": [vp, i32, i64, i32, u32, i64, vp, vp, vp, vp, vp, vp, vp],
         "lv_timing_enable": [vp, i32],
+        "lv_pack_pages": [vp, vp, i64, vp, vp],
+        "lv_unpack_pages": [vp, vp, vp, i64, vp],
         "lv_timing_read": [vp, ctypes.POINTER(lv_kernel_timing), i32],
         "lv_remap": [vp, vp, i64, vp],
         "lv_cancel": [vp, vp, i64, vp],
@@ -136,6 +139,8 @@ def _load():
         f.restype = ctypes.c_int
     lib.lv_pool_host_ptr.argtypes = [vp]
     lib.lv_pool_host_ptr.restype = vp
+    lib.lv_pool_host_device_ptr.argtypes = [vp]
+    lib.lv_pool_host_device_ptr.restype = vp
     lib.lv_status_str.argtypes = [ctypes.c_int]
     lib.lv_status_str.restype = ctypes.c_char_p
     lib.lv_version.argtypes = []
@@ -150,7 +155,8 @@ EXPORTED = ("lv_pool_create", "lv_pool_destroy", "lv_pool_host_ptr", "lv_pool_im
             "lv_swap_out", "lv_swap_in", "lv_swap_exchange", "lv_make_resident", "lv_remap", "lv_cancel", "lv_session_append",
             "lv_session_counts", "lv_session_blocks", "lv_read_tables", "lv_sync",
             "lv_get_stats", "lv_clear_error", "lv_status_str", "lv_version",
-            "lv_select_victims_noalloc", "lv_timing_enable", "lv_timing_read")
+            "lv_select_victims_noalloc", "lv_timing_enable", "lv_timing_read", "lv_pack_pages",
+            "lv_unpack_pages", "lv_pool_host_device_ptr")
 
 
 def lib():
@@ -203,6 +209,18 @@ def lv_pool_destroy(pool, stream=None):
 
 def lv_pool_host_ptr(pool) -> int:
     return _lib.lv_pool_host_ptr(pool)
+
+
+def lv_pool_host_device_ptr(pool) -> int:
+    return _lib.lv_pool_host_device_ptr(pool)
+
+
+def lv_pack_pages(pool, pages, n, dst, stream=None):
+    _check(_lib.lv_pack_pages(pool, ptr(pages), n, ptr(dst), stream_handle(stream)), "lv_pack_pages")
+
+
+def lv_unpack_pages(pool, src, pages, n, stream=None):
+    _check(_lib.lv_unpack_pages(pool, ptr(src), ptr(pages), n, stream_handle(stream)), "lv_unpack_pages")
 
 
 def lv_pool_import(pool, placement, ctx_tokens, stream=None):

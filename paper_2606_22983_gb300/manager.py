@@ -7,6 +7,9 @@ Consumes monitor event scripts (records ``(t_us, kind, sid, a, b, c, d)``):
          the host tier takes the turn (perms[d][0] when none has)
   kind 3 PLAYBACK(sid, a=delta_us)    kind 4 SPEECH_START(sid)
   kind 5 BARGE_IN(sid)                kind 6 SPEECH_STOP(sid)
+  kind 7 TURN_SCATTER(d=row, a=key): as TURN_ANY, host blocks reloaded in the
+         order ``order_fn(key, blocks)`` (given by the caller)
+  kind 8 EVICT(a=k): free k pages now, in the next-use order
 
 A turn makes the session fully resident (a synchronous foreground load),
 grows its context, then records the reply.  By default (``driver="device"``)
@@ -34,6 +37,7 @@ from . import lv
 from .pool import KVPool
 
 EV_TURN, EV_TURN_ANY, EV_PLAYBACK, EV_SPEECH_START, EV_BARGE_IN, EV_SPEECH_STOP = 1, 2, 3, 4, 5, 6
+EV_TURN_SCATTER, EV_EVICT = 7, 8
 
 _STATE_EVENT = {EV_PLAYBACK: lv.LV_EV_PLAYBACK, EV_SPEECH_START: lv.LV_EV_SPEECH_START,
                 EV_BARGE_IN: lv.LV_EV_BARGE_IN, EV_SPEECH_STOP: lv.LV_EV_SPEECH_STOP}
@@ -47,7 +51,7 @@ def _event(kind, sid, t, a=0, b=0):
 
 class KVManager:
     def __init__(self, pool: KVPool, perms=None, on_append=None, rank_on="none", admit=None,
-                 mode=lv.LV_MODE_AUTO, record=True, driver="device"):
+                 mode=lv.LV_MODE_AUTO, record=True, driver="device", order_fn=None):
         self.pool = pool
         self.perms = perms
         self.on_append = on_append      # callback(sid, old_ctx, new_ctx, pages) after growth
@@ -60,6 +64,7 @@ class KVManager:
         # device: one lv_make_resident per step, no host round trip;
         # exchange: select, then one lv_swap_exchange; sequential: the four calls
         self.driver = driver
+        self.order_fn = order_fn        # (key, blocks) -> blocks, for TURN_SCATTER
         self.res_h = torch.zeros(lv.RESIDENT_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
         self.counters = dict(victims=0, pages_out=0, pages_in=0, preloads=0,
                              preload_skipped=0, turns=0, sync_loads=0, appended=0)
@@ -127,8 +132,8 @@ class KVManager:
             self.on_append(sid, old_ctx, old_ctx + append_tokens)
         return status
 
-    def make_resident(self, sid, now_us, append_tokens, foreground, rec):
-        if self.driver == "device":
+    def make_resident(self, sid, now_us, append_tokens, foreground, rec, order_key=None):
+        if self.driver == "device" and order_key is None:
             status = self._device(sid, now_us, append_tokens, foreground, rec)
             if status == lv.LV_RESIDENT_FAILED:
                 raise lv.LvError(self.pool.sync(raise_on_error=False) or lv.LV_ERR_NO_HBM,
@@ -136,6 +141,9 @@ class KVManager:
             return status
         pool = self.pool
         hblk, nh = self.host_blocks(sid)
+        if order_key is not None and nh:
+            order = np.asarray(self.order_fn(order_key, hblk.cpu().numpy()), dtype=np.int32)
+            hblk = torch.from_numpy(order).to(pool.device)
         new_blocks = 0
         if append_tokens:
             ctx = self.ctx_tokens(sid)
@@ -144,7 +152,7 @@ class KVManager:
         need = nh + new_blocks
         k = max(0, need - self.free_budget())
         rec["k"] = k
-        if self.driver == "exchange":
+        if self.driver != "sequential":
             if not self._exchange(sid, now_us, k, hblk, nh, foreground, rec):
                 return False
         else:
@@ -235,6 +243,8 @@ class KVManager:
         return True
 
     def preload(self, sid, now_us, rec):
+        if self.pool.policy == lv.LV_POLICY_LRU:
+            return              # the LRU baseline loads at turn start only
         if self.driver == "device" and self.admit is None:
             status = self._device(sid, now_us, 0, False, rec)
             if status == lv.LV_RESIDENT_DONE:
@@ -259,6 +269,26 @@ class KVManager:
             self.counters["preload_skipped"] += 1
             rec["preload"] = "skipped"
 
+    def evict(self, now_us, k, rec):
+        """Free k pages now: the first k of the victim order (fewer if there are fewer)."""
+        pool = self.pool
+        victims, n = pool.select(now_us, k, 0)
+        rec["k"] = int(k)
+        if self.record:
+            rec["victims"] = victims.cpu().numpy().astype(np.int64)
+        if n == 0:
+            return
+        if self.driver == "sequential":
+            slots, commit = pool.swap_out(victims, n, self.mode)
+            pool.remap(commit, n)
+        else:
+            slots, _ = pool.exchange(victims, n, 0, None, 0, self.mode)
+        if self.record:
+            rec["slots"] = slots.cpu().numpy().astype(np.int64)
+        self.counters["victims"] += n
+        self.counters["pages_out"] += n
+        self.bytes_moved += n * pool.J * pool.P
+
     def turn_target(self, row):
         _, host = self.pool.counts()
         for s in self.perms[row]:
@@ -276,19 +306,27 @@ class KVManager:
             pool.events(_event(_STATE_EVENT[kind], sid, t, a))
             if kind in (EV_SPEECH_START, EV_BARGE_IN):
                 self.preload(sid, t, rec)
-        elif kind in (EV_TURN, EV_TURN_ANY):
-            if kind == EV_TURN_ANY:
+        elif kind in (EV_TURN, EV_TURN_ANY, EV_TURN_SCATTER):
+            order_key = None
+            if kind == EV_TURN_SCATTER:
+                sid = self.turn_target(d)
+                order_key, a = a, 0
+            elif kind == EV_TURN_ANY:
                 sid = self.turn_target(d)
             pool.events(_event(lv.LV_EV_TURN_BEGIN, sid, t))
-            if self.driver != "device" and self.host_blocks(sid)[1]:
+            host_path = self.driver != "device" or order_key is not None
+            if host_path and self.host_blocks(sid)[1]:
                 self.counters["sync_loads"] += 1
-            self.make_resident(sid, t, a, foreground=True, rec=rec)
+            self.make_resident(sid, t, a, foreground=True, rec=rec, order_key=order_key)
             pool.events(_event(lv.LV_EV_TURN_END, sid, t, b, c))
             self.counters["turns"] += 1
+        elif kind == EV_EVICT:
+            self.evict(t, a, rec)
         else:
             raise ValueError(f"unknown script event kind {kind}")
         rec["sid"] = sid
-        if self.rank_on == "all" or (self.rank_on == "turns" and kind in (EV_TURN, EV_TURN_ANY)):
+        if self.rank_on == "all" or (self.rank_on == "turns" and kind in (EV_TURN, EV_TURN_ANY,
+                                                                           EV_TURN_SCATTER)):
             order, n = pool.select(t, lv.LV_ALL, 0)
             rec["order"] = order.cpu().numpy().astype(np.int64)
         return rec

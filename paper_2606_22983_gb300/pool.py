@@ -13,12 +13,20 @@ import torch
 from . import lv
 
 
+class _CudaArray:
+    """__cuda_array_interface__ of a raw device address (no ownership)."""
+
+    def __init__(self, ptr, nbytes):
+        self.__cuda_array_interface__ = {"shape": (nbytes,), "typestr": "|u1",
+                                         "data": (int(ptr), False), "version": 3, "strides": None}
+
+
 class KVPool:
     def __init__(self, *, layers, kv_heads, head_dim, max_sessions, max_blocks, hbm_pages,
                  hbm_budget_pages, host_pages, page_tokens=16, elem_bytes=2,
                  reply_prior_us=3_000_000, protect_us=2_000_000, unit_us=80_000,
                  within_order=lv.LV_SUFFIX_FIRST, t_play_mode=lv.LV_PLAY_PLAYBACK,
-                 device=None, stream=None, kv=None):
+                 device=None, stream=None, kv=None, policy=lv.LV_POLICY_NEXT_USE):
         if not torch.cuda.is_available():
             raise RuntimeError("KVPool needs a CUDA device (liblv has no CPU path)")
         self.device = torch.device(device or "cuda", torch.cuda.current_device()) \
@@ -30,6 +38,7 @@ class KVPool:
         self.S, self.max_blocks = max_sessions, max_blocks
         self.hbm_pages, self.budget, self.host_pages = hbm_pages, hbm_budget_pages, host_pages
         self.launches = 0      # liblv kernels launched through this object
+        self.policy = policy
         with torch.cuda.device(self.device):
             if kv is None:
                 # one allocation, viewed as 2L sub-page arrays [hbm_pages][P]
@@ -45,7 +54,7 @@ class KVPool:
             d.hbm_kv = ctypes.cast(ptrs, ctypes.POINTER(ctypes.c_void_p))
             d.host_kv = None
             d.reply_prior_us, d.protect_us, d.unit_us = reply_prior_us, protect_us, unit_us
-            d.t_play_mode, d.reserved = t_play_mode, 0
+            d.t_play_mode, d.policy = t_play_mode, policy
             self.handle = lv.lv_pool_create(d, stream)
             cap = max(hbm_budget_pages, max_blocks, 1)
             self.cap = cap
@@ -59,13 +68,20 @@ class KVPool:
             self.count_h = torch.zeros(4, dtype=torch.int64).pin_memory()
         hp = lv.lv_pool_host_ptr(self.handle)
         self.host = None
+        self.host_dev = None
         if host_pages:
-            buf = (ctypes.c_uint8 * (host_pages * self.J * self.P)).from_address(hp)
+            nbytes = host_pages * self.J * self.P
+            buf = (ctypes.c_uint8 * nbytes).from_address(hp)
             self.host = np.frombuffer(buf, dtype=np.uint8).reshape(host_pages, self.J, self.P)
+            # the same host pool as a CUDA tensor (device-side alias of the mapped memory)
+            cai = _CudaArray(lv.lv_pool_host_device_ptr(self.handle), nbytes)
+            with torch.cuda.device(self.device):
+                self.host_dev = torch.as_tensor(cai, device=self.device).view(host_pages, self.J, self.P)
 
     # ------------------------------------------------------------------ life
     def close(self):
         if getattr(self, "handle", None):
+            self.host_dev = None
             lv.lv_pool_destroy(self.handle, self.stream)
             self.handle = None
             self.host = None

@@ -7,13 +7,13 @@ import torch
 
 from oracle import OracleManager
 from paper_2606_22983_gb300 import lv
-from paper_2606_22983_gb300.harness import ContentWriter, pool_for
+from paper_2606_22983_gb300.harness import ContentWriter, pool_for, zero_host
 from paper_2606_22983_gb300.manager import KVManager
-from workloads import value_table
+from workloads import scatter_order, value_table
 
 REC_KEYS = ("sid", "k", "victims", "slots", "in_blocks", "in_pages", "append_pages", "order", "preload")
 SESSION_FIELDS = ("ctx_tokens", "flags", "gen_us", "play_us", "t_done_us", "reply_ema_us",
-                  "reply_n", "reply_tokens", "protect_until_us")
+                  "reply_n", "reply_tokens", "protect_until_us", "last_use_us")
 
 
 def compare_records(ro, rg, where):
@@ -63,11 +63,11 @@ def make_pair(workload, with_bytes, rank_on="all", mode=lv.LV_MODE_AUTO, driver=
     writer = None
     if with_bytes:
         writer = ContentWriter(pool, workload)
-        pool.host[:] = 0
+        zero_host(pool)
         writer.write_initial(workload)
     gm = KVManager(pool, perms=workload.perms,
                    on_append=writer.write_appended if writer else None,
-                   rank_on=rank_on, mode=mode, driver=driver)
+                   rank_on=rank_on, mode=mode, driver=driver, order_fn=scatter_order)
     return om, pool, gm
 
 

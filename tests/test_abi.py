@@ -64,9 +64,10 @@ int main(void) {
   F(lv_session_state, ctx_tokens); F(lv_session_state, flags); F(lv_session_state, gen_us);
   F(lv_session_state, play_us); F(lv_session_state, t_done_us); F(lv_session_state, reply_ema_us);
   F(lv_session_state, reply_n); F(lv_session_state, reply_tokens); F(lv_session_state, protect_until_us);
+  F(lv_session_state, last_use_us);
   F(lv_event, kind); F(lv_event, sid); F(lv_event, t_us); F(lv_event, a); F(lv_event, b);
   F(lv_pool_desc, hbm_pages); F(lv_pool_desc, hbm_kv); F(lv_pool_desc, host_kv);
-  F(lv_pool_desc, reply_prior_us); F(lv_pool_desc, t_play_mode); F(lv_pool_desc, reserved);
+  F(lv_pool_desc, reply_prior_us); F(lv_pool_desc, t_play_mode); F(lv_pool_desc, policy);
   return 0;
 }
 ''')
@@ -99,7 +100,7 @@ int main(void) {
     for name in lv.EVENT_DTYPE.names:
         off, size = got[f"lv_event.{name}"]
         assert lv.EVENT_DTYPE.fields[name][1] == off
-    for name in ("hbm_pages", "hbm_kv", "host_kv", "reply_prior_us", "t_play_mode", "reserved"):
+    for name in ("hbm_pages", "hbm_kv", "host_kv", "reply_prior_us", "t_play_mode", "policy"):
         assert getattr(lv.lv_pool_desc, name).offset == got[f"lv_pool_desc.{name}"][0], name
 
 

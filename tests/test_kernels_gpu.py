@@ -1,0 +1,286 @@
+"""Kernel-level GPU tests through the C ABI: the ranker against the oracle on random
+session states (and at 2^20 resident pages), pack/unpack against the content
+definition, remap / cancel / allocation error paths, degenerate sizes, and host
+versus device pointer arguments."""
+import os
+import time
+
+import numpy as np
+import pytest
+
+pytestmark = pytest.mark.gpu
+
+
+def _tiny_pool(**kw):
+    from paper_2606_22983_gb300.pool import KVPool
+    args = dict(layers=2, kv_heads=2, head_dim=64, max_sessions=8, max_blocks=16, hbm_pages=64,
+                hbm_budget_pages=64, host_pages=64)
+    args.update(kw)
+    return KVPool(**args)
+
+
+def _oracle_states(st):
+    from oracle import sessions as se
+    out = []
+    for r in st:
+        out.append(se.SessionState(ctx_tokens=int(r["ctx_tokens"]), flags=int(r["flags"]),
+                                   gen_us=int(r["gen_us"]), play_us=int(r["play_us"]),
+                                   t_done_us=int(r["t_done_us"]), reply_ema_us=int(r["reply_ema_us"]),
+                                   reply_n=int(r["reply_n"]), reply_tokens=int(r["reply_tokens"]),
+                                   protect_until_us=int(r["protect_until_us"]),
+                                   last_use_us=int(r["last_use_us"])))
+    return out
+
+
+def _random_states(rng, S):
+    from paper_2606_22983_gb300 import lv
+    st = np.zeros(S, dtype=lv.SESSION_DTYPE)
+    st["gen_us"] = rng.integers(0, 6, S) * 1_000_000
+    st["play_us"] = (rng.random(S) * st["gen_us"]).astype(np.int64) // 500_000 * 500_000
+    st["reply_n"] = rng.integers(0, 2, S)
+    st["reply_ema_us"] = rng.integers(0, 4, S) * 700_000
+    st["reply_tokens"] = rng.integers(0, 80, S)
+    fl = np.zeros(S, np.int32)
+    fl |= np.where(rng.random(S) < 0.5, lv.LV_RESP_OPEN, 0).astype(np.int32)
+    r = rng.random(S)
+    fl |= np.where(r < 0.15, lv.LV_RUNNING, 0).astype(np.int32)
+    fl |= np.where((r >= 0.15) & (r < 0.3), lv.LV_IMMEDIATE, 0).astype(np.int32)
+    st["flags"] = fl
+    st["protect_until_us"] = np.where((r >= 0.3) & (r < 0.45), 10_000_000, 0)
+    return st
+
+
+def _random_placement(rng, S, maxb, T, hbm_pages, host_pages, p_host=0.3):
+    ctx = rng.integers(0, maxb * T + 1, S).astype(np.int32)
+    nb = -(-ctx // T)
+    placement = np.full((S, maxb), -1, np.int32)
+    pages = rng.permutation(hbm_pages)
+    slots = rng.permutation(host_pages)
+    pi = hi = 0
+    for s in range(S):
+        for b in range(nb[s]):
+            if rng.random() < p_host and hi < host_pages:
+                placement[s, b] = -(int(slots[hi]) + 2)
+                hi += 1
+            elif pi < hbm_pages:
+                placement[s, b] = int(pages[pi])
+                pi += 1
+            else:
+                placement[s, b] = -(int(slots[hi]) + 2)
+                hi += 1
+    return placement, ctx
+
+
+@pytest.mark.parametrize("within,tplay", [(0, 0), (1, 0), (0, 1)])
+def test_ranker_matches_oracle_on_random_states(within, tplay):
+    from paper_2606_22983_gb300 import lv
+    from oracle.policy import order_global
+    rng = np.random.default_rng(11 + within + 2 * tplay)
+    S, maxb, T = 64, 24, 16
+    pool = _tiny_pool(max_sessions=S, max_blocks=maxb, hbm_pages=1024, hbm_budget_pages=1024,
+                      host_pages=1024, within_order=within, t_play_mode=tplay,
+                      reply_prior_us=1_500_000, unit_us=40_000)
+    try:
+        for trial in range(12):
+            placement, ctx = _random_placement(rng, S, maxb, T, 1024, 1024)
+            pool.import_placement(placement, ctx)
+            st = _random_states(rng, S)
+            pool.set_sessions(st)
+            pool.sync()
+            gs = pool.get_sessions()
+            osess = _oracle_states(gs)
+            tables = placement.astype(np.int64)
+            nb = -(-ctx.astype(np.int64) // T)
+            now = int(rng.integers(0, 12_000_000))
+            for fallback in (False, True):
+                want = np.stack(order_global(tables, nb, osess, now, tplay, 1_500_000, 40_000,
+                                             within, fallback), axis=1)
+                flags = lv.LV_SELECT_FALLBACK if fallback else 0
+                got, n = pool.select(now, lv.LV_ALL, flags)
+                assert np.array_equal(got.cpu().numpy().astype(np.int64), want), (trial, fallback)
+                for k in (0, 1, 7, len(want), len(want) + 3):
+                    got, n = pool.select(now, k, flags)
+                    assert n == min(k, len(want))
+                    assert np.array_equal(got.cpu().numpy().astype(np.int64), want[:n])
+        assert pool.sync(raise_on_error=False) == 0
+    finally:
+        pool.close()
+
+
+def test_ranker_at_two_to_the_twenty_resident_pages():
+    """1024 sessions x 1024 blocks all resident (a metadata-sized page shape):
+    the full order and a top-256 match the oracle; reports microseconds per decision."""
+    import torch
+    from paper_2606_22983_gb300 import lv
+    from oracle.policy import order_global
+    rng = np.random.default_rng(5)
+    S, maxb, T = 1024, 1024, 16
+    n = S * maxb
+    pool = _tiny_pool(layers=1, kv_heads=1, head_dim=8, max_sessions=S, max_blocks=maxb,
+                      hbm_pages=n, hbm_budget_pages=n, host_pages=16)
+    try:
+        placement = rng.permutation(n).astype(np.int32).reshape(S, maxb)
+        ctx = np.full(S, maxb * T, np.int32)
+        pool.import_placement(placement, ctx)
+        st = _random_states(rng, S)
+        st["flags"] &= ~(lv.LV_RUNNING | lv.LV_IMMEDIATE)
+        st["protect_until_us"] = 0
+        st["gen_us"] = rng.integers(0, 10_000_000, S)          # distinct-ish keys
+        st["play_us"] = 0
+        pool.set_sessions(st)
+        pool.sync()
+        osess = _oracle_states(pool.get_sessions())
+        want = np.stack(order_global(placement.astype(np.int64), np.full(S, maxb), osess, 0, 0,
+                                     3_000_000, 80_000), axis=1)
+        assert want.shape[0] == n
+        got, cnt = pool.select(0, lv.LV_ALL, 0, capacity=n)
+        assert cnt == n and np.array_equal(got.cpu().numpy().astype(np.int64), want)
+        out = torch.empty((256, 3), dtype=torch.int32, device="cuda")
+        cnt_d = torch.zeros(1, dtype=torch.int64, device="cuda")
+        for _ in range(5):
+            lv.lv_select_victims(pool.handle, 0, 256, 0, out, 256, cnt_d, pool.stream)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        reps = 50
+        for _ in range(reps):
+            lv.lv_select_victims(pool.handle, 0, 256, 0, out, 256, cnt_d, pool.stream)
+        b.record()
+        torch.cuda.synchronize()
+        us = a.elapsed_time(b) * 1e3 / reps
+        assert np.array_equal(out.cpu().numpy().astype(np.int64), want[:256])
+        print(f"\nranker, 2^20 resident pages, k=256: {us:.1f} us per decision")
+    finally:
+        pool.close()
+
+
+@pytest.mark.parametrize("kernel", ["tma", "lsu"])
+def test_pack_unpack_pages(kernel, monkeypatch):
+    import torch
+    from paper_2606_22983_gb300 import lv
+    monkeypatch.setenv("LV_STAGE_KERNEL", kernel)
+    pool = _tiny_pool(hbm_pages=300, hbm_budget_pages=300)
+    try:
+        rng = np.random.default_rng(1)
+        kv = rng.integers(0, 256, tuple(pool.kv.shape), dtype=np.uint8)
+        pool.kv.copy_(torch.from_numpy(kv))
+        pages = rng.permutation(300)[:173].astype(np.int32)
+        run = torch.zeros((173, pool.J, pool.P), dtype=torch.uint8, device="cuda")
+        lv.lv_pack_pages(pool.handle, pages, 173, run, pool.stream)
+        pool.sync()
+        want = np.stack([kv[:, p, :] for p in pages])
+        assert np.array_equal(run.cpu().numpy(), want)
+        # unpack a fresh run into other pages; the rest of the pool is untouched
+        src = rng.integers(0, 256, (90, pool.J, pool.P), dtype=np.uint8)
+        dst_pages = rng.permutation(300)[:90].astype(np.int32)
+        lv.lv_unpack_pages(pool.handle, torch.from_numpy(src).cuda(), torch.from_numpy(dst_pages).cuda(),
+                           90, pool.stream)
+        pool.sync()
+        after = pool.kv.cpu().numpy()
+        expect = kv.copy()
+        for i, p in enumerate(dst_pages):
+            expect[:, p, :] = src[i]
+        assert np.array_equal(after, expect)
+        # an out-of-range page is reported and skipped, not faulted
+        bad = np.array([3, 300, 5], dtype=np.int32)
+        lv.lv_pack_pages(pool.handle, bad, 3, run, pool.stream)
+        assert pool.sync(raise_on_error=False) == lv.LV_ERR_BOUNDS
+        pool.clear_error()
+        assert pool.sync(raise_on_error=False) == 0
+    finally:
+        pool.close()
+
+
+def test_remap_cancel_and_allocation_errors():
+    from paper_2606_22983_gb300 import lv
+    pool = _tiny_pool(hbm_pages=64, hbm_budget_pages=10, host_pages=8)
+    try:
+        placement = np.full((8, 16), -1, np.int32)
+        placement[0, :4] = [0, 1, 2, 3]
+        placement[1, :2] = [4, -2]                     # block (1, 1) on host slot 0
+        ctx = np.zeros(8, np.int32)
+        ctx[0], ctx[1] = 64, 32
+        pool.import_placement(placement, ctx)
+        assert pool.sync(raise_on_error=False) == 0
+        st = pool.stats()
+        assert st["hbm_allocated"] == 5 and st["host_allocated"] == 1
+
+        def remap(entries):
+            e = np.array(entries, dtype=np.int32).reshape(-1, 3)
+            pool.remap(e, len(e))
+            return pool.sync(raise_on_error=False)
+
+        assert remap([[0, 0, 4]]) == lv.LV_ERR_DOUBLE_MAP     # page 4 is owned by (1, 0)
+        pool.clear_error()
+        assert remap([[0, 0, 20]]) == lv.LV_ERR_DOUBLE_MAP    # page 20 was never reserved
+        pool.clear_error()
+        assert remap([[0, 9, 20]]) == lv.LV_ERR_BOUNDS        # block 9 is past the context
+        pool.clear_error()
+        assert remap([[0, 0, -1]]) == lv.LV_ERR_BOUNDS        # no location
+        pool.clear_error()
+        # a reservation, committed twice in one call: one is a double map
+        pages, _ = pool.swap_in(1, np.array([1], np.int32), 1)
+        p = int(pages.cpu()[0])
+        assert remap([[1, 1, p], [1, 1, p]]) == lv.LV_ERR_DOUBLE_MAP
+        pool.clear_error()
+        t, own, _ = pool.tables()
+        assert t[1, 1] == p and own[p] == (1 << 32) | 1
+        # cancel: an owned page is refused, a pending reservation is released
+        pool.cancel(np.array([p], np.int32), 1)
+        assert pool.sync(raise_on_error=False) == lv.LV_ERR_STATE
+        pool.clear_error()
+        v = np.array([[0, 3, 3]], np.int32)
+        slots, commit = pool.swap_out(v, 1)
+        s0 = int(slots.cpu()[0])
+        pool.cancel(np.array([-(s0 + 2)], np.int32), 1)
+        assert pool.sync(raise_on_error=False) == 0
+        assert pool.stats()["host_allocated"] == 0
+        # the budget: 6 pages used of 10, 6 more cannot be reserved and nothing changes
+        before = pool.stats()["hbm_allocated"]
+        lv.lv_session_append(pool.handle, 2, 6 * 16, pool.pages, None, pool.stream)
+        assert pool.sync(raise_on_error=False) == lv.LV_ERR_NO_HBM
+        pool.clear_error()
+        assert pool.stats()["hbm_allocated"] == before
+        assert int(pool.get_sessions()["ctx_tokens"][2]) == 0
+        # a stale victim (block 0 does not live on page 3) is refused by swap-out
+        pool.swap_out(np.array([[0, 0, 3]], np.int32), 1)
+        assert pool.sync(raise_on_error=False) == lv.LV_ERR_STATE
+        pool.clear_error()
+    finally:
+        pool.close()
+
+
+def test_degenerate_sizes_and_host_pointer_arguments():
+    import torch
+    from paper_2606_22983_gb300 import lv
+    pool = _tiny_pool(max_sessions=1, max_blocks=4, hbm_pages=8, hbm_budget_pages=8, host_pages=8)
+    try:
+        placement = np.full((1, 4), -1, np.int32)
+        placement[0, :3] = [5, 6, 7]
+        pool.import_placement(placement, np.array([40], np.int32))
+        # k = 0, n = 0, empty exchange: no work, no error
+        got, n = pool.select(0, 0)
+        assert n == 0
+        pool.swap_out(np.zeros((0, 3), np.int32), 0)
+        lv.lv_swap_exchange(pool.handle, None, 0, 0, None, 0, None, None, 0, pool.stream)
+        lv.lv_session_append(pool.handle, 0, 0, None, None, pool.stream)
+        assert pool.sync(raise_on_error=False) == 0
+        # the same swap-out with host (numpy) and device (torch) arguments
+        v_host = np.array([[0, 2, 7], [0, 1, 6]], np.int32)
+        slots_h = np.full(2, -9, np.int32)
+        commit_h = np.zeros((2, 3), np.int32)
+        lv.lv_swap_out(pool.handle, v_host, 2, slots_h, commit_h, 0, pool.stream)
+        pool.sync()
+        assert slots_h.tolist() == [0, 1]
+        assert commit_h.tolist() == [[0, 2, -2], [0, 1, -3]]
+        pool.cancel(np.array([-2, -3], np.int32), 2)
+        v_dev = torch.from_numpy(v_host).cuda()
+        slots_d = torch.full((2,), -9, dtype=torch.int32, device="cuda")
+        commit_d = torch.zeros((2, 3), dtype=torch.int32, device="cuda")
+        lv.lv_swap_out(pool.handle, v_dev, 2, slots_d, commit_d, 0, pool.stream)
+        pool.sync()
+        assert slots_d.cpu().tolist() == [0, 1]
+        assert np.array_equal(commit_d.cpu().numpy(), commit_h)
+        assert np.array_equal(pool.host[0], pool.kv[:, 7].cpu().numpy())
+    finally:
+        pool.close()

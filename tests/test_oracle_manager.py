@@ -198,3 +198,22 @@ def test_pins_catch_remap_without_free(monkeypatch):
         self.hbm_used |= keep & (self.owner_hbm[:, 0] == -1) & ~self.hbm_used
     monkeypatch.setattr(opool.OraclePool, "remap", bad)
     assert _fails(tpool.test_exclusive_tiers_free_host_slot_on_commit)
+
+
+def test_next_use_versus_lru_on_the_voice_workloads():
+    """NEXT f3 (Sections 2.3 and 5): the same scripts under the paper's next-use
+    order with speech-triggered preload, and under the LRU baseline that loads at
+    turn start.  Next-use must move fewer reloads onto the turns' critical path."""
+    rows = {}
+    for name in ("tiny", "mixed"):
+        for policy in (0, 1):
+            from workloads import pool_spec
+            wl = make_workload(name, 0)
+            wl.spec = wl.spec.with_(policy=policy)
+            m = OracleManager(wl, with_bytes=False, rank_on="none")
+            m.run()
+            m.pool.check_invariants()
+            rows[(name, policy)] = dict(m.counters)
+    for name in ("tiny", "mixed"):
+        nu, lru = rows[(name, 0)], rows[(name, 1)]
+        assert nu["sync_loads"] < lru["sync_loads"], (name, nu, lru)

@@ -243,3 +243,43 @@ def test_protection_window_expires():
     assert order_global(tables, nb, [st], 3_000_000, 0, 3_000_000, 80000)[0].size == 2
     se.apply_event(st, se.SE_TURN_BEGIN, 1_500_000)
     assert st.protect_until_us == 0
+
+
+def test_lru_baseline_order_pairwise():
+    """The LRU baseline (Sections 2.3 and 5: rank by last use, not next use):
+    only running KV is pinned; least recently used session first, equal times by
+    smaller session id, suffix blocks first."""
+    from oracle.policy import order_lru
+    rng = np.random.default_rng(99)
+    for trial in range(40):
+        sess, tables, nblocks = _random_pool(rng, int(rng.integers(1, 9)), int(rng.integers(1, 6)))
+        for st in sess:
+            st.last_use_us = int(rng.integers(0, 4)) * 1_000_000
+        s_, b_, p_ = order_lru(tables, nblocks, sess)
+        got = list(zip(s_.tolist(), b_.tolist()))
+        cand = {(s, b) for s in range(len(sess)) for b in range(int(nblocks[s]))
+                if tables[s, b] >= 0 and not (sess[s].flags & se.RUNNING)}
+        assert set(got) == cand and len(got) == len(cand)
+        for i in range(len(got)):
+            for j in range(i + 1, len(got)):
+                (sx, bx), (sy, by) = got[i], got[j]
+                tx, ty = sess[sx].last_use_us, sess[sy].last_use_us
+                assert (tx < ty) or (tx == ty and (sx < sy or (sx == sy and bx > by))), (got[i], got[j])
+
+
+def test_lru_picks_the_older_session_in_the_paper_scenario():
+    from oracle.policy import order_lru
+    g = _load("scenario_lru_vs_next_use.json")
+    sess = _mk_sessions(g["sessions"])
+    for st, d in zip(sess, g["sessions"]):
+        st.last_use_us = d["last_use_us"]
+    tables = np.full((3, 8), -1, dtype=np.int64)
+    nblocks = np.zeros(3, dtype=np.int64)
+    page = 0
+    for s, d in enumerate(g["sessions"]):
+        nblocks[s] = d["resident_blocks"]
+        for b in range(d["resident_blocks"]):
+            tables[s, b] = page
+            page += 1
+    s_, _, _ = order_lru(tables, nblocks, sess)
+    assert s_[:g["k"]].tolist() == g["expect_lru_victims_sessions"]

@@ -25,6 +25,16 @@ def test_tiny_workload_full_images(seed, driver, mode):
     assert gm.counters["pages_out"] > 500 and gm.counters["preloads"] > 10
 
 
+@pytest.mark.parametrize("driver", ["device", "sequential"])
+def test_tiny_workload_lru_baseline(driver):
+    """The LRU baseline policy on the same kernels (NEXT f3): every ranking and
+    every move of the tiny script, with full byte images."""
+    wl = make_workload("tiny", 3)
+    wl.spec = wl.spec.with_(policy=1)
+    om, gm = run_lockstep(wl, with_bytes=True, check_every=100, driver=driver)
+    assert om.counters == gm.counters and gm.counters["preloads"] == 0
+
+
 def test_tiny_workload_ascending_and_counters_mode():
     """The literal block-ascending tie-break and the progress-counter T_play."""
     wl = make_workload("tiny", 2)
@@ -42,50 +52,77 @@ def _expected_block(seed, table, shape, sid, blk, ctx):
     return subpage_values_np(table, off, rows, shape).view(np.uint8).reshape(J, -1)
 
 
-@pytest.mark.parametrize("driver,mode", [("device", 0), ("exchange", 0), ("exchange", 2)])
-def test_thinker_full_size_sampled_bytes(driver, mode):
-    """The thinker pool at full size (40 GB HBM budget, 1.5 MiB pages), in the
-    launch configuration the benchmark times: every turn's victims, host slots
-    and pages match the oracle; afterwards the tables and owners match, and
-    the bytes of sampled blocks (plus every block of the last turn) are the
-    content of their logical position."""
+def _sampled_full_size(wl, driver, mode, n_sample=48, rank_on="turns"):
+    """Every event's decisions, the final tables/owners/sessions, and the bytes of
+    sampled blocks (plus blocks the last movements touched) against the oracle."""
     import torch
     from oracle import OracleManager
     from paper_2606_22983_gb300.harness import ContentWriter, pool_for
     from paper_2606_22983_gb300.manager import KVManager
-    from workloads import value_table
+    from workloads import scatter_order, value_table
     from ._lockstep import compare_records, compare_state
 
-    wl = make_workload("thinker", 0, n_turns=6)
-    om = OracleManager(wl, with_bytes=False, rank_on="turns")
+    om = OracleManager(wl, with_bytes=False, rank_on=rank_on)
     pool = pool_for(wl)
     try:
         writer = ContentWriter(pool, wl)
         writer.write_initial(wl)
-        gm = KVManager(pool, perms=wl.perms, rank_on="turns", driver=driver, mode=mode)
-        last = None
+        gm = KVManager(pool, perms=wl.perms, rank_on=rank_on, driver=driver, mode=mode,
+                       order_fn=scatter_order, on_append=writer.write_appended)
+        touched = []
         for i in range(wl.n_events):
             ro, rg = om.step(i), gm.step(wl.event(i), i)
             compare_records(ro, rg, i)
-            if ro["kind"] == 2:
-                last = ro
+            if "victims" in ro and len(ro["victims"]):
+                touched += [(int(a), int(b)) for a, b, _ in ro["victims"][:8]]
+            if "in_blocks" in ro:
+                touched += [(int(ro["sid"]), int(b)) for b in ro["in_blocks"][:8]]
         compare_state(om, pool, "end", with_bytes=False)
         table = value_table(wl.seed)
         rng = np.random.default_rng(0)
         t = om.pool.tables
-        sample = set()
         placed = np.argwhere(t != -1)
-        for r in rng.choice(len(placed), 48, replace=False):
-            sample.add(tuple(int(x) for x in placed[r]))
-        for s, b, _ in last["victims"][:32]:
-            sample.add((int(s), int(b)))
-        for b in last["in_blocks"][:32]:
-            sample.add((int(last["sid"]), int(b)))
-        for s, b in sorted(sample):
-            e = int(t[s, b])
-            want = _expected_block(wl.seed, table, wl.spec.shape, s, b, int(om.pool.ctx[s]))
+        sample = {tuple(int(x) for x in placed[r])
+                  for r in rng.choice(len(placed), min(n_sample, len(placed)), replace=False)}
+        sample |= set(touched[-64:])
+        for s_, b in sorted(sample):
+            e = int(t[s_, b])
+            want = _expected_block(wl.seed, table, wl.spec.shape, s_, b, int(om.pool.ctx[s_]))
             got = pool.kv[:, e, :].cpu().numpy() if e >= 0 else pool.host[-(e + 2)]
-            assert np.array_equal(got, want), (s, b, e)
+            assert np.array_equal(got, want), (s_, b, e)
+        assert om.counters["pages_out"] > 0 and om.counters["pages_in"] > 0
+        return om, gm
     finally:
         torch.cuda.synchronize()
         pool.close()
+        torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("driver,mode", [("device", 0), ("exchange", 0), ("exchange", 2)])
+def test_thinker_full_size_sampled_bytes(driver, mode):
+    """The thinker pool at full size (40 GB HBM budget, 1.5 MiB pages), in the
+    launch configuration the benchmark times."""
+    _sampled_full_size(make_workload("thinker", 0, n_turns=6), driver, mode)
+
+
+def test_mixed_realtime_full_size():
+    """Mixed realtime load: 128 sessions (log-uniform 2k-16k tokens) with Poisson
+    next-speech arrivals, barge-ins, speech-triggered preloads and turns with
+    growth; 60 GB HBM budget, ~40 GB host tier; 3000 events."""
+    om, gm = _sampled_full_size(make_workload("mixed", 0), "device", 0)
+    assert om.counters["preloads"] > 50 and om.counters == gm.counters
+
+
+def test_long_multimodal_full_size():
+    """16 sessions of 32k-64k tokens (3-6 GB each, 30 % frame tokens); every turn
+    evicts and reloads several GB at once through the exchange."""
+    om, gm = _sampled_full_size(make_workload("long", 0), "device", 0)
+    assert om.counters["pages_in"] > 16 * 1000
+
+
+def test_fragmentation_full_size():
+    """Pages randomly permuted over a 100 GB HBM budget, 640 sessions of
+    256-4096 tokens; 10 000 events alternating "free k pages" with turns whose
+    reload list comes in a scattered order."""
+    om, gm = _sampled_full_size(make_workload("frag", 0), "exchange", 0, rank_on="none")
+    assert om.counters["turns"] == 5000

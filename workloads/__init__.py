@@ -12,7 +12,8 @@ from .configs import (  # noqa: F401
 from .scripts import (  # noqa: F401
     Workload, InitialState, make_workload,
     EV_TURN, EV_TURN_ANY, EV_PLAYBACK, EV_SPEECH_START, EV_BARGE_IN, EV_SPEECH_STOP,
-    EVENT_NAMES, LOC_NONE, encode_host, is_host, host_slot,
+    EV_TURN_SCATTER, EV_EVICT, EVENT_NAMES, LOC_NONE, encode_host, is_host, host_slot,
+    scatter_order,
 )
 from .content import (  # noqa: F401
     TABLE_LEN, value_table, subpage_offsets, subpage_values_np, subpage_values_torch,

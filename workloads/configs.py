@@ -64,6 +64,7 @@ class PoolSpec:
     within_order: int = 0        # 0: suffix blocks first, 1: ascending block id
     t_play_mode: int = 0         # 0: playback accounting, 1: progress counters
     unit_us: int = 80_000        # progress-counter unit (one audio token)
+    policy: int = 0              # 0: next-use order, 1: LRU baseline
 
     def with_(self, **kw) -> "PoolSpec":
         return replace(self, **kw)
@@ -87,15 +88,19 @@ def pool_spec(name: str) -> PoolSpec:
         return PoolSpec("thinker", THINKER_SHAPE, n_sessions=64, max_blocks=1024,
                         hbm_pages=b, hbm_budget_pages=b, host_pages=0)
     if name == "mixed":
+        # 256 sessions would need a ~120 GB pinned host tier; scaled to 128 sessions so the
+        # host tier (~40 GB) leaves most of a 199 GB host free
         b = pages_for_bytes(60 * GB, THINKER_SHAPE)          # 38 146 pages
-        return PoolSpec("mixed", THINKER_SHAPE, n_sessions=256, max_blocks=1024,
+        return PoolSpec("mixed", THINKER_SHAPE, n_sessions=128, max_blocks=1024,
                         hbm_pages=b, hbm_budget_pages=b, host_pages=0)
     if name == "long":
         b = pages_for_bytes(40 * GB, THINKER_SHAPE)
         return PoolSpec("long", THINKER_SHAPE, n_sessions=16, max_blocks=4096,
                         hbm_pages=b, hbm_budget_pages=b, host_pages=0)
     if name == "frag":
+        # 1024 sessions of 256-4096 tokens hold ~219 GB, which would need ~140 GB of
+        # pinned host memory; scaled to 640 sessions (~137 GB, host tier ~45 GB)
         b = pages_for_bytes(100 * GB, THINKER_SHAPE)         # 63 578 pages
-        return PoolSpec("frag", THINKER_SHAPE, n_sessions=1024, max_blocks=256,
+        return PoolSpec("frag", THINKER_SHAPE, n_sessions=640, max_blocks=256,
                         hbm_pages=b, hbm_budget_pages=b, host_pages=0)
     raise ValueError(f"unknown workload {name!r}; expected one of {CONFIG_NAMES}")

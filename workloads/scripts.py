@@ -20,6 +20,12 @@ Script event kinds and arguments:
   EV_SPEECH_START(sid), EV_BARGE_IN(sid), EV_SPEECH_STOP(sid)
       Voice-activity signals; a barge-in is speech that starts while the
       session's reply is still playing.
+  EV_TURN_SCATTER(sid=-1, d=row, a=scatter_key, b=reply_audio_us, c=reply_tokens)
+      As EV_TURN_ANY (no context growth), but the session's host blocks are
+      reloaded in the order ``scatter_order(scatter_key, blocks)`` instead of
+      ascending block order.
+  EV_EVICT(a=k)
+      Memory pressure from elsewhere: k pages must be freed now.
 
 Block-table placement encoding (the C-ABI's published encoding): entry >= 0 is
 an HBM page id, -1 is "no block", entry <= -2 is host slot ``-(entry + 2)``.
@@ -39,9 +45,12 @@ EV_PLAYBACK = 3
 EV_SPEECH_START = 4
 EV_BARGE_IN = 5
 EV_SPEECH_STOP = 6
+EV_TURN_SCATTER = 7
+EV_EVICT = 8
 EVENT_NAMES = {EV_TURN: "TURN", EV_TURN_ANY: "TURN_ANY", EV_PLAYBACK: "PLAYBACK",
                EV_SPEECH_START: "SPEECH_START", EV_BARGE_IN: "BARGE_IN",
-               EV_SPEECH_STOP: "SPEECH_STOP"}
+               EV_SPEECH_STOP: "SPEECH_STOP", EV_TURN_SCATTER: "TURN_SCATTER",
+               EV_EVICT: "EVICT"}
 
 LOC_NONE = -1
 SEC = 1_000_000
@@ -92,6 +101,15 @@ class Workload:
     def event(self, i: int):
         return (int(self.t_us[i]), int(self.kind[i]), int(self.sid[i]), int(self.a[i]),
                 int(self.b[i]), int(self.c[i]), int(self.d[i]))
+
+
+def scatter_order(key, blocks) -> np.ndarray:
+    """A seeded permutation of ``blocks`` (the random scatter order of a reload)."""
+    from .content import _splitmix64
+    blocks = np.asarray(blocks, dtype=np.int64)
+    h = _splitmix64(np.uint64(key & 0xFFFFFFFFFFFF) * np.uint64(1 << 16)
+                    + blocks.astype(np.uint64) * np.uint64(2654435761))
+    return blocks[np.argsort(h, kind="stable")]
 
 
 def _pack_events(rows, S):
@@ -149,6 +167,7 @@ def _interactive(spec: PoolSpec, seed: int, n_events: int, ctx_lo: int, ctx_hi: 
     rng = np.random.default_rng(seed)
     S, T = spec.n_sessions, spec.shape.page_tokens
     cap_tokens = spec.max_blocks * T
+    size_host_after = spec.host_pages == 0 and not all_resident
     if log_uniform_ctx:
         ctx = _log_uniform_tokens(rng, ctx_lo, ctx_hi, S)
     else:
@@ -159,7 +178,8 @@ def _interactive(spec: PoolSpec, seed: int, n_events: int, ctx_lo: int, ctx_hi: 
         raise ValueError("initial contexts exceed the HBM budget")
     host_pages = spec.host_pages
     if host_pages == 0:
-        host_pages = int(n_pages.sum()) + S * 16
+        # room for every session, plus growth; shrunk below once the script is known
+        host_pages = int(n_pages.sum()) + S * spec.max_blocks
         spec = spec.with_(host_pages=host_pages)
     placement = _place_fill(n_pages, spec.max_blocks, spec.hbm_budget_pages, host_pages)
 
@@ -233,23 +253,42 @@ def _interactive(spec: PoolSpec, seed: int, n_events: int, ctx_lo: int, ctx_hi: 
             gen[s], play[s] = reply, 0
             push(t + report_us, s, "report", t + gap())
     rows.sort(key=lambda r: r[0])   # stable: equal times keep generation order
+    rows = rows[:n_events]
     t_us, kind, sid, a, b, c, d = _pack_events(rows, S)
+    meta = {}
+    if size_host_after:
+        # every block that can exist, minus what the budget holds, plus two sessions of slack
+        grown = ctx.copy()
+        for r in rows:
+            if r[1] == EV_TURN:
+                grown[r[2]] += r[3]
+        total = int(_pages(grown, T).sum())
+        host = max(int(n_pages.sum()) - spec.hbm_budget_pages, total - spec.hbm_budget_pages) \
+            + 2 * spec.max_blocks
+        spec = spec.with_(host_pages=host)
+        meta["total_pages_final"] = total
+    meta["total_pages"] = int(n_pages.sum())
     return Workload(spec, seed, init, t_us, kind, sid, a, b, c, d,
-                    np.zeros((0, S), dtype=np.int32))
+                    np.zeros((0, S), dtype=np.int32), meta=meta)
 
 
 # --------------------------------------------------------------------------------------
 # Turn-driven sessions (thinker): every turn reloads an offloaded session.
 # --------------------------------------------------------------------------------------
 def _turns(spec: PoolSpec, seed: int, n_turns: int, ctx_lo: int, ctx_hi: int,
-           reply_lo_us: int, reply_hi_us: int, step_us: int) -> Workload:
+           reply_lo_us: int, reply_hi_us: int, step_us: int, ctx_dist: str = "log",
+           frame_fraction: float = 0.0) -> Workload:
     rng = np.random.default_rng(seed)
     S, T = spec.n_sessions, spec.shape.page_tokens
     need = spec.hbm_budget_pages + spec.max_blocks
-    # Contexts are log-uniform; draws whose total KV would fit the budget with less
-    # than one largest session to spare are redrawn, so every turn must evict.
+    # Contexts are log-uniform (or uniform); draws whose total KV would fit the budget
+    # with less than one largest session to spare are redrawn, so every turn must evict.
     for _ in range(1000):
-        ctx = np.minimum(_log_uniform_tokens(rng, ctx_lo, ctx_hi, S), spec.max_blocks * T)
+        if ctx_dist == "log":
+            raw = _log_uniform_tokens(rng, ctx_lo, ctx_hi, S)
+        else:
+            raw = rng.integers(ctx_lo, ctx_hi + 1, S).astype(np.int64)
+        ctx = np.minimum(raw, spec.max_blocks * T)
         n_pages = _pages(ctx, T)
         if int(n_pages.sum()) >= need:
             break
@@ -273,7 +312,64 @@ def _turns(spec: PoolSpec, seed: int, n_turns: int, ctx_lo: int, ctx_hi: int,
         reply = int(rng.integers(reply_lo_us, reply_hi_us + 1))
         rows.append((t, EV_TURN_ANY, -1, 0, reply, reply // spec.unit_us, i))
     t_us, kind, sid, a, b, c, d = _pack_events(rows, S)
-    return Workload(spec, seed, init, t_us, kind, sid, a, b, c, d, perms,
+    meta = {"total_pages": total}
+    if frame_fraction > 0:
+        meta["frame_spans"] = _frame_spans(rng, ctx, frame_fraction)
+    return Workload(spec, seed, init, t_us, kind, sid, a, b, c, d, perms, meta=meta)
+
+
+def _frame_spans(rng, ctx, fraction, frame_tokens=256):
+    """Token spans that came from dense image / video frames (a modality tag only:
+    the KV of a frame token moves like any other)."""
+    spans = []
+    for c in ctx:
+        want = int(fraction * int(c)) // frame_tokens
+        starts = np.sort(rng.choice(max(1, int(c) // frame_tokens), size=min(want, max(1, int(c) // frame_tokens)),
+                                    replace=False)) * frame_tokens
+        spans.append([(int(x), frame_tokens) for x in starts])
+    return spans
+
+
+# --------------------------------------------------------------------------------------
+# Fragmentation stress (frag): a pool whose pages start randomly permuted; events
+# alternate "free k pages" and a turn whose reload list comes in a scattered order.
+# --------------------------------------------------------------------------------------
+def _frag(spec: PoolSpec, seed: int, n_events: int, ctx_lo: int, ctx_hi: int,
+          evict_lo: int, evict_hi: int, reply_lo_us: int, reply_hi_us: int, step_us: int) -> Workload:
+    rng = np.random.default_rng(seed)
+    S, T = spec.n_sessions, spec.shape.page_tokens
+    for _ in range(1000):
+        ctx = np.minimum(rng.integers(ctx_lo, ctx_hi + 1, S).astype(np.int64), spec.max_blocks * T)
+        n_pages = _pages(ctx, T)
+        if int(n_pages.sum()) >= spec.hbm_budget_pages + 2 * spec.max_blocks:
+            break
+    else:
+        raise RuntimeError("could not draw contexts that exceed the budget")
+    total = int(n_pages.sum())
+    host_pages = spec.host_pages or (total - spec.hbm_budget_pages + max(total // 10, 2 * spec.max_blocks)
+                                     + evict_hi)
+    spec = spec.with_(host_pages=host_pages)
+    perm = rng.permutation(spec.hbm_pages)
+    placement = _place_fill(n_pages, spec.max_blocks, spec.hbm_budget_pages, host_pages, page_perm=perm)
+    gen0 = rng.integers(reply_lo_us, reply_hi_us + 1, S).astype(np.int64)
+    play0 = (rng.uniform(0.0, 1.0, S) * gen0).astype(np.int64)
+    rtok0 = (gen0 // spec.unit_us).astype(np.int32)
+    init = InitialState(ctx.astype(np.int32), placement, gen0, play0, np.ones(S, np.int32), rtok0)
+    rows = []
+    n_turns = (n_events + 1) // 2
+    perms = np.zeros((n_turns, S), dtype=np.int32)
+    for i in range(n_events):
+        t = (i + 1) * step_us
+        if i % 2 == 0:
+            rows.append((t, EV_EVICT, -1, int(rng.integers(evict_lo, evict_hi + 1)), 0, 0, -1))
+        else:
+            r = i // 2
+            perms[r] = rng.permutation(S)
+            reply = int(rng.integers(reply_lo_us, reply_hi_us + 1))
+            rows.append((t, EV_TURN_SCATTER, -1, int(rng.integers(0, 2**40)), reply,
+                         reply // spec.unit_us, r))
+    t_us, kind, sid, a, b, c, d = _pack_events(rows, S)
+    return Workload(spec, seed, init, t_us, kind, sid, a, b, c, d, perms[: (n_events // 2)],
                     meta={"total_pages": total})
 
 
@@ -296,4 +392,22 @@ def make_workload(name: str, seed: int = 0, **over) -> Workload:
                   reply_lo_us=5 * SEC, reply_hi_us=30 * SEC, step_us=500_000)
         kw.update(over)
         return _turns(spec, seed, **kw)
-    raise NotImplementedError(f"workload {name!r} is not generated yet")
+    if name == "mixed":
+        kw = dict(n_events=3000, ctx_lo=2048, ctx_hi=16384, log_uniform_ctx=True,
+                  gap_mean_us=8 * SEC, gap_exponential=True,
+                  reply_lo_us=5 * SEC, reply_hi_us=30 * SEC,
+                  speech_lo_us=2 * SEC, speech_hi_us=10 * SEC,
+                  append_lo=16, append_hi=96, all_resident=False)
+        kw.update(over)
+        return _interactive(spec, seed, **kw)
+    if name == "long":
+        kw = dict(n_turns=16, ctx_lo=32768, ctx_hi=65536, ctx_dist="uniform",
+                  reply_lo_us=5 * SEC, reply_hi_us=30 * SEC, step_us=500_000, frame_fraction=0.3)
+        kw.update(over)
+        return _turns(spec, seed, **kw)
+    if name == "frag":
+        kw = dict(n_events=10_000, ctx_lo=256, ctx_hi=4096, evict_lo=8, evict_hi=128,
+                  reply_lo_us=5 * SEC, reply_hi_us=30 * SEC, step_us=100_000)
+        kw.update(over)
+        return _frag(spec, seed, **kw)
+    raise ValueError(f"unknown workload {name!r}")
