@@ -336,6 +336,7 @@ def ours(args, torch):
     if line is not None and args.micro:
         micro = kernel_micro(torch, pool, args.seed)
         line["ranker"] = micro.pop("ranker")
+        line["scheduler"] = micro.pop("scheduler")
         line["hbm_kernels"] = micro
     pool.close()
     if line is not None and args.cpu_baseline:
@@ -381,6 +382,33 @@ def kernel_micro(torch, pool, seed=0):
         out[name] = {"pages": n, "bytes_per_launch": 2 * payload, "avg_ms": round(ms, 4),
                      "achieved_gbs": round(gbs, 1), "peak_gbs": HBM_PEAK, "frac": round(gbs / HBM_PEAK, 3)}
     del run
+    # one urgency-scheduling round over 4096 ready requests (Algorithm 1)
+    rng = np.random.default_rng(seed)
+    R = lv.LV_SCHED_MAX_REQUESTS
+    reqs = np.zeros(R, dtype=lv.REQUEST_DTYPE)
+    reqs["id"] = np.arange(R)
+    reqs["started"] = rng.random(R) < 0.7
+    reqs["play_buffer_us"] = rng.integers(0, 8, R) * 700_000
+    reqs["ready_age_us"] = rng.integers(0, 10_000_000, R)
+    reqs["kv_pages"] = rng.integers(0, 2048, R)
+    reqs["tokens"] = rng.integers(1, 512, R)
+    reqs["kv_needed"] = rng.integers(0, 64, R)
+    q = lv.lv_sched_params(p_safe_us=2_000_000, alpha=4, beta=1, occupied=30_000, allocatable=40_000,
+                           token_budget=8192, kv_budget=4096)
+    reqs_d = torch.from_numpy(reqs.view(np.uint8).copy()).to(pool.device)
+    order = torch.empty(R, dtype=torch.int32, device=pool.device)
+    nb = torch.empty(1, dtype=torch.int32, device=pool.device)
+    for _ in range(5):
+        lv.lv_schedule(pool.handle, q, reqs_d, R, order, nb, pool.stream)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(50):
+        lv.lv_schedule(pool.handle, q, reqs_d, R, order, nb, pool.stream)
+    b.record()
+    torch.cuda.synchronize()
+    out["scheduler"] = {"ready_requests": R, "us_per_round": round(a.elapsed_time(b) * 1e3 / 50, 2),
+                        "admitted": int(nb.item())}
     # a metadata-sized pool: 1024 sessions x 1024 resident blocks = 2^20 pages
     S = B = 1024
     N = S * B

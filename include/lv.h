@@ -92,7 +92,8 @@ enum {
   LV_EV_SPEECH_START = 4,
   LV_EV_BARGE_IN = 5,      /* speech while the reply plays: unplayed audio discarded */
   LV_EV_SPEECH_STOP = 6,   /* the user input is complete */
-  LV_EV_PRELOADED = 7      /* a preload completed at t_us: protect the warmed KV */
+  LV_EV_PRELOADED = 7,     /* a preload completed at t_us: protect the warmed KV */
+  LV_EV_UNPROTECT = 8      /* the warmed KV's protection ends now (the cap, Section 5.2) */
 };
 
 typedef struct lv_pool_desc {
@@ -220,7 +221,7 @@ lv_status lv_session_get(lv_pool* pool, lv_session_state* out, int32_t first, in
    completion time, sets IMMEDIATE.  SPEECH_STOP clears IMMEDIATE and, when the
    reply had completed, folds x = t - t_done_us into the reply-interval average
    (first sample: ema = x; later: ema = floor((3*ema + x) / 4)).  PRELOADED
-   sets protect_until_us = t + protect_us.  Device-detected: LV_ERR_BOUNDS for an
+   sets protect_until_us = t + protect_us; UNPROTECT sets it to 0.  Device-detected: LV_ERR_BOUNDS for an
    unknown kind or session id (that event is skipped). */
 lv_status lv_session_events(lv_pool* pool, const lv_event* events, int64_t n, lv_stream stream);
 
@@ -382,9 +383,10 @@ lv_status lv_session_blocks(lv_pool* pool, int32_t sid, int32_t where, int32_t* 
                             int64_t* count_out, lv_stream stream);
 
 /* Copies the block tables (int32 [S][max_blocks]) and, if not NULL, the owner
-   tables (int64 [hbm_pages] and [host_pages]: sid << 32 | blk, or -1). */
-lv_status lv_read_tables(lv_pool* pool, int32_t* tables, int64_t* hbm_owner,
-                         int64_t* host_owner, lv_stream stream);
+   tables (int32 [hbm_pages] and [host_pages]: sid << 16 | blk for an owned
+   location, -1 free, -2 reserved by a swap and not yet committed). */
+lv_status lv_read_tables(lv_pool* pool, int32_t* tables, int32_t* hbm_owner,
+                         int32_t* host_owner, lv_stream stream);
 
 /* ------------------------------------------- ranking without allocation */
 
@@ -433,6 +435,44 @@ lv_status lv_select_victims_noalloc(const lv_rank_params* params, const lv_sessi
                                     const int32_t* tables, int64_t now_us, int64_t k,
                                     lv_victim* out, int64_t capacity, int64_t* count_out,
                                     lv_stream stream);
+
+/* --------------------------------------------------- request scheduling */
+
+/* One ready request of a stage for lv_schedule (48 bytes). */
+typedef struct lv_request {
+  int32_t id;                  /* caller's request id (echoed in the order) */
+  int32_t started;             /* 1 once its first playable audio went out */
+  int64_t play_buffer_us;      /* P_i: audio the client holds, 0..2^40 */
+  int64_t ready_age_us;        /* A_i: time since it became ready, 0..2^62 */
+  int64_t kv_pages;            /* K_i: GPU KV it occupies, 0..2^24 pages */
+  int64_t tokens;              /* token budget it consumes if admitted (>= 0) */
+  int64_t kv_needed;           /* KV blocks it needs if admitted (>= 0) */
+} lv_request;
+
+typedef struct lv_sched_params {
+  int64_t p_safe_us;           /* P_safe, 1..2^32 */
+  int64_t alpha, beta;         /* Eq. 1 weights, 0..2^16 */
+  int64_t occupied;            /* occupied GPU KV of the stage, 0..2^32 */
+  int64_t allocatable;         /* allocatable GPU KV of the stage, 1..2^32 */
+  int64_t token_budget;        /* round budgets M_s */
+  int64_t kv_budget;
+} lv_sched_params;
+
+#define LV_SCHED_MAX_REQUESTS 4096
+
+/* Section 4.1 (urgency classes, Eqs. 1-3) and Section 4.2 (Algorithm 1): one
+   scheduling round over n ready requests (reqs, lv_request [n]).  Class U0
+   (started, P_i <= P_safe) by P_i ascending; U1 (not started) by A_i
+   descending; U2 (started, P_i > P_safe) by U_i = beta*K_i*R_occ -
+   alpha*max(0, P_i - P_safe)/P_safe descending, R_occ = occupied/allocatable;
+   ties keep the ready set's order.  order_out (int32 [n]) receives the request
+   ids in priority order U0-U1-U2; *batch_out (int32) the length of the
+   admitted prefix: admission stops at the first request whose tokens or KV
+   blocks exceed what is left of the round budgets.  Runs on one CTA with
+   exact integer arithmetic.  n is 0..LV_SCHED_MAX_REQUESTS.  Device-detected:
+   LV_ERR_BOUNDS for a field outside its range (it is clamped). */
+lv_status lv_schedule(lv_pool* pool, const lv_sched_params* params, const lv_request* reqs, int32_t n,
+                      int32_t* order_out, int32_t* batch_out, lv_stream stream);
 
 /* ------------------------------------------------------------- status */
 

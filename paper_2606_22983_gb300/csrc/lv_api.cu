@@ -396,8 +396,8 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       cudaMemsetAsync(d.sess, 0, d.S * sizeof(lv_session_state), s) != cudaSuccess ||
       cudaMemsetAsync(d.table, 0xff, tb * sizeof(int32_t), s) != cudaSuccess ||
       cudaMemsetAsync(d.mark, 0, tb * sizeof(int32_t), s) != cudaSuccess ||
-      cudaMemsetAsync(d.own_hbm, 0xff, (size_t)d.hbm_pages * 8, s) != cudaSuccess ||
-      cudaMemsetAsync(d.own_host, 0xff, (size_t)(d.host_pages ? d.host_pages : 1) * 8, s) != cudaSuccess ||
+      cudaMemsetAsync(d.own_hbm, 0xff, (size_t)d.hbm_pages * 4, s) != cudaSuccess ||
+      cudaMemsetAsync(d.own_host, 0xff, (size_t)(d.host_pages ? d.host_pages : 1) * 4, s) != cudaSuccess ||
       cudaMemsetAsync(d.bits_hbm, 0, wh * 4, s) != cudaSuccess ||
       cudaMemsetAsync(d.bits_host, 0, (wo ? wo : 1) * 4, s) != cudaSuccess ||
       cudaMemsetAsync(d.ctl, 0, lv::C_N * sizeof(long long), s) != cudaSuccess ||
@@ -473,8 +473,8 @@ lv_status lv_pool_import(lv_pool* pool, const int32_t* placement, const int32_t*
     lv_status r;
     if ((r = st.in(placement, (size_t)d.S * d.maxB * 4, &pl)) != LV_OK) return r;
     if ((r = st.in(ctx_tokens, (size_t)d.S * 4, &cx)) != LV_OK) return r;
-    LV_TRY(cudaMemsetAsync(d.own_hbm, 0xff, (size_t)d.hbm_pages * 8, s));
-    if (d.host_pages) LV_TRY(cudaMemsetAsync(d.own_host, 0xff, (size_t)d.host_pages * 8, s));
+    LV_TRY(cudaMemsetAsync(d.own_hbm, 0xff, (size_t)d.hbm_pages * 4, s));
+    if (d.host_pages) LV_TRY(cudaMemsetAsync(d.own_host, 0xff, (size_t)d.host_pages * 4, s));
     LV_TRY(cudaMemsetAsync(d.bits_hbm, 0, (size_t)((d.hbm_pages + 31) / 32) * 4, s));
     if (d.host_pages) LV_TRY(cudaMemsetAsync(d.bits_host, 0, (size_t)((d.host_pages + 31) / 32) * 4, s));
     LV_TRY(cudaMemsetAsync(d.ctl, 0, 2 * sizeof(long long), s));   // allocation counts
@@ -768,6 +768,36 @@ lv_status lv_unpack_pages(lv_pool* pool, const void* src, const int32_t* pages, 
 
 void* lv_pool_host_device_ptr(lv_pool* pool) { return pool ? pool->d.host : nullptr; }
 
+lv_status lv_schedule(lv_pool* pool, const lv_sched_params* q, const lv_request* reqs, int32_t n,
+                      int32_t* order_out, int32_t* batch_out, lv_stream stream) {
+  if (!pool || !q || n < 0 || n > LV_SCHED_MAX_REQUESTS || !batch_out || (n > 0 && (!reqs || !order_out)))
+    return LV_ERR_INVALID;
+  if (q->p_safe_us < 1 || q->p_safe_us > (1ll << 32) || q->alpha < 0 || q->alpha > (1 << 16) ||
+      q->beta < 0 || q->beta > (1 << 16) || q->occupied < 0 || q->occupied > (1ll << 32) ||
+      q->allocatable < 1 || q->allocatable > (1ll << 32))
+    return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  try {
+    Staging st(pool, s);
+    const void* rin = nullptr;
+    void *odev = nullptr, *bdev = nullptr;
+    lv_status r;
+    if ((r = st.in(reqs, (size_t)n * sizeof(lv_request), &rin)) != LV_OK) return r;
+    if ((r = st.out(order_out, (size_t)n * 4, &odev, true)) != LV_OK) return r;
+    if ((r = st.out(batch_out, 4, &bdev, true)) != LV_OK) return r;
+    if (n == 0) {
+      LV_TRY(cudaMemsetAsync(bdev, 0, 4, s));
+      return st.finish();
+    }
+    LV_TRY(lv::launch_schedule(*q, static_cast<const lv_request*>(rin), n, static_cast<int32_t*>(odev),
+                               static_cast<int32_t*>(bdev), pool->d.ctl, s));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
 lv_status lv_remap(lv_pool* pool, const lv_remap_entry* entries, int64_t n, lv_stream stream) {
   if (!pool || n < 0 || (n > 0 && !entries)) return LV_ERR_INVALID;
   if (n == 0) return LV_OK;
@@ -861,7 +891,7 @@ lv_status lv_session_blocks(lv_pool* pool, int32_t sid, int32_t where, int32_t* 
   }
 }
 
-lv_status lv_read_tables(lv_pool* pool, int32_t* tables, int64_t* hbm_owner, int64_t* host_owner,
+lv_status lv_read_tables(lv_pool* pool, int32_t* tables, int32_t* hbm_owner, int32_t* host_owner,
                          lv_stream stream) {
   if (!pool) return LV_ERR_INVALID;
   DeviceGuard g(pool->device);
@@ -870,9 +900,9 @@ lv_status lv_read_tables(lv_pool* pool, int32_t* tables, int64_t* hbm_owner, int
   if (tables)
     LV_TRY(cudaMemcpyAsync(tables, d.table, (size_t)d.S * d.maxB * 4, cudaMemcpyDefault, s));
   if (hbm_owner)
-    LV_TRY(cudaMemcpyAsync(hbm_owner, d.own_hbm, (size_t)d.hbm_pages * 8, cudaMemcpyDefault, s));
+    LV_TRY(cudaMemcpyAsync(hbm_owner, d.own_hbm, (size_t)d.hbm_pages * 4, cudaMemcpyDefault, s));
   if (host_owner && d.host_pages)
-    LV_TRY(cudaMemcpyAsync(host_owner, d.own_host, (size_t)d.host_pages * 8, cudaMemcpyDefault, s));
+    LV_TRY(cudaMemcpyAsync(host_owner, d.own_host, (size_t)d.host_pages * 4, cudaMemcpyDefault, s));
   return LV_OK;
 }
 

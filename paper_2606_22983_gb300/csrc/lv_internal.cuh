@@ -8,7 +8,9 @@
 
 namespace lv {
 
-constexpr unsigned long long kOwnerNone = ~0ull;
+// Owner words: the (sid << 16 | blk) that owns a page or slot, or one of two states.
+constexpr uint32_t kOwnerNone = 0xFFFFFFFFu;       // free
+constexpr uint32_t kOwnerReserved = 0xFFFFFFFEu;   // reserved by a swap, not yet committed
 constexpr long long kKeyMax = 0xFFFFFFFFll;   // T_next is clamped to 32 bits (microseconds)
 
 // Layout of the per-pool int64 control block in device memory.
@@ -51,8 +53,8 @@ struct DevPool {
   lv_session_state* sess; // [S]
   int32_t* table;         // [S][maxB]
   int32_t* mark;          // [S][maxB] epoch of the last remap that touched the block
-  unsigned long long* own_hbm;   // [hbm_pages] sid << 32 | blk, or kOwnerNone
-  unsigned long long* own_host;  // [host_pages]
+  uint32_t* own_hbm;      // [hbm_pages] owner word (kOwnerNone / kOwnerReserved / sid << 16 | blk)
+  uint32_t* own_host;     // [host_pages]
   uint32_t* bits_hbm;     // allocation bitmap, 1 = reserved or owned
   uint32_t* bits_host;
   long long* ctl;         // [C_N]
@@ -65,8 +67,8 @@ struct DevPool {
   unsigned long long* page_tag;  // [hbm_pages] epoch << 32 | victim index (| paired bit)
 };
 
-__host__ __device__ inline unsigned long long owner_key(int32_t sid, int32_t blk) {
-  return ((unsigned long long)(uint32_t)sid << 32) | (uint32_t)blk;
+__host__ __device__ inline uint32_t owner_key(int32_t sid, int32_t blk) {
+  return ((uint32_t)sid << 16) | ((uint32_t)blk & 0xFFFFu);   // sid < 4096, blk < 65536
 }
 
 // Optional CUDA events recorded around a copy kernel launch.
@@ -137,6 +139,9 @@ cudaError_t launch_stage(const DevPool& p, bool pack, const int4* tasks, int64_t
 cudaError_t launch_tasks_pages(const DevPool& p, const int32_t* pages, int64_t n, bool pack,
                                int4* tasks, cudaStream_t s);
 cudaError_t configure_stage_kernels(const DevPool& p);
+// lv_sched.cu
+cudaError_t launch_schedule(const lv_sched_params& q, const lv_request* reqs, int n, int32_t* order,
+                            int32_t* batch, long long* ctl, cudaStream_t s);
 cudaError_t configure_kernels();   // once per device, before the first launch
 
 }  // namespace lv

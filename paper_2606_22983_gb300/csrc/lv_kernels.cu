@@ -119,7 +119,7 @@ __global__ void k_import(DevPool p, const int32_t* __restrict__ placement,
       if (e != -1) set_error(p.ctl, LV_ERR_BOUNDS, idx);
       continue;
     }
-    const unsigned long long key = owner_key(s, b);
+    const uint32_t key = owner_key(s, b);
     if (e >= 0) {
       if (e >= p.hbm_pages) { set_error(p.ctl, LV_ERR_BOUNDS, idx); continue; }
       if (atomicCAS(&p.own_hbm[e], kOwnerNone, key) != kOwnerNone) {
@@ -164,7 +164,7 @@ __global__ void k_events(DevPool p, const lv_event* __restrict__ ev, long long n
   const int s = blockIdx.x * blockDim.x + threadIdx.x;
   if (s == 0) {
     for (long long e = 0; e < n; ++e) {
-      if (ev[e].kind < LV_EV_TURN_BEGIN || ev[e].kind > LV_EV_PRELOADED || ev[e].sid < 0 ||
+      if (ev[e].kind < LV_EV_TURN_BEGIN || ev[e].kind > LV_EV_UNPROTECT || ev[e].sid < 0 ||
           ev[e].sid >= p.S) {
         set_error(p.ctl, LV_ERR_BOUNDS, e);
       }
@@ -225,6 +225,9 @@ __global__ void k_events(DevPool p, const lv_event* __restrict__ ev, long long n
         break;
       case LV_EV_PRELOADED:
         st.protect_until_us = x.t_us + p.protect_us;
+        break;
+      case LV_EV_UNPROTECT:
+        st.protect_until_us = 0;
         break;
       default:
         break;   // reported above
@@ -409,6 +412,9 @@ k_alloc(DevPool p, bool hbm, long long n, int32_t* __restrict__ out) {
     return;
   }
   block_alloc_lowest<kAllocThreads>(bits, nbits, n, out);
+  __syncthreads();
+  uint32_t* own = hbm ? p.own_hbm : p.own_host;
+  for (long long i = threadIdx.x; i < n; i += kAllocThreads) own[out[i]] = kOwnerReserved;
 }
 
 // ------------------------------------------------------------------ copy
@@ -571,7 +577,7 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
   const unsigned long long tag = (unsigned long long)(uint32_t)epoch << 32;
   for (long long i = threadIdx.x; i < n_out; i += kPlanThreads) {
     const lv_victim x = v[i];
-    const unsigned long long key = owner_key(x.sid, x.blk);
+    const uint32_t key = owner_key(x.sid, x.blk);
     p.table[(size_t)x.sid * p.maxB + x.blk] = -(slots[i] + 2);
     p.own_host[slots[i]] = key;
     p.own_hbm[x.page] = kOwnerNone;
@@ -907,10 +913,6 @@ __global__ void k_tasks_pages(DevPool p, const int32_t* __restrict__ pages, long
 }
 
 // ---------------------------------------------------------------- commit
-__device__ __forceinline__ bool bit_is_set(const uint32_t* bits, long long i) {
-  return (bits[i >> 5] >> (i & 31)) & 1u;
-}
-
 constexpr int kRemapThreads = 256;
 
 // One thread per entry.  The allocation counts and the commit counter change
@@ -929,18 +931,16 @@ k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t ep
       ti = (size_t)x.sid * p.maxB + x.blk;
       if (atomicExch(&p.mark[ti], epoch) == epoch) err = LV_ERR_DOUBLE_MAP;   // same block twice
     }
-    const unsigned long long key = err ? 0ull : owner_key(x.sid, x.blk);
+    const uint32_t key = err ? 0u : owner_key(x.sid, x.blk);
     if (!err) {
+      // the new location must be a reservation nobody owns yet: one CAS checks and takes it
       if (x.loc >= 0) {
         if (x.loc >= p.hbm_pages) err = LV_ERR_BOUNDS;
-        else if (!bit_is_set(p.bits_hbm, x.loc) ||
-                 atomicCAS(&p.own_hbm[x.loc], kOwnerNone, key) != kOwnerNone)
-          err = LV_ERR_DOUBLE_MAP;
+        else if (atomicCAS(&p.own_hbm[x.loc], kOwnerReserved, key) != kOwnerReserved) err = LV_ERR_DOUBLE_MAP;
       } else if (x.loc <= -2) {
         const long long h = -(long long)x.loc - 2;
         if (h >= p.host_pages) err = LV_ERR_BOUNDS;
-        else if (!bit_is_set(p.bits_host, h) || atomicCAS(&p.own_host[h], kOwnerNone, key) != kOwnerNone)
-          err = LV_ERR_DOUBLE_MAP;
+        else if (atomicCAS(&p.own_host[h], kOwnerReserved, key) != kOwnerReserved) err = LV_ERR_DOUBLE_MAP;
       } else {
         err = LV_ERR_BOUNDS;
       }
@@ -950,13 +950,16 @@ k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t ep
     } else {
       const int32_t old = p.table[ti];
       p.table[ti] = x.loc;
+      // the old location belongs to this block alone (one entry per block per call)
       if (old >= 0 && old < p.hbm_pages) {
-        if (atomicCAS(&p.own_hbm[old], key, kOwnerNone) != key) set_error(p.ctl, LV_ERR_STATE, i);
+        if (p.own_hbm[old] != key) set_error(p.ctl, LV_ERR_STATE, i);
+        p.own_hbm[old] = kOwnerNone;
         atomicAnd(&p.bits_hbm[old >> 5], ~(1u << (old & 31)));
         freed_hbm = true;
       } else if (old <= -2 && (-(long long)old - 2) < p.host_pages) {
         const long long h = -(long long)old - 2;
-        if (atomicCAS(&p.own_host[h], key, kOwnerNone) != key) set_error(p.ctl, LV_ERR_STATE, i);
+        if (p.own_host[h] != key) set_error(p.ctl, LV_ERR_STATE, i);
+        p.own_host[h] = kOwnerNone;
         atomicAnd(&p.bits_host[h >> 5], ~(1u << (h & 31)));
         freed_host = true;
       }
@@ -978,7 +981,7 @@ __global__ void k_cancel(DevPool p, const int32_t* __restrict__ locs, long long 
   if (i >= n) return;
   const int32_t loc = locs[i];
   uint32_t* bits;
-  unsigned long long* own;
+  uint32_t* own;
   long long idx;
   int which;
   if (loc >= 0 && loc < p.hbm_pages) {
@@ -989,10 +992,13 @@ __global__ void k_cancel(DevPool p, const int32_t* __restrict__ locs, long long 
     set_error(p.ctl, LV_ERR_BOUNDS, i);
     return;
   }
-  if (own[idx] != kOwnerNone) { set_error(p.ctl, LV_ERR_STATE, i); return; }
+  // only a pending reservation can be released
+  if (atomicCAS(&own[idx], kOwnerReserved, kOwnerNone) != kOwnerReserved) {
+    set_error(p.ctl, LV_ERR_STATE, i);
+    return;
+  }
   const uint32_t m = 1u << (idx & 31);
-  const uint32_t before = atomicAnd(&bits[idx >> 5], ~m);
-  if (!(before & m)) { set_error(p.ctl, LV_ERR_STATE, i); return; }
+  atomicAnd(&bits[idx >> 5], ~m);
   atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[which]), (unsigned long long)-1ll);
   atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_CANCELS]), 1ull);
 }

@@ -31,7 +31,7 @@ LV_SELECT_FALLBACK = 1
 LV_POLICY_NEXT_USE, LV_POLICY_LRU = 0, 1
 LV_RUNNING, LV_IMMEDIATE, LV_RESP_OPEN, LV_DONE_VALID = 1, 2, 4, 8
 (LV_EV_TURN_BEGIN, LV_EV_TURN_END, LV_EV_PLAYBACK, LV_EV_SPEECH_START, LV_EV_BARGE_IN,
- LV_EV_SPEECH_STOP, LV_EV_PRELOADED) = 1, 2, 3, 4, 5, 6, 7
+ LV_EV_SPEECH_STOP, LV_EV_PRELOADED, LV_EV_UNPROTECT) = 1, 2, 3, 4, 5, 6, 7, 8
 
 
 class LvError(RuntimeError):
@@ -81,6 +81,15 @@ class lv_rank_params(ctypes.Structure):
                 ("reply_prior_us", ctypes.c_int64), ("unit_us", ctypes.c_int64)]
 
 
+class lv_sched_params(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int64) for n in ("p_safe_us", "alpha", "beta", "occupied",
+                                               "allocatable", "token_budget", "kv_budget")]
+
+
+REQUEST_DTYPE = np.dtype([("id", "<i4"), ("started", "<i4"), ("play_buffer_us", "<i8"),
+                          ("ready_age_us", "<i8"), ("kv_pages", "<i8"), ("tokens", "<i8"),
+                          ("kv_needed", "<i8")])
+LV_SCHED_MAX_REQUESTS = 4096
 LV_NOALLOC_MAX_SESSIONS = 4096
 LV_RESIDENT_PRELOAD = 1
 LV_RESIDENT_DONE, LV_RESIDENT_SKIPPED, LV_RESIDENT_NOTHING, LV_RESIDENT_FAILED = 0, 1, 2, 3
@@ -119,6 +128,7 @@ def _load():
         "lv_make_resident": [vp, i32, i64, i32, u32, i64, vp, vp, vp, vp, vp, vp, vp],
         "lv_timing_enable": [vp, i32],
         "lv_pack_pages": [vp, vp, i64, vp, vp],
+        "lv_schedule": [vp, ctypes.POINTER(lv_sched_params), vp, i32, vp, vp, vp],
         "lv_unpack_pages": [vp, vp, vp, i64, vp],
         "lv_timing_read": [vp, ctypes.POINTER(lv_kernel_timing), i32],
         "lv_remap": [vp, vp, i64, vp],
@@ -156,7 +166,7 @@ EXPORTED = ("lv_pool_create", "lv_pool_destroy", "lv_pool_host_ptr", "lv_pool_im
             "lv_session_counts", "lv_session_blocks", "lv_read_tables", "lv_sync",
             "lv_get_stats", "lv_clear_error", "lv_status_str", "lv_version",
             "lv_select_victims_noalloc", "lv_timing_enable", "lv_timing_read", "lv_pack_pages",
-            "lv_unpack_pages", "lv_pool_host_device_ptr")
+            "lv_unpack_pages", "lv_pool_host_device_ptr", "lv_schedule")
 
 
 def lib():
@@ -331,6 +341,11 @@ def lv_timing_read(pool, reset=False) -> dict:
     return {TIMING_NAMES[i]: {"launches": int(arr[i].launches), "total_ms": arr[i].total_ms,
                               "min_ms": arr[i].min_ms, "max_ms": arr[i].max_ms}
             for i in range(LV_TIMING_KINDS)}
+
+
+def lv_schedule(pool, params: lv_sched_params, reqs, n, order_out, batch_out, stream=None):
+    _check(_lib.lv_schedule(pool, ctypes.byref(params), ptr(reqs), n, ptr(order_out), ptr(batch_out),
+                            stream_handle(stream)), "lv_schedule")
 
 
 def lv_status_str(status: int) -> str:

@@ -180,8 +180,8 @@ class KVPool:
 
     def tables(self):
         t = np.zeros((self.S, self.max_blocks), dtype=np.int32)
-        oh = np.zeros(self.hbm_pages, dtype=np.int64)
-        oo = np.zeros(max(self.host_pages, 1), dtype=np.int64)
+        oh = np.zeros(self.hbm_pages, dtype=np.int32)
+        oo = np.zeros(max(self.host_pages, 1), dtype=np.int32)
         lv.lv_read_tables(self.handle, t, oh, oo if self.host_pages else None, self.stream)
         self.sync()
         return t, oh, oo[:self.host_pages]

@@ -30,16 +30,18 @@ def compare_records(ro, rg, where):
         assert a.shape == b.shape and np.array_equal(a, b), (where, key, a, b)
 
 
-def owners_encoded(owner_pairs):
+def owners_encoded(owner_pairs, used):
+    """The C ABI's owner words: sid << 16 | blk when owned, -2 when reserved by a
+    swap and not yet committed, -1 when free."""
     sid, blk = owner_pairs[:, 0], owner_pairs[:, 1]
-    return np.where(sid < 0, -1, (sid << 32) | blk)
+    return np.where(sid >= 0, (sid << 16) | blk, np.where(used, -2, -1)).astype(np.int32)
 
 
 def compare_state(om: OracleManager, pool, where, with_bytes):
     tables, own_hbm, own_host = pool.tables()
     assert np.array_equal(om.pool.tables.astype(np.int32), tables), where
-    assert np.array_equal(owners_encoded(om.pool.owner_hbm), own_hbm), where
-    assert np.array_equal(owners_encoded(om.pool.owner_host), own_host), where
+    assert np.array_equal(owners_encoded(om.pool.owner_hbm, om.pool.hbm_used), own_hbm), where
+    assert np.array_equal(owners_encoded(om.pool.owner_host, om.pool.host_used), own_host), where
     st = pool.stats()
     assert st["error"] == 0, (where, st)
     assert st["hbm_allocated"] == int(om.pool.hbm_used.sum()), where

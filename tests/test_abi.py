@@ -59,6 +59,9 @@ int main(void) {
   printf("sizeof lv_remap_entry %zu\n", sizeof(lv_remap_entry));
   printf("sizeof lv_stats %zu\n", sizeof(lv_stats));
   printf("sizeof lv_resident_result %zu\n", sizeof(lv_resident_result));
+  printf("sizeof lv_request %zu\n", sizeof(lv_request));
+  printf("sizeof lv_sched_params %zu\n", sizeof(lv_sched_params));
+  F(lv_request, play_buffer_us); F(lv_request, kv_needed);
   F(lv_resident_result, k); F(lv_resident_result, n_found); F(lv_resident_result, n_victims);
   F(lv_resident_result, n_loaded); F(lv_resident_result, n_appended); F(lv_resident_result, status);
   F(lv_session_state, ctx_tokens); F(lv_session_state, flags); F(lv_session_state, gen_us);
@@ -89,6 +92,10 @@ int main(void) {
     assert got["lv_pool_desc"] == ctypes.sizeof(lv.lv_pool_desc)
     assert got["lv_stats"] == ctypes.sizeof(lv.lv_stats)
     assert got["lv_resident_result"] == lv.RESIDENT_DTYPE.itemsize
+    assert got["lv_request"] == lv.REQUEST_DTYPE.itemsize == 48
+    assert got["lv_sched_params"] == ctypes.sizeof(lv.lv_sched_params)
+    assert got["lv_request.play_buffer_us"][0] == lv.REQUEST_DTYPE.fields["play_buffer_us"][1]
+    assert got["lv_request.kv_needed"][0] == lv.REQUEST_DTYPE.fields["kv_needed"][1]
     for name in lv.RESIDENT_DTYPE.names:
         if name != "pad":
             assert lv.RESIDENT_DTYPE.fields[name][1] == got[f"lv_resident_result.{name}"][0], name

@@ -224,7 +224,7 @@ def test_remap_cancel_and_allocation_errors():
         assert remap([[1, 1, p], [1, 1, p]]) == lv.LV_ERR_DOUBLE_MAP
         pool.clear_error()
         t, own, _ = pool.tables()
-        assert t[1, 1] == p and own[p] == (1 << 32) | 1
+        assert t[1, 1] == p and own[p] == (1 << 16) | 1
         # cancel: an owned page is refused, a pending reservation is released
         pool.cancel(np.array([p], np.int32), 1)
         assert pool.sync(raise_on_error=False) == lv.LV_ERR_STATE
