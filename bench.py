@@ -454,6 +454,21 @@ def kernel_micro(torch, pool, seed=0):
     return out
 
 
+def micro_only(args, torch):
+    """kernel_micro on a 2048-page thinker-shaped pool (3.2 GB) instead of the bench pool."""
+    from paper_2606_22983_gb300 import build
+    build()
+    from paper_2606_22983_gb300.harness import fill_random
+    from paper_2606_22983_gb300.pool import KVPool
+    pool = KVPool(layers=48, kv_heads=4, head_dim=128, max_sessions=8, max_blocks=16,
+                  hbm_pages=2048, hbm_budget_pages=2048, host_pages=16)
+    try:
+        fill_random(pool, args.seed)
+        return {"micro": kernel_micro(torch, pool, args.seed)}
+    finally:
+        pool.close()
+
+
 def _profiled_traffic(kernel, bytes_per_launch):
     """DRAM bytes per launch from the committed ncu summary, or None when that
     summary does not cover this kernel or the kernel source changed since."""
@@ -558,6 +573,8 @@ def main():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", dest="cpu_baseline", action="store_false")
+    ap.add_argument("--micro-only", action="store_true",
+                    help="only the standalone kernel timings, on a small pool (profiling case)")
     ap.add_argument("--no-micro", dest="micro", action="store_false",
                     help="skip the standalone pack/unpack/remap/ranker timings")
     ap.add_argument("--sessions", type=int, default=0,
@@ -569,6 +586,9 @@ def main():
         ap.error("--warmup must be at least 3")
     if args.impl == "reference":
         line = reference(args)
+    elif args.micro_only:
+        import torch
+        line = micro_only(args, torch)
     else:
         import torch
         line = ours(args, torch)

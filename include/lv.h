@@ -504,6 +504,21 @@ typedef struct lv_kernel_timing {
 lv_status lv_timing_enable(lv_pool* pool, int32_t enable);
 lv_status lv_timing_read(lv_pool* pool, lv_kernel_timing* out /* [LV_TIMING_KINDS] */, int32_t reset);
 
+/* Failure paths without a GPU fault (Section 5.2: a failed or cancelled
+   transfer must leave the old mapping valid).  lv_inject_fault arms a one-shot
+   fault: the (after+1)-th later host-slot allocation (LV_FAULT_HOST_ALLOC) or
+   HBM-page allocation (LV_FAULT_HBM_ALLOC) fails as if that tier were full --
+   the device reports LV_ERR_NO_HOST / LV_ERR_NO_HBM and nothing is reserved or
+   copied -- or the (after+1)-th later copy-engine transfer of the staged path
+   (LV_FAULT_COPY) is not issued and the call returns LV_ERR_CUDA, leaving the
+   reservations made so far uncommitted (release them with lv_cancel).
+   LV_FAULT_NONE disarms.  lv_selftest_wait runs the library's bounded device
+   wait on a barrier that nothing completes, with a limit of limit_us; the
+   device then reports LV_ERR_TIMEOUT and the context stays usable. */
+enum { LV_FAULT_NONE = 0, LV_FAULT_HOST_ALLOC = 1, LV_FAULT_HBM_ALLOC = 2, LV_FAULT_COPY = 3 };
+lv_status lv_inject_fault(lv_pool* pool, int32_t kind, int32_t after);
+lv_status lv_selftest_wait(lv_pool* pool, int64_t limit_us, lv_stream stream);
+
 const char* lv_status_str(lv_status s);
 int32_t lv_version(void);
 

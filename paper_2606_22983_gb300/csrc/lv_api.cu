@@ -23,6 +23,8 @@ struct lv_pool {
   std::vector<cudaEvent_t> sync_events;
   int stage_ctas = 0;
   bool stage_tma = true;           // pack/unpack with TMA bulk copies (else 16-byte LSU copies)
+  int32_t fault_kind = LV_FAULT_NONE;   // lv_inject_fault: one-shot, after `fault_after` more events
+  int32_t fault_after = 0;
   // copy-kernel timing (lv_timing_enable): event pairs recorded per kind, reused
   bool timing = false;
   std::vector<lv::EventPair> ev_free;
@@ -169,6 +171,17 @@ const lv::EventPair* timing_pair(lv_pool* pool, int kind) {
   return &pool->ev_used[kind].back();
 }
 
+// True when the armed fault of this kind fires now (then it disarms).
+bool fault_fires(lv_pool* pool, int32_t kind) {
+  if (pool->fault_kind != kind) return false;
+  if (pool->fault_after > 0) {
+    --pool->fault_after;
+    return false;
+  }
+  pool->fault_kind = LV_FAULT_NONE;
+  return true;
+}
+
 // At least n timing-free events, created on first use and reused.
 lv_status sync_events(lv_pool* pool, size_t n) {
   while (pool->sync_events.size() < n) {
@@ -182,7 +195,8 @@ lv_status sync_events(lv_pool* pool, size_t n) {
 // The staged data movement of n validated tasks {out page, out slot, in slot, in page}
 // on `s`: pack out pages into staging, copy-engine runs of consecutive slots in each
 // direction on the side streams, unpack into the in pages; joined back into `s`.
-lv_status staged_move(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStream_t s) {
+lv_status staged_move_inner(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStream_t s,
+                            void** staging_out) {
   const lv::DevPool& d = pool->d;
   if (n <= 0) return LV_OK;
   if ((size_t)n > pool->tasks_host_cap) return LV_ERR_INVALID;
@@ -209,6 +223,7 @@ lv_status staged_move(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStrea
     const size_t bytes = (size_t)n * pb * ((any_out ? 1 : 0) + (any_in ? 1 : 0));
     cudaError_t e = cudaMallocFromPoolAsync(&staging, bytes, pool->mp, s);
     if (e != cudaSuccess) return lv_cuda_fail(e);
+    *staging_out = staging;
   }
   uint8_t* stg_out = static_cast<uint8_t*>(staging);
   uint8_t* stg_in = stg_out + (any_out ? (size_t)n * pb : 0);
@@ -223,6 +238,7 @@ lv_status staged_move(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStrea
       if (t[i].z < 0) { ++i; continue; }
       int64_t j = i + 1;
       while (j < b && t[j].z == t[j - 1].z + 1) ++j;
+      if (fault_fires(pool, LV_FAULT_COPY)) return LV_ERR_CUDA;
       LV_TRY(cudaMemcpyAsync(stg_in + (size_t)i * pb, host + (size_t)t[i].z * pb, (size_t)(j - i) * pb,
                              cudaMemcpyHostToDevice, pool->s_h2d));
       i = j;
@@ -240,6 +256,7 @@ lv_status staged_move(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStrea
       if (t[i].x < 0) { ++i; continue; }
       int64_t j = i + 1;
       while (j < b && t[j].x >= 0 && t[j].y == t[j - 1].y + 1) ++j;
+      if (fault_fires(pool, LV_FAULT_COPY)) return LV_ERR_CUDA;
       LV_TRY(cudaMemcpyAsync(host + (size_t)t[i].y * pb, stg_out + (size_t)i * pb, (size_t)(j - i) * pb,
                              cudaMemcpyDeviceToHost, pool->s_d2h));
       i = j;
@@ -252,12 +269,23 @@ lv_status staged_move(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStrea
     LV_TRY(lv::launch_stage(d, false, tasks_dev, a, b, stg_in, s, pool->stage_ctas,
                             timing_pair(pool, LV_TIMING_UNPACK), pool->stage_tma));
   }
-  LV_TRY(cudaEventRecord(ev_d2h_done, pool->s_d2h));
-  LV_TRY(cudaEventRecord(ev_h2d_done, pool->s_h2d));
-  LV_TRY(cudaStreamWaitEvent(s, ev_d2h_done, 0));
-  LV_TRY(cudaStreamWaitEvent(s, ev_h2d_done, 0));
-  LV_TRY(cudaFreeAsync(staging, s));
   return LV_OK;
+}
+
+// staged_move_inner, then (also after an early error) join the side streams back
+// into `s` and release the staging run in stream order.
+lv_status staged_move(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStream_t s) {
+  void* staging = nullptr;
+  const lv_status st = staged_move_inner(pool, tasks_dev, n, s, &staging);
+  if (staging) {
+    cudaEvent_t* ev = pool->sync_events.data();
+    cudaEventRecord(ev[1], pool->s_d2h);
+    cudaEventRecord(ev[2], pool->s_h2d);
+    cudaStreamWaitEvent(s, ev[1], 0);
+    cudaStreamWaitEvent(s, ev[2], 0);
+    cudaFreeAsync(staging, s);
+  }
+  return st;
 }
 
 void free_pool(lv_pool* pool) {
@@ -572,7 +600,7 @@ lv_status lv_swap_out(lv_pool* pool, const lv_victim* victims, int64_t n, int32_
     if ((r = st.out(slots_out, (size_t)n * 4, &sdev, true)) != LV_OK) return r;
     if ((r = st.out(commit_out, (size_t)n * sizeof(lv_remap_entry), &cdev, false)) != LV_OK) return r;
     int32_t* slots = static_cast<int32_t*>(sdev);
-    LV_TRY(lv::launch_alloc(pool->d, false, n, slots, s));
+    LV_TRY(lv::launch_alloc(pool->d, false, n, slots, s, fault_fires(pool, LV_FAULT_HOST_ALLOC)));
     if (mode == LV_MODE_STAGED) {
       void* tdev = nullptr;
       if ((r = st.out(nullptr, (size_t)n * sizeof(int4), &tdev, true)) != LV_OK) return r;
@@ -608,7 +636,7 @@ lv_status lv_swap_in(lv_pool* pool, int32_t sid, const int32_t* blks, int64_t n,
     if ((r = st.out(pages_out, (size_t)n * 4, &pdev, true)) != LV_OK) return r;
     if ((r = st.out(commit_out, (size_t)n * sizeof(lv_remap_entry), &cdev, false)) != LV_OK) return r;
     int32_t* pages = static_cast<int32_t*>(pdev);
-    LV_TRY(lv::launch_alloc(pool->d, true, n, pages, s));
+    LV_TRY(lv::launch_alloc(pool->d, true, n, pages, s, fault_fires(pool, LV_FAULT_HBM_ALLOC)));
     if (mode == LV_MODE_STAGED) {
       void* tdev = nullptr;
       if ((r = st.out(nullptr, (size_t)n * sizeof(int4), &tdev, true)) != LV_OK) return r;
@@ -985,6 +1013,20 @@ lv_status lv_timing_read(lv_pool* pool, lv_kernel_timing* out, int32_t reset) {
       pool->ev_used[kind].clear();
     }
   }
+  return LV_OK;
+}
+
+lv_status lv_inject_fault(lv_pool* pool, int32_t kind, int32_t after) {
+  if (!pool || kind < LV_FAULT_NONE || kind > LV_FAULT_COPY || after < 0) return LV_ERR_INVALID;
+  pool->fault_kind = kind;
+  pool->fault_after = after;
+  return LV_OK;
+}
+
+lv_status lv_selftest_wait(lv_pool* pool, int64_t limit_us, lv_stream stream) {
+  if (!pool || limit_us < 1 || limit_us > 10000000) return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  LV_TRY(lv::launch_selftest_wait(pool->d, limit_us * 1000, as_stream(stream)));
   return LV_OK;
 }
 

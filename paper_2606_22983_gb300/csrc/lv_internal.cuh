@@ -86,7 +86,8 @@ cudaError_t launch_events(const DevPool& p, const lv_event* ev, int64_t n, cudaS
 cudaError_t launch_select(const DevPool& p, int64_t now_us, int64_t k, bool fallback,
                           lv_victim* out, long long* count_dev, cudaStream_t s, int num_sms,
                           const long long* k_dev = nullptr);
-cudaError_t launch_alloc(const DevPool& p, bool hbm, int64_t n, int32_t* out, cudaStream_t s);
+cudaError_t launch_alloc(const DevPool& p, bool hbm, int64_t n, int32_t* out, cudaStream_t s,
+                         bool injected_fail = false);
 cudaError_t launch_swap_out(const DevPool& p, const lv_victim* v, const int32_t* slots,
                             int64_t n, lv_remap_entry* commit, cudaStream_t s, int num_sms,
                             const EventPair* ev = nullptr);
@@ -139,6 +140,7 @@ cudaError_t launch_stage(const DevPool& p, bool pack, const int4* tasks, int64_t
 cudaError_t launch_tasks_pages(const DevPool& p, const int32_t* pages, int64_t n, bool pack,
                                int4* tasks, cudaStream_t s);
 cudaError_t configure_stage_kernels(const DevPool& p);
+cudaError_t launch_selftest_wait(const DevPool& p, long long limit_ns, cudaStream_t s);
 // lv_sched.cu
 cudaError_t launch_schedule(const lv_sched_params& q, const lv_request* reqs, int n, int32_t* order,
                             int32_t* batch, long long* ctl, cudaStream_t s);

@@ -391,7 +391,7 @@ k_rank_emit(DevPool p, lv_victim* __restrict__ out) {
 constexpr int kAllocThreads = 1024;
 
 __global__ void __launch_bounds__(kAllocThreads)
-k_alloc(DevPool p, bool hbm, long long n, int32_t* __restrict__ out) {
+k_alloc(DevPool p, bool hbm, long long n, int32_t* __restrict__ out, bool injected_fail) {
   __shared__ int ok;
   uint32_t* bits = hbm ? p.bits_hbm : p.bits_host;
   const long long nbits = hbm ? p.hbm_pages : p.host_pages;
@@ -400,7 +400,7 @@ k_alloc(DevPool p, bool hbm, long long n, int32_t* __restrict__ out) {
   if (threadIdx.x == 0) {
     const long long before = (long long)atomicAdd(reinterpret_cast<unsigned long long*>(counter),
                                                   (unsigned long long)n);
-    ok = before + n <= cap;
+    ok = before + n <= cap && !injected_fail;
     if (!ok) {
       atomicAdd(reinterpret_cast<unsigned long long*>(counter), (unsigned long long)(-n));
       set_error(p.ctl, hbm ? LV_ERR_NO_HBM : LV_ERR_NO_HOST, n);
@@ -785,16 +785,24 @@ __device__ __forceinline__ void bulk_wait_read_1() {
 }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
-// Bounded wait on a stage barrier: false after `limit` polls (the data never came).
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, long long limit) {
-  for (long long it = 0; it < limit; ++it)
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Bounded wait on a stage barrier: false once `limit_ns` have passed (the data never came).
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, long long limit_ns) {
+  const unsigned long long t0 = global_ns();
+  for (;;) {
     if (mbar_try_wait(bar, parity)) return true;
-  return false;
+    if ((long long)(global_ns() - t0) > limit_ns) return false;
+  }
 }
 
 constexpr int kStageThreads = 32;     // one warp per CTA; lane 0 issues the bulk copies
 constexpr int kMaxStages = 8;
-constexpr long long kWaitPolls = 1ll << 22;   // each poll may also suspend briefly in hardware
+constexpr long long kWaitLimitNs = 1000000000ll;   // one second per stage wait
 
 // Moves units u = (task t, sub-page j) of P bytes through `stages` shared-memory
 // buffers: unit i's load is issued `stages` units ahead of its store.
@@ -850,7 +858,7 @@ k_stage_tasks(DevPool p, const int4* __restrict__ tasks, long long t_begin, long
     const int s = (int)(k % stages);
     bool stored = false;
     if (live[s]) {
-      if (!mbar_wait_bounded(&bars[s], phase[s], kWaitPolls)) {
+      if (!mbar_wait_bounded(&bars[s], phase[s], kWaitLimitNs)) {
         failed = true;
         break;
       }
@@ -870,7 +878,7 @@ k_stage_tasks(DevPool p, const int4* __restrict__ tasks, long long t_begin, long
     set_error(p.ctl, LV_ERR_TIMEOUT, blockIdx.x);
     // let every load still in flight land before the shared memory is released
     for (int s = 0; s < stages; ++s)
-      if (live[s]) mbar_wait_bounded(&bars[s], phase[s], kWaitPolls);
+      if (live[s]) mbar_wait_bounded(&bars[s], phase[s], kWaitLimitNs);
   }
   bulk_wait_all();
 }
@@ -910,6 +918,18 @@ __global__ void k_tasks_pages(DevPool p, const int32_t* __restrict__ pages, long
     return;
   }
   tasks[i] = pack ? make_int4(pg, -1, -1, -1) : make_int4(-1, -1, 0, pg);
+}
+
+// Self-test of the bounded wait: one thread arms a stage barrier for bytes that no
+// copy will ever deliver and waits on it with the given limit; the timeout must be
+// reported in the error word and the kernel must return.
+__global__ void k_selftest_wait(long long* ctl, long long limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  mbar_expect_tx(&bar, 16);                       // 16 bytes that never arrive
+  if (!mbar_wait_bounded(&bar, 0, limit_ns)) set_error(ctl, LV_ERR_TIMEOUT, limit_ns);
 }
 
 // ---------------------------------------------------------------- commit
@@ -1251,8 +1271,9 @@ cudaError_t configure_kernels() {
   return cudaFuncSetAttribute(k_rank_sort, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * 1024);
 }
 
-cudaError_t launch_alloc(const DevPool& p, bool hbm, int64_t n, int32_t* out, cudaStream_t s) {
-  k_alloc<<<1, kAllocThreads, 0, s>>>(p, hbm, n, out);
+cudaError_t launch_alloc(const DevPool& p, bool hbm, int64_t n, int32_t* out, cudaStream_t s,
+                         bool injected_fail) {
+  k_alloc<<<1, kAllocThreads, 0, s>>>(p, hbm, n, out, injected_fail);
   return cudaGetLastError();
 }
 
@@ -1311,6 +1332,11 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
     if (e != cudaSuccess) return e;
   }
   k_resident_finish<<<1, 32, 0, s>>>(p, sid, now_us, preload, R, result);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_selftest_wait(const DevPool& p, long long limit_ns, cudaStream_t s) {
+  k_selftest_wait<<<1, 32, 0, s>>>(p.ctl, limit_ns);
   return cudaGetLastError();
 }
 

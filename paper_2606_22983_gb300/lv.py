@@ -129,6 +129,8 @@ def _load():
         "lv_timing_enable": [vp, i32],
         "lv_pack_pages": [vp, vp, i64, vp, vp],
         "lv_schedule": [vp, ctypes.POINTER(lv_sched_params), vp, i32, vp, vp, vp],
+        "lv_inject_fault": [vp, i32, i32],
+        "lv_selftest_wait": [vp, i64, vp],
         "lv_unpack_pages": [vp, vp, vp, i64, vp],
         "lv_timing_read": [vp, ctypes.POINTER(lv_kernel_timing), i32],
         "lv_remap": [vp, vp, i64, vp],
@@ -166,7 +168,8 @@ EXPORTED = ("lv_pool_create", "lv_pool_destroy", "lv_pool_host_ptr", "lv_pool_im
             "lv_session_counts", "lv_session_blocks", "lv_read_tables", "lv_sync",
             "lv_get_stats", "lv_clear_error", "lv_status_str", "lv_version",
             "lv_select_victims_noalloc", "lv_timing_enable", "lv_timing_read", "lv_pack_pages",
-            "lv_unpack_pages", "lv_pool_host_device_ptr", "lv_schedule")
+            "lv_unpack_pages", "lv_pool_host_device_ptr", "lv_schedule", "lv_inject_fault",
+            "lv_selftest_wait")
 
 
 def lib():
@@ -346,6 +349,17 @@ def lv_timing_read(pool, reset=False) -> dict:
 def lv_schedule(pool, params: lv_sched_params, reqs, n, order_out, batch_out, stream=None):
     _check(_lib.lv_schedule(pool, ctypes.byref(params), ptr(reqs), n, ptr(order_out), ptr(batch_out),
                             stream_handle(stream)), "lv_schedule")
+
+
+LV_FAULT_NONE, LV_FAULT_HOST_ALLOC, LV_FAULT_HBM_ALLOC, LV_FAULT_COPY = 0, 1, 2, 3
+
+
+def lv_inject_fault(pool, kind, after=0):
+    _check(_lib.lv_inject_fault(pool, kind, after), "lv_inject_fault")
+
+
+def lv_selftest_wait(pool, limit_us, stream=None):
+    _check(_lib.lv_selftest_wait(pool, limit_us, stream_handle(stream)), "lv_selftest_wait")
 
 
 def lv_status_str(status: int) -> str:
