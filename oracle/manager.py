@@ -49,7 +49,8 @@ class OracleManager:
         self.shape = sh
         self.pool = OraclePool(sh.layers, sh.kv_heads, sh.head_dim, sh.page_tokens, sh.elem_bytes,
                                spec.n_sessions, spec.max_blocks, spec.hbm_pages,
-                               spec.hbm_budget_pages, spec.host_pages, with_bytes=with_bytes)
+                               spec.hbm_budget_pages, spec.host_pages, with_bytes=with_bytes,
+                               inclusive=spec.tiers == 1)
         init = workload.init
         self.pool.import_placement(init.placement, init.ctx_tokens)
         self.sessions = []

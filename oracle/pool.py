@@ -21,9 +21,20 @@ Operations follow their plain definitions:
     failed or cancelled transfer is never committed, so the old mapping stays
     valid (Section 5.2: preloading affects latency but not correctness).
 
-Reading: the tiers are exclusive -- a block lives in exactly one tier, and a
-host slot is freed when its block is committed back to HBM (the paper does
-not say whether the host copy is kept).
+Tiers (the paper does not say whether the host copy is kept after a reload):
+  * exclusive (default): a block lives in exactly one tier; its host slot is
+    freed when the block is committed back to HBM.
+  * inclusive: the host slot of a block committed back to HBM stays allocated
+    and owned by the block as its *clean copy* (``shadow[s, b]``), as long as
+    the block's bytes are unchanged.  KV rows are written once, when their
+    token is appended, so only a session's last, partially filled block can
+    change: appending tokens into it drops its clean copy (the slot is freed).
+    Evicting a block that has a clean copy moves no bytes: its "slot" is the
+    clean copy, no slot is reserved, and the commit points the table back to
+    it.  Committing a block to any other host slot drops its clean copy.
+    Clean copies are never reclaimed for other blocks, so the host tier must
+    be able to hold every block (otherwise an eviction fails with NO_HOST,
+    exactly as in the exclusive mode).
 """
 from __future__ import annotations
 
@@ -50,7 +61,8 @@ def _enc_host(slot: int) -> int:
 
 class OraclePool:
     def __init__(self, layers, kv_heads, head_dim, page_tokens, elem_bytes, n_sessions,
-                 max_blocks, hbm_pages, hbm_budget_pages, host_pages, with_bytes=True):
+                 max_blocks, hbm_pages, hbm_budget_pages, host_pages, with_bytes=True,
+                 inclusive=False):
         self.L, self.T = layers, page_tokens
         self.P = page_tokens * kv_heads * head_dim * elem_bytes
         self.J = 2 * layers
@@ -69,6 +81,10 @@ class OraclePool:
             self.host = np.zeros((host_pages, self.J, self.P), dtype=np.uint8)
         self.bytes_out = 0
         self.bytes_in = 0
+        self.inclusive = bool(inclusive)
+        self.shadow = np.full((n_sessions, max_blocks), -1, dtype=np.int64)   # clean copies
+        self.clean_out = 0        # evictions that moved no bytes
+        self.clean_dropped = 0    # clean copies dropped because their block changed
 
     # ---------------------------------------------------------------- set-up
     def import_placement(self, placement: np.ndarray, ctx_tokens: np.ndarray) -> None:
@@ -126,7 +142,10 @@ class OraclePool:
 
     # ------------------------------------------------------------------ copy
     def swap_out(self, sid, blk, page) -> np.ndarray:
-        """Copy victim pages to freshly reserved host slots; returns the slots."""
+        """Copy victim pages to freshly reserved host slots; returns the slots.
+
+        Inclusive tiers: a victim with a clean copy gets that slot and moves no
+        bytes; the others reserve the lowest free slots, in victim order."""
         sid, blk, page = (np.asarray(x, dtype=np.int64) for x in (sid, blk, page))
         for s, b, p in zip(sid, blk, page):
             s, b, p = int(s), int(b), int(p)
@@ -134,12 +153,19 @@ class OraclePool:
                 raise OracleError("BOUNDS", f"victim ({s},{b},{p})")
             if self.tables[s, b] != p or tuple(self.owner_hbm[p]) != (s, b):
                 raise OracleError("STATE", f"victim ({s},{b},{p}) is not resident there")
-        slots = self.alloc_host(sid.size)
+        clean = np.array([self.inclusive and self.shadow[int(s), int(b)] >= 0
+                          for s, b in zip(sid, blk)], dtype=bool)
+        slots = np.empty(sid.size, dtype=np.int64)
+        slots[~clean] = self.alloc_host(int((~clean).sum()))
+        slots[clean] = self.shadow[sid[clean], blk[clean]]
         if self.with_bytes:
-            for p, h in zip(page, slots):
+            for p, h, c in zip(page, slots, clean):
+                if c:
+                    continue
                 for j in range(self.J):
                     self.host[h, j, :] = self.hbm[j, p, :]
-        self.bytes_out += int(sid.size) * self.J * self.P
+        self.bytes_out += int((~clean).sum()) * self.J * self.P
+        self.clean_out += int(clean.sum())
         return slots
 
     def swap_in(self, sid: int, blks) -> np.ndarray:
@@ -183,21 +209,33 @@ class OraclePool:
                 h = _slot_of(e)
                 if h >= self.host_pages:
                     raise OracleError("BOUNDS", f"slot {h}")
-                if not self.host_used[h] or self.owner_host[h, 0] != -1:
+                own_copy = self.inclusive and self.shadow[s, b] == h
+                if not own_copy and (not self.host_used[h] or self.owner_host[h, 0] != -1):
                     raise OracleError("DOUBLE_MAP", f"slot {h} is not a free reservation")
                 self.owner_host[h] = (s, b)
             else:
                 raise OracleError("BOUNDS", "new location -1")
             old = int(self.tables[s, b])
             self.tables[s, b] = e
+            if _is_host(e):
+                g = int(self.shadow[s, b])
+                if g >= 0 and g != _slot_of(e):          # committed elsewhere: the copy goes
+                    self._free_host(g)
+                self.shadow[s, b] = -1
             if old >= 0:
                 self.owner_hbm[old] = (-1, -1)
                 self.hbm_used[old] = False
             elif _is_host(old):
-                self.owner_host[_slot_of(old)] = (-1, -1)
-                self.host_used[_slot_of(old)] = False
+                if self.inclusive and e >= 0:            # the host copy stays, clean
+                    self.shadow[s, b] = _slot_of(old)
+                else:
+                    self._free_host(_slot_of(old))
         if int(self.hbm_used.sum()) > self.budget:
             raise OracleError("BUDGET", "HBM budget exceeded after commit")
+
+    def _free_host(self, h: int) -> None:
+        self.owner_host[h] = (-1, -1)
+        self.host_used[h] = False
 
     def cancel(self, locs) -> None:
         """Release reservations that were never committed."""
@@ -209,7 +247,10 @@ class OraclePool:
                 self.hbm_used[e] = False
             elif _is_host(e):
                 h = _slot_of(e)
-                if not self.host_used[h] or self.owner_host[h, 0] != -1:
+                o_s, o_b = (int(x) for x in self.owner_host[h])
+                if self.inclusive and o_s >= 0 and self.shadow[o_s, o_b] == h:
+                    continue                             # a clean copy: nothing was reserved
+                if not self.host_used[h] or o_s != -1:
                     raise OracleError("STATE", f"slot {h} is not a pending reservation")
                 self.host_used[h] = False
 
@@ -222,6 +263,12 @@ class OraclePool:
             raise OracleError("BOUNDS", f"session {sid} would need {nb} blocks")
         first = int(self.nblocks[sid])
         pages = self.alloc_hbm(nb - first)
+        tail = int(self.ctx[sid]) % self.T
+        if n_tokens > 0 and tail and self.shadow[sid, first - 1] >= 0:
+            # the partially filled last block gains rows: its clean copy is stale
+            self._free_host(int(self.shadow[sid, first - 1]))
+            self.shadow[sid, first - 1] = -1
+            self.clean_dropped += 1
         for i, p in enumerate(pages):
             b = first + i
             self.tables[sid, b] = int(p)
@@ -241,14 +288,19 @@ class OraclePool:
     def free_budget(self) -> int:
         return self.budget - self.resident_count()
 
+    def clean_copies(self) -> int:
+        return int((self.shadow >= 0).sum())
+
     def check_invariants(self) -> None:
-        """Owner tables and block tables are mutually inverse; budget holds."""
-        n_hbm = n_host = 0
+        """Owner tables and block tables (plus clean copies) are mutually inverse;
+        budget holds."""
+        n_hbm = n_host = n_clean = 0
         for s in range(self.S):
             for b in range(self.max_blocks):
                 e = int(self.tables[s, b])
+                g = int(self.shadow[s, b])
                 if b >= self.nblocks[s]:
-                    assert e == -1, (s, b, e)
+                    assert e == -1 and g == -1, (s, b, e, g)
                     continue
                 if e >= 0:
                     assert tuple(self.owner_hbm[e]) == (s, b), (s, b, e)
@@ -257,8 +309,12 @@ class OraclePool:
                     assert _is_host(e), (s, b, e)
                     assert tuple(self.owner_host[_slot_of(e)]) == (s, b), (s, b, e)
                     n_host += 1
+                if g >= 0:
+                    assert self.inclusive and e >= 0, (s, b, e, g)
+                    assert tuple(self.owner_host[g]) == (s, b) and self.host_used[g], (s, b, g)
+                    n_clean += 1
         assert int((self.owner_hbm[:, 0] >= 0).sum()) == n_hbm
-        assert int((self.owner_host[:, 0] >= 0).sum()) == n_host
+        assert int((self.owner_host[:, 0] >= 0).sum()) == n_host + n_clean
         assert np.all(self.hbm_used[self.owner_hbm[:, 0] >= 0])
         assert np.all(self.host_used[self.owner_host[:, 0] >= 0])
         assert int(self.hbm_used.sum()) <= self.budget

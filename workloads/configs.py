@@ -65,6 +65,7 @@ class PoolSpec:
     t_play_mode: int = 0         # 0: playback accounting, 1: progress counters
     unit_us: int = 80_000        # progress-counter unit (one audio token)
     policy: int = 0              # 0: next-use order, 1: LRU baseline
+    tiers: int = 0               # 0: exclusive, 1: inclusive (clean host copies kept)
 
     def with_(self, **kw) -> "PoolSpec":
         return replace(self, **kw)

@@ -265,6 +265,8 @@ def _interactive(spec: PoolSpec, seed: int, n_events: int, ctx_lo: int, ctx_hi: 
         total = int(_pages(grown, T).sum())
         host = max(int(n_pages.sum()) - spec.hbm_budget_pages, total - spec.hbm_budget_pages) \
             + 2 * spec.max_blocks
+        if spec.tiers == 1:          # inclusive tiers: room for a host copy of every block
+            host = total + 2 * spec.max_blocks
         spec = spec.with_(host_pages=host)
         meta["total_pages_final"] = total
     meta["total_pages"] = int(n_pages.sum())
@@ -295,7 +297,8 @@ def _turns(spec: PoolSpec, seed: int, n_turns: int, ctx_lo: int, ctx_hi: int,
     else:
         raise RuntimeError("could not draw contexts that exceed the budget")
     total = int(n_pages.sum())
-    host_pages = spec.host_pages or (total - spec.hbm_budget_pages + 2 * spec.max_blocks)
+    host_pages = spec.host_pages or (total - spec.hbm_budget_pages + 2 * spec.max_blocks
+                                     if spec.tiers == 0 else total + 2 * spec.max_blocks)
     spec = spec.with_(host_pages=host_pages)
     placement = _place_fill(n_pages, spec.max_blocks, spec.hbm_budget_pages, host_pages)
     gen0 = rng.integers(reply_lo_us, reply_hi_us + 1, S).astype(np.int64)
@@ -346,8 +349,8 @@ def _frag(spec: PoolSpec, seed: int, n_events: int, ctx_lo: int, ctx_hi: int,
     else:
         raise RuntimeError("could not draw contexts that exceed the budget")
     total = int(n_pages.sum())
-    host_pages = spec.host_pages or (total - spec.hbm_budget_pages + max(total // 10, 2 * spec.max_blocks)
-                                     + evict_hi)
+    keep = total if spec.tiers == 1 else total - spec.hbm_budget_pages   # inclusive: every block
+    host_pages = spec.host_pages or (keep + max(total // 10, 2 * spec.max_blocks) + evict_hi)
     spec = spec.with_(host_pages=host_pages)
     perm = rng.permutation(spec.hbm_pages)
     placement = _place_fill(n_pages, spec.max_blocks, spec.hbm_budget_pages, host_pages, page_perm=perm)
