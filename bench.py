@@ -168,8 +168,12 @@ def run_turns(gm, wl, lo, hi, dev_events=None):
 
 
 def _moved_pages(pool):
+    """Pages whose bytes crossed the host link (an eviction that found a clean
+    copy under inclusive tiers moves none): (both ways, out, in)."""
     st = pool.stats()
-    return st["pages_out"] + st["pages_in"], st["pages_out"], st["pages_in"]
+    page = pool.J * pool.P
+    out, inn = st["bytes_out"] // page, st["bytes_in"] // page
+    return out + inn, out, inn
 
 
 def ours(args, torch):
@@ -187,12 +191,12 @@ def ours(args, torch):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     K, W = args.steps, args.warmup
     over = {}
-    if args.sessions or args.budget_pages:
+    if args.sessions or args.budget_pages or args.tiers:
         from workloads import pool_spec
         sp = pool_spec(WORKLOAD)
         b = args.budget_pages or sp.hbm_budget_pages
         over["spec"] = sp.with_(n_sessions=args.sessions or sp.n_sessions, hbm_pages=b,
-                                hbm_budget_pages=b)
+                                hbm_budget_pages=b, tiers=args.tiers)
     wl = make_workload(WORKLOAD, args.seed + rank, n_turns=W + 2 * K, **over)
     pool = pool_for(wl)
     fill_random(pool, args.seed + rank)
@@ -294,11 +298,21 @@ def ours(args, torch):
         if link_kern:
             dom = max(link_kern, key=lambda n: kern[n]["total_ms"])
             dk = kern[dom]
-            peak = {"swap_out": peaks["d2h"], "swap_in": peaks["h2d"]}.get(dom, peaks.get("bidir"))
-            peak_dir = {"swap_out": "D2H", "swap_in": "H2D"}.get(dom, "D2H and H2D concurrently")
+            peak = {"swap_out": peaks["d2h"], "swap_in": peaks["h2d"]}.get(dom)
+            peak_dir = {"swap_out": "D2H", "swap_in": "H2D"}.get(dom)
+            if peak is None:
+                # the exchange moves O bytes out and I in at once: the link's best time for
+                # that mix is max(O / d2h, I / h2d, (O + I) / bidir)
+                O, I = (o1 - o0) * page_bytes, (i1 - i0) * page_bytes
+                best_s = max(O / peaks["d2h"], I / peaks["h2d"], (O + I) / peaks["bidir"])
+                peak = (O + I) / best_s if best_s > 0 else peaks["bidir"]
+                peak_dir = (f"D2H and H2D concurrently, weighted by this run's mix: "
+                            f"{O / 1e9:.1f} GB out, {I / 1e9:.1f} GB in")
+            # the profiled DRAM ratio holds for the exclusive tiers' two-way mix only
+            traffic = _profiled_traffic(dom, dk["bytes_per_launch"]) if args.tiers == 0 else None
             roof = {"kernel": dom, "bound": "host_link", "achieved": round(dk["gbs"], 1),
                     "peak": round(peak, 1), "unit": "GB/s", "frac": round(dk["gbs"] / peak, 3),
-                    "traffic": _profiled_traffic(dom, dk["bytes_per_launch"]),
+                    "traffic": traffic,
                     "peak_source": "same-run contiguous page-locked cudaMemcpyAsync "
                                    f"({peak_dir}, mean-turn byte count)"}
         else:   # staged: the copy engines carry the link traffic, the kernels are HBM-bound
@@ -319,10 +333,12 @@ def ours(args, torch):
                        "hbm_budget_pages": wl.spec.hbm_budget_pages, "host_pages": wl.spec.host_pages,
                        "mode": {0: "auto", 1: "zero_copy", 2: "staged"}[args.mode],
                        "driver": args.driver,
+                       "tiers": ("exclusive", "inclusive")[args.tiers],
                        "l2": "inputs larger than L2 (mean turn moves "
                              f"{mean_turn / 1e6:.0f} MB each way from a 40 GB pool)",
                        "parallelism": f"replicas x{ws}"},
             "blocks_per_s": round(moved / page_bytes / t_max, 1),
+            "turns_per_s": round(K * ws / t_max, 2),
             "link_peak_gbs": {k: round(v, 1) for k, v in peaks.items()},
             "link_frac": round(value / peaks["bidir"], 3) if "bidir" in peaks else None,
             "roofline": roof,
@@ -620,6 +636,8 @@ def main():
                     help="smaller case for profiling: number of sessions")
     ap.add_argument("--budget-pages", type=int, default=0,
                     help="smaller case for profiling: HBM budget in pages")
+    ap.add_argument("--tiers", type=int, default=0, choices=(0, 1),
+                    help="0 exclusive tiers, 1 inclusive (clean host copies kept)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")

@@ -75,6 +75,19 @@ enum { LV_SELECT_FALLBACK = 1 };                       /* lv_select_victims flag
    not running, ranked by last use ascending (then session id ascending, suffix
    blocks first); speech, barge-in and preload protection are ignored. */
 enum { LV_POLICY_NEXT_USE = 0, LV_POLICY_LRU = 1 };
+/* Host-tier mode (lv_pool_desc.tiers).  The paper does not say whether a
+   reloaded block keeps its host copy.  LV_TIERS_EXCLUSIVE: a block lives in
+   one tier; its host slot is freed when it is committed back to HBM.
+   LV_TIERS_INCLUSIVE: that slot stays allocated and owned by the block as its
+   clean copy while the block's bytes are unchanged, so evicting the block
+   again moves no bytes (lv_swap_out, lv_swap_exchange, lv_make_resident).  KV
+   rows are written once, when their token is appended, so only the last,
+   partially filled block of a session changes: lv_session_append and
+   lv_make_resident drop that block's clean copy when they add rows to it.
+   Clean copies are not reclaimed for other blocks: the host tier should hold
+   a slot for every block (with fewer, an eviction fails with LV_ERR_NO_HOST as
+   in the exclusive mode). */
+enum { LV_TIERS_EXCLUSIVE = 0, LV_TIERS_INCLUSIVE = 1 };
 
 /* session flag bits (lv_session_state.flags) */
 enum {
@@ -117,6 +130,8 @@ typedef struct lv_pool_desc {
   int64_t unit_us;             /* progress-counter unit, 1..2^31 */
   int32_t t_play_mode;         /* LV_PLAY_PLAYBACK or LV_PLAY_COUNTERS */
   int32_t policy;              /* LV_POLICY_NEXT_USE (Section 5.1) or LV_POLICY_LRU */
+  int32_t tiers;               /* LV_TIERS_EXCLUSIVE (default) or LV_TIERS_INCLUSIVE */
+  int32_t reserved;            /* must be 0 */
 } lv_pool_desc;
 
 /* Per-session interaction state (72 bytes).  ctx_tokens is maintained by
@@ -168,6 +183,10 @@ typedef struct lv_stats {
   int64_t selects, victims, shortfalls, pages_out, pages_in, bytes_out, bytes_in;
   int64_t remap_entries, appended_pages, cancels, events, fallback_selects;
   int64_t preloads, preloads_skipped;   /* lv_make_resident with LV_RESIDENT_PRELOAD */
+  /* LV_TIERS_INCLUSIVE: clean copies held now (part of host_allocated), evictions
+     that found one and moved no bytes (part of pages_out, not of bytes_out), and
+     copies dropped because their block gained rows */
+  int64_t clean_copies, clean_out, clean_dropped;
 } lv_stats;
 
 /* ---------------------------------------------------------------- pool */
@@ -251,7 +270,9 @@ lv_status lv_select_victims(lv_pool* pool, int64_t now_us, int64_t k, uint32_t f
    (lv_remap_entry [n], may be NULL) ready-to-commit entries.  mode:
    LV_MODE_ZERO_COPY (SM copies straight into the mapped host pool),
    LV_MODE_STAGED (pack into HBM staging, then copy-engine transfer) or
-   LV_MODE_AUTO (zero-copy).  LV_MODE_STAGED reads the reserved slots back
+   LV_MODE_AUTO (zero-copy).  LV_TIERS_INCLUSIVE: a victim that has a clean
+   copy gets that slot, reserves nothing and moves no bytes; the others reserve
+   the lowest free slots in victim order.  LV_MODE_STAGED reads the reserved slots back
    to build one copy per contiguous slot run, so it waits on the host for the
    work queued before it on `stream` (and for the reservation).  Device-detected: LV_ERR_NO_HOST (nothing reserved or copied),
    LV_ERR_BOUNDS, LV_ERR_STATE (a victim is not resident where it says). */
@@ -338,15 +359,21 @@ lv_status lv_make_resident(lv_pool* pool, int32_t sid, int64_t now_us, int32_t a
 /* Section 6 (side tables) and Section 5.2 ("preloading affects latency but not
    correctness"): commits n entries.  For each, the new location must be a
    reservation not yet owned; it becomes owned by (sid, blk), the block table
-   points to it and the old location is freed.  Entries are independent;
+   points to it and the old location is freed.  LV_TIERS_INCLUSIVE: a host
+   location may also be the block's own clean copy (it then stops being a
+   copy); a block committed to HBM from the host tier keeps its slot as its
+   clean copy; a block committed to another host slot loses its clean copy
+   (freed).  Entries are independent;
    a bad one is skipped.  Device-detected: LV_ERR_DOUBLE_MAP (location not a
    free reservation, or the same block twice in one call), LV_ERR_BOUNDS,
    LV_ERR_BUDGET. */
 lv_status lv_remap(lv_pool* pool, const lv_remap_entry* entries, int64_t n, lv_stream stream);
 
 /* Releases reservations that will never be committed (a cancelled or failed
-   transfer, Section 5.2).  locs are encoded locations.  Device-detected:
-   LV_ERR_STATE when a location is owned or not reserved. */
+   transfer, Section 5.2).  locs are encoded locations.  A host slot that is
+   its owner's clean copy (LV_TIERS_INCLUSIVE) was not reserved and is left as
+   it is.  Device-detected: LV_ERR_STATE when a location is owned or not
+   reserved. */
 lv_status lv_cancel(lv_pool* pool, const int32_t* locs, int64_t n, lv_stream stream);
 
 /* The staged path's building blocks (Section 6, offload connector), usable on
@@ -363,7 +390,8 @@ lv_status lv_unpack_pages(lv_pool* pool, const void* src, const int32_t* pages, 
 
 /* Block-level allocation kept (Section 5.1): grows session sid's context by
    n_tokens; each new block takes the lowest free HBM page, in block order, and
-   is committed at once.  pages_out (int32, capacity ceil(n_tokens/T)+1, may be
+   is committed at once.  LV_TIERS_INCLUSIVE: when n_tokens > 0 and the last
+   block is partially filled, its clean copy (if any) is dropped.  pages_out (int32, capacity ceil(n_tokens/T)+1, may be
    NULL) receives the new pages; *count_out (int32, may be NULL) their number.
    Device-detected: LV_ERR_NO_HBM (nothing changes), LV_ERR_BOUNDS (the block
    table would overflow). */

@@ -326,6 +326,8 @@ lv_status validate_desc(const lv_pool_desc* d) {
   if (d->t_play_mode != LV_PLAY_PLAYBACK && d->t_play_mode != LV_PLAY_COUNTERS) return LV_ERR_INVALID;
   if (d->within_order != LV_SUFFIX_FIRST && d->within_order != LV_ASCENDING) return LV_ERR_INVALID;
   if (d->policy != LV_POLICY_NEXT_USE && d->policy != LV_POLICY_LRU) return LV_ERR_INVALID;
+  if (d->tiers != LV_TIERS_EXCLUSIVE && d->tiers != LV_TIERS_INCLUSIVE) return LV_ERR_INVALID;
+  if (d->reserved != 0) return LV_ERR_INVALID;
   if (d->hbm_kv == nullptr) return LV_ERR_INVALID;
   return LV_OK;
 }
@@ -357,6 +359,7 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
   d.within = desc->within_order;
   d.tplay = desc->t_play_mode;
   d.policy = desc->policy;
+  d.incl = desc->tiers == LV_TIERS_INCLUSIVE ? 1 : 0;
 
   // the caller's HBM sub-page arrays
   std::vector<uint8_t*> kv(d.J);
@@ -399,6 +402,7 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       (st = dev_alloc(pool, &d.sess, d.S)) != LV_OK ||
       (st = dev_alloc(pool, &d.table, tb)) != LV_OK ||
       (st = dev_alloc(pool, &d.mark, tb)) != LV_OK ||
+      (st = dev_alloc(pool, &d.shadow, tb)) != LV_OK ||
       (st = dev_alloc(pool, &d.own_hbm, (size_t)d.hbm_pages)) != LV_OK ||
       (st = dev_alloc(pool, &d.own_host, (size_t)d.host_pages)) != LV_OK ||
       (st = dev_alloc(pool, &d.bits_hbm, wh)) != LV_OK ||
@@ -424,6 +428,7 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       cudaMemsetAsync(d.sess, 0, d.S * sizeof(lv_session_state), s) != cudaSuccess ||
       cudaMemsetAsync(d.table, 0xff, tb * sizeof(int32_t), s) != cudaSuccess ||
       cudaMemsetAsync(d.mark, 0, tb * sizeof(int32_t), s) != cudaSuccess ||
+      cudaMemsetAsync(d.shadow, 0xff, tb * sizeof(int32_t), s) != cudaSuccess ||
       cudaMemsetAsync(d.own_hbm, 0xff, (size_t)d.hbm_pages * 4, s) != cudaSuccess ||
       cudaMemsetAsync(d.own_host, 0xff, (size_t)(d.host_pages ? d.host_pages : 1) * 4, s) != cudaSuccess ||
       cudaMemsetAsync(d.bits_hbm, 0, wh * 4, s) != cudaSuccess ||
@@ -506,6 +511,7 @@ lv_status lv_pool_import(lv_pool* pool, const int32_t* placement, const int32_t*
     LV_TRY(cudaMemsetAsync(d.bits_hbm, 0, (size_t)((d.hbm_pages + 31) / 32) * 4, s));
     if (d.host_pages) LV_TRY(cudaMemsetAsync(d.bits_host, 0, (size_t)((d.host_pages + 31) / 32) * 4, s));
     LV_TRY(cudaMemsetAsync(d.ctl, 0, 2 * sizeof(long long), s));   // allocation counts
+    LV_TRY(cudaMemsetAsync(d.ctl + lv::C_CLEAN, 0, sizeof(long long), s));   // no clean copies
     LV_TRY(lv::launch_import(d, static_cast<const int32_t*>(pl), static_cast<const int32_t*>(cx), s));
     LV_TRY(lv::launch_check_budget(d, s));
     return st.finish();
@@ -600,7 +606,11 @@ lv_status lv_swap_out(lv_pool* pool, const lv_victim* victims, int64_t n, int32_
     if ((r = st.out(slots_out, (size_t)n * 4, &sdev, true)) != LV_OK) return r;
     if ((r = st.out(commit_out, (size_t)n * sizeof(lv_remap_entry), &cdev, false)) != LV_OK) return r;
     int32_t* slots = static_cast<int32_t*>(sdev);
-    LV_TRY(lv::launch_alloc(pool->d, false, n, slots, s, fault_fires(pool, LV_FAULT_HOST_ALLOC)));
+    const bool fail_alloc = fault_fires(pool, LV_FAULT_HOST_ALLOC);
+    if (pool->d.incl)
+      LV_TRY(lv::launch_alloc_out(pool->d, static_cast<const lv_victim*>(vin), n, slots, s, fail_alloc));
+    else
+      LV_TRY(lv::launch_alloc(pool->d, false, n, slots, s, fail_alloc));
     if (mode == LV_MODE_STAGED) {
       void* tdev = nullptr;
       if ((r = st.out(nullptr, (size_t)n * sizeof(int4), &tdev, true)) != LV_OK) return r;
@@ -968,7 +978,7 @@ lv_status lv_get_stats(lv_pool* pool, lv_stats* out, lv_stream stream) {
   out->shortfalls = c[lv::C_SHORTFALLS];
   out->pages_out = c[lv::C_PAGES_OUT];
   out->pages_in = c[lv::C_PAGES_IN];
-  out->bytes_out = c[lv::C_PAGES_OUT] * page_bytes;
+  out->bytes_out = (c[lv::C_PAGES_OUT] - c[lv::C_CLEAN_OUT]) * page_bytes;
   out->bytes_in = c[lv::C_PAGES_IN] * page_bytes;
   out->remap_entries = c[lv::C_REMAP];
   out->appended_pages = c[lv::C_APPENDED];
@@ -977,6 +987,9 @@ lv_status lv_get_stats(lv_pool* pool, lv_stats* out, lv_stream stream) {
   out->fallback_selects = c[lv::C_FALLBACK];
   out->preloads = c[lv::C_PRELOADS];
   out->preloads_skipped = c[lv::C_PRELOADS_SKIPPED];
+  out->clean_copies = c[lv::C_CLEAN];
+  out->clean_out = c[lv::C_CLEAN_OUT];
+  out->clean_dropped = c[lv::C_CLEAN_DROPPED];
   return LV_OK;
 }
 

@@ -21,6 +21,7 @@ enum Ctl : int {
   C_ERR_DETAIL = 3,
   C_SEL_COUNT = 4,     // victims written by the last select
   C_SEL_TOTAL = 5,     // candidates seen by the last select
+  C_CLEAN = 6,         // clean host copies held now (inclusive tiers; part of C_HOST_ALLOC)
   C_SELECTS = 8,
   C_VICTIMS,
   C_SHORTFALLS,
@@ -33,6 +34,8 @@ enum Ctl : int {
   C_FALLBACK,
   C_PRELOADS,
   C_PRELOADS_SKIPPED,
+  C_CLEAN_OUT,         // evictions that found a clean copy (moved no bytes)
+  C_CLEAN_DROPPED,     // clean copies dropped because their block gained rows
   C_N = 32
 };
 
@@ -48,11 +51,13 @@ struct DevPool {
   int32_t within;         // LV_SUFFIX_FIRST / LV_ASCENDING
   int32_t tplay;          // LV_PLAY_PLAYBACK / LV_PLAY_COUNTERS
   int32_t policy;         // LV_POLICY_NEXT_USE / LV_POLICY_LRU
+  int32_t incl;           // 1: LV_TIERS_INCLUSIVE
   uint8_t* const* kv;     // [J] device pointers, sub-page j of page p at kv[j] + p*P
   uint8_t* host;          // device view of the host pool [host_pages][J][P]
   lv_session_state* sess; // [S]
   int32_t* table;         // [S][maxB]
   int32_t* mark;          // [S][maxB] epoch of the last remap that touched the block
+  int32_t* shadow;        // [S][maxB] host slot holding the block's clean copy, or -1
   uint32_t* own_hbm;      // [hbm_pages] owner word (kOwnerNone / kOwnerReserved / sid << 16 | blk)
   uint32_t* own_host;     // [host_pages]
   uint32_t* bits_hbm;     // allocation bitmap, 1 = reserved or owned
@@ -88,6 +93,10 @@ cudaError_t launch_select(const DevPool& p, int64_t now_us, int64_t k, bool fall
                           const long long* k_dev = nullptr);
 cudaError_t launch_alloc(const DevPool& p, bool hbm, int64_t n, int32_t* out, cudaStream_t s,
                          bool injected_fail = false);
+// host slots for n victims: a clean copy where the block has one (inclusive
+// tiers), else the lowest free slots in victim order (reserved)
+cudaError_t launch_alloc_out(const DevPool& p, const lv_victim* v, int64_t n, int32_t* out,
+                             cudaStream_t s, bool injected_fail = false);
 cudaError_t launch_swap_out(const DevPool& p, const lv_victim* v, const int32_t* slots,
                             int64_t n, lv_remap_entry* commit, cudaStream_t s, int num_sms,
                             const EventPair* ev = nullptr);

@@ -96,6 +96,45 @@ __device__ void block_alloc_lowest(uint32_t* bits, long long nbits, long long n,
   }
 }
 
+// Inclusive tiers: the host slot holding victim x's clean copy, or -1.
+__device__ __forceinline__ int32_t clean_copy_of(const DevPool& p, const lv_victim& x) {
+  if (!p.incl || x.sid < 0 || x.sid >= p.S || x.blk < 0 || x.blk >= p.maxB) return -1;
+  return p.shadow[(size_t)x.sid * p.maxB + x.blk];
+}
+
+// Host slots for n victims when nd of them have no clean copy: the nd lowest
+// free slots are taken (ascending) into out[0..nd), then spread in place so
+// that the r-th victim without a copy gets the r-th slot and every other
+// victim its copy.  The spreading runs from the last chunk to the first: a
+// victim's rank r is at most its index, so each read position still holds its
+// compact value when it is read.
+template <int NT>
+__device__ void block_alloc_out(const DevPool& p, const lv_victim* __restrict__ v, long long n,
+                                long long nd, int32_t* out) {
+  if (nd > 0) block_alloc_lowest<NT>(p.bits_host, p.host_pages, nd, out);
+  __syncthreads();
+  for (long long r = threadIdx.x; r < nd; r += NT) p.own_host[out[r]] = kOwnerReserved;
+  __syncthreads();
+  if (nd == n) return;
+  long long after = 0;   // victims without a copy in the chunks already spread
+  for (long long c = (n + NT - 1) / NT - 1; c >= 0; --c) {
+    const long long i = c * NT + threadIdx.x;
+    int32_t cp = -1;
+    long long d = 0;
+    if (i < n) {
+      cp = clean_copy_of(p, v[i]);
+      d = cp < 0;
+    }
+    long long chunk;
+    const long long excl = block_excl_scan<NT>(d, &chunk);
+    const int32_t val = (i < n && d) ? out[nd - after - chunk + excl] : cp;
+    __syncthreads();
+    if (i < n) out[i] = val;
+    __syncthreads();
+    after += chunk;
+  }
+}
+
 // ---------------------------------------------------------------- import
 __global__ void k_import(DevPool p, const int32_t* __restrict__ placement,
                          const int32_t* __restrict__ ctx) {
@@ -115,6 +154,7 @@ __global__ void k_import(DevPool p, const int32_t* __restrict__ placement,
     const int32_t e = placement[idx];
     p.table[idx] = -1;
     p.mark[idx] = 0;
+    p.shadow[idx] = -1;
     if (b >= nb) {
       if (e != -1) set_error(p.ctl, LV_ERR_BOUNDS, idx);
       continue;
@@ -417,6 +457,36 @@ k_alloc(DevPool p, bool hbm, long long n, int32_t* __restrict__ out, bool inject
   for (long long i = threadIdx.x; i < n; i += kAllocThreads) own[out[i]] = kOwnerReserved;
 }
 
+// Host slots of a swap-out under inclusive tiers (one CTA): victims with a clean
+// copy take it; only the others count against the host tier and reserve slots.
+__global__ void __launch_bounds__(kAllocThreads)
+k_alloc_out(DevPool p, const lv_victim* __restrict__ v, long long n, int32_t* __restrict__ out,
+            bool injected_fail) {
+  __shared__ int ok;
+  __shared__ long long nd_s;
+  long long cnt = 0;
+  for (long long i = threadIdx.x; i < n; i += kAllocThreads) cnt += clean_copy_of(p, v[i]) < 0;
+  long long nd;
+  block_excl_scan<kAllocThreads>(cnt, &nd);
+  if (threadIdx.x == 0) {
+    long long* counter = &p.ctl[C_HOST_ALLOC];
+    const long long before = (long long)atomicAdd(reinterpret_cast<unsigned long long*>(counter),
+                                                  (unsigned long long)nd);
+    ok = before + nd <= p.host_pages && !injected_fail;
+    if (!ok) {
+      atomicAdd(reinterpret_cast<unsigned long long*>(counter), (unsigned long long)(-nd));
+      set_error(p.ctl, LV_ERR_NO_HOST, nd);
+    }
+    nd_s = nd;
+  }
+  __syncthreads();
+  if (!ok) {
+    for (long long i = threadIdx.x; i < n; i += kAllocThreads) out[i] = -1;
+    return;
+  }
+  block_alloc_out<kAllocThreads>(p, v, n, nd_s, out);
+}
+
 // ------------------------------------------------------------------ copy
 constexpr int kCopyThreads = 256;
 constexpr int kCopyUnroll = 4;
@@ -456,12 +526,14 @@ k_swap_out(DevPool p, const lv_victim* __restrict__ v, const int32_t* __restrict
     ok = ok && x.blk < nblocks_of(p, x.sid);
     ok = ok && p.table[(size_t)x.sid * p.maxB + x.blk] == x.page &&
          p.own_hbm[x.page] == owner_key(x.sid, x.blk);
+    const bool clean = ok && clean_copy_of(p, x) == slot;   // its clean copy: nothing to move
     if (j == 0 && threadIdx.x == 0) {
       if (!ok) set_error(p.ctl, LV_ERR_STATE, i);
       else atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PAGES_OUT]), 1ull);
+      if (clean) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_CLEAN_OUT]), 1ull);
       if (commit) commit[i] = lv_remap_entry{x.sid, x.blk, ok ? -(slot + 2) : -1};
     }
-    if (!ok) continue;
+    if (!ok || clean) continue;
     const int4* src = reinterpret_cast<const int4*>(p.kv[j] + (size_t)x.page * p.P);
     int4* dst = reinterpret_cast<int4*>(p.host + ((size_t)slot * p.J + j) * p.P);
     copy_subpage(src, dst, nvec);
@@ -551,12 +623,16 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
     }
     if (!ok) { set_error(p.ctl, sid_ok ? LV_ERR_STATE : LV_ERR_BOUNDS, n_out + i); bad = 1; }
   }
-  __syncthreads();
+  // victims without a clean copy (all of them unless the tiers are inclusive)
+  long long cnt = 0;
+  for (long long i = threadIdx.x; i < n_out; i += kPlanThreads) cnt += clean_copy_of(p, v[i]) < 0;
+  long long n_dirty;
+  block_excl_scan<kPlanThreads>(cnt, &n_dirty);
   if (threadIdx.x == 0 && !bad) {
     // capacity, as the sequential calls see it: host slots before any is freed,
     // HBM pages after the victims' pages are freed
-    if (p.ctl[C_HOST_ALLOC] + n_out > p.host_pages) {
-      set_error(p.ctl, LV_ERR_NO_HOST, n_out);
+    if (p.ctl[C_HOST_ALLOC] + n_dirty > p.host_pages) {
+      set_error(p.ctl, LV_ERR_NO_HOST, n_dirty);
       bad = 1;
     } else if (p.ctl[C_HBM_ALLOC] - n_out + n_in > p.budget) {
       set_error(p.ctl, LV_ERR_NO_HBM, n_in);
@@ -570,19 +646,23 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
     if (threadIdx.x == 0) *n_tasks = 0;
     return;
   }
-  // host slots for the victims
-  if (n_out > 0) block_alloc_lowest<kPlanThreads>(p.bits_host, p.host_pages, n_out, slots);
+  // host slots for the victims: a clean copy, or the lowest free slots in victim order
+  if (n_out > 0) block_alloc_out<kPlanThreads>(p, v, n_out, n_dirty, slots);
   __syncthreads();
-  // out-commit: victims now live in their slots, their pages are free
+  // out-commit: victims now live in their slots, their pages are free; only a
+  // victim that moves bytes tags its page (a clean one has nothing to read)
   const unsigned long long tag = (unsigned long long)(uint32_t)epoch << 32;
   for (long long i = threadIdx.x; i < n_out; i += kPlanThreads) {
     const lv_victim x = v[i];
     const uint32_t key = owner_key(x.sid, x.blk);
-    p.table[(size_t)x.sid * p.maxB + x.blk] = -(slots[i] + 2);
+    const size_t ti = (size_t)x.sid * p.maxB + x.blk;
+    const bool clean = p.incl && p.shadow[ti] == slots[i];
+    p.table[ti] = -(slots[i] + 2);
+    if (clean) p.shadow[ti] = -1;
     p.own_host[slots[i]] = key;
     p.own_hbm[x.page] = kOwnerNone;
     atomicAnd(&p.bits_hbm[x.page >> 5], ~(1u << (x.page & 31)));
-    page_tag[x.page] = tag | (unsigned long long)i;
+    if (!clean) page_tag[x.page] = tag | (unsigned long long)i;
   }
   __syncthreads();
   // HBM pages for the incoming blocks
@@ -596,8 +676,12 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
     const int32_t pg = pages[i];
     p.table[ti] = pg;
     p.own_hbm[pg] = owner_key(sid, b);
-    p.own_host[g] = kOwnerNone;
-    atomicAnd(&p.bits_host[g >> 5], ~(1u << (g & 31)));
+    if (p.incl) {
+      p.shadow[ti] = (int32_t)g;             // the host slot stays as its clean copy
+    } else {
+      p.own_host[g] = kOwnerNone;
+      atomicAnd(&p.bits_host[g >> 5], ~(1u << (g & 31)));
+    }
     int4 t = make_int4(-1, -1, (int32_t)g, pg);
     const unsigned long long pt = page_tag[pg];
     if ((pt >> 32) == (unsigned long long)(uint32_t)epoch && !(pt & kPairedBit)) {
@@ -617,7 +701,8 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
     int32_t pg = -1;
     if (i < n_out) {
       pg = v[i].page;
-      flag = (page_tag[pg] & kPairedBit) ? 0 : 1;
+      const unsigned long long pt = page_tag[pg];
+      flag = ((pt >> 32) == (unsigned long long)(uint32_t)epoch && !(pt & kPairedBit)) ? 1 : 0;
     }
     long long chunk;
     const long long pos = run + block_excl_scan<kPlanThreads>(flag, &chunk);
@@ -626,7 +711,13 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
   }
   if (threadIdx.x == 0) {
     *n_tasks = n_in + run;
-    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HOST_ALLOC]), (unsigned long long)(n_out - n_in));
+    const long long n_clean = n_out - n_dirty;
+    const long long host_delta = p.incl ? n_dirty : n_dirty - n_in;
+    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HOST_ALLOC]), (unsigned long long)host_delta);
+    if (p.incl) {
+      atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_CLEAN]), (unsigned long long)(n_in - n_clean));
+      atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_CLEAN_OUT]), (unsigned long long)n_clean);
+    }
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HBM_ALLOC]), (unsigned long long)(n_in - n_out));
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PAGES_OUT]), (unsigned long long)n_out);
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PAGES_IN]), (unsigned long long)n_in);
@@ -696,8 +787,11 @@ __global__ void k_tasks_out(DevPool p, const lv_victim* __restrict__ v, const in
          p.own_hbm[x.page] == owner_key(x.sid, x.blk);
     if (!ok) set_error(p.ctl, LV_ERR_STATE, i);
     else {
-      t = make_int4(x.page, slot, -1, -1);
       atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PAGES_OUT]), 1ull);
+      if (clean_copy_of(p, x) == slot)        // its clean copy: no task
+        atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_CLEAN_OUT]), 1ull);
+      else
+        t = make_int4(x.page, slot, -1, -1);
     }
     if (commit) commit[i] = lv_remap_entry{x.sid, x.blk, ok ? -(slot + 2) : -1};
   } else if (commit) {
@@ -937,10 +1031,13 @@ constexpr int kRemapThreads = 256;
 
 // One thread per entry.  The allocation counts and the commit counter change
 // by block totals (one atomic per block and counter, not one per entry).
+// Inclusive tiers: a host location may be the block's own clean copy; a block
+// committed to HBM from the host tier keeps its slot as its clean copy; a
+// block committed to another host slot loses its copy.
 __global__ void __launch_bounds__(kRemapThreads)
 k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t epoch) {
   const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
-  bool ok = false, freed_hbm = false, freed_host = false;
+  bool ok = false, freed_hbm = false, freed_host = false, copy_kept = false, copy_gone = false;
   if (i < n) {
     const lv_remap_entry x = e[i];
     int err = 0;
@@ -960,7 +1057,9 @@ k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t ep
       } else if (x.loc <= -2) {
         const long long h = -(long long)x.loc - 2;
         if (h >= p.host_pages) err = LV_ERR_BOUNDS;
-        else if (atomicCAS(&p.own_host[h], kOwnerReserved, key) != kOwnerReserved) err = LV_ERR_DOUBLE_MAP;
+        else if (atomicCAS(&p.own_host[h], kOwnerReserved, key) != kOwnerReserved &&
+                 !(p.incl && p.shadow[ti] == (int32_t)h && p.own_host[h] == key))
+          err = LV_ERR_DOUBLE_MAP;
       } else {
         err = LV_ERR_BOUNDS;
       }
@@ -970,6 +1069,18 @@ k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t ep
     } else {
       const int32_t old = p.table[ti];
       p.table[ti] = x.loc;
+      if (x.loc <= -2 && p.incl) {
+        const int32_t g = p.shadow[ti];
+        if (g >= 0) {                       // the copy becomes the location, or goes
+          p.shadow[ti] = -1;
+          copy_gone = true;
+          if ((long long)g != -(long long)x.loc - 2) {
+            p.own_host[g] = kOwnerNone;
+            atomicAnd(&p.bits_host[g >> 5], ~(1u << (g & 31)));
+            freed_host = true;
+          }
+        }
+      }
       // the old location belongs to this block alone (one entry per block per call)
       if (old >= 0 && old < p.hbm_pages) {
         if (p.own_hbm[old] != key) set_error(p.ctl, LV_ERR_STATE, i);
@@ -979,9 +1090,14 @@ k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t ep
       } else if (old <= -2 && (-(long long)old - 2) < p.host_pages) {
         const long long h = -(long long)old - 2;
         if (p.own_host[h] != key) set_error(p.ctl, LV_ERR_STATE, i);
-        p.own_host[h] = kOwnerNone;
-        atomicAnd(&p.bits_host[h >> 5], ~(1u << (h & 31)));
-        freed_host = true;
+        if (p.incl && x.loc >= 0) {         // back in HBM: the host slot stays as its clean copy
+          p.shadow[ti] = (int32_t)h;
+          copy_kept = true;
+        } else {
+          p.own_host[h] = kOwnerNone;
+          atomicAnd(&p.bits_host[h >> 5], ~(1u << (h & 31)));
+          freed_host = true;
+        }
       }
       ok = true;
     }
@@ -989,10 +1105,13 @@ k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t ep
   const int n_ok = __syncthreads_count(ok);
   const int n_hbm = __syncthreads_count(freed_hbm);
   const int n_host = __syncthreads_count(freed_host);
+  int n_clean = 0;
+  if (p.incl) n_clean = __syncthreads_count(copy_kept) - __syncthreads_count(copy_gone);
   if (threadIdx.x == 0) {
     if (n_hbm) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HBM_ALLOC]), (unsigned long long)-(long long)n_hbm);
     if (n_host) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HOST_ALLOC]), (unsigned long long)-(long long)n_host);
     if (n_ok) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_REMAP]), (unsigned long long)n_ok);
+    if (n_clean) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_CLEAN]), (unsigned long long)(long long)n_clean);
   }
 }
 
@@ -1012,9 +1131,13 @@ __global__ void k_cancel(DevPool p, const int32_t* __restrict__ locs, long long 
     set_error(p.ctl, LV_ERR_BOUNDS, i);
     return;
   }
-  // only a pending reservation can be released
-  if (atomicCAS(&own[idx], kOwnerReserved, kOwnerNone) != kOwnerReserved) {
-    set_error(p.ctl, LV_ERR_STATE, i);
+  // only a pending reservation can be released; a clean copy was never reserved
+  const uint32_t o = atomicCAS(&own[idx], kOwnerReserved, kOwnerNone);
+  if (o != kOwnerReserved) {
+    const int32_t os = (int32_t)(o >> 16), ob = (int32_t)(o & 0xFFFFu);
+    const bool copy = p.incl && which == C_HOST_ALLOC && o != kOwnerNone && os < p.S &&
+                      ob < p.maxB && p.shadow[(size_t)os * p.maxB + ob] == idx;
+    if (!copy) set_error(p.ctl, LV_ERR_STATE, i);
     return;
   }
   const uint32_t m = 1u << (idx & 31);
@@ -1075,6 +1198,20 @@ k_append(DevPool p, int32_t sid, int32_t n_tokens, int32_t* __restrict__ pages,
     p.own_hbm[pg] = owner_key(sid, b);
   }
   if (threadIdx.x == 0) {
+    // inclusive tiers: the partially filled last block gains rows, its clean copy is stale
+    const long long old_ctx = ctx_s - n_tokens;
+    if (p.incl && n_tokens > 0 && nb_s > 0 && old_ctx % p.T != 0) {
+      const size_t ti = (size_t)sid * p.maxB + (nb_s - 1);
+      const int32_t g = p.shadow[ti];
+      if (g >= 0 && g < p.host_pages) {
+        p.shadow[ti] = -1;
+        p.own_host[g] = kOwnerNone;
+        atomicAnd(&p.bits_host[g >> 5], ~(1u << (g & 31)));
+        atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HOST_ALLOC]), (unsigned long long)-1ll);
+        atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_CLEAN]), (unsigned long long)-1ll);
+        atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_CLEAN_DROPPED]), 1ull);
+      }
+    }
     p.sess[sid].ctx_tokens = (int32_t)ctx_s;
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_APPENDED]), (unsigned long long)m);
     if (count) *count = (int32_t)m;
@@ -1274,6 +1411,13 @@ cudaError_t configure_kernels() {
 cudaError_t launch_alloc(const DevPool& p, bool hbm, int64_t n, int32_t* out, cudaStream_t s,
                          bool injected_fail) {
   k_alloc<<<1, kAllocThreads, 0, s>>>(p, hbm, n, out, injected_fail);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_alloc_out(const DevPool& p, const lv_victim* v, int64_t n, int32_t* out,
+                             cudaStream_t s, bool injected_fail) {
+  if (n <= 0) return cudaSuccess;
+  k_alloc_out<<<1, kAllocThreads, 0, s>>>(p, v, n, out, injected_fail);
   return cudaGetLastError();
 }
 

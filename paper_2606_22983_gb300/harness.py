@@ -31,7 +31,7 @@ def pool_for(workload, device=None, stream=None, kv=None) -> KVPool:
                   host_pages=spec.host_pages, reply_prior_us=spec.reply_prior_us,
                   protect_us=spec.protect_us, unit_us=spec.unit_us,
                   within_order=spec.within_order, t_play_mode=spec.t_play_mode,
-                  device=device, stream=stream, kv=kv, policy=spec.policy)
+                  device=device, stream=stream, kv=kv, policy=spec.policy, tiers=spec.tiers)
     init = workload.init
     pool.import_placement(init.placement, init.ctx_tokens)
     st = np.zeros(spec.n_sessions, dtype=lv.SESSION_DTYPE)

@@ -29,6 +29,7 @@ LV_PLAY_PLAYBACK, LV_PLAY_COUNTERS = 0, 1
 LV_MODE_AUTO, LV_MODE_ZERO_COPY, LV_MODE_STAGED = 0, 1, 2
 LV_SELECT_FALLBACK = 1
 LV_POLICY_NEXT_USE, LV_POLICY_LRU = 0, 1
+LV_TIERS_EXCLUSIVE, LV_TIERS_INCLUSIVE = 0, 1
 LV_RUNNING, LV_IMMEDIATE, LV_RESP_OPEN, LV_DONE_VALID = 1, 2, 4, 8
 (LV_EV_TURN_BEGIN, LV_EV_TURN_END, LV_EV_PLAYBACK, LV_EV_SPEECH_START, LV_EV_BARGE_IN,
  LV_EV_SPEECH_STOP, LV_EV_PRELOADED, LV_EV_UNPROTECT) = 1, 2, 3, 4, 5, 6, 7, 8
@@ -49,7 +50,8 @@ class lv_pool_desc(ctypes.Structure):
                 ("host_pages", ctypes.c_int64), ("hbm_kv", ctypes.POINTER(ctypes.c_void_p)),
                 ("host_kv", ctypes.c_void_p), ("reply_prior_us", ctypes.c_int64),
                 ("protect_us", ctypes.c_int64), ("unit_us", ctypes.c_int64),
-                ("t_play_mode", ctypes.c_int32), ("policy", ctypes.c_int32)]
+                ("t_play_mode", ctypes.c_int32), ("policy", ctypes.c_int32),
+                ("tiers", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
 class lv_stats(ctypes.Structure):
@@ -58,7 +60,7 @@ class lv_stats(ctypes.Structure):
         "error_detail", "last_select_count", "last_select_total", "selects", "victims",
         "shortfalls", "pages_out", "pages_in", "bytes_out", "bytes_in", "remap_entries",
         "appended_pages", "cancels", "events", "fallback_selects", "preloads",
-        "preloads_skipped")]
+        "preloads_skipped", "clean_copies", "clean_out", "clean_dropped")]
 
     def as_dict(self):
         return {n: int(getattr(self, n)) for n, _ in self._fields_}

@@ -26,7 +26,8 @@ class KVPool:
                  hbm_budget_pages, host_pages, page_tokens=16, elem_bytes=2,
                  reply_prior_us=3_000_000, protect_us=2_000_000, unit_us=80_000,
                  within_order=lv.LV_SUFFIX_FIRST, t_play_mode=lv.LV_PLAY_PLAYBACK,
-                 device=None, stream=None, kv=None, policy=lv.LV_POLICY_NEXT_USE):
+                 device=None, stream=None, kv=None, policy=lv.LV_POLICY_NEXT_USE,
+                 tiers=lv.LV_TIERS_EXCLUSIVE):
         if not torch.cuda.is_available():
             raise RuntimeError("KVPool needs a CUDA device (liblv has no CPU path)")
         self.device = torch.device(device or "cuda", torch.cuda.current_device()) \
@@ -39,6 +40,7 @@ class KVPool:
         self.hbm_pages, self.budget, self.host_pages = hbm_pages, hbm_budget_pages, host_pages
         self.launches = 0      # liblv kernels launched through this object
         self.policy = policy
+        self.tiers = tiers
         with torch.cuda.device(self.device):
             if kv is None:
                 # one allocation, viewed as 2L sub-page arrays [hbm_pages][P]
@@ -54,7 +56,7 @@ class KVPool:
             d.hbm_kv = ctypes.cast(ptrs, ctypes.POINTER(ctypes.c_void_p))
             d.host_kv = None
             d.reply_prior_us, d.protect_us, d.unit_us = reply_prior_us, protect_us, unit_us
-            d.t_play_mode, d.policy = t_play_mode, policy
+            d.t_play_mode, d.policy, d.tiers = t_play_mode, policy, tiers
             self.handle = lv.lv_pool_create(d, stream)
             cap = max(hbm_budget_pages, max_blocks, 1)
             self.cap = cap

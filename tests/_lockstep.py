@@ -46,6 +46,9 @@ def compare_state(om: OracleManager, pool, where, with_bytes):
     assert st["error"] == 0, (where, st)
     assert st["hbm_allocated"] == int(om.pool.hbm_used.sum()), where
     assert st["host_allocated"] == int(om.pool.host_used.sum()), where
+    assert st["clean_copies"] == om.pool.clean_copies(), where
+    assert st["clean_out"] == om.pool.clean_out, where
+    assert st["clean_dropped"] == om.pool.clean_dropped, where
     gs = pool.get_sessions()
     oa = om.session_arrays()
     for f in SESSION_FIELDS:

@@ -71,6 +71,7 @@ int main(void) {
   F(lv_event, kind); F(lv_event, sid); F(lv_event, t_us); F(lv_event, a); F(lv_event, b);
   F(lv_pool_desc, hbm_pages); F(lv_pool_desc, hbm_kv); F(lv_pool_desc, host_kv);
   F(lv_pool_desc, reply_prior_us); F(lv_pool_desc, t_play_mode); F(lv_pool_desc, policy);
+  F(lv_pool_desc, tiers); F(lv_pool_desc, reserved);
   return 0;
 }
 ''')
