@@ -674,6 +674,7 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
     const size_t ti = (size_t)sid * p.maxB + b;
     const long long g = -(long long)p.table[ti] - 2;
     const int32_t pg = pages[i];
+    const unsigned long long pt = page_tag[pg];   // read before this thread's stores
     p.table[ti] = pg;
     p.own_hbm[pg] = owner_key(sid, b);
     if (p.incl) {
@@ -683,7 +684,6 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
       atomicAnd(&p.bits_host[g >> 5], ~(1u << (g & 31)));
     }
     int4 t = make_int4(-1, -1, (int32_t)g, pg);
-    const unsigned long long pt = page_tag[pg];
     if ((pt >> 32) == (unsigned long long)(uint32_t)epoch && !(pt & kPairedBit)) {
       const long long vi = (long long)(pt & 0x7fffffffull);
       t.x = pg;
@@ -1034,32 +1034,50 @@ constexpr int kRemapThreads = 256;
 // Inclusive tiers: a host location may be the block's own clean copy; a block
 // committed to HBM from the host tier keeps its slot as its clean copy; a
 // block committed to another host slot loses its copy.
+//
+// Every read that does not depend on a check (the block's table entry, the
+// owner word of its old location, its clean-copy slot) is issued first, before
+// any atomic or store: a random load issued after this thread's stores costs
+// several times more.  The early reads are race-free within one call: a block
+// has at most one accepted entry (the epoch mark), and another entry can take
+// an owned location only through a CAS, which then fails.
 __global__ void __launch_bounds__(kRemapThreads)
 k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t epoch) {
   const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
   bool ok = false, freed_hbm = false, freed_host = false, copy_kept = false, copy_gone = false;
   if (i < n) {
     const lv_remap_entry x = e[i];
+    const bool in_range = x.sid >= 0 && x.sid < p.S && x.blk >= 0 && x.blk < p.maxB;
+    const size_t ti = in_range ? (size_t)x.sid * p.maxB + x.blk : 0;
+    // early reads
+    const int32_t old = in_range ? p.table[ti] : -1;
+    const long long old_slot = -(long long)old - 2;
+    const bool old_hbm = old >= 0 && old < p.hbm_pages;
+    const bool old_host = old <= -2 && old_slot < p.host_pages;
+    uint32_t old_owner = kOwnerNone;
+    if (old_hbm) old_owner = p.own_hbm[old];
+    else if (old_host) old_owner = p.own_host[old_slot];
+    const int32_t g = (in_range && p.incl) ? p.shadow[ti] : -1;
+    // checks
     int err = 0;
-    size_t ti = 0;
-    if (x.sid < 0 || x.sid >= p.S || x.blk < 0 || x.blk >= nblocks_of(p, x.sid)) {
+    if (!in_range || x.blk >= nblocks_of(p, x.sid)) {
       err = LV_ERR_BOUNDS;
-    } else {
-      ti = (size_t)x.sid * p.maxB + x.blk;
-      if (atomicExch(&p.mark[ti], epoch) == epoch) err = LV_ERR_DOUBLE_MAP;   // same block twice
+    } else if (atomicExch(&p.mark[ti], epoch) == epoch) {
+      err = LV_ERR_DOUBLE_MAP;   // same block twice
     }
     const uint32_t key = err ? 0u : owner_key(x.sid, x.blk);
+    const long long h = -(long long)x.loc - 2;
     if (!err) {
       // the new location must be a reservation nobody owns yet: one CAS checks and takes it
       if (x.loc >= 0) {
         if (x.loc >= p.hbm_pages) err = LV_ERR_BOUNDS;
         else if (atomicCAS(&p.own_hbm[x.loc], kOwnerReserved, key) != kOwnerReserved) err = LV_ERR_DOUBLE_MAP;
       } else if (x.loc <= -2) {
-        const long long h = -(long long)x.loc - 2;
         if (h >= p.host_pages) err = LV_ERR_BOUNDS;
-        else if (atomicCAS(&p.own_host[h], kOwnerReserved, key) != kOwnerReserved &&
-                 !(p.incl && p.shadow[ti] == (int32_t)h && p.own_host[h] == key))
-          err = LV_ERR_DOUBLE_MAP;
+        else {
+          const uint32_t o = atomicCAS(&p.own_host[h], kOwnerReserved, key);
+          if (o != kOwnerReserved && !(p.incl && (long long)g == h && o == key)) err = LV_ERR_DOUBLE_MAP;
+        }
       } else {
         err = LV_ERR_BOUNDS;
       }
@@ -1067,35 +1085,29 @@ k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t ep
     if (err) {
       set_error(p.ctl, err, i);
     } else {
-      const int32_t old = p.table[ti];
       p.table[ti] = x.loc;
-      if (x.loc <= -2 && p.incl) {
-        const int32_t g = p.shadow[ti];
-        if (g >= 0) {                       // the copy becomes the location, or goes
-          p.shadow[ti] = -1;
-          copy_gone = true;
-          if ((long long)g != -(long long)x.loc - 2) {
-            p.own_host[g] = kOwnerNone;
-            atomicAnd(&p.bits_host[g >> 5], ~(1u << (g & 31)));
-            freed_host = true;
-          }
+      if (x.loc <= -2 && g >= 0) {          // the copy becomes the location, or goes
+        p.shadow[ti] = -1;
+        copy_gone = true;
+        if ((long long)g != h) {
+          p.own_host[g] = kOwnerNone;
+          atomicAnd(&p.bits_host[g >> 5], ~(1u << (g & 31)));
+          freed_host = true;
         }
       }
       // the old location belongs to this block alone (one entry per block per call)
-      if (old >= 0 && old < p.hbm_pages) {
-        if (p.own_hbm[old] != key) set_error(p.ctl, LV_ERR_STATE, i);
-        p.own_hbm[old] = kOwnerNone;
-        atomicAnd(&p.bits_hbm[old >> 5], ~(1u << (old & 31)));
-        freed_hbm = true;
-      } else if (old <= -2 && (-(long long)old - 2) < p.host_pages) {
-        const long long h = -(long long)old - 2;
-        if (p.own_host[h] != key) set_error(p.ctl, LV_ERR_STATE, i);
-        if (p.incl && x.loc >= 0) {         // back in HBM: the host slot stays as its clean copy
-          p.shadow[ti] = (int32_t)h;
+      if (old_hbm || old_host) {
+        if (old_owner != key) set_error(p.ctl, LV_ERR_STATE, i);
+        if (old_hbm) {
+          p.own_hbm[old] = kOwnerNone;
+          atomicAnd(&p.bits_hbm[old >> 5], ~(1u << (old & 31)));
+          freed_hbm = true;
+        } else if (p.incl && x.loc >= 0) {   // back in HBM: the host slot stays as its clean copy
+          p.shadow[ti] = (int32_t)old_slot;
           copy_kept = true;
         } else {
-          p.own_host[h] = kOwnerNone;
-          atomicAnd(&p.bits_host[h >> 5], ~(1u << (h & 31)));
+          p.own_host[old_slot] = kOwnerNone;
+          atomicAnd(&p.bits_host[old_slot >> 5], ~(1u << (old_slot & 31)));
           freed_host = true;
         }
       }
