@@ -202,7 +202,7 @@ def ours(args, torch):
     fill_random(pool, args.seed + rank)
     page_bytes = pool.J * pool.P
     gm = KVManager(pool, perms=wl.perms, rank_on="none", mode=args.mode, record=False,
-                   driver=args.driver)
+                   driver=args.driver, async_copy=args.async_copy)
     S = wl.spec.n_sessions
     # the PLAYBACK batches of the device-timed pass, resident before timing
     dev_events = []
@@ -229,6 +229,7 @@ def ours(args, torch):
     t1 = torch.cuda.Event(enable_timing=True)
     t0.record()
     run_turns(gm, wl, W, W + K, dev_events)
+    lv.lv_join(pool.handle, pool.stream)       # every turn's copy is inside the timed region
     t1.record()
     torch.cuda.synchronize()
     if dist:
@@ -334,6 +335,7 @@ def ours(args, torch):
                        "mode": {0: "auto", 1: "zero_copy", 2: "staged"}[args.mode],
                        "driver": args.driver,
                        "tiers": ("exclusive", "inclusive")[args.tiers],
+                       "async_copy": bool(args.async_copy and args.driver == "device"),
                        "l2": "inputs larger than L2 (mean turn moves "
                              f"{mean_turn / 1e6:.0f} MB each way from a 40 GB pool)",
                        "parallelism": f"replicas x{ws}"},
@@ -639,6 +641,9 @@ def main():
                     help="smaller case for profiling: number of sessions")
     ap.add_argument("--budget-pages", type=int, default=0,
                     help="smaller case for profiling: HBM budget in pages")
+    ap.add_argument("--no-async-copy", dest="async_copy", action="store_false",
+                    help="device driver: copy on the caller's stream (no overlap of the next "
+                         "turn's decisions with this turn's copy)")
     ap.add_argument("--tiers", type=int, default=0, choices=(0, 1),
                     help="0 exclusive tiers, 1 inclusive (clean host copies kept)")
     args = ap.parse_args()

@@ -317,8 +317,14 @@ lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_ou
                            const int32_t* blks, int64_t n_in, int32_t* slots_out,
                            int32_t* pages_out, int32_t mode, lv_stream stream);
 
-/* lv_make_resident flags and result */
-enum { LV_RESIDENT_PRELOAD = 1 };
+/* lv_make_resident flags and result.  LV_RESIDENT_ASYNC_COPY (lv_make_resident,
+   lv_turn): the step's page copies run on the pool's own copy stream, after the
+   step's decisions and after every earlier asynchronous copy, so that the work
+   queued next on `stream` (the next step's ranking and planning) overlaps
+   them.  Until lv_join(pool, stream) the moved KV bytes must not be read or
+   written by the caller; every liblv call that moves or reads KV bytes, and
+   lv_sync, joins first by itself. */
+enum { LV_RESIDENT_PRELOAD = 1, LV_RESIDENT_ASYNC_COPY = 2 };
 enum { LV_RESIDENT_DONE = 0, LV_RESIDENT_SKIPPED = 1, LV_RESIDENT_NOTHING = 2,
        LV_RESIDENT_FAILED = 3 /* a device-detected error stopped it (see lv_sync) */ };
 
@@ -329,7 +335,7 @@ typedef struct lv_resident_result {
   int64_t n_loaded;       /* host blocks loaded */
   int64_t n_appended;     /* new pages for appended tokens */
   int32_t status;         /* LV_RESIDENT_DONE / _SKIPPED / _NOTHING */
-  int32_t pad;
+  int32_t sid;            /* the session made resident (lv_turn: the one it picked) */
 } lv_resident_result;
 
 /* Sections 5.1 and 5.2, one step with no host round trip: makes session sid
@@ -375,6 +381,37 @@ lv_status lv_remap(lv_pool* pool, const lv_remap_entry* entries, int64_t n, lv_s
    it is.  Device-detected: LV_ERR_STATE when a location is owned or not
    reserved. */
 lv_status lv_cancel(lv_pool* pool, const int32_t* locs, int64_t n, lv_stream stream);
+
+/* One turn of a voice session as one call (Section 3: the user's input is
+   complete and the request runs; Sections 5.1 and 5.2: its KV is made
+   resident first), with no host round trip.  In stream order on the device:
+   the turn's session is d->sid, or, when d->sid is -1, the first of
+   d->candidates (num_candidates session ids, device or host memory, read at
+   call time) that has at least one block in the host tier -- the first
+   candidate when none has; then LV_EV_TURN_BEGIN at now_us; then
+   lv_make_resident(sid, now_us, append_tokens, foreground); then, unless that
+   failed, LV_EV_TURN_END at now_us with a = reply_audio_us, b = reply_units.
+   The outputs are those of lv_make_resident (each may be NULL), with
+   result.sid the session.  Host-detected: LV_ERR_INVALID.
+   Device-detected: as lv_make_resident, LV_ERR_BOUNDS for a candidate out of
+   range. */
+typedef struct lv_turn_desc {
+  int32_t sid;                 /* the session, or -1: pick from candidates */
+  int32_t num_candidates;      /* 1..max_sessions when sid == -1 */
+  const int32_t* candidates;   /* session ids in pick order */
+  int64_t now_us;              /* the turn's start */
+  int64_t reply_audio_us;      /* LV_EV_TURN_END a: audio of the reply */
+  int64_t reply_units;         /* LV_EV_TURN_END b: reply length in progress units */
+  int32_t append_tokens;       /* context growth (>= 0) */
+  uint32_t flags;              /* 0 or LV_RESIDENT_ASYNC_COPY */
+} lv_turn_desc;
+lv_status lv_turn(lv_pool* pool, const lv_turn_desc* d, lv_victim* victims_out, int32_t* slots_out,
+                  int32_t* blocks_out, int32_t* pages_out, int32_t* append_out,
+                  lv_resident_result* result_out, lv_stream stream);
+
+/* Makes `stream` wait for every page copy issued so far with
+   LV_RESIDENT_ASYNC_COPY (nothing to wait for: no effect). */
+lv_status lv_join(lv_pool* pool, lv_stream stream);
 
 /* The staged path's building blocks (Section 6, offload connector), usable on
    their own: lv_pack_pages gathers the 2L sub-pages of each listed HBM page into

@@ -15,7 +15,15 @@ struct lv_pool {
   int num_sms = 0;
   int32_t epoch = 0;
   int exchange_ctas = 0;           // grid of the exchange copy kernel
-  lv::ResidentScratch rs{};        // lv_make_resident buffers
+  lv::ResidentScratch rs{};        // lv_make_resident / lv_turn buffers
+  // LV_RESIDENT_ASYNC_COPY: the copies run on s_copy; consecutive steps alternate
+  // between two task lists and control-word sets (rs_alt shares everything else)
+  lv::ResidentScratch rs_alt{};
+  uint32_t rs_seq = 0;
+  cudaStream_t s_copy = nullptr;
+  cudaEvent_t ev_planned = nullptr;
+  cudaEvent_t ev_copied[2] = {nullptr, nullptr};
+  bool copied_pending[2] = {false, false};   // an async copy used scratch set b
   // staged path: side streams for the copy engines, a host copy of the tasks, sync events
   cudaStream_t s_d2h = nullptr, s_h2d = nullptr;
   int4* tasks_host = nullptr;
@@ -288,7 +296,38 @@ lv_status staged_move(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStrea
   return st;
 }
 
+// Makes `s` wait for every asynchronous page copy issued so far.
+cudaError_t join_copies(lv_pool* pool, cudaStream_t s) {
+  for (int b = 0; b < 2; ++b) {
+    if (!pool->copied_pending[b]) continue;
+    const cudaError_t e = cudaStreamWaitEvent(s, pool->ev_copied[b], 0);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+// The scratch set of the next device-driven step, ordered on `s` after the
+// copy that last used it (async); a synchronous step first joins every copy.
+cudaError_t next_scratch(lv_pool* pool, cudaStream_t s, bool async, const lv::ResidentScratch** rs,
+                         lv::CopyOffload* off) {
+  const int b = (int)(pool->rs_seq++ & 1u);
+  *rs = b ? &pool->rs_alt : &pool->rs;
+  if (!async) return join_copies(pool, s);
+  if (pool->copied_pending[b]) {
+    const cudaError_t e = cudaStreamWaitEvent(s, pool->ev_copied[b], 0);
+    if (e != cudaSuccess) return e;
+  }
+  *off = lv::CopyOffload{pool->s_copy, pool->ev_planned, pool->ev_copied[b]};
+  pool->copied_pending[b] = true;
+  return cudaSuccess;
+}
+
 void free_pool(lv_pool* pool) {
+  if (pool->s_copy) cudaStreamSynchronize(pool->s_copy);
+  if (pool->s_copy) cudaStreamDestroy(pool->s_copy);
+  if (pool->ev_planned) cudaEventDestroy(pool->ev_planned);
+  for (cudaEvent_t e : pool->ev_copied)
+    if (e) cudaEventDestroy(e);
   for (cudaEvent_t e : pool->sync_events) cudaEventDestroy(e);
   if (pool->s_d2h) cudaStreamDestroy(pool->s_d2h);
   if (pool->s_h2d) cudaStreamDestroy(pool->s_h2d);
@@ -421,8 +460,18 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       (st = dev_alloc(pool, &rs.pages, (size_t)d.maxB)) != LV_OK ||
       (st = dev_alloc(pool, &rs.append, (size_t)d.maxB + 2)) != LV_OK ||
       (st = dev_alloc(pool, &rs.tasks, (size_t)d.budget + d.maxB)) != LV_OK ||
-      (st = dev_alloc(pool, &rs.words, 16)) != LV_OK)
+      (st = dev_alloc(pool, &rs.words, 16)) != LV_OK ||
+      (st = dev_alloc(pool, &rs.hits, (size_t)d.S)) != LV_OK)
     return fail(st);
+  pool->rs_alt = rs;
+  if ((st = dev_alloc(pool, &pool->rs_alt.tasks, (size_t)d.budget + d.maxB)) != LV_OK ||
+      (st = dev_alloc(pool, &pool->rs_alt.words, 16)) != LV_OK)
+    return fail(st);
+  if (cudaStreamCreateWithFlags(&pool->s_copy, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&pool->ev_planned, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&pool->ev_copied[0], cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&pool->ev_copied[1], cudaEventDisableTiming) != cudaSuccess)
+    return fail(LV_ERR_CUDA);
   d.kv = kv_dev;
   if (cudaMemcpyAsync(kv_dev, kv.data(), d.J * sizeof(uint8_t*), cudaMemcpyHostToDevice, s) != cudaSuccess ||
       cudaMemsetAsync(d.sess, 0, d.S * sizeof(lv_session_state), s) != cudaSuccess ||
@@ -487,7 +536,8 @@ lv_status lv_pool_create(const lv_pool_desc* desc, lv_stream stream, lv_pool** o
 lv_status lv_pool_destroy(lv_pool* pool, lv_stream stream) {
   if (!pool) return LV_ERR_INVALID;
   DeviceGuard g(pool->device);
-  cudaError_t e = cudaStreamSynchronize(as_stream(stream));
+  cudaError_t e = join_copies(pool, as_stream(stream));
+  if (e == cudaSuccess) e = cudaStreamSynchronize(as_stream(stream));
   free_pool(pool);
   return e == cudaSuccess ? LV_OK : LV_ERR_CUDA;
 }
@@ -598,6 +648,7 @@ lv_status lv_swap_out(lv_pool* pool, const lv_victim* victims, int64_t n, int32_
   DeviceGuard g(pool->device);
   cudaStream_t s = as_stream(stream);
   try {
+    LV_TRY(join_copies(pool, s));   // earlier asynchronous copies move bytes too
     Staging st(pool, s);
     const void* vin = nullptr;
     void *sdev = nullptr, *cdev = nullptr;
@@ -638,6 +689,7 @@ lv_status lv_swap_in(lv_pool* pool, int32_t sid, const int32_t* blks, int64_t n,
   DeviceGuard g(pool->device);
   cudaStream_t s = as_stream(stream);
   try {
+    LV_TRY(join_copies(pool, s));   // earlier asynchronous copies move bytes too
     Staging st(pool, s);
     const void* bin = nullptr;
     void *pdev = nullptr, *cdev = nullptr;
@@ -678,6 +730,7 @@ lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_ou
   DeviceGuard g(pool->device);
   cudaStream_t s = as_stream(stream);
   try {
+    LV_TRY(join_copies(pool, s));   // earlier asynchronous copies move bytes too
     Staging st(pool, s);
     const void *vin = nullptr, *bin = nullptr;
     void *sdev = nullptr, *pdev = nullptr, *tdev = nullptr, *ndev = nullptr;
@@ -711,39 +764,102 @@ lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_ou
   }
 }
 
+// Optional copies of a device-driven step's decisions (whole buffers: the counts
+// live on the device).
+cudaError_t copy_resident_outputs(lv_pool* pool, int32_t append_tokens, lv_victim* victims_out,
+                                  int32_t* slots_out, int32_t* blocks_out, int32_t* pages_out,
+                                  int32_t* append_out, cudaStream_t s) {
+  const lv::DevPool& d = pool->d;
+  const lv::ResidentScratch& rs = pool->rs;
+  const struct { void* user; const void* dev; size_t bytes; } outs[] = {
+      {victims_out, rs.victims, (size_t)d.budget * sizeof(lv_victim)},
+      {slots_out, rs.slots, (size_t)d.budget * 4},
+      {blocks_out, rs.blocks, (size_t)d.maxB * 4},
+      {pages_out, rs.pages, (size_t)d.maxB * 4},
+      {append_out, rs.append,
+       (size_t)(append_tokens / d.T + 2 < d.maxB + 2 ? append_tokens / d.T + 2 : d.maxB + 2) * 4}};
+  for (const auto& o : outs) {
+    if (!o.user) continue;
+    const cudaError_t e = cudaMemcpyAsync(o.user, o.dev, o.bytes, cudaMemcpyDefault, s);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
 lv_status lv_make_resident(lv_pool* pool, int32_t sid, int64_t now_us, int32_t append_tokens,
                            uint32_t flags, int64_t max_load_pages, lv_victim* victims_out,
                            int32_t* slots_out, int32_t* blocks_out, int32_t* pages_out,
                            int32_t* append_out, lv_resident_result* result_out, lv_stream stream) {
   if (!pool || sid < 0 || sid >= pool->d.S || append_tokens < 0) return LV_ERR_INVALID;
-  if (flags & ~(uint32_t)LV_RESIDENT_PRELOAD) return LV_ERR_INVALID;
+  if (flags & ~(uint32_t)(LV_RESIDENT_PRELOAD | LV_RESIDENT_ASYNC_COPY)) return LV_ERR_INVALID;
   const bool preload = (flags & LV_RESIDENT_PRELOAD) != 0;
+  const bool async = (flags & LV_RESIDENT_ASYNC_COPY) != 0;
   if (preload && append_tokens != 0) return LV_ERR_INVALID;
   if (pool->d.host_pages == 0) return LV_ERR_INVALID;
   DeviceGuard g(pool->device);
   cudaStream_t s = as_stream(stream);
   const DevPool& d = pool->d;
-  const lv::ResidentScratch& rs = pool->rs;
   try {
     Staging st(pool, s);
     void* rdev = nullptr;
     lv_status r;
     if ((r = st.out(result_out, sizeof(lv_resident_result), &rdev, false)) != LV_OK) return r;
     if (++pool->epoch <= 0) pool->epoch = 1;
-    LV_TRY(lv::launch_make_resident(d, rs, sid, now_us, append_tokens, preload, max_load_pages,
+    const lv::ResidentScratch* rs = nullptr;
+    lv::CopyOffload off{};
+    LV_TRY(next_scratch(pool, s, async, &rs, &off));
+    LV_TRY(lv::launch_make_resident(d, *rs, sid, now_us, append_tokens, preload, max_load_pages,
                                     pool->epoch, s, pool->exchange_ctas,
                                     static_cast<lv_resident_result*>(rdev),
-                                    timing_pair(pool, LV_TIMING_EXCHANGE)));
-    // optional copies of the decisions (whole buffers: the counts live on the device)
-    const struct { void* user; const void* dev; size_t bytes; } outs[] = {
-        {victims_out, rs.victims, (size_t)d.budget * sizeof(lv_victim)},
-        {slots_out, rs.slots, (size_t)d.budget * 4},
-        {blocks_out, rs.blocks, (size_t)d.maxB * 4},
-        {pages_out, rs.pages, (size_t)d.maxB * 4},
-        {append_out, rs.append,
-         (size_t)(append_tokens / d.T + 2 < d.maxB + 2 ? append_tokens / d.T + 2 : d.maxB + 2) * 4}};
-    for (const auto& o : outs)
-      if (o.user) LV_TRY(cudaMemcpyAsync(o.user, o.dev, o.bytes, cudaMemcpyDefault, s));
+                                    timing_pair(pool, LV_TIMING_EXCHANGE), nullptr,
+                                    async ? &off : nullptr));
+    LV_TRY(copy_resident_outputs(pool, append_tokens, victims_out, slots_out, blocks_out, pages_out,
+                                 append_out, s));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
+lv_status lv_join(lv_pool* pool, lv_stream stream) {
+  if (!pool) return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  LV_TRY(join_copies(pool, as_stream(stream)));
+  return LV_OK;
+}
+
+lv_status lv_turn(lv_pool* pool, const lv_turn_desc* d, lv_victim* victims_out, int32_t* slots_out,
+                  int32_t* blocks_out, int32_t* pages_out, int32_t* append_out,
+                  lv_resident_result* result_out, lv_stream stream) {
+  if (!pool || !d || d->append_tokens < 0 || (d->flags & ~(uint32_t)LV_RESIDENT_ASYNC_COPY))
+    return LV_ERR_INVALID;
+  const bool async = (d->flags & LV_RESIDENT_ASYNC_COPY) != 0;
+  if (d->sid < -1 || d->sid >= pool->d.S) return LV_ERR_INVALID;
+  if (d->sid == -1 && (d->num_candidates < 1 || d->num_candidates > pool->d.S || !d->candidates))
+    return LV_ERR_INVALID;
+  if (pool->d.host_pages == 0) return LV_ERR_INVALID;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  try {
+    Staging st(pool, s);
+    const void* cdev = nullptr;
+    void* rdev = nullptr;
+    lv_status r;
+    if (d->sid == -1 &&
+        (r = st.in(d->candidates, (size_t)d->num_candidates * 4, &cdev)) != LV_OK)
+      return r;
+    if ((r = st.out(result_out, sizeof(lv_resident_result), &rdev, false)) != LV_OK) return r;
+    if (++pool->epoch <= 0) pool->epoch = 1;
+    const lv::ResidentScratch* rs = nullptr;
+    lv::CopyOffload off{};
+    LV_TRY(next_scratch(pool, s, async, &rs, &off));
+    LV_TRY(lv::launch_turn(pool->d, *rs, d->sid, static_cast<const int32_t*>(cdev),
+                           d->sid == -1 ? d->num_candidates : 0, d->now_us, d->append_tokens,
+                           d->reply_audio_us, d->reply_units, pool->epoch, s, pool->exchange_ctas,
+                           static_cast<lv_resident_result*>(rdev), timing_pair(pool, LV_TIMING_EXCHANGE),
+                           async ? &off : nullptr));
+    LV_TRY(copy_resident_outputs(pool, d->append_tokens, victims_out, slots_out, blocks_out, pages_out,
+                                 append_out, s));
     return st.finish();
   } catch (const std::bad_alloc&) {
     return LV_ERR_OOM;
@@ -766,6 +882,7 @@ void* device_alias(const void* p) {
 lv_status pack_impl(lv_pool* pool, const int32_t* pages, int64_t n, void* run, bool pack, cudaStream_t s) {
   void* rdev = device_alias(run);
   if (!rdev || (reinterpret_cast<uintptr_t>(rdev) & 15)) return LV_ERR_INVALID;
+  LV_TRY(join_copies(pool, s));
   Staging st(pool, s);
   const void* pin = nullptr;
   void* tdev = nullptr;
@@ -949,7 +1066,8 @@ lv_status lv_sync(lv_pool* pool, lv_stream stream) {
   DeviceGuard g(pool->device);
   long long ctl[2] = {0, 0};
   cudaStream_t s = as_stream(stream);
-  if (cudaMemcpyAsync(ctl, pool->d.ctl + lv::C_ERR, sizeof(ctl), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+  if (join_copies(pool, s) != cudaSuccess ||
+      cudaMemcpyAsync(ctl, pool->d.ctl + lv::C_ERR, sizeof(ctl), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
       cudaStreamSynchronize(s) != cudaSuccess)
     return LV_ERR_CUDA;
   return static_cast<lv_status>(ctl[0]);

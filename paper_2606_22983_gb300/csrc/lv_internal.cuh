@@ -82,6 +82,15 @@ struct EventPair {
   cudaEvent_t end;
 };
 
+// Page copies moved off the caller's stream (LV_RESIDENT_ASYNC_COPY): the copy
+// waits for `planned` (recorded on the caller's stream after the plan), runs on
+// `stream`, and records `copied` there.
+struct CopyOffload {
+  cudaStream_t stream;
+  cudaEvent_t planned;
+  cudaEvent_t copied;
+};
+
 // ---- launch wrappers (lv_kernels.cu); each returns cudaGetLastError() ----
 cudaError_t launch_import(const DevPool& p, const int32_t* placement, const int32_t* ctx,
                           cudaStream_t s);
@@ -108,12 +117,14 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
                             int4* tasks, long long* n_tasks, int32_t epoch,
                             unsigned long long* page_tag, cudaStream_t s, int copy_ctas,
                             const long long* counts_dev = nullptr, long long max_units = 0,
-                            const EventPair* ev = nullptr);
+                            const EventPair* ev = nullptr, const long long* sid_dev = nullptr,
+                            const CopyOffload* off = nullptr);
 cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, int32_t epoch,
                          cudaStream_t s);
 cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cudaStream_t s);
 cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32_t* pages,
-                          int32_t* count, cudaStream_t s, const long long* gate = nullptr);
+                          int32_t* count, cudaStream_t s, const long long* gate = nullptr,
+                          const long long* sid_dev = nullptr);
 
 // Device buffers of lv_make_resident, owned by the pool.
 struct ResidentScratch {
@@ -124,11 +135,19 @@ struct ResidentScratch {
   int32_t* append;      // [maxB + 2]
   int4* tasks;          // [budget + maxB]
   long long* words;     // [16]
+  int32_t* hits;        // [S] lv_turn's pick
 };
 cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, int32_t sid,
                                  int64_t now_us, int32_t append_tokens, bool preload,
                                  int64_t max_load, int32_t epoch, cudaStream_t s, int copy_ctas,
-                                 lv_resident_result* result, const EventPair* ev = nullptr);
+                                 lv_resident_result* result, const EventPair* ev = nullptr,
+                                 const long long* sid_dev = nullptr, const CopyOffload* off = nullptr);
+// lv_turn: pick (sid < 0), LV_EV_TURN_BEGIN, make resident, LV_EV_TURN_END
+cudaError_t launch_turn(const DevPool& p, const ResidentScratch& rs, int32_t sid, const int32_t* cand,
+                        int32_t n_cand, int64_t now_us, int32_t append_tokens, int64_t audio_us,
+                        int64_t units, int32_t epoch, cudaStream_t s, int copy_ctas,
+                        lv_resident_result* result, const EventPair* ev = nullptr,
+                        const CopyOffload* off = nullptr);
 cudaError_t launch_counts(const DevPool& p, int32_t* hbm, int32_t* host, cudaStream_t s);
 cudaError_t launch_blocks(const DevPool& p, int32_t sid, int32_t where, int32_t* out,
                           long long* count, cudaStream_t s);

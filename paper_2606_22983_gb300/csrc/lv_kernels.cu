@@ -199,6 +199,65 @@ __global__ void k_session_set(DevPool p, const lv_session_state* __restrict__ in
   p.sess[first + i] = st;
 }
 
+// One monitor event applied to a session's state (Section 3 signals; Section
+// 5.1 reply interval and immediate reuse; Section 5.2 protection).
+__device__ __forceinline__ void apply_event(const DevPool& p, lv_session_state& st, const lv_event& x) {
+  switch (x.kind) {
+    case LV_EV_TURN_BEGIN:
+      st.flags = (st.flags | LV_RUNNING) & ~LV_IMMEDIATE;
+      st.protect_until_us = 0;
+      st.last_use_us = x.t_us;
+      break;
+    case LV_EV_TURN_END:
+      st.last_use_us = x.t_us;
+      st.flags &= ~(LV_RUNNING | LV_DONE_VALID);
+      st.gen_us = x.a;
+      st.play_us = 0;
+      st.reply_tokens = x.b;
+      if (st.gen_us > 0) {
+        st.flags |= LV_RESP_OPEN;
+      } else {
+        st.flags = (st.flags & ~LV_RESP_OPEN) | LV_DONE_VALID;
+        st.t_done_us = x.t_us;
+      }
+      break;
+    case LV_EV_PLAYBACK:
+      if (st.flags & LV_RESP_OPEN) {
+        const long long np = st.play_us + x.a;
+        st.play_us = np < st.gen_us ? np : st.gen_us;
+        if (st.play_us >= st.gen_us) {
+          st.flags = (st.flags & ~LV_RESP_OPEN) | LV_DONE_VALID;
+          st.t_done_us = x.t_us;
+        }
+      }
+      break;
+    case LV_EV_SPEECH_START:
+      st.flags |= LV_IMMEDIATE;
+      break;
+    case LV_EV_BARGE_IN:
+      st.gen_us = st.play_us;
+      st.flags = (st.flags | LV_IMMEDIATE) & ~(LV_RESP_OPEN | LV_DONE_VALID);
+      break;
+    case LV_EV_SPEECH_STOP:
+      if (st.flags & LV_DONE_VALID) {
+        long long xs = x.t_us - st.t_done_us;
+        if (xs < 0) xs = 0;
+        st.reply_ema_us = st.reply_n == 0 ? xs : (3 * st.reply_ema_us + xs) / 4;
+        if (st.reply_n < 0x7fffffff) st.reply_n += 1;
+      }
+      st.flags &= ~(LV_IMMEDIATE | LV_DONE_VALID);
+      break;
+    case LV_EV_PRELOADED:
+      st.protect_until_us = x.t_us + p.protect_us;
+      break;
+    case LV_EV_UNPROTECT:
+      st.protect_until_us = 0;
+      break;
+    default:
+      break;   // reported by the caller
+  }
+}
+
 // One thread per session applies, in order, the events addressed to it.
 __global__ void k_events(DevPool p, const lv_event* __restrict__ ev, long long n) {
   const int s = blockIdx.x * blockDim.x + threadIdx.x;
@@ -216,62 +275,8 @@ __global__ void k_events(DevPool p, const lv_event* __restrict__ ev, long long n
   bool touched = false;
   for (long long e = 0; e < n; ++e) {
     if (ev[e].sid != s) continue;
-    const lv_event x = ev[e];
     touched = true;
-    switch (x.kind) {
-      case LV_EV_TURN_BEGIN:
-        st.flags = (st.flags | LV_RUNNING) & ~LV_IMMEDIATE;
-        st.protect_until_us = 0;
-        st.last_use_us = x.t_us;
-        break;
-      case LV_EV_TURN_END:
-        st.last_use_us = x.t_us;
-        st.flags &= ~(LV_RUNNING | LV_DONE_VALID);
-        st.gen_us = x.a;
-        st.play_us = 0;
-        st.reply_tokens = x.b;
-        if (st.gen_us > 0) {
-          st.flags |= LV_RESP_OPEN;
-        } else {
-          st.flags = (st.flags & ~LV_RESP_OPEN) | LV_DONE_VALID;
-          st.t_done_us = x.t_us;
-        }
-        break;
-      case LV_EV_PLAYBACK:
-        if (st.flags & LV_RESP_OPEN) {
-          const long long np = st.play_us + x.a;
-          st.play_us = np < st.gen_us ? np : st.gen_us;
-          if (st.play_us >= st.gen_us) {
-            st.flags = (st.flags & ~LV_RESP_OPEN) | LV_DONE_VALID;
-            st.t_done_us = x.t_us;
-          }
-        }
-        break;
-      case LV_EV_SPEECH_START:
-        st.flags |= LV_IMMEDIATE;
-        break;
-      case LV_EV_BARGE_IN:
-        st.gen_us = st.play_us;
-        st.flags = (st.flags | LV_IMMEDIATE) & ~(LV_RESP_OPEN | LV_DONE_VALID);
-        break;
-      case LV_EV_SPEECH_STOP:
-        if (st.flags & LV_DONE_VALID) {
-          long long xs = x.t_us - st.t_done_us;
-          if (xs < 0) xs = 0;
-          st.reply_ema_us = st.reply_n == 0 ? xs : (3 * st.reply_ema_us + xs) / 4;
-          if (st.reply_n < 0x7fffffff) st.reply_n += 1;
-        }
-        st.flags &= ~(LV_IMMEDIATE | LV_DONE_VALID);
-        break;
-      case LV_EV_PRELOADED:
-        st.protect_until_us = x.t_us + p.protect_us;
-        break;
-      case LV_EV_UNPROTECT:
-        st.protect_until_us = 0;
-        break;
-      default:
-        break;   // reported above
-    }
+    apply_event(p, st, ev[e]);
   }
   if (touched) p.sess[s] = st;
 }
@@ -591,11 +596,12 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
                 const int32_t* __restrict__ blks, long long n_in, int32_t* __restrict__ slots,
                 int32_t* __restrict__ pages, int4* __restrict__ tasks, long long* n_tasks,
                 int32_t epoch, unsigned long long* __restrict__ page_tag,
-                const long long* __restrict__ counts_dev) {
+                const long long* __restrict__ counts_dev, const long long* __restrict__ sid_dev) {
   if (counts_dev) {          // counts decided on the device (lv_make_resident)
     n_out = counts_dev[0];
     n_in = counts_dev[1];
   }
+  if (sid_dev) sid = (int32_t)*sid_dev;
   __shared__ int bad;
   if (threadIdx.x == 0) bad = 0;
   __syncthreads();
@@ -1160,12 +1166,14 @@ __global__ void k_cancel(DevPool p, const int32_t* __restrict__ locs, long long 
 
 __global__ void __launch_bounds__(kAllocThreads)
 k_append(DevPool p, int32_t sid, int32_t n_tokens, int32_t* __restrict__ pages,
-         int32_t* __restrict__ count, const long long* __restrict__ gate) {
+         int32_t* __restrict__ count, const long long* __restrict__ gate,
+         const long long* __restrict__ sid_dev) {
   __shared__ long long m_s, nb_s, ctx_s;
   if (gate && *gate != 0) {   // an earlier step of lv_make_resident did not complete
     if (threadIdx.x == 0 && count) *count = 0;
     return;
   }
+  if (sid_dev) sid = (int32_t)*sid_dev;
   if (threadIdx.x == 0) {
     long long m = -1;
     if (sid >= 0 && sid < p.S && n_tokens >= 0) {
@@ -1241,13 +1249,23 @@ enum ResWord : int {
   R_GATE = 5,       // 0: the append may run
   R_N_TASKS = 6,
   R_APPENDED = 7,   // int32 count of appended pages, in the low half
-  R_FOUND = 8       // victims the ranking found
+  R_FOUND = 8,      // victims the ranking found
+  R_SID = 9         // lv_turn: the turn's session (-1 when the pick failed)
 };
 
 // One CTA: sid's host-tier blocks (ascending), the deficit k and the admission.
 __global__ void __launch_bounds__(kCensusThreads)
 k_resident_prepare(DevPool p, int32_t sid, int32_t append_tokens, bool preload,
-                   long long max_load, int32_t* __restrict__ blocks, long long* __restrict__ R) {
+                   long long max_load, int32_t* __restrict__ blocks, long long* __restrict__ R,
+                   const long long* __restrict__ sid_dev) {
+  if (sid_dev) sid = (int32_t)*sid_dev;
+  if (sid < 0 || sid >= p.S) {        // lv_turn's pick failed (already reported)
+    if (threadIdx.x == 0) {
+      R[R_K_SELECT] = 0; R[R_N_OUT] = 0; R[R_N_IN] = 0; R[R_STATUS] = LV_RESIDENT_FAILED;
+      R[R_K] = 0; R[R_GATE] = 1; R[R_APPENDED] = 0; R[R_FOUND] = 0;
+    }
+    return;
+  }
   const int32_t nb = nblocks_of(p, sid);
   const int32_t* row = p.table + (size_t)sid * p.maxB;
   long long run = 0;
@@ -1313,8 +1331,10 @@ __global__ void k_resident_gate(DevPool p, bool preload, long long* __restrict__
 }
 
 __global__ void k_resident_finish(DevPool p, int32_t sid, long long now_us, bool preload,
-                                  long long* __restrict__ R, lv_resident_result* __restrict__ out) {
+                                  long long* __restrict__ R, lv_resident_result* __restrict__ out,
+                                  const long long* __restrict__ sid_dev) {
   if (threadIdx.x != 0) return;
+  if (sid_dev) sid = (int32_t)*sid_dev;
   const int status = (int)R[R_STATUS];
   if (preload && status == LV_RESIDENT_DONE) {
     p.sess[sid].protect_until_us = now_us + p.protect_us;   // warmed KV (Section 5.2)
@@ -1328,9 +1348,77 @@ __global__ void k_resident_finish(DevPool p, int32_t sid, long long now_us, bool
     r.n_loaded = R[R_N_IN];
     r.n_appended = (int32_t)R[R_APPENDED];
     r.status = status;
-    r.pad = 0;
+    r.sid = sid;
     *out = r;
   }
+}
+
+// ------------------------------------------------------------------ turn
+// lv_turn's pick: CTA c reports whether candidate c has a block in the host tier.
+__global__ void __launch_bounds__(kCensusThreads)
+k_pick_scan(DevPool p, const int32_t* __restrict__ cand, int32_t* __restrict__ hit) {
+  const int32_t s = cand[blockIdx.x];
+  int any = 0;
+  if (s >= 0 && s < p.S) {
+    const int32_t nb = nblocks_of(p, s);
+    const int32_t* row = p.table + (size_t)s * p.maxB;
+    for (int32_t b = threadIdx.x; b < nb && !any; b += kCensusThreads) any = row[b] <= -2;
+  }
+  any = __syncthreads_or(any);
+  if (threadIdx.x == 0) hit[blockIdx.x] = any;
+}
+
+// The turn's session (sid, or the first candidate with a hit, else the first
+// candidate) into R[R_SID], then LV_EV_TURN_BEGIN for it.
+__global__ void __launch_bounds__(1024)
+k_turn_begin(DevPool p, int32_t sid, const int32_t* __restrict__ cand, int32_t n,
+             const int32_t* __restrict__ hit, long long now_us, long long* __restrict__ R) {
+  __shared__ int first;
+  if (threadIdx.x == 0) first = n;
+  __syncthreads();
+  if (sid < 0) {
+    int mine = n;
+    for (int c = threadIdx.x; c < n; c += blockDim.x)
+      if (hit[c]) { mine = c; break; }
+    if (mine < n) atomicMin(&first, mine);
+  }
+  __syncthreads();
+  if (threadIdx.x != 0) return;
+  if (sid < 0) {
+    sid = cand[first < n ? first : 0];
+    if (sid < 0 || sid >= p.S) {
+      set_error(p.ctl, LV_ERR_BOUNDS, first < n ? first : 0);
+      R[R_SID] = -1;
+      return;
+    }
+  }
+  R[R_SID] = sid;
+  lv_session_state st = p.sess[sid];
+  lv_event x{};
+  x.kind = LV_EV_TURN_BEGIN;
+  x.sid = sid;
+  x.t_us = now_us;
+  apply_event(p, st, x);
+  p.sess[sid] = st;
+  atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_EVENTS]), 1ull);
+}
+
+// LV_EV_TURN_END for the turn's session, unless its KV could not be made resident.
+__global__ void k_turn_end(DevPool p, long long now_us, long long audio_us, long long units,
+                           const long long* __restrict__ R) {
+  if (threadIdx.x != 0) return;
+  const long long sid = R[R_SID];
+  if (sid < 0 || sid >= p.S || R[R_STATUS] == LV_RESIDENT_FAILED) return;
+  lv_session_state st = p.sess[sid];
+  lv_event x{};
+  x.kind = LV_EV_TURN_END;
+  x.sid = (int32_t)sid;
+  x.t_us = now_us;
+  x.a = audio_us;
+  x.b = units;
+  apply_event(p, st, x);
+  p.sess[sid] = st;
+  atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_EVENTS]), 1ull);
 }
 
 // ----------------------------------------------------------------- views
@@ -1458,36 +1546,64 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
                             const int32_t* blks, int64_t n_in, int32_t* slots, int32_t* pages,
                             int4* tasks, long long* n_tasks, int32_t epoch,
                             unsigned long long* page_tag, cudaStream_t s, int copy_ctas,
-                            const long long* counts_dev, long long max_units, const EventPair* ev) {
+                            const long long* counts_dev, long long max_units, const EventPair* ev,
+                            const long long* sid_dev, const CopyOffload* off) {
   k_exchange_plan<<<1, kPlanThreads, 0, s>>>(p, v, n_out, sid, blks, n_in, slots, pages, tasks,
-                                             n_tasks, epoch, page_tag, counts_dev);
+                                             n_tasks, epoch, page_tag, counts_dev, sid_dev);
   const long long units = counts_dev ? max_units : (n_out + n_in) * (long long)p.J;
-  if (ev) cudaEventRecord(ev->start, s);
-  k_exchange_copy<<<blocks_for(units, 1, copy_ctas), kCopyThreads, 0, s>>>(p, tasks, n_tasks);
-  if (ev) cudaEventRecord(ev->end, s);
+  cudaStream_t cs = s;
+  if (off) {
+    cudaError_t e = cudaEventRecord(off->planned, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(off->stream, off->planned, 0);
+    if (e != cudaSuccess) return e;
+    cs = off->stream;
+  }
+  if (ev) cudaEventRecord(ev->start, cs);
+  k_exchange_copy<<<blocks_for(units, 1, copy_ctas), kCopyThreads, 0, cs>>>(p, tasks, n_tasks);
+  if (ev) cudaEventRecord(ev->end, cs);
+  if (off) {
+    const cudaError_t e = cudaEventRecord(off->copied, cs);
+    if (e != cudaSuccess) return e;
+  }
   return cudaGetLastError();
 }
 
 cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, int32_t sid,
                                  int64_t now_us, int32_t append_tokens, bool preload,
                                  int64_t max_load, int32_t epoch, cudaStream_t s, int copy_ctas,
-                                 lv_resident_result* result, const EventPair* ev) {
+                                 lv_resident_result* result, const EventPair* ev,
+                                 const long long* sid_dev, const CopyOffload* off) {
   long long* R = rs.words;
   k_resident_prepare<<<1, kCensusThreads, 0, s>>>(p, sid, append_tokens, preload, max_load,
-                                                  rs.blocks, R);
+                                                  rs.blocks, R, sid_dev);
   cudaError_t e = launch_select(p, now_us, 0, !preload, rs.victims, nullptr, s, 0, R + R_K_SELECT);
   if (e != cudaSuccess) return e;
   k_resident_gate<<<1, 32, 0, s>>>(p, preload, R);
   const long long max_units = ((long long)p.budget + p.maxB) * p.J;
   e = launch_exchange(p, rs.victims, 0, sid, rs.blocks, 0, rs.slots, rs.pages, rs.tasks,
-                      R + R_N_TASKS, epoch, p.page_tag, s, copy_ctas, R + R_N_OUT, max_units, ev);
+                      R + R_N_TASKS, epoch, p.page_tag, s, copy_ctas, R + R_N_OUT, max_units, ev,
+                      sid_dev, off);
   if (e != cudaSuccess) return e;
   if (append_tokens > 0) {
     e = launch_append(p, sid, append_tokens, rs.append, reinterpret_cast<int32_t*>(R + R_APPENDED), s,
-                      R + R_GATE);
+                      R + R_GATE, sid_dev);
     if (e != cudaSuccess) return e;
   }
-  k_resident_finish<<<1, 32, 0, s>>>(p, sid, now_us, preload, R, result);
+  k_resident_finish<<<1, 32, 0, s>>>(p, sid, now_us, preload, R, result, sid_dev);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_turn(const DevPool& p, const ResidentScratch& rs, int32_t sid, const int32_t* cand,
+                        int32_t n_cand, int64_t now_us, int32_t append_tokens, int64_t audio_us,
+                        int64_t units, int32_t epoch, cudaStream_t s, int copy_ctas,
+                        lv_resident_result* result, const EventPair* ev, const CopyOffload* off) {
+  long long* R = rs.words;
+  if (sid < 0) k_pick_scan<<<n_cand, kCensusThreads, 0, s>>>(p, cand, rs.hits);
+  k_turn_begin<<<1, 1024, 0, s>>>(p, sid, cand, n_cand, rs.hits, now_us, R);
+  cudaError_t e = launch_make_resident(p, rs, sid, now_us, append_tokens, false, -1, epoch, s,
+                                       copy_ctas, result, ev, R + R_SID, off);
+  if (e != cudaSuccess) return e;
+  k_turn_end<<<1, 32, 0, s>>>(p, now_us, audio_us, units, R);
   return cudaGetLastError();
 }
 
@@ -1555,7 +1671,7 @@ cudaError_t launch_exchange_plan(const DevPool& p, const lv_victim* v, int64_t n
                                  int4* tasks, long long* n_tasks, int32_t epoch,
                                  unsigned long long* page_tag, cudaStream_t s) {
   k_exchange_plan<<<1, kPlanThreads, 0, s>>>(p, v, n_out, sid, blks, n_in, slots, pages, tasks,
-                                             n_tasks, epoch, page_tag, nullptr);
+                                             n_tasks, epoch, page_tag, nullptr, nullptr);
   return cudaGetLastError();
 }
 
@@ -1571,8 +1687,9 @@ cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cuda
 }
 
 cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32_t* pages,
-                          int32_t* count, cudaStream_t s, const long long* gate) {
-  k_append<<<1, kAllocThreads, 0, s>>>(p, sid, n_tokens, pages, count, gate);
+                          int32_t* count, cudaStream_t s, const long long* gate,
+                          const long long* sid_dev) {
+  k_append<<<1, kAllocThreads, 0, s>>>(p, sid, n_tokens, pages, count, gate, sid_dev);
   return cudaGetLastError();
 }
 

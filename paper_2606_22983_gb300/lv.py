@@ -30,6 +30,7 @@ LV_MODE_AUTO, LV_MODE_ZERO_COPY, LV_MODE_STAGED = 0, 1, 2
 LV_SELECT_FALLBACK = 1
 LV_POLICY_NEXT_USE, LV_POLICY_LRU = 0, 1
 LV_TIERS_EXCLUSIVE, LV_TIERS_INCLUSIVE = 0, 1
+LV_RESIDENT_ASYNC_COPY = 2
 LV_RUNNING, LV_IMMEDIATE, LV_RESP_OPEN, LV_DONE_VALID = 1, 2, 4, 8
 (LV_EV_TURN_BEGIN, LV_EV_TURN_END, LV_EV_PLAYBACK, LV_EV_SPEECH_START, LV_EV_BARGE_IN,
  LV_EV_SPEECH_STOP, LV_EV_PRELOADED, LV_EV_UNPROTECT) = 1, 2, 3, 4, 5, 6, 7, 8
@@ -52,6 +53,13 @@ class lv_pool_desc(ctypes.Structure):
                 ("protect_us", ctypes.c_int64), ("unit_us", ctypes.c_int64),
                 ("t_play_mode", ctypes.c_int32), ("policy", ctypes.c_int32),
                 ("tiers", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+class lv_turn_desc(ctypes.Structure):
+    _fields_ = [("sid", ctypes.c_int32), ("num_candidates", ctypes.c_int32),
+                ("candidates", ctypes.c_void_p), ("now_us", ctypes.c_int64),
+                ("reply_audio_us", ctypes.c_int64), ("reply_units", ctypes.c_int64),
+                ("append_tokens", ctypes.c_int32), ("flags", ctypes.c_uint32)]
 
 
 class lv_stats(ctypes.Structure):
@@ -104,7 +112,7 @@ SESSION_DTYPE = np.dtype([("ctx_tokens", "<i4"), ("flags", "<i4"), ("gen_us", "<
 EVENT_DTYPE = np.dtype([("kind", "<i4"), ("sid", "<i4"), ("t_us", "<i8"), ("a", "<i8"), ("b", "<i8")])
 VICTIM_DTYPE = np.dtype([("sid", "<i4"), ("blk", "<i4"), ("page", "<i4")])
 RESIDENT_DTYPE = np.dtype([("k", "<i8"), ("n_found", "<i8"), ("n_victims", "<i8"), ("n_loaded", "<i8"),
-                           ("n_appended", "<i8"), ("status", "<i4"), ("pad", "<i4")])
+                           ("n_appended", "<i8"), ("status", "<i4"), ("sid", "<i4")])
 REMAP_DTYPE = np.dtype([("sid", "<i4"), ("blk", "<i4"), ("loc", "<i4")])
 assert SESSION_DTYPE.itemsize == 72 and EVENT_DTYPE.itemsize == 32
 assert VICTIM_DTYPE.itemsize == 12 and REMAP_DTYPE.itemsize == 12
@@ -128,6 +136,8 @@ def _load():
         "lv_swap_in": [vp, i32, vp, i64, vp, vp, i32, vp],
         "lv_swap_exchange": [vp, vp, i64, i32, vp, i64, vp, vp, i32, vp],
         "lv_make_resident": [vp, i32, i64, i32, u32, i64, vp, vp, vp, vp, vp, vp, vp],
+        "lv_turn": [vp, ctypes.POINTER(lv_turn_desc), vp, vp, vp, vp, vp, vp, vp],
+        "lv_join": [vp, vp],
         "lv_timing_enable": [vp, i32],
         "lv_pack_pages": [vp, vp, i64, vp, vp],
         "lv_schedule": [vp, ctypes.POINTER(lv_sched_params), vp, i32, vp, vp, vp],
@@ -171,7 +181,7 @@ EXPORTED = ("lv_pool_create", "lv_pool_destroy", "lv_pool_host_ptr", "lv_pool_im
             "lv_get_stats", "lv_clear_error", "lv_status_str", "lv_version",
             "lv_select_victims_noalloc", "lv_timing_enable", "lv_timing_read", "lv_pack_pages",
             "lv_unpack_pages", "lv_pool_host_device_ptr", "lv_schedule", "lv_inject_fault",
-            "lv_selftest_wait")
+            "lv_selftest_wait", "lv_turn", "lv_join")
 
 
 def lib():
@@ -282,6 +292,21 @@ def lv_make_resident(pool, sid, now_us, append_tokens, flags, max_load_pages, vi
                                  ptr(victims_out), ptr(slots_out), ptr(blocks_out), ptr(pages_out),
                                  ptr(append_out), ptr(result_out), stream_handle(stream)),
            "lv_make_resident")
+
+
+def lv_turn(pool, sid, now_us, append_tokens, reply_audio_us, reply_units, outs=(None,) * 5,
+            result_out=None, candidates=None, num_candidates=0, stream=None, flags=0):
+    """One turn (pick when sid == -1, turn begin, make resident, turn end); outs =
+    (victims, slots, blocks, pages, append) as for lv_make_resident."""
+    d = lv_turn_desc(sid=sid, num_candidates=num_candidates, candidates=ptr(candidates),
+                     now_us=now_us, reply_audio_us=reply_audio_us, reply_units=reply_units,
+                     append_tokens=append_tokens, flags=flags)
+    _check(_lib.lv_turn(pool, ctypes.byref(d), *(ptr(o) for o in outs), ptr(result_out),
+                        stream_handle(stream)), "lv_turn")
+
+
+def lv_join(pool, stream=None):
+    _check(_lib.lv_join(pool, stream_handle(stream)), "lv_join")
 
 
 def lv_remap(pool, entries, n, stream=None):

@@ -51,8 +51,12 @@ def _event(kind, sid, t, a=0, b=0):
 
 class KVManager:
     def __init__(self, pool: KVPool, perms=None, on_append=None, rank_on="none", admit=None,
-                 mode=lv.LV_MODE_AUTO, record=True, driver="device", order_fn=None):
+                 mode=lv.LV_MODE_AUTO, record=True, driver="device", order_fn=None,
+                 async_copy=False):
         self.pool = pool
+        # device driver: turns' page copies on the pool's copy stream, overlapping the
+        # next turn's decisions (LV_RESIDENT_ASYNC_COPY); pool.sync() joins them
+        self.async_copy = async_copy
         self.perms = perms
         self.on_append = on_append      # callback(sid, old_ctx, new_ctx, pages) after growth
         self.rank_on = rank_on          # 'all' events, 'turns' only, or 'none'
@@ -66,6 +70,10 @@ class KVManager:
         self.driver = driver
         self.order_fn = order_fn        # (key, blocks) -> blocks, for TURN_SCATTER
         self.res_h = torch.zeros(lv.RESIDENT_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
+        # the turn-target candidate rows, resident for lv_turn's on-device pick
+        self.perms_dev = None
+        if perms is not None and len(perms):
+            self.perms_dev = torch.from_numpy(np.ascontiguousarray(perms, dtype=np.int32)).to(pool.device)
         self.counters = dict(victims=0, pages_out=0, pages_in=0, preloads=0,
                              preload_skipped=0, turns=0, sync_loads=0, appended=0)
         self.bytes_moved = 0
@@ -131,6 +139,53 @@ class KVManager:
         if status == lv.LV_RESIDENT_DONE and append_tokens and self.on_append is not None:
             self.on_append(sid, old_ctx, old_ctx + append_tokens)
         return status
+
+    def _device_turn(self, sid, row, now_us, append_tokens, reply_us, reply_units, rec):
+        """One lv_turn: (pick,) turn begin, make resident, turn end -- no host round trip
+        unless the decisions are recorded.  Returns the session id (-1 when not read back)."""
+        pool = self.pool
+        cand = self.perms_dev[row] if sid < 0 else None
+        rec_bufs = self.record or (self.on_append is not None and append_tokens > 0)
+        outs = (pool.victims, pool.slots, pool.blks, pool.pages, pool.app) if self.record else (None,) * 5
+        lv.lv_turn(pool.handle, sid, now_us, append_tokens, reply_us, reply_units, outs, self.res_h,
+                   cand, int(cand.numel()) if cand is not None else 0, pool.stream,
+                   lv.LV_RESIDENT_ASYNC_COPY if self.async_copy else 0)
+        pool.launches += 10 + (1 if sid < 0 else 0) + (1 if append_tokens else 0)
+        if not rec_bufs:
+            return sid
+        pool.sync(raise_on_error=False)
+        r = self.res_h.numpy().view(lv.RESIDENT_DTYPE)[0]
+        sid = int(r["sid"])
+        status = int(r["status"])
+        if status == lv.LV_RESIDENT_FAILED:
+            raise lv.LvError(pool.sync(raise_on_error=False) or lv.LV_ERR_NO_HBM, f"turn of session {sid}")
+        k, found, nv, nl, na = (int(r["k"]), int(r["n_found"]), int(r["n_victims"]),
+                                int(r["n_loaded"]), int(r["n_appended"]))
+        rec["k"] = k
+        if self.record:
+            if k > 0:
+                rec["victims"] = pool.victims[:found].cpu().numpy().astype(np.int64)
+                self.last_readback_bytes += found * 12
+            if nv:
+                rec["slots"] = pool.slots[:nv].cpu().numpy().astype(np.int64)
+                self.last_readback_bytes += nv * 4
+            if nl:
+                rec["in_blocks"] = pool.blks[:nl].cpu().numpy().astype(np.int64)
+                rec["in_pages"] = pool.pages[:nl].cpu().numpy().astype(np.int64)
+                self.last_readback_bytes += nl * 8
+            if append_tokens:
+                rec["append_pages"] = pool.app[:na].cpu().numpy().astype(np.int64)
+        self.counters["victims"] += nv
+        self.counters["pages_out"] += nv
+        self.counters["pages_in"] += nl
+        self.counters["appended"] += na
+        self.bytes_moved += (nv + nl) * pool.J * pool.P
+        if nl:
+            self.counters["sync_loads"] += 1
+        if append_tokens and self.on_append is not None:
+            new_ctx = self.ctx_tokens(sid)
+            self.on_append(sid, new_ctx - append_tokens, new_ctx)
+        return sid
 
     def make_resident(self, sid, now_us, append_tokens, foreground, rec, order_key=None):
         if self.driver == "device" and order_key is None:
@@ -306,6 +361,9 @@ class KVManager:
             pool.events(_event(_STATE_EVENT[kind], sid, t, a))
             if kind in (EV_SPEECH_START, EV_BARGE_IN):
                 self.preload(sid, t, rec)
+        elif kind in (EV_TURN, EV_TURN_ANY) and self.driver == "device":
+            sid = self._device_turn(sid if kind == EV_TURN else -1, d, t, a, b, c, rec)
+            self.counters["turns"] += 1
         elif kind in (EV_TURN, EV_TURN_ANY, EV_TURN_SCATTER):
             order_key = None
             if kind == EV_TURN_SCATTER:

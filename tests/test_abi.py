@@ -64,6 +64,11 @@ int main(void) {
   F(lv_request, play_buffer_us); F(lv_request, kv_needed);
   F(lv_resident_result, k); F(lv_resident_result, n_found); F(lv_resident_result, n_victims);
   F(lv_resident_result, n_loaded); F(lv_resident_result, n_appended); F(lv_resident_result, status);
+  F(lv_resident_result, sid);
+  printf("sizeof lv_turn_desc %zu\n", sizeof(lv_turn_desc));
+  F(lv_turn_desc, sid); F(lv_turn_desc, num_candidates); F(lv_turn_desc, candidates);
+  F(lv_turn_desc, now_us); F(lv_turn_desc, reply_audio_us); F(lv_turn_desc, reply_units);
+  F(lv_turn_desc, append_tokens); F(lv_turn_desc, flags);
   F(lv_session_state, ctx_tokens); F(lv_session_state, flags); F(lv_session_state, gen_us);
   F(lv_session_state, play_us); F(lv_session_state, t_done_us); F(lv_session_state, reply_ema_us);
   F(lv_session_state, reply_n); F(lv_session_state, reply_tokens); F(lv_session_state, protect_until_us);
@@ -95,6 +100,9 @@ int main(void) {
     assert got["lv_resident_result"] == lv.RESIDENT_DTYPE.itemsize
     assert got["lv_request"] == lv.REQUEST_DTYPE.itemsize == 48
     assert got["lv_sched_params"] == ctypes.sizeof(lv.lv_sched_params)
+    assert got["lv_turn_desc"] == ctypes.sizeof(lv.lv_turn_desc)
+    for name, _ in lv.lv_turn_desc._fields_:
+        assert getattr(lv.lv_turn_desc, name).offset == got[f"lv_turn_desc.{name}"][0], name
     assert got["lv_request.play_buffer_us"][0] == lv.REQUEST_DTYPE.fields["play_buffer_us"][1]
     assert got["lv_request.kv_needed"][0] == lv.REQUEST_DTYPE.fields["kv_needed"][1]
     for name in lv.RESIDENT_DTYPE.names:

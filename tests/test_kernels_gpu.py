@@ -284,3 +284,81 @@ def test_degenerate_sizes_and_host_pointer_arguments():
         assert np.array_equal(pool.host[0], pool.kv[:, 7].cpu().numpy())
     finally:
         pool.close()
+
+
+def test_turn_picks_the_first_candidate_with_host_blocks():
+    """lv_turn with sid = -1: the first listed session that has a block in the host
+    tier (else the first listed), then turn begin, make resident, turn end -- the
+    same state as the separate calls."""
+    import torch
+    from paper_2606_22983_gb300 import lv
+    S, B, T = 8, 16, 16
+    placement = np.full((S, B), -1, np.int32)
+    ctx = np.zeros(S, np.int32)
+    # sessions 1 and 3: 4 blocks in HBM; session 5: 3 blocks on the host; session 6: 2 + 2
+    nxt = 0
+    for s, (n_hbm, n_host) in {1: (4, 0), 3: (4, 0), 5: (0, 3), 6: (2, 2)}.items():
+        for b in range(n_hbm + n_host):
+            placement[s, b] = nxt if b < n_hbm else -(s * 4 + b + 2)
+            nxt += b < n_hbm
+        ctx[s] = (n_hbm + n_host) * T
+    results = []
+    for how in ("turn", "calls"):
+        pool = _tiny_pool(max_sessions=S, max_blocks=B, hbm_pages=64, hbm_budget_pages=64, host_pages=64)
+        try:
+            pool.import_placement(placement, ctx)
+            res = np.zeros(1, dtype=lv.RESIDENT_DTYPE)
+            if how == "turn":
+                cand = torch.tensor([3, 1, 6, 5], dtype=torch.int32, device=pool.device)
+                lv.lv_turn(pool.handle, -1, 7_000_000, 20, 4_000_000, 50, result_out=res,
+                           candidates=cand, num_candidates=4, stream=pool.stream)
+            else:
+                ev = np.zeros(1, dtype=lv.EVENT_DTYPE)
+                ev["kind"], ev["sid"], ev["t_us"] = lv.LV_EV_TURN_BEGIN, 6, 7_000_000
+                pool.events(ev)
+                lv.lv_make_resident(pool.handle, 6, 7_000_000, 20, 0, -1, None, None, None, None,
+                                    None, res, pool.stream)
+                ev["kind"], ev["a"], ev["b"] = lv.LV_EV_TURN_END, 4_000_000, 50
+                pool.events(ev)
+            assert pool.sync(raise_on_error=False) == 0
+            r = res[0]
+            assert int(r["sid"]) == 6 and int(r["status"]) == lv.LV_RESIDENT_DONE
+            assert int(r["n_loaded"]) == 2 and int(r["n_appended"]) == 2
+            results.append((pool.tables(), pool.get_sessions().copy(), pool.stats()))
+        finally:
+            pool.close()
+    (ta, sa, xa), (tb, sb, xb) = results
+    for a, b in zip(ta, tb):
+        assert np.array_equal(a, b)
+    assert np.array_equal(sa, sb)
+    assert sa[6]["gen_us"] == 4_000_000 and not (sa[6]["flags"] & lv.LV_RUNNING)
+    for k in ("hbm_allocated", "host_allocated", "pages_in", "appended_pages", "events"):
+        assert xa[k] == xb[k], k
+
+
+def test_turn_pick_fallback_and_bad_candidate():
+    import torch
+    from paper_2606_22983_gb300 import lv
+    pool = _tiny_pool()
+    try:
+        placement = np.full((8, 16), -1, np.int32)
+        placement[2, :2] = [0, 1]
+        pool.import_placement(placement, np.array([0, 0, 32, 0, 0, 0, 0, 0], np.int32))
+        res = np.zeros(1, dtype=lv.RESIDENT_DTYPE)
+        cand = torch.tensor([4, 2], dtype=torch.int32, device=pool.device)
+        lv.lv_turn(pool.handle, -1, 1_000, 0, 0, 0, result_out=res, candidates=cand,
+                   num_candidates=2, stream=pool.stream)
+        assert pool.sync(raise_on_error=False) == 0
+        assert int(res[0]["sid"]) == 4 and int(res[0]["n_loaded"]) == 0   # nobody offloaded
+        bad = torch.tensor([8 + 3], dtype=torch.int32, device=pool.device)
+        lv.lv_turn(pool.handle, -1, 2_000, 16, 0, 0, result_out=res, candidates=bad,
+                   num_candidates=1, stream=pool.stream)
+        assert pool.sync(raise_on_error=False) == lv.LV_ERR_BOUNDS
+        assert int(res[0]["status"]) == lv.LV_RESIDENT_FAILED and int(res[0]["sid"]) == -1
+        assert pool.stats()["appended_pages"] == 0
+        pool.clear_error()
+        with pytest.raises(lv.LvError):
+            lv.lv_turn(pool.handle, -1, 3_000, 0, 0, 0, candidates=None, num_candidates=0,
+                       stream=pool.stream)
+    finally:
+        pool.close()

@@ -52,9 +52,11 @@ def _expected_block(seed, table, shape, sid, blk, ctx):
     return subpage_values_np(table, off, rows, shape).view(np.uint8).reshape(J, -1)
 
 
-def _sampled_full_size(wl, driver, mode, n_sample=48, rank_on="turns"):
-    """Every event's decisions, the final tables/owners/sessions, and the bytes of
-    sampled blocks (plus blocks the last movements touched) against the oracle."""
+def _sampled_full_size(wl, driver, mode, n_sample=48, rank_on="turns", record=True,
+                       async_copy=False):
+    """Every event's decisions (when recorded), the final tables/owners/sessions, and
+    the bytes of sampled blocks (plus blocks the last movements touched) against the
+    oracle."""
     import torch
     from oracle import OracleManager
     from paper_2606_22983_gb300.harness import ContentWriter, pool_for
@@ -67,12 +69,14 @@ def _sampled_full_size(wl, driver, mode, n_sample=48, rank_on="turns"):
     try:
         writer = ContentWriter(pool, wl)
         writer.write_initial(wl)
-        gm = KVManager(pool, perms=wl.perms, rank_on=rank_on, driver=driver, mode=mode,
-                       order_fn=scatter_order, on_append=writer.write_appended)
+        gm = KVManager(pool, perms=wl.perms, rank_on=rank_on if record else "none", driver=driver,
+                       mode=mode, order_fn=scatter_order, on_append=writer.write_appended,
+                       record=record, async_copy=async_copy)
         touched = []
         for i in range(wl.n_events):
             ro, rg = om.step(i), gm.step(wl.event(i), i)
-            compare_records(ro, rg, i)
+            if record:
+                compare_records(ro, rg, i)
             if "victims" in ro and len(ro["victims"]):
                 touched += [(int(a), int(b)) for a, b, _ in ro["victims"][:8]]
             if "in_blocks" in ro:
@@ -96,6 +100,14 @@ def _sampled_full_size(wl, driver, mode, n_sample=48, rank_on="turns"):
         torch.cuda.synchronize()
         pool.close()
         torch.cuda.empty_cache()
+
+
+def test_thinker_full_size_async_copies():
+    """Thinker turns with each turn's copy on the pool's copy stream and no host
+    round trip between turns (the next turn ranks and plans while the previous
+    turn's pages still move): the end state and sampled bytes equal the oracle's."""
+    _sampled_full_size(make_workload("thinker", 1, n_turns=30), "device", 0, record=False,
+                       async_copy=True)
 
 
 @pytest.mark.parametrize("driver,mode", [("device", 0), ("exchange", 0), ("exchange", 2)])
