@@ -197,7 +197,8 @@ def ours(args, torch):
         b = args.budget_pages or sp.hbm_budget_pages
         over["spec"] = sp.with_(n_sessions=args.sessions or sp.n_sessions, hbm_pages=b,
                                 hbm_budget_pages=b, tiers=args.tiers)
-    wl = make_workload(WORKLOAD, args.seed + rank, n_turns=W + 2 * K, **over)
+    KO = OVERLAP_TURNS if (args.overlap and args.driver == "device") else 0
+    wl = make_workload(WORKLOAD, args.seed + rank, n_turns=W + 2 * K + 4 * KO + 6, **over)
     pool = pool_for(wl)
     fill_random(pool, args.seed + rank)
     page_bytes = pool.J * pool.P
@@ -253,21 +254,34 @@ def ours(args, torch):
                           "bytes_per_launch": nb / t["launches"],
                           "gbs": nb / 1e9 / (t["total_ms"] / 1e3)}
 
-    # e2e: the next K turns through the C ABI with host buffers
-    gm.record = True
-    h2d = d2h = 0
+    # e2e: K further turns through the public API from host buffers, timed on the host
+    # clock: every step copies its event batch from page-locked host memory to the
+    # device and reads the turn's result (lv_resident_result) back into page-locked
+    # host memory, in stream order; the results are checked after the final join
+    gm.record = False
+    ev_h = torch.empty((K, S * lv.EVENT_DTYPE.itemsize), dtype=torch.uint8).pin_memory()
+    for j, i in enumerate(range(W + K, W + 2 * K)):
+        base = i * (S + 1)
+        ev = ev_h[j].numpy().view(lv.EVENT_DTYPE)
+        ev["kind"], ev["sid"], ev["t_us"], ev["a"], ev["b"] = (
+            lv.LV_EV_PLAYBACK, wl.sid[base:base + S], int(wl.t_us[base]), wl.a[base:base + S], 0)
+    res_h = torch.zeros((K, lv.RESIDENT_DTYPE.itemsize), dtype=torch.uint8).pin_memory()
+    own_res = gm.res_h
+    h2d = K * S * lv.EVENT_DTYPE.itemsize
+    d2h = K * lv.RESIDENT_DTYPE.itemsize
     torch.cuda.synchronize()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
     q0 = _moved_pages(pool)[0]
-    e0.record()
-    for i in range(W + K, W + 2 * K):
-        run_turns(gm, wl, i, i + 1, None)
-        h2d += (S + 2) * lv.EVENT_DTYPE.itemsize
-        d2h += gm.last_readback_bytes + lv.RESIDENT_DTYPE.itemsize
-    e1.record()
+    w0 = time.perf_counter()
+    for j, i in enumerate(range(W + K, W + 2 * K)):
+        lv.lv_session_events(pool.handle, ev_h[j], S, pool.stream)
+        gm.res_h = res_h[j]
+        gm.step(wl.event(i * (S + 1) + S), i * (S + 1) + S)
+    lv.lv_join(pool.handle, pool.stream)
     torch.cuda.synchronize()
-    e2e_s = e0.elapsed_time(e1) / 1e3
+    e2e_s = time.perf_counter() - w0
+    gm.res_h = own_res
+    status = res_h.numpy().view(lv.RESIDENT_DTYPE)["status"]
+    assert (status == lv.LV_RESIDENT_DONE).all(), "a turn of the end-to-end pass failed"
     moved_e2e = (_moved_pages(pool)[0] - q0) * page_bytes
     if dist:
         tt = torch.tensor([dev_s, e2e_s, moved, moved_e2e], dtype=torch.float64, device="cuda")
@@ -351,6 +365,8 @@ def ours(args, torch):
             "gpu_launches": int(launches),
             "clocks": clk,
         }
+    if line is not None and KO:
+        line["overlap"] = overlap_measure(torch, pool, wl, W + 2 * K, KO)
     if line is not None and args.micro:
         micro = kernel_micro(torch, pool, args.seed)
         line["ranker"] = micro.pop("ranker")
@@ -364,7 +380,84 @@ def ours(args, torch):
     return line
 
 
+OVERLAP_TURNS = 40
 REMAP_BYTES_PER_ENTRY = 52   # entry 12; read+write of: table 4+4, epoch 4+4, new owner 4+4, old owner 4+4, old bitmap 4+4
+
+
+def overlap_measure(torch, pool, wl, first_turn, n_turns):
+    """Config 3's overlap of KV movement with serving work: a consumer standing in
+    for the engine's attention reads (a torch sum over 4096 resident pages, 6.4 GB,
+    on its own stream; not part of liblv) runs alone, then throughout n_turns
+    thinker turns moved by the zero-copy device-driven path (SM copies, async) and
+    then by the staged path (copy engines).  The consumer's pages may change under
+    it; its sums are not used."""
+    from paper_2606_22983_gb300 import lv
+    from paper_2606_22983_gb300.manager import KVManager
+    n_pages = min(4096, pool.hbm_pages)
+    view = pool.kv[:, :n_pages, :].view(torch.int64)
+    read_bytes = view.numel() * 8
+    cs = torch.cuda.Stream(device=pool.device)
+
+    def consume(k):
+        with torch.cuda.stream(cs):
+            for _ in range(k):
+                view.sum(dtype=torch.int64)
+
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    consume(3)
+    torch.cuda.synchronize()
+    a0, a1 = ev(), ev()
+    a0.record(cs)
+    consume(20)
+    a1.record(cs)
+    torch.cuda.synchronize()
+    alone_ms = a0.elapsed_time(a1) / 20
+    out = {"consumer": "torch sum over 4096 resident pages (6.4 GB read), its own stream",
+           "consumer_alone_gbs": round(read_bytes / alone_ms / 1e6, 1)}
+    page_bytes = pool.J * pool.P
+    per_turn = 3          # consumer reads queued per turn: it never runs dry
+    turn = first_turn
+    for label, driver, mode, async_copy in (("zero_copy_sm", "device", 0, True),
+                                            ("staged_copy_engine", "exchange", 2, False)):
+        gm = KVManager(pool, perms=wl.perms, rank_on="none", mode=mode, record=False,
+                       driver=driver, async_copy=async_copy)
+        run_turns(gm, wl, turn, turn + 3, None)             # warm-up of this driver
+        turn += 3
+        lv.lv_join(pool.handle, pool.stream)
+        torch.cuda.synchronize()
+        # the turns alone
+        p0 = _moved_pages(pool)[0]
+        t0, t1 = ev(), ev()
+        t0.record()
+        run_turns(gm, wl, turn, turn + n_turns, None)
+        lv.lv_join(pool.handle, pool.stream)
+        t1.record()
+        torch.cuda.synchronize()
+        alone_gbs = (_moved_pages(pool)[0] - p0) * page_bytes / (t0.elapsed_time(t1) / 1e3) / 1e9
+        turn += n_turns
+        # the turns with the consumer running throughout
+        p0 = _moved_pages(pool)[0]
+        c0, c1 = ev(), ev()
+        c0.record(cs)
+        t0.record()
+        calls = 0
+        for i in range(turn, turn + n_turns):
+            consume(per_turn)
+            calls += per_turn
+            run_turns(gm, wl, i, i + 1, None)
+        lv.lv_join(pool.handle, pool.stream)
+        t1.record()
+        c1.record(cs)
+        torch.cuda.synchronize()
+        turn += n_turns
+        both_gbs = (_moved_pages(pool)[0] - p0) * page_bytes / (t0.elapsed_time(t1) / 1e3) / 1e9
+        cons_gbs = calls * read_bytes / (c0.elapsed_time(c1) / 1e3) / 1e9
+        out[label] = {"turns": n_turns, "turns_alone_gbs": round(alone_gbs, 1),
+                      "turns_with_consumer_gbs": round(both_gbs, 1),
+                      "consumer_with_turns_gbs": round(cons_gbs, 1),
+                      "consumer_frac_kept": round(cons_gbs / out["consumer_alone_gbs"], 3)}
+    assert pool.sync(raise_on_error=False) == 0, "device error during the overlap turns"
+    return out
 
 
 def kernel_micro(torch, pool, seed=0):
@@ -641,6 +734,8 @@ def main():
                     help="smaller case for profiling: number of sessions")
     ap.add_argument("--budget-pages", type=int, default=0,
                     help="smaller case for profiling: HBM budget in pages")
+    ap.add_argument("--no-overlap", dest="overlap", action="store_false",
+                    help="skip the consumer-overlap measurement")
     ap.add_argument("--no-async-copy", dest="async_copy", action="store_false",
                     help="device driver: copy on the caller's stream (no overlap of the next "
                          "turn's decisions with this turn's copy)")

@@ -425,6 +425,18 @@ lv_status lv_pack_pages(lv_pool* pool, const int32_t* pages, int64_t n, void* ds
 lv_status lv_unpack_pages(lv_pool* pool, const void* src, const int32_t* pages, int64_t n,
                           lv_stream stream);
 
+/* Reads listed HBM pages and reduces each to a 64-bit checksum: with the
+   page's 2L sub-pages concatenated in order (sub-page j = 2*layer + kv) and
+   read as little-endian 64-bit words w_0 .. w_{m-1} (m = 2L*P/8),
+       sums_out[i] = sum over q of w_q * (2q + 1)   (mod 2^64).
+   The weights make the sum depend on where each word sits.  It stands in for
+   a consumer that reads running sessions' KV (attention reads every byte of
+   a page) and verifies page contents without copying them to the host.  Not
+   from the paper: an instrument.  sums_out (uint64 [n], device or host).
+   Device-detected: LV_ERR_BOUNDS for a page outside the pool (its sum is 0). */
+lv_status lv_page_checksums(lv_pool* pool, const int32_t* pages, int64_t n, uint64_t* sums_out,
+                            lv_stream stream);
+
 /* Block-level allocation kept (Section 5.1): grows session sid's context by
    n_tokens; each new block takes the lowest free HBM page, in block order, and
    is committed at once.  LV_TIERS_INCLUSIVE: when n_tokens > 0 and the last

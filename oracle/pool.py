@@ -278,6 +278,15 @@ class OraclePool:
         return pages
 
     # ----------------------------------------------------------------- views
+    def page_checksum(self, page: int) -> int:
+        """Position-weighted sum of an HBM page (an instrument, not from the paper):
+        the 2L sub-pages concatenated in order, read as little-endian 64-bit words
+        w_q, and sum_q w_q * (2q + 1) mod 2^64."""
+        data = np.ascontiguousarray(self.hbm[:, int(page), :]).reshape(-1)
+        w = data.view("<u8")
+        weights = 2 * np.arange(w.size, dtype=np.uint64) + np.uint64(1)
+        return int(np.sum(w * weights, dtype=np.uint64))
+
     def host_blocks(self, sid: int) -> np.ndarray:
         row = self.tables[sid, :int(self.nblocks[sid])]
         return np.nonzero(row <= -2)[0].astype(np.int64)

@@ -7,7 +7,18 @@
 #include <new>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "lv_internal.cuh"
+
+// One NVTX range per entry point, so that a profiler's timeline shows which liblv call
+// launched which kernels (no cost without a tool attached).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 struct lv_pool {
   lv::DevPool d{};
@@ -524,6 +535,7 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
 extern "C" {
 
 lv_status lv_pool_create(const lv_pool_desc* desc, lv_stream stream, lv_pool** out) {
+  NvtxRange nvtx_range("lv_pool_create");
   if (!out) return LV_ERR_INVALID;
   *out = nullptr;
   try {
@@ -534,6 +546,7 @@ lv_status lv_pool_create(const lv_pool_desc* desc, lv_stream stream, lv_pool** o
 }
 
 lv_status lv_pool_destroy(lv_pool* pool, lv_stream stream) {
+  NvtxRange nvtx_range("lv_pool_destroy");
   if (!pool) return LV_ERR_INVALID;
   DeviceGuard g(pool->device);
   cudaError_t e = join_copies(pool, as_stream(stream));
@@ -546,6 +559,7 @@ void* lv_pool_host_ptr(lv_pool* pool) { return pool ? pool->host_base : nullptr;
 
 lv_status lv_pool_import(lv_pool* pool, const int32_t* placement, const int32_t* ctx_tokens,
                          lv_stream stream) {
+  NvtxRange nvtx_range("lv_pool_import");
   if (!pool || !placement || !ctx_tokens) return LV_ERR_INVALID;
   DeviceGuard g(pool->device);
   cudaStream_t s = as_stream(stream);
@@ -572,6 +586,7 @@ lv_status lv_pool_import(lv_pool* pool, const int32_t* placement, const int32_t*
 
 lv_status lv_session_set(lv_pool* pool, const lv_session_state* states, int32_t first, int32_t n,
                          lv_stream stream) {
+  NvtxRange nvtx_range("lv_session_set");
   if (!pool || first < 0 || n < 0 || (long long)first + n > pool->d.S) return LV_ERR_INVALID;
   if (n == 0) return LV_OK;
   DeviceGuard g(pool->device);
@@ -599,6 +614,7 @@ lv_status lv_session_get(lv_pool* pool, lv_session_state* out, int32_t first, in
 }
 
 lv_status lv_session_events(lv_pool* pool, const lv_event* events, int64_t n, lv_stream stream) {
+  NvtxRange nvtx_range("lv_session_events");
   if (!pool || n < 0 || (n > 0 && !events)) return LV_ERR_INVALID;
   if (n == 0) return LV_OK;
   DeviceGuard g(pool->device);
@@ -618,6 +634,7 @@ lv_status lv_session_events(lv_pool* pool, const lv_event* events, int64_t n, lv
 lv_status lv_select_victims(lv_pool* pool, int64_t now_us, int64_t k, uint32_t flags,
                             lv_victim* out, int64_t capacity, int64_t* count_out,
                             lv_stream stream) {
+  NvtxRange nvtx_range("lv_select_victims");
   if (!pool || k < 0 || capacity < 0 || (flags & ~(uint32_t)LV_SELECT_FALLBACK)) return LV_ERR_INVALID;
   const int64_t keff = k < capacity ? k : capacity;
   if (keff > 0 && !out) return LV_ERR_INVALID;
@@ -640,6 +657,7 @@ lv_status lv_select_victims(lv_pool* pool, int64_t now_us, int64_t k, uint32_t f
 
 lv_status lv_swap_out(lv_pool* pool, const lv_victim* victims, int64_t n, int32_t* slots_out,
                       lv_remap_entry* commit_out, int32_t mode, lv_stream stream) {
+  NvtxRange nvtx_range("lv_swap_out");
   if (!pool || n < 0 || n > 0x7fffffffll || (n > 0 && !victims)) return LV_ERR_INVALID;
   if (mode != LV_MODE_AUTO && mode != LV_MODE_ZERO_COPY && mode != LV_MODE_STAGED) return LV_ERR_INVALID;
   if (n == 0) return LV_OK;
@@ -681,6 +699,7 @@ lv_status lv_swap_out(lv_pool* pool, const lv_victim* victims, int64_t n, int32_
 
 lv_status lv_swap_in(lv_pool* pool, int32_t sid, const int32_t* blks, int64_t n, int32_t* pages_out,
                      lv_remap_entry* commit_out, int32_t mode, lv_stream stream) {
+  NvtxRange nvtx_range("lv_swap_in");
   if (!pool || n < 0 || n > 0x7fffffffll || (n > 0 && !blks)) return LV_ERR_INVALID;
   if (mode != LV_MODE_AUTO && mode != LV_MODE_ZERO_COPY && mode != LV_MODE_STAGED) return LV_ERR_INVALID;
   if (sid < 0 || sid >= pool->d.S) return LV_ERR_INVALID;
@@ -719,6 +738,7 @@ lv_status lv_swap_in(lv_pool* pool, int32_t sid, const int32_t* blks, int64_t n,
 lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_out, int32_t sid,
                            const int32_t* blks, int64_t n_in, int32_t* slots_out, int32_t* pages_out,
                            int32_t mode, lv_stream stream) {
+  NvtxRange nvtx_range("lv_swap_exchange");
   if (!pool || n_out < 0 || n_in < 0 || n_out > 0x7fffffffll || n_in > 0x7fffffffll ||
       (n_out > 0 && !victims) || (n_in > 0 && !blks))
     return LV_ERR_INVALID;
@@ -790,6 +810,7 @@ lv_status lv_make_resident(lv_pool* pool, int32_t sid, int64_t now_us, int32_t a
                            uint32_t flags, int64_t max_load_pages, lv_victim* victims_out,
                            int32_t* slots_out, int32_t* blocks_out, int32_t* pages_out,
                            int32_t* append_out, lv_resident_result* result_out, lv_stream stream) {
+  NvtxRange nvtx_range("lv_make_resident");
   if (!pool || sid < 0 || sid >= pool->d.S || append_tokens < 0) return LV_ERR_INVALID;
   if (flags & ~(uint32_t)(LV_RESIDENT_PRELOAD | LV_RESIDENT_ASYNC_COPY)) return LV_ERR_INVALID;
   const bool preload = (flags & LV_RESIDENT_PRELOAD) != 0;
@@ -822,6 +843,7 @@ lv_status lv_make_resident(lv_pool* pool, int32_t sid, int64_t now_us, int32_t a
 }
 
 lv_status lv_join(lv_pool* pool, lv_stream stream) {
+  NvtxRange nvtx_range("lv_join");
   if (!pool) return LV_ERR_INVALID;
   DeviceGuard g(pool->device);
   LV_TRY(join_copies(pool, as_stream(stream)));
@@ -831,6 +853,7 @@ lv_status lv_join(lv_pool* pool, lv_stream stream) {
 lv_status lv_turn(lv_pool* pool, const lv_turn_desc* d, lv_victim* victims_out, int32_t* slots_out,
                   int32_t* blocks_out, int32_t* pages_out, int32_t* append_out,
                   lv_resident_result* result_out, lv_stream stream) {
+  NvtxRange nvtx_range("lv_turn");
   if (!pool || !d || d->append_tokens < 0 || (d->flags & ~(uint32_t)LV_RESIDENT_ASYNC_COPY))
     return LV_ERR_INVALID;
   const bool async = (d->flags & LV_RESIDENT_ASYNC_COPY) != 0;
@@ -899,6 +922,7 @@ lv_status pack_impl(lv_pool* pool, const int32_t* pages, int64_t n, void* run, b
 }  // namespace
 
 lv_status lv_pack_pages(lv_pool* pool, const int32_t* pages, int64_t n, void* dst, lv_stream stream) {
+  NvtxRange nvtx_range("lv_pack_pages");
   if (!pool || n < 0 || n > 0x7fffffffll || (n > 0 && (!pages || !dst))) return LV_ERR_INVALID;
   if (n == 0) return LV_OK;
   DeviceGuard g(pool->device);
@@ -911,6 +935,7 @@ lv_status lv_pack_pages(lv_pool* pool, const int32_t* pages, int64_t n, void* ds
 
 lv_status lv_unpack_pages(lv_pool* pool, const void* src, const int32_t* pages, int64_t n,
                           lv_stream stream) {
+  NvtxRange nvtx_range("lv_unpack_pages");
   if (!pool || n < 0 || n > 0x7fffffffll || (n > 0 && (!pages || !src))) return LV_ERR_INVALID;
   if (n == 0) return LV_OK;
   DeviceGuard g(pool->device);
@@ -921,10 +946,35 @@ lv_status lv_unpack_pages(lv_pool* pool, const void* src, const int32_t* pages, 
   }
 }
 
+lv_status lv_page_checksums(lv_pool* pool, const int32_t* pages, int64_t n, uint64_t* sums_out,
+                            lv_stream stream) {
+  NvtxRange nvtx_range("lv_page_checksums");
+  if (!pool || n < 0 || n > 0x7fffffffll || (n > 0 && (!pages || !sums_out))) return LV_ERR_INVALID;
+  if (n == 0) return LV_OK;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  try {
+    LV_TRY(join_copies(pool, s));   // reads KV bytes: after earlier asynchronous copies
+    Staging st(pool, s);
+    const void* pin = nullptr;
+    void* sdev = nullptr;
+    lv_status r;
+    if ((r = st.in(pages, (size_t)n * 4, &pin)) != LV_OK) return r;
+    if ((r = st.out(sums_out, (size_t)n * 8, &sdev, true)) != LV_OK) return r;
+    LV_TRY(cudaMemsetAsync(sdev, 0, (size_t)n * 8, s));
+    LV_TRY(lv::launch_checksums(pool->d, static_cast<const int32_t*>(pin), n,
+                                static_cast<unsigned long long*>(sdev), s, pool->stage_ctas * 8));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
 void* lv_pool_host_device_ptr(lv_pool* pool) { return pool ? pool->d.host : nullptr; }
 
 lv_status lv_schedule(lv_pool* pool, const lv_sched_params* q, const lv_request* reqs, int32_t n,
                       int32_t* order_out, int32_t* batch_out, lv_stream stream) {
+  NvtxRange nvtx_range("lv_schedule");
   if (!pool || !q || n < 0 || n > LV_SCHED_MAX_REQUESTS || !batch_out || (n > 0 && (!reqs || !order_out)))
     return LV_ERR_INVALID;
   if (q->p_safe_us < 1 || q->p_safe_us > (1ll << 32) || q->alpha < 0 || q->alpha > (1 << 16) ||
@@ -954,6 +1004,7 @@ lv_status lv_schedule(lv_pool* pool, const lv_sched_params* q, const lv_request*
 }
 
 lv_status lv_remap(lv_pool* pool, const lv_remap_entry* entries, int64_t n, lv_stream stream) {
+  NvtxRange nvtx_range("lv_remap");
   if (!pool || n < 0 || (n > 0 && !entries)) return LV_ERR_INVALID;
   if (n == 0) return LV_OK;
   DeviceGuard g(pool->device);
@@ -972,6 +1023,7 @@ lv_status lv_remap(lv_pool* pool, const lv_remap_entry* entries, int64_t n, lv_s
 }
 
 lv_status lv_cancel(lv_pool* pool, const int32_t* locs, int64_t n, lv_stream stream) {
+  NvtxRange nvtx_range("lv_cancel");
   if (!pool || n < 0 || (n > 0 && !locs)) return LV_ERR_INVALID;
   if (n == 0) return LV_OK;
   DeviceGuard g(pool->device);
@@ -990,6 +1042,7 @@ lv_status lv_cancel(lv_pool* pool, const int32_t* locs, int64_t n, lv_stream str
 
 lv_status lv_session_append(lv_pool* pool, int32_t sid, int32_t n_tokens, int32_t* pages_out,
                             int32_t* count_out, lv_stream stream) {
+  NvtxRange nvtx_range("lv_session_append");
   if (!pool || sid < 0 || sid >= pool->d.S || n_tokens < 0) return LV_ERR_INVALID;
   DeviceGuard g(pool->device);
   cudaStream_t s = as_stream(stream);
@@ -1009,6 +1062,7 @@ lv_status lv_session_append(lv_pool* pool, int32_t sid, int32_t n_tokens, int32_
 }
 
 lv_status lv_session_counts(lv_pool* pool, int32_t* hbm_blocks, int32_t* host_blocks, lv_stream stream) {
+  NvtxRange nvtx_range("lv_session_counts");
   if (!pool) return LV_ERR_INVALID;
   if (!hbm_blocks && !host_blocks) return LV_OK;
   DeviceGuard g(pool->device);
@@ -1028,6 +1082,7 @@ lv_status lv_session_counts(lv_pool* pool, int32_t* hbm_blocks, int32_t* host_bl
 
 lv_status lv_session_blocks(lv_pool* pool, int32_t sid, int32_t where, int32_t* blks_out,
                             int64_t* count_out, lv_stream stream) {
+  NvtxRange nvtx_range("lv_session_blocks");
   if (!pool || sid < 0 || sid >= pool->d.S || (where != 0 && where != 1) || !blks_out)
     return LV_ERR_INVALID;
   DeviceGuard g(pool->device);
@@ -1048,6 +1103,7 @@ lv_status lv_session_blocks(lv_pool* pool, int32_t sid, int32_t where, int32_t* 
 
 lv_status lv_read_tables(lv_pool* pool, int32_t* tables, int32_t* hbm_owner, int32_t* host_owner,
                          lv_stream stream) {
+  NvtxRange nvtx_range("lv_read_tables");
   if (!pool) return LV_ERR_INVALID;
   DeviceGuard g(pool->device);
   cudaStream_t s = as_stream(stream);
@@ -1062,6 +1118,7 @@ lv_status lv_read_tables(lv_pool* pool, int32_t* tables, int32_t* hbm_owner, int
 }
 
 lv_status lv_sync(lv_pool* pool, lv_stream stream) {
+  NvtxRange nvtx_range("lv_sync");
   if (!pool) return LV_ERR_INVALID;
   DeviceGuard g(pool->device);
   long long ctl[2] = {0, 0};

@@ -149,6 +149,9 @@ cudaError_t launch_turn(const DevPool& p, const ResidentScratch& rs, int32_t sid
                         lv_resident_result* result, const EventPair* ev = nullptr,
                         const CopyOffload* off = nullptr);
 cudaError_t launch_counts(const DevPool& p, int32_t* hbm, int32_t* host, cudaStream_t s);
+// sums[i] = position-weighted 64-bit sum of page pages[i] (sums zeroed by the caller)
+cudaError_t launch_checksums(const DevPool& p, const int32_t* pages, int64_t n,
+                             unsigned long long* sums, cudaStream_t s, int ctas);
 cudaError_t launch_blocks(const DevPool& p, int32_t sid, int32_t where, int32_t* out,
                           long long* count, cudaStream_t s);
 cudaError_t launch_check_budget(const DevPool& p, cudaStream_t s);

@@ -1421,6 +1421,60 @@ __global__ void k_turn_end(DevPool p, long long now_us, long long audio_us, long
   atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_EVENTS]), 1ull);
 }
 
+// ------------------------------------------------------------- checksums
+constexpr int kSumThreads = 256;
+constexpr int kSumUnroll = 4;
+
+// Unit u = (page i, sub-page j); the sub-page's words are q0 + k (q0 = j*P/8).
+// Each thread keeps kSumUnroll 16-byte loads in flight; the per-unit partial sum
+// goes to sums[i] with one atomic add (addition mod 2^64 is order-free).
+__global__ void __launch_bounds__(kSumThreads)
+k_checksum(DevPool p, const int32_t* __restrict__ pages, long long n, unsigned long long* __restrict__ sums) {
+  __shared__ unsigned long long warp_part[kSumThreads / 32];
+  const long long units = n * p.J;
+  const int nvec = (int)(p.P >> 4);                   // 16-byte vectors per sub-page
+  for (long long u = blockIdx.x; u < units; u += gridDim.x) {
+    const long long i = u / p.J;
+    const int j = (int)(u % p.J);
+    const int32_t pg = pages[i];
+    const bool ok = pg >= 0 && pg < p.hbm_pages;
+    unsigned long long acc = 0;
+    if (ok) {
+      const ulonglong2* src = reinterpret_cast<const ulonglong2*>(p.kv[j] + (size_t)pg * p.P);
+      const unsigned long long q0 = (unsigned long long)j * (unsigned long long)(p.P >> 3);
+      for (int base = threadIdx.x; base < nvec; base += kSumThreads * kSumUnroll) {
+        ulonglong2 r[kSumUnroll];
+#pragma unroll
+        for (int k = 0; k < kSumUnroll; ++k) {
+          const int v = base + k * kSumThreads;
+          if (v < nvec) r[k] = src[v];
+        }
+#pragma unroll
+        for (int k = 0; k < kSumUnroll; ++k) {
+          const int v = base + k * kSumThreads;
+          if (v < nvec) {
+            const unsigned long long q = q0 + 2ull * (unsigned long long)v;   // word index of r.x
+            acc += r[k].x * (2ull * q + 1ull) + r[k].y * (2ull * q + 3ull);
+          }
+        }
+      }
+    } else if (j == 0 && threadIdx.x == 0) {
+      set_error(p.ctl, LV_ERR_BOUNDS, i);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_down_sync(0xffffffffu, acc, o);
+    if ((threadIdx.x & 31) == 0) warp_part[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      unsigned long long t = 0;
+#pragma unroll
+      for (int w = 0; w < kSumThreads / 32; ++w) t += warp_part[w];
+      if (ok) atomicAdd(&sums[i], t);
+    }
+    __syncthreads();
+  }
+}
+
 // ----------------------------------------------------------------- views
 __global__ void __launch_bounds__(kCensusThreads)
 k_counts(DevPool p, int32_t* __restrict__ hbm, int32_t* __restrict__ host) {
@@ -1604,6 +1658,13 @@ cudaError_t launch_turn(const DevPool& p, const ResidentScratch& rs, int32_t sid
                                        copy_ctas, result, ev, R + R_SID, off);
   if (e != cudaSuccess) return e;
   k_turn_end<<<1, 32, 0, s>>>(p, now_us, audio_us, units, R);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_checksums(const DevPool& p, const int32_t* pages, int64_t n,
+                             unsigned long long* sums, cudaStream_t s, int ctas) {
+  if (n <= 0) return cudaSuccess;
+  k_checksum<<<blocks_for(n * p.J, 1, ctas), kSumThreads, 0, s>>>(p, pages, n, sums);
   return cudaGetLastError();
 }
 

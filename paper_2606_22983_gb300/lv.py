@@ -138,6 +138,7 @@ def _load():
         "lv_make_resident": [vp, i32, i64, i32, u32, i64, vp, vp, vp, vp, vp, vp, vp],
         "lv_turn": [vp, ctypes.POINTER(lv_turn_desc), vp, vp, vp, vp, vp, vp, vp],
         "lv_join": [vp, vp],
+        "lv_page_checksums": [vp, vp, i64, vp, vp],
         "lv_timing_enable": [vp, i32],
         "lv_pack_pages": [vp, vp, i64, vp, vp],
         "lv_schedule": [vp, ctypes.POINTER(lv_sched_params), vp, i32, vp, vp, vp],
@@ -181,7 +182,7 @@ EXPORTED = ("lv_pool_create", "lv_pool_destroy", "lv_pool_host_ptr", "lv_pool_im
             "lv_get_stats", "lv_clear_error", "lv_status_str", "lv_version",
             "lv_select_victims_noalloc", "lv_timing_enable", "lv_timing_read", "lv_pack_pages",
             "lv_unpack_pages", "lv_pool_host_device_ptr", "lv_schedule", "lv_inject_fault",
-            "lv_selftest_wait", "lv_turn", "lv_join")
+            "lv_selftest_wait", "lv_turn", "lv_join", "lv_page_checksums")
 
 
 def lib():
@@ -303,6 +304,11 @@ def lv_turn(pool, sid, now_us, append_tokens, reply_audio_us, reply_units, outs=
                      append_tokens=append_tokens, flags=flags)
     _check(_lib.lv_turn(pool, ctypes.byref(d), *(ptr(o) for o in outs), ptr(result_out),
                         stream_handle(stream)), "lv_turn")
+
+
+def lv_page_checksums(pool, pages, n, sums_out, stream=None):
+    _check(_lib.lv_page_checksums(pool, ptr(pages), n, ptr(sums_out), stream_handle(stream)),
+           "lv_page_checksums")
 
 
 def lv_join(pool, stream=None):

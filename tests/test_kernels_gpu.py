@@ -362,3 +362,41 @@ def test_turn_pick_fallback_and_bad_candidate():
                        stream=pool.stream)
     finally:
         pool.close()
+
+
+@pytest.mark.parametrize("shape", [(2, 2, 64), (48, 4, 128)])
+def test_page_checksums_match_the_oracle(shape):
+    """lv_page_checksums against the oracle's definition on the same bytes: every
+    page of a randomly filled pool (tiny and thinker-shaped sub-pages), host and
+    device argument buffers, and a page id outside the pool."""
+    import torch
+    from oracle.pool import OraclePool
+    from paper_2606_22983_gb300 import lv
+    L, H, D = shape
+    pages = 64 if L == 2 else 24
+    pool = _tiny_pool(layers=L, kv_heads=H, head_dim=D, hbm_pages=pages, hbm_budget_pages=pages,
+                      host_pages=4)
+    try:
+        g = torch.Generator(device=pool.device).manual_seed(5)
+        pool.kv.copy_(torch.randint(0, 256, pool.kv.shape, generator=g, device=pool.device,
+                                    dtype=torch.int32).to(torch.uint8))
+        om = OraclePool(L, H, D, 16, 2, n_sessions=1, max_blocks=1, hbm_pages=pages,
+                        hbm_budget_pages=pages, host_pages=0)
+        om.hbm[:] = pool.kv.cpu().numpy()
+        want = np.array([om.page_checksum(q) for q in range(pages)], dtype=np.uint64)
+        order = np.random.default_rng(0).permutation(pages).astype(np.int32)
+        got_h = np.zeros(pages, np.uint64)
+        lv.lv_page_checksums(pool.handle, order, pages, got_h, pool.stream)
+        assert pool.sync(raise_on_error=False) == 0
+        assert np.array_equal(got_h, want[order])
+        got_d = torch.zeros(pages, dtype=torch.int64, device=pool.device)
+        lv.lv_page_checksums(pool.handle, torch.from_numpy(order).to(pool.device), pages, got_d,
+                             pool.stream)
+        assert np.array_equal(got_d.cpu().numpy().view(np.uint64), want[order])
+        bad = np.array([1, pages + 7], np.int32)
+        sums = np.ones(2, np.uint64)
+        lv.lv_page_checksums(pool.handle, bad, 2, sums, pool.stream)
+        assert pool.sync(raise_on_error=False) == lv.LV_ERR_BOUNDS
+        assert sums[0] == want[1] and sums[1] == 0
+    finally:
+        pool.close()
