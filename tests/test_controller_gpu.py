@@ -27,18 +27,20 @@ def _compare_controller(ro, rg, where):
                                       for a, b in zip(vo, vg)), where
 
 
-@pytest.mark.parametrize("name,bw,lead,cap,with_bytes", [
-    ("tiny", 1, 1_000_000, 40, True),
-    ("mixed", 2_000, 2_000_000, 2000, False),
+@pytest.mark.parametrize("name,bw,lead,cap,with_bytes,tiers", [
+    ("tiny", 1, 1_000_000, 40, True, 0),
+    ("tiny", 1, 1_000_000, 40, True, 1),
+    ("mixed", 2_000, 2_000_000, 2000, False, 0),
 ])
-def test_controller_matches_oracle(name, bw, lead, cap, with_bytes):
+def test_controller_matches_oracle(name, bw, lead, cap, with_bytes, tiers):
     import torch
     from oracle.preload import ControlledOracleManager, PreloadController
     from paper_2606_22983_gb300.controller import ControlledKVManager
     from paper_2606_22983_gb300.harness import ContentWriter, pool_for, zero_host
     from ._lockstep import compare_state
 
-    wl = make_workload(name, 0)
+    from workloads import pool_spec
+    wl = make_workload(name, 0, spec=pool_spec(name).with_(tiers=tiers))
     table = value_table(wl.seed)
     om = ControlledOracleManager(wl, PreloadController(link_bytes_per_us=bw, lead_prior_us=lead,
                                                        cap_pages=cap),

@@ -181,3 +181,25 @@ def test_commit_elsewhere_drops_the_copy():
     p.remap([0], [0], _enc_host(h))
     assert p.shadow[0, 0] == -1 and not p.host_used[0] and p.tables[0, 0] == _enc_host(int(h[0]))
     p.check_invariants()
+
+
+def test_tier_mode_changes_no_controller_decision():
+    """Under the Section 5.2 preload controller (admissions, deferred commits,
+    cancellations) the inclusive tiers still change where bytes sit only."""
+    from oracle.preload import ControlledOracleManager, PreloadController
+    runs = []
+    for tiers in (0, 1):
+        wl = make_workload("tiny", 0, spec=pool_spec("tiny").with_(tiers=tiers))
+        om = ControlledOracleManager(wl, PreloadController(link_bytes_per_us=1, lead_prior_us=1_000_000,
+                                                           cap_pages=40),
+                                     with_bytes=False, rank_on="none")
+        runs.append((om, om.run()))
+    (ex, ra), (inc, rb) = runs
+    for a, b in zip(ra, rb):
+        for key in DECISIONS + ("admitted", "completed", "cancelled", "unprotected"):
+            assert (key in a) == (key in b), key
+            if key in a and key != "admitted":
+                assert np.array_equal(np.asarray(a[key]), np.asarray(b[key])), key
+    assert ex.counters == inc.counters
+    assert inc.pool.clean_out > 0 and inc.pool.bytes_out < ex.pool.bytes_out
+    inc.pool.check_invariants()

@@ -35,3 +35,10 @@ def test_thinker_inclusive_full_size():
     om, gm = _sampled_full_size(_inclusive("thinker", 0, n_turns=20), "device", 0)
     assert om.pool.clean_out > 0
     assert om.pool.clean_dropped == 0
+
+
+def test_tiny_inclusive_lru_baseline():
+    """Inclusive tiers under the LRU baseline policy (no preloads)."""
+    wl = make_workload("tiny", 3, spec=pool_spec("tiny").with_(tiers=1, policy=1))
+    om, gm = run_lockstep(wl, with_bytes=True, check_every=100, driver="device")
+    assert om.counters == gm.counters and om.pool.clean_out > 0
