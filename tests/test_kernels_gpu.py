@@ -400,3 +400,43 @@ def test_page_checksums_match_the_oracle(shape):
         assert sums[0] == want[1] and sums[1] == 0
     finally:
         pool.close()
+
+
+def test_async_copy_is_joined_by_the_next_reader():
+    """lv_make_resident with LV_RESIDENT_ASYNC_COPY moves 96 thinker pages on the
+    pool's copy stream; lv_page_checksums queued right after it on the same stream,
+    with no host wait, must see every moved byte (it joins the copies first)."""
+    import torch
+    from oracle.pool import OraclePool
+    from paper_2606_22983_gb300 import lv
+    n = 96
+    pool = _tiny_pool(layers=48, kv_heads=4, head_dim=128, max_sessions=2, max_blocks=128,
+                      hbm_pages=256, hbm_budget_pages=256, host_pages=128)
+    try:
+        placement = np.full((2, 128), -1, np.int32)
+        placement[0, :n] = -(np.arange(n, dtype=np.int32) + 2)         # session 0 on the host
+        pool.import_placement(placement, np.array([n * 16, 0], np.int32))
+        g = torch.Generator(device=pool.device).manual_seed(9)
+        pool.host_dev[:n].copy_(torch.randint(0, 256, pool.host_dev[:n].shape, generator=g,
+                                              device=pool.device, dtype=torch.int32).to(torch.uint8))
+        torch.cuda.synchronize()
+        om = OraclePool(48, 4, 128, 16, 2, n_sessions=1, max_blocks=1, hbm_pages=1,
+                        hbm_budget_pages=1, host_pages=0)
+        want = []
+        for h in range(n):
+            om.hbm[:, 0, :] = pool.host[h]
+            want.append(om.page_checksum(0))
+        blocks = torch.empty(128, dtype=torch.int32, device=pool.device)
+        pages = torch.empty(128, dtype=torch.int32, device=pool.device)
+        sums = torch.zeros(n, dtype=torch.int64, device=pool.device)
+        res = torch.zeros(lv.RESIDENT_DTYPE.itemsize, dtype=torch.uint8).pin_memory()
+        lv.lv_make_resident(pool.handle, 0, 1_000, 0, lv.LV_RESIDENT_ASYNC_COPY, -1, None, None,
+                            blocks, pages, None, res, pool.stream)
+        lv.lv_page_checksums(pool.handle, pages, n, sums, pool.stream)
+        assert pool.sync(raise_on_error=False) == 0
+        r = res.numpy().view(lv.RESIDENT_DTYPE)[0]
+        assert int(r["n_loaded"]) == n and int(r["status"]) == lv.LV_RESIDENT_DONE
+        assert np.array_equal(blocks[:n].cpu().numpy(), np.arange(n))
+        assert np.array_equal(sums.cpu().numpy().view(np.uint64), np.array(want, np.uint64))
+    finally:
+        pool.close()

@@ -42,3 +42,10 @@ def test_tiny_inclusive_lru_baseline():
     wl = make_workload("tiny", 3, spec=pool_spec("tiny").with_(tiers=1, policy=1))
     om, gm = run_lockstep(wl, with_bytes=True, check_every=100, driver="device")
     assert om.counters == gm.counters and om.pool.clean_out > 0
+
+
+def test_thinker_inclusive_async_copies():
+    """Inclusive tiers with asynchronous turn copies and no host round trip."""
+    om, gm = _sampled_full_size(_inclusive("thinker", 2, n_turns=30), "device", 0, record=False,
+                                async_copy=True)
+    assert om.pool.clean_out > 0
