@@ -460,6 +460,75 @@ def overlap_measure(torch, pool, wl, first_turn, n_turns):
     return out
 
 
+def ab_measure(torch, seed, n_events):
+    """NEXT rows f1 and f3 on the GPU: the mixed real-time workload at full size
+    (128 sessions, 60 GB HBM budget) under three policies -- next-use ranking with
+    the Section 5.2 preload controller (a 200 GB/s modelled link), next-use with
+    every preload admitted, and the LRU baseline (no preloads).  For each turn it
+    records whether the session's KV had to be loaded at turn start, on the turn's
+    critical path, and the device time of the turn's calls (CUDA events, a host wait
+    per turn to read its decisions)."""
+    from paper_2606_22983_gb300.controller import ControlledKVManager
+    from paper_2606_22983_gb300.harness import pool_for
+    from paper_2606_22983_gb300.manager import KVManager
+    from workloads import make_workload, pool_spec, scatter_order
+    out = {"workload": f"mixed (128 sessions, 60 GB HBM budget), {n_events} events, seed {seed}"}
+    turn_kinds = (1, 2, 7)
+    for label in ("next_use_controller", "next_use_preload", "lru"):
+        spec = pool_spec("mixed").with_(policy=1 if label == "lru" else 0)
+        wl = make_workload("mixed", seed, spec=spec, n_events=n_events)
+        pool = pool_for(wl)
+        try:
+            if label == "next_use_controller":
+                gm = ControlledKVManager(pool, link_bytes_per_us=200_000, lead_prior_us=2_000_000,
+                                         cap_pages=spec.hbm_budget_pages // 10, perms=wl.perms,
+                                         order_fn=scatter_order)
+            else:
+                gm = KVManager(pool, perms=wl.perms, rank_on="none", record=True, driver="device",
+                               order_fn=scatter_order)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            on_path_ms, on_path_pages, turn_ms = [], [], []
+            w0 = time.perf_counter()
+            for i in range(wl.n_events):
+                e = wl.event(i)
+                if int(e[1]) not in turn_kinds:
+                    gm.step(e, i)
+                    continue
+                torch.cuda.synchronize()
+                a.record()
+                rec = gm.step(e, i)
+                b.record()
+                torch.cuda.synchronize()
+                ms = a.elapsed_time(b)
+                turn_ms.append(ms)
+                loaded = len(rec.get("in_blocks", ()))
+                if loaded:
+                    on_path_ms.append(ms)
+                    on_path_pages.append(loaded)
+            wall = time.perf_counter() - w0
+            assert pool.sync(raise_on_error=False) == 0, f"device error in the {label} run"
+            st = pool.stats()
+            q = lambda xs, f: round(float(np.percentile(xs, f)), 3) if xs else None
+            out[label] = {
+                "turns": len(turn_ms), "turns_loading_on_path": len(on_path_ms),
+                "on_path_load_ms": {"mean": round(float(np.mean(on_path_ms)), 3) if on_path_ms else None,
+                                    "p50": q(on_path_ms, 50), "p90": q(on_path_ms, 90),
+                                    "max": q(on_path_ms, 100)},
+                "on_path_pages_mean": round(float(np.mean(on_path_pages)), 1) if on_path_pages else 0,
+                "turn_ms_mean": round(float(np.mean(turn_ms)), 3),
+                "preloads": int(gm.counters.get("preloads", 0)),
+                "gb_out": round(st["bytes_out"] / 1e9, 2), "gb_in": round(st["bytes_in"] / 1e9, 2),
+                "wall_s": round(wall, 1)}
+            for k in ("admitted", "completed", "cancelled", "given_up", "hits"):
+                if k in gm.counters:
+                    out[label][k] = int(gm.counters[k])
+        finally:
+            torch.cuda.synchronize()
+            pool.close()
+            torch.cuda.empty_cache()
+    return out
+
+
 def kernel_micro(torch, pool, seed=0):
     """Standalone timings of the HBM-bound kernels and the ranker (rank 0, after the turns).
 
@@ -734,6 +803,9 @@ def main():
                     help="smaller case for profiling: number of sessions")
     ap.add_argument("--budget-pages", type=int, default=0,
                     help="smaller case for profiling: HBM budget in pages")
+    ap.add_argument("--ab", action="store_true",
+                    help="only the policy A/B on the mixed workload (NEXT rows f1 and f3)")
+    ap.add_argument("--ab-events", type=int, default=3000)
     ap.add_argument("--no-overlap", dest="overlap", action="store_false",
                     help="skip the consumer-overlap measurement")
     ap.add_argument("--no-async-copy", dest="async_copy", action="store_false",
@@ -749,6 +821,11 @@ def main():
     elif args.micro_only:
         import torch
         line = micro_only(args, torch)
+    elif args.ab:
+        import torch
+        from paper_2606_22983_gb300 import build
+        build()
+        line = {"ab": ab_measure(torch, args.seed, args.ab_events)}
     else:
         import torch
         line = ours(args, torch)
