@@ -514,7 +514,13 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
   }
 
   if (lv::configure_kernels() != cudaSuccess) return fail(LV_ERR_CUDA);
-  if (lv::configure_stage_kernels(d) != cudaSuccess) return fail(LV_ERR_CUDA);
+  if (const char* env = std::getenv("LV_STAGE_STAGES")) {   // TMA pack/unpack stages per CTA
+    const int st = std::atoi(env);
+    if (st >= 2 && st <= 16) d.stages = st;
+  }
+  // two TMA stages must fit in a CTA's shared memory; larger sub-pages use 16-byte copies
+  const bool tma_fits = 2 * d.P <= 227 * 1024;
+  if (tma_fits && lv::configure_stage_kernels(d) != cudaSuccess) return fail(LV_ERR_CUDA);
   if (cudaStreamCreateWithFlags(&pool->s_d2h, cudaStreamNonBlocking) != cudaSuccess ||
       cudaStreamCreateWithFlags(&pool->s_h2d, cudaStreamNonBlocking) != cudaSuccess)
     return fail(LV_ERR_CUDA);
@@ -524,8 +530,13 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
     pool->tasks_host = nullptr;
     return fail(LV_ERR_OOM);
   }
-  pool->stage_ctas = pool->num_sms;
+  pool->stage_ctas = 2 * pool->num_sms;   // two TMA pack/unpack CTAs per SM (see stage_count)
+  if (const char* env = std::getenv("LV_STAGE_CTAS_PER_SM")) {
+    const int per = std::atoi(env);
+    if (per >= 1 && per <= 4) pool->stage_ctas = pool->num_sms * per;
+  }
   if (const char* env = std::getenv("LV_STAGE_KERNEL")) pool->stage_tma = std::strcmp(env, "lsu") != 0;
+  if (!tma_fits) pool->stage_tma = false;
   cudaMemPoolProps props{};
   props.allocType = cudaMemAllocationTypePinned;
   props.location.type = cudaMemLocationTypeDevice;
@@ -974,7 +985,7 @@ lv_status lv_page_checksums(lv_pool* pool, const int32_t* pages, int64_t n, uint
     if ((r = st.out(sums_out, (size_t)n * 8, &sdev, true)) != LV_OK) return r;
     LV_TRY(cudaMemsetAsync(sdev, 0, (size_t)n * 8, s));
     LV_TRY(lv::launch_checksums(pool->d, static_cast<const int32_t*>(pin), n,
-                                static_cast<unsigned long long*>(sdev), s, pool->stage_ctas * 8));
+                                static_cast<unsigned long long*>(sdev), s, pool->num_sms * 8));
     return st.finish();
   } catch (const std::bad_alloc&) {
     return LV_ERR_OOM;

@@ -52,6 +52,7 @@ struct DevPool {
   int32_t tplay;          // LV_PLAY_PLAYBACK / LV_PLAY_COUNTERS
   int32_t policy;         // LV_POLICY_NEXT_USE / LV_POLICY_LRU
   int32_t incl;           // 1: LV_TIERS_INCLUSIVE
+  int32_t stages;         // shared-memory stages of the TMA pack/unpack kernel (0: from P)
   uint8_t* const* kv;     // [J] device pointers, sub-page j of page p at kv[j] + p*P
   uint8_t* host;          // device view of the host pool [host_pages][J][P]
   lv_session_state* sess; // [S]

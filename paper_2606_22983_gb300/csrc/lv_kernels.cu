@@ -901,7 +901,7 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
 }
 
 constexpr int kStageThreads = 32;     // one warp per CTA; lane 0 issues the bulk copies
-constexpr int kMaxStages = 8;
+constexpr int kMaxStages = 16;
 constexpr long long kWaitLimitNs = 1000000000ll;   // one second per stage wait
 
 // Moves units u = (task t, sub-page j) of P bytes through `stages` shared-memory
@@ -1685,9 +1685,15 @@ cudaError_t launch_tasks_in(const DevPool& p, int32_t sid, const int32_t* blks, 
   return cudaGetLastError();
 }
 
+// About 48 KiB of stages per CTA, two CTAs per SM: on GB300 three 16 KiB stages per CTA
+// moved 4096 scattered thinker pages at 6.82-6.94 TB/s (read + write), against 6.2-6.4
+// with eight stages and one CTA per SM, and 5.5 with two stages.
 int stage_count(const DevPool& p) {
-  int st = (int)((160 * 1024) / p.P);
-  return st < 2 ? 2 : (st > kMaxStages ? kMaxStages : st);
+  int st = p.stages > 0 ? p.stages : (int)((48 * 1024) / p.P);
+  if (st < 3) st = 3;
+  if (st > kMaxStages) st = kMaxStages;
+  if ((long long)st * p.P > 227 * 1024) st = (int)((227 * 1024) / p.P);
+  return st < 2 ? 2 : st;
 }
 
 cudaError_t configure_stage_kernels(const DevPool& p) {

@@ -440,3 +440,35 @@ def test_async_copy_is_joined_by_the_next_reader():
         assert np.array_equal(sums.cpu().numpy().view(np.uint64), np.array(want, np.uint64))
     finally:
         pool.close()
+
+
+def test_large_subpages_fall_back_to_plain_copies():
+    """Sub-pages too large for two TMA stages (32 KV heads x 128, 16 tokens, bf16 =
+    128 KiB) are packed and staged with 16-byte copies: a round trip through the
+    staged swap path returns every byte."""
+    import torch
+    from paper_2606_22983_gb300 import lv
+    pool = _tiny_pool(layers=1, kv_heads=32, head_dim=128, max_sessions=2, max_blocks=8,
+                      hbm_pages=8, hbm_budget_pages=8, host_pages=8)
+    try:
+        placement = np.full((2, 8), -1, np.int32)
+        placement[0, :4] = [0, 1, 2, 3]
+        pool.import_placement(placement, np.array([64, 0], np.int32))
+        g = torch.Generator(device=pool.device).manual_seed(3)
+        pool.kv.copy_(torch.randint(0, 256, pool.kv.shape, generator=g, device=pool.device,
+                                    dtype=torch.int32).to(torch.uint8))
+        before = pool.kv[:, :4, :].clone()
+        victims, n = pool.select(0, 4)
+        slots, commit = pool.swap_out(victims, n, lv.LV_MODE_STAGED)
+        pool.remap(commit, n)
+        assert pool.sync(raise_on_error=False) == 0
+        blks, nb = pool.blocks(0, 1)
+        pool.kv[:, :4, :].zero_()
+        pages, commit = pool.swap_in(0, blks, nb, lv.LV_MODE_STAGED)
+        pool.remap(commit, nb)
+        assert pool.sync(raise_on_error=False) == 0
+        t, _, _ = pool.tables()
+        for b in range(4):
+            assert torch.equal(pool.kv[:, int(t[0, b]), :], before[:, b, :])
+    finally:
+        pool.close()
