@@ -355,25 +355,57 @@ k_rank_sort(DevPool p, long long k, const long long* k_dev, bool fallback, long 
   extern __shared__ unsigned char smem_raw[];
   unsigned long long* keys = reinterpret_cast<unsigned long long*>(smem_raw);
   int32_t* vals = reinterpret_cast<int32_t*>(keys + N);
-  for (int i = threadIdx.x; i < N; i += kSortThreads) {
-    keys[i] = i < p.S ? p.skey[i] : 0ull;
-    vals[i] = i;
-  }
-  __syncthreads();
-  for (int kk = 2; kk <= N; kk <<= 1) {
-    for (int j = kk >> 1; j > 0; j >>= 1) {
-      for (int i = threadIdx.x; i < N; i += kSortThreads) {
-        const int ixj = i ^ j;
-        if (ixj > i) {
-          const unsigned long long a = keys[i], b = keys[ixj];
-          const bool swap = ((i & kk) == 0) ? (a < b) : (a > b);
-          if (swap) {
-            keys[i] = b; keys[ixj] = a;
-            const int32_t t = vals[i]; vals[i] = vals[ixj]; vals[ixj] = t;
-          }
+  if (N <= kSortThreads) {
+    // one key per thread: partners closer than a warp trade through shuffles, the
+    // others through shared memory; the pair (lower, upper) swaps exactly when the
+    // shared-memory network below would
+    const int i = threadIdx.x;
+    unsigned long long key = (i < N && i < p.S) ? p.skey[i] : 0ull;
+    int32_t val = i;
+    for (int kk = 2; kk <= N; kk <<= 1) {
+      for (int j = kk >> 1; j > 0; j >>= 1) {
+        unsigned long long pk;
+        int32_t pv;
+        if (j >= 32) {
+          if (i < N) { keys[i] = key; vals[i] = val; }
+          __syncthreads();
+          if (i < N) { pk = keys[i ^ j]; pv = vals[i ^ j]; }
+          __syncthreads();
+        } else {
+          pk = __shfl_xor_sync(0xffffffffu, key, j);
+          pv = __shfl_xor_sync(0xffffffffu, val, j);
+        }
+        if (i < N) {
+          const bool lower = (i & j) == 0;
+          const unsigned long long lo = lower ? key : pk, hi = lower ? pk : key;
+          const bool swap = ((i & kk) == 0) ? (lo < hi) : (lo > hi);
+          if (swap) { key = pk; val = pv; }
         }
       }
-      __syncthreads();
+    }
+    if (i < N) { keys[i] = key; vals[i] = val; }
+    __syncthreads();
+  } else {
+    for (int i = threadIdx.x; i < N; i += kSortThreads) {
+      keys[i] = i < p.S ? p.skey[i] : 0ull;
+      vals[i] = i;
+    }
+    __syncthreads();
+    for (int kk = 2; kk <= N; kk <<= 1) {
+      for (int j = kk >> 1; j > 0; j >>= 1) {
+        for (int i = threadIdx.x; i < N; i += kSortThreads) {
+          const int ixj = i ^ j;
+          if (ixj > i) {
+            const unsigned long long a = keys[i], b = keys[ixj];
+            const bool swap = ((i & kk) == 0) ? (a < b) : (a > b);
+            if (swap) {
+              keys[i] = b; keys[ixj] = a;
+              const int32_t t = vals[i]; vals[i] = vals[ixj]; vals[ixj] = t;
+            }
+          }
+        }
+        __syncthreads();
+      }
     }
   }
   // counts in rank order, each thread a contiguous run of ranks
