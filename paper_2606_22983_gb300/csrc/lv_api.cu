@@ -212,8 +212,13 @@ lv_status sync_events(lv_pool* pool, size_t n) {
 }
 
 // The staged data movement of n validated tasks {out page, out slot, in slot, in page}
-// on `s`: pack out pages into staging, copy-engine runs of consecutive slots in each
-// direction on the side streams, unpack into the in pages; joined back into `s`.
+// on `s`.  The task list is read back once; its out halves are sorted by host slot and
+// so are its in halves, so that consecutive slots become one copy-engine transfer
+// whatever order the blocks were listed in (a session evicted suffix first sits in
+// descending slots).  Then: pack the out pages into staging in slot order; copy-engine
+// runs in each direction on the side streams; unpack into the in pages; joined back
+// into `s`.  Every pack precedes every unpack on `s`, so a page that an incoming block
+// takes is read before it is overwritten.
 lv_status staged_move_inner(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStream_t s,
                             void** staging_out) {
   const lv::DevPool& d = pool->d;
@@ -221,71 +226,78 @@ lv_status staged_move_inner(lv_pool* pool, const int4* tasks_dev, int64_t n, cud
   if ((size_t)n > pool->tasks_host_cap) return LV_ERR_INVALID;
   LV_TRY(cudaMemcpyAsync(pool->tasks_host, tasks_dev, (size_t)n * sizeof(int4), cudaMemcpyDeviceToHost, s));
   LV_TRY(cudaStreamSynchronize(s));
+  // split and sort, in the second and third thirds of the page-locked task buffer
   const int4* t = pool->tasks_host;
+  int4* tout = pool->tasks_host + n;
+  int64_t n_out = 0, n_in = 0;
+  for (int64_t i = 0; i < n; ++i)
+    if (t[i].x >= 0) tout[n_out++] = make_int4(t[i].x, t[i].y, -1, -1);
+  int4* tin = tout + n_out;
+  for (int64_t i = 0; i < n; ++i)
+    if (t[i].z >= 0) tin[n_in++] = make_int4(-1, -1, t[i].z, t[i].w);
+  std::stable_sort(tout, tout + n_out, [](const int4& u, const int4& v) { return u.y < v.y; });
+  std::stable_sort(tin, tin + n_in, [](const int4& u, const int4& v) { return u.z < v.z; });
+  if (n_out + n_in == 0) return LV_OK;      // every task was refused (errors already set)
   const size_t pb = (size_t)d.J * d.P;
   const int64_t chunk = std::max<int64_t>(1, (int64_t)((96u << 20) / pb));
-  const int64_t nchunks = (n + chunk - 1) / chunk;
+  const int64_t nchunks = (std::max(n_out, n_in) + chunk - 1) / chunk;
   lv_status st = sync_events(pool, (size_t)(2 * nchunks + 3));
   if (st != LV_OK) return st;
   cudaEvent_t* ev = pool->sync_events.data();
-  cudaEvent_t ev_start = ev[0], ev_d2h_done = ev[1], ev_h2d_done = ev[2];
+  cudaEvent_t ev_start = ev[0];
   cudaEvent_t* ev_pack = ev + 3;            // [nchunks]
   cudaEvent_t* ev_h2d = ev + 3 + nchunks;   // [nchunks]
-  bool any_out = false, any_in = false;
-  for (int64_t i = 0; i < n; ++i) {
-    any_out |= t[i].x >= 0;
-    any_in |= t[i].z >= 0;
-  }
-  // staging[t] per direction: out pages are packed into one run, in pages land in another
+  // staging: out run [n_out][2L][P], in run [n_in][2L][P], then the sorted task lists
   void* staging = nullptr;
   {
-    const size_t bytes = (size_t)n * pb * ((any_out ? 1 : 0) + (any_in ? 1 : 0));
+    const size_t bytes = (size_t)(n_out + n_in) * pb + (size_t)(n_out + n_in) * sizeof(int4);
     cudaError_t e = cudaMallocFromPoolAsync(&staging, bytes, pool->mp, s);
     if (e != cudaSuccess) return lv_cuda_fail(e);
     *staging_out = staging;
   }
   uint8_t* stg_out = static_cast<uint8_t*>(staging);
-  uint8_t* stg_in = stg_out + (any_out ? (size_t)n * pb : 0);
+  uint8_t* stg_in = stg_out + (size_t)n_out * pb;
+  int4* tout_dev = reinterpret_cast<int4*>(stg_in + (size_t)n_in * pb);
+  int4* tin_dev = tout_dev + n_out;
+  LV_TRY(cudaMemcpyAsync(tout_dev, tout, (size_t)(n_out + n_in) * sizeof(int4), cudaMemcpyHostToDevice, s));
   uint8_t* host = static_cast<uint8_t*>(pool->host_base);
   LV_TRY(cudaEventRecord(ev_start, s));
   LV_TRY(cudaStreamWaitEvent(pool->s_d2h, ev_start, 0));
   LV_TRY(cudaStreamWaitEvent(pool->s_h2d, ev_start, 0));
-  // H2D first so that the inbound copies start at once
-  for (int64_t c = 0; c < nchunks && any_in; ++c) {
-    const int64_t a = c * chunk, b = std::min(n, a + chunk);
+  // H2D first so that the inbound copies start at once: runs of consecutive slots
+  for (int64_t c = 0; c * chunk < n_in; ++c) {
+    const int64_t a = c * chunk, b = std::min(n_in, a + chunk);
     for (int64_t i = a; i < b;) {
-      if (t[i].z < 0) { ++i; continue; }
       int64_t j = i + 1;
-      while (j < b && t[j].z == t[j - 1].z + 1) ++j;
+      while (j < b && tin[j].z == tin[j - 1].z + 1) ++j;
       if (fault_fires(pool, LV_FAULT_COPY)) return LV_ERR_CUDA;
-      LV_TRY(cudaMemcpyAsync(stg_in + (size_t)i * pb, host + (size_t)t[i].z * pb, (size_t)(j - i) * pb,
+      LV_TRY(cudaMemcpyAsync(stg_in + (size_t)i * pb, host + (size_t)tin[i].z * pb, (size_t)(j - i) * pb,
                              cudaMemcpyHostToDevice, pool->s_h2d));
       i = j;
     }
     LV_TRY(cudaEventRecord(ev_h2d[c], pool->s_h2d));
   }
   // pack every chunk on s; the D2H runs of chunk c follow its pack
-  for (int64_t c = 0; c < nchunks && any_out; ++c) {
-    const int64_t a = c * chunk, b = std::min(n, a + chunk);
-    LV_TRY(lv::launch_stage(d, true, tasks_dev, a, b, stg_out, s, pool->stage_ctas,
+  for (int64_t c = 0; c * chunk < n_out; ++c) {
+    const int64_t a = c * chunk, b = std::min(n_out, a + chunk);
+    LV_TRY(lv::launch_stage(d, true, tout_dev, a, b, stg_out, s, pool->stage_ctas,
                             timing_pair(pool, LV_TIMING_PACK), pool->stage_tma));
     LV_TRY(cudaEventRecord(ev_pack[c], s));
     LV_TRY(cudaStreamWaitEvent(pool->s_d2h, ev_pack[c], 0));
     for (int64_t i = a; i < b;) {
-      if (t[i].x < 0) { ++i; continue; }
       int64_t j = i + 1;
-      while (j < b && t[j].x >= 0 && t[j].y == t[j - 1].y + 1) ++j;
+      while (j < b && tout[j].y == tout[j - 1].y + 1) ++j;
       if (fault_fires(pool, LV_FAULT_COPY)) return LV_ERR_CUDA;
-      LV_TRY(cudaMemcpyAsync(host + (size_t)t[i].y * pb, stg_out + (size_t)i * pb, (size_t)(j - i) * pb,
+      LV_TRY(cudaMemcpyAsync(host + (size_t)tout[i].y * pb, stg_out + (size_t)i * pb, (size_t)(j - i) * pb,
                              cudaMemcpyDeviceToHost, pool->s_d2h));
       i = j;
     }
   }
   // unpack each chunk once it has arrived (every pack precedes it on s)
-  for (int64_t c = 0; c < nchunks && any_in; ++c) {
-    const int64_t a = c * chunk, b = std::min(n, a + chunk);
+  for (int64_t c = 0; c * chunk < n_in; ++c) {
+    const int64_t a = c * chunk, b = std::min(n_in, a + chunk);
     LV_TRY(cudaStreamWaitEvent(s, ev_h2d[c], 0));
-    LV_TRY(lv::launch_stage(d, false, tasks_dev, a, b, stg_in, s, pool->stage_ctas,
+    LV_TRY(lv::launch_stage(d, false, tin_dev, a, b, stg_in, s, pool->stage_ctas,
                             timing_pair(pool, LV_TIMING_UNPACK), pool->stage_tma));
   }
   return LV_OK;
@@ -525,7 +537,8 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       cudaStreamCreateWithFlags(&pool->s_h2d, cudaStreamNonBlocking) != cudaSuccess)
     return fail(LV_ERR_CUDA);
   pool->tasks_host_cap = (size_t)d.budget + d.maxB + (size_t)d.host_pages;
-  if (cudaHostAlloc((void**)&pool->tasks_host, pool->tasks_host_cap * sizeof(int4), cudaHostAllocDefault) !=
+  // the task list read back, then its sorted out and in halves
+  if (cudaHostAlloc((void**)&pool->tasks_host, 3 * pool->tasks_host_cap * sizeof(int4), cudaHostAllocDefault) !=
       cudaSuccess) {
     pool->tasks_host = nullptr;
     return fail(LV_ERR_OOM);
