@@ -190,15 +190,8 @@ def ours(args, torch):
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     K, W = args.steps, args.warmup
-    over = {}
-    if args.sessions or args.budget_pages or args.tiers:
-        from workloads import pool_spec
-        sp = pool_spec(WORKLOAD)
-        b = args.budget_pages or sp.hbm_budget_pages
-        over["spec"] = sp.with_(n_sessions=args.sessions or sp.n_sessions, hbm_pages=b,
-                                hbm_budget_pages=b, tiers=args.tiers)
     KO = OVERLAP_TURNS if (args.overlap and args.driver == "device") else 0
-    wl = make_workload(WORKLOAD, args.seed + rank, n_turns=W + 2 * K + 4 * KO + 6, **over)
+    wl = _arm_spec(args, args.seed + rank)
     pool = pool_for(wl)
     fill_random(pool, args.seed + rank)
     page_bytes = pool.J * pool.P
@@ -342,17 +335,8 @@ def ours(args, torch):
             "steps": K, "warmup": W, "ms_per_step": round(t_max * 1e3 / K, 4),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "u8", "data": "synthetic",
-            "config": {"workload": "thinker: 48 layers, 4 KV heads x 128, bf16, 16-token pages "
-                                   "(1.5 MiB), 64 sessions log-uniform 2k-16k tokens, 40 GB HBM "
-                                   "budget, one turn = evict + reload",
-                       "hbm_budget_pages": wl.spec.hbm_budget_pages, "host_pages": wl.spec.host_pages,
-                       "mode": {0: "auto", 1: "zero_copy", 2: "staged"}[args.mode],
-                       "driver": args.driver,
-                       "tiers": ("exclusive", "inclusive")[args.tiers],
-                       "async_copy": bool(args.async_copy and args.driver == "device"),
-                       "l2": "inputs larger than L2 (mean turn moves "
-                             f"{mean_turn / 1e6:.0f} MB each way from a 40 GB pool)",
-                       "parallelism": f"replicas x{ws}"},
+            "config": arm_config(args, wl.spec, ws),
+            "mean_turn_mb_each_way": round(mean_turn / 1e6, 1),
             "blocks_per_s": round(moved / page_bytes / t_max, 1),
             "turns_per_s": round(K * ws / t_max, 2),
             "link_peak_gbs": {k: round(v, 1) for k, v in peaks.items()},
@@ -745,6 +729,35 @@ def cpu_baseline(seconds, seed, steps=None):
             "seconds": round(el, 2)}
 
 
+def arm_config(args, spec, ws):
+    """The workload description both arms report (identical for the same arguments)."""
+    return {"workload": "thinker: 48 layers, 4 KV heads x 128, bf16, 16-token pages (1.5 MiB), "
+                        f"{spec.n_sessions} sessions log-uniform 2k-16k tokens, "
+                        f"{spec.hbm_budget_pages}-page HBM budget, one turn = evict + reload",
+            "hbm_budget_pages": spec.hbm_budget_pages, "host_pages": spec.host_pages,
+            "mode": {0: "auto", 1: "zero_copy", 2: "staged"}[args.mode],
+            "driver": args.driver,
+            "tiers": ("exclusive", "inclusive")[args.tiers],
+            "async_copy": bool(args.async_copy and args.driver == "device"),
+            "l2": "inputs larger than L2 (a turn moves about 0.6 GB each way out of a "
+                  "40 GB pool)",
+            "parallelism": f"replicas x{ws}"}
+
+
+def _arm_spec(args, seed):
+    """The pool spec of the timed workload, as ours() builds it."""
+    from workloads import make_workload, pool_spec
+    over = {}
+    if args.sessions or args.budget_pages or args.tiers:
+        sp = pool_spec(WORKLOAD)
+        b = args.budget_pages or sp.hbm_budget_pages
+        over["spec"] = sp.with_(n_sessions=args.sessions or sp.n_sessions, hbm_pages=b,
+                                hbm_budget_pages=b, tiers=args.tiers)
+    KO = OVERLAP_TURNS if (args.overlap and args.driver == "device") else 0
+    return make_workload(WORKLOAD, seed, n_turns=args.warmup + 2 * args.steps + 4 * KO + 6,
+                         **over)
+
+
 def reference(args):
     ws, rank, _ = _dist()
     if rank != 0:
@@ -774,10 +787,11 @@ def reference(args):
             "n_gpus": ws, "steps": K, "warmup": W, "ms_per_step": round(el * 1e3 / K, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
             "data": "synthetic",
-            "config": {"workload": "thinker-shaped pages; the oracle's bounded sample "
-                                   "(8 sessions, 1500-page HBM image)"},
+            "config": arm_config(args, _arm_spec(args, args.seed).spec, ws),
             "cpu_baseline": {"value": round(v, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
-                             "sample": f"{K} turns after {W} warm-up, {moved / 1e9:.2f} GB moved"},
+                             "sample": f"{K} turns of the oracle's bounded sample of this workload "
+                                       f"(thinker-shaped pages, 8 sessions, 1500-page HBM image) "
+                                       f"after {W} warm-up, {moved / 1e9:.2f} GB moved"},
             "e2e": {"value": round(v, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
 
