@@ -726,7 +726,29 @@ def cpu_baseline(seconds, seed, steps=None):
     return {"value": round(moved / el / 1e9, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
             "sample": f"{turns} turns of a thinker-shaped pool (8 sessions, 1500-page HBM image, "
                       f"{wl.spec.host_pages} host slots), {moved / 1e9:.2f} GB moved in {el:.1f} s",
-            "seconds": round(el, 2)}
+            "seconds": round(el, 2), "ranker": _oracle_ranker(seed)}
+
+
+def _oracle_ranker(seed):
+    """The oracle's top-256 decision over the 2^20-page metadata state the GPU ranker is
+    timed on (1024 sessions x 1024 resident blocks, random placement and states)."""
+    from oracle import sessions as se
+    from oracle.policy import select_victims
+    rng = np.random.default_rng(seed)
+    S = B = 1024
+    tables = rng.permutation(S * B).reshape(S, B).astype(np.int64)
+    nblocks = np.full(S, B, np.int64)
+    sts = [se.SessionState(gen_us=int(g)) for g in rng.integers(0, 10_000_000, S)]
+    t0 = time.perf_counter()
+    n = 0
+    while True:
+        select_victims(tables, nblocks, sts, 0, 256, se.MODE_PLAYBACK, 3_000_000, 80_000)
+        n += 1
+        el = time.perf_counter() - t0
+        if el > 2.0 or n >= 5:
+            break
+    return {"ms_per_decision": round(el * 1e3 / n, 1), "resident_pages": S * B, "k": 256,
+            "decisions": n}
 
 
 def arm_config(args, spec, ws):
