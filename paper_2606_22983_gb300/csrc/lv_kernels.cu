@@ -1,13 +1,20 @@
 // CUDA kernels of the KV swap path (sm_103a).
 //
 //   ranking   k_rank_census -> k_rank_sort -> k_rank_emit   (Section 5.1, Eq. 4)
-//   allocate  k_alloc                                        (lowest free, Section 5.1)
+//   allocate  k_alloc, k_alloc_out                           (lowest free, Section 5.1)
 //   move      k_swap_out / k_swap_in                         (Section 5, Fig. 6; Section 5.2)
+//             k_exchange_plan -> k_exchange_copy             (both directions in one step)
+//             k_stage_tasks (TMA) / k_stage_tasks_lsu         (staged copy-engine path)
 //   commit    k_remap, k_cancel, k_append                    (Section 6 side tables)
 //   monitor   k_events                                       (Section 3, Sections 5.1-5.2)
+//   turn      k_resident_*, k_pick_scan, k_turn_begin/end    (a whole turn on the device)
+//   verify    k_checksum                                     (page checksums)
 //
-// No kernel waits on another agent, so none can hang; every index read from
-// memory is range-checked and a bad item is skipped with the sticky error set.
+// The only waits are the TMA stage kernel's mbarrier waits for its own copies,
+// each limited by %globaltimer to one second, after which the kernel reports
+// LV_ERR_TIMEOUT and returns; no kernel waits on another kernel or agent.  Every
+// index read from memory is range-checked and a bad item is skipped with the
+// sticky error set.
 #include <cstdint>
 
 #include "lv_internal.cuh"
