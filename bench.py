@@ -402,7 +402,7 @@ def overlap_measure(torch, pool, wl, first_turn, n_turns):
     per_turn = 3          # consumer reads queued per turn: it never runs dry
     turn = first_turn
     for label, driver, mode, async_copy in (("zero_copy_sm", "device", 0, True),
-                                            ("staged_copy_engine", "exchange", 2, False)):
+                                            ("staged_copy_engine", "exchange", 2, True)):
         gm = KVManager(pool, perms=wl.perms, rank_on="none", mode=mode, record=False,
                        driver=driver, async_copy=async_copy)
         run_turns(gm, wl, turn, turn + 3, None)             # warm-up of this driver
@@ -760,7 +760,7 @@ def arm_config(args, spec, ws):
             "mode": {0: "auto", 1: "zero_copy", 2: "staged"}[args.mode],
             "driver": args.driver,
             "tiers": ("exclusive", "inclusive")[args.tiers],
-            "async_copy": bool(args.async_copy and args.driver == "device"),
+            "async_copy": bool(args.async_copy and (args.driver == "device" or args.mode == 2)),
             "l2": "inputs larger than L2 (a turn moves about 0.6 GB each way out of a "
                   "40 GB pool)",
             "parallelism": f"replicas x{ws}"}

@@ -35,6 +35,12 @@ struct lv_pool {
   cudaEvent_t ev_planned = nullptr;
   cudaEvent_t ev_copied[2] = {nullptr, nullptr};
   bool copied_pending[2] = {false, false};   // an async copy used scratch set b
+  // LV_MODE_STAGED | LV_MODE_ASYNC: unpacks on s_unpack; the last call's D2H, H2D and
+  // unpack completions (each next call's transfers wait on them) and its whole end
+  cudaStream_t s_unpack = nullptr;
+  cudaEvent_t ev_st_d2h = nullptr, ev_st_h2d = nullptr, ev_st_unpack = nullptr,
+              ev_st_packed = nullptr, ev_st_done = nullptr;
+  bool st_pending = false;
   // staged path: side streams for the copy engines, a host copy of the tasks, sync events
   cudaStream_t s_d2h = nullptr, s_h2d = nullptr;
   int4* tasks_host = nullptr;
@@ -220,7 +226,7 @@ lv_status sync_events(lv_pool* pool, size_t n) {
 // into `s`.  Every pack precedes every unpack on `s`, so a page that an incoming block
 // takes is read before it is overwritten.
 lv_status staged_move_inner(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStream_t s,
-                            void** staging_out) {
+                            void** staging_out, bool async) {
   const lv::DevPool& d = pool->d;
   if (n <= 0) return LV_OK;
   if ((size_t)n > pool->tasks_host_cap) return LV_ERR_INVALID;
@@ -264,6 +270,14 @@ lv_status staged_move_inner(lv_pool* pool, const int4* tasks_dev, int64_t n, cud
   LV_TRY(cudaEventRecord(ev_start, s));
   LV_TRY(cudaStreamWaitEvent(pool->s_d2h, ev_start, 0));
   LV_TRY(cudaStreamWaitEvent(pool->s_h2d, ev_start, 0));
+  const bool after_async = async && pool->st_pending;   // the previous asynchronous call
+  if (after_async) {
+    // a block it wrote out may come back now; a slot it read may be written now;
+    // a page it loaded may be packed now
+    LV_TRY(cudaStreamWaitEvent(pool->s_h2d, pool->ev_st_d2h, 0));
+    LV_TRY(cudaStreamWaitEvent(pool->s_d2h, pool->ev_st_h2d, 0));
+    LV_TRY(cudaStreamWaitEvent(s, pool->ev_st_unpack, 0));
+  }
   // H2D first so that the inbound copies start at once: runs of consecutive slots
   for (int64_t c = 0; c * chunk < n_in; ++c) {
     const int64_t a = c * chunk, b = std::min(n_in, a + chunk);
@@ -293,11 +307,18 @@ lv_status staged_move_inner(lv_pool* pool, const int4* tasks_dev, int64_t n, cud
       i = j;
     }
   }
-  // unpack each chunk once it has arrived (every pack precedes it on s)
+  // unpack each chunk once it has arrived, after every pack (on s, or on s_unpack
+  // when asynchronous)
+  cudaStream_t us = s;
+  if (async) {
+    us = pool->s_unpack;
+    LV_TRY(cudaEventRecord(pool->ev_st_packed, s));
+    LV_TRY(cudaStreamWaitEvent(us, pool->ev_st_packed, 0));
+  }
   for (int64_t c = 0; c * chunk < n_in; ++c) {
     const int64_t a = c * chunk, b = std::min(n_in, a + chunk);
-    LV_TRY(cudaStreamWaitEvent(s, ev_h2d[c], 0));
-    LV_TRY(lv::launch_stage(d, false, tin_dev, a, b, stg_in, s, pool->stage_ctas,
+    LV_TRY(cudaStreamWaitEvent(us, ev_h2d[c], 0));
+    LV_TRY(lv::launch_stage(d, false, tin_dev, a, b, stg_in, us, pool->stage_ctas,
                             timing_pair(pool, LV_TIMING_UNPACK), pool->stage_tma));
   }
   return LV_OK;
@@ -305,27 +326,47 @@ lv_status staged_move_inner(lv_pool* pool, const int4* tasks_dev, int64_t n, cud
 
 // staged_move_inner, then (also after an early error) join the side streams back
 // into `s` and release the staging run in stream order.
-lv_status staged_move(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStream_t s) {
+lv_status staged_move(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStream_t s,
+                      bool async = false) {
   void* staging = nullptr;
-  const lv_status st = staged_move_inner(pool, tasks_dev, n, s, &staging);
-  if (staging) {
-    cudaEvent_t* ev = pool->sync_events.data();
-    cudaEventRecord(ev[1], pool->s_d2h);
-    cudaEventRecord(ev[2], pool->s_h2d);
-    cudaStreamWaitEvent(s, ev[1], 0);
-    cudaStreamWaitEvent(s, ev[2], 0);
-    cudaFreeAsync(staging, s);
+  const lv_status st = staged_move_inner(pool, tasks_dev, n, s, &staging, async);
+  if (!staging) return st;
+  if (async && st == LV_OK) {
+    // the next asynchronous call orders itself on these; the staging run is freed
+    // once both directions and the unpacks are done
+    cudaEventRecord(pool->ev_st_d2h, pool->s_d2h);
+    cudaEventRecord(pool->ev_st_h2d, pool->s_h2d);
+    cudaEventRecord(pool->ev_st_unpack, pool->s_unpack);
+    cudaStreamWaitEvent(pool->s_unpack, pool->ev_st_d2h, 0);
+    cudaStreamWaitEvent(pool->s_unpack, pool->ev_st_h2d, 0);
+    cudaFreeAsync(staging, pool->s_unpack);
+    cudaEventRecord(pool->ev_st_done, pool->s_unpack);
+    pool->st_pending = true;
+    return st;
   }
+  cudaEvent_t* ev = pool->sync_events.data();
+  cudaEventRecord(ev[1], pool->s_d2h);
+  cudaEventRecord(ev[2], pool->s_h2d);
+  cudaStreamWaitEvent(s, ev[1], 0);
+  cudaStreamWaitEvent(s, ev[2], 0);
+  if (async) {   // stopped early: everything joins the caller's stream
+    cudaEventRecord(pool->ev_st_unpack, pool->s_unpack);
+    cudaStreamWaitEvent(s, pool->ev_st_unpack, 0);
+  }
+  cudaFreeAsync(staging, s);
   return st;
 }
 
-// Makes `s` wait for every asynchronous page copy issued so far.
-cudaError_t join_copies(lv_pool* pool, cudaStream_t s) {
+// Makes `s` wait for every asynchronous page copy issued so far (with
+// staged = false: not for the asynchronous staged exchanges, which order
+// themselves against each other).
+cudaError_t join_copies(lv_pool* pool, cudaStream_t s, bool staged = true) {
   for (int b = 0; b < 2; ++b) {
     if (!pool->copied_pending[b]) continue;
     const cudaError_t e = cudaStreamWaitEvent(s, pool->ev_copied[b], 0);
     if (e != cudaSuccess) return e;
   }
+  if (staged && pool->st_pending) return cudaStreamWaitEvent(s, pool->ev_st_done, 0);
   return cudaSuccess;
 }
 
@@ -336,6 +377,10 @@ cudaError_t next_scratch(lv_pool* pool, cudaStream_t s, bool async, const lv::Re
   const int b = (int)(pool->rs_seq++ & 1u);
   *rs = b ? &pool->rs_alt : &pool->rs;
   if (!async) return join_copies(pool, s);
+  if (pool->st_pending) {   // an asynchronous staged exchange may still move bytes
+    const cudaError_t e = cudaStreamWaitEvent(s, pool->ev_st_done, 0);
+    if (e != cudaSuccess) return e;
+  }
   if (pool->copied_pending[b]) {
     const cudaError_t e = cudaStreamWaitEvent(s, pool->ev_copied[b], 0);
     if (e != cudaSuccess) return e;
@@ -346,6 +391,11 @@ cudaError_t next_scratch(lv_pool* pool, cudaStream_t s, bool async, const lv::Re
 }
 
 void free_pool(lv_pool* pool) {
+  if (pool->s_unpack) cudaStreamSynchronize(pool->s_unpack);
+  if (pool->s_unpack) cudaStreamDestroy(pool->s_unpack);
+  for (cudaEvent_t e : {pool->ev_st_d2h, pool->ev_st_h2d, pool->ev_st_unpack, pool->ev_st_packed,
+                        pool->ev_st_done})
+    if (e) cudaEventDestroy(e);
   if (pool->s_copy) cudaStreamSynchronize(pool->s_copy);
   if (pool->s_copy) cudaStreamDestroy(pool->s_copy);
   if (pool->ev_planned) cudaEventDestroy(pool->ev_planned);
@@ -534,7 +584,13 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
   const bool tma_fits = 2 * d.P <= 227 * 1024;
   if (tma_fits && lv::configure_stage_kernels(d) != cudaSuccess) return fail(LV_ERR_CUDA);
   if (cudaStreamCreateWithFlags(&pool->s_d2h, cudaStreamNonBlocking) != cudaSuccess ||
-      cudaStreamCreateWithFlags(&pool->s_h2d, cudaStreamNonBlocking) != cudaSuccess)
+      cudaStreamCreateWithFlags(&pool->s_h2d, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&pool->s_unpack, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&pool->ev_st_d2h, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&pool->ev_st_h2d, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&pool->ev_st_unpack, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&pool->ev_st_packed, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&pool->ev_st_done, cudaEventDisableTiming) != cudaSuccess)
     return fail(LV_ERR_CUDA);
   pool->tasks_host_cap = (size_t)d.budget + d.maxB + (size_t)d.host_pages;
   // the task list read back, then its sorted out and in halves
@@ -560,6 +616,10 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
   }
   uint64_t threshold = UINT64_MAX;
   cudaMemPoolSetAttribute(pool->mp, cudaMemPoolAttrReleaseThreshold, &threshold);
+  // never make one stream wait for another to reuse a freed run (asynchronous staged
+  // exchanges free on their own stream): grow the pool instead
+  int no_internal = 0;
+  cudaMemPoolSetAttribute(pool->mp, cudaMemPoolReuseAllowInternalDependencies, &no_internal);
   if (cudaStreamSynchronize(s) != cudaSuccess) return fail(LV_ERR_CUDA);
   *out = pool;
   return LV_OK;
@@ -777,7 +837,10 @@ lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_ou
   if (!pool || n_out < 0 || n_in < 0 || n_out > 0x7fffffffll || n_in > 0x7fffffffll ||
       (n_out > 0 && !victims) || (n_in > 0 && !blks))
     return LV_ERR_INVALID;
+  const bool async = (mode & LV_MODE_ASYNC) != 0;
+  mode &= ~LV_MODE_ASYNC;
   if (mode != LV_MODE_AUTO && mode != LV_MODE_ZERO_COPY && mode != LV_MODE_STAGED) return LV_ERR_INVALID;
+  if (async && mode != LV_MODE_STAGED) return LV_ERR_INVALID;
   if (n_in > 0 && (sid < 0 || sid >= pool->d.S)) return LV_ERR_INVALID;
   if (mode == LV_MODE_STAGED && (size_t)(n_out + n_in) > pool->tasks_host_cap) return LV_ERR_INVALID;
   if (n_out > 0 && pool->d.host_pages == 0) return LV_ERR_INVALID;
@@ -785,7 +848,9 @@ lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_ou
   DeviceGuard g(pool->device);
   cudaStream_t s = as_stream(stream);
   try {
-    LV_TRY(join_copies(pool, s));   // earlier asynchronous copies move bytes too
+    // earlier asynchronous copies move bytes too (an asynchronous staged exchange
+    // orders itself against the previous one, transfer by transfer)
+    LV_TRY(join_copies(pool, s, !async));
     Staging st(pool, s);
     const void *vin = nullptr, *bin = nullptr;
     void *sdev = nullptr, *pdev = nullptr, *tdev = nullptr, *ndev = nullptr;
@@ -805,7 +870,7 @@ lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_ou
       long long nt = 0;
       LV_TRY(cudaMemcpyAsync(&nt, ndev, sizeof(nt), cudaMemcpyDeviceToHost, s));
       LV_TRY(cudaStreamSynchronize(s));
-      if ((r = staged_move(pool, static_cast<int4*>(tdev), nt, s)) != LV_OK) return r;
+      if ((r = staged_move(pool, static_cast<int4*>(tdev), nt, s, async)) != LV_OK) return r;
       return st.finish();
     }
     LV_TRY(lv::launch_exchange(pool->d, static_cast<const lv_victim*>(vin), n_out, sid,

@@ -55,7 +55,8 @@ class KVManager:
                  async_copy=False):
         self.pool = pool
         # device driver: turns' page copies on the pool's copy stream, overlapping the
-        # next turn's decisions (LV_RESIDENT_ASYNC_COPY); pool.sync() joins them
+        # next turn's decisions (LV_RESIDENT_ASYNC_COPY); exchange driver, staged mode:
+        # consecutive exchanges pipelined (LV_MODE_ASYNC); pool.sync() joins them
         self.async_copy = async_copy
         self.perms = perms
         self.on_append = on_append      # callback(sid, old_ctx, new_ctx, pages) after growth
@@ -223,6 +224,13 @@ class KVManager:
                 self.on_append(sid, old_ctx, old_ctx + append_tokens)
         return True
 
+    def _xmode(self):
+        """The exchange's mode: staged exchanges are pipelined across calls when the
+        manager runs with asynchronous copies (LV_MODE_ASYNC; pool.sync() joins)."""
+        if self.async_copy and self.mode == lv.LV_MODE_STAGED:
+            return self.mode | lv.LV_MODE_ASYNC
+        return self.mode
+
     def _victims(self, sid, now_us, k, foreground, rec):
         flags = lv.LV_SELECT_FALLBACK if foreground else 0
         victims, n = self.pool.select(now_us, k, flags)
@@ -247,7 +255,7 @@ class KVManager:
         nbytes = (n + nh) * pool.J * pool.P
         if self.timer:
             self.timer.start("exchange")
-        slots, pages = pool.exchange(victims, n, sid, hblk, nh, self.mode)
+        slots, pages = pool.exchange(victims, n, sid, hblk, nh, self._xmode())
         if self.timer:
             self.timer.stop("exchange", nbytes)
         if self.record:
@@ -337,7 +345,7 @@ class KVManager:
             slots, commit = pool.swap_out(victims, n, self.mode)
             pool.remap(commit, n)
         else:
-            slots, _ = pool.exchange(victims, n, 0, None, 0, self.mode)
+            slots, _ = pool.exchange(victims, n, 0, None, 0, self._xmode())
         if self.record:
             rec["slots"] = slots.cpu().numpy().astype(np.int64)
         self.counters["victims"] += n

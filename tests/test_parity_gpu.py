@@ -12,7 +12,7 @@ pytestmark = pytest.mark.gpu
 
 @pytest.mark.parametrize("seed,driver,mode", [(0, "device", 0), (1, "device", 0), (0, "exchange", 0),
                                               (1, "sequential", 0), (0, "exchange", 2),
-                                              (1, "sequential", 2)])
+                                              (1, "sequential", 2), (2, "exchange", 18)])
 def test_tiny_workload_full_images(seed, driver, mode):
     """1000 scripted events of the tiny pool: every ranking (full order after
     each event), eviction, preload, reload and growth, with full HBM and host
@@ -100,6 +100,14 @@ def _sampled_full_size(wl, driver, mode, n_sample=48, rank_on="turns", record=Tr
         torch.cuda.synchronize()
         pool.close()
         torch.cuda.empty_cache()
+
+
+def test_thinker_full_size_pipelined_staged_exchanges():
+    """Staged (copy-engine) exchanges with LV_MODE_ASYNC: each call's transfers and
+    unpacks overlap the next calls, ordered transfer by transfer; no byte readback
+    between turns.  The end state and sampled bytes equal the oracle's."""
+    _sampled_full_size(make_workload("thinker", 3, n_turns=30), "exchange", 2, record=False,
+                       async_copy=True)
 
 
 def test_thinker_full_size_async_copies():
