@@ -49,3 +49,64 @@ def test_thinker_inclusive_async_copies():
     om, gm = _sampled_full_size(_inclusive("thinker", 2, n_turns=30), "device", 0, record=False,
                                 async_copy=True)
     assert om.pool.clean_out > 0
+
+
+def test_inclusive_swap_out_over_several_chunks():
+    """One swap-out of 1500 victims (more than a CTA's 1024 threads), 800 without a
+    clean copy and 700 with one, in suffix-first order: the in-place spread of the
+    compact slot allocation over two chunks gives the oracle's slots, tables and bytes."""
+    import numpy as np
+    import torch
+    from oracle.pool import OraclePool, _enc_host
+    from paper_2606_22983_gb300.pool import KVPool
+    S, B, N = 2, 2048, 2000
+    pool = KVPool(layers=1, kv_heads=1, head_dim=8, max_sessions=S, max_blocks=B, hbm_pages=4096,
+                  hbm_budget_pages=4096, host_pages=4096, tiers=1)
+    om = OraclePool(1, 1, 8, 16, 2, S, B, 4096, 4096, 4096, with_bytes=True, inclusive=True)
+    try:
+        rng = np.random.default_rng(7)
+        placement = np.full((S, B), -1, np.int64)
+        order = rng.permutation(N)
+        hbm_blocks, host_blocks = np.sort(order[:800]), np.sort(order[800:])
+        placement[0, hbm_blocks] = rng.permutation(4096)[:800]
+        placement[0, host_blocks] = -(rng.permutation(4096)[:1200] + 2)
+        ctx = np.array([N * 16, 0])
+        om.import_placement(placement, ctx)
+        pool.import_placement(placement.astype(np.int32), ctx.astype(np.int32))
+        om.hbm[:] = rng.integers(0, 256, om.hbm.shape, dtype=np.uint8)
+        om.host[:] = rng.integers(0, 256, om.host.shape, dtype=np.uint8)
+        pool.kv.copy_(torch.from_numpy(om.hbm).to(pool.device))
+        pool.host[:] = om.host
+        torch.cuda.synchronize()
+        # reload 700 of the host blocks: they keep their slots as clean copies
+        back = np.sort(rng.permutation(host_blocks)[:700])
+        pages = om.swap_in(0, back)
+        om.remap(np.zeros(700, np.int64), back, pages)
+        gp, commit = pool.swap_in(0, torch.from_numpy(back.astype(np.int32)).to(pool.device), 700)
+        pool.remap(commit, 700)
+        assert np.array_equal(gp.cpu().numpy(), pages.astype(np.int32))
+        assert om.clean_copies() == 700
+        # evict every resident block at once
+        from oracle import sessions as se
+        from oracle.policy import select_victims
+        vs, vb, vp = select_victims(om.tables, om.nblocks, [se.SessionState(ctx_tokens=N * 16),
+                                                            se.SessionState()], 0, 1500, 0,
+                                    3_000_000, 80_000)
+        victims, n = pool.select(0, 1500)
+        assert n == 1500 and np.array_equal(victims.cpu().numpy(), np.stack([vs, vb, vp], 1).astype(np.int32))
+        slots = om.swap_out(vs, vb, vp)
+        gs, commit = pool.swap_out(victims, n)
+        assert np.array_equal(gs.cpu().numpy(), slots.astype(np.int32))
+        om.remap(vs, vb, _enc_host(slots))
+        pool.remap(commit, n)
+        assert pool.sync(raise_on_error=False) == 0
+        assert om.clean_out == 700
+        t, oh, oo = pool.tables()
+        assert np.array_equal(t, om.tables.astype(np.int32))
+        assert np.array_equal(pool.host, om.host)
+        st = pool.stats()
+        assert st["clean_out"] == 700 and st["clean_copies"] == 0
+        assert st["host_allocated"] == int(om.host_used.sum())
+    finally:
+        torch.cuda.synchronize()
+        pool.close()
