@@ -472,3 +472,35 @@ def test_large_subpages_fall_back_to_plain_copies():
             assert torch.equal(pool.kv[:, int(t[0, b]), :], before[:, b, :])
     finally:
         pool.close()
+
+
+@pytest.mark.parametrize("S", [1025, 1500, 4096])
+def test_ranker_beyond_a_thousand_sessions(S):
+    """More sessions than the sort kernel's threads (up to the 4096 maximum): the
+    shared-memory sorting network, against the oracle's full order."""
+    from paper_2606_22983_gb300 import lv
+    from oracle.policy import order_global
+    rng = np.random.default_rng(S)
+    maxb, T = 4, 16
+    pages = S * maxb
+    pool = _tiny_pool(max_sessions=S, max_blocks=maxb, hbm_pages=pages, hbm_budget_pages=pages,
+                      host_pages=pages)
+    try:
+        placement, ctx = _random_placement(rng, S, maxb, T, pages, pages)
+        pool.import_placement(placement, ctx)
+        st = _random_states(rng, S)
+        pool.set_sessions(st)
+        pool.sync()
+        osess = _oracle_states(pool.get_sessions())
+        nb = -(-ctx.astype(np.int64) // T)
+        now = int(rng.integers(0, 12_000_000))
+        for fallback in (False, True):
+            want = np.stack(order_global(placement.astype(np.int64), nb, osess, now, 0, 3_000_000,
+                                         80_000, 0, fallback), axis=1)
+            got, n = pool.select(now, lv.LV_ALL, lv.LV_SELECT_FALLBACK if fallback else 0)
+            assert np.array_equal(got.cpu().numpy().astype(np.int64), want), fallback
+            got, n = pool.select(now, 100, lv.LV_SELECT_FALLBACK if fallback else 0)
+            assert np.array_equal(got.cpu().numpy().astype(np.int64), want[:100]), fallback
+        assert pool.sync(raise_on_error=False) == 0
+    finally:
+        pool.close()
