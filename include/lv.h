@@ -205,7 +205,12 @@ typedef struct lv_stats {
    counters) and, when desc->host_kv is NULL, a mapped page-locked host pool.
    All tables start empty.  Returns LV_ERR_INVALID for a bad descriptor (sizes
    out of range, P not a multiple of 16, a misaligned or non-device KV pointer,
-   a host_kv that is not page-locked), LV_ERR_OOM or LV_ERR_CUDA. */
+   a host_kv that is not page-locked), LV_ERR_OOM or LV_ERR_CUDA.
+   Launch shapes can be overridden through the environment at creation time (for
+   tuning sweeps): LV_EXCHANGE_CTAS (the exchange copy's grid, default a third of
+   the SMs) or LV_EXCHANGE_CTAS_PER_SM; LV_STAGE_STAGES and LV_STAGE_CTAS_PER_SM
+   (the TMA pack/unpack kernel, default about 48 KiB of stages per CTA and two
+   CTAs per SM); LV_STAGE_KERNEL=lsu (16-byte copies instead of TMA). */
 lv_status lv_pool_create(const lv_pool_desc* desc, lv_stream stream, lv_pool** out);
 
 /* Waits for the pool's outstanding work on `stream`, then frees everything the
