@@ -609,6 +609,69 @@ enum { LV_FAULT_NONE = 0, LV_FAULT_HOST_ALLOC = 1, LV_FAULT_HBM_ALLOC = 2, LV_FA
 lv_status lv_inject_fault(lv_pool* pool, int32_t kind, int32_t after);
 lv_status lv_selftest_wait(lv_pool* pool, int64_t limit_us, lv_stream stream);
 
+/* ------------------------------------------------------ preload controller */
+
+/* Section 5.2, the preload controller, over the pool's own calls.  Readings (the
+   paper describes it in prose):
+   - Admission: a preload of B bytes requested at time t is admitted if, queued
+     behind the transfers already on a modelled host->device link of
+     link_bytes_per_us, it finishes by the predicted start of the session's turn,
+     t_speech + lead (lead: the session's moving average of turn start minus
+     speech start, integer EMA of weight 1/4, first sample sets it; lead_prior_us
+     before any sample), and if the pages it must evict fit in the host tier with
+     max_blocks slots still free.
+   - A refused preload waits and is re-checked at every later tick until it is
+     admitted, its deadline passes (given up), or the turn begins (given up).
+   - An admitted preload evicts what it needs (the ranked order, no fallback tier)
+     and commits that at once; it reserves and fills its HBM pages at once but
+     commits them only at the first tick at or after its modelled finish.  A turn
+     that begins first cancels the reservation (the turn then loads itself).
+   - A completed preload protects the session until finish + protect_us; when the
+     protected sessions' resident pages exceed cap_pages, the oldest protections
+     (earliest end, then lower session id) are dropped.
+   - A turn's own synchronous load occupies the modelled link too
+     (lv_controller_turn_loaded).
+   The hooks are called in event order: lv_controller_tick at every event, then
+   lv_controller_turn_begin before a turn, lv_controller_speech at a speech start
+   or barge-in.  Each hook waits on the host for the work queued before it on
+   `stream` (it reads host blocks, allocation counts and session states). */
+typedef struct lv_controller lv_controller;
+typedef struct lv_controller_desc {
+  int64_t link_bytes_per_us;   /* > 0 */
+  int64_t lead_prior_us;       /* >= 0 */
+  int64_t cap_pages;           /* resident pages of protected sessions at most; -1: no cap */
+  int32_t mode;                /* LV_MODE_* of the preloads' and evictions' copies */
+  int32_t reserved;            /* must be 0 */
+} lv_controller_desc;
+/* decision records, in the order the decisions were taken */
+enum { LV_CTL_ADMITTED = 1, LV_CTL_COMPLETED = 2, LV_CTL_CANCELLED = 3, LV_CTL_GIVEN_UP = 4,
+       LV_CTL_UNPROTECTED = 5, LV_CTL_EVICTED = 6 };
+typedef struct lv_controller_record {
+  int32_t kind;                /* LV_CTL_* */
+  int32_t sid;                 /* the session (EVICTED: the session being preloaded) */
+  int64_t start_us, finish_us, deadline_us;   /* ADMITTED: the modelled transfer */
+  int64_t n;                   /* ADMITTED: pages loaded; EVICTED: victims */
+  int64_t data_offset;         /* ADMITTED: n HBM pages; EVICTED: n (sid, blk, page) triples */
+} lv_controller_record;
+typedef struct lv_controller_counters {
+  int64_t admitted, completed, waited, given_up, cancelled, hits, victims, pages_in;
+} lv_controller_counters;
+lv_status lv_controller_create(lv_pool* pool, const lv_controller_desc* d, lv_controller** out);
+/* Cancels pending preloads (their reservations are released) and frees the
+   controller; call it before lv_pool_destroy of its pool. */
+lv_status lv_controller_destroy(lv_controller* c, lv_stream stream);
+lv_status lv_controller_tick(lv_controller* c, int64_t now_us, lv_stream stream);
+lv_status lv_controller_speech(lv_controller* c, int32_t sid, int64_t now_us, lv_stream stream);
+lv_status lv_controller_turn_begin(lv_controller* c, int32_t sid, int64_t now_us, lv_stream stream);
+lv_status lv_controller_turn_loaded(lv_controller* c, int64_t now_us, int64_t pages);
+/* Moves the records taken since the last call (and their int32 data) to the caller.
+   With too small a capacity nothing moves, *n_records and *n_data receive the sizes
+   needed, and the call returns LV_ERR_INVALID. */
+lv_status lv_controller_records(lv_controller* c, lv_controller_record* records, int64_t capacity,
+                                int64_t* n_records, int32_t* data, int64_t data_capacity,
+                                int64_t* n_data);
+lv_status lv_controller_counters_get(lv_controller* c, lv_controller_counters* out);
+
 const char* lv_status_str(lv_status s);
 int32_t lv_version(void);
 

@@ -627,6 +627,17 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
 
 }  // namespace
 
+namespace lv {
+void pool_shape(const lv_pool* pool, int32_t* sessions, int32_t* max_blocks, int64_t* page_bytes,
+                int64_t* budget, int64_t* host_pages) {
+  *sessions = pool->d.S;
+  *max_blocks = pool->d.maxB;
+  *page_bytes = (int64_t)pool->d.J * pool->d.P;
+  *budget = pool->d.budget;
+  *host_pages = pool->d.host_pages;
+}
+}  // namespace lv
+
 extern "C" {
 
 lv_status lv_pool_create(const lv_pool_desc* desc, lv_stream stream, lv_pool** out) {

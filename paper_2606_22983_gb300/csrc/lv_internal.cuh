@@ -177,5 +177,8 @@ cudaError_t launch_selftest_wait(const DevPool& p, long long limit_ns, cudaStrea
 cudaError_t launch_schedule(const lv_sched_params& q, const lv_request* reqs, int n, int32_t* order,
                             int32_t* batch, long long* ctl, cudaStream_t s);
 cudaError_t configure_kernels();   // once per device, before the first launch
+// lv_api.cu: the shape of a pool (for the controller)
+void pool_shape(const lv_pool* pool, int32_t* sessions, int32_t* max_blocks, int64_t* page_bytes,
+                int64_t* budget, int64_t* host_pages);
 
 }  // namespace lv

@@ -63,6 +63,19 @@ class lv_turn_desc(ctypes.Structure):
                 ("append_tokens", ctypes.c_int32), ("flags", ctypes.c_uint32)]
 
 
+class lv_controller_desc(ctypes.Structure):
+    _fields_ = [("link_bytes_per_us", ctypes.c_int64), ("lead_prior_us", ctypes.c_int64),
+                ("cap_pages", ctypes.c_int64), ("mode", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+class lv_controller_counters(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int64) for n in ("admitted", "completed", "waited", "given_up",
+                                               "cancelled", "hits", "victims", "pages_in")]
+
+    def as_dict(self):
+        return {n: int(getattr(self, n)) for n, _ in self._fields_}
+
+
 class lv_stats(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int64) for n in (
         "hbm_allocated", "host_allocated", "hbm_budget_pages", "host_pages", "error",
@@ -115,6 +128,10 @@ VICTIM_DTYPE = np.dtype([("sid", "<i4"), ("blk", "<i4"), ("page", "<i4")])
 RESIDENT_DTYPE = np.dtype([("k", "<i8"), ("n_found", "<i8"), ("n_victims", "<i8"), ("n_loaded", "<i8"),
                            ("n_appended", "<i8"), ("status", "<i4"), ("sid", "<i4")])
 REMAP_DTYPE = np.dtype([("sid", "<i4"), ("blk", "<i4"), ("loc", "<i4")])
+CTL_RECORD_DTYPE = np.dtype([("kind", "<i4"), ("sid", "<i4"), ("start_us", "<i8"), ("finish_us", "<i8"),
+                             ("deadline_us", "<i8"), ("n", "<i8"), ("data_offset", "<i8")])
+LV_CTL_ADMITTED, LV_CTL_COMPLETED, LV_CTL_CANCELLED, LV_CTL_GIVEN_UP, LV_CTL_UNPROTECTED, \
+    LV_CTL_EVICTED = 1, 2, 3, 4, 5, 6
 assert SESSION_DTYPE.itemsize == 72 and EVENT_DTYPE.itemsize == 32
 assert VICTIM_DTYPE.itemsize == 12 and REMAP_DTYPE.itemsize == 12
 
@@ -140,6 +157,14 @@ def _load():
         "lv_turn": [vp, ctypes.POINTER(lv_turn_desc), vp, vp, vp, vp, vp, vp, vp],
         "lv_join": [vp, vp],
         "lv_page_checksums": [vp, vp, i64, vp, vp],
+        "lv_controller_create": [vp, ctypes.POINTER(lv_controller_desc), ctypes.POINTER(vp)],
+        "lv_controller_destroy": [vp, vp],
+        "lv_controller_tick": [vp, i64, vp],
+        "lv_controller_speech": [vp, i32, i64, vp],
+        "lv_controller_turn_begin": [vp, i32, i64, vp],
+        "lv_controller_turn_loaded": [vp, i64, i64],
+        "lv_controller_records": [vp, vp, i64, vp, vp, i64, vp],
+        "lv_controller_counters_get": [vp, ctypes.POINTER(lv_controller_counters)],
         "lv_timing_enable": [vp, i32],
         "lv_pack_pages": [vp, vp, i64, vp, vp],
         "lv_schedule": [vp, ctypes.POINTER(lv_sched_params), vp, i32, vp, vp, vp],
@@ -183,7 +208,10 @@ EXPORTED = ("lv_pool_create", "lv_pool_destroy", "lv_pool_host_ptr", "lv_pool_im
             "lv_get_stats", "lv_clear_error", "lv_status_str", "lv_version",
             "lv_select_victims_noalloc", "lv_timing_enable", "lv_timing_read", "lv_pack_pages",
             "lv_unpack_pages", "lv_pool_host_device_ptr", "lv_schedule", "lv_inject_fault",
-            "lv_selftest_wait", "lv_turn", "lv_join", "lv_page_checksums")
+            "lv_selftest_wait", "lv_turn", "lv_join", "lv_page_checksums",
+            "lv_controller_create", "lv_controller_destroy", "lv_controller_tick",
+            "lv_controller_speech", "lv_controller_turn_begin", "lv_controller_turn_loaded",
+            "lv_controller_records", "lv_controller_counters_get")
 
 
 def lib():
@@ -310,6 +338,54 @@ def lv_turn(pool, sid, now_us, append_tokens, reply_audio_us, reply_units, outs=
 def lv_page_checksums(pool, pages, n, sums_out, stream=None):
     _check(_lib.lv_page_checksums(pool, ptr(pages), n, ptr(sums_out), stream_handle(stream)),
            "lv_page_checksums")
+
+
+def lv_controller_create(pool, link_bytes_per_us, lead_prior_us, cap_pages=None, mode=LV_MODE_AUTO):
+    d = lv_controller_desc(link_bytes_per_us=link_bytes_per_us, lead_prior_us=lead_prior_us,
+                           cap_pages=-1 if cap_pages is None else cap_pages, mode=mode, reserved=0)
+    out = ctypes.c_void_p()
+    _check(_lib.lv_controller_create(pool, ctypes.byref(d), ctypes.byref(out)), "lv_controller_create")
+    return out.value
+
+
+def lv_controller_destroy(ctl, stream=None):
+    _check(_lib.lv_controller_destroy(ctl, stream_handle(stream)), "lv_controller_destroy")
+
+
+def lv_controller_tick(ctl, now_us, stream=None):
+    _check(_lib.lv_controller_tick(ctl, now_us, stream_handle(stream)), "lv_controller_tick")
+
+
+def lv_controller_speech(ctl, sid, now_us, stream=None):
+    _check(_lib.lv_controller_speech(ctl, sid, now_us, stream_handle(stream)), "lv_controller_speech")
+
+
+def lv_controller_turn_begin(ctl, sid, now_us, stream=None):
+    _check(_lib.lv_controller_turn_begin(ctl, sid, now_us, stream_handle(stream)),
+           "lv_controller_turn_begin")
+
+
+def lv_controller_turn_loaded(ctl, now_us, pages):
+    _check(_lib.lv_controller_turn_loaded(ctl, now_us, pages), "lv_controller_turn_loaded")
+
+
+def lv_controller_records(ctl):
+    """The decision records since the last call and their int32 data."""
+    n, nd = ctypes.c_int64(), ctypes.c_int64()
+    st = _lib.lv_controller_records(ctl, None, 0, ctypes.byref(n), None, 0, ctypes.byref(nd))
+    if st == LV_OK:
+        return np.zeros(0, CTL_RECORD_DTYPE), np.zeros(0, np.int32)
+    recs = np.zeros(n.value, CTL_RECORD_DTYPE)
+    data = np.zeros(max(nd.value, 1), np.int32)
+    _check(_lib.lv_controller_records(ctl, recs.ctypes.data, n.value, ctypes.byref(n), data.ctypes.data,
+                                      data.size, ctypes.byref(nd)), "lv_controller_records")
+    return recs, data[:nd.value]
+
+
+def lv_controller_counters_get(ctl) -> dict:
+    c = lv_controller_counters()
+    _check(_lib.lv_controller_counters_get(ctl, ctypes.byref(c)), "lv_controller_counters_get")
+    return c.as_dict()
 
 
 def lv_join(pool, stream=None):

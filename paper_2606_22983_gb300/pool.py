@@ -81,8 +81,18 @@ class KVPool:
                 self.host_dev = torch.as_tensor(cai, device=self.device).view(host_pages, self.J, self.P)
 
     # ------------------------------------------------------------------ life
+    def attach(self, obj):
+        """Objects holding native state over this pool (a preload controller); they are
+        closed before the pool is destroyed."""
+        if not hasattr(self, "_attached"):
+            self._attached = []
+        self._attached.append(obj)
+
     def close(self):
         if getattr(self, "handle", None):
+            for obj in getattr(self, "_attached", []):
+                obj.close()
+            self._attached = []
             self.host_dev = None
             lv.lv_pool_destroy(self.handle, self.stream)
             self.handle = None
