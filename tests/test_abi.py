@@ -66,6 +66,12 @@ int main(void) {
   F(lv_resident_result, n_loaded); F(lv_resident_result, n_appended); F(lv_resident_result, status);
   F(lv_resident_result, sid);
   printf("sizeof lv_turn_desc %zu\n", sizeof(lv_turn_desc));
+  printf("sizeof lv_controller_desc %zu\n", sizeof(lv_controller_desc));
+  printf("sizeof lv_controller_counters %zu\n", sizeof(lv_controller_counters));
+  printf("sizeof lv_controller_record %zu\n", sizeof(lv_controller_record));
+  F(lv_controller_record, kind); F(lv_controller_record, sid); F(lv_controller_record, start_us);
+  F(lv_controller_record, finish_us); F(lv_controller_record, deadline_us); F(lv_controller_record, n);
+  F(lv_controller_record, data_offset);
   F(lv_turn_desc, sid); F(lv_turn_desc, num_candidates); F(lv_turn_desc, candidates);
   F(lv_turn_desc, now_us); F(lv_turn_desc, reply_audio_us); F(lv_turn_desc, reply_units);
   F(lv_turn_desc, append_tokens); F(lv_turn_desc, flags);
@@ -101,6 +107,11 @@ int main(void) {
     assert got["lv_request"] == lv.REQUEST_DTYPE.itemsize == 48
     assert got["lv_sched_params"] == ctypes.sizeof(lv.lv_sched_params)
     assert got["lv_turn_desc"] == ctypes.sizeof(lv.lv_turn_desc)
+    assert got["lv_controller_desc"] == ctypes.sizeof(lv.lv_controller_desc)
+    assert got["lv_controller_counters"] == ctypes.sizeof(lv.lv_controller_counters)
+    assert got["lv_controller_record"] == lv.CTL_RECORD_DTYPE.itemsize
+    for name in lv.CTL_RECORD_DTYPE.names:
+        assert lv.CTL_RECORD_DTYPE.fields[name][1] == got[f"lv_controller_record.{name}"][0], name
     for name, _ in lv.lv_turn_desc._fields_:
         assert getattr(lv.lv_turn_desc, name).offset == got[f"lv_turn_desc.{name}"][0], name
     assert got["lv_request.play_buffer_us"][0] == lv.REQUEST_DTYPE.fields["play_buffer_us"][1]
