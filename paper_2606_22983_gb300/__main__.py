@@ -25,6 +25,10 @@ def main(argv=None) -> int:
     ap.add_argument("--tiers", type=int, choices=(0, 1), default=0, help="1: inclusive tiers")
     ap.add_argument("--policy", type=int, choices=(0, 1), default=0, help="1: LRU baseline")
     ap.add_argument("--events", type=int, default=0, help="run only the first N events")
+    ap.add_argument("--controller", type=int, default=0, metavar="BYTES_PER_US",
+                    help="preloads through the Section 5.2 controller with this modelled link "
+                         "(host-driven exchange driver; 0: every preload admitted)")
+    ap.add_argument("--cap-pages", type=int, default=-1, help="the controller's protected-KV cap")
     args = ap.parse_args(argv)
 
     import torch
@@ -38,8 +42,14 @@ def main(argv=None) -> int:
     pool = pool_for(wl)
     try:
         fill_random(pool, args.seed)
-        gm = KVManager(pool, perms=wl.perms, rank_on="none", record=True, driver=args.driver,
-                       mode=args.mode, order_fn=scatter_order)
+        if args.controller > 0:
+            from .controller import ControlledKVManager
+            gm = ControlledKVManager(pool, link_bytes_per_us=args.controller,
+                                     cap_pages=None if args.cap_pages < 0 else args.cap_pages,
+                                     perms=wl.perms, mode=args.mode, order_fn=scatter_order)
+        else:
+            gm = KVManager(pool, perms=wl.perms, rank_on="none", record=True, driver=args.driver,
+                           mode=args.mode, order_fn=scatter_order)
         n = wl.n_events if args.events <= 0 else min(args.events, wl.n_events)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         turn_ms, load_ms = [], []
@@ -65,6 +75,7 @@ def main(argv=None) -> int:
         print(json.dumps({
             "workload": args.workload, "seed": args.seed, "events": n, "driver": args.driver,
             "mode": args.mode, "tiers": args.tiers, "policy": args.policy,
+            "controller_link_bytes_per_us": args.controller or None,
             "sessions": spec.n_sessions, "hbm_budget_pages": spec.hbm_budget_pages,
             "host_pages": wl.spec.host_pages, "page_bytes": pool.J * pool.P,
             "turns": len(turn_ms), "turns_loading_on_path": len(load_ms),
