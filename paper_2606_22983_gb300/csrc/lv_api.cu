@@ -671,6 +671,7 @@ lv_status lv_pool_import(lv_pool* pool, const int32_t* placement, const int32_t*
   cudaStream_t s = as_stream(stream);
   DevPool& d = pool->d;
   try {
+    LV_TRY(join_copies(pool, s));   // a new placement: no copy of the old one may still run
     Staging st(pool, s);
     const void *pl = nullptr, *cx = nullptr;
     lv_status r;
