@@ -23,6 +23,11 @@ Readings:
     foreground turn that cannot otherwise run), protected sessions that are
     not running form a second tier, ordered by the same rule after every
     normally eligible block.  Pinned running KV is never a candidate.
+
+Parity status: formulation A is pinned against formulation B, against brute
+force over all block orders on tiny pools, and against hand-worked orders of
+Section 5.1's rules.  The tie-breaks and the T_play reading of the counter
+mode are readings: parity unpinned against the paper for those choices.
 """
 from __future__ import annotations
 

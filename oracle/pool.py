@@ -35,6 +35,12 @@ Tiers (the paper does not say whether the host copy is kept after a reload):
     Clean copies are never reclaimed for other blocks, so the host tier must
     be able to hold every block (otherwise an eviction fails with NO_HOST,
     exactly as in the exclusive mode).
+
+Parity status: allocation, copy and remap are pinned by closed forms and
+invariants (owners and tables stay inverse, every byte lands where its block
+is mapped, a failed transfer leaves the mapping unchanged).  The inclusive
+tier is a reading: it is pinned by invariance (the same workload leaves the
+same bytes and tables under both tiers) and is otherwise parity unpinned.
 """
 from __future__ import annotations
 

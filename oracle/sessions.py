@@ -20,6 +20,11 @@ Readings (the paper does not fix these):
   * A barge-in discards the unplayed part of the reply (Section 3), so the
     remaining playback becomes zero and the reply is finished without a
     completion time.
+
+Parity status: the event updates are pinned by hand-worked timelines and by
+invariants (a barge-in leaves no playback, protection ends at the turn start).
+The EMA weight 1/4, the first-sample rule and the protection window are
+readings: parity unpinned against the paper for those constants.
 """
 from __future__ import annotations
 
