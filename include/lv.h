@@ -497,14 +497,13 @@ lv_status lv_read_tables(lv_pool* pool, int32_t* tables, int32_t* hbm_owner,
    pageable host pointers are rejected with LV_ERR_INVALID because staging them
    would need an allocation.
 
-   Its working memory is one array of LV_NOALLOC_MAX_SESSIONS x 24 bytes plus
-   256 bytes (96.25 KiB) compiled into liblv as device memory: every GPU that
+   Its working memory is one array of LV_NOALLOC_MAX_SESSIONS x 12 bytes plus
+   256 bytes (48.25 KiB) compiled into liblv as device memory: every GPU that
    loads the library holds it until the process exits.  num_sessions above
    LV_NOALLOC_MAX_SESSIONS is rejected with LV_ERR_INVALID.  The call allocates
    nothing (no cudaMalloc, cudaFree or allocating library routine).  The first
-   call on a device looks up that array's device address (cudaGetSymbolAddress)
-   and sets a kernel attribute, so make the first call on each device before
-   any stream capture.  All calls on a device share the one array and each call
+   call on a device looks up that array's device address (cudaGetSymbolAddress),
+   so make the first call on each device before any stream capture.  All calls on a device share the one array and each call
    starts by clearing its counters: calls whose execution overlaps on the GPU
    (two streams, or two host threads) race and may return wrong victims, so
    order them, for example on one stream. */

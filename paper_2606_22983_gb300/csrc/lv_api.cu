@@ -522,8 +522,6 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       (st = dev_alloc(pool, &d.ctl, (size_t)lv::C_N)) != LV_OK ||
       (st = dev_alloc(pool, &d.skey, d.S)) != LV_OK ||
       (st = dev_alloc(pool, &d.scount, d.S)) != LV_OK ||
-      (st = dev_alloc(pool, &d.sorder, d.S)) != LV_OK ||
-      (st = dev_alloc(pool, &d.soff, d.S)) != LV_OK ||
       (st = dev_alloc(pool, &d.page_tag, (size_t)d.hbm_pages)) != LV_OK)
     return fail(st);
   lv::ResidentScratch& rs = pool->rs;
@@ -575,7 +573,6 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
     if (n >= 1 && n <= pool->num_sms * 16) pool->exchange_ctas = n;
   }
 
-  if (lv::configure_kernels() != cudaSuccess) return fail(LV_ERR_CUDA);
   if (const char* env = std::getenv("LV_STAGE_STAGES")) {   // TMA pack/unpack stages per CTA
     const int st = std::atoi(env);
     if (st >= 2 && st <= 16) d.stages = st;

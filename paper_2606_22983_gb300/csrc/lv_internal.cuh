@@ -67,8 +67,6 @@ struct DevPool {
   // ranking scratch
   unsigned long long* skey;  // [S] session sort key (0 = not a candidate)
   int32_t* scount;           // [S] resident blocks of the session
-  int32_t* sorder;           // [S] session id at rank r
-  long long* soff;           // [S] first victim position of rank r
   // exchange scratch
   unsigned long long* page_tag;  // [hbm_pages] epoch << 32 | victim index (| paired bit)
 };
@@ -176,7 +174,6 @@ cudaError_t launch_selftest_wait(const DevPool& p, long long limit_ns, cudaStrea
 // lv_sched.cu
 cudaError_t launch_schedule(const lv_sched_params& q, const lv_request* reqs, int n, int32_t* order,
                             int32_t* batch, long long* ctl, cudaStream_t s);
-cudaError_t configure_kernels();   // once per device, before the first launch
 // lv_api.cu: the shape of a pool (for the controller)
 void pool_shape(const lv_pool* pool, int32_t* sessions, int32_t* max_blocks, int64_t* page_bytes,
                 int64_t* budget, int64_t* host_pages);

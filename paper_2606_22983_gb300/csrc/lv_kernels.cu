@@ -1,6 +1,6 @@
 // CUDA kernels of the KV swap path (sm_103a).
 //
-//   ranking   k_rank_census -> k_rank_sort -> k_rank_emit   (Section 5.1, Eq. 4)
+//   ranking   k_rank_census -> k_rank_emit                (Section 5.1, Eq. 4)
 //   allocate  k_alloc, k_alloc_out                           (lowest free, Section 5.1)
 //   move      k_swap_out / k_swap_in                         (Section 5, Fig. 6; Section 5.2)
 //             k_exchange_plan -> k_exchange_copy             (both directions in one step)
@@ -351,86 +351,34 @@ k_rank_census(DevPool p, long long now_us, bool fallback) {
   }
 }
 
-constexpr int kSortThreads = 1024;
+constexpr int kEmitThreads = 256;
 
-// One CTA: bitonic sort of the session keys (descending), scan of the counts
-// in rank order, and the number of victims to emit.
-__global__ void __launch_bounds__(kSortThreads)
-k_rank_sort(DevPool p, long long k, const long long* k_dev, bool fallback, long long* count_dev,
-            int N) {
+// One CTA per session.  The victim order takes the sessions by decreasing key
+// (keys are distinct: each holds its session id), so a session's first
+// position in the order is the number of resident blocks of the sessions with
+// a larger key; the CTA sums those counts over the census, then writes its
+// own resident blocks, suffix first (or ascending), while positions stay below
+// the selection count min(k, all resident candidates).  CTA 0 publishes the
+// count and the counters.
+__global__ void __launch_bounds__(kEmitThreads)
+k_rank_emit(DevPool p, long long k, const long long* k_dev, bool fallback, long long* count_dev,
+            lv_victim* __restrict__ out) {
+  const int32_t sid = blockIdx.x;
+  const unsigned long long key = p.skey[sid];
+  if (key == 0ull && sid != 0) return;
   if (k_dev) k = *k_dev;   // k decided on the device (lv_make_resident)
-  extern __shared__ unsigned char smem_raw[];
-  unsigned long long* keys = reinterpret_cast<unsigned long long*>(smem_raw);
-  int32_t* vals = reinterpret_cast<int32_t*>(keys + N);
-  if (N <= kSortThreads) {
-    // one key per thread: partners closer than a warp trade through shuffles, the
-    // others through shared memory; the pair (lower, upper) swaps exactly when the
-    // shared-memory network below would
-    const int i = threadIdx.x;
-    unsigned long long key = (i < N && i < p.S) ? p.skey[i] : 0ull;
-    int32_t val = i;
-    for (int kk = 2; kk <= N; kk <<= 1) {
-      for (int j = kk >> 1; j > 0; j >>= 1) {
-        unsigned long long pk;
-        int32_t pv;
-        if (j >= 32) {
-          if (i < N) { keys[i] = key; vals[i] = val; }
-          __syncthreads();
-          if (i < N) { pk = keys[i ^ j]; pv = vals[i ^ j]; }
-          __syncthreads();
-        } else {
-          pk = __shfl_xor_sync(0xffffffffu, key, j);
-          pv = __shfl_xor_sync(0xffffffffu, val, j);
-        }
-        if (i < N) {
-          const bool lower = (i & j) == 0;
-          const unsigned long long lo = lower ? key : pk, hi = lower ? pk : key;
-          const bool swap = ((i & kk) == 0) ? (lo < hi) : (lo > hi);
-          if (swap) { key = pk; val = pv; }
-        }
-      }
-    }
-    if (i < N) { keys[i] = key; vals[i] = val; }
-    __syncthreads();
-  } else {
-    for (int i = threadIdx.x; i < N; i += kSortThreads) {
-      keys[i] = i < p.S ? p.skey[i] : 0ull;
-      vals[i] = i;
-    }
-    __syncthreads();
-    for (int kk = 2; kk <= N; kk <<= 1) {
-      for (int j = kk >> 1; j > 0; j >>= 1) {
-        for (int i = threadIdx.x; i < N; i += kSortThreads) {
-          const int ixj = i ^ j;
-          if (ixj > i) {
-            const unsigned long long a = keys[i], b = keys[ixj];
-            const bool swap = ((i & kk) == 0) ? (a < b) : (a > b);
-            if (swap) {
-              keys[i] = b; keys[ixj] = a;
-              const int32_t t = vals[i]; vals[i] = vals[ixj]; vals[ixj] = t;
-            }
-          }
-        }
-        __syncthreads();
-      }
-    }
+  long long before = 0, all = 0;
+  for (int32_t j = threadIdx.x; j < p.S; j += kEmitThreads) {
+    const unsigned long long kj = p.skey[j];
+    const long long cj = kj ? p.scount[j] : 0;
+    all += cj;
+    before += kj > key ? cj : 0;
   }
-  // counts in rank order, each thread a contiguous run of ranks
-  const int per = (N + kSortThreads - 1) / kSortThreads;
-  const int r0 = min(N, (int)threadIdx.x * per), r1 = min(N, r0 + per);
-  long long local = 0;
-  for (int r = r0; r < r1; ++r) local += keys[r] ? p.scount[vals[r]] : 0;
-  long long total;
-  long long run = block_excl_scan<kSortThreads>(local, &total);
-  for (int r = r0; r < r1; ++r) {
-    if (r < p.S) {
-      p.sorder[r] = vals[r];
-      p.soff[r] = run;
-    }
-    run += keys[r] ? p.scount[vals[r]] : 0;
-  }
-  if (threadIdx.x == 0) {
-    const long long n_out = k < total ? k : total;
+  long long off, total;
+  block_excl_scan<kEmitThreads>(before, &off);
+  block_excl_scan<kEmitThreads>(all, &total);
+  const long long n_out = k < total ? k : total;
+  if (sid == 0 && threadIdx.x == 0) {
     p.ctl[C_SEL_COUNT] = n_out;
     p.ctl[C_SEL_TOTAL] = total;
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_SELECTS]), 1ull);
@@ -440,20 +388,7 @@ k_rank_sort(DevPool p, long long k, const long long* k_dev, bool fallback, long 
     if (fallback) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_FALLBACK]), 1ull);
     if (count_dev) *count_dev = n_out;
   }
-}
-
-constexpr int kEmitThreads = 256;
-
-// One CTA per rank: writes the session's resident blocks, suffix first (or
-// ascending), to its slice of the victim list, up to the global count.
-__global__ void __launch_bounds__(kEmitThreads)
-k_rank_emit(DevPool p, lv_victim* __restrict__ out) {
-  const int r = blockIdx.x;
-  const long long n_out = p.ctl[C_SEL_COUNT];
-  const long long off = p.soff[r];
-  if (off >= n_out) return;
-  const int32_t sid = p.sorder[r];
-  if (sid < 0 || sid >= p.S || p.skey[sid] == 0ull) return;
+  if (key == 0ull || off >= n_out) return;
   const int32_t nb = nblocks_of(p, sid);
   const int32_t* row = p.table + (size_t)sid * p.maxB;
   const bool suffix = p.within == LV_SUFFIX_FIRST;
@@ -1587,19 +1522,11 @@ cudaError_t launch_events(const DevPool& p, const lv_event* ev, int64_t n, cudaS
 cudaError_t launch_select(const DevPool& p, int64_t now_us, int64_t k, bool fallback,
                           lv_victim* out, long long* count_dev, cudaStream_t s, int /*num_sms*/,
                           const long long* k_dev) {
-  int N = 1;
-  while (N < p.S) N <<= 1;
-  const size_t smem = (size_t)N * (sizeof(unsigned long long) + sizeof(int32_t));
   k_rank_census<<<p.S, kCensusThreads, 0, s>>>(p, now_us, fallback);
-  k_rank_sort<<<1, kSortThreads, smem, s>>>(p, k, k_dev, fallback, count_dev, N);
-  k_rank_emit<<<p.S, kEmitThreads, 0, s>>>(p, out);
+  k_rank_emit<<<p.S, kEmitThreads, 0, s>>>(p, k, k_dev, fallback, count_dev, out);
   return cudaGetLastError();
 }
 
-cudaError_t configure_kernels() {
-  // the session sort keeps up to 4096 keys and ids in dynamic shared memory (48 KiB)
-  return cudaFuncSetAttribute(k_rank_sort, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * 1024);
-}
 
 cudaError_t launch_alloc(const DevPool& p, bool hbm, int64_t n, int32_t* out, cudaStream_t s,
                          bool injected_fail) {

@@ -16,13 +16,11 @@ namespace {
 
 constexpr int kMaxSessions = LV_NOALLOC_MAX_SESSIONS;
 constexpr size_t kKeyBytes = sizeof(unsigned long long) * kMaxSessions;
-constexpr size_t kOffBytes = sizeof(long long) * kMaxSessions;
 constexpr size_t kCountBytes = sizeof(int32_t) * kMaxSessions;
-constexpr size_t kOrderBytes = sizeof(int32_t) * kMaxSessions;
 constexpr size_t kCtlBytes = sizeof(long long) * lv::C_N;
-constexpr size_t kScratchBytes = kKeyBytes + kOffBytes + kCountBytes + kOrderBytes + kCtlBytes;
+constexpr size_t kScratchBytes = kKeyBytes + kCountBytes + kCtlBytes;
 
-// The ranking scratch of every call on a device (96 KiB + 256 B).  Every GPU
+// The ranking scratch of every call on a device (48 KiB + 256 B).  Every GPU
 // that loads liblv holds one copy until the process exits.
 static __device__ __align__(256) unsigned char g_rank_scratch[kScratchBytes];
 
@@ -42,7 +40,6 @@ lv_status scratch_for_current_device(unsigned char** out) {
       cudaGetLastError();
       return LV_ERR_CUDA;
     }
-    if (lv::configure_kernels() != cudaSuccess) return LV_ERR_CUDA;
     g_scratch_dev[dev] = ptr;
   }
   *out = static_cast<unsigned char*>(g_scratch_dev[dev]);
@@ -99,14 +96,12 @@ extern "C" lv_status lv_select_victims_noalloc(const lv_rank_params* prm,
   p.sess = const_cast<lv_session_state*>(static_cast<const lv_session_state*>(sess));
   p.table = const_cast<int32_t*>(static_cast<const int32_t*>(tab));
   p.skey = reinterpret_cast<unsigned long long*>(scratch);
-  p.soff = reinterpret_cast<long long*>(scratch + kKeyBytes);
-  p.scount = reinterpret_cast<int32_t*>(scratch + kKeyBytes + kOffBytes);
-  p.sorder = reinterpret_cast<int32_t*>(scratch + kKeyBytes + kOffBytes + kCountBytes);
-  p.ctl = reinterpret_cast<long long*>(scratch + kKeyBytes + kOffBytes + kCountBytes + kOrderBytes);
+  p.scount = reinterpret_cast<int32_t*>(scratch + kKeyBytes);
+  p.ctl = reinterpret_cast<long long*>(scratch + kKeyBytes + kCountBytes);
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   // the counters and counts left by the previous call start again from zero;
-  // keys, counts, order and offsets are rewritten for every session each call
+  // keys and counts are rewritten for every session each call
   if (cudaMemsetAsync(p.ctl, 0, kCtlBytes, s) != cudaSuccess) return LV_ERR_CUDA;
   if (lv::launch_select(p, now_us, keff, (prm->flags & LV_SELECT_FALLBACK) != 0,
                         static_cast<lv_victim*>(vout), static_cast<long long*>(cout), s, 0) !=

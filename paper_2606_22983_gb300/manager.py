@@ -105,7 +105,7 @@ class KVManager:
             self.timer.start("resident")
         lv.lv_make_resident(pool.handle, sid, now_us, append_tokens, flags, -1, *outs,
                             self.res_h, pool.stream)
-        pool.launches += 8 + (1 if append_tokens else 0)
+        pool.launches += 7 + (1 if append_tokens else 0)
         if self.timer:
             self.timer.stop("resident", None)
         if not rec_bufs:
@@ -151,7 +151,7 @@ class KVManager:
         lv.lv_turn(pool.handle, sid, now_us, append_tokens, reply_us, reply_units, outs, self.res_h,
                    cand, int(cand.numel()) if cand is not None else 0, pool.stream,
                    lv.LV_RESIDENT_ASYNC_COPY if self.async_copy else 0)
-        pool.launches += 10 + (1 if sid < 0 else 0) + (1 if append_tokens else 0)
+        pool.launches += 9 + (1 if sid < 0 else 0) + (1 if append_tokens else 0)
         if not rec_bufs:
             return sid
         pool.sync(raise_on_error=False)

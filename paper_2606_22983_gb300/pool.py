@@ -135,7 +135,7 @@ class KVPool:
                                                                 device=self.device)
         lv.lv_select_victims(self.handle, now_us, min(k, lv.LV_ALL), flags, out, cap,
                              self.count_h[0:1], self.stream)
-        self.launches += 3
+        self.launches += 2
         self.sync()
         n = int(self.count_h[0])
         return out[:n], n

@@ -286,6 +286,82 @@ def test_degenerate_sizes_and_host_pointer_arguments():
         pool.close()
 
 
+def test_largest_pool_shape_and_ids():
+    """The largest shape the descriptor allows: 4096 sessions x 65536 blocks per
+    session.  Session 4095 holds a full 65536-block table (its top 1536 blocks in HBM,
+    the rest on the host), so its owner words carry the largest session and block ids.
+    The full victim order matches the oracle; evicting the top 1536 blocks fills the
+    host tier to its last slot; the tables, owners and bytes follow, and the highest
+    block comes back."""
+    import torch
+    from paper_2606_22983_gb300 import lv
+    from oracle.policy import order_global
+    S, maxb, T, hbm, host = 4096, 65536, 16, 2048, 65536
+    rng = np.random.default_rng(23)
+    pool = _tiny_pool(layers=1, kv_heads=1, head_dim=8, max_sessions=S, max_blocks=maxb,
+                      hbm_pages=hbm, hbm_budget_pages=hbm, host_pages=host)
+    try:
+        g = torch.Generator().manual_seed(23)
+        pool.kv.copy_(torch.randint(0, 256, tuple(pool.kv.shape), generator=g, dtype=torch.uint8))
+        kv0 = pool.kv.cpu().numpy()
+        pages = rng.permutation(hbm).astype(np.int32)
+        placement = np.full((S, maxb), -1, np.int32)
+        ctx = np.zeros(S, np.int32)
+        top, n_top = S - 1, 1536
+        ctx[top] = maxb * T
+        placement[top, :maxb - n_top] = -(np.arange(maxb - n_top, dtype=np.int32) + 2)
+        placement[top, maxb - n_top:] = pages[:n_top]
+        ctx[0], ctx[2047] = 70, 100 * T
+        placement[0, :5] = pages[n_top:n_top + 5]
+        placement[2047, :100] = pages[n_top + 5:n_top + 105]
+        pool.import_placement(placement, ctx)
+        st = np.zeros(S, dtype=lv.SESSION_DTYPE)
+        st["reply_n"] = 1
+        st["reply_ema_us"] = 1_000_000
+        st["reply_ema_us"][top], st["reply_ema_us"][0], st["reply_ema_us"][2047] = 9e6, 5e6, 2e6
+        pool.set_sessions(st)
+        pool.sync()
+        osess = _oracle_states(pool.get_sessions())
+        nb = -(-ctx.astype(np.int64) // T)
+        want = np.stack(order_global(placement, nb, osess, 0, 0, 3_000_000, 80_000), axis=1)
+        assert want.shape[0] == n_top + 105
+        got, n = pool.select(0, lv.LV_ALL, 0, capacity=len(want))
+        assert n == len(want) and np.array_equal(got.cpu().numpy().astype(np.int64), want)
+        # evict the top 1536: blocks 65535 .. 64000 of session 4095 into slots 64000 ..
+        v, n = pool.select(0, n_top)
+        assert n == n_top and np.array_equal(v.cpu().numpy().astype(np.int64), want[:n_top])
+        slots, commit = pool.swap_out(v, n)
+        pool.remap(commit, n)
+        pool.sync()
+        blk = np.arange(maxb - 1, maxb - 1 - n_top, -1)
+        want_slots = np.arange(maxb - n_top, maxb)
+        assert np.array_equal(slots.cpu().numpy(), want_slots)
+        tables, own_hbm, own_host = pool.tables()
+        assert np.array_equal(tables[top, blk], -(want_slots + 2))
+        assert np.array_equal(own_host[want_slots].astype(np.int64), (top << 16) | blk)
+        assert own_host[want_slots[0]] == (4095 << 16) | 65535
+        assert np.all(own_host[:maxb - n_top] == ((top << 16) | np.arange(maxb - n_top)))
+        assert np.all(own_hbm[pages[:n_top]] == -1)
+        host_img = pool.host.reshape(host, pool.J, pool.P)
+        for i in (0, 1, 700, n_top - 1):
+            assert np.array_equal(host_img[want_slots[i]], kv0[:, pages[n_top - 1 - i]])
+        assert pool.stats()["host_allocated"] == host
+        # the highest block comes back into the lowest free HBM page
+        free = np.sort(pages[:n_top])
+        pg, commit = pool.swap_in(top, torch.tensor([maxb - 1], dtype=torch.int32,
+                                                    device="cuda"), 1)
+        pool.remap(commit, 1)
+        pool.sync()
+        assert int(pg[0]) == free[0]
+        assert np.array_equal(pool.kv[:, free[0]].cpu().numpy(), kv0[:, pages[n_top - 1]])
+        tables, own_hbm, own_host = pool.tables()
+        assert tables[top, maxb - 1] == free[0] and own_hbm[free[0]] == (4095 << 16) | 65535
+        assert own_host[maxb - n_top] == -1
+        assert pool.sync(raise_on_error=False) == 0
+    finally:
+        pool.close()
+
+
 def test_turn_picks_the_first_candidate_with_host_blocks():
     """lv_turn with sid = -1: the first listed session that has a block in the host
     tier (else the first listed), then turn begin, make resident, turn end -- the

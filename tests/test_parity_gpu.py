@@ -12,7 +12,8 @@ pytestmark = pytest.mark.gpu
 
 @pytest.mark.parametrize("seed,driver,mode", [(0, "device", 0), (1, "device", 0), (0, "exchange", 0),
                                               (1, "sequential", 0), (0, "exchange", 2),
-                                              (1, "sequential", 2), (2, "exchange", 18)])
+                                              (1, "sequential", 2), (2, "exchange", 18),
+                                              (3, "device", 0), (4, "device", 0)])
 def test_tiny_workload_full_images(seed, driver, mode):
     """1000 scripted events of the tiny pool: every ranking (full order after
     each event), eviction, preload, reload and growth, with full HBM and host
