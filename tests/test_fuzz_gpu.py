@@ -1,8 +1,11 @@
 """Randomized differential test of the C ABI against the oracle: random sequences of
-ranking, swap-out, swap-in, commit, cancel, exchange, growth and monitor events on a
-tiny pool with random bytes, plus single-item calls that must be refused with the
-right status and change nothing.  After every call the block and owner tables,
-allocation counts, clean copies, session states and both byte images are compared."""
+ranking, swap-out, swap-in, commit, cancel, exchange, growth, monitor events and whole
+device-driven turns (lv_turn, most with their copies left running on the pool's copy
+stream) on a tiny pool with random bytes, plus single-item calls that must be refused
+with the right status and change nothing.  After a random half of the calls (so that a
+turn's copies are often still in flight when the next call starts, and that call must
+join them), and after the last one, the block and owner tables, allocation counts,
+clean copies, session states and both byte images are compared."""
 import numpy as np
 import pytest
 
@@ -79,12 +82,12 @@ def test_random_call_sequences_match_the_oracle(seed, tiers):
     from oracle.pool import OracleError, _enc_host
     rng, pool, om, sts, lv, se = _setup(seed, tiers)
     now = 1_000_000
-    done = dict.fromkeys(("select", "out", "in", "exchange", "append", "events", "bad"), 0)
+    done = dict.fromkeys(("select", "out", "in", "exchange", "append", "events", "turn", "bad"), 0)
     try:
         for step in range(300):
             now += int(rng.integers(0, 400_000))
-            op = rng.choice(["select", "out", "in", "exchange", "append", "events", "bad"],
-                            p=[0.1, 0.2, 0.2, 0.15, 0.1, 0.2, 0.05])
+            op = rng.choice(["select", "out", "in", "exchange", "append", "events", "turn", "bad"],
+                            p=[0.08, 0.17, 0.17, 0.13, 0.1, 0.15, 0.15, 0.05])
             where = (seed, tiers, step, op)
             if op in ("select", "out", "exchange"):
                 k = int(rng.integers(0, 12))
@@ -179,6 +182,39 @@ def test_random_call_sequences_match_the_oracle(seed, tiers):
                     ev[e] = (kind, sid, now, a, bb)
                     se.apply_event(sts[sid], kind, now, a, bb, protect_us=2_000_000)
                 pool.events(ev)
+            elif op == "turn":
+                # the oracle's turn (Section 5.1): turn begin, evict the first k of the
+                # order (protected KV as a last resort), reload every host block in block
+                # order, grow, turn end -- tried on copies first, since a turn that
+                # cannot fit is an error on the GPU
+                sid = int(rng.integers(0, S))
+                n_app = min(int(rng.integers(0, 40)) if rng.random() < 0.5 else 0,
+                            B * T - int(om.ctx[sid]))
+                trial = [x.copy() for x in sts]
+                se.apply_event(trial[sid], se.SE_TURN_BEGIN, now)
+                hb = om.host_blocks(sid)
+                new_blocks = -(-(int(om.ctx[sid]) + n_app) // T) - int(om.nblocks[sid])
+                k = max(0, int(hb.size) + new_blocks - (BUDGET - int(om.hbm_used.sum())))
+                vs, vb, vp = select_victims(om.tables, om.nblocks, trial, now, k, 0, 3_000_000,
+                                            80_000, 0, True)
+                need = int(sum(om.shadow[s_, b_] < 0 for s_, b_ in zip(vs, vb)))
+                if vs.size < k or need > HOST - int(om.host_used.sum()):
+                    continue
+                sts[sid] = trial[sid]
+                if k:
+                    slots = om.swap_out(vs, vb, vp)
+                    om.remap(vs, vb, _enc_host(slots))
+                if hb.size:
+                    pages = om.swap_in(sid, hb)
+                    om.remap(np.full(hb.size, sid), hb, pages)
+                if n_app:
+                    om.append(sid, n_app)
+                    sts[sid].ctx_tokens = int(om.ctx[sid])
+                audio, units = int(rng.integers(0, 3_000_000)), int(rng.integers(0, 60))
+                se.apply_event(sts[sid], se.SE_TURN_END, now, audio, units)
+                flags = lv.LV_RESIDENT_ASYNC_COPY if rng.random() < 0.7 else 0
+                lv.lv_turn(pool.handle, sid, now, n_app, audio, units, stream=pool.stream,
+                           flags=flags)
             else:   # a single-item call that must be refused and change nothing
                 which = int(rng.integers(0, 3))
                 if which == 0:      # commit to a page nobody reserved
@@ -216,8 +252,10 @@ def test_random_call_sequences_match_the_oracle(seed, tiers):
                     _refused(pool, lv, lv.LV_ERR_STATE, where)
                     with pytest.raises(OracleError):
                         om.cancel([int(owned[0])])
-            _compare(pool, om, sts, where)
+            if op == "bad" or rng.random() < 0.5:
+                _compare(pool, om, sts, where)
             done[op] += 1
+        _compare(pool, om, sts, (seed, tiers, "end"))
         om.check_invariants()
         # every kind of call ran, not only the ones that are always possible
         assert min(done.values()) >= 5, done
