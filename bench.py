@@ -366,6 +366,13 @@ def ours(args, torch):
 
 OVERLAP_TURNS = 40
 REMAP_BYTES_PER_ENTRY = 52   # entry 12; read+write of: table 4+4, epoch 4+4, new owner 4+4, old owner 4+4, old bitmap 4+4
+# The scattered requests one k_remap entry makes when the micro commits every page to
+# the host tier: the old location's owner is loaded and cleared and its bitmap bit
+# reduced at a random position (pages are a random permutation); the epoch mark
+# (exchange) and the new slot's owner (CAS) are returning atomics, at consecutive
+# positions here (entries follow the victim order, slots ascend).  The entry, the
+# table word and the session's length are coalesced or cached loads and are left out.
+REMAP_REQUESTS = {"load": 1, "store": 1, "reduce": 1, "atomic": 2}
 
 
 def overlap_measure(torch, pool, wl, first_turn, n_turns):
@@ -625,6 +632,30 @@ def kernel_micro(torch, pool, seed=0):
                            "entries_per_s": round(N / (ms / 1e3)), "achieved_gbs": round(gbs, 1),
                            "peak_gbs": HBM_PEAK, "frac": round(gbs / HBM_PEAK, 3),
                            "l2": "flushed before each launch"}
+        # The ceiling for remap's own traffic: the rate of each kind of scattered 4-byte
+        # request alone (lv_probe_scattered over a 16 MB array, timed like the remap, L2
+        # flushed first), each request of an entry taking its kind's share of time.
+        arr = torch.zeros(1 << 22, dtype=torch.int32, device=pool.device)
+        rates = {}
+        for i, kind in enumerate(("load", "atomic", "store", "reduce")):
+            mix = [0, 0, 0, 0]
+            mix[i] = 8
+            t = []
+            for rep in range(4):
+                flush.fill_(rep)
+                a.record()
+                lv.lv_probe_scattered(mix, arr, arr.numel(), N, None, mp.stream)
+                b.record()
+                torch.cuda.synchronize()
+                if rep:
+                    t.append(a.elapsed_time(b))
+            rates[kind] = N * 8 / (float(np.mean(t)) / 1e3)
+        model_ms = N * sum(c / rates[k] for k, c in REMAP_REQUESTS.items()) * 1e3
+        out["remap_1m"]["scattered_ceiling"] = {
+            "requests_per_entry": REMAP_REQUESTS,
+            "g_requests_per_s": {k: round(v / 1e9, 1) for k, v in rates.items()},
+            "model_ms": round(model_ms, 4), "frac": round(model_ms / ms, 3)}
+        del arr
         # and at a turn's size: 1024 entries (one whole thinker session), latency
         mp.import_placement(placement, ctx)
         lat = []

@@ -210,7 +210,9 @@ typedef struct lv_stats {
    tuning sweeps): LV_EXCHANGE_CTAS (the exchange copy's grid, default a third of
    the SMs) or LV_EXCHANGE_CTAS_PER_SM; LV_STAGE_STAGES and LV_STAGE_CTAS_PER_SM
    (the TMA pack/unpack kernel, default about 48 KiB of stages per CTA and two
-   CTAs per SM); LV_STAGE_KERNEL=lsu (16-byte copies instead of TMA). */
+   CTAs per SM); LV_STAGE_KERNEL=lsu (16-byte copies instead of TMA);
+   LV_REMAP_ENTRIES_PER_THREAD = 1, 2 or 4 (lv_remap's entries per thread,
+   default 1 while the GPU holds one thread per entry at once, else 2 or 4). */
 lv_status lv_pool_create(const lv_pool_desc* desc, lv_stream stream, lv_pool** out);
 
 /* Waits for the pool's outstanding work on `stream`, then frees everything the
@@ -449,6 +451,29 @@ lv_status lv_unpack_pages(lv_pool* pool, const void* src, const int32_t* pages, 
    Device-detected: LV_ERR_BOUNDS for a page outside the pool (its sum is 0). */
 lv_status lv_page_checksums(lv_pool* pool, const int32_t* pages, int64_t n, uint64_t* sums_out,
                             lv_stream stream);
+
+/* Scattered-access probe (an instrument, not from the paper).  Launches one
+   kernel on `stream` with `threads` threads; each makes mix->loads loads,
+   mix->atomics returning atomics (atomicExch), mix->stores stores and
+   mix->reductions reductions (atomicAnd with a constant), in that order, to
+   4-byte words of `array` (device memory, uint32 [words], owned by the caller;
+   words a power of two up to 2^32) at hashed positions, no request depending
+   on another.  Stores and atomics overwrite array words.  The caller times the
+   launch (CUDA events on `stream`).  One kind alone measures the rate at which
+   the GPU serves that kind of scattered request; a kernel's own mix per work
+   item, one thread per item, measures the ceiling of that kernel (k_remap
+   commits one entry with two loads, two returning atomics, two stores and
+   one reduction).  sink (uint32 [1], device, may be NULL) is never written in
+   practice; it keeps the loads from being removed.  LV_ERR_INVALID for a
+   count outside 0..64 or a bad size, LV_ERR_CUDA if the launch fails. */
+typedef struct lv_probe_mix {
+  int32_t loads;
+  int32_t atomics;
+  int32_t stores;
+  int32_t reductions;
+} lv_probe_mix;
+lv_status lv_probe_scattered(const lv_probe_mix* mix, uint32_t* array, int64_t words,
+                             int64_t threads, uint32_t* sink, lv_stream stream);
 
 /* Block-level allocation kept (Section 5.1): grows session sid's context by
    n_tokens; each new block takes the lowest free HBM page, in block order, and

@@ -26,6 +26,7 @@ struct lv_pool {
   int num_sms = 0;
   int32_t epoch = 0;
   int exchange_ctas = 0;           // grid of the exchange copy kernel
+  int remap_per_thread = 0;        // entries per thread of k_remap (0: by batch size)
   lv::ResidentScratch rs{};        // lv_make_resident / lv_turn buffers
   // LV_RESIDENT_ASYNC_COPY: the copies run on s_copy; consecutive steps alternate
   // between two task lists and control-word sets (rs_alt shares everything else)
@@ -602,6 +603,10 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
     if (per >= 1 && per <= 4) pool->stage_ctas = pool->num_sms * per;
   }
   if (const char* env = std::getenv("LV_STAGE_KERNEL")) pool->stage_tma = std::strcmp(env, "lsu") != 0;
+  if (const char* env = std::getenv("LV_REMAP_ENTRIES_PER_THREAD")) {   // 1, 2 or 4
+    const int e = std::atoi(env);
+    if (e == 1 || e == 2 || e == 4) pool->remap_per_thread = e;
+  }
   if (!tma_fits) pool->stage_tma = false;
   cudaMemPoolProps props{};
   props.allocType = cudaMemAllocationTypePinned;
@@ -1124,7 +1129,8 @@ lv_status lv_remap(lv_pool* pool, const lv_remap_entry* entries, int64_t n, lv_s
     lv_status r = st.in(entries, (size_t)n * sizeof(lv_remap_entry), &in);
     if (r != LV_OK) return r;
     if (++pool->epoch <= 0) pool->epoch = 1;
-    LV_TRY(lv::launch_remap(pool->d, static_cast<const lv_remap_entry*>(in), n, pool->epoch, s));
+    LV_TRY(lv::launch_remap(pool->d, static_cast<const lv_remap_entry*>(in), n, pool->epoch, s,
+                            pool->num_sms, pool->remap_per_thread));
     return st.finish();
   } catch (const std::bad_alloc&) {
     return LV_ERR_OOM;

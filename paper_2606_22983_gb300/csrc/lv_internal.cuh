@@ -119,7 +119,7 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
                             const EventPair* ev = nullptr, const long long* sid_dev = nullptr,
                             const CopyOffload* off = nullptr);
 cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, int32_t epoch,
-                         cudaStream_t s);
+                         cudaStream_t s, int num_sms, int per_thread);
 cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cudaStream_t s);
 cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32_t* pages,
                           int32_t* count, cudaStream_t s, const long long* gate = nullptr,

@@ -1009,101 +1009,184 @@ __global__ void k_selftest_wait(long long* ctl, long long limit_ns) {
 // ---------------------------------------------------------------- commit
 constexpr int kRemapThreads = 256;
 
-// One thread per entry.  The allocation counts and the commit counter change
-// by block totals (one atomic per block and counter, not one per entry).
+// The reads of one entry that do not depend on a check.
+struct RemapRead {
+  lv_remap_entry x;
+  size_t ti;            // table index (0 when out of range)
+  int32_t old;          // the block's current location
+  int32_t g;            // its clean-copy slot (inclusive tiers), or -1
+  int32_t nb;           // blocks of its session
+  uint32_t old_owner;   // owner word of the current location
+  bool in_range;
+};
+
+struct RemapCounts {
+  int ok, hbm, host, clean;
+};
+
+__device__ __forceinline__ void remap_read_entry(const DevPool& p, const lv_remap_entry* e, long long i,
+                                                 long long n, RemapRead& r) {
+  r.x = i < n ? e[i] : lv_remap_entry{-1, -1, -1};
+  r.in_range = i < n && r.x.sid >= 0 && r.x.sid < p.S && r.x.blk >= 0 && r.x.blk < p.maxB;
+  r.ti = r.in_range ? (size_t)r.x.sid * p.maxB + r.x.blk : 0;
+}
+
+__device__ __forceinline__ void remap_read_table(const DevPool& p, RemapRead& r) {
+  r.old = r.in_range ? p.table[r.ti] : -1;
+  r.g = (r.in_range && p.incl) ? p.shadow[r.ti] : -1;
+  r.nb = r.in_range ? nblocks_of(p, r.x.sid) : 0;
+}
+
+__device__ __forceinline__ void remap_read_owner(const DevPool& p, RemapRead& r) {
+  const long long old_slot = -(long long)r.old - 2;
+  r.old_owner = kOwnerNone;
+  if (r.old >= 0 && r.old < p.hbm_pages) r.old_owner = p.own_hbm[r.old];
+  else if (r.old <= -2 && old_slot < p.host_pages) r.old_owner = p.own_host[old_slot];
+}
+
+// The block's epoch mark: one accepted entry per block per call.  Returns the
+// entry's error so far (a returning atomic; the caller issues every entry's
+// mark before it looks at any result).
+__device__ __forceinline__ int remap_mark(const DevPool& p, const RemapRead& r, int32_t epoch,
+                                          int32_t& seen) {
+  if (!r.in_range || r.x.blk >= r.nb) return LV_ERR_BOUNDS;
+  seen = atomicExch(&p.mark[r.ti], epoch);
+  return 0;
+}
+
+// The new location must be a reservation nobody owns yet: one CAS checks and
+// takes it.  Issued for every entry that passed its mark, before any result is read.
+__device__ __forceinline__ int remap_claim(const DevPool& p, const RemapRead& r, int err,
+                                           uint32_t& got) {
+  if (err) return err;
+  const lv_remap_entry& x = r.x;
+  const uint32_t key = owner_key(x.sid, x.blk);
+  if (x.loc >= 0) {
+    if (x.loc >= p.hbm_pages) return LV_ERR_BOUNDS;
+    got = atomicCAS(&p.own_hbm[x.loc], kOwnerReserved, key);
+  } else if (x.loc <= -2) {
+    if (-(long long)x.loc - 2 >= p.host_pages) return LV_ERR_BOUNDS;
+    got = atomicCAS(&p.own_host[-(long long)x.loc - 2], kOwnerReserved, key);
+  } else {
+    return LV_ERR_BOUNDS;
+  }
+  return 0;
+}
+
+// Judges the claim and applies the entry: table, clean copy, old location.
+__device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& r, int err,
+                                            uint32_t got, long long i, RemapCounts& c) {
+  const lv_remap_entry& x = r.x;
+  const int32_t old = r.old, g = r.g;
+  const long long old_slot = -(long long)old - 2;
+  const bool old_hbm = old >= 0 && old < p.hbm_pages;
+  const bool old_host = old <= -2 && old_slot < p.host_pages;
+  const long long h = -(long long)x.loc - 2;
+  const uint32_t key = owner_key(x.sid, x.blk);
+  if (!err && got != kOwnerReserved) {
+    // a host location already owned by this block is fine only as its own clean copy
+    if (!(x.loc <= -2 && p.incl && (long long)g == h && got == key)) err = LV_ERR_DOUBLE_MAP;
+  }
+  if (err) {
+    set_error(p.ctl, err, i);
+    return;
+  }
+  p.table[r.ti] = x.loc;
+  if (x.loc <= -2 && g >= 0) {          // the copy becomes the location, or goes
+    p.shadow[r.ti] = -1;
+    c.clean -= 1;
+    if ((long long)g != h) {
+      p.own_host[g] = kOwnerNone;
+      atomicAnd(&p.bits_host[g >> 5], ~(1u << (g & 31)));
+      c.host += 1;
+    }
+  }
+  // the old location belongs to this block alone (one entry per block per call)
+  if (old_hbm || old_host) {
+    if (r.old_owner != key) set_error(p.ctl, LV_ERR_STATE, i);
+    if (old_hbm) {
+      p.own_hbm[old] = kOwnerNone;
+      atomicAnd(&p.bits_hbm[old >> 5], ~(1u << (old & 31)));
+      c.hbm += 1;
+    } else if (p.incl && x.loc >= 0) {   // back in HBM: the host slot stays as its clean copy
+      p.shadow[r.ti] = (int32_t)old_slot;
+      c.clean += 1;
+    } else {
+      p.own_host[old_slot] = kOwnerNone;
+      atomicAnd(&p.bits_host[old_slot >> 5], ~(1u << (old_slot & 31)));
+      c.host += 1;
+    }
+  }
+  c.ok += 1;
+}
+
+// Each thread commits E entries, i0, i0 + stride, ... (stride = the grid's
+// threads, so a warp's entries stay contiguous).  The allocation counts and the
+// commit counter change by block totals (one atomic per block and counter).
 // Inclusive tiers: a host location may be the block's own clean copy; a block
 // committed to HBM from the host tier keeps its slot as its clean copy; a
 // block committed to another host slot loses its copy.
 //
-// Every read that does not depend on a check (the block's table entry, the
-// owner word of its old location, its clean-copy slot) is issued first, before
-// any atomic or store: a random load issued after this thread's stores costs
-// several times more.  The early reads are race-free within one call: a block
-// has at most one accepted entry (the epoch mark), and another entry can take
-// an owned location only through a CAS, which then fails.
+// The kernel is bound by the latency of dependent scattered accesses (entry ->
+// table entry -> owner of the old location -> epoch mark -> claim of the new
+// location), so each step is issued for all E entries of the thread before any
+// of its results is used: every read that does not depend on a check, then
+// every mark, then every claim, then the stores.  E chains then wait together.  The early
+// reads are race-free within one call: a block has at most one accepted entry
+// (the epoch mark), a location freed by one entry is never the new location of
+// another (new locations are reservations), and another entry can take an
+// owned location only through a CAS, which then fails.  A thread's own
+// entries apply in order, so a duplicate among them meets the epoch mark too.
+template <int E>
 __global__ void __launch_bounds__(kRemapThreads)
 k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t epoch) {
-  const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
-  bool ok = false, freed_hbm = false, freed_host = false, copy_kept = false, copy_gone = false;
-  if (i < n) {
-    const lv_remap_entry x = e[i];
-    const bool in_range = x.sid >= 0 && x.sid < p.S && x.blk >= 0 && x.blk < p.maxB;
-    const size_t ti = in_range ? (size_t)x.sid * p.maxB + x.blk : 0;
-    // early reads
-    const int32_t old = in_range ? p.table[ti] : -1;
-    const long long old_slot = -(long long)old - 2;
-    const bool old_hbm = old >= 0 && old < p.hbm_pages;
-    const bool old_host = old <= -2 && old_slot < p.host_pages;
-    uint32_t old_owner = kOwnerNone;
-    if (old_hbm) old_owner = p.own_hbm[old];
-    else if (old_host) old_owner = p.own_host[old_slot];
-    const int32_t g = (in_range && p.incl) ? p.shadow[ti] : -1;
-    // checks
-    int err = 0;
-    if (!in_range || x.blk >= nblocks_of(p, x.sid)) {
-      err = LV_ERR_BOUNDS;
-    } else if (atomicExch(&p.mark[ti], epoch) == epoch) {
-      err = LV_ERR_DOUBLE_MAP;   // same block twice
-    }
-    const uint32_t key = err ? 0u : owner_key(x.sid, x.blk);
-    const long long h = -(long long)x.loc - 2;
-    if (!err) {
-      // the new location must be a reservation nobody owns yet: one CAS checks and takes it
-      if (x.loc >= 0) {
-        if (x.loc >= p.hbm_pages) err = LV_ERR_BOUNDS;
-        else if (atomicCAS(&p.own_hbm[x.loc], kOwnerReserved, key) != kOwnerReserved) err = LV_ERR_DOUBLE_MAP;
-      } else if (x.loc <= -2) {
-        if (h >= p.host_pages) err = LV_ERR_BOUNDS;
-        else {
-          const uint32_t o = atomicCAS(&p.own_host[h], kOwnerReserved, key);
-          if (o != kOwnerReserved && !(p.incl && (long long)g == h && o == key)) err = LV_ERR_DOUBLE_MAP;
-        }
-      } else {
-        err = LV_ERR_BOUNDS;
-      }
-    }
-    if (err) {
-      set_error(p.ctl, err, i);
-    } else {
-      p.table[ti] = x.loc;
-      if (x.loc <= -2 && g >= 0) {          // the copy becomes the location, or goes
-        p.shadow[ti] = -1;
-        copy_gone = true;
-        if ((long long)g != h) {
-          p.own_host[g] = kOwnerNone;
-          atomicAnd(&p.bits_host[g >> 5], ~(1u << (g & 31)));
-          freed_host = true;
-        }
-      }
-      // the old location belongs to this block alone (one entry per block per call)
-      if (old_hbm || old_host) {
-        if (old_owner != key) set_error(p.ctl, LV_ERR_STATE, i);
-        if (old_hbm) {
-          p.own_hbm[old] = kOwnerNone;
-          atomicAnd(&p.bits_hbm[old >> 5], ~(1u << (old & 31)));
-          freed_hbm = true;
-        } else if (p.incl && x.loc >= 0) {   // back in HBM: the host slot stays as its clean copy
-          p.shadow[ti] = (int32_t)old_slot;
-          copy_kept = true;
-        } else {
-          p.own_host[old_slot] = kOwnerNone;
-          atomicAnd(&p.bits_host[old_slot >> 5], ~(1u << (old_slot & 31)));
-          freed_host = true;
-        }
-      }
-      ok = true;
-    }
+  const long long stride = (long long)gridDim.x * kRemapThreads;
+  const long long i0 = blockIdx.x * (long long)kRemapThreads + threadIdx.x;
+  RemapRead r[E];
+#pragma unroll
+  for (int j = 0; j < E; ++j) remap_read_entry(p, e, i0 + j * stride, n, r[j]);
+#pragma unroll
+  for (int j = 0; j < E; ++j) remap_read_table(p, r[j]);
+#pragma unroll
+  for (int j = 0; j < E; ++j) remap_read_owner(p, r[j]);
+  // the atomics of all E entries: every mark, then every claim, each group in flight
+  // together; a thread's own duplicate meets the mark of its earlier entry
+  int err[E];
+  int32_t seen[E];
+  uint32_t got[E];
+#pragma unroll
+  for (int j = 0; j < E; ++j) {
+    seen[j] = 0;
+    err[j] = i0 + j * stride < n ? remap_mark(p, r[j], epoch, seen[j]) : -1;
   }
-  const int n_ok = __syncthreads_count(ok);
-  const int n_hbm = __syncthreads_count(freed_hbm);
-  const int n_host = __syncthreads_count(freed_host);
-  int n_clean = 0;
-  if (p.incl) n_clean = __syncthreads_count(copy_kept) - __syncthreads_count(copy_gone);
+#pragma unroll
+  for (int j = 0; j < E; ++j) {
+    if (err[j] == 0 && seen[j] == epoch) err[j] = LV_ERR_DOUBLE_MAP;   // same block twice
+    got[j] = kOwnerReserved;
+    if (err[j] >= 0) err[j] = remap_claim(p, r[j], err[j], got[j]);
+  }
+  RemapCounts c{0, 0, 0, 0};
+#pragma unroll
+  for (int j = 0; j < E; ++j)
+    if (err[j] >= 0) remap_apply(p, r[j], err[j], got[j], i0 + j * stride, c);
+  // block totals: warp sums, one shared atomic per warp, one global atomic per block
+  __shared__ int tot[4];
+  if (threadIdx.x < 4) tot[threadIdx.x] = 0;
+  __syncthreads();
+  const int ok = __reduce_add_sync(0xffffffffu, c.ok), fh = __reduce_add_sync(0xffffffffu, c.hbm);
+  const int fo = __reduce_add_sync(0xffffffffu, c.host), cl = __reduce_add_sync(0xffffffffu, c.clean);
+  if ((threadIdx.x & 31) == 0) {
+    if (ok) atomicAdd(&tot[0], ok);
+    if (fh) atomicAdd(&tot[1], fh);
+    if (fo) atomicAdd(&tot[2], fo);
+    if (cl) atomicAdd(&tot[3], cl);
+  }
+  __syncthreads();
   if (threadIdx.x == 0) {
-    if (n_hbm) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HBM_ALLOC]), (unsigned long long)-(long long)n_hbm);
-    if (n_host) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HOST_ALLOC]), (unsigned long long)-(long long)n_host);
-    if (n_ok) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_REMAP]), (unsigned long long)n_ok);
-    if (n_clean) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_CLEAN]), (unsigned long long)(long long)n_clean);
+    if (tot[1]) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HBM_ALLOC]), (unsigned long long)-(long long)tot[1]);
+    if (tot[2]) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HOST_ALLOC]), (unsigned long long)-(long long)tot[2]);
+    if (tot[0]) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_REMAP]), (unsigned long long)tot[0]);
+    if (tot[3]) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_CLEAN]), (unsigned long long)(long long)tot[3]);
   }
 }
 
@@ -1709,8 +1792,17 @@ cudaError_t launch_exchange_plan(const DevPool& p, const lv_victim* v, int64_t n
 }
 
 cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, int32_t epoch,
-                         cudaStream_t s) {
-  k_remap<<<blocks_for(n, kRemapThreads, 1ll << 30), kRemapThreads, 0, s>>>(p, e, n, epoch);
+                         cudaStream_t s, int num_sms, int per_thread) {
+  if (n <= 0) return cudaSuccess;
+  // one entry per thread while the GPU holds every thread at once; beyond that, up
+  // to four entries per thread so that their reads overlap
+  const long long resident = (long long)(num_sms > 0 ? num_sms : 1) * 2048;
+  int E = per_thread;
+  if (E != 1 && E != 2 && E != 4) E = n <= resident ? 1 : (n <= 2 * resident ? 2 : 4);
+  const unsigned grid = blocks_for((n + E - 1) / E, kRemapThreads, 1ll << 30);
+  if (E == 1) k_remap<1><<<grid, kRemapThreads, 0, s>>>(p, e, n, epoch);
+  else if (E == 2) k_remap<2><<<grid, kRemapThreads, 0, s>>>(p, e, n, epoch);
+  else k_remap<4><<<grid, kRemapThreads, 0, s>>>(p, e, n, epoch);
   return cudaGetLastError();
 }
 

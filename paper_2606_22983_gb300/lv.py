@@ -68,6 +68,10 @@ class lv_controller_desc(ctypes.Structure):
                 ("cap_pages", ctypes.c_int64), ("mode", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
+class lv_probe_mix(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in ("loads", "atomics", "stores", "reductions")]
+
+
 class lv_controller_counters(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int64) for n in ("admitted", "completed", "waited", "given_up",
                                                "cancelled", "hits", "victims", "pages_in")]
@@ -157,6 +161,7 @@ def _load():
         "lv_turn": [vp, ctypes.POINTER(lv_turn_desc), vp, vp, vp, vp, vp, vp, vp],
         "lv_join": [vp, vp],
         "lv_page_checksums": [vp, vp, i64, vp, vp],
+        "lv_probe_scattered": [ctypes.POINTER(lv_probe_mix), vp, i64, i64, vp, vp],
         "lv_controller_create": [vp, ctypes.POINTER(lv_controller_desc), ctypes.POINTER(vp)],
         "lv_controller_destroy": [vp, vp],
         "lv_controller_tick": [vp, i64, vp],
@@ -208,7 +213,7 @@ EXPORTED = ("lv_pool_create", "lv_pool_destroy", "lv_pool_host_ptr", "lv_pool_im
             "lv_get_stats", "lv_clear_error", "lv_status_str", "lv_version",
             "lv_select_victims_noalloc", "lv_timing_enable", "lv_timing_read", "lv_pack_pages",
             "lv_unpack_pages", "lv_pool_host_device_ptr", "lv_schedule", "lv_inject_fault",
-            "lv_selftest_wait", "lv_turn", "lv_join", "lv_page_checksums",
+            "lv_selftest_wait", "lv_turn", "lv_join", "lv_page_checksums", "lv_probe_scattered",
             "lv_controller_create", "lv_controller_destroy", "lv_controller_tick",
             "lv_controller_speech", "lv_controller_turn_begin", "lv_controller_turn_loaded",
             "lv_controller_records", "lv_controller_counters_get")
@@ -338,6 +343,13 @@ def lv_turn(pool, sid, now_us, append_tokens, reply_audio_us, reply_units, outs=
 def lv_page_checksums(pool, pages, n, sums_out, stream=None):
     _check(_lib.lv_page_checksums(pool, ptr(pages), n, ptr(sums_out), stream_handle(stream)),
            "lv_page_checksums")
+
+
+def lv_probe_scattered(mix, array, words, threads, sink=None, stream=None):
+    """mix = (loads, atomics, stores, reductions) per thread."""
+    m = lv_probe_mix(*(int(x) for x in mix))
+    _check(_lib.lv_probe_scattered(ctypes.byref(m), ptr(array), words, threads, ptr(sink),
+                                   stream_handle(stream)), "lv_probe_scattered")
 
 
 def lv_controller_create(pool, link_bytes_per_us, lead_prior_us, cap_pages=None, mode=LV_MODE_AUTO):

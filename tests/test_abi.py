@@ -69,6 +69,8 @@ int main(void) {
   printf("sizeof lv_controller_desc %zu\n", sizeof(lv_controller_desc));
   printf("sizeof lv_controller_counters %zu\n", sizeof(lv_controller_counters));
   printf("sizeof lv_controller_record %zu\n", sizeof(lv_controller_record));
+  printf("sizeof lv_probe_mix %zu\n", sizeof(lv_probe_mix));
+  F(lv_probe_mix, loads); F(lv_probe_mix, atomics); F(lv_probe_mix, stores); F(lv_probe_mix, reductions);
   F(lv_controller_record, kind); F(lv_controller_record, sid); F(lv_controller_record, start_us);
   F(lv_controller_record, finish_us); F(lv_controller_record, deadline_us); F(lv_controller_record, n);
   F(lv_controller_record, data_offset);
@@ -110,6 +112,9 @@ int main(void) {
     assert got["lv_controller_desc"] == ctypes.sizeof(lv.lv_controller_desc)
     assert got["lv_controller_counters"] == ctypes.sizeof(lv.lv_controller_counters)
     assert got["lv_controller_record"] == lv.CTL_RECORD_DTYPE.itemsize
+    assert got["lv_probe_mix"] == ctypes.sizeof(lv.lv_probe_mix)
+    for name, _ in lv.lv_probe_mix._fields_:
+        assert getattr(lv.lv_probe_mix, name).offset == got[f"lv_probe_mix.{name}"][0], name
     for name in lv.CTL_RECORD_DTYPE.names:
         assert lv.CTL_RECORD_DTYPE.fields[name][1] == got[f"lv_controller_record.{name}"][0], name
     for name, _ in lv.lv_turn_desc._fields_:
