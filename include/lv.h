@@ -582,8 +582,9 @@ typedef struct lv_sched_params {
    ties keep the ready set's order.  order_out (int32 [n]) receives the request
    ids in priority order U0-U1-U2; *batch_out (int32) the length of the
    admitted prefix: admission stops at the first request whose tokens or KV
-   blocks exceed what is left of the round budgets.  Runs on one CTA with
-   exact integer arithmetic.  n is 0..LV_SCHED_MAX_REQUESTS.  Device-detected:
+   blocks exceed what is left of the round budgets.  Exact integer arithmetic;
+   the pool's scheduling scratch (128 KiB), so calls on one pool are ordered on
+   one stream.  n is 0..LV_SCHED_MAX_REQUESTS.  Device-detected:
    LV_ERR_BOUNDS for a field outside its range (it is clamped). */
 lv_status lv_schedule(lv_pool* pool, const lv_sched_params* params, const lv_request* reqs, int32_t n,
                       int32_t* order_out, int32_t* batch_out, lv_stream stream);

@@ -27,6 +27,7 @@ struct lv_pool {
   int32_t epoch = 0;
   int exchange_ctas = 0;           // grid of the exchange copy kernel
   int remap_per_thread = 0;        // entries per thread of k_remap (0: by batch size)
+  unsigned char* sched_scratch = nullptr;   // lv_schedule's keys and costs
   lv::ResidentScratch rs{};        // lv_make_resident / lv_turn buffers
   // LV_RESIDENT_ASYNC_COPY: the copies run on s_copy; consecutive steps alternate
   // between two task lists and control-word sets (rs_alt shares everything else)
@@ -533,7 +534,8 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       (st = dev_alloc(pool, &rs.append, (size_t)d.maxB + 2)) != LV_OK ||
       (st = dev_alloc(pool, &rs.tasks, (size_t)d.budget + d.maxB)) != LV_OK ||
       (st = dev_alloc(pool, &rs.words, 16)) != LV_OK ||
-      (st = dev_alloc(pool, &rs.hits, (size_t)d.S)) != LV_OK)
+      (st = dev_alloc(pool, &rs.hits, (size_t)d.S)) != LV_OK ||
+      (st = dev_alloc(pool, &pool->sched_scratch, (size_t)32 * LV_SCHED_MAX_REQUESTS)) != LV_OK)
     return fail(st);
   pool->rs_alt = rs;
   if ((st = dev_alloc(pool, &pool->rs_alt.tasks, (size_t)d.budget + d.maxB)) != LV_OK ||
@@ -1110,7 +1112,7 @@ lv_status lv_schedule(lv_pool* pool, const lv_sched_params* q, const lv_request*
       return st.finish();
     }
     LV_TRY(lv::launch_schedule(*q, static_cast<const lv_request*>(rin), n, static_cast<int32_t*>(odev),
-                               static_cast<int32_t*>(bdev), pool->d.ctl, s));
+                               static_cast<int32_t*>(bdev), pool->d.ctl, pool->sched_scratch, s));
     return st.finish();
   } catch (const std::bad_alloc&) {
     return LV_ERR_OOM;

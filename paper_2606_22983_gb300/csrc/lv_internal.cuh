@@ -172,8 +172,9 @@ cudaError_t launch_tasks_pages(const DevPool& p, const int32_t* pages, int64_t n
 cudaError_t configure_stage_kernels(const DevPool& p);
 cudaError_t launch_selftest_wait(const DevPool& p, long long limit_ns, cudaStream_t s);
 // lv_sched.cu
+// scratch: device memory of 32 * LV_SCHED_MAX_REQUESTS bytes (keys and costs)
 cudaError_t launch_schedule(const lv_sched_params& q, const lv_request* reqs, int n, int32_t* order,
-                            int32_t* batch, long long* ctl, cudaStream_t s);
+                            int32_t* batch, long long* ctl, void* scratch, cudaStream_t s);
 // lv_api.cu: the shape of a pool (for the controller)
 void pool_shape(const lv_pool* pool, int32_t* sessions, int32_t* max_blocks, int64_t* page_bytes,
                 int64_t* budget, int64_t* host_pages);

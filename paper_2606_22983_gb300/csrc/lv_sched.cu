@@ -1,10 +1,11 @@
 // lv_schedule: the interaction-aware request scheduler of Section 4 (Algorithm 1).
 //
-// One CTA ranks a ready set of up to LV_SCHED_MAX_REQUESTS requests: every request
-// gets a 128-bit key (urgency class, the class's own order, its position in the
-// ready set), a bitonic sort orders the keys in shared memory, and a scan of the
-// token and KV costs in that order finds the longest prefix that fits the round
-// budgets ("admission stops" at the first request that does not fit).
+// A ready set of up to LV_SCHED_MAX_REQUESTS requests: every request gets a
+// 128-bit key (urgency class, the class's own order, its position in the ready
+// set); then each request counts the smaller keys (its place in the order) and
+// sums their token and KV costs, which decides whether it lies in the
+// longest prefix that fits the round budgets ("admission stops" at the first
+// request that does not fit).  Nothing is sorted; the work spreads over the GPU.
 #include <cstdint>
 
 #include "lv_internal.cuh"
@@ -15,7 +16,10 @@ namespace {
 using u128 = unsigned __int128;
 using i128 = __int128;
 
-constexpr int kSchedThreads = 1024;
+constexpr int kKeyThreads = 256;
+constexpr int kPerWarp = 2;                                   // requests a warp places
+constexpr int kPlaceThreads = 512;
+constexpr int kPlaceRequests = kPlaceThreads / 32 * kPerWarp;  // requests a CTA places
 constexpr u128 kLow114 = (((u128)1) << 114) - 1;
 
 __device__ __forceinline__ void sched_error(long long* ctl, int code) {
@@ -52,81 +56,95 @@ __device__ u128 request_key(const lv_request& r, int idx, const lv_sched_params&
   return ((u128)cls << 126) | ((v & kLow114) << 12) | (u128)(unsigned)idx;
 }
 
-__global__ void __launch_bounds__(kSchedThreads)
-k_schedule(lv_sched_params q, const lv_request* __restrict__ reqs, int n, int N,
-           int32_t* __restrict__ order, int32_t* __restrict__ batch, long long* __restrict__ err) {
+// Every request's 128-bit key and its two costs (negative costs count as 0).
+__global__ void __launch_bounds__(kKeyThreads)
+k_sched_keys(lv_sched_params q, const lv_request* __restrict__ reqs, int n, u128* __restrict__ keys,
+             longlong2* __restrict__ cost, int32_t* __restrict__ batch, long long* __restrict__ err) {
+  const int i = blockIdx.x * kKeyThreads + threadIdx.x;
+  if (i == 0) *batch = 0;
+  if (i >= n) return;
+  const lv_request& r = reqs[i];
+  keys[i] = request_key(r, i, q, err);
+  cost[i] = make_longlong2(r.tokens > 0 ? r.tokens : 0, r.kv_needed > 0 ? r.kv_needed : 0);
+}
+
+// A CTA places 32 requests: each warp holds kPerWarp of them and its lanes
+// stride over the ready set, comparing every key (staged in shared memory) with
+// the warp's requests.  Keys are distinct (each holds its request's index), so a
+// request's place in the priority order is the number of smaller keys, and the
+// tokens and KV admitted before it are the sums of their costs.  Costs are never
+// negative, so the requests that fit -- cumulative costs through their own
+// within both budgets -- are exactly the prefix that admission reaches before it
+// stops.
+__global__ void __launch_bounds__(kPlaceThreads)
+k_sched_place(lv_sched_params q, const lv_request* __restrict__ reqs, int n,
+              const u128* __restrict__ keys, const longlong2* __restrict__ cost,
+              int32_t* __restrict__ order, int32_t* __restrict__ batch) {
   extern __shared__ __align__(16) unsigned char smem[];
-  u128* keys = reinterpret_cast<u128*>(smem);
-  for (int i = threadIdx.x; i < N; i += kSchedThreads)
-    keys[i] = i < n ? request_key(reqs[i], i, q, err) : ~(u128)0;
+  u128* sk = reinterpret_cast<u128*>(smem);
+  longlong2* sc = reinterpret_cast<longlong2*>(sk + n);
+  __shared__ int s_admitted;
+  if (threadIdx.x == 0) s_admitted = 0;
+  for (int j = threadIdx.x; j < n; j += kPlaceThreads) {
+    sk[j] = keys[j];
+    sc[j] = cost[j];
+  }
   __syncthreads();
-  for (int k = 2; k <= N; k <<= 1) {
-    for (int j = k >> 1; j > 0; j >>= 1) {
-      for (int i = threadIdx.x; i < N; i += kSchedThreads) {
-        const int ixj = i ^ j;
-        if (ixj > i) {
-          const u128 a = keys[i], b = keys[ixj];
-          if (((i & k) == 0) ? (a > b) : (a < b)) {
-            keys[i] = b;
-            keys[ixj] = a;
-          }
-        }
-      }
-      __syncthreads();
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int base = blockIdx.x * kPlaceRequests + w * kPerWarp;
+  u128 mine[kPerWarp];
+  int rank[kPerWarp];
+  long long tok[kPerWarp], kv[kPerWarp];
+#pragma unroll
+  for (int r = 0; r < kPerWarp; ++r) {
+    mine[r] = base + r < n ? sk[base + r] : ~(u128)0;
+    rank[r] = 0;
+    tok[r] = kv[r] = 0;
+  }
+  for (int j = lane; j < n; j += 32) {
+    const u128 k = sk[j];
+    const longlong2 c = sc[j];
+#pragma unroll
+    for (int r = 0; r < kPerWarp; ++r) {
+      const long long m = k < mine[r] ? -1ll : 0ll;
+      rank[r] -= (int)m;
+      tok[r] += c.x & m;
+      kv[r] += c.y & m;
     }
   }
-  // cumulative token and KV costs in priority order; the admitted set is a prefix
-  const int per = (N + kSchedThreads - 1) / kSchedThreads;
-  const int r0 = min(N, (int)threadIdx.x * per), r1 = min(N, r0 + per);
-  long long tok = 0, kv = 0;
-  for (int r = r0; r < r1 && r < n; ++r) {
-    const lv_request& x = reqs[(int)(keys[r] & 0xFFF)];
-    tok += x.tokens > 0 ? x.tokens : 0;
-    kv += x.kv_needed > 0 ? x.kv_needed : 0;
+#pragma unroll
+  for (int r = 0; r < kPerWarp; ++r) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      rank[r] += __shfl_xor_sync(0xffffffffu, rank[r], o);
+      tok[r] += __shfl_xor_sync(0xffffffffu, tok[r], o);
+      kv[r] += __shfl_xor_sync(0xffffffffu, kv[r], o);
+    }
+    const int i = base + r;
+    if (lane == r && i < n) {
+      order[rank[r]] = reqs[i].id;
+      if (tok[r] + sc[i].x <= q.token_budget && kv[r] + sc[i].y <= q.kv_budget)
+        atomicAdd(&s_admitted, 1);
+    }
   }
-  __shared__ long long s_tok[kSchedThreads], s_kv[kSchedThreads];
-  __shared__ int s_cnt[kSchedThreads];
-  s_tok[threadIdx.x] = tok;
-  s_kv[threadIdx.x] = kv;
   __syncthreads();
-  // exclusive prefix over threads (a simple two-array Hillis-Steele scan)
-  for (int off = 1; off < kSchedThreads; off <<= 1) {
-    const long long at = threadIdx.x >= off ? s_tok[threadIdx.x - off] : 0;
-    const long long ak = threadIdx.x >= off ? s_kv[threadIdx.x - off] : 0;
-    __syncthreads();
-    s_tok[threadIdx.x] += at;
-    s_kv[threadIdx.x] += ak;
-    __syncthreads();
-  }
-  long long ctok = s_tok[threadIdx.x] - tok, ckv = s_kv[threadIdx.x] - kv;
-  int admitted = 0;
-  for (int r = r0; r < r1 && r < n; ++r) {
-    const int idx = (int)(keys[r] & 0xFFF);
-    const lv_request& x = reqs[idx];
-    order[r] = x.id;
-    ctok += x.tokens > 0 ? x.tokens : 0;
-    ckv += x.kv_needed > 0 ? x.kv_needed : 0;
-    admitted += (ctok <= q.token_budget && ckv <= q.kv_budget) ? 1 : 0;
-  }
-  s_cnt[threadIdx.x] = admitted;
-  __syncthreads();
-  for (int off = kSchedThreads / 2; off > 0; off >>= 1) {
-    if (threadIdx.x < off) s_cnt[threadIdx.x] += s_cnt[threadIdx.x + off];
-    __syncthreads();
-  }
-  if (threadIdx.x == 0) *batch = s_cnt[0];
+  if (threadIdx.x == 0 && s_admitted) atomicAdd(batch, s_admitted);
 }
 
 }  // namespace
 
 cudaError_t launch_schedule(const lv_sched_params& q, const lv_request* reqs, int n, int32_t* order,
-                            int32_t* batch, long long* ctl, cudaStream_t s) {
-  int N = 1;
-  while (N < n) N <<= 1;
-  const size_t smem = (size_t)N * sizeof(u128);
-  cudaError_t e = cudaFuncSetAttribute(k_schedule, cudaFuncAttributeMaxDynamicSharedMemorySize, 64 * 1024);
+                            int32_t* batch, long long* ctl, void* scratch, cudaStream_t s) {
+  u128* keys = static_cast<u128*>(scratch);
+  longlong2* cost = reinterpret_cast<longlong2*>(keys + LV_SCHED_MAX_REQUESTS);
+  // every CTA stages all keys and costs: 32 B per request, up to 128 KiB
+  cudaError_t e = cudaFuncSetAttribute(k_sched_place, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)(32 * LV_SCHED_MAX_REQUESTS));
   if (e != cudaSuccess) return e;
-  k_schedule<<<1, kSchedThreads, smem, s>>>(q, reqs, n, N, order, batch, ctl);
+  k_sched_keys<<<(n + kKeyThreads - 1) / kKeyThreads, kKeyThreads, 0, s>>>(q, reqs, n, keys, cost,
+                                                                          batch, ctl);
+  k_sched_place<<<(n + kPlaceRequests - 1) / kPlaceRequests, kPlaceThreads, (size_t)n * 32, s>>>(
+      q, reqs, n, keys, cost, order, batch);
   return cudaGetLastError();
 }
 
