@@ -69,9 +69,10 @@ enum { LV_SUFFIX_FIRST = 0, LV_ASCENDING = 1 };        /* lv_pool_desc.within_or
 enum { LV_PLAY_PLAYBACK = 0, LV_PLAY_COUNTERS = 1 };   /* lv_pool_desc.t_play_mode */
 enum { LV_MODE_AUTO = 0, LV_MODE_ZERO_COPY = 1, LV_MODE_STAGED = 2 };   /* swap modes */
 /* lv_swap_exchange with LV_MODE_STAGED | LV_MODE_ASYNC: the call returns once its
-   transfers are queued; its copy-engine transfers and unpacks run after the
-   previous asynchronous call's (each direction waits for the transfer that last
-   used the same host slots or HBM pages), overlapping the caller's next calls.
+   transfers are queued; its copy-engine transfers and unpacks overlap the
+   caller's next calls.  A later asynchronous call waits for an earlier one's
+   transfers of a direction only when it touches an HBM page or host slot that
+   they may still be using.
    Until lv_join(pool, stream) the caller must not read or write the pool's KV
    arrays or host pool; calls that move or read KV bytes (other than another
    asynchronous staged exchange) and lv_sync join first by themselves. */

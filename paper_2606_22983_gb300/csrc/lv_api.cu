@@ -20,6 +20,25 @@ struct NvtxRange {
   NvtxRange& operator=(const NvtxRange&) = delete;
 };
 
+// Pages or slots touched by transfers that may still be running: a byte per
+// index for lookups, and the list of marked indices for clearing.
+struct MarkSet {
+  std::vector<uint8_t> on;
+  std::vector<int32_t> list;
+  void resize(int64_t n) { on.assign((size_t)(n > 0 ? n : 1), 0); }
+  void add(int32_t x) {
+    if (x >= 0 && (size_t)x < on.size() && !on[x]) {
+      on[x] = 1;
+      list.push_back(x);
+    }
+  }
+  bool has(int32_t x) const { return x < 0 || (size_t)x >= on.size() || on[x] != 0; }
+  void clear() {
+    for (int32_t x : list) on[x] = 0;
+    list.clear();
+  }
+};
+
 struct lv_pool {
   lv::DevPool d{};
   int device = 0;
@@ -43,6 +62,10 @@ struct lv_pool {
   cudaEvent_t ev_st_d2h = nullptr, ev_st_h2d = nullptr, ev_st_unpack = nullptr,
               ev_st_packed = nullptr, ev_st_done = nullptr;
   bool st_pending = false;
+  // what those calls touch while they may still run: pages their unpacks write, slots
+  // their D2H copies write, slots their H2D copies read; a new call waits for an event
+  // only when it touches a marked page or slot
+  MarkSet st_loaded, st_written, st_read;
   // staged path: side streams for the copy engines, a host copy of the tasks, sync events
   cudaStream_t s_d2h = nullptr, s_h2d = nullptr;
   int4* tasks_host = nullptr;
@@ -227,6 +250,17 @@ lv_status sync_events(lv_pool* pool, size_t n) {
 // runs in each direction on the side streams; unpack into the in pages; joined back
 // into `s`.  Every pack precedes every unpack on `s`, so a page that an incoming block
 // takes is read before it is overwritten.
+// Drops the marks of `m` once `ev` (recorded after every transfer that marked it)
+// has completed; a query that finds it still running keeps them.
+cudaError_t prune_marks(cudaEvent_t ev, MarkSet& m) {
+  if (m.list.empty()) return cudaSuccess;
+  const cudaError_t e = cudaEventQuery(ev);
+  if (e == cudaErrorNotReady) return cudaSuccess;
+  if (e != cudaSuccess) return e;
+  m.clear();
+  return cudaSuccess;
+}
+
 lv_status staged_move_inner(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStream_t s,
                             void** staging_out, bool async) {
   const lv::DevPool& d = pool->d;
@@ -272,13 +306,31 @@ lv_status staged_move_inner(lv_pool* pool, const int4* tasks_dev, int64_t n, cud
   LV_TRY(cudaEventRecord(ev_start, s));
   LV_TRY(cudaStreamWaitEvent(pool->s_d2h, ev_start, 0));
   LV_TRY(cudaStreamWaitEvent(pool->s_h2d, ev_start, 0));
-  const bool after_async = async && pool->st_pending;   // the previous asynchronous call
-  if (after_async) {
-    // a block it wrote out may come back now; a slot it read may be written now;
-    // a page it loaded may be packed now
-    LV_TRY(cudaStreamWaitEvent(pool->s_h2d, pool->ev_st_d2h, 0));
-    LV_TRY(cudaStreamWaitEvent(pool->s_d2h, pool->ev_st_h2d, 0));
-    LV_TRY(cudaStreamWaitEvent(s, pool->ev_st_unpack, 0));
+  if (async && pool->st_pending) {
+    // Earlier asynchronous calls: a block one wrote out may come back now, a slot one
+    // read may be written now, a page one loaded may be packed now.  Marks of
+    // transfers that have finished are dropped; the event of a direction is waited
+    // for only when this call touches a page or slot still marked for it.  Each event
+    // was recorded after every earlier transfer of its stream, so one wait covers all.
+    LV_TRY(prune_marks(pool->ev_st_unpack, pool->st_loaded));
+    LV_TRY(prune_marks(pool->ev_st_d2h, pool->st_written));
+    LV_TRY(prune_marks(pool->ev_st_h2d, pool->st_read));
+    bool h2d_after_d2h = false, d2h_after_h2d = false, pack_after_unpack = false;
+    for (int64_t i = 0; i < n_in && !h2d_after_d2h; ++i) h2d_after_d2h = pool->st_written.has(tin[i].z);
+    for (int64_t i = 0; i < n_out && !(d2h_after_h2d && pack_after_unpack); ++i) {
+      d2h_after_h2d = d2h_after_h2d || pool->st_read.has(tout[i].y);
+      pack_after_unpack = pack_after_unpack || pool->st_loaded.has(tout[i].x);
+    }
+    if (h2d_after_d2h) LV_TRY(cudaStreamWaitEvent(pool->s_h2d, pool->ev_st_d2h, 0));
+    if (d2h_after_h2d) LV_TRY(cudaStreamWaitEvent(pool->s_d2h, pool->ev_st_h2d, 0));
+    if (pack_after_unpack) LV_TRY(cudaStreamWaitEvent(s, pool->ev_st_unpack, 0));
+  }
+  if (async) {
+    for (int64_t i = 0; i < n_in; ++i) {
+      pool->st_loaded.add(tin[i].w);
+      pool->st_read.add(tin[i].z);
+    }
+    for (int64_t i = 0; i < n_out; ++i) pool->st_written.add(tout[i].y);
   }
   // H2D first so that the inbound copies start at once: runs of consecutive slots
   for (int64_t c = 0; c * chunk < n_in; ++c) {
@@ -593,6 +645,9 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       cudaEventCreateWithFlags(&pool->ev_st_done, cudaEventDisableTiming) != cudaSuccess)
     return fail(LV_ERR_CUDA);
   pool->tasks_host_cap = (size_t)d.budget + d.maxB + (size_t)d.host_pages;
+  pool->st_loaded.resize(d.hbm_pages);
+  pool->st_written.resize(d.host_pages);
+  pool->st_read.resize(d.host_pages);
   // the task list read back, then its sorted out and in halves
   if (cudaHostAlloc((void**)&pool->tasks_host, 3 * pool->tasks_host_cap * sizeof(int4), cudaHostAllocDefault) !=
       cudaSuccess) {
