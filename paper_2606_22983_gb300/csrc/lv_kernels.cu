@@ -331,6 +331,9 @@ constexpr int kCensusThreads = 256;
 // One CTA per session: its key and its count of HBM-resident blocks.
 __global__ void __launch_bounds__(kCensusThreads)
 k_rank_census(DevPool p, long long now_us, bool fallback) {
+  // the emit kernel may be scheduled as soon as every census CTA has started; it
+  // waits for the whole census (griddepcontrol.wait) before it reads anything
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int32_t s = blockIdx.x;
   __shared__ unsigned long long key;
   if (threadIdx.x == 0) key = session_key(p, s, now_us, fallback);
@@ -363,6 +366,7 @@ constexpr int kEmitThreads = 256;
 __global__ void __launch_bounds__(kEmitThreads)
 k_rank_emit(DevPool p, long long k, const long long* k_dev, bool fallback, long long* count_dev,
             lv_victim* __restrict__ out) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");   // the census is complete and visible
   const int32_t sid = blockIdx.x;
   const unsigned long long key = p.skey[sid];
   if (key == 0ull && sid != 0) return;
@@ -1606,7 +1610,19 @@ cudaError_t launch_select(const DevPool& p, int64_t now_us, int64_t k, bool fall
                           lv_victim* out, long long* count_dev, cudaStream_t s, int /*num_sms*/,
                           const long long* k_dev) {
   k_rank_census<<<p.S, kCensusThreads, 0, s>>>(p, now_us, fallback);
-  k_rank_emit<<<p.S, kEmitThreads, 0, s>>>(p, k, k_dev, fallback, count_dev, out);
+  // programmatic dependent launch: the emit grid's launch overlaps the census
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((unsigned)p.S);
+  cfg.blockDim = dim3(kEmitThreads);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, k_rank_emit, p, (long long)k, k_dev, fallback,
+                                           count_dev, out);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
