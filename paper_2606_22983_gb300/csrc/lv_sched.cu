@@ -60,6 +60,9 @@ __device__ u128 request_key(const lv_request& r, int idx, const lv_sched_params&
 __global__ void __launch_bounds__(kKeyThreads)
 k_sched_keys(lv_sched_params q, const lv_request* __restrict__ reqs, int n, u128* __restrict__ keys,
              longlong2* __restrict__ cost, int32_t* __restrict__ batch, long long* __restrict__ err) {
+  // the placement grid may be scheduled once every key CTA has started; it waits
+  // for all keys (griddepcontrol.wait) before it reads them
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int i = blockIdx.x * kKeyThreads + threadIdx.x;
   if (i == 0) *batch = 0;
   if (i >= n) return;
@@ -80,6 +83,7 @@ __global__ void __launch_bounds__(kPlaceThreads)
 k_sched_place(lv_sched_params q, const lv_request* __restrict__ reqs, int n,
               const u128* __restrict__ keys, const longlong2* __restrict__ cost,
               int32_t* __restrict__ order, int32_t* __restrict__ batch) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");   // every key, cost and the zeroed batch
   extern __shared__ __align__(16) unsigned char smem[];
   u128* sk = reinterpret_cast<u128*>(smem);
   longlong2* sc = reinterpret_cast<longlong2*>(sk + n);
@@ -143,8 +147,20 @@ cudaError_t launch_schedule(const lv_sched_params& q, const lv_request* reqs, in
   if (e != cudaSuccess) return e;
   k_sched_keys<<<(n + kKeyThreads - 1) / kKeyThreads, kKeyThreads, 0, s>>>(q, reqs, n, keys, cost,
                                                                           batch, ctl);
-  k_sched_place<<<(n + kPlaceRequests - 1) / kPlaceRequests, kPlaceThreads, (size_t)n * 32, s>>>(
-      q, reqs, n, keys, cost, order, batch);
+  // programmatic dependent launch: the placement grid's launch overlaps the keys
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((unsigned)((n + kPlaceRequests - 1) / kPlaceRequests));
+  cfg.blockDim = dim3(kPlaceThreads);
+  cfg.dynamicSmemBytes = (size_t)n * 32;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, k_sched_place, q, reqs, n, (const u128*)keys, (const longlong2*)cost,
+                         order, batch);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
