@@ -266,26 +266,42 @@ __device__ __forceinline__ void apply_event(const DevPool& p, lv_session_state& 
 }
 
 // One thread per session applies, in order, the events addressed to it.
-__global__ void k_events(DevPool p, const lv_event* __restrict__ ev, long long n) {
-  const int s = blockIdx.x * blockDim.x + threadIdx.x;
-  if (s == 0) {
-    for (long long e = 0; e < n; ++e) {
-      if (ev[e].kind < LV_EV_TURN_BEGIN || ev[e].kind > LV_EV_UNPROTECT || ev[e].sid < 0 ||
-          ev[e].sid >= p.S) {
-        set_error(p.ctl, LV_ERR_BOUNDS, e);
+constexpr int kEventThreads = 128;
+constexpr int kEventChunk = 512;   // events staged in shared memory at a time (16 KiB)
+
+// One thread per session.  The CTA stages the event list in shared memory, a
+// chunk at a time (coalesced loads, each event read once per CTA), and every
+// thread applies, in list order, the events of its own session.  CTA 0 checks
+// every event's kind and session and counts them.
+__global__ void __launch_bounds__(kEventThreads)
+k_events(DevPool p, const lv_event* __restrict__ ev, long long n) {
+  __shared__ lv_event chunk[kEventChunk];
+  const int s = blockIdx.x * kEventThreads + threadIdx.x;
+  lv_session_state st;
+  if (s < p.S) st = p.sess[s];
+  bool touched = false;
+  for (long long c0 = 0; c0 < n; c0 += kEventChunk) {
+    const int m = (int)(n - c0 < kEventChunk ? n - c0 : kEventChunk);
+    __syncthreads();   // the previous chunk is no longer read
+    for (int e = threadIdx.x; e < m; e += kEventThreads) {
+      const lv_event x = ev[c0 + e];
+      chunk[e] = x;
+      if (blockIdx.x == 0 && (x.kind < LV_EV_TURN_BEGIN || x.kind > LV_EV_UNPROTECT || x.sid < 0 ||
+                              x.sid >= p.S))
+        set_error(p.ctl, LV_ERR_BOUNDS, c0 + e);
+    }
+    __syncthreads();
+    if (s < p.S) {
+      for (int e = 0; e < m; ++e) {
+        if (chunk[e].sid != s) continue;
+        touched = true;
+        apply_event(p, st, chunk[e]);
       }
     }
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0)
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_EVENTS]), (unsigned long long)n);
-  }
-  if (s >= p.S) return;
-  lv_session_state st = p.sess[s];
-  bool touched = false;
-  for (long long e = 0; e < n; ++e) {
-    if (ev[e].sid != s) continue;
-    touched = true;
-    apply_event(p, st, ev[e]);
-  }
-  if (touched) p.sess[s] = st;
+  if (s < p.S && touched) p.sess[s] = st;
 }
 
 // --------------------------------------------------------------- ranking
@@ -1602,7 +1618,7 @@ cudaError_t launch_session_set(const DevPool& p, const lv_session_state* in, int
 }
 
 cudaError_t launch_events(const DevPool& p, const lv_event* ev, int64_t n, cudaStream_t s) {
-  k_events<<<blocks_for(p.S, 128, 1 << 20), 128, 0, s>>>(p, ev, n);
+  k_events<<<blocks_for(p.S, kEventThreads, 1 << 20), kEventThreads, 0, s>>>(p, ev, n);
   return cudaGetLastError();
 }
 
