@@ -65,7 +65,7 @@ struct DevPool {
   uint32_t* bits_host;
   long long* ctl;         // [C_N]
   // ranking scratch
-  unsigned long long* skey;  // [S] session sort key (0 = not a candidate)
+  unsigned long long* skey;  // [S] session order key (0 = not a candidate)
   int32_t* scount;           // [S] resident blocks of the session
   // exchange scratch
   unsigned long long* page_tag;  // [hbm_pages] epoch << 32 | victim index (| paired bit)

@@ -305,7 +305,7 @@ k_events(DevPool p, const lv_event* __restrict__ ev, long long n) {
 }
 
 // --------------------------------------------------------------- ranking
-// Sort key of a session, 0 when it is not a candidate.  Larger keys are
+// Order key of a session, 0 when it is not a candidate.  Larger keys are
 // evicted first: bit 63 = normal tier, bits 31..62 = T_next (Eq. 4), bits
 // 0..30 = 2^31-1-sid so that equal T_next rank by ascending session id.
 __device__ __forceinline__ unsigned long long session_key(const DevPool& p, int32_t s,
