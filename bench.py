@@ -111,44 +111,6 @@ class ClockSampler:
 
 
 # --------------------------------------------------------------- our arm
-def link_peaks(torch, pool, nbytes, reps=5):
-    """Contiguous page-locked cudaMemcpyAsync of nbytes each way, and both at once."""
-    src = pool.kv.view(-1)[:nbytes]
-    host = torch.from_numpy(pool.host.reshape(-1)[:nbytes])
-    dev2 = torch.empty(nbytes, dtype=torch.uint8, device=pool.device)
-    host2 = torch.from_numpy(pool.host.reshape(-1)[nbytes:2 * nbytes]) \
-        if pool.host.size >= 2 * nbytes else None
-    res = {}
-    for name, fn in (("d2h", lambda: host.copy_(src, non_blocking=True)),
-                     ("h2d", lambda: dev2.copy_(host, non_blocking=True))):
-        best = 1e30
-        for _ in range(reps):
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            a.record()
-            fn()
-            b.record()
-            b.synchronize()
-            best = min(best, a.elapsed_time(b))
-        res[name] = nbytes / (best / 1e3) / 1e9
-    if host2 is not None:
-        s2 = torch.cuda.Stream()
-        best = 1e30
-        for _ in range(reps):
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            a.record()
-            s2.wait_event(a)
-            host.copy_(src, non_blocking=True)
-            with torch.cuda.stream(s2):
-                dev2.copy_(host2, non_blocking=True)
-            torch.cuda.current_stream().wait_stream(s2)
-            b.record()
-            b.synchronize()
-            best = min(best, a.elapsed_time(b))
-        res["bidir"] = 2 * nbytes / (best / 1e3) / 1e9
-    del dev2
-    return res
-
-
 def run_turns(gm, wl, lo, hi, dev_events=None):
     """Turns lo..hi of a turn-driven script (playback batch, then the turn)."""
     from paper_2606_22983_gb300 import lv
@@ -179,7 +141,7 @@ def _moved_pages(pool):
 def ours(args, torch):
     from paper_2606_22983_gb300 import build, lv
     build()
-    from paper_2606_22983_gb300.harness import fill_random, pool_for
+    from paper_2606_22983_gb300.harness import fill_random, link_peaks, pool_for
     from paper_2606_22983_gb300.manager import KVManager
     from workloads import make_workload
 
@@ -292,7 +254,7 @@ def ours(args, torch):
     line = None
     if rank == 0:
         mean_turn = moved / K / 2
-        peaks = link_peaks(torch, pool, int(min(mean_turn, 1 << 30)) // 4096 * 4096)
+        peaks = link_peaks(pool, int(min(mean_turn, 1 << 30)) // 4096 * 4096)
         # roofline of the dominant kernel (longest total time) among the link-bound copies;
         # the staged path's pack/unpack are HBM-bound and reported against the HBM peak
         link_kern = {n: d for n, d in kern.items() if n in ("swap_out", "swap_in", "exchange")}

@@ -398,6 +398,23 @@ lv_status lv_remap(lv_pool* pool, const lv_remap_entry* entries, int64_t n, lv_s
    reserved. */
 lv_status lv_cancel(lv_pool* pool, const int32_t* locs, int64_t n, lv_stream stream);
 
+/* Section 5.1 under memory pressure from outside the manager, with no host
+   round trip: frees up to k HBM pages now.  On the device, in stream order:
+   rank with lv_select_victims' order (normal eligibility, no fallback tier),
+   take the first k -- every candidate when there are fewer -- and evict them
+   exactly as lv_swap_exchange does with no incoming blocks.  The results
+   equal those of lv_select_victims followed by lv_swap_exchange.
+   flags: 0 or LV_RESIDENT_ASYNC_COPY.  Optional outputs (host or device, NULL
+   to skip): victims_out (lv_victim [hbm_budget_pages]: the victims chosen),
+   slots_out (int32 [hbm_budget_pages]: their host slots), result_out (k, and
+   n_found = n_victims = victims evicted; n_loaded = 0; status
+   LV_RESIDENT_DONE, or LV_RESIDENT_NOTHING when nothing was a candidate;
+   sid = -1).  k above hbm_budget_pages is taken as hbm_budget_pages.
+   Device-detected: LV_ERR_NO_HOST when the host tier cannot take the victims
+   (then nothing moves). */
+lv_status lv_evict(lv_pool* pool, int64_t now_us, int64_t k, uint32_t flags, lv_victim* victims_out,
+                   int32_t* slots_out, lv_resident_result* result_out, lv_stream stream);
+
 /* One turn of a voice session as one call (Section 3: the user's input is
    complete and the request runs; Sections 5.1 and 5.2: its KV is made
    resident first), with no host round trip.  In stream order on the device:

@@ -2,9 +2,12 @@
 
     python -m paper_2606_22983_gb300 --workload mixed --seed 0 --driver device
 
-Prints one JSON line: the workload's size, the bytes moved each way, the device time
-of the turns (CUDA events around each turn's calls, with a host wait per turn so that
-each turn's time is its own), the wall time, and the manager's and pool's counters.
+Prints one JSON line: the workload's size, the bytes moved each way, the device time of
+every event that moved bytes (CUDA events around each event's calls, with a host wait per
+event so that each event's time is its own), the turns' latencies, the wall time, the
+manager's and pool's counters, and the host link's peaks measured afterwards in the same
+process.  ``link_frac`` compares the moving events' time with the link's best time for
+each event's own mix of bytes out and in: max(out / d2h, in / h2d, (out + in) / bidir).
 Workloads: tiny, thinker, mixed, long, frag (see workloads.configs)."""
 from __future__ import annotations
 
@@ -34,7 +37,7 @@ def main(argv=None) -> int:
     import torch
     from . import build
     build()
-    from .harness import fill_random, pool_for
+    from .harness import fill_random, link_peaks, pool_for
     from .manager import KVManager
 
     spec = pool_spec(args.workload).with_(tiers=args.tiers, policy=args.policy)
@@ -52,32 +55,55 @@ def main(argv=None) -> int:
                            mode=args.mode, order_fn=scatter_order)
         n = wl.n_events if args.events <= 0 else min(args.events, wl.n_events)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        turn_ms, load_ms = [], []
+        page = pool.J * pool.P
+        turn_ms, load_ms, moves = [], [], []      # moves: (ms, bytes out, bytes in)
+        st0 = pool.stats()
         w0 = time.perf_counter()
         for i in range(n):
             e = wl.event(i)
-            if int(e[1]) not in (1, 2, 7):
-                gm.step(e, i)
-                continue
             torch.cuda.synchronize()
             a.record()
             rec = gm.step(e, i)
             b.record()
             torch.cuda.synchronize()
             ms = a.elapsed_time(b)
-            turn_ms.append(ms)
-            if len(rec.get("in_blocks", ())):
-                load_ms.append(ms)
+            st1 = pool.stats()
+            out, inn = st1["bytes_out"] - st0["bytes_out"], st1["bytes_in"] - st0["bytes_in"]
+            st0 = st1
+            if out or inn:
+                moves.append((ms, out, inn))
+            if int(e[1]) in (1, 2, 7):
+                turn_ms.append(ms)
+                if len(rec.get("in_blocks", ())):
+                    load_ms.append(ms)
         assert pool.sync(raise_on_error=False) == 0
         wall = time.perf_counter() - w0
         st = pool.stats()
+        mv = np.array(moves, dtype=np.float64).reshape(-1, 3)
+        mean_move = float(mv[:, 1:].sum(axis=1).mean()) if len(mv) else 0.0
+        nbytes = int(min(max(mean_move / 2, 1 << 26), 1 << 30, pool.kv.numel(),
+                         pool.host.size // 2 if pool.host is not None else 0))
+        nbytes = nbytes // 4096 * 4096
+        peaks = link_peaks(pool, nbytes) if nbytes > 0 else {}
+        link = None
+        if len(mv) and "bidir" in peaks:
+            best_s = np.maximum(np.maximum(mv[:, 1] / (peaks["d2h"] * 1e9), mv[:, 2] / (peaks["h2d"] * 1e9)),
+                                (mv[:, 1] + mv[:, 2]) / (peaks["bidir"] * 1e9))
+            t_s = mv[:, 0].sum() / 1e3
+            link = {"moving_events": int(len(mv)), "device_s": round(float(t_s), 4),
+                    "gbs": round(float(mv[:, 1:].sum() / t_s / 1e9), 1),
+                    "link_best_s": round(float(best_s.sum()), 4),
+                    "link_frac": round(float(best_s.sum() / t_s), 3),
+                    "peaks_gbs": {k: round(v, 1) for k, v in peaks.items()},
+                    "peak_copy_bytes": nbytes}
         q = lambda xs, f: round(float(np.percentile(xs, f)), 3) if xs else None
         print(json.dumps({
             "workload": args.workload, "seed": args.seed, "events": n, "driver": args.driver,
             "mode": args.mode, "tiers": args.tiers, "policy": args.policy,
             "controller_link_bytes_per_us": args.controller or None,
             "sessions": spec.n_sessions, "hbm_budget_pages": spec.hbm_budget_pages,
-            "host_pages": wl.spec.host_pages, "page_bytes": pool.J * pool.P,
+            "host_pages": wl.spec.host_pages, "page_bytes": page,
+            "moves": link,
             "turns": len(turn_ms), "turns_loading_on_path": len(load_ms),
             "turn_ms": {"mean": round(float(np.mean(turn_ms)), 3) if turn_ms else None,
                         "p50": q(turn_ms, 50), "p90": q(turn_ms, 90), "max": q(turn_ms, 100)},

@@ -1013,6 +1013,34 @@ lv_status lv_make_resident(lv_pool* pool, int32_t sid, int64_t now_us, int32_t a
   }
 }
 
+lv_status lv_evict(lv_pool* pool, int64_t now_us, int64_t k, uint32_t flags, lv_victim* victims_out,
+                   int32_t* slots_out, lv_resident_result* result_out, lv_stream stream) {
+  NvtxRange nvtx_range("lv_evict");
+  if (!pool || k < 0 || (flags & ~(uint32_t)LV_RESIDENT_ASYNC_COPY)) return LV_ERR_INVALID;
+  if (pool->d.host_pages == 0) return LV_ERR_INVALID;
+  const bool async = (flags & LV_RESIDENT_ASYNC_COPY) != 0;
+  DeviceGuard g(pool->device);
+  cudaStream_t s = as_stream(stream);
+  try {
+    Staging st(pool, s);
+    void* rdev = nullptr;
+    lv_status r;
+    if ((r = st.out(result_out, sizeof(lv_resident_result), &rdev, false)) != LV_OK) return r;
+    if (++pool->epoch <= 0) pool->epoch = 1;
+    const lv::ResidentScratch* rs = nullptr;
+    lv::CopyOffload off{};
+    LV_TRY(next_scratch(pool, s, async, &rs, &off));
+    const int64_t kk = k < (int64_t)pool->d.budget ? k : (int64_t)pool->d.budget;
+    LV_TRY(lv::launch_evict(pool->d, *rs, now_us, kk, pool->epoch, s, pool->exchange_ctas,
+                            static_cast<lv_resident_result*>(rdev),
+                            timing_pair(pool, LV_TIMING_EXCHANGE), async ? &off : nullptr));
+    LV_TRY(copy_resident_outputs(pool, 0, victims_out, slots_out, nullptr, nullptr, nullptr, s));
+    return st.finish();
+  } catch (const std::bad_alloc&) {
+    return LV_ERR_OOM;
+  }
+}
+
 lv_status lv_join(lv_pool* pool, lv_stream stream) {
   NvtxRange nvtx_range("lv_join");
   if (!pool) return LV_ERR_INVALID;

@@ -142,6 +142,10 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
                                  lv_resident_result* result, const EventPair* ev = nullptr,
                                  const long long* sid_dev = nullptr, const CopyOffload* off = nullptr);
 // lv_turn: pick (sid < 0), LV_EV_TURN_BEGIN, make resident, LV_EV_TURN_END
+// lv_evict: rank, evict up to k victims (no loads), finish
+cudaError_t launch_evict(const DevPool& p, const ResidentScratch& rs, int64_t now_us, int64_t k,
+                         int32_t epoch, cudaStream_t s, int copy_ctas, lv_resident_result* result,
+                         const EventPair* ev, const CopyOffload* off);
 cudaError_t launch_turn(const DevPool& p, const ResidentScratch& rs, int32_t sid, const int32_t* cand,
                         int32_t n_cand, int64_t now_us, int32_t append_tokens, int64_t audio_us,
                         int64_t units, int32_t epoch, cudaStream_t s, int copy_ctas,

@@ -1430,6 +1430,30 @@ __global__ void k_resident_finish(DevPool p, int32_t sid, long long now_us, bool
   }
 }
 
+// ----------------------------------------------------------------- evict
+// lv_evict: up to k victims by the normal order (no fallback tier), fewer when
+// there are fewer candidates; nothing is loaded.
+__global__ void k_evict_prepare(long long k, long long* __restrict__ R) {
+  if (threadIdx.x != 0) return;
+  R[R_K_SELECT] = k;
+  R[R_N_OUT] = 0;
+  R[R_N_IN] = 0;
+  R[R_STATUS] = LV_RESIDENT_DONE;
+  R[R_K] = k;
+  R[R_GATE] = 1;
+  R[R_APPENDED] = 0;
+  R[R_FOUND] = 0;
+  R[R_SID] = -1;
+}
+
+__global__ void k_evict_gate(DevPool p, long long* __restrict__ R) {
+  if (threadIdx.x != 0) return;
+  const long long found = p.ctl[C_SEL_COUNT];   // min(k, candidates)
+  R[R_FOUND] = found;
+  R[R_N_OUT] = found;
+  if (found == 0) R[R_STATUS] = LV_RESIDENT_NOTHING;
+}
+
 // ------------------------------------------------------------------ turn
 // lv_turn's pick: CTA c reports whether candidate c has a block in the host tier.
 __global__ void __launch_bounds__(kCensusThreads)
@@ -1725,6 +1749,23 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
     if (e != cudaSuccess) return e;
   }
   k_resident_finish<<<1, 32, 0, s>>>(p, sid, now_us, preload, R, result, sid_dev);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_evict(const DevPool& p, const ResidentScratch& rs, int64_t now_us, int64_t k,
+                         int32_t epoch, cudaStream_t s, int copy_ctas, lv_resident_result* result,
+                         const EventPair* ev, const CopyOffload* off) {
+  long long* R = rs.words;
+  k_evict_prepare<<<1, 32, 0, s>>>(k, R);
+  cudaError_t e = launch_select(p, now_us, 0, false, rs.victims, nullptr, s, 0, R + R_K_SELECT);
+  if (e != cudaSuccess) return e;
+  k_evict_gate<<<1, 32, 0, s>>>(p, R);
+  const long long max_units = (long long)p.budget * p.J;
+  e = launch_exchange(p, rs.victims, 0, -1, rs.blocks, 0, rs.slots, rs.pages, rs.tasks,
+                      R + R_N_TASKS, epoch, p.page_tag, s, copy_ctas, R + R_N_OUT, max_units, ev,
+                      nullptr, off);
+  if (e != cudaSuccess) return e;
+  k_resident_finish<<<1, 32, 0, s>>>(p, -1, now_us, false, R, result, nullptr);
   return cudaGetLastError();
 }
 

@@ -124,3 +124,43 @@ def fill_random(pool: KVPool, seed: int = 0):
                             dtype=torch.float32).to(torch.bfloat16)
             pool.host_dev[lo:lo + n].copy_(v.view(torch.uint8).view(n, pool.J, pool.P))
     torch.cuda.synchronize(pool.device)
+
+
+def link_peaks(pool: KVPool, nbytes: int, reps: int = 5) -> dict:
+    """The host link's measured peaks in GB/s: a contiguous page-locked cudaMemcpyAsync of
+    nbytes device-to-host, host-to-device, and both at once ('bidir', counting both).
+    It overwrites the first 2 * nbytes of the host pool: measure after the workload."""
+    src = pool.kv.view(-1)[:nbytes]
+    host = torch.from_numpy(pool.host.reshape(-1)[:nbytes])
+    dev2 = torch.empty(nbytes, dtype=torch.uint8, device=pool.device)
+    host2 = torch.from_numpy(pool.host.reshape(-1)[nbytes:2 * nbytes]) \
+        if pool.host.size >= 2 * nbytes else None
+    res = {}
+    for name, fn in (("d2h", lambda: host.copy_(src, non_blocking=True)),
+                     ("h2d", lambda: dev2.copy_(host, non_blocking=True))):
+        best = 1e30
+        for _ in range(reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            b.synchronize()
+            best = min(best, a.elapsed_time(b))
+        res[name] = nbytes / (best / 1e3) / 1e9
+    if host2 is not None:
+        s2 = torch.cuda.Stream()
+        best = 1e30
+        for _ in range(reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            s2.wait_event(a)
+            host.copy_(src, non_blocking=True)
+            with torch.cuda.stream(s2):
+                dev2.copy_(host2, non_blocking=True)
+            torch.cuda.current_stream().wait_stream(s2)
+            b.record()
+            b.synchronize()
+            best = min(best, a.elapsed_time(b))
+        res["bidir"] = 2 * nbytes / (best / 1e3) / 1e9
+    del dev2
+    return res

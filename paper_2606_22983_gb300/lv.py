@@ -160,6 +160,7 @@ def _load():
         "lv_make_resident": [vp, i32, i64, i32, u32, i64, vp, vp, vp, vp, vp, vp, vp],
         "lv_turn": [vp, ctypes.POINTER(lv_turn_desc), vp, vp, vp, vp, vp, vp, vp],
         "lv_join": [vp, vp],
+        "lv_evict": [vp, i64, i64, u32, vp, vp, vp, vp],
         "lv_page_checksums": [vp, vp, i64, vp, vp],
         "lv_probe_scattered": [ctypes.POINTER(lv_probe_mix), vp, i64, i64, vp, vp],
         "lv_controller_create": [vp, ctypes.POINTER(lv_controller_desc), ctypes.POINTER(vp)],
@@ -213,7 +214,7 @@ EXPORTED = ("lv_pool_create", "lv_pool_destroy", "lv_pool_host_ptr", "lv_pool_im
             "lv_get_stats", "lv_clear_error", "lv_status_str", "lv_version",
             "lv_select_victims_noalloc", "lv_timing_enable", "lv_timing_read", "lv_pack_pages",
             "lv_unpack_pages", "lv_pool_host_device_ptr", "lv_schedule", "lv_inject_fault",
-            "lv_selftest_wait", "lv_turn", "lv_join", "lv_page_checksums", "lv_probe_scattered",
+            "lv_selftest_wait", "lv_turn", "lv_evict", "lv_join", "lv_page_checksums", "lv_probe_scattered",
             "lv_controller_create", "lv_controller_destroy", "lv_controller_tick",
             "lv_controller_speech", "lv_controller_turn_begin", "lv_controller_turn_loaded",
             "lv_controller_records", "lv_controller_counters_get")
@@ -338,6 +339,12 @@ def lv_turn(pool, sid, now_us, append_tokens, reply_audio_us, reply_units, outs=
                      append_tokens=append_tokens, flags=flags)
     _check(_lib.lv_turn(pool, ctypes.byref(d), *(ptr(o) for o in outs), ptr(result_out),
                         stream_handle(stream)), "lv_turn")
+
+
+def lv_evict(pool, now_us, k, flags=0, victims_out=None, slots_out=None, result_out=None,
+             stream=None):
+    _check(_lib.lv_evict(pool, now_us, k, flags, ptr(victims_out), ptr(slots_out), ptr(result_out),
+                         stream_handle(stream)), "lv_evict")
 
 
 def lv_page_checksums(pool, pages, n, sums_out, stream=None):

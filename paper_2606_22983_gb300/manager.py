@@ -335,6 +335,9 @@ class KVManager:
     def evict(self, now_us, k, rec):
         """Free k pages now: the first k of the victim order (fewer if there are fewer)."""
         pool = self.pool
+        if self.driver == "device":
+            self._device_evict(now_us, k, rec)
+            return
         victims, n = pool.select(now_us, k, 0)
         rec["k"] = int(k)
         if self.record:
@@ -348,6 +351,27 @@ class KVManager:
             slots, _ = pool.exchange(victims, n, 0, None, 0, self._xmode())
         if self.record:
             rec["slots"] = slots.cpu().numpy().astype(np.int64)
+        self.counters["victims"] += n
+        self.counters["pages_out"] += n
+        self.bytes_moved += n * pool.J * pool.P
+
+    def _device_evict(self, now_us, k, rec):
+        """lv_evict: ranking and eviction on the device, no host round trip unless the
+        decisions are recorded."""
+        pool = self.pool
+        outs = (pool.victims, pool.slots) if self.record else (None, None)
+        lv.lv_evict(pool.handle, now_us, int(k), lv.LV_RESIDENT_ASYNC_COPY if self.async_copy else 0,
+                    *outs, self.res_h, pool.stream)
+        pool.launches += 7
+        rec["k"] = int(k)
+        if not self.record:
+            return
+        pool.sync()
+        r = self.res_h.numpy().view(lv.RESIDENT_DTYPE)[0]
+        n = int(r["n_victims"])
+        rec["victims"] = pool.victims[:int(r["n_found"])].cpu().numpy().astype(np.int64)
+        if n:
+            rec["slots"] = pool.slots[:n].cpu().numpy().astype(np.int64)
         self.counters["victims"] += n
         self.counters["pages_out"] += n
         self.bytes_moved += n * pool.J * pool.P

@@ -1,7 +1,7 @@
 """Randomized differential test of the C ABI against the oracle: random sequences of
-ranking, swap-out, swap-in, commit, cancel, exchange, growth, monitor events and whole
+ranking, swap-out, swap-in, commit, cancel, exchange, growth, monitor events, whole
 device-driven turns (lv_turn, most with their copies left running on the pool's copy
-stream) on a tiny pool with random bytes, plus single-item calls that must be refused
+stream) and device-driven evictions (lv_evict) on a tiny pool with random bytes, plus single-item calls that must be refused
 with the right status and change nothing.  After a random half of the calls (so that a
 turn's copies are often still in flight when the next call starts, and that call must
 join them), and after the last one, the block and owner tables, allocation counts,
@@ -82,12 +82,13 @@ def test_random_call_sequences_match_the_oracle(seed, tiers):
     from oracle.pool import OracleError, _enc_host
     rng, pool, om, sts, lv, se = _setup(seed, tiers)
     now = 1_000_000
-    done = dict.fromkeys(("select", "out", "in", "exchange", "append", "events", "turn", "bad"), 0)
+    done = dict.fromkeys(("select", "out", "in", "exchange", "append", "events", "turn", "evict",
+                          "bad"), 0)
     try:
         for step in range(300):
             now += int(rng.integers(0, 400_000))
-            op = rng.choice(["select", "out", "in", "exchange", "append", "events", "turn", "bad"],
-                            p=[0.08, 0.17, 0.17, 0.13, 0.1, 0.15, 0.15, 0.05])
+            op = rng.choice(["select", "out", "in", "exchange", "append", "events", "turn", "evict",
+                             "bad"], p=[0.07, 0.15, 0.15, 0.12, 0.09, 0.14, 0.14, 0.09, 0.05])
             where = (seed, tiers, step, op)
             if op in ("select", "out", "exchange"):
                 k = int(rng.integers(0, 12))
@@ -215,6 +216,29 @@ def test_random_call_sequences_match_the_oracle(seed, tiers):
                 flags = lv.LV_RESIDENT_ASYNC_COPY if rng.random() < 0.7 else 0
                 lv.lv_turn(pool.handle, sid, now, n_app, audio, units, stream=pool.stream,
                            flags=flags)
+            elif op == "evict":
+                # lv_evict (Section 5.1 under outside pressure): the first k of the normal
+                # order, fewer when there are fewer, evicted with no load
+                k = int(rng.integers(0, 16))
+                vs, vb, vp = select_victims(om.tables, om.nblocks, sts, now, k, 0, 3_000_000,
+                                            80_000, 0, False)
+                need = int(sum(om.shadow[s_, b_] < 0 for s_, b_ in zip(vs, vb)))
+                if need > HOST - int(om.host_used.sum()):
+                    continue
+                if vs.size:
+                    slots = om.swap_out(vs, vb, vp)
+                    om.remap(vs, vb, _enc_host(slots))
+                res = np.zeros(1, dtype=lv.RESIDENT_DTYPE)
+                flags = lv.LV_RESIDENT_ASYNC_COPY if rng.random() < 0.5 else 0
+                lv.lv_evict(pool.handle, now, k, flags, pool.victims, pool.slots, res, pool.stream)
+                pool.sync()
+                assert int(res["n_victims"][0]) == vs.size and int(res["k"][0]) == k, where
+                assert int(res["status"][0]) == (lv.LV_RESIDENT_DONE if vs.size else
+                                                 lv.LV_RESIDENT_NOTHING), where
+                got = pool.victims[:vs.size].cpu().numpy()
+                assert np.array_equal(got, np.stack([vs, vb, vp], 1).astype(np.int32)), where
+                if vs.size:
+                    assert np.array_equal(pool.slots[:vs.size].cpu().numpy(), slots.astype(np.int32)), where
             else:   # a single-item call that must be refused and change nothing
                 which = int(rng.integers(0, 3))
                 if which == 0:      # commit to a page nobody reserved

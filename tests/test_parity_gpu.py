@@ -141,9 +141,11 @@ def test_long_multimodal_full_size():
     assert om.counters["pages_in"] > 16 * 1000
 
 
-def test_fragmentation_full_size():
+@pytest.mark.parametrize("driver", ["exchange", "device"])
+def test_fragmentation_full_size(driver):
     """Pages randomly permuted over a 100 GB HBM budget, 640 sessions of
     256-4096 tokens; 10 000 events alternating "free k pages" with turns whose
-    reload list comes in a scattered order."""
-    om, gm = _sampled_full_size(make_workload("frag", 0), "exchange", 0, rank_on="none")
+    reload list comes in a scattered order (with the device driver, the evictions
+    run through lv_evict)."""
+    om, gm = _sampled_full_size(make_workload("frag", 0), driver, 0, rank_on="none")
     assert om.counters["turns"] == 5000
