@@ -425,9 +425,14 @@ lv_status lv_evict(lv_pool* pool, int64_t now_us, int64_t k, uint32_t flags, lv_
    lv_make_resident(sid, now_us, append_tokens, foreground); then, unless that
    failed, LV_EV_TURN_END at now_us with a = reply_audio_us, b = reply_units.
    The outputs are those of lv_make_resident (each may be NULL), with
-   result.sid the session.  Host-detected: LV_ERR_INVALID.
-   Device-detected: as lv_make_resident, LV_ERR_BOUNDS for a candidate out of
-   range. */
+   result.sid the session.  load_keys (optional, uint64 [max_blocks], device
+   or host memory, indexed by block id) sets the order in which the session's
+   host-tier blocks are loaded -- ascending (key, block id) instead of
+   ascending block id -- and so which of the lowest free HBM pages each block
+   takes; blocks_out then lists them in that order.  Ordering costs one warp
+   per host block, each comparing it with every other.  Host-detected:
+   LV_ERR_INVALID.  Device-detected: as lv_make_resident, LV_ERR_BOUNDS for a
+   candidate out of range. */
 typedef struct lv_turn_desc {
   int32_t sid;                 /* the session, or -1: pick from candidates */
   int32_t num_candidates;      /* 1..max_sessions when sid == -1 */
@@ -437,6 +442,7 @@ typedef struct lv_turn_desc {
   int64_t reply_units;         /* LV_EV_TURN_END b: reply length in progress units */
   int32_t append_tokens;       /* context growth (>= 0) */
   uint32_t flags;              /* 0 or LV_RESIDENT_ASYNC_COPY */
+  const uint64_t* load_keys;   /* NULL, or the load order's key of every block */
 } lv_turn_desc;
 lv_status lv_turn(lv_pool* pool, const lv_turn_desc* d, lv_victim* victims_out, int32_t* slots_out,
                   int32_t* blocks_out, int32_t* pages_out, int32_t* append_out,

@@ -582,6 +582,7 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
   if ((st = dev_alloc(pool, &rs.victims, (size_t)d.budget)) != LV_OK ||
       (st = dev_alloc(pool, &rs.slots, (size_t)d.budget)) != LV_OK ||
       (st = dev_alloc(pool, &rs.blocks, (size_t)d.maxB)) != LV_OK ||
+      (st = dev_alloc(pool, &rs.loads, (size_t)d.maxB)) != LV_OK ||
       (st = dev_alloc(pool, &rs.pages, (size_t)d.maxB)) != LV_OK ||
       (st = dev_alloc(pool, &rs.append, (size_t)d.maxB + 2)) != LV_OK ||
       (st = dev_alloc(pool, &rs.tasks, (size_t)d.budget + d.maxB)) != LV_OK ||
@@ -959,13 +960,13 @@ lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_ou
 // live on the device).
 cudaError_t copy_resident_outputs(lv_pool* pool, int32_t append_tokens, lv_victim* victims_out,
                                   int32_t* slots_out, int32_t* blocks_out, int32_t* pages_out,
-                                  int32_t* append_out, cudaStream_t s) {
+                                  int32_t* append_out, cudaStream_t s, bool ordered = false) {
   const lv::DevPool& d = pool->d;
   const lv::ResidentScratch& rs = pool->rs;
   const struct { void* user; const void* dev; size_t bytes; } outs[] = {
       {victims_out, rs.victims, (size_t)d.budget * sizeof(lv_victim)},
       {slots_out, rs.slots, (size_t)d.budget * 4},
-      {blocks_out, rs.blocks, (size_t)d.maxB * 4},
+      {blocks_out, ordered ? rs.loads : rs.blocks, (size_t)d.maxB * 4},
       {pages_out, rs.pages, (size_t)d.maxB * 4},
       {append_out, rs.append,
        (size_t)(append_tokens / d.T + 2 < d.maxB + 2 ? append_tokens / d.T + 2 : d.maxB + 2) * 4}};
@@ -1065,10 +1066,14 @@ lv_status lv_turn(lv_pool* pool, const lv_turn_desc* d, lv_victim* victims_out, 
   try {
     Staging st(pool, s);
     const void* cdev = nullptr;
+    const void* kdev = nullptr;
     void* rdev = nullptr;
     lv_status r;
     if (d->sid == -1 &&
         (r = st.in(d->candidates, (size_t)d->num_candidates * 4, &cdev)) != LV_OK)
+      return r;
+    if (d->load_keys &&
+        (r = st.in(d->load_keys, (size_t)pool->d.maxB * sizeof(uint64_t), &kdev)) != LV_OK)
       return r;
     if ((r = st.out(result_out, sizeof(lv_resident_result), &rdev, false)) != LV_OK) return r;
     if (++pool->epoch <= 0) pool->epoch = 1;
@@ -1079,9 +1084,9 @@ lv_status lv_turn(lv_pool* pool, const lv_turn_desc* d, lv_victim* victims_out, 
                            d->sid == -1 ? d->num_candidates : 0, d->now_us, d->append_tokens,
                            d->reply_audio_us, d->reply_units, pool->epoch, s, pool->exchange_ctas,
                            static_cast<lv_resident_result*>(rdev), timing_pair(pool, LV_TIMING_EXCHANGE),
-                           async ? &off : nullptr));
+                           async ? &off : nullptr, static_cast<const unsigned long long*>(kdev)));
     LV_TRY(copy_resident_outputs(pool, d->append_tokens, victims_out, slots_out, blocks_out, pages_out,
-                                 append_out, s));
+                                 append_out, s, d->load_keys != nullptr));
     return st.finish();
   } catch (const std::bad_alloc&) {
     return LV_ERR_OOM;

@@ -129,7 +129,8 @@ cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32
 struct ResidentScratch {
   lv_victim* victims;   // [budget]
   int32_t* slots;       // [budget]
-  int32_t* blocks;      // [maxB]
+  int32_t* blocks;      // [maxB] the session's host-tier blocks, ascending
+  int32_t* loads;       // [maxB] the same blocks in the caller's load order (load keys)
   int32_t* pages;       // [maxB]
   int32_t* append;      // [maxB + 2]
   int4* tasks;          // [budget + maxB]
@@ -140,7 +141,8 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
                                  int64_t now_us, int32_t append_tokens, bool preload,
                                  int64_t max_load, int32_t epoch, cudaStream_t s, int copy_ctas,
                                  lv_resident_result* result, const EventPair* ev = nullptr,
-                                 const long long* sid_dev = nullptr, const CopyOffload* off = nullptr);
+                                 const long long* sid_dev = nullptr, const CopyOffload* off = nullptr,
+                                 const unsigned long long* load_keys = nullptr);
 // lv_turn: pick (sid < 0), LV_EV_TURN_BEGIN, make resident, LV_EV_TURN_END
 // lv_evict: rank, evict up to k victims (no loads), finish
 cudaError_t launch_evict(const DevPool& p, const ResidentScratch& rs, int64_t now_us, int64_t k,
@@ -150,7 +152,7 @@ cudaError_t launch_turn(const DevPool& p, const ResidentScratch& rs, int32_t sid
                         int32_t n_cand, int64_t now_us, int32_t append_tokens, int64_t audio_us,
                         int64_t units, int32_t epoch, cudaStream_t s, int copy_ctas,
                         lv_resident_result* result, const EventPair* ev = nullptr,
-                        const CopyOffload* off = nullptr);
+                        const CopyOffload* off = nullptr, const unsigned long long* load_keys = nullptr);
 cudaError_t launch_counts(const DevPool& p, int32_t* hbm, int32_t* host, cudaStream_t s);
 // sums[i] = position-weighted 64-bit sum of page pages[i] (sums zeroed by the caller)
 cudaError_t launch_checksums(const DevPool& p, const int32_t* pages, int64_t n,

@@ -1385,6 +1385,31 @@ k_resident_prepare(DevPool p, int32_t sid, int32_t append_tokens, bool preload,
   }
 }
 
+constexpr int kOrderThreads = 256;
+
+// The caller's load order: host-tier block i of the session (ascending in
+// `blocks`, R[R_N_IN] of them) goes to position #{j : (key[b_j], b_j) <
+// (key[b_i], b_i)} of `loads` -- ascending (key, block id).  One warp per block.
+__global__ void __launch_bounds__(kOrderThreads)
+k_order_loads(const long long* __restrict__ R, const int32_t* __restrict__ blocks,
+              const unsigned long long* __restrict__ key, int32_t* __restrict__ loads) {
+  const long long nh = R[R_N_IN];
+  const long long i = blockIdx.x * (long long)(kOrderThreads / 32) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (i >= nh) return;
+  const int32_t bi = blocks[i];
+  const unsigned long long ki = key[bi];
+  int rank = 0;
+  for (long long j = lane; j < nh; j += 32) {
+    const int32_t bj = blocks[j];
+    const unsigned long long kj = key[bj];
+    rank += (kj < ki || (kj == ki && bj < bi)) ? 1 : 0;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) rank += __shfl_xor_sync(0xffffffffu, rank, o);
+  if (lane == 0) loads[rank] = bi;
+}
+
 // After the ranking: a shortfall stops the step (a preload is skipped, a
 // foreground turn fails), otherwise the exchange evicts exactly k victims.
 __global__ void k_resident_gate(DevPool p, bool preload, long long* __restrict__ R) {
@@ -1731,17 +1756,21 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
                                  int64_t now_us, int32_t append_tokens, bool preload,
                                  int64_t max_load, int32_t epoch, cudaStream_t s, int copy_ctas,
                                  lv_resident_result* result, const EventPair* ev,
-                                 const long long* sid_dev, const CopyOffload* off) {
+                                 const long long* sid_dev, const CopyOffload* off,
+                                 const unsigned long long* load_keys) {
   long long* R = rs.words;
   k_resident_prepare<<<1, kCensusThreads, 0, s>>>(p, sid, append_tokens, preload, max_load,
                                                   rs.blocks, R, sid_dev);
+  if (load_keys)
+    k_order_loads<<<blocks_for(p.maxB, kOrderThreads / 32, 1ll << 30), kOrderThreads, 0, s>>>(
+        R, rs.blocks, load_keys, rs.loads);
   cudaError_t e = launch_select(p, now_us, 0, !preload, rs.victims, nullptr, s, 0, R + R_K_SELECT);
   if (e != cudaSuccess) return e;
   k_resident_gate<<<1, 32, 0, s>>>(p, preload, R);
   const long long max_units = ((long long)p.budget + p.maxB) * p.J;
-  e = launch_exchange(p, rs.victims, 0, sid, rs.blocks, 0, rs.slots, rs.pages, rs.tasks,
-                      R + R_N_TASKS, epoch, p.page_tag, s, copy_ctas, R + R_N_OUT, max_units, ev,
-                      sid_dev, off);
+  e = launch_exchange(p, rs.victims, 0, sid, load_keys ? rs.loads : rs.blocks, 0, rs.slots, rs.pages,
+                      rs.tasks, R + R_N_TASKS, epoch, p.page_tag, s, copy_ctas, R + R_N_OUT, max_units,
+                      ev, sid_dev, off);
   if (e != cudaSuccess) return e;
   if (append_tokens > 0) {
     e = launch_append(p, sid, append_tokens, rs.append, reinterpret_cast<int32_t*>(R + R_APPENDED), s,
@@ -1772,12 +1801,13 @@ cudaError_t launch_evict(const DevPool& p, const ResidentScratch& rs, int64_t no
 cudaError_t launch_turn(const DevPool& p, const ResidentScratch& rs, int32_t sid, const int32_t* cand,
                         int32_t n_cand, int64_t now_us, int32_t append_tokens, int64_t audio_us,
                         int64_t units, int32_t epoch, cudaStream_t s, int copy_ctas,
-                        lv_resident_result* result, const EventPair* ev, const CopyOffload* off) {
+                        lv_resident_result* result, const EventPair* ev, const CopyOffload* off,
+                        const unsigned long long* load_keys) {
   long long* R = rs.words;
   if (sid < 0) k_pick_scan<<<n_cand, kCensusThreads, 0, s>>>(p, cand, rs.hits);
   k_turn_begin<<<1, 1024, 0, s>>>(p, sid, cand, n_cand, rs.hits, now_us, R);
   cudaError_t e = launch_make_resident(p, rs, sid, now_us, append_tokens, false, -1, epoch, s,
-                                       copy_ctas, result, ev, R + R_SID, off);
+                                       copy_ctas, result, ev, R + R_SID, off, load_keys);
   if (e != cudaSuccess) return e;
   k_turn_end<<<1, 32, 0, s>>>(p, now_us, audio_us, units, R);
   return cudaGetLastError();

@@ -60,7 +60,8 @@ class lv_turn_desc(ctypes.Structure):
     _fields_ = [("sid", ctypes.c_int32), ("num_candidates", ctypes.c_int32),
                 ("candidates", ctypes.c_void_p), ("now_us", ctypes.c_int64),
                 ("reply_audio_us", ctypes.c_int64), ("reply_units", ctypes.c_int64),
-                ("append_tokens", ctypes.c_int32), ("flags", ctypes.c_uint32)]
+                ("append_tokens", ctypes.c_int32), ("flags", ctypes.c_uint32),
+                ("load_keys", ctypes.c_void_p)]
 
 
 class lv_controller_desc(ctypes.Structure):
@@ -331,12 +332,14 @@ def lv_make_resident(pool, sid, now_us, append_tokens, flags, max_load_pages, vi
 
 
 def lv_turn(pool, sid, now_us, append_tokens, reply_audio_us, reply_units, outs=(None,) * 5,
-            result_out=None, candidates=None, num_candidates=0, stream=None, flags=0):
+            result_out=None, candidates=None, num_candidates=0, stream=None, flags=0,
+            load_keys=None):
     """One turn (pick when sid == -1, turn begin, make resident, turn end); outs =
-    (victims, slots, blocks, pages, append) as for lv_make_resident."""
+    (victims, slots, blocks, pages, append) as for lv_make_resident; load_keys (uint64
+    [max_blocks]) orders the loads."""
     d = lv_turn_desc(sid=sid, num_candidates=num_candidates, candidates=ptr(candidates),
                      now_us=now_us, reply_audio_us=reply_audio_us, reply_units=reply_units,
-                     append_tokens=append_tokens, flags=flags)
+                     append_tokens=append_tokens, flags=flags, load_keys=ptr(load_keys))
     _check(_lib.lv_turn(pool, ctypes.byref(d), *(ptr(o) for o in outs), ptr(result_out),
                         stream_handle(stream)), "lv_turn")
 

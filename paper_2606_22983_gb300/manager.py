@@ -8,7 +8,9 @@ Consumes monitor event scripts (records ``(t_us, kind, sid, a, b, c, d)``):
   kind 3 PLAYBACK(sid, a=delta_us)    kind 4 SPEECH_START(sid)
   kind 5 BARGE_IN(sid)                kind 6 SPEECH_STOP(sid)
   kind 7 TURN_SCATTER(d=row, a=key): as TURN_ANY, host blocks reloaded in the
-         order ``order_fn(key, blocks)`` (given by the caller)
+         order ``order_fn(key, blocks)`` (given by the caller; it must order blocks
+         by a key of each block alone, so that the device driver can pass it as
+         per-block load keys)
   kind 8 EVICT(a=k): free k pages now, in the next-use order
 
 A turn makes the session fully resident (a synchronous foreground load),
@@ -141,7 +143,18 @@ class KVManager:
             self.on_append(sid, old_ctx, old_ctx + append_tokens)
         return status
 
-    def _device_turn(self, sid, row, now_us, append_tokens, reply_us, reply_units, rec):
+    def _load_keys(self, order_key):
+        """Per-block keys whose ascending order is ``order_fn(order_key, blocks)`` for any
+        set of blocks: the rank of each block in the order of all of them (``order_fn``
+        orders blocks by a key of the block alone, as the workloads' scatter order does)."""
+        nb = self.pool.max_blocks
+        perm = np.asarray(self.order_fn(order_key, np.arange(nb)), dtype=np.int64)
+        keys = np.empty(nb, dtype=np.uint64)
+        keys[perm] = np.arange(nb, dtype=np.uint64)
+        return keys
+
+    def _device_turn(self, sid, row, now_us, append_tokens, reply_us, reply_units, rec,
+                     load_keys=None):
         """One lv_turn: (pick,) turn begin, make resident, turn end -- no host round trip
         unless the decisions are recorded.  Returns the session id (-1 when not read back)."""
         pool = self.pool
@@ -150,7 +163,8 @@ class KVManager:
         outs = (pool.victims, pool.slots, pool.blks, pool.pages, pool.app) if self.record else (None,) * 5
         lv.lv_turn(pool.handle, sid, now_us, append_tokens, reply_us, reply_units, outs, self.res_h,
                    cand, int(cand.numel()) if cand is not None else 0, pool.stream,
-                   lv.LV_RESIDENT_ASYNC_COPY if self.async_copy else 0)
+                   lv.LV_RESIDENT_ASYNC_COPY if self.async_copy else 0, load_keys)
+        pool.launches += 1 if load_keys is not None else 0
         pool.launches += 9 + (1 if sid < 0 else 0) + (1 if append_tokens else 0)
         if not rec_bufs:
             return sid
@@ -395,6 +409,10 @@ class KVManager:
                 self.preload(sid, t, rec)
         elif kind in (EV_TURN, EV_TURN_ANY) and self.driver == "device":
             sid = self._device_turn(sid if kind == EV_TURN else -1, d, t, a, b, c, rec)
+            self.counters["turns"] += 1
+        elif kind == EV_TURN_SCATTER and self.driver == "device" and self.order_fn is not None:
+            # the reload order is the script's scatter order, given as per-block keys
+            sid = self._device_turn(-1, d, t, 0, b, c, rec, load_keys=self._load_keys(a))
             self.counters["turns"] += 1
         elif kind in (EV_TURN, EV_TURN_ANY, EV_TURN_SCATTER):
             order_key = None

@@ -76,7 +76,7 @@ int main(void) {
   F(lv_controller_record, data_offset);
   F(lv_turn_desc, sid); F(lv_turn_desc, num_candidates); F(lv_turn_desc, candidates);
   F(lv_turn_desc, now_us); F(lv_turn_desc, reply_audio_us); F(lv_turn_desc, reply_units);
-  F(lv_turn_desc, append_tokens); F(lv_turn_desc, flags);
+  F(lv_turn_desc, append_tokens); F(lv_turn_desc, flags); F(lv_turn_desc, load_keys);
   F(lv_session_state, ctx_tokens); F(lv_session_state, flags); F(lv_session_state, gen_us);
   F(lv_session_state, play_us); F(lv_session_state, t_done_us); F(lv_session_state, reply_ema_us);
   F(lv_session_state, reply_n); F(lv_session_state, reply_tokens); F(lv_session_state, protect_until_us);
