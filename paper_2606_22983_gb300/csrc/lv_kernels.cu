@@ -16,6 +16,7 @@
 // index read from memory is range-checked and a bad item is skipped with the
 // sticky error set.
 #include <cstdint>
+#include <utility>
 
 #include "lv_internal.cuh"
 
@@ -28,6 +29,18 @@ __device__ __forceinline__ void set_error(long long* ctl, int code, long long de
                 (unsigned long long)code) == 0ull) {
     ctl[C_ERR_DETAIL] = detail;
   }
+}
+
+// Programmatic dependent launch.  The kernels of a device-driven step are
+// launched so that each may be scheduled while the previous kernel on the
+// stream still runs (its launch latency overlaps that kernel).  Each of them
+// begins with pdl_entry(): it waits until the previous kernel has completed
+// and its writes are visible -- nothing of the kernel runs earlier -- and then
+// lets the next kernel of the stream be scheduled.  In a kernel launched the
+// ordinary way both instructions have no effect.
+__device__ __forceinline__ void pdl_entry() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 __device__ __forceinline__ int32_t nblocks_of(const DevPool& p, int32_t sid) {
@@ -347,9 +360,7 @@ constexpr int kCensusThreads = 256;
 // One CTA per session: its key and its count of HBM-resident blocks.
 __global__ void __launch_bounds__(kCensusThreads)
 k_rank_census(DevPool p, long long now_us, bool fallback) {
-  // the emit kernel may be scheduled as soon as every census CTA has started; it
-  // waits for the whole census (griddepcontrol.wait) before it reads anything
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  pdl_entry();
   const int32_t s = blockIdx.x;
   __shared__ unsigned long long key;
   if (threadIdx.x == 0) key = session_key(p, s, now_us, fallback);
@@ -382,7 +393,7 @@ constexpr int kEmitThreads = 256;
 __global__ void __launch_bounds__(kEmitThreads)
 k_rank_emit(DevPool p, long long k, const long long* k_dev, bool fallback, long long* count_dev,
             lv_victim* __restrict__ out) {
-  asm volatile("griddepcontrol.wait;" ::: "memory");   // the census is complete and visible
+  pdl_entry();   // the census is complete and visible
   const int32_t sid = blockIdx.x;
   const unsigned long long key = p.skey[sid];
   if (key == 0ull && sid != 0) return;
@@ -591,6 +602,7 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
                 int32_t* __restrict__ pages, int4* __restrict__ tasks, long long* n_tasks,
                 int32_t epoch, unsigned long long* __restrict__ page_tag,
                 const long long* __restrict__ counts_dev, const long long* __restrict__ sid_dev) {
+  pdl_entry();
   if (counts_dev) {          // counts decided on the device (lv_make_resident)
     n_out = counts_dev[0];
     n_in = counts_dev[1];
@@ -730,6 +742,7 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
 // stores either, so a paired task reads the old page before overwriting it.
 __global__ void __launch_bounds__(kCopyThreads)
 k_exchange_copy(DevPool p, const int4* __restrict__ tasks, const long long* __restrict__ n_tasks) {
+  pdl_entry();
   const long long units = *n_tasks * p.J;
   const int nvec = (int)(p.P >> 4);
   for (long long u = blockIdx.x; u < units; u += gridDim.x) {
@@ -1245,6 +1258,7 @@ __global__ void __launch_bounds__(kAllocThreads)
 k_append(DevPool p, int32_t sid, int32_t n_tokens, int32_t* __restrict__ pages,
          int32_t* __restrict__ count, const long long* __restrict__ gate,
          const long long* __restrict__ sid_dev) {
+  pdl_entry();
   __shared__ long long m_s, nb_s, ctx_s;
   if (gate && *gate != 0) {   // an earlier step of lv_make_resident did not complete
     if (threadIdx.x == 0 && count) *count = 0;
@@ -1335,6 +1349,7 @@ __global__ void __launch_bounds__(kCensusThreads)
 k_resident_prepare(DevPool p, int32_t sid, int32_t append_tokens, bool preload,
                    long long max_load, int32_t* __restrict__ blocks, long long* __restrict__ R,
                    const long long* __restrict__ sid_dev) {
+  pdl_entry();
   if (sid_dev) sid = (int32_t)*sid_dev;
   if (sid < 0 || sid >= p.S) {        // lv_turn's pick failed (already reported)
     if (threadIdx.x == 0) {
@@ -1393,6 +1408,7 @@ constexpr int kOrderThreads = 256;
 __global__ void __launch_bounds__(kOrderThreads)
 k_order_loads(const long long* __restrict__ R, const int32_t* __restrict__ blocks,
               const unsigned long long* __restrict__ key, int32_t* __restrict__ loads) {
+  pdl_entry();
   const long long nh = R[R_N_IN];
   const long long i = blockIdx.x * (long long)(kOrderThreads / 32) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -1413,6 +1429,7 @@ k_order_loads(const long long* __restrict__ R, const int32_t* __restrict__ block
 // After the ranking: a shortfall stops the step (a preload is skipped, a
 // foreground turn fails), otherwise the exchange evicts exactly k victims.
 __global__ void k_resident_gate(DevPool p, bool preload, long long* __restrict__ R) {
+  pdl_entry();
   if (threadIdx.x != 0 || R[R_STATUS] != LV_RESIDENT_DONE) return;
   const long long found = p.ctl[C_SEL_COUNT], k = R[R_K];
   R[R_FOUND] = found;
@@ -1435,6 +1452,7 @@ __global__ void k_resident_gate(DevPool p, bool preload, long long* __restrict__
 __global__ void k_resident_finish(DevPool p, int32_t sid, long long now_us, bool preload,
                                   long long* __restrict__ R, lv_resident_result* __restrict__ out,
                                   const long long* __restrict__ sid_dev) {
+  pdl_entry();
   if (threadIdx.x != 0) return;
   if (sid_dev) sid = (int32_t)*sid_dev;
   const int status = (int)R[R_STATUS];
@@ -1459,6 +1477,7 @@ __global__ void k_resident_finish(DevPool p, int32_t sid, long long now_us, bool
 // lv_evict: up to k victims by the normal order (no fallback tier), fewer when
 // there are fewer candidates; nothing is loaded.
 __global__ void k_evict_prepare(long long k, long long* __restrict__ R) {
+  pdl_entry();
   if (threadIdx.x != 0) return;
   R[R_K_SELECT] = k;
   R[R_N_OUT] = 0;
@@ -1472,6 +1491,7 @@ __global__ void k_evict_prepare(long long k, long long* __restrict__ R) {
 }
 
 __global__ void k_evict_gate(DevPool p, long long* __restrict__ R) {
+  pdl_entry();
   if (threadIdx.x != 0) return;
   const long long found = p.ctl[C_SEL_COUNT];   // min(k, candidates)
   R[R_FOUND] = found;
@@ -1483,6 +1503,7 @@ __global__ void k_evict_gate(DevPool p, long long* __restrict__ R) {
 // lv_turn's pick: CTA c reports whether candidate c has a block in the host tier.
 __global__ void __launch_bounds__(kCensusThreads)
 k_pick_scan(DevPool p, const int32_t* __restrict__ cand, int32_t* __restrict__ hit) {
+  pdl_entry();
   const int32_t s = cand[blockIdx.x];
   int any = 0;
   if (s >= 0 && s < p.S) {
@@ -1499,6 +1520,7 @@ k_pick_scan(DevPool p, const int32_t* __restrict__ cand, int32_t* __restrict__ h
 __global__ void __launch_bounds__(1024)
 k_turn_begin(DevPool p, int32_t sid, const int32_t* __restrict__ cand, int32_t n,
              const int32_t* __restrict__ hit, long long now_us, long long* __restrict__ R) {
+  pdl_entry();
   __shared__ int first;
   if (threadIdx.x == 0) first = n;
   __syncthreads();
@@ -1532,6 +1554,7 @@ k_turn_begin(DevPool p, int32_t sid, const int32_t* __restrict__ cand, int32_t n
 // LV_EV_TURN_END for the turn's session, unless its KV could not be made resident.
 __global__ void k_turn_end(DevPool p, long long now_us, long long audio_us, long long units,
                            const long long* __restrict__ R) {
+  pdl_entry();
   if (threadIdx.x != 0) return;
   const long long sid = R[R_SID];
   if (sid < 0 || sid >= p.S || R[R_STATUS] == LV_RESIDENT_FAILED) return;
@@ -1666,6 +1689,24 @@ cudaError_t launch_session_set(const DevPool& p, const lv_session_state* in, int
   return cudaGetLastError();
 }
 
+// A launch that lets the kernel be scheduled while the previous kernel on `s`
+// still runs; the kernel must begin with pdl_entry().
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), unsigned grid, unsigned block, size_t smem,
+                       cudaStream_t s, Args&&... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(block);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 cudaError_t launch_events(const DevPool& p, const lv_event* ev, int64_t n, cudaStream_t s) {
   k_events<<<blocks_for(p.S, kEventThreads, 1 << 20), kEventThreads, 0, s>>>(p, ev, n);
   return cudaGetLastError();
@@ -1674,19 +1715,11 @@ cudaError_t launch_events(const DevPool& p, const lv_event* ev, int64_t n, cudaS
 cudaError_t launch_select(const DevPool& p, int64_t now_us, int64_t k, bool fallback,
                           lv_victim* out, long long* count_dev, cudaStream_t s, int /*num_sms*/,
                           const long long* k_dev) {
-  k_rank_census<<<p.S, kCensusThreads, 0, s>>>(p, now_us, fallback);
-  // programmatic dependent launch: the emit grid's launch overlaps the census
-  cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3((unsigned)p.S);
-  cfg.blockDim = dim3(kEmitThreads);
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  const cudaError_t e = cudaLaunchKernelEx(&cfg, k_rank_emit, p, (long long)k, k_dev, fallback,
-                                           count_dev, out);
+  cudaError_t e = launch_pdl(k_rank_census, (unsigned)p.S, kCensusThreads, 0, s, p, (long long)now_us,
+                             fallback);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(k_rank_emit, (unsigned)p.S, kEmitThreads, 0, s, p, (long long)k, k_dev, fallback,
+                 count_dev, out);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
@@ -1732,8 +1765,10 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
                             unsigned long long* page_tag, cudaStream_t s, int copy_ctas,
                             const long long* counts_dev, long long max_units, const EventPair* ev,
                             const long long* sid_dev, const CopyOffload* off) {
-  k_exchange_plan<<<1, kPlanThreads, 0, s>>>(p, v, n_out, sid, blks, n_in, slots, pages, tasks,
-                                             n_tasks, epoch, page_tag, counts_dev, sid_dev);
+  cudaError_t le = launch_pdl(k_exchange_plan, 1, kPlanThreads, 0, s, p, v, (long long)n_out, sid,
+                              blks, (long long)n_in, slots, pages, tasks, n_tasks, epoch, page_tag,
+                              counts_dev, sid_dev);
+  if (le != cudaSuccess) return le;
   const long long units = counts_dev ? max_units : (n_out + n_in) * (long long)p.J;
   cudaStream_t cs = s;
   if (off) {
@@ -1743,7 +1778,13 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
     cs = off->stream;
   }
   if (ev) cudaEventRecord(ev->start, cs);
-  k_exchange_copy<<<blocks_for(units, 1, copy_ctas), kCopyThreads, 0, cs>>>(p, tasks, n_tasks);
+  if (off || ev) {   // after an event wait or record: an ordinary launch
+    k_exchange_copy<<<blocks_for(units, 1, copy_ctas), kCopyThreads, 0, cs>>>(p, tasks, n_tasks);
+  } else {
+    le = launch_pdl(k_exchange_copy, blocks_for(units, 1, copy_ctas), kCopyThreads, 0, cs, p,
+                    (const int4*)tasks, (const long long*)n_tasks);
+    if (le != cudaSuccess) return le;
+  }
   if (ev) cudaEventRecord(ev->end, cs);
   if (off) {
     const cudaError_t e = cudaEventRecord(off->copied, cs);
@@ -1759,14 +1800,18 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
                                  const long long* sid_dev, const CopyOffload* off,
                                  const unsigned long long* load_keys) {
   long long* R = rs.words;
-  k_resident_prepare<<<1, kCensusThreads, 0, s>>>(p, sid, append_tokens, preload, max_load,
-                                                  rs.blocks, R, sid_dev);
-  if (load_keys)
-    k_order_loads<<<blocks_for(p.maxB, kOrderThreads / 32, 1ll << 30), kOrderThreads, 0, s>>>(
-        R, rs.blocks, load_keys, rs.loads);
-  cudaError_t e = launch_select(p, now_us, 0, !preload, rs.victims, nullptr, s, 0, R + R_K_SELECT);
+  cudaError_t e = launch_pdl(k_resident_prepare, 1, kCensusThreads, 0, s, p, sid, append_tokens,
+                             preload, (long long)max_load, rs.blocks, R, sid_dev);
   if (e != cudaSuccess) return e;
-  k_resident_gate<<<1, 32, 0, s>>>(p, preload, R);
+  if (load_keys) {
+    e = launch_pdl(k_order_loads, blocks_for(p.maxB, kOrderThreads / 32, 1ll << 30), kOrderThreads, 0,
+                   s, (const long long*)R, (const int32_t*)rs.blocks, load_keys, rs.loads);
+    if (e != cudaSuccess) return e;
+  }
+  e = launch_select(p, now_us, 0, !preload, rs.victims, nullptr, s, 0, R + R_K_SELECT);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(k_resident_gate, 1, 32, 0, s, p, preload, R);
+  if (e != cudaSuccess) return e;
   const long long max_units = ((long long)p.budget + p.maxB) * p.J;
   e = launch_exchange(p, rs.victims, 0, sid, load_keys ? rs.loads : rs.blocks, 0, rs.slots, rs.pages,
                       rs.tasks, R + R_N_TASKS, epoch, p.page_tag, s, copy_ctas, R + R_N_OUT, max_units,
@@ -1777,7 +1822,9 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
                       R + R_GATE, sid_dev);
     if (e != cudaSuccess) return e;
   }
-  k_resident_finish<<<1, 32, 0, s>>>(p, sid, now_us, preload, R, result, sid_dev);
+  e = launch_pdl(k_resident_finish, 1, 32, 0, s, p, sid, (long long)now_us, preload, R, result,
+                 sid_dev);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
@@ -1785,16 +1832,20 @@ cudaError_t launch_evict(const DevPool& p, const ResidentScratch& rs, int64_t no
                          int32_t epoch, cudaStream_t s, int copy_ctas, lv_resident_result* result,
                          const EventPair* ev, const CopyOffload* off) {
   long long* R = rs.words;
-  k_evict_prepare<<<1, 32, 0, s>>>(k, R);
-  cudaError_t e = launch_select(p, now_us, 0, false, rs.victims, nullptr, s, 0, R + R_K_SELECT);
+  cudaError_t e = launch_pdl(k_evict_prepare, 1, 32, 0, s, (long long)k, R);
   if (e != cudaSuccess) return e;
-  k_evict_gate<<<1, 32, 0, s>>>(p, R);
+  e = launch_select(p, now_us, 0, false, rs.victims, nullptr, s, 0, R + R_K_SELECT);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(k_evict_gate, 1, 32, 0, s, p, R);
+  if (e != cudaSuccess) return e;
   const long long max_units = (long long)p.budget * p.J;
   e = launch_exchange(p, rs.victims, 0, -1, rs.blocks, 0, rs.slots, rs.pages, rs.tasks,
                       R + R_N_TASKS, epoch, p.page_tag, s, copy_ctas, R + R_N_OUT, max_units, ev,
                       nullptr, off);
   if (e != cudaSuccess) return e;
-  k_resident_finish<<<1, 32, 0, s>>>(p, -1, now_us, false, R, result, nullptr);
+  e = launch_pdl(k_resident_finish, 1, 32, 0, s, p, (int32_t)-1, (long long)now_us, false, R, result,
+                 (const long long*)nullptr);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
@@ -1804,12 +1855,20 @@ cudaError_t launch_turn(const DevPool& p, const ResidentScratch& rs, int32_t sid
                         lv_resident_result* result, const EventPair* ev, const CopyOffload* off,
                         const unsigned long long* load_keys) {
   long long* R = rs.words;
-  if (sid < 0) k_pick_scan<<<n_cand, kCensusThreads, 0, s>>>(p, cand, rs.hits);
-  k_turn_begin<<<1, 1024, 0, s>>>(p, sid, cand, n_cand, rs.hits, now_us, R);
+  cudaError_t e0 = cudaSuccess;
+  if (sid < 0) {
+    e0 = launch_pdl(k_pick_scan, (unsigned)n_cand, kCensusThreads, 0, s, p, cand, rs.hits);
+    if (e0 != cudaSuccess) return e0;
+  }
+  e0 = launch_pdl(k_turn_begin, 1, 1024, 0, s, p, sid, cand, n_cand, (const int32_t*)rs.hits,
+                  (long long)now_us, R);
+  if (e0 != cudaSuccess) return e0;
   cudaError_t e = launch_make_resident(p, rs, sid, now_us, append_tokens, false, -1, epoch, s,
                                        copy_ctas, result, ev, R + R_SID, off, load_keys);
   if (e != cudaSuccess) return e;
-  k_turn_end<<<1, 32, 0, s>>>(p, now_us, audio_us, units, R);
+  e = launch_pdl(k_turn_end, 1, 32, 0, s, p, (long long)now_us, (long long)audio_us, (long long)units,
+                 (const long long*)R);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
@@ -1917,7 +1976,9 @@ cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cuda
 cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32_t* pages,
                           int32_t* count, cudaStream_t s, const long long* gate,
                           const long long* sid_dev) {
-  k_append<<<1, kAllocThreads, 0, s>>>(p, sid, n_tokens, pages, count, gate, sid_dev);
+  const cudaError_t e = launch_pdl(k_append, 1, kAllocThreads, 0, s, p, sid, n_tokens, pages, count,
+                                   gate, sid_dev);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
