@@ -225,7 +225,7 @@ def ours(args, torch):
     h2d = K * S * lv.EVENT_DTYPE.itemsize
     d2h = K * lv.RESIDENT_DTYPE.itemsize
     torch.cuda.synchronize()
-    q0 = _moved_pages(pool)[0]
+    q0, qo0, qi0 = _moved_pages(pool)
     w0 = time.perf_counter()
     for j, i in enumerate(range(W + K, W + 2 * K)):
         lv.lv_session_events(pool.handle, ev_h[j], S, pool.stream)
@@ -237,7 +237,9 @@ def ours(args, torch):
     gm.res_h = own_res
     status = res_h.numpy().view(lv.RESIDENT_DTYPE)["status"]
     assert (status == lv.LV_RESIDENT_DONE).all(), "a turn of the end-to-end pass failed"
-    moved_e2e = (_moved_pages(pool)[0] - q0) * page_bytes
+    q1, qo1, qi1 = _moved_pages(pool)
+    moved_e2e = (q1 - q0) * page_bytes
+    e2e_out, e2e_in = (qo1 - qo0) * page_bytes, (qi1 - qi0) * page_bytes
     if dist:
         tt = torch.tensor([dev_s, e2e_s, moved, moved_e2e], dtype=torch.float64, device="cuda")
         gathered = [torch.zeros_like(tt) for _ in range(ws)]
@@ -307,7 +309,12 @@ def ours(args, torch):
             "kernels": {n: {k: round(v, 3) for k, v in d.items()} for n, d in kern.items()},
             "in_turn_hbm_kernels": hbm_kern or None,
             "e2e": {"value": round(e2e_value, 3), "unit": UNIT,
-                    "h2d_bytes_per_step": int(h2d / K), "d2h_bytes_per_step": int(d2h / K)},
+                    "h2d_bytes_per_step": int(h2d / K), "d2h_bytes_per_step": int(d2h / K),
+                    # its own turns (the K after the device-timed ones) and their link roofline
+                    "mean_turn_mb_each_way": round(moved_e2e / K / 2 / 1e6, 1),
+                    "link_frac": (round(max(e2e_out / peaks["d2h"], e2e_in / peaks["h2d"],
+                                            moved_e2e / peaks["bidir"]) / 1e9 / e2e_s, 3)
+                                  if "bidir" in peaks and ws == 1 else None)},
             "gpu_launches": int(launches),
             "clocks": clk,
         }

@@ -54,6 +54,7 @@ struct lv_pool {
   uint32_t rs_seq = 0;
   cudaStream_t s_copy = nullptr;
   cudaEvent_t ev_planned = nullptr;
+  cudaEvent_t ev_copy_start = nullptr, ev_copy_end = nullptr;
   cudaEvent_t ev_copied[2] = {nullptr, nullptr};
   bool copied_pending[2] = {false, false};   // an async copy used scratch set b
   // LV_MODE_STAGED | LV_MODE_ASYNC: unpacks on s_unpack; the last call's D2H, H2D and
@@ -439,7 +440,8 @@ cudaError_t next_scratch(lv_pool* pool, cudaStream_t s, bool async, const lv::Re
     const cudaError_t e = cudaStreamWaitEvent(s, pool->ev_copied[b], 0);
     if (e != cudaSuccess) return e;
   }
-  *off = lv::CopyOffload{pool->s_copy, pool->ev_planned, pool->ev_copied[b]};
+  *off = lv::CopyOffload{pool->s_copy, pool->ev_planned, pool->ev_copied[b], pool->ev_copy_start,
+                         pool->ev_copy_end};
   pool->copied_pending[b] = true;
   return cudaSuccess;
 }
@@ -453,6 +455,8 @@ void free_pool(lv_pool* pool) {
   if (pool->s_copy) cudaStreamSynchronize(pool->s_copy);
   if (pool->s_copy) cudaStreamDestroy(pool->s_copy);
   if (pool->ev_planned) cudaEventDestroy(pool->ev_planned);
+  if (pool->ev_copy_start) cudaEventDestroy(pool->ev_copy_start);
+  if (pool->ev_copy_end) cudaEventDestroy(pool->ev_copy_end);
   for (cudaEvent_t e : pool->ev_copied)
     if (e) cudaEventDestroy(e);
   for (cudaEvent_t e : pool->sync_events) cudaEventDestroy(e);
@@ -599,6 +603,8 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
   if (cudaDeviceGetStreamPriorityRange(&prio_least, &prio_greatest) != cudaSuccess) prio_greatest = 0;
   if (cudaStreamCreateWithPriority(&pool->s_copy, cudaStreamNonBlocking, prio_greatest) != cudaSuccess ||
       cudaEventCreateWithFlags(&pool->ev_planned, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreate(&pool->ev_copy_start) != cudaSuccess ||
+      cudaEventCreate(&pool->ev_copy_end) != cudaSuccess ||
       cudaEventCreateWithFlags(&pool->ev_copied[0], cudaEventDisableTiming) != cudaSuccess ||
       cudaEventCreateWithFlags(&pool->ev_copied[1], cudaEventDisableTiming) != cudaSuccess)
     return fail(LV_ERR_CUDA);

@@ -1778,6 +1778,7 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
     cs = off->stream;
   }
   if (ev) cudaEventRecord(ev->start, cs);
+  else if (off && off->started) cudaEventRecord(off->started, cs);
   if (off || ev) {   // after an event wait or record: an ordinary launch
     k_exchange_copy<<<blocks_for(units, 1, copy_ctas), kCopyThreads, 0, cs>>>(p, tasks, n_tasks);
   } else {
@@ -1786,6 +1787,7 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
     if (le != cudaSuccess) return le;
   }
   if (ev) cudaEventRecord(ev->end, cs);
+  else if (off && off->finished) cudaEventRecord(off->finished, cs);
   if (off) {
     const cudaError_t e = cudaEventRecord(off->copied, cs);
     if (e != cudaSuccess) return e;
