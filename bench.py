@@ -381,8 +381,10 @@ def overlap_measure(torch, pool, wl, first_turn, n_turns):
                                             ("staged_copy_engine", "exchange", 2, True)):
         gm = KVManager(pool, perms=wl.perms, rank_on="none", mode=mode, record=False,
                        driver=driver, async_copy=async_copy)
-        run_turns(gm, wl, turn, turn + 3, None)             # warm-up of this driver
-        turn += 3
+        # warm-up of this driver (the staged path's stream-ordered staging pool grows
+        # during its first calls)
+        run_turns(gm, wl, turn, turn + 10, None)
+        turn += 10
         lv.lv_join(pool.handle, pool.stream)
         torch.cuda.synchronize()
         # the turns alone
@@ -776,7 +778,7 @@ def _arm_spec(args, seed):
         over["spec"] = sp.with_(n_sessions=args.sessions or sp.n_sessions, hbm_pages=b,
                                 hbm_budget_pages=b, tiers=args.tiers)
     KO = OVERLAP_TURNS if (args.overlap and args.driver == "device") else 0
-    return make_workload(WORKLOAD, seed, n_turns=args.warmup + 2 * args.steps + 4 * KO + 6,
+    return make_workload(WORKLOAD, seed, n_turns=args.warmup + 2 * args.steps + 4 * KO + 26,
                          **over)
 
 
