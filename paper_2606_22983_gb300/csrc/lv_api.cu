@@ -67,6 +67,13 @@ struct lv_pool {
   // their D2H copies write, slots their H2D copies read; a new call waits for an event
   // only when it touches a marked page or slot
   MarkSet st_loaded, st_written, st_read;
+  // staging runs of the staged path, used by alternate calls and kept between calls;
+  // st_buf_done[b] completes when the call that last used run b has finished with it
+  void* st_buf[2] = {nullptr, nullptr};
+  size_t st_buf_bytes[2] = {0, 0};
+  cudaEvent_t st_buf_done[2] = {nullptr, nullptr};
+  bool st_buf_used[2] = {false, false};
+  uint32_t st_seq = 0;
   // staged path: side streams for the copy engines, a host copy of the tasks, sync events
   cudaStream_t s_d2h = nullptr, s_h2d = nullptr;
   int4* tasks_host = nullptr;
@@ -243,14 +250,6 @@ lv_status sync_events(lv_pool* pool, size_t n) {
   return LV_OK;
 }
 
-// The staged data movement of n validated tasks {out page, out slot, in slot, in page}
-// on `s`.  The task list is read back once; its out halves are sorted by host slot and
-// so are its in halves, so that consecutive slots become one copy-engine transfer
-// whatever order the blocks were listed in (a session evicted suffix first sits in
-// descending slots).  Then: pack the out pages into staging in slot order; copy-engine
-// runs in each direction on the side streams; unpack into the in pages; joined back
-// into `s`.  Every pack precedes every unpack on `s`, so a page that an incoming block
-// takes is read before it is overwritten.
 // Drops the marks of `m` once `ev` (recorded after every transfer that marked it)
 // has completed; a query that finds it still running keeps them.
 cudaError_t prune_marks(cudaEvent_t ev, MarkSet& m) {
@@ -262,6 +261,14 @@ cudaError_t prune_marks(cudaEvent_t ev, MarkSet& m) {
   return cudaSuccess;
 }
 
+// The staged data movement of n validated tasks {out page, out slot, in slot, in page}
+// on `s`.  The task list is read back once; its out halves are sorted by host slot and
+// so are its in halves, so that consecutive slots become one copy-engine transfer
+// whatever order the blocks were listed in (a session evicted suffix first sits in
+// descending slots).  Then: pack the out pages into staging in slot order; copy-engine
+// runs in each direction on the side streams; unpack into the in pages; joined back
+// into `s`.  Every pack precedes every unpack on `s`, so a page that an incoming block
+// takes is read before it is overwritten.
 lv_status staged_move_inner(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStream_t s,
                             void** staging_out, bool async) {
   const lv::DevPool& d = pool->d;
@@ -290,14 +297,29 @@ lv_status staged_move_inner(lv_pool* pool, const int4* tasks_dev, int64_t n, cud
   cudaEvent_t ev_start = ev[0];
   cudaEvent_t* ev_pack = ev + 3;            // [nchunks]
   cudaEvent_t* ev_h2d = ev + 3 + nchunks;   // [nchunks]
-  // staging: out run [n_out][2L][P], in run [n_in][2L][P], then the sorted task lists
-  void* staging = nullptr;
+  // staging: out run [n_out][2L][P], in run [n_in][2L][P], then the sorted task lists, in
+  // the pool's run b (alternate calls); `s` waits until the call that used run b last is
+  // done with it, and the run grows (with a quarter to spare) when this call needs more
+  const int b = (int)(pool->st_seq++ & 1u);
+  *staging_out = &pool->st_buf[b];
+  if (pool->st_buf_used[b]) LV_TRY(cudaStreamWaitEvent(s, pool->st_buf_done[b], 0));
+  pool->st_buf_used[b] = true;
   {
     const size_t bytes = (size_t)(n_out + n_in) * pb + (size_t)(n_out + n_in) * sizeof(int4);
-    cudaError_t e = cudaMallocFromPoolAsync(&staging, bytes, pool->mp, s);
-    if (e != cudaSuccess) return lv_cuda_fail(e);
-    *staging_out = staging;
+    if (bytes > pool->st_buf_bytes[b]) {
+      if (pool->st_buf[b]) LV_TRY(cudaFreeAsync(pool->st_buf[b], s));
+      pool->st_buf[b] = nullptr;
+      pool->st_buf_bytes[b] = 0;
+      const size_t want = (bytes + bytes / 4 + (64u << 20) - 1) / (64u << 20) * (64u << 20);
+      cudaError_t e = cudaMallocFromPoolAsync(&pool->st_buf[b], want, pool->mp, s);
+      if (e != cudaSuccess) {
+        pool->st_buf[b] = nullptr;
+        return lv_cuda_fail(e);
+      }
+      pool->st_buf_bytes[b] = want;
+    }
   }
+  void* staging = pool->st_buf[b];
   uint8_t* stg_out = static_cast<uint8_t*>(staging);
   uint8_t* stg_in = stg_out + (size_t)n_out * pb;
   int4* tout_dev = reinterpret_cast<int4*>(stg_in + (size_t)n_in * pb);
@@ -380,21 +402,22 @@ lv_status staged_move_inner(lv_pool* pool, const int4* tasks_dev, int64_t n, cud
 }
 
 // staged_move_inner, then (also after an early error) join the side streams back
-// into `s` and release the staging run in stream order.
+// into `s` and mark the staging run free in stream order.
 lv_status staged_move(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStream_t s,
                       bool async = false) {
-  void* staging = nullptr;
-  const lv_status st = staged_move_inner(pool, tasks_dev, n, s, &staging, async);
-  if (!staging) return st;
+  void* slot = nullptr;   // &pool->st_buf[b] once the call has taken run b
+  const lv_status st = staged_move_inner(pool, tasks_dev, n, s, &slot, async);
+  if (!slot) return st;
+  const int b = static_cast<void**>(slot) == &pool->st_buf[0] ? 0 : 1;
   if (async && st == LV_OK) {
-    // the next asynchronous call orders itself on these; the staging run is freed
-    // once both directions and the unpacks are done
+    // the next asynchronous calls order themselves on these; run b is free again once
+    // both directions and the unpacks are done
     cudaEventRecord(pool->ev_st_d2h, pool->s_d2h);
     cudaEventRecord(pool->ev_st_h2d, pool->s_h2d);
     cudaEventRecord(pool->ev_st_unpack, pool->s_unpack);
     cudaStreamWaitEvent(pool->s_unpack, pool->ev_st_d2h, 0);
     cudaStreamWaitEvent(pool->s_unpack, pool->ev_st_h2d, 0);
-    cudaFreeAsync(staging, pool->s_unpack);
+    cudaEventRecord(pool->st_buf_done[b], pool->s_unpack);
     cudaEventRecord(pool->ev_st_done, pool->s_unpack);
     pool->st_pending = true;
     return st;
@@ -408,7 +431,7 @@ lv_status staged_move(lv_pool* pool, const int4* tasks_dev, int64_t n, cudaStrea
     cudaEventRecord(pool->ev_st_unpack, pool->s_unpack);
     cudaStreamWaitEvent(s, pool->ev_st_unpack, 0);
   }
-  cudaFreeAsync(staging, s);
+  cudaEventRecord(pool->st_buf_done[b], s);
   return st;
 }
 
@@ -450,7 +473,7 @@ void free_pool(lv_pool* pool) {
   if (pool->s_unpack) cudaStreamSynchronize(pool->s_unpack);
   if (pool->s_unpack) cudaStreamDestroy(pool->s_unpack);
   for (cudaEvent_t e : {pool->ev_st_d2h, pool->ev_st_h2d, pool->ev_st_unpack, pool->ev_st_packed,
-                        pool->ev_st_done})
+                        pool->ev_st_done, pool->st_buf_done[0], pool->st_buf_done[1]})
     if (e) cudaEventDestroy(e);
   if (pool->s_copy) cudaStreamSynchronize(pool->s_copy);
   if (pool->s_copy) cudaStreamDestroy(pool->s_copy);
@@ -469,6 +492,8 @@ void free_pool(lv_pool* pool) {
     cudaEventDestroy(e.start);
     cudaEventDestroy(e.end);
   }
+  for (void* b : pool->st_buf)
+    if (b) cudaFree(b);   // after every stream above has been synchronised
   for (void* p : pool->dev_allocs) cudaFree(p);
   pool->dev_allocs.clear();
   if (pool->own_host && pool->host_base) cudaFreeHost(pool->host_base);
@@ -649,7 +674,9 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       cudaEventCreateWithFlags(&pool->ev_st_h2d, cudaEventDisableTiming) != cudaSuccess ||
       cudaEventCreateWithFlags(&pool->ev_st_unpack, cudaEventDisableTiming) != cudaSuccess ||
       cudaEventCreateWithFlags(&pool->ev_st_packed, cudaEventDisableTiming) != cudaSuccess ||
-      cudaEventCreateWithFlags(&pool->ev_st_done, cudaEventDisableTiming) != cudaSuccess)
+      cudaEventCreateWithFlags(&pool->ev_st_done, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&pool->st_buf_done[0], cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&pool->st_buf_done[1], cudaEventDisableTiming) != cudaSuccess)
     return fail(LV_ERR_CUDA);
   pool->tasks_host_cap = (size_t)d.budget + d.maxB + (size_t)d.host_pages;
   pool->st_loaded.resize(d.hbm_pages);
