@@ -646,11 +646,12 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       cudaMemsetAsync(d.ctl, 0, lv::C_N * sizeof(long long), s) != cudaSuccess ||
       cudaMemsetAsync(d.page_tag, 0, (size_t)d.hbm_pages * 8, s) != cudaSuccess)
     return fail(LV_ERR_CUDA);
-  // A third of the SMs keeps both link directions saturated (341 GB/s on GB300, the
-  // same as one CTA per SM) and leaves the rest of the GPU to the serving work that
-  // runs meanwhile: next to a consumer reading resident KV at HBM speed, 48 CTAs
-  // moved 208 GB/s and left it 0.83 of its rate, against 167 GB/s and 0.67 for 152.
-  pool->exchange_ctas = pool->num_sms / 3 > 0 ? pool->num_sms / 3 : 1;
+  // A fifth of the SMs (30 CTAs on GB300) keeps both link directions saturated (338 GB/s,
+  // the same as 50 CTAs or one per SM; 25 CTAs fall to 326) and leaves the rest of the
+  // GPU to the serving work that runs meanwhile: next to a consumer reading resident KV
+  // at HBM speed, 30 CTAs moved 211 GB/s and left it 0.88 of its rate, against 197 GB/s
+  // and 0.835 for 50 CTAs and 167 GB/s and 0.67 for 152.
+  pool->exchange_ctas = pool->num_sms / 5 > 0 ? pool->num_sms / 5 : 1;
   if (const char* env = std::getenv("LV_EXCHANGE_CTAS_PER_SM")) {
     const int per = std::atoi(env);
     if (per >= 1 && per <= 16) pool->exchange_ctas = pool->num_sms * per;
