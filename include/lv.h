@@ -705,6 +705,7 @@ typedef struct lv_controller_record {
 typedef struct lv_controller_counters {
   int64_t admitted, completed, waited, given_up, cancelled, hits, victims, pages_in;
 } lv_controller_counters;
+/* A controller over `pool` (one per pool).  LV_ERR_INVALID for a bad descriptor. */
 lv_status lv_controller_create(lv_pool* pool, const lv_controller_desc* d, lv_controller** out);
 /* Cancels pending preloads (their reservations are released) and frees the
    controller; call it before lv_pool_destroy of its pool. */
@@ -719,9 +720,12 @@ lv_status lv_controller_turn_loaded(lv_controller* c, int64_t now_us, int64_t pa
 lv_status lv_controller_records(lv_controller* c, lv_controller_record* records, int64_t capacity,
                                 int64_t* n_records, int32_t* data, int64_t data_capacity,
                                 int64_t* n_data);
+/* The controller's counters since it was created (host memory). */
 lv_status lv_controller_counters_get(lv_controller* c, lv_controller_counters* out);
 
+/* A static, human-readable name of a status. */
 const char* lv_status_str(lv_status s);
+/* The library's interface version (1 for this header). */
 int32_t lv_version(void);
 
 #ifdef __cplusplus
