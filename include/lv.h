@@ -725,7 +725,9 @@ lv_status lv_controller_counters_get(lv_controller* c, lv_controller_counters* o
 
 /* A static, human-readable name of a status. */
 const char* lv_status_str(lv_status s);
-/* The library's interface version (1 for this header). */
+/* The library's interface version: LV_VERSION of the header it was built with.  A
+   caller built against another header must not use the library. */
+#define LV_VERSION 2
 int32_t lv_version(void);
 
 #ifdef __cplusplus

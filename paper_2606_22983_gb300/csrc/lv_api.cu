@@ -1474,6 +1474,6 @@ const char* lv_status_str(lv_status s) {
   return "LV_ERR_UNKNOWN";
 }
 
-int32_t lv_version(void) { return 1; }
+int32_t lv_version(void) { return LV_VERSION; }
 
 }  // extern "C"

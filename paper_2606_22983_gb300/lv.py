@@ -31,6 +31,7 @@ LV_SELECT_FALLBACK = 1
 LV_POLICY_NEXT_USE, LV_POLICY_LRU = 0, 1
 LV_TIERS_EXCLUSIVE, LV_TIERS_INCLUSIVE = 0, 1
 LV_RESIDENT_ASYNC_COPY = 2
+LV_VERSION = 2                     # include/lv.h
 LV_MODE_ASYNC = 16
 LV_RUNNING, LV_IMMEDIATE, LV_RESP_OPEN, LV_DONE_VALID = 1, 2, 4, 8
 (LV_EV_TURN_BEGIN, LV_EV_TURN_END, LV_EV_PLAYBACK, LV_EV_SPEECH_START, LV_EV_BARGE_IN,
@@ -203,6 +204,9 @@ def _load():
     lib.lv_status_str.restype = ctypes.c_char_p
     lib.lv_version.argtypes = []
     lib.lv_version.restype = i32
+    if lib.lv_version() != LV_VERSION:
+        raise ImportError(f"{LIB_PATH} implements interface version {lib.lv_version()}, this "
+                          f"binding version {LV_VERSION}: rebuild it")
     return lib
 
 

@@ -41,6 +41,10 @@ def test_binding_names_match_header():
     assert sorted(lv.EXPORTED) == _declared_functions()
     for n in lv.EXPORTED:
         assert callable(getattr(lv, n)), n
+    import re
+    with open(HEADER) as f:
+        m = re.search(r"#define LV_VERSION (\d+)", f.read())
+    assert m and int(m.group(1)) == lv.LV_VERSION
 
 
 def test_struct_layouts_match_header(tmp_path):
@@ -140,7 +144,7 @@ def test_status_strings_and_argument_checks(lib):
     from paper_2606_22983_gb300 import lv
     for code, name in lv.STATUS_NAMES.items():
         assert lv.lv_status_str(code) == name
-    assert lv.lv_version() >= 1
+    assert lv.lv_version() == lv.LV_VERSION == 2
     # argument checks that need no device: a NULL descriptor / NULL out pointer
     L = lv.lib()
     h = ctypes.c_void_p()
