@@ -51,6 +51,18 @@ def _event(kind, sid, t, a=0, b=0):
     return e
 
 
+def load_keys(order_fn, order_key, n_blocks):
+    """Per-block keys (uint64 [n_blocks]) whose ascending order is ``order_fn(order_key,
+    blocks)`` for any set of blocks: the rank of each block in the order of all of them.
+    ``order_fn`` must order blocks by a key of each block alone (ties by block id), as the
+    workloads' scatter order does; then its order of any subset is the subset's order in
+    the whole."""
+    perm = np.asarray(order_fn(order_key, np.arange(n_blocks)), dtype=np.int64)
+    keys = np.empty(n_blocks, dtype=np.uint64)
+    keys[perm] = np.arange(n_blocks, dtype=np.uint64)
+    return keys
+
+
 class KVManager:
     def __init__(self, pool: KVPool, perms=None, on_append=None, rank_on="none", admit=None,
                  mode=lv.LV_MODE_AUTO, record=True, driver="device", order_fn=None,
@@ -144,14 +156,7 @@ class KVManager:
         return status
 
     def _load_keys(self, order_key):
-        """Per-block keys whose ascending order is ``order_fn(order_key, blocks)`` for any
-        set of blocks: the rank of each block in the order of all of them (``order_fn``
-        orders blocks by a key of the block alone, as the workloads' scatter order does)."""
-        nb = self.pool.max_blocks
-        perm = np.asarray(self.order_fn(order_key, np.arange(nb)), dtype=np.int64)
-        keys = np.empty(nb, dtype=np.uint64)
-        keys[perm] = np.arange(nb, dtype=np.uint64)
-        return keys
+        return load_keys(self.order_fn, order_key, self.pool.max_blocks)
 
     def _device_turn(self, sid, row, now_us, append_tokens, reply_us, reply_units, rec,
                      load_keys=None):

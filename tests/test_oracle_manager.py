@@ -84,6 +84,26 @@ def test_workload_scripts_are_deterministic_and_ordered():
     assert int(t.meta["total_pages"]) >= t.spec.hbm_budget_pages + t.spec.max_blocks
 
 
+def test_load_keys_reproduce_the_scatter_order_of_any_subset():
+    """The device driver passes a scattered reload order as per-block keys: for every
+    subset of blocks, ascending (key, block id) must be the scatter order the oracle
+    uses for that subset."""
+    from paper_2606_22983_gb300 import build
+    build()                      # the manager module loads liblv (no GPU call)
+    from paper_2606_22983_gb300.manager import load_keys
+    from workloads import scatter_order
+    rng = np.random.default_rng(4)
+    for trial in range(40):
+        nb = int(rng.integers(1, 300))
+        key = int(rng.integers(0, 1 << 40))
+        keys = load_keys(scatter_order, key, nb)
+        assert sorted(keys.tolist()) == list(range(nb))
+        sub = np.sort(rng.choice(nb, size=int(rng.integers(0, nb + 1)), replace=False))
+        want = scatter_order(key, sub)
+        got = sub[np.lexsort((sub, keys[sub]))]
+        assert np.array_equal(got, want), (trial, nb)
+
+
 def test_content_numpy_and_torch_agree():
     import torch
     from workloads import TINY_SHAPE, THINKER_SHAPE, subpage_values_torch
