@@ -628,8 +628,8 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
   if (cudaDeviceGetStreamPriorityRange(&prio_least, &prio_greatest) != cudaSuccess) prio_greatest = 0;
   if (cudaStreamCreateWithPriority(&pool->s_copy, cudaStreamNonBlocking, prio_greatest) != cudaSuccess ||
       cudaEventCreateWithFlags(&pool->ev_planned, cudaEventDisableTiming) != cudaSuccess ||
-      cudaEventCreate(&pool->ev_copy_start) != cudaSuccess ||
-      cudaEventCreate(&pool->ev_copy_end) != cudaSuccess ||
+      cudaEventCreateWithFlags(&pool->ev_copy_start, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&pool->ev_copy_end, cudaEventDisableTiming) != cudaSuccess ||
       cudaEventCreateWithFlags(&pool->ev_copied[0], cudaEventDisableTiming) != cudaSuccess ||
       cudaEventCreateWithFlags(&pool->ev_copied[1], cudaEventDisableTiming) != cudaSuccess)
     return fail(LV_ERR_CUDA);

@@ -88,9 +88,9 @@ struct CopyOffload {
   cudaStream_t stream;
   cudaEvent_t planned;
   cudaEvent_t copied;
-  // timing events recorded on `stream` just before and just after the copy kernel when
-  // the timing instrument is off (it records its own pair there when on): measured, the
-  // asynchronous turns run at 338 GB/s with a pair there and at 316 GB/s without one
+  // events recorded on `stream` just before and just after the copy kernel when the timing
+  // instrument is off (it records its own pair there when on): measured, the asynchronous
+  // turns run at 334-338 GB/s with a pair there (timing or not) and at 316 GB/s without one
   cudaEvent_t started;
   cudaEvent_t finished;
 };
