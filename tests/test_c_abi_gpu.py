@@ -1,7 +1,8 @@
 """The C ABI used from C alone (no Python, no PyTorch): a program linked against
 liblv.so and the CUDA runtime creates a pool over its own cudaMalloc'd KV arrays,
 ranks, swaps out, commits, checks the bytes in the host pool, reloads and checks
-the bytes in HBM."""
+the bytes in HBM; then frees pages with lv_evict and runs one lv_turn whose load
+keys set the reload order."""
 import os
 import subprocess
 
@@ -107,6 +108,39 @@ int main(void) {
   CHECK(lv_read_tables(pool, tables, NULL, NULL, NULL));
   CHECK(lv_sync(pool, NULL));
   if (tables[0] != 10 || tables[1] != 0 || tables[2] != 1 || tables[3] != 2) { printf("tables\n"); return 1; }
+
+  /* free 2 pages now on the device: the suffix of session 0 (session 1 runs) */
+  static lv_victim ev[PAGES];
+  static int32_t evs[PAGES];
+  lv_resident_result res;
+  CHECK(lv_evict(pool, 0, 2, 0, ev, evs, &res, NULL));
+  CHECK(lv_sync(pool, NULL));
+  if (res.status != LV_RESIDENT_DONE || res.n_victims != 2 || ev[0].sid != 0 || ev[0].blk != 3 ||
+      ev[1].blk != 2 || evs[0] != 0 || evs[1] != 1) { printf("evict\n"); return 1; }
+
+  /* one turn of session 0 whose load keys reverse its host blocks: block 3 loads first and
+     takes the lowest free page (1), block 2 the next (2) */
+  static uint64_t keys[MAXB];
+  for (int b = 0; b < MAXB; ++b) keys[b] = (uint64_t)(MAXB - b);
+  lv_turn_desc td;
+  memset(&td, 0, sizeof td);
+  td.sid = 0; td.now_us = 10; td.reply_audio_us = 1000; td.reply_units = 1; td.load_keys = keys;
+  int32_t tblocks[MAXB], tpages[MAXB];
+  CHECK(lv_turn(pool, &td, NULL, NULL, tblocks, tpages, NULL, &res, NULL));
+  CHECK(lv_sync(pool, NULL));
+  if (res.status != LV_RESIDENT_DONE || res.n_loaded != 2 || res.sid != 0 || tblocks[0] != 3 ||
+      tblocks[1] != 2 || tpages[0] != 1 || tpages[1] != 2) { printf("turn\n"); return 1; }
+  for (int i = 0; i < 2; ++i) {
+    for (int j = 0; j < J; ++j) {
+      CUDA(cudaMemcpy(sub, kv[j] + (size_t)tpages[i] * P, P, cudaMemcpyDeviceToHost));
+      const uint8_t want = (uint8_t)(((10 + tblocks[i]) * 2 + j + 1) & 255);   /* block b began on page 10+b */
+      for (size_t b = 0; b < P; ++b)
+        if (sub[b] != want) { printf("turn byte %d/%d/%zu\n", i, j, b); return 1; }
+    }
+  }
+  CHECK(lv_read_tables(pool, tables, NULL, NULL, NULL));
+  CHECK(lv_sync(pool, NULL));
+  if (tables[0] != 10 || tables[1] != 0 || tables[2] != 2 || tables[3] != 1) { printf("tables 2\n"); return 1; }
   CHECK(lv_pool_destroy(pool, NULL));
   for (int j = 0; j < J; ++j) CUDA(cudaFree(kv[j]));
   printf("ok\n");
