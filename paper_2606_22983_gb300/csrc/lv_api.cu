@@ -5,6 +5,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <new>
+#include <deque>
 #include <vector>
 
 #include <nvtx3/nvToolsExt.h>
@@ -86,7 +87,8 @@ struct lv_pool {
   // copy-kernel timing (lv_timing_enable): event pairs recorded per kind, reused
   bool timing = false;
   std::vector<lv::EventPair> ev_free;
-  std::vector<lv::EventPair> ev_used[LV_TIMING_KINDS];
+  // a deque: the pointer timing_pair returns stays valid while later pairs are added
+  std::deque<lv::EventPair> ev_used[LV_TIMING_KINDS];
   bool own_host = false;
   void* host_base = nullptr;       // host-visible address of the host pool
   std::vector<void*> dev_allocs;
