@@ -35,6 +35,11 @@
  * by a copy queued on the stream: read it after the stream has completed.
  * Calls that allocate from the same tier (swap-out: host slots; swap-in and
  * append: HBM pages) must be ordered with respect to each other.
+ *
+ * Threads.  A pool keeps host-side state (scratch alternation, pending
+ * asynchronous copies, staging runs, timing records): calls on one pool must
+ * not run concurrently from several host threads.  Distinct pools are
+ * independent, and so is one pool per GPU.
  */
 #ifndef LV_H
 #define LV_H
