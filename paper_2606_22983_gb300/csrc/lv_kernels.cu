@@ -614,32 +614,37 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
   const bool sid_ok = sid >= 0 && sid < p.S;
   const int32_t nb_in = sid_ok ? nblocks_of(p, sid) : 0;
   // validation: every victim is resident where it says, every incoming block is in
-  // the host tier, and no block appears twice
-  for (long long i = threadIdx.x; i < n_out; i += kPlanThreads) {
-    const lv_victim x = v[i];
-    bool ok = x.sid >= 0 && x.sid < p.S && x.blk >= 0 && x.page >= 0 && x.page < p.hbm_pages;
-    ok = ok && x.blk < nblocks_of(p, x.sid);
-    ok = ok && p.table[(size_t)x.sid * p.maxB + x.blk] == x.page &&
-         p.own_hbm[x.page] == owner_key(x.sid, x.blk);
-    ok = ok && atomicExch(&p.mark[(size_t)x.sid * p.maxB + x.blk], epoch) != epoch;
-    if (!ok) { set_error(p.ctl, LV_ERR_STATE, i); bad = 1; }
-  }
-  for (long long i = threadIdx.x; i < n_in; i += kPlanThreads) {
-    const int32_t b = blks[i];
-    bool ok = sid_ok && b >= 0 && b < nb_in;
-    if (ok) {
-      const int32_t e = p.table[(size_t)sid * p.maxB + b];
-      const long long h = -(long long)e - 2;
-      ok = e <= -2 && h < p.host_pages && p.own_host[h] == owner_key(sid, b);
-      ok = ok && atomicExch(&p.mark[(size_t)sid * p.maxB + b], epoch) != epoch;
+  // the host tier, and no block appears twice (victims and incoming blocks side by
+  // side: item i < n_out is victim i, item n_out + i incoming block i)
+  for (long long it = threadIdx.x; it < n_out + n_in; it += kPlanThreads) {
+    if (it < n_out) {
+      const lv_victim x = v[it];
+      bool ok = x.sid >= 0 && x.sid < p.S && x.blk >= 0 && x.page >= 0 && x.page < p.hbm_pages;
+      ok = ok && x.blk < nblocks_of(p, x.sid);
+      ok = ok && p.table[(size_t)x.sid * p.maxB + x.blk] == x.page &&
+           p.own_hbm[x.page] == owner_key(x.sid, x.blk);
+      ok = ok && atomicExch(&p.mark[(size_t)x.sid * p.maxB + x.blk], epoch) != epoch;
+      if (!ok) { set_error(p.ctl, LV_ERR_STATE, it); bad = 1; }
+    } else {
+      const int32_t b = blks[it - n_out];
+      bool ok = sid_ok && b >= 0 && b < nb_in;
+      if (ok) {
+        const int32_t e = p.table[(size_t)sid * p.maxB + b];
+        const long long h = -(long long)e - 2;
+        ok = e <= -2 && h < p.host_pages && p.own_host[h] == owner_key(sid, b);
+        ok = ok && atomicExch(&p.mark[(size_t)sid * p.maxB + b], epoch) != epoch;
+      }
+      if (!ok) { set_error(p.ctl, sid_ok ? LV_ERR_STATE : LV_ERR_BOUNDS, it); bad = 1; }
     }
-    if (!ok) { set_error(p.ctl, sid_ok ? LV_ERR_STATE : LV_ERR_BOUNDS, n_out + i); bad = 1; }
   }
-  // victims without a clean copy (all of them unless the tiers are inclusive)
-  long long cnt = 0;
-  for (long long i = threadIdx.x; i < n_out; i += kPlanThreads) cnt += clean_copy_of(p, v[i]) < 0;
-  long long n_dirty;
-  block_excl_scan<kPlanThreads>(cnt, &n_dirty);
+  __syncthreads();   // every validation verdict is in `bad` before the capacity check
+  // victims without a clean copy: all of them unless the tiers are inclusive
+  long long n_dirty = n_out;
+  if (p.incl) {
+    long long cnt = 0;
+    for (long long i = threadIdx.x; i < n_out; i += kPlanThreads) cnt += clean_copy_of(p, v[i]) < 0;
+    block_excl_scan<kPlanThreads>(cnt, &n_dirty);
+  }
   if (threadIdx.x == 0 && !bad) {
     // capacity, as the sequential calls see it: host slots before any is freed,
     // HBM pages after the victims' pages are freed
