@@ -524,6 +524,23 @@ def kernel_micro(torch, pool, seed=0):
         out[name] = {"pages": n, "bytes_per_launch": 2 * payload, "avg_ms": round(ms, 4),
                      "achieved_gbs": round(gbs, 1), "peak_gbs": HBM_PEAK, "frac": round(gbs / HBM_PEAK, 3)}
     del run
+    # page checksums (an HBM-bound reader): the same scattered pages, each read once
+    sums = torch.empty(n, dtype=torch.int64, device=pool.device)
+    for _ in range(2):
+        lv.lv_page_checksums(pool.handle, pages, n, sums, pool.stream)
+    torch.cuda.synchronize()
+    c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    c0.record()
+    for _ in range(5):
+        lv.lv_page_checksums(pool.handle, pages, n, sums, pool.stream)
+    c1.record()
+    torch.cuda.synchronize()
+    assert pool.sync(raise_on_error=False) == 0
+    ms = c0.elapsed_time(c1) / 5
+    gbs = payload / (ms / 1e3) / 1e9
+    out["checksum"] = {"pages": n, "bytes_per_launch": payload, "avg_ms": round(ms, 4),
+                       "achieved_gbs": round(gbs, 1), "peak_gbs": HBM_PEAK, "frac": round(gbs / HBM_PEAK, 3)}
+    del sums
     # one urgency-scheduling round over 4096 ready requests (Algorithm 1)
     rng = np.random.default_rng(seed)
     R = lv.LV_SCHED_MAX_REQUESTS
