@@ -122,7 +122,7 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
                             unsigned long long* page_tag, cudaStream_t s, int copy_ctas,
                             const long long* counts_dev = nullptr, long long max_units = 0,
                             const EventPair* ev = nullptr, const long long* sid_dev = nullptr,
-                            const CopyOffload* off = nullptr);
+                            const CopyOffload* off = nullptr, int gate = 0);
 cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, int32_t epoch,
                          cudaStream_t s, int num_sms, int per_thread);
 cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cudaStream_t s);
@@ -147,7 +147,8 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
                                  int64_t max_load, int32_t epoch, cudaStream_t s, int copy_ctas,
                                  lv_resident_result* result, const EventPair* ev = nullptr,
                                  const long long* sid_dev = nullptr, const CopyOffload* off = nullptr,
-                                 const unsigned long long* load_keys = nullptr);
+                                 const unsigned long long* load_keys = nullptr, bool turn_end = false,
+                                 int64_t audio_us = 0, int64_t units = 0);
 // lv_turn: pick (sid < 0), LV_EV_TURN_BEGIN, make resident, LV_EV_TURN_END
 // lv_evict: rank, evict up to k victims (no loads), finish
 cudaError_t launch_evict(const DevPool& p, const ResidentScratch& rs, int64_t now_us, int64_t k,

@@ -7,7 +7,8 @@
 //             k_stage_tasks (TMA) / k_stage_tasks_lsu         (staged copy-engine path)
 //   commit    k_remap, k_cancel, k_append                    (Section 6 side tables)
 //   monitor   k_events                                       (Section 3, Sections 5.1-5.2)
-//   turn      k_resident_*, k_pick_scan, k_turn_begin/end    (a whole turn on the device)
+//   turn      k_resident_*, k_pick_scan, k_turn_begin,        (a whole turn on the device;
+//             k_order_loads, k_evict_prepare                 the gate runs in the plan)
 //   verify    k_checksum                                     (page checksums)
 //
 // The only waits are the TMA stage kernel's mbarrier waits for its own copies,
@@ -596,21 +597,73 @@ k_swap_in(DevPool p, int32_t sid, const int32_t* __restrict__ blks,
 constexpr int kPlanThreads = 1024;
 constexpr unsigned long long kPairedBit = 1ull << 31;
 
+// Words shared by the steps of one lv_make_resident call.
+enum ResWord : int {
+  R_K_SELECT = 0,   // k handed to the ranker (0 when nothing is to be evicted)
+  R_N_OUT = 1,      // victims the exchange evicts
+  R_N_IN = 2,       // host blocks the exchange loads
+  R_STATUS = 3,     // LV_RESIDENT_*
+  R_K = 4,          // pages the budget was short
+  R_GATE = 5,       // 0: the append may run
+  R_N_TASKS = 6,
+  R_APPENDED = 7,   // int32 count of appended pages, in the low half
+  R_FOUND = 8,      // victims the ranking found
+  R_SID = 9         // lv_turn: the turn's session (-1 when the pick failed)
+};
+
+// The gate after a device-driven step's ranking, run by the exchange plan's first
+// thread before it reads the counts.  GATE_RESIDENT / GATE_PRELOAD (lv_make_resident):
+// a shortfall stops the step (a preload is skipped, a foreground turn fails),
+// otherwise the exchange evicts exactly k victims.  GATE_EVICT (lv_evict): every
+// victim found is evicted; none found is LV_RESIDENT_NOTHING.
+enum { GATE_NONE = 0, GATE_RESIDENT = 1, GATE_PRELOAD = 2, GATE_EVICT = 3 };
+
+__device__ __forceinline__ void step_gate(const DevPool& p, long long* __restrict__ R, int gate) {
+  const long long found = p.ctl[C_SEL_COUNT];   // min(k, candidates)
+  if (gate == GATE_EVICT) {
+    R[R_FOUND] = found;
+    R[R_N_OUT] = found;
+    if (found == 0) R[R_STATUS] = LV_RESIDENT_NOTHING;
+    return;
+  }
+  if (R[R_STATUS] != LV_RESIDENT_DONE) return;
+  const long long k = R[R_K];
+  R[R_FOUND] = found;
+  if (found < k) {
+    if (gate == GATE_PRELOAD) {
+      R[R_STATUS] = LV_RESIDENT_SKIPPED;
+      atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PRELOADS_SKIPPED]), 1ull);
+    } else {
+      set_error(p.ctl, LV_ERR_NO_HBM, k);
+      R[R_STATUS] = LV_RESIDENT_FAILED;
+    }
+    R[R_N_OUT] = 0;
+    R[R_N_IN] = 0;
+    R[R_GATE] = 1;
+  } else {
+    R[R_N_OUT] = k;
+  }
+}
+
 __global__ void __launch_bounds__(kPlanThreads)
 k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int32_t sid,
                 const int32_t* __restrict__ blks, long long n_in, int32_t* __restrict__ slots,
                 int32_t* __restrict__ pages, int4* __restrict__ tasks, long long* n_tasks,
                 int32_t epoch, unsigned long long* __restrict__ page_tag,
-                const long long* __restrict__ counts_dev, const long long* __restrict__ sid_dev) {
+                const long long* counts_dev, const long long* __restrict__ sid_dev,
+                long long* R, int gate) {
   pdl_entry();
-  if (counts_dev) {          // counts decided on the device (lv_make_resident)
+  __shared__ int bad;
+  if (threadIdx.x == 0) {
+    bad = 0;
+    if (gate != GATE_NONE) step_gate(p, R, gate);   // a device-driven step: may set the counts
+  }
+  __syncthreads();
+  if (counts_dev) {          // counts decided on the device (lv_make_resident, lv_evict)
     n_out = counts_dev[0];
     n_in = counts_dev[1];
   }
   if (sid_dev) sid = (int32_t)*sid_dev;
-  __shared__ int bad;
-  if (threadIdx.x == 0) bad = 0;
-  __syncthreads();
   const bool sid_ok = sid >= 0 && sid < p.S;
   const int32_t nb_in = sid_ok ? nblocks_of(p, sid) : 0;
   // validation: every victim is resident where it says, every incoming block is in
@@ -1335,19 +1388,6 @@ k_append(DevPool p, int32_t sid, int32_t n_tokens, int32_t* __restrict__ pages,
 }
 
 // -------------------------------------------------------- make_resident
-// Words shared by the steps of one lv_make_resident call.
-enum ResWord : int {
-  R_K_SELECT = 0,   // k handed to the ranker (0 when nothing is to be evicted)
-  R_N_OUT = 1,      // victims the exchange evicts
-  R_N_IN = 2,       // host blocks the exchange loads
-  R_STATUS = 3,     // LV_RESIDENT_*
-  R_K = 4,          // pages the budget was short
-  R_GATE = 5,       // 0: the append may run
-  R_N_TASKS = 6,
-  R_APPENDED = 7,   // int32 count of appended pages, in the low half
-  R_FOUND = 8,      // victims the ranking found
-  R_SID = 9         // lv_turn: the turn's session (-1 when the pick failed)
-};
 
 // One CTA: sid's host-tier blocks (ascending), the deficit k and the admission.
 __global__ void __launch_bounds__(kCensusThreads)
@@ -1431,36 +1471,29 @@ k_order_loads(const long long* __restrict__ R, const int32_t* __restrict__ block
   if (lane == 0) loads[rank] = bi;
 }
 
-// After the ranking: a shortfall stops the step (a preload is skipped, a
-// foreground turn fails), otherwise the exchange evicts exactly k victims.
-__global__ void k_resident_gate(DevPool p, bool preload, long long* __restrict__ R) {
-  pdl_entry();
-  if (threadIdx.x != 0 || R[R_STATUS] != LV_RESIDENT_DONE) return;
-  const long long found = p.ctl[C_SEL_COUNT], k = R[R_K];
-  R[R_FOUND] = found;
-  if (found < k) {
-    if (preload) {
-      R[R_STATUS] = LV_RESIDENT_SKIPPED;
-      atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PRELOADS_SKIPPED]), 1ull);
-    } else {
-      set_error(p.ctl, LV_ERR_NO_HBM, k);
-      R[R_STATUS] = LV_RESIDENT_FAILED;
-    }
-    R[R_N_OUT] = 0;
-    R[R_N_IN] = 0;
-    R[R_GATE] = 1;
-  } else {
-    R[R_N_OUT] = k;
-  }
-}
 
+// The step's result and, for lv_turn (turn_end), LV_EV_TURN_END for the turn's session
+// unless its KV could not be made resident.
 __global__ void k_resident_finish(DevPool p, int32_t sid, long long now_us, bool preload,
                                   long long* __restrict__ R, lv_resident_result* __restrict__ out,
-                                  const long long* __restrict__ sid_dev) {
+                                  const long long* __restrict__ sid_dev, bool turn_end,
+                                  long long audio_us, long long units) {
   pdl_entry();
   if (threadIdx.x != 0) return;
   if (sid_dev) sid = (int32_t)*sid_dev;
   const int status = (int)R[R_STATUS];
+  if (turn_end && sid >= 0 && sid < p.S && status != LV_RESIDENT_FAILED) {
+    lv_session_state st = p.sess[sid];
+    lv_event x{};
+    x.kind = LV_EV_TURN_END;
+    x.sid = sid;
+    x.t_us = now_us;
+    x.a = audio_us;
+    x.b = units;
+    apply_event(p, st, x);
+    p.sess[sid] = st;
+    atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_EVENTS]), 1ull);
+  }
   if (preload && status == LV_RESIDENT_DONE) {
     p.sess[sid].protect_until_us = now_us + p.protect_us;   // warmed KV (Section 5.2)
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PRELOADS]), 1ull);
@@ -1480,7 +1513,7 @@ __global__ void k_resident_finish(DevPool p, int32_t sid, long long now_us, bool
 
 // ----------------------------------------------------------------- evict
 // lv_evict: up to k victims by the normal order (no fallback tier), fewer when
-// there are fewer candidates; nothing is loaded.
+// there are fewer candidates (GATE_EVICT); nothing is loaded.
 __global__ void k_evict_prepare(long long k, long long* __restrict__ R) {
   pdl_entry();
   if (threadIdx.x != 0) return;
@@ -1495,14 +1528,6 @@ __global__ void k_evict_prepare(long long k, long long* __restrict__ R) {
   R[R_SID] = -1;
 }
 
-__global__ void k_evict_gate(DevPool p, long long* __restrict__ R) {
-  pdl_entry();
-  if (threadIdx.x != 0) return;
-  const long long found = p.ctl[C_SEL_COUNT];   // min(k, candidates)
-  R[R_FOUND] = found;
-  R[R_N_OUT] = found;
-  if (found == 0) R[R_STATUS] = LV_RESIDENT_NOTHING;
-}
 
 // ------------------------------------------------------------------ turn
 // lv_turn's pick: CTA c reports whether candidate c has a block in the host tier.
@@ -1556,24 +1581,6 @@ k_turn_begin(DevPool p, int32_t sid, const int32_t* __restrict__ cand, int32_t n
   atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_EVENTS]), 1ull);
 }
 
-// LV_EV_TURN_END for the turn's session, unless its KV could not be made resident.
-__global__ void k_turn_end(DevPool p, long long now_us, long long audio_us, long long units,
-                           const long long* __restrict__ R) {
-  pdl_entry();
-  if (threadIdx.x != 0) return;
-  const long long sid = R[R_SID];
-  if (sid < 0 || sid >= p.S || R[R_STATUS] == LV_RESIDENT_FAILED) return;
-  lv_session_state st = p.sess[sid];
-  lv_event x{};
-  x.kind = LV_EV_TURN_END;
-  x.sid = (int32_t)sid;
-  x.t_us = now_us;
-  x.a = audio_us;
-  x.b = units;
-  apply_event(p, st, x);
-  p.sess[sid] = st;
-  atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_EVENTS]), 1ull);
-}
 
 // ------------------------------------------------------------- checksums
 constexpr int kSumThreads = 256;
@@ -1769,10 +1776,11 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
                             int4* tasks, long long* n_tasks, int32_t epoch,
                             unsigned long long* page_tag, cudaStream_t s, int copy_ctas,
                             const long long* counts_dev, long long max_units, const EventPair* ev,
-                            const long long* sid_dev, const CopyOffload* off) {
+                            const long long* sid_dev, const CopyOffload* off, int gate) {
+  long long* R = gate != GATE_NONE ? const_cast<long long*>(counts_dev) - R_N_OUT : nullptr;
   cudaError_t le = launch_pdl(k_exchange_plan, 1, kPlanThreads, 0, s, p, v, (long long)n_out, sid,
                               blks, (long long)n_in, slots, pages, tasks, n_tasks, epoch, page_tag,
-                              counts_dev, sid_dev);
+                              counts_dev, sid_dev, R, gate);
   if (le != cudaSuccess) return le;
   const long long units = counts_dev ? max_units : (n_out + n_in) * (long long)p.J;
   cudaStream_t cs = s;
@@ -1805,7 +1813,8 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
                                  int64_t max_load, int32_t epoch, cudaStream_t s, int copy_ctas,
                                  lv_resident_result* result, const EventPair* ev,
                                  const long long* sid_dev, const CopyOffload* off,
-                                 const unsigned long long* load_keys) {
+                                 const unsigned long long* load_keys, bool turn_end,
+                                 int64_t audio_us, int64_t units) {
   long long* R = rs.words;
   cudaError_t e = launch_pdl(k_resident_prepare, 1, kCensusThreads, 0, s, p, sid, append_tokens,
                              preload, (long long)max_load, rs.blocks, R, sid_dev);
@@ -1817,12 +1826,10 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
   }
   e = launch_select(p, now_us, 0, !preload, rs.victims, nullptr, s, 0, R + R_K_SELECT);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(k_resident_gate, 1, 32, 0, s, p, preload, R);
-  if (e != cudaSuccess) return e;
   const long long max_units = ((long long)p.budget + p.maxB) * p.J;
   e = launch_exchange(p, rs.victims, 0, sid, load_keys ? rs.loads : rs.blocks, 0, rs.slots, rs.pages,
                       rs.tasks, R + R_N_TASKS, epoch, p.page_tag, s, copy_ctas, R + R_N_OUT, max_units,
-                      ev, sid_dev, off);
+                      ev, sid_dev, off, preload ? GATE_PRELOAD : GATE_RESIDENT);
   if (e != cudaSuccess) return e;
   if (append_tokens > 0) {
     e = launch_append(p, sid, append_tokens, rs.append, reinterpret_cast<int32_t*>(R + R_APPENDED), s,
@@ -1830,7 +1837,7 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
     if (e != cudaSuccess) return e;
   }
   e = launch_pdl(k_resident_finish, 1, 32, 0, s, p, sid, (long long)now_us, preload, R, result,
-                 sid_dev);
+                 sid_dev, turn_end, (long long)audio_us, (long long)units);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
@@ -1843,15 +1850,13 @@ cudaError_t launch_evict(const DevPool& p, const ResidentScratch& rs, int64_t no
   if (e != cudaSuccess) return e;
   e = launch_select(p, now_us, 0, false, rs.victims, nullptr, s, 0, R + R_K_SELECT);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(k_evict_gate, 1, 32, 0, s, p, R);
-  if (e != cudaSuccess) return e;
   const long long max_units = (long long)p.budget * p.J;
   e = launch_exchange(p, rs.victims, 0, -1, rs.blocks, 0, rs.slots, rs.pages, rs.tasks,
                       R + R_N_TASKS, epoch, p.page_tag, s, copy_ctas, R + R_N_OUT, max_units, ev,
-                      nullptr, off);
+                      nullptr, off, GATE_EVICT);
   if (e != cudaSuccess) return e;
   e = launch_pdl(k_resident_finish, 1, 32, 0, s, p, (int32_t)-1, (long long)now_us, false, R, result,
-                 (const long long*)nullptr);
+                 (const long long*)nullptr, false, 0ll, 0ll);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
@@ -1870,11 +1875,10 @@ cudaError_t launch_turn(const DevPool& p, const ResidentScratch& rs, int32_t sid
   e0 = launch_pdl(k_turn_begin, 1, 1024, 0, s, p, sid, cand, n_cand, (const int32_t*)rs.hits,
                   (long long)now_us, R);
   if (e0 != cudaSuccess) return e0;
+  // make resident, then (in its finish kernel) LV_EV_TURN_END
   cudaError_t e = launch_make_resident(p, rs, sid, now_us, append_tokens, false, -1, epoch, s,
-                                       copy_ctas, result, ev, R + R_SID, off, load_keys);
-  if (e != cudaSuccess) return e;
-  e = launch_pdl(k_turn_end, 1, 32, 0, s, p, (long long)now_us, (long long)audio_us, (long long)units,
-                 (const long long*)R);
+                                       copy_ctas, result, ev, R + R_SID, off, load_keys, true,
+                                       audio_us, units);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
@@ -1956,7 +1960,8 @@ cudaError_t launch_exchange_plan(const DevPool& p, const lv_victim* v, int64_t n
                                  int4* tasks, long long* n_tasks, int32_t epoch,
                                  unsigned long long* page_tag, cudaStream_t s) {
   k_exchange_plan<<<1, kPlanThreads, 0, s>>>(p, v, n_out, sid, blks, n_in, slots, pages, tasks,
-                                             n_tasks, epoch, page_tag, nullptr, nullptr);
+                                             n_tasks, epoch, page_tag, nullptr, nullptr, nullptr,
+                                             (int)GATE_NONE);
   return cudaGetLastError();
 }
 
