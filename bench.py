@@ -5,11 +5,12 @@ One step = one turn of the thinker-shaped workload (48 layers, 4 KV heads x
 128, 16-token pages of 1.5 MiB, 64 sessions with log-uniform 2k-16k token
 contexts, 40 GB HBM budget): playback reports for every session, then the
 turn's session is made fully resident -- next-use ranking (census, then
-rank and top-k emission), host-slot allocation, swap-out, commit, HBM-page allocation, swap-in,
-commit.  ``value`` is the payload moved over the host link in both
+rank and top-k emission), host-slot allocation, swap-out, commit, HBM-page
+allocation, swap-in, commit -- in one lv_turn with no host round trip.  ``value`` is the payload moved over the host link in both
 directions per second (GB/s, 1e9 B) with every input resident before timing;
-``e2e`` is the same through the C ABI with host buffers (event batches copied
-in, victim / slot / page lists read back every step).
+``e2e`` is the same through the C ABI with host buffers (every step copies its
+event batch in from page-locked host memory and reads the turn's result back
+into it), timed on the host clock.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
