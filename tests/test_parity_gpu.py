@@ -134,6 +134,21 @@ def test_mixed_realtime_full_size():
     assert om.counters["preloads"] > 50 and om.counters == gm.counters
 
 
+def test_mixed_realtime_full_size_async_copies():
+    """The mixed workload with every turn's and preload's copy left running on the pool's
+    copy stream (turns, preloads and growth overlap earlier copies): the end state and
+    sampled bytes equal the oracle's."""
+    om, gm = _sampled_full_size(make_workload("mixed", 1), "device", 0, record=False,
+                                async_copy=True)
+
+
+def test_long_multimodal_full_size_pipelined_staged():
+    """The long workload's multi-GB turns through the copy-engine path with pipelined
+    (asynchronous) staged exchanges: the staging runs grow to several GB and are reused
+    by alternate calls.  The end state and sampled bytes equal the oracle's."""
+    _sampled_full_size(make_workload("long", 1), "exchange", 2, record=False, async_copy=True)
+
+
 def test_long_multimodal_full_size():
     """16 sessions of 32k-64k tokens (3-6 GB each, 30 % frame tokens); every turn
     evicts and reloads several GB at once through the exchange."""
