@@ -156,11 +156,14 @@ def test_long_multimodal_full_size():
     assert om.counters["pages_in"] > 16 * 1000
 
 
-@pytest.mark.parametrize("driver", ["exchange", "device"])
-def test_fragmentation_full_size(driver):
+@pytest.mark.parametrize("driver,async_copy", [("exchange", False), ("device", False),
+                                               ("device", True)])
+def test_fragmentation_full_size(driver, async_copy):
     """Pages randomly permuted over a 100 GB HBM budget, 640 sessions of
     256-4096 tokens; 10 000 events alternating "free k pages" with turns whose
     reload list comes in a scattered order (with the device driver, the evictions
-    run through lv_evict)."""
-    om, gm = _sampled_full_size(make_workload("frag", 0), driver, 0, rank_on="none")
+    run through lv_evict and the turns through lv_turn with load keys; with
+    asynchronous copies, nothing is read back between events)."""
+    om, gm = _sampled_full_size(make_workload("frag", 0), driver, 0, rank_on="none",
+                                record=not async_copy, async_copy=async_copy)
     assert om.counters["turns"] == 5000
