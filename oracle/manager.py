@@ -60,7 +60,7 @@ class OracleManager:
             if int(init.resp_open[s]):
                 st.flags |= se.RESP_OPEN
             self.sessions.append(st)
-        self.content = content        # (seed, value table) used to write KV bytes
+        self.content = content        # (seed, value table) or "tagged": how KV bytes are made
         self.admit = admit
         self.rank_on = rank_on          # 'all' events, 'turns' only, or 'none'
         self.counters = dict(victims=0, pages_out=0, pages_in=0, preloads=0,
@@ -70,12 +70,17 @@ class OracleManager:
 
     # ------------------------------------------------------------ content
     def _subpage_content(self, sid, blk, ctx):
-        from workloads.content import subpage_offsets, subpage_values_np, valid_rows
-        seed, table = self.content
+        from workloads.content import (subpage_offsets, subpage_values_np, tagged_values_np,
+                                       valid_rows)
         sh = self.shape
         J = 2 * sh.layers
         layer = np.arange(J) // 2
         kv = np.arange(J) % 2
+        if self.content == "tagged":      # address-tagged chunks (a debugging mode)
+            rows = np.full(J, int(valid_rows(ctx, blk, sh)))
+            return tagged_values_np(np.full(J, sid), np.full(J, blk), layer, kv, rows,
+                                    sh).view(np.uint8).reshape(J, sh.subpage_bytes)
+        seed, table = self.content
         off = subpage_offsets(seed, np.full(J, sid), np.full(J, blk), layer, kv, sh)
         rows = np.full(J, int(valid_rows(ctx, blk, sh)))
         return subpage_values_np(table, off, rows, sh).view(np.uint8).reshape(J, sh.subpage_bytes)

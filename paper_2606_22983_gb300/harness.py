@@ -9,7 +9,8 @@ from __future__ import annotations
 import numpy as np
 import torch
 
-from workloads.content import subpage_offsets, subpage_values_torch, valid_rows, value_table
+from workloads.content import (subpage_offsets, subpage_values_torch, tagged_values_torch,
+                               valid_rows, value_table)
 
 from . import lv
 from .pool import KVPool
@@ -47,15 +48,19 @@ def pool_for(workload, device=None, stream=None, kv=None) -> KVPool:
 class ContentWriter:
     """Writes tagged KV contents into a pool's HBM arrays and host pool."""
 
-    def __init__(self, pool: KVPool, workload, seed=None, chunk=2048):
+    def __init__(self, pool: KVPool, workload, seed=None, chunk=2048, tagged=False):
         self.pool = pool
         self.shape = workload.spec.shape
         self.seed = workload.seed if seed is None else seed
-        self.table_np = value_table(self.seed)
-        self.table = torch.from_numpy(self.table_np.view(np.int16)).to(pool.device)
+        self.tagged = tagged            # address-tagged chunks instead of seeded values
+        if not tagged:
+            self.table_np = value_table(self.seed)
+            self.table = torch.from_numpy(self.table_np.view(np.int16)).to(pool.device)
         self.chunk = chunk
 
     def _values(self, sids, blks, layer, kv, rows):
+        if self.tagged:
+            return tagged_values_torch(sids, blks, layer, kv, rows, self.shape, self.pool.device)
         off = subpage_offsets(self.seed, sids, blks, np.full(len(sids), layer),
                               np.full(len(sids), kv), self.shape)
         return subpage_values_torch(self.table, torch.from_numpy(off).to(self.pool.device),

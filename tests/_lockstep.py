@@ -55,19 +55,35 @@ def compare_state(om: OracleManager, pool, where, with_bytes):
         assert np.array_equal(gs[f].astype(np.int64), oa[f]), (where, f)
     if with_bytes:
         hbm = pool.kv.cpu().numpy()
-        assert np.array_equal(hbm, om.pool.hbm), (where, "hbm bytes")
-        assert np.array_equal(pool.host, om.pool.host), (where, "host bytes")
+        assert np.array_equal(hbm, om.pool.hbm), (where, "hbm bytes", _first_difference(hbm, om.pool.hbm))
+        assert np.array_equal(pool.host, om.pool.host), (where, "host bytes",
+                                                         _first_difference(pool.host, om.pool.host))
 
 
-def make_pair(workload, with_bytes, rank_on="all", mode=lv.LV_MODE_AUTO, driver="device"):
+def _first_difference(got, want):
+    """Where two byte images first differ, with both 16-byte chunks decoded as
+    address tags (meaningful when the contents are address-tagged)."""
+    from workloads.content import decode_tag
+    g, w = np.ascontiguousarray(got).reshape(-1), np.ascontiguousarray(want).reshape(-1)
+    bad = np.nonzero(g != w)[0]
+    if not bad.size:
+        return None
+    at = int(bad[0]) // 16 * 16
+    return {"byte": int(bad[0]), "got (sid, token, layer, kv, chunk)": decode_tag(g[at:at + 16]),
+            "want": decode_tag(w[at:at + 16])}
+
+
+def make_pair(workload, with_bytes, rank_on="all", mode=lv.LV_MODE_AUTO, driver="device",
+              tagged=False):
     seed = workload.seed
-    table = value_table(seed)
-    om = OracleManager(workload, with_bytes=with_bytes, content=(seed, table) if with_bytes else None,
-                       rank_on=rank_on)
+    content = None
+    if with_bytes:
+        content = "tagged" if tagged else (seed, value_table(seed))
+    om = OracleManager(workload, with_bytes=with_bytes, content=content, rank_on=rank_on)
     pool = pool_for(workload)
     writer = None
     if with_bytes:
-        writer = ContentWriter(pool, workload)
+        writer = ContentWriter(pool, workload, tagged=tagged)
         zero_host(pool)
         writer.write_initial(workload)
     gm = KVManager(pool, perms=workload.perms,
@@ -77,8 +93,8 @@ def make_pair(workload, with_bytes, rank_on="all", mode=lv.LV_MODE_AUTO, driver=
 
 
 def run_lockstep(workload, with_bytes=True, check_every=50, n_events=None, rank_on="all",
-                 mode=lv.LV_MODE_AUTO, driver="device"):
-    om, pool, gm = make_pair(workload, with_bytes, rank_on, mode, driver)
+                 mode=lv.LV_MODE_AUTO, driver="device", tagged=False):
+    om, pool, gm = make_pair(workload, with_bytes, rank_on, mode, driver, tagged)
     n = workload.n_events if n_events is None else n_events
     try:
         compare_state(om, pool, "initial", with_bytes)

@@ -26,6 +26,16 @@ def test_tiny_workload_full_images(seed, driver, mode):
     assert gm.counters["pages_out"] > 500 and gm.counters["preloads"] > 10
 
 
+@pytest.mark.parametrize("driver,mode", [("device", 0), ("exchange", 2)])
+def test_tiny_workload_address_tagged_bytes(driver, mode):
+    """The tiny script with address-tagged KV contents (every 16-byte chunk holds its
+    session, token, layer, K/V and chunk): full byte images after every 25 events, so a
+    misplaced byte would be reported with where it came from."""
+    wl = make_workload("tiny", 5)
+    om, gm = run_lockstep(wl, with_bytes=True, check_every=25, driver=driver, mode=mode, tagged=True)
+    assert om.counters == gm.counters and gm.counters["pages_out"] > 300
+
+
 @pytest.mark.parametrize("driver", ["device", "sequential"])
 def test_tiny_workload_lru_baseline(driver):
     """The LRU baseline policy on the same kernels (NEXT f3): every ranking and

@@ -88,3 +88,54 @@ def subpage_values_torch(table_t, offsets_t, rows_t, shape: KVShape):
     tok = ar // shape.row_elems
     out.masked_fill_(tok[None, :] >= rows_t[:, None], 0)
     return out
+
+
+# ------------------------------------------------------------- address-tagged content
+# A debugging mode: every 16-byte chunk of a sub-page holds where it belongs, as four
+# little-endian uint32 words (sid, token = blk * T + row, 2 * layer + kv, chunk within
+# the row), so a byte found in the wrong place says which token, layer and chunk it
+# is.  Rows past the context end are zero, as in the seeded mode.  Needs token rows
+# of a multiple of 16 bytes.
+
+def tagged_values_np(sid, blk, layer, kv, rows, shape: KVShape) -> np.ndarray:
+    """uint16 [n, T*H*D] address-tagged contents of n sub-pages (host)."""
+    sid = np.atleast_1d(np.asarray(sid, dtype=np.uint32))
+    n = sid.size
+    blk = np.broadcast_to(np.asarray(blk, dtype=np.uint32), (n,))
+    jj = np.broadcast_to(np.asarray(layer, dtype=np.uint32) * 2 + np.asarray(kv, dtype=np.uint32), (n,))
+    rows = np.broadcast_to(np.asarray(rows, dtype=np.int64), (n,))
+    T = shape.page_tokens
+    cpr = shape.row_elems * shape.elem_bytes // 16           # chunks per token row
+    assert cpr * 16 == shape.row_elems * shape.elem_bytes
+    w = np.zeros((n, T, cpr, 4), dtype=np.uint32)
+    w[..., 0] = sid[:, None, None]
+    w[..., 1] = blk[:, None, None] * np.uint32(T) + np.arange(T, dtype=np.uint32)[None, :, None]
+    w[..., 2] = jj[:, None, None]
+    w[..., 3] = np.arange(cpr, dtype=np.uint32)[None, None, :]
+    w[np.arange(T)[None, :] >= rows[:, None]] = 0
+    return w.reshape(n, -1).view(np.uint16).reshape(n, shape.subpage_elems)
+
+
+def tagged_values_torch(sid, blk, layer, kv, rows, shape: KVShape, device):
+    """int16 [n, T*H*D]: the same contents built on ``device``."""
+    import torch
+    as_t = lambda a: torch.as_tensor(np.asarray(a, dtype=np.int64), device=device)
+    sid, blk, rows = as_t(sid), as_t(blk), as_t(rows)
+    jj = as_t(np.asarray(layer) * 2 + np.asarray(kv)).expand(sid.shape[0])
+    n = sid.shape[0]
+    T = shape.page_tokens
+    cpr = shape.row_elems * shape.elem_bytes // 16
+    tok = torch.arange(T, device=device, dtype=torch.int64)
+    w = torch.zeros((n, T, cpr, 4), dtype=torch.int64, device=device)
+    w[..., 0] = sid[:, None, None]
+    w[..., 1] = blk[:, None, None] * T + tok[None, :, None]
+    w[..., 2] = jj[:, None, None]
+    w[..., 3] = torch.arange(cpr, device=device, dtype=torch.int64)[None, None, :]
+    w.masked_fill_((tok[None, :] >= rows[:, None])[:, :, None, None], 0)
+    return w.to(torch.int32).reshape(n, -1).view(torch.int16).reshape(n, shape.subpage_elems)
+
+
+def decode_tag(chunk16: bytes):
+    """(sid, token, layer, kv, chunk) of a 16-byte address-tagged chunk."""
+    w = np.frombuffer(bytes(chunk16), dtype="<u4")
+    return int(w[0]), int(w[1]), int(w[2]) // 2, int(w[2]) % 2, int(w[3])
