@@ -193,7 +193,7 @@ typedef struct lv_stats {
   int64_t error_detail;        /* index of the offending item */
   int64_t last_select_count;   /* victims written by the last lv_select_victims */
   int64_t last_select_total;   /* candidates it saw */
-  /* counters ("counters for policy fallbacks and preload outcomes", Section 6) */
+  /* counters of policy fallbacks and of preload outcomes (Section 6) */
   int64_t selects, victims, shortfalls, pages_out, pages_in, bytes_out, bytes_in;
   int64_t remap_entries, appended_pages, cancels, events, fallback_selects;
   int64_t preloads, preloads_skipped;   /* lv_make_resident with LV_RESIDENT_PRELOAD */
@@ -314,7 +314,7 @@ lv_status lv_swap_in(lv_pool* pool, int32_t sid, const int32_t* blks, int64_t n,
                      int32_t* pages_out, lv_remap_entry* commit_out, int32_t mode,
                      lv_stream stream);
 
-/* Section 5.1 (evict "until enough HBM is released") followed by the load of
+/* Section 5.1 (evict until enough HBM is free) followed by the load of
    Section 5.2 / Section 6, as one step: evicts n_out victims to the host tier
    and loads n_in host-resident blocks of session sid, committing both.  The
    result -- slots_out (int32 [n_out], victim order), pages_out (int32 [n_in],

@@ -41,6 +41,9 @@ EV_TURN_SCATTER, EV_EVICT = 7, 8
 
 
 class OracleManager:
+    """The KV manager of Section 5 over an event script: turns make their session
+    resident (Section 5.1 eviction, Section 6 loading), speech start and barge-in
+    trigger preloads (Section 5.2), monitor events update the sessions (Section 3)."""
     def __init__(self, workload, with_bytes=True, content=None, admit=None, rank_on="all"):
         spec = workload.spec
         sh = spec.shape
@@ -113,6 +116,8 @@ class OracleManager:
 
     # ------------------------------------------------------------- ranking
     def full_order(self, now_us):
+        """The whole victim order at now_us: Section 5.1 (Eq. 4 keys), or the LRU
+        baseline of Sections 2.3 and 5."""
         sp = self.spec
         if sp.policy == LRU:
             return order_lru(self.pool.tables, self.pool.nblocks, self.sessions, sp.within_order)
@@ -120,6 +125,8 @@ class OracleManager:
                             sp.t_play_mode, sp.reply_prior_us, sp.unit_us, sp.within_order)
 
     def select(self, now_us, k, fallback=False):
+        """The first k victims of the order (Section 5.1); with ``fallback`` the
+        protected, non-running tier follows the normal one (Section 5.2)."""
         sp = self.spec
         if sp.policy == LRU:
             s_, b_, p_ = order_lru(self.pool.tables, self.pool.nblocks, self.sessions, sp.within_order)
@@ -131,6 +138,10 @@ class OracleManager:
 
     # ------------------------------------------------------------ movement
     def make_resident(self, sid, now_us, append_tokens, foreground, rec, order_key=None):
+        """Make session sid fully resident, then grow it: evict exactly the deficit in
+        the Section 5.1 order, load the host blocks (Sections 5.2 and 6; block order, or
+        the script's scattered order), allocate pages for new tokens (Section 5.1 keeps
+        block-level allocation).  False when a preload finds too few victims."""
         pool = self.pool
         host_blks = pool.host_blocks(sid)
         if order_key is not None:
@@ -173,6 +184,8 @@ class OracleManager:
         return True
 
     def preload(self, sid, now_us, rec):
+        """Speech-triggered preload of sid's host blocks (Section 5.2): admitted by
+        ``admit`` when given, skipped when too few victims, protected once complete."""
         if self.spec.policy == LRU:
             return              # the baseline loads at turn start only
         host_blks = self.pool.host_blocks(sid)
@@ -192,8 +205,9 @@ class OracleManager:
             rec["preload"] = "skipped"
 
     def evict(self, now_us, k, rec):
-        """Free k pages now (memory pressure from elsewhere): the first k of the victim
-        order, or all candidates when there are fewer."""
+        """Free k pages now (memory pressure from elsewhere): the first k of the
+        Section 5.1 victim order with normal eligibility, or all candidates when there
+        are fewer."""
         pool = self.pool
         vs, vb, vp = self.select(now_us, k)
         rec["k"] = int(k)
@@ -206,6 +220,8 @@ class OracleManager:
             self.counters["pages_out"] += int(vs.size)
 
     def turn_target(self, perm_row):
+        """The session a TURN_ANY / TURN_SCATTER event picks: the first of the script's
+        seeded order that has offloaded KV (a workload construct, not from the paper)."""
         perm = self.wl.perms[perm_row]
         for s in perm:
             if self.pool.host_blocks(int(s)).size:
@@ -214,7 +230,8 @@ class OracleManager:
 
     # --------------------------------------------------------------- events
     def step(self, i):
-        """Process script event i; returns a record of everything it decided."""
+        """Process script event i (Section 3 monitor events; the decisions of Sections
+        5.1 and 5.2); returns a record of everything it decided."""
         t, kind, sid, a, b, c, d = self.wl.event(i)
         rec = {"i": i, "t": t, "kind": kind}
         sts = self.sessions
@@ -252,11 +269,13 @@ class OracleManager:
         return rec
 
     def run(self, lo=0, hi=None):
+        """Process script events lo..hi (harness helper)."""
         hi = self.wl.n_events if hi is None else hi
         return [self.step(i) for i in range(lo, hi)]
 
     # ------------------------------------------------------------- snapshot
     def session_arrays(self):
+        """The session table as arrays (harness helper for comparisons)."""
         keys = ("ctx_tokens", "flags", "gen_us", "play_us", "t_done_us", "reply_ema_us",
                 "reply_n", "reply_tokens", "protect_until_us", "last_use_us")
         return {k: np.array([getattr(s, k) for s in self.sessions], dtype=np.int64) for k in keys}

@@ -19,7 +19,7 @@ Readings:
     unfinished responses" mean later reuse, Section 5.1); like the playback
     horizon it is never negative.
   * Protection holds against *normal* eviction only (Section 5.1), and warmed
-    KV may be "evicted before reuse" (Section 5.2).  With ``fallback`` set (a
+    KV may still be evicted before it is reused (Section 5.2).  With ``fallback`` set (a
     foreground turn that cannot otherwise run), protected sessions that are
     not running form a second tier, ordered by the same rule after every
     normally eligible block.  Pinned running KV is never a candidate.
@@ -71,7 +71,7 @@ def is_eligible(st: SessionState, now_us: int) -> bool:
 
 
 def tier(st: SessionState, now_us: int, fallback: bool):
-    """0: normally eligible; 1: protected, a candidate only with ``fallback``; None: never."""
+    """0: normally eligible; 1: protected, a candidate only with ``fallback``; None: never (Section 5.1 eligibility; Section 5.2 protection)."""
     if is_eligible(st, now_us):
         return 0
     if fallback and not (st.flags & RUNNING):
@@ -83,7 +83,7 @@ def order_lru(tables, nblocks, sessions, within=SUFFIX_FIRST):
     """The LRU baseline: every HBM-resident block of a session that is not running,
     least recently used session first (last turn time ascending, then session id
     ascending), suffix blocks first within a session.  Immediate reuse and preload
-    protection do not exist for it."""
+    protection do not exist for it (Sections 2.3 and 5)."""
     cands = [(s, st.last_use_us) for s, st in enumerate(sessions) if not (st.flags & RUNNING)]
     cands.sort(key=lambda c: (min(max(c[1], 0), KEY_MAX), c[0]))
     out_s, out_b, out_p = [], [], []
@@ -107,7 +107,7 @@ def _resident_blocks(table_row: np.ndarray, nblocks: int) -> np.ndarray:
 
 def order_global(tables, nblocks, sessions, now_us, mode, reply_prior_us, unit_us,
                  within=SUFFIX_FIRST, fallback=False):
-    """Formulation A. Returns int64 arrays (sid, blk, page) of the full victim order."""
+    """Formulation A. Returns int64 arrays (sid, blk, page) of the full victim order (Section 5.1)."""
     sids, blks, keys, tiers = [], [], [], []
     for s, st in enumerate(sessions):
         tr = tier(st, now_us, fallback)
@@ -137,7 +137,7 @@ def order_global(tables, nblocks, sessions, now_us, mode, reply_prior_us, unit_u
 
 def order_scan(tables, nblocks, sessions, now_us, mode, reply_prior_us, unit_us,
                within=SUFFIX_FIRST, k=None, fallback=False):
-    """Formulation B (the paper's session scan). Returns (sid, blk, page) lists."""
+    """Formulation B (the paper's session scan). Returns (sid, blk, page) lists (Section 5.1)."""
     elig = []
     for s, st in enumerate(sessions):
         tr = tier(st, now_us, fallback)
@@ -162,7 +162,7 @@ def order_scan(tables, nblocks, sessions, now_us, mode, reply_prior_us, unit_us,
 
 def select_victims(tables, nblocks, sessions, now_us, k, mode, reply_prior_us, unit_us,
                    within=SUFFIX_FIRST, fallback=False):
-    """The first min(k, #candidates) blocks of the victim order."""
+    """The first min(k, #candidates) blocks of the victim order (Section 5.1)."""
     sid, blk, page = order_global(tables, nblocks, sessions, now_us, mode,
                                   reply_prior_us, unit_us, within, fallback)
     k = min(int(k), sid.size)

@@ -12,7 +12,7 @@ State
 Operations follow their plain definitions:
   * allocation takes the lowest-numbered free pages / slots, in ascending
     order, and hands them out in request order; the HBM tier may hold at most
-    ``budget`` allocated pages ("keeps the block allocator", Section 5.1);
+    ``budget`` allocated pages (the block allocator is kept, Section 5.1);
   * swap-out copies every sub-page of each victim page to its host slot and
     swap-in copies every sub-page of a host slot back, one ``memcpy`` per
     sub-page; neither changes the block tables;
@@ -94,7 +94,8 @@ class OraclePool:
 
     # ---------------------------------------------------------------- set-up
     def import_placement(self, placement: np.ndarray, ctx_tokens: np.ndarray) -> None:
-        """Load an initial placement (encoded block tables) and context lengths."""
+        """Load an initial placement (encoded block tables) and context lengths (Section 6,
+        paged KV tables)."""
         S = self.S
         for s in range(S):
             self.ctx[s] = int(ctx_tokens[s])
@@ -141,14 +142,17 @@ class OraclePool:
         return got
 
     def alloc_hbm(self, n: int) -> np.ndarray:
+        """Reserve the n lowest free HBM pages within the budget (Section 5.1)."""
         return self._alloc_lowest(self.hbm_used, n, self.budget, "NO_HBM")
 
     def alloc_host(self, n: int) -> np.ndarray:
+        """Reserve the n lowest free host slots of the swap pool (Section 5.1)."""
         return self._alloc_lowest(self.host_used, n, self.host_pages, "NO_HOST")
 
     # ------------------------------------------------------------------ copy
     def swap_out(self, sid, blk, page) -> np.ndarray:
-        """Copy victim pages to freshly reserved host slots; returns the slots.
+        """Copy victim pages to freshly reserved host slots; returns the slots (Section 5,
+        the swap-out of Fig. 6).
 
         Inclusive tiers: a victim with a clean copy gets that slot and moves no
         bytes; the others reserve the lowest free slots, in victim order."""
@@ -175,7 +179,8 @@ class OraclePool:
         return slots
 
     def swap_in(self, sid: int, blks) -> np.ndarray:
-        """Copy host-resident blocks of ``sid`` into freshly reserved HBM pages."""
+        """Copy host-resident blocks of ``sid`` into freshly reserved HBM pages
+        (Sections 5.2 and 6)."""
         blks = np.asarray(blks, dtype=np.int64)
         slots = []
         for b in blks:
@@ -196,7 +201,7 @@ class OraclePool:
 
     # ----------------------------------------------------------------- remap
     def remap(self, sid, blk, new_loc) -> None:
-        """Commit (sid, blk, new location) entries in order."""
+        """Commit (sid, blk, new location) entries in order (Section 6, block-table update)."""
         seen = set()
         for s, b, e in zip(np.asarray(sid), np.asarray(blk), np.asarray(new_loc)):
             s, b, e = int(s), int(b), int(e)
@@ -244,7 +249,7 @@ class OraclePool:
         self.host_used[h] = False
 
     def cancel(self, locs) -> None:
-        """Release reservations that were never committed."""
+        """Release reservations that were never committed (Section 5.2, a cancelled preload)."""
         for e in np.asarray(locs):
             e = int(e)
             if e >= 0:
@@ -262,7 +267,7 @@ class OraclePool:
 
     # ---------------------------------------------------------------- growth
     def append(self, sid: int, n_tokens: int) -> np.ndarray:
-        """Grow a session's context; new blocks take the lowest free HBM pages."""
+        """Grow a session's context; new blocks take the lowest free HBM pages (Section 5.1)."""
         new_ctx = int(self.ctx[sid]) + int(n_tokens)
         nb = -(-new_ctx // self.T)
         if nb > self.max_blocks:
@@ -294,21 +299,26 @@ class OraclePool:
         return int(np.sum(w * weights, dtype=np.uint64))
 
     def host_blocks(self, sid: int) -> np.ndarray:
+        """Block indices of ``sid`` that live in host slots (Section 6)."""
         row = self.tables[sid, :int(self.nblocks[sid])]
         return np.nonzero(row <= -2)[0].astype(np.int64)
 
     def resident_count(self) -> int:
+        """HBM pages in use (Section 5.1, the capacity check)."""
         return int(self.hbm_used.sum())
 
     def free_budget(self) -> int:
+        """HBM pages still free under the budget (Section 5.1)."""
         return self.budget - self.resident_count()
 
     def clean_copies(self) -> int:
+        """Host slots that still hold a clean copy of a resident block (inclusive tiers,
+        a reading of Section 5)."""
         return int((self.shadow >= 0).sum())
 
     def check_invariants(self) -> None:
         """Owner tables and block tables (plus clean copies) are mutually inverse;
-        budget holds."""
+        budget holds (Section 6)."""
         n_hbm = n_host = n_clean = 0
         for s in range(self.S):
             for b in range(self.max_blocks):

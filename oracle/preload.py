@@ -8,7 +8,7 @@ reading -- parity unpinned against the paper):
     the predicted start of the session's LLM stage:
         start  = max(t, link_free_at);  finish = start + ceil(B / link_bytes_per_us)
         admit  iff finish <= t_speech + lead
-    ("enough time to hide the transfer cost under current pressure"), and only
+    (the transfer must be hidden before the turn under the current load), and only
     if the victims it must evict fit in the host tier with ``max_blocks`` slots
     still free (room for a foreground turn's synchronous eviction).  lead is
     the session's moving average of (turn start - speech start) -- integer EMA
@@ -20,8 +20,8 @@ reading -- parity unpinned against the paper):
   * An admitted preload evicts what it needs (next-use order, normal tier only)
     and reserves and copies at once, but commits only when its transfer
     completes (at the first event with time >= finish).  If the turn arrives
-    first, the reservation is cancelled and the turn loads synchronously
-    ("falls back to synchronous loading").
+    first, the reservation is cancelled and the turn loads synchronously (the
+    paper's fallback).
   * Protection and its cap: a completed preload protects the session until
     finish + protect_us; if the protected sessions' resident pages then exceed
     ``cap_pages``, the oldest protections (smallest protect_until, then lower
@@ -43,6 +43,9 @@ from .pool import _enc_host
 
 
 class PreloadController:
+    """The preload controller's constants (Section 5.2): the host link's speed, the
+    prior speech-to-turn lead and an optional cap on warmed pages."""
+
     def __init__(self, link_bytes_per_us=200_000, lead_prior_us=2_000_000, cap_pages=None):
         self.bw = int(link_bytes_per_us)
         self.lead_prior_us = int(lead_prior_us)
@@ -147,6 +150,8 @@ class ControlledOracleManager(OracleManager):
 
     # ------------------------------------------------------------- events
     def preload(self, sid, now_us, rec):
+        """A speech start (or barge-in) asks for ``sid``'s host blocks; the request waits
+        until the link can finish it before the predicted turn (Section 5.2)."""
         self.speech_t.setdefault(sid, now_us)
         if sid in self.pending or sid in self.waiting:
             return
@@ -156,6 +161,8 @@ class ControlledOracleManager(OracleManager):
         self._try_admit(sid, now_us, rec)
 
     def step(self, i):
+        """One event, with the controller's admissions, completions and lead updates
+        around it (Section 5.2)."""
         t, kind, sid, a, b, c, d = self.wl.event(i)
         pre = {}
         self._housekeeping(t, pre)

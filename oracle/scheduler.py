@@ -25,6 +25,7 @@ from fractions import Fraction
 
 
 def classify(started: bool, play_buffer_us: int, p_safe_us: int) -> int:
+    """Urgency class (Section 4.1): 0 playback at risk, 1 not yet started, 2 safe."""
     if not started:
         return 1
     return 0 if play_buffer_us <= p_safe_us else 2

@@ -7,7 +7,7 @@ KV cache manager").  This module is that state, updated one event at a time in
 event order.  Times are integer microseconds.
 
 Readings (the paper does not fix these):
-  * T_reply is "a per-session moving average" of the time from playback
+  * T_reply is a moving average, kept per session, of the time from playback
     completion to the next completed user input (Section 5.1, after Eq. 4).
     Reading: an integer exponential moving average with weight 1/4,
     ``ema <- floor((3*ema + x) / 4)``; the first sample sets ``ema = x``.
@@ -54,6 +54,8 @@ INT32_MAX = 2**31 - 1
 
 @dataclass
 class SessionState:
+    """What the interaction monitor knows about one session (Section 5.1)."""
+
     ctx_tokens: int = 0
     flags: int = 0
     gen_us: int = 0            # audio generated for the current reply
@@ -71,7 +73,7 @@ class SessionState:
 
 def apply_event(st: SessionState, kind: int, t_us: int, a: int = 0, b: int = 0,
                 protect_us: int = 0) -> None:
-    """Apply one monitor event to ``st`` in place."""
+    """Apply one monitor event to ``st`` in place (Sections 5.1 and 5.2)."""
     if kind == SE_TURN_BEGIN:
         # The turn's request runs: its KV is pinned running KV (Section 5, Fig. 6),
         # immediate-reuse ends, warmed KV has been reused (Section 5.2).
