@@ -712,10 +712,10 @@ def _profiled_traffic(kernel, bytes_per_launch):
 
 
 # ----------------------------------------------------------- the oracle arm
-def _oracle_sample(seed):
+def _oracle_sample(seed, n_turns=400):
     from workloads import make_workload, pool_spec
     spec = pool_spec(WORKLOAD).with_(n_sessions=8, hbm_pages=1500, hbm_budget_pages=1500)
-    return make_workload(WORKLOAD, seed, spec=spec, n_turns=400)
+    return make_workload(WORKLOAD, seed, spec=spec, n_turns=max(400, int(n_turns)))
 
 
 def cpu_baseline(seconds, seed, steps=None):
@@ -806,12 +806,13 @@ def reference(args):
         return None
     K, W = args.steps, args.warmup
     from oracle import OracleManager
-    wl = _oracle_sample(args.seed)
+    wl = _oracle_sample(args.seed, n_turns=W + K + 1)
     om = OracleManager(wl, with_bytes=True, content=None, rank_on="none")
     om.pool.hbm.fill(1)
     om.pool.host.fill(1)
     S = wl.spec.n_sessions
     per_turn = S + 1
+    assert (W + K) * per_turn <= wl.n_events
 
     def turn(i):
         b0 = om.pool.bytes_out + om.pool.bytes_in
