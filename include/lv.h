@@ -26,7 +26,10 @@
  * lv_sync / lv_get_stats report; the kernels skip the offending item instead of
  * faulting, and no call traps, aborts or falls back to the CPU.  Nothing in the
  * library waits on the device except lv_sync, lv_get_stats and the readers
- * named as synchronous below.
+ * named as synchronous below.  Every call returns LV_ERR_INVALID for a NULL
+ * pool or a NULL required pointer, LV_ERR_OOM when staging a host argument
+ * needs memory that cannot be had, and LV_ERR_CUDA when a CUDA runtime call
+ * fails; the comments below name the other statuses.
  *
  * Pointers.  Array arguments may point to device memory or to host memory.  A
  * host input is copied to the device in stream order before use (pageable host
@@ -242,11 +245,13 @@ lv_status lv_pool_import(lv_pool* pool, const int32_t* placement, const int32_t*
 
 /* ------------------------------------------------------------ sessions */
 
-/* Writes states[0..n) to sessions first..first+n (ctx_tokens is ignored). */
+/* Writes states[0..n) to sessions first..first+n (ctx_tokens is ignored).
+   LV_ERR_INVALID when [first, first+n) is not within 0..max_sessions. */
 lv_status lv_session_set(lv_pool* pool, const lv_session_state* states, int32_t first,
                          int32_t n, lv_stream stream);
 
-/* Reads sessions first..first+n into out (host or device). */
+/* Reads sessions first..first+n into out (host or device).  LV_ERR_INVALID
+   when [first, first+n) is not within 0..max_sessions. */
 lv_status lv_session_get(lv_pool* pool, lv_session_state* out, int32_t first, int32_t n,
                          lv_stream stream);
 
