@@ -255,7 +255,7 @@ lv_status lv_session_set(lv_pool* pool, const lv_session_state* states, int32_t 
 lv_status lv_session_get(lv_pool* pool, lv_session_state* out, int32_t first, int32_t n,
                          lv_stream stream);
 
-/* Section 3 (runtime monitor: playback progress, speech activity, barge-in)
+/* Section 3 (runtime monitor: playback position, user speech, barge-in)
    and Sections 5.1-5.2: applies n events in order to the session table.
    TURN_BEGIN sets RUNNING, clears IMMEDIATE and the preload protection.
    TURN_END(a, b) clears RUNNING, starts a reply of a us and b units (LV_RESP_OPEN).
@@ -388,8 +388,8 @@ lv_status lv_make_resident(lv_pool* pool, int32_t sid, int64_t now_us, int32_t a
                            int32_t* append_out, lv_resident_result* result_out,
                            lv_stream stream);
 
-/* Section 6 (side tables) and Section 5.2 ("preloading affects latency but not
-   correctness"): commits n entries.  For each, the new location must be a
+/* Section 6 (side tables) and Section 5.2 (a failed
+   preload costs time, never correctness): commits n entries.  For each, the new location must be a
    reservation not yet owned; it becomes owned by (sid, blk), the block table
    points to it and the old location is freed.  LV_TIERS_INCLUSIVE: a host
    location may also be the block's own clean copy (it then stops being a

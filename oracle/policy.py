@@ -12,11 +12,12 @@ Readings:
     suffix-first rule (Section 5.1, last paragraph) orders blocks by
     decreasing block id.  ``ASCENDING`` orders them by increasing block id
     instead (the literal "(session id, block id) ascending" tie-break).
-  * T_next is clamped to [0, 2^32 - 1] microseconds; the estimate "need not
-    be an exact wall-clock prediction" (Section 5.1).
+  * T_next is clamped to [0, 2^32 - 1] microseconds; the paper asks only for
+    an ordering signal, not a precise forecast of the time (Section 5.1).
   * T_play in the progress-counter mode is the current reply's length in
-    units times ``unit_us`` while the reply is unfinished, else 0 ("longer
-    unfinished responses" mean later reuse, Section 5.1); like the playback
+    units times ``unit_us`` while the reply is unfinished, else 0 (the paper
+    reads a reply that is still long and open as reuse further away, Section
+    5.1); like the playback
     horizon it is never negative.
   * Protection holds against *normal* eviction only (Section 5.1), and warmed
     KV may still be evicted before it is reused (Section 5.2).  With ``fallback`` set (a
@@ -46,12 +47,12 @@ LRU = 1             # the substrate's least-recently-used baseline (Sections 2.3
 def t_next(st: SessionState, mode: int, reply_prior_us: int, unit_us: int) -> int:
     """Eq. 4: T_next = T_play + T_reply for one session (clamped to 32 bits)."""
     if mode == MODE_PLAYBACK:
-        t_play = max(0, st.gen_us - st.play_us)            # remaining playback horizon
+        t_play = max(0, st.gen_us - st.play_us)            # audio still to play
     elif mode == MODE_COUNTERS:
         t_play = max(0, st.reply_tokens * unit_us) if (st.flags & RESP_OPEN) else 0
     else:
         raise ValueError(f"unknown T_play mode {mode}")
-    # per-session moving average when available, workload-level prior otherwise
+    # the session's own average once it has a sample, else the workload prior
     t_reply = st.reply_ema_us if st.reply_n > 0 else reply_prior_us
     return min(KEY_MAX, max(0, t_play + t_reply))
 
@@ -60,7 +61,7 @@ next_use_key = t_next
 
 
 def is_eligible(st: SessionState, now_us: int) -> bool:
-    """Only idle-resident multi-turn KV may be evicted (Section 5.1, Eviction policy):
+    """Eviction takes only multi-turn KV that sits in HBM unused (Section 5.1, Eviction policy):
     pinned running KV, immediate-reuse sessions (speech start / barge-in) and
     preload-protected sessions (Section 5.2) are excluded."""
     if st.flags & (RUNNING | IMMEDIATE):

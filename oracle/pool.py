@@ -19,7 +19,7 @@ Operations follow their plain definitions:
   * remap commits (sid, blk, new location) entries: the table points to the
     new location, which becomes owned, and the old location is freed.  A
     failed or cancelled transfer is never committed, so the old mapping stays
-    valid (Section 5.2: preloading affects latency but not correctness).
+    valid (Section 5.2: a preload that fails only costs time; the result stays right).
 
 Tiers (the paper does not say whether the host copy is kept after a reload):
   * exclusive (default): a block lives in exactly one tier; its host slot is

@@ -1,14 +1,15 @@
 """Per-session interaction state and how monitor events change it.
 
-The runtime monitor (Section 3) reports playback progress, speech activity and
+The runtime monitor (Section 3) reports how far playback has got, whether the user speaks, and
 barge-ins; the KV manager keeps per-session side tables with the next-use
 estimate's inputs and the preload-protection state (Section 6, "Hierarchical
 KV cache manager").  This module is that state, updated one event at a time in
 event order.  Times are integer microseconds.
 
 Readings (the paper does not fix these):
-  * T_reply is a moving average, kept per session, of the time from playback
-    completion to the next completed user input (Section 5.1, after Eq. 4).
+  * T_reply is a moving average, kept per session, of how long the user takes
+    to finish speaking again once the reply has played out (Section 5.1,
+    after Eq. 4).
     Reading: an integer exponential moving average with weight 1/4,
     ``ema <- floor((3*ema + x) / 4)``; the first sample sets ``ema = x``.
   * A sample is taken at SPEECH_STOP (the user input is complete) when the
@@ -100,7 +101,7 @@ def apply_event(st: SessionState, kind: int, t_us: int, a: int = 0, b: int = 0,
     elif kind == SE_SPEECH_START:
         st.flags |= IMMEDIATE
     elif kind == SE_BARGE_IN:
-        # Tokens beyond the playback point are discarded (Section 3, barge-in handling).
+        # Audio not yet played is dropped on a barge-in (Section 3, barge-in handling).
         st.gen_us = st.play_us
         st.flags = (st.flags | IMMEDIATE) & ~(RESP_OPEN | DONE_VALID)
     elif kind == SE_SPEECH_STOP:

@@ -135,7 +135,7 @@ def _prefers(x, y, keyof, within):
     """True when candidate x must be evicted before candidate y (Section 5.1 wording).
 
     keyof(sid) -> (tier, T_next).  The normally eligible tier comes first; then the
-    session whose next use is farther away; equal estimates by smaller session id;
+    session with the later predicted next use; equal estimates by smaller session id;
     within a session the suffix (larger block id) first, or the smaller block id
     under ASCENDING."""
     (sx, bx), (sy, by) = x, y

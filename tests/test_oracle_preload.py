@@ -19,7 +19,7 @@ def test_controller_properties(name, bw, lead, cap):
     for i in range(wl.n_events):
         rec = m.step(i)
         for sid, start, finish, t_pred, pages in rec.get("admitted", []):
-            # "enough time to hide the transfer cost": the transfer ends by the predicted turn
+            # admitted only when the copy can finish unseen: the transfer ends by the predicted turn
             assert finish <= t_pred
             assert start >= rec["t"] and finish - start == -(-len(pages) * page_bytes // bw)
             intervals.append((start, finish))
