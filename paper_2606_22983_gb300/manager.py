@@ -443,9 +443,3 @@ class KVManager:
             order, n = pool.select(t, lv.LV_ALL, 0)
             rec["order"] = order.cpu().numpy().astype(np.int64)
         return rec
-
-    def playback_batch(self, t_us, sids, deltas):
-        """Many PLAYBACK reports at once (one kernel launch)."""
-        ev = np.zeros(len(sids), dtype=lv.EVENT_DTYPE)
-        ev["kind"], ev["sid"], ev["t_us"], ev["a"] = lv.LV_EV_PLAYBACK, sids, t_us, deltas
-        self.pool.events(ev)
