@@ -28,6 +28,11 @@ reading -- parity unpinned against the paper):
     session id) are dropped until they fit -- the new one too if it alone
     exceeds the cap.
 
+The code is pinned to these readings by two scenarios whose every decision was
+worked by hand (tests/golden/preload_controller_hand.json: admission, queueing on
+the link, victims, waiting, completion, cancellation, the cap, hits, give-ups,
+the lead average) and by properties on the generated workloads.
+
 Counters: admitted, completed, waited (admitted after at least one refusal),
 given_up, cancelled, hits (turns whose session needed no synchronous load after
 a completed preload), sync_loads.
