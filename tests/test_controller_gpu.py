@@ -68,3 +68,46 @@ def test_controller_matches_oracle(name, bw, lead, cap, with_bytes, tiers):
         torch.cuda.synchronize()
         pool.close()
         torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("index", [0, 1])
+def test_controller_hand_worked_scenarios(index):
+    """The two scenarios of tests/golden/preload_controller_hand.json through the native
+    controller: every decision against the oracle's, which the CPU tests pin to the
+    hand-worked values; byte images compared after every event."""
+    import torch
+    from oracle.preload import ControlledOracleManager, PreloadController
+    from paper_2606_22983_gb300.controller import ControlledKVManager
+    from paper_2606_22983_gb300.harness import ContentWriter, pool_for, zero_host
+    from ._hand import hand_workload, load
+    from ._lockstep import compare_state
+
+    sc = load("preload_controller_hand.json")["scenarios"][index]
+    c = sc["controller"]
+    wl = hand_workload(sc)
+    om = ControlledOracleManager(wl, PreloadController(link_bytes_per_us=c["link_bytes_per_us"],
+                                                       lead_prior_us=c["lead_prior_us"],
+                                                       cap_pages=c["cap_pages"]),
+                                 with_bytes=True, content=(wl.seed, value_table(wl.seed)),
+                                 rank_on="none")
+    pool = pool_for(wl)
+    try:
+        writer = ContentWriter(pool, wl)
+        zero_host(pool)
+        writer.write_initial(wl)
+        gm = ControlledKVManager(pool, link_bytes_per_us=c["link_bytes_per_us"],
+                                 lead_prior_us=c["lead_prior_us"],
+                                 cap_pages=c["cap_pages"],
+                                 perms=wl.perms, on_append=writer.write_appended,
+                                 order_fn=scatter_order)
+        for i in range(wl.n_events):
+            ro, rg = om.step(i), gm.step(wl.event(i), i)
+            _compare_controller(ro, rg, (i, wl.event(i)))
+            compare_state(om, pool, i, True)
+        for k, v in sc["expect_counters"].items():
+            if k in gm.counters:
+                assert gm.counters[k] == v, k
+        assert om.pool.tables.tolist() == sc["expect_tables"]
+    finally:
+        torch.cuda.synchronize()
+        pool.close()

@@ -237,3 +237,23 @@ def test_next_use_versus_lru_on_the_voice_workloads():
     for name in ("tiny", "mixed"):
         nu, lru = rows[(name, 0)], rows[(name, 1)]
         assert nu["sync_loads"] < lru["sync_loads"], (name, nu, lru)
+
+
+def test_turns_preload_fallback_and_eviction_hand_worked():
+    """Every decision of a small script worked by hand (tests/golden/manager_turns_hand.json):
+    a preload, turns with growth, the foreground fallback tier and an eviction request
+    with fewer candidates than asked for."""
+    from oracle.manager import OracleManager
+    from ._hand import hand_workload, load
+    g = load("manager_turns_hand.json")
+    m = OracleManager(hand_workload(g), with_bytes=True, content="tagged", rank_on="none")
+    for i, want in enumerate(g["expect"]):
+        rec = m.step(i)
+        got = {k: np.asarray(rec[k]).tolist() for k in want if k in rec}
+        assert got == want, (i, got)
+        assert not any(k in rec for k in ("k", "victims", "in_blocks", "append_pages") if k not in want), i
+        m.pool.check_invariants()
+    assert m.pool.tables.tolist() == g["expect_tables"]
+    assert [s.ctx_tokens for s in m.sessions] == g["expect_ctx_tokens"]
+    assert [s.protect_until_us for s in m.sessions] == g["expect_protect_until_us"]
+    assert {k: m.counters[k] for k in g["expect_counters"]} == g["expect_counters"]

@@ -64,49 +64,19 @@ def test_fast_link_admits_every_preload_and_hides_reloads():
 
 
 # ------------------------------------------------------ hand-worked scenarios
-import json
-import os
-
-from oracle.preload import ControlledOracleManager as _CM
-from workloads.configs import PoolSpec, TINY_SHAPE
-from workloads.scripts import (InitialState, Workload, EV_TURN, EV_PLAYBACK, EV_SPEECH_START,
-                               EV_SPEECH_STOP)
-
-_GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "preload_controller_hand.json")
-_KINDS = {"TURN": EV_TURN, "PLAYBACK": EV_PLAYBACK, "SPEECH_START": EV_SPEECH_START,
-          "SPEECH_STOP": EV_SPEECH_STOP}
-
-
-def _hand_workload(sc):
-    p = sc["pool"]
-    spec = PoolSpec("hand", TINY_SHAPE, n_sessions=p["n_sessions"], max_blocks=p["max_blocks"],
-                    hbm_pages=p["hbm_pages"], hbm_budget_pages=p["hbm_budget_pages"],
-                    host_pages=p["host_pages"], reply_prior_us=p["reply_prior_us"],
-                    protect_us=p["protect_us"])
-    S = spec.n_sessions
-    z = np.zeros(S, np.int64)
-    init = InitialState(ctx_tokens=np.array(sc["initial"]["ctx_tokens"], np.int32),
-                        placement=np.array(sc["initial"]["placement"], np.int32),
-                        gen_us=z.copy(), play_us=z.copy(), resp_open=np.zeros(S, np.int32),
-                        reply_tokens=np.zeros(S, np.int32))
-    ev = sc["events"]
-    col = lambda key, dt: np.array([e.get(key, 0) for e in ev], dt)
-    return Workload(spec=spec, seed=0, init=init, t_us=col("t", np.int64),
-                    kind=np.array([_KINDS[e["ev"]] for e in ev], np.int32), sid=col("sid", np.int32),
-                    a=col("a", np.int64), b=col("b", np.int64), c=np.zeros(len(ev), np.int64),
-                    d=np.full(len(ev), -1, np.int32), perms=np.zeros((0, S), np.int32))
+from ._hand import hand_workload, load as _load_hand
 
 
 @pytest.mark.parametrize("index", [0, 1])
 def test_controller_hand_worked_scenarios(index):
     """Every decision of two small scenarios, worked by hand from the controller's
     reading of Section 5.2 (tests/golden/preload_controller_hand.json)."""
-    sc = json.load(open(_GOLDEN))["scenarios"][index]
+    sc = _load_hand("preload_controller_hand.json")["scenarios"][index]
     c = sc["controller"]
-    m = _CM(_hand_workload(sc), PreloadController(link_bytes_per_us=c["link_bytes_per_us"],
-                                                   lead_prior_us=c["lead_prior_us"],
-                                                   cap_pages=c["cap_pages"]),
-            with_bytes=True, content="tagged", rank_on="none")
+    m = ControlledOracleManager(hand_workload(sc), PreloadController(link_bytes_per_us=c["link_bytes_per_us"],
+                                                                     lead_prior_us=c["lead_prior_us"],
+                                                                     cap_pages=c["cap_pages"]),
+                                with_bytes=True, content="tagged", rank_on="none")
     admitted, victims, completed, cancelled, unprotected = [], {}, {}, {}, {}
     for i in range(m.wl.n_events):
         rec = m.step(i)

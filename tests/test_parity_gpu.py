@@ -36,6 +36,19 @@ def test_tiny_workload_address_tagged_bytes(driver, mode):
     assert om.counters == gm.counters and gm.counters["pages_out"] > 300
 
 
+@pytest.mark.parametrize("driver,mode", [("device", 0), ("exchange", 0), ("exchange", 2),
+                                         ("sequential", 0)])
+def test_hand_worked_turns(driver, mode):
+    """The hand-worked script of tests/golden/manager_turns_hand.json (a preload, growth,
+    the foreground fallback tier, an eviction with a shortfall): every decision and the
+    state with address-tagged bytes after every event."""
+    from ._hand import hand_workload, load
+    g = load("manager_turns_hand.json")
+    om, gm = run_lockstep(hand_workload(g), with_bytes=True, check_every=1, driver=driver,
+                          mode=mode, tagged=True)
+    assert om.pool.tables.tolist() == g["expect_tables"]
+
+
 @pytest.mark.parametrize("driver", ["device", "sequential"])
 def test_tiny_workload_lru_baseline(driver):
     """The LRU baseline policy on the same kernels (NEXT f3): every ranking and
