@@ -677,7 +677,8 @@ lv_status lv_selftest_wait(lv_pool* pool, int64_t limit_us, lv_stream stream);
      link_bytes_per_us, it finishes by the predicted start of the session's turn,
      t_speech + lead (lead: the session's moving average of turn start minus
      speech start, integer EMA of weight 1/4, first sample sets it; lead_prior_us
-     before any sample), and if the pages it must evict fit in the host tier with
+     before any sample; t_speech is the first speech start or barge-in since the
+     session's last turn), and if the pages it must evict fit in the host tier with
      max_blocks slots still free.
    - A refused preload waits and is re-checked at every later tick until it is
      admitted, its deadline passes (given up), or the turn begins (given up).

@@ -13,6 +13,8 @@ reading -- parity unpinned against the paper):
     still free (room for a foreground turn's synchronous eviction).  lead is
     the session's moving average of (turn start - speech start) -- integer EMA
     with weight 1/4, first sample sets it -- or ``lead_prior_us`` before any
+    sample.  t_speech is the first speech start (or barge-in) since the session's
+    last turn: later ones before the same turn move neither the deadline nor the
     sample.  A sync load at a turn also occupies the link.
   * Brief wait and re-check: a preload that is not admitted waits; at every later
     event before the turn it is re-evaluated at that event's time (the slack
