@@ -92,3 +92,40 @@ def test_reply_interval_events():
         assert pool.sync() == 0
     finally:
         pool.close()
+
+
+def test_scenario_on_the_allocation_free_ranker():
+    """The same scenario through lv_select_victims_noalloc, from caller-held session and
+    block tables: the next-use victims, then the state a barge-in of session 1 leaves
+    (its unplayed audio dropped, immediate reuse)."""
+    import torch
+    from paper_2606_22983_gb300 import lv
+    g = _load("scenario_lru_vs_next_use.json")
+    S, maxb, T = len(g["sessions"]), 8, 16
+    st = np.zeros(S, dtype=lv.SESSION_DTYPE)
+    tables = np.full((S, maxb), -1, np.int32)
+    page = 0
+    for s, d in enumerate(g["sessions"]):
+        st[s]["ctx_tokens"] = d["resident_blocks"] * T
+        st[s]["gen_us"], st[s]["play_us"] = d["gen_us"], d["play_us"]
+        st[s]["flags"] = lv.LV_RUNNING if "RUNNING" in d["flags"] else 0
+        for b in range(d["resident_blocks"]):
+            tables[s, b] = page
+            page += 1
+    prm = lv.lv_rank_params(num_sessions=S, max_blocks=maxb, page_tokens=T, within_order=0,
+                            t_play_mode=0, flags=0, reply_prior_us=g["reply_prior_us"], unit_us=80_000)
+    tab = torch.from_numpy(tables).cuda()
+    cap = 16
+
+    def rank(states):
+        sess = torch.from_numpy(states.view(np.uint8).copy()).cuda()
+        out = torch.full((cap, 3), -7, dtype=torch.int32, device="cuda")
+        cnt = torch.full((1,), -1, dtype=torch.int64, device="cuda")
+        lv.lv_select_victims_noalloc(prm, sess, tab, g["now_us"], g["k"], out, cap, cnt, None)
+        torch.cuda.synchronize()
+        return out[:int(cnt.item())].cpu().numpy()
+
+    assert rank(st)[:, :2].tolist() == g["expect_next_use_victims"]
+    st[1]["gen_us"] = st[1]["play_us"]
+    st[1]["flags"] |= lv.LV_IMMEDIATE
+    assert rank(st)[:, :2].tolist() == g["barge_in_variant"]["expect_victims"]
