@@ -39,8 +39,9 @@ def test_controller_matches_oracle(name, bw, lead, cap, with_bytes, tiers):
     from paper_2606_22983_gb300.harness import ContentWriter, pool_for, zero_host
     from ._lockstep import compare_state
 
-    from workloads import pool_spec
-    wl = make_workload(name, 0, spec=pool_spec(name).with_(tiers=tiers))
+    from workloads import host_tier_limit, pool_spec
+    wl = make_workload(name, 0, spec=pool_spec(name).with_(tiers=tiers),
+                       host_limit=host_tier_limit() if name == "mixed" else None)
     table = value_table(wl.seed)
     om = ControlledOracleManager(wl, PreloadController(link_bytes_per_us=bw, lead_prior_us=lead,
                                                        cap_pages=cap),
@@ -63,7 +64,13 @@ def test_controller_matches_oracle(name, bw, lead, cap, with_bytes, tiers):
         for k in ("admitted", "completed", "waited", "given_up", "cancelled", "hits", "sync_loads",
                   "pages_in", "pages_out"):
             assert om.counters[k] == gm.counters[k], k
-        assert gm.counters["cancelled"] > 0 and gm.counters["given_up"] > 0
+        assert gm.counters["given_up"] > 0 and gm.counters["admitted"] > 0
+        if name == "tiny":
+            assert gm.counters["cancelled"] > 0
+        else:
+            # 256 sessions on a 60 GB budget: the host tier is tight, so most preloads wait
+            # for room and are given up; the admitted ones complete before their turns
+            assert gm.counters["waited"] > 0 and gm.counters["hits"] > 0
     finally:
         torch.cuda.synchronize()
         pool.close()

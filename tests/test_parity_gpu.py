@@ -149,11 +149,28 @@ def test_thinker_full_size_sampled_bytes(driver, mode):
     _sampled_full_size(make_workload("thinker", 0, n_turns=6), driver, mode)
 
 
+def _at_stated_size(name, seed):
+    """The workload at its stated session count (256 mixed, 1024 frag) when this host
+    can page-lock its host tier within min(400 GB, 0.8 * MemAvailable), else scaled
+    down to that limit; the sizing is printed (pytest -rP shows it) and checked."""
+    from workloads import STATED_SESSIONS, host_tier_limit, mem_available_bytes
+    mem = mem_available_bytes()
+    wl = make_workload(name, seed, host_limit=host_tier_limit(mem))
+    sz = wl.meta["sizing"]
+    print(f"sizing {name} seed {seed}: MemAvailable {mem} B, limit {sz['host_limit_bytes']} B, "
+          f"sessions {sz['sessions']} of {sz['stated_sessions']}, host tier {sz['host_tier_bytes']} B")
+    assert sz["host_tier_bytes"] <= sz["host_limit_bytes"]
+    assert sz["stated_sessions"] == STATED_SESSIONS[name]
+    if not sz["scaled"]:
+        assert wl.spec.n_sessions == STATED_SESSIONS[name]
+    return wl
+
+
 def test_mixed_realtime_full_size():
-    """Mixed realtime load: 128 sessions (log-uniform 2k-16k tokens) with Poisson
+    """Mixed realtime load: 256 sessions (log-uniform 2k-16k tokens) with Poisson
     next-speech arrivals, barge-ins, speech-triggered preloads and turns with
-    growth; 60 GB HBM budget, ~40 GB host tier; 3000 events."""
-    om, gm = _sampled_full_size(make_workload("mixed", 0), "device", 0)
+    growth; 60 GB HBM budget, a ~115-135 GB host tier; 3000 events."""
+    om, gm = _sampled_full_size(_at_stated_size("mixed", 0), "device", 0)
     assert om.counters["preloads"] > 50 and om.counters == gm.counters
 
 
@@ -161,7 +178,7 @@ def test_mixed_realtime_full_size_async_copies():
     """The mixed workload with every turn's and preload's copy left running on the pool's
     copy stream (turns, preloads and growth overlap earlier copies): the end state and
     sampled bytes equal the oracle's."""
-    om, gm = _sampled_full_size(make_workload("mixed", 1), "device", 0, record=False,
+    om, gm = _sampled_full_size(_at_stated_size("mixed", 1), "device", 0, record=False,
                                 async_copy=True)
 
 
@@ -182,11 +199,11 @@ def test_long_multimodal_full_size():
 @pytest.mark.parametrize("driver,async_copy", [("exchange", False), ("device", False),
                                                ("device", True)])
 def test_fragmentation_full_size(driver, async_copy):
-    """Pages randomly permuted over a 100 GB HBM budget, 640 sessions of
-    256-4096 tokens; 10 000 events alternating "free k pages" with turns whose
-    reload list comes in a scattered order (with the device driver, the evictions
-    run through lv_evict and the turns through lv_turn with load keys; with
-    asynchronous copies, nothing is read back between events)."""
-    om, gm = _sampled_full_size(make_workload("frag", 0), driver, 0, rank_on="none",
+    """Pages randomly permuted over a 100 GB HBM budget, 1024 sessions of
+    256-4096 tokens (~219 GB of KV, a ~148 GB host tier); 10 000 events alternating
+    "free k pages" with turns whose reload list comes in a scattered order (with the
+    device driver, the evictions run through lv_evict and the turns through lv_turn
+    with load keys; with asynchronous copies, nothing is read back between events)."""
+    om, gm = _sampled_full_size(_at_stated_size("frag", 0), driver, 0, rank_on="none",
                                 record=not async_copy, async_copy=async_copy)
     assert om.counters["turns"] == 5000

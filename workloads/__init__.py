@@ -8,6 +8,7 @@ same generated inputs, and neither is imported here.
 """
 from .configs import (  # noqa: F401
     KVShape, PoolSpec, TINY_SHAPE, THINKER_SHAPE, CONFIG_NAMES, pool_spec, GB,
+    STATED_SESSIONS, host_tier_limit, mem_available_bytes,
 )
 from .scripts import (  # noqa: F401
     Workload, InitialState, make_workload,

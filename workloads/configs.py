@@ -73,6 +73,31 @@ class PoolSpec:
 
 CONFIG_NAMES = ("tiny", "thinker", "mixed", "long", "frag")
 
+# Session counts of the two workloads whose host tier is the largest.  Where the host
+# cannot page-lock that much, the count is scaled down (``host_tier_limit``).
+STATED_SESSIONS = {"mixed": 256, "frag": 1024}
+HOST_TIER_CAP = 400 * GB       # the mixed workload's stated host tier
+
+
+def mem_available_bytes(path: str = "/proc/meminfo"):
+    """MemAvailable of this host in bytes, or None where /proc/meminfo has none."""
+    try:
+        with open(path) as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    return None
+
+
+def host_tier_limit(mem_available=None) -> int:
+    """Page-locked host tier a workload may take: min(400 GB, 0.8 * MemAvailable)."""
+    m = mem_available_bytes() if mem_available is None else int(mem_available)
+    if m is None:
+        return HOST_TIER_CAP
+    return min(HOST_TIER_CAP, int(0.8 * m))
+
 
 def pages_for_bytes(nbytes: int, shape: KVShape) -> int:
     return nbytes // shape.page_bytes
@@ -89,19 +114,17 @@ def pool_spec(name: str) -> PoolSpec:
         return PoolSpec("thinker", THINKER_SHAPE, n_sessions=64, max_blocks=1024,
                         hbm_pages=b, hbm_budget_pages=b, host_pages=0)
     if name == "mixed":
-        # 256 sessions would need a ~120 GB pinned host tier; scaled to 128 sessions so the
-        # host tier (~40 GB) leaves most of a 199 GB host free
+        # 256 sessions: the host tier comes to ~115-135 GB of page-locked memory
         b = pages_for_bytes(60 * GB, THINKER_SHAPE)          # 38 146 pages
-        return PoolSpec("mixed", THINKER_SHAPE, n_sessions=128, max_blocks=1024,
-                        hbm_pages=b, hbm_budget_pages=b, host_pages=0)
+        return PoolSpec("mixed", THINKER_SHAPE, n_sessions=STATED_SESSIONS["mixed"],
+                        max_blocks=1024, hbm_pages=b, hbm_budget_pages=b, host_pages=0)
     if name == "long":
         b = pages_for_bytes(40 * GB, THINKER_SHAPE)
         return PoolSpec("long", THINKER_SHAPE, n_sessions=16, max_blocks=4096,
                         hbm_pages=b, hbm_budget_pages=b, host_pages=0)
     if name == "frag":
-        # 1024 sessions of 256-4096 tokens hold ~219 GB, which would need ~140 GB of
-        # pinned host memory; scaled to 640 sessions (~137 GB, host tier ~45 GB)
+        # 1024 sessions of 256-4096 tokens hold ~219 GB: a host tier of ~140-150 GB
         b = pages_for_bytes(100 * GB, THINKER_SHAPE)         # 63 578 pages
-        return PoolSpec("frag", THINKER_SHAPE, n_sessions=640, max_blocks=256,
-                        hbm_pages=b, hbm_budget_pages=b, host_pages=0)
+        return PoolSpec("frag", THINKER_SHAPE, n_sessions=STATED_SESSIONS["frag"],
+                        max_blocks=256, hbm_pages=b, hbm_budget_pages=b, host_pages=0)
     raise ValueError(f"unknown workload {name!r}; expected one of {CONFIG_NAMES}")

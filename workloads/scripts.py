@@ -263,7 +263,7 @@ def _interactive(spec: PoolSpec, seed: int, n_events: int, ctx_lo: int, ctx_hi: 
             if r[1] == EV_TURN:
                 grown[r[2]] += r[3]
         total = int(_pages(grown, T).sum())
-        host = max(int(n_pages.sum()) - spec.hbm_budget_pages, total - spec.hbm_budget_pages) \
+        host = max(int(n_pages.sum()) - spec.hbm_budget_pages, total - spec.hbm_budget_pages, 0) \
             + 2 * spec.max_blocks
         if spec.tiers == 1:          # inclusive tiers: room for a host copy of every block
             host = total + 2 * spec.max_blocks
@@ -376,11 +376,44 @@ def _frag(spec: PoolSpec, seed: int, n_events: int, ctx_lo: int, ctx_hi: int,
                     meta={"total_pages": total})
 
 
-def make_workload(name: str, seed: int = 0, **over) -> Workload:
+def make_workload(name: str, seed: int = 0, host_limit=None, **over) -> Workload:
     """Build the seeded workload ``name`` (see ``workloads.configs.CONFIG_NAMES``).
 
     Keyword overrides change the scale (e.g. ``n_events``, ``n_turns``, ``spec``).
+    ``host_limit`` (bytes, for a caller that page-locks the host tier): when the
+    workload's host tier would exceed it, the session count is scaled down by the
+    ratio of the two and the script drawn again (then by 1 % steps until it fits);
+    ``meta["sizing"]`` records the limit, the stated and the used session counts.
     """
+    if host_limit is None:
+        return _make(name, seed, **over)
+    wl = _make(name, seed, **dict(over))
+    n0 = wl.spec.n_sessions
+    need = wl.spec.host_pages * wl.spec.shape.page_bytes
+    n = n0
+    # the host tier is about (all pages - budget + slack): linear in the session count
+    per_session = (need + wl.spec.hbm_budget_pages * wl.spec.shape.page_bytes) / max(n0, 1)
+    while need > host_limit and n > 1:
+        guess = int((host_limit + wl.spec.hbm_budget_pages * wl.spec.shape.page_bytes) / per_session)
+        n = max(1, min(n - 1, guess))
+        sp = (over.get("spec") or pool_spec(name)).with_(n_sessions=n)
+        wl = _make(name, seed, **dict(over, spec=sp))
+        need = wl.spec.host_pages * wl.spec.shape.page_bytes
+    # the estimate may undershoot: take the largest count that still fits
+    while wl.spec.n_sessions < n0 and need <= host_limit:
+        sp = (over.get("spec") or pool_spec(name)).with_(n_sessions=wl.spec.n_sessions + 1)
+        nxt = _make(name, seed, **dict(over, spec=sp))
+        nneed = nxt.spec.host_pages * nxt.spec.shape.page_bytes
+        if nneed > host_limit:
+            break
+        wl, need = nxt, nneed
+    wl.meta["sizing"] = {"host_limit_bytes": int(host_limit), "stated_sessions": n0,
+                         "sessions": wl.spec.n_sessions, "host_tier_bytes": int(need),
+                         "scaled": wl.spec.n_sessions != n0}
+    return wl
+
+
+def _make(name: str, seed: int = 0, **over) -> Workload:
     spec = over.pop("spec", None) or pool_spec(name)
     if name == "tiny":
         kw = dict(n_events=1000, ctx_lo=64, ctx_hi=512, log_uniform_ctx=False,
