@@ -486,29 +486,6 @@ lv_status lv_unpack_pages(lv_pool* pool, const void* src, const int32_t* pages, 
 lv_status lv_page_checksums(lv_pool* pool, const int32_t* pages, int64_t n, uint64_t* sums_out,
                             lv_stream stream);
 
-/* Scattered-access probe (an instrument, not from the paper).  Launches one
-   kernel on `stream` with `threads` threads; each makes mix->loads loads,
-   mix->atomics returning atomics (atomicExch), mix->stores stores and
-   mix->reductions reductions (atomicAnd with a constant), in that order, to
-   4-byte words of `array` (device memory, uint32 [words], owned by the caller;
-   words a power of two up to 2^32) at hashed positions, no request depending
-   on another.  Stores and atomics overwrite array words.  The caller times the
-   launch (CUDA events on `stream`).  One kind alone measures the rate at which
-   the GPU serves that kind of scattered request; a kernel's own mix per work
-   item, one thread per item, measures the ceiling of that kernel (k_remap
-   commits one entry with two loads, two returning atomics, two stores and
-   one reduction).  sink (uint32 [1], device, may be NULL) is never written in
-   practice; it keeps the loads from being removed.  LV_ERR_INVALID for a
-   count outside 0..64 or a bad size, LV_ERR_CUDA if the launch fails. */
-typedef struct lv_probe_mix {
-  int32_t loads;
-  int32_t atomics;
-  int32_t stores;
-  int32_t reductions;
-} lv_probe_mix;
-lv_status lv_probe_scattered(const lv_probe_mix* mix, uint32_t* array, int64_t words,
-                             int64_t threads, uint32_t* sink, lv_stream stream);
-
 /* Block-level allocation kept (Section 5.1): grows session sid's context by
    n_tokens; each new block takes the lowest free HBM page, in block order, and
    is committed at once.  LV_TIERS_INCLUSIVE: when n_tokens > 0 and the last
@@ -546,26 +523,36 @@ lv_status lv_read_tables(lv_pool* pool, int32_t* tables, int32_t* hbm_owner,
    latency-critical scheduler thread, where cudaMalloc / cudaFree can
    synchronise the device.
 
-   lv_select_victims_noalloc computes exactly what lv_select_victims computes
-   (same order, same count, same fallback tier), but from a session table and
-   block tables that the caller passes in, without a pool: sessions is
-   lv_session_state [num_sessions] (ctx_tokens gives each session's block
-   count), tables is int32 [num_sessions][max_blocks] in the block-table
-   encoding above.  Both, and out (lv_victim [capacity]) and count_out (int64,
-   may be NULL), must be device memory or mapped page-locked host memory;
-   pageable host pointers are rejected with LV_ERR_INVALID because staging them
-   would need an allocation.
+   lv_select_victims_noalloc computes what lv_select_victims computes on a pool
+   of the same policy, within order and T_play mode (same order, same count,
+   same fallback tier), but from a session table and block tables that the
+   caller passes in, without a pool: sessions is lv_session_state
+   [num_sessions] (ctx_tokens gives each session's block count), tables is
+   int32 [num_sessions][max_blocks] in the block-table encoding above.  Both,
+   and out (lv_victim [capacity]) and count_out (int64, may be NULL), must be
+   memory that the current device can address: device memory of the current
+   device, managed memory, or mapped page-locked host memory with a device
+   alias for it.  Pageable host pointers (staging them would need an
+   allocation) and device memory of another device are rejected with
+   LV_ERR_INVALID.
 
-   Its working memory is one array of LV_NOALLOC_MAX_SESSIONS x 12 bytes plus
-   256 bytes (48.25 KiB) compiled into liblv as device memory: every GPU that
+   Its working memory is one array of LV_NOALLOC_MAX_SESSIONS x 20 bytes plus
+   256 bytes (80.25 KiB) compiled into liblv as device memory: every GPU that
    loads the library holds it until the process exits.  num_sessions above
-   LV_NOALLOC_MAX_SESSIONS is rejected with LV_ERR_INVALID.  The call allocates
-   nothing (no cudaMalloc, cudaFree or allocating library routine).  The first
-   call on a device looks up that array's device address (cudaGetSymbolAddress),
-   so make the first call on each device before any stream capture.  All calls on a device share the one array and each call
-   starts by clearing its counters: calls whose execution overlaps on the GPU
-   (two streams, or two host threads) race and may return wrong victims, so
-   order them, for example on one stream. */
+   LV_NOALLOC_MAX_SESSIONS is rejected with LV_ERR_INVALID.  The call issues no
+   cudaMalloc, cudaFree or allocating library routine.  The first call on a
+   device looks up that array's device address (cudaGetSymbolAddress) and
+   keeps it for the rest of the process, so make the first call on each device
+   before any stream capture; under lazy module loading (the CUDA default) that
+   first call, or the first ranking of any kind on the device, may also load
+   liblv's kernels, which takes device memory once.  A warm-up call at
+   start-up, before the memory is given away, leaves every later call free of
+   allocations.  The kept address does not survive cudaDeviceReset or the
+   destruction of the device's primary context: do not call it after either.
+   All calls on a device share the one array and each call starts by clearing
+   its counters: calls whose execution overlaps on the GPU (two streams, or two
+   host threads) race and may return wrong victims, so order them, for example
+   on one stream. */
 #define LV_NOALLOC_MAX_SESSIONS 4096
 
 typedef struct lv_rank_params {
@@ -577,6 +564,8 @@ typedef struct lv_rank_params {
   uint32_t flags;              /* 0 or LV_SELECT_FALLBACK */
   int64_t reply_prior_us;      /* >= 0 */
   int64_t unit_us;             /* 1..2^31 */
+  int32_t policy;              /* LV_POLICY_NEXT_USE or LV_POLICY_LRU */
+  int32_t reserved;            /* must be 0 */
 } lv_rank_params;
 
 lv_status lv_select_victims_noalloc(const lv_rank_params* params, const lv_session_state* sessions,
@@ -738,7 +727,7 @@ lv_status lv_controller_counters_get(lv_controller* c, lv_controller_counters* o
 const char* lv_status_str(lv_status s);
 /* The library's interface version: LV_VERSION of the header it was built with.  A
    caller built against another header must not use the library. */
-#define LV_VERSION 2
+#define LV_VERSION 3
 int32_t lv_version(void);
 
 #ifdef __cplusplus

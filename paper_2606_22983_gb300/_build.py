@@ -17,8 +17,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "liblv.so")
 
-SOURCES = ["lv_api.cu", "lv_kernels.cu", "lv_noalloc.cu", "lv_sched.cu", "lv_controller.cu",
-           "lv_probe.cu"]
+SOURCES = ["lv_api.cu", "lv_kernels.cu", "lv_noalloc.cu", "lv_sched.cu", "lv_controller.cu"]
 HEADERS = [os.path.join(CSRC, "lv_internal.cuh"), os.path.join(INCLUDE, "lv.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2", "--expt-relaxed-constexpr"]

@@ -22,6 +22,7 @@ enum Ctl : int {
   C_SEL_COUNT = 4,     // victims written by the last select
   C_SEL_TOTAL = 5,     // candidates seen by the last select
   C_CLEAN = 6,         // clean host copies held now (inclusive tiers; part of C_HOST_ALLOC)
+  C_RANK_TOTAL = 7,    // ranking scratch: resident blocks of all candidate sessions
   C_SELECTS = 8,
   C_VICTIMS,
   C_SHORTFALLS,
@@ -67,8 +68,14 @@ struct DevPool {
   // ranking scratch
   unsigned long long* skey;  // [S] session order key (0 = not a candidate)
   int32_t* scount;           // [S] resident blocks of the session
+  long long* sbefore;        // [S] resident blocks of the candidates ranked ahead of it
   // exchange scratch
   unsigned long long* page_tag;  // [hbm_pages] epoch << 32 | victim index (| paired bit)
+  // lv_remap's tags (0xFFFFFFFF between calls): the first entry of a call naming a
+  // block or a location
+  uint32_t* rtag_blk;     // [S][maxB]
+  uint32_t* rtag_hbm;     // [hbm_pages]
+  uint32_t* rtag_host;    // [host_pages]
 };
 
 __host__ __device__ inline uint32_t owner_key(int32_t sid, int32_t blk) {
@@ -123,8 +130,9 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
                             const long long* counts_dev = nullptr, long long max_units = 0,
                             const EventPair* ev = nullptr, const long long* sid_dev = nullptr,
                             const CopyOffload* off = nullptr, int gate = 0);
-cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, int32_t epoch,
-                         cudaStream_t s, int num_sms, int per_thread);
+// n <= 2^32 - 2 (entry indices are the 32-bit tags of the two passes)
+cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, cudaStream_t s,
+                         int num_sms, int per_thread);
 cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cudaStream_t s);
 cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32_t* pages,
                           int32_t* count, cudaStream_t s, const long long* gate = nullptr,

@@ -357,6 +357,10 @@ __device__ __forceinline__ unsigned long long session_key(const DevPool& p, int3
 }
 
 constexpr int kCensusThreads = 256;
+// Up to this many sessions every emit CTA finds its session's place by reading all
+// S keys itself; above it, k_rank_prefix computes every place once, between the
+// census and the emission (S^2 key comparisons, but S^2 / 256 key reads).
+constexpr int kEmitScanMax = 256;
 
 // One CTA per session: its key and its count of HBM-resident blocks.
 __global__ void __launch_bounds__(kCensusThreads)
@@ -364,7 +368,13 @@ k_rank_census(DevPool p, long long now_us, bool fallback) {
   pdl_entry();
   const int32_t s = blockIdx.x;
   __shared__ unsigned long long key;
-  if (threadIdx.x == 0) key = session_key(p, s, now_us, fallback);
+  if (threadIdx.x == 0) {
+    key = session_key(p, s, now_us, fallback);
+    if (p.S > kEmitScanMax) {       // k_rank_prefix accumulates into these
+      p.sbefore[s] = 0;
+      if (s == 0) p.ctl[C_RANK_TOTAL] = 0;
+    }
+  }
   __syncthreads();
   if (key == 0ull) {
     if (threadIdx.x == 0) { p.skey[s] = 0ull; p.scount[s] = 0; }
@@ -379,6 +389,51 @@ k_rank_census(DevPool p, long long now_us, bool fallback) {
   if (threadIdx.x == 0) {
     p.skey[s] = key;
     p.scount[s] = (int32_t)total;
+  }
+}
+
+constexpr int kPrefixTile = 128;    // sessions placed by one CTA (one per thread)
+constexpr int kPrefixChunk = 256;   // keys staged by one CTA in shared memory
+
+// The place of every candidate session in the victim order, for S > kEmitScanMax:
+// sbefore[s] = the resident blocks of the candidate sessions with a larger key
+// (keys are distinct).  CTA (x, y) compares the sessions of tile x with the keys
+// of chunk y, read once into shared memory (every thread reads the same key at
+// once: a broadcast), and adds its partial sums; the CTAs of tile 0 also add up
+// all candidates' blocks into C_RANK_TOTAL.  The census zeroed both.
+__global__ void __launch_bounds__(kPrefixTile)
+k_rank_prefix(DevPool p) {
+  pdl_entry();   // the census is complete and visible
+  __shared__ unsigned long long kc[kPrefixChunk];
+  __shared__ int32_t cc[kPrefixChunk];
+  __shared__ long long part[kPrefixTile / 32];
+  const int32_t j0 = blockIdx.y * kPrefixChunk;
+  const int32_t nj = min(kPrefixChunk, p.S - j0);
+  for (int32_t j = threadIdx.x; j < nj; j += kPrefixTile) {
+    const unsigned long long kj = p.skey[j0 + j];
+    kc[j] = kj;
+    cc[j] = kj ? p.scount[j0 + j] : 0;
+  }
+  __syncthreads();
+  const int32_t s = blockIdx.x * kPrefixTile + threadIdx.x;
+  const unsigned long long key = s < p.S ? p.skey[s] : 0ull;
+  if (key != 0ull) {
+    long long before = 0;
+#pragma unroll 8
+    for (int32_t j = 0; j < nj; ++j) before += kc[j] > key ? cc[j] : 0;
+    if (before) atomicAdd(reinterpret_cast<unsigned long long*>(&p.sbefore[s]), (unsigned long long)before);
+  }
+  if (blockIdx.x == 0) {
+    long long t = 0;
+    for (int32_t j = threadIdx.x; j < nj; j += kPrefixTile) t += cc[j];
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = t;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      long long all = 0;
+      for (int w = 0; w < kPrefixTile / 32; ++w) all += part[w];
+      if (all) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_RANK_TOTAL]), (unsigned long long)all);
+    }
   }
 }
 
@@ -399,16 +454,21 @@ k_rank_emit(DevPool p, long long k, const long long* k_dev, bool fallback, long 
   const unsigned long long key = p.skey[sid];
   if (key == 0ull && sid != 0) return;
   if (k_dev) k = *k_dev;   // k decided on the device (lv_make_resident)
-  long long before = 0, all = 0;
-  for (int32_t j = threadIdx.x; j < p.S; j += kEmitThreads) {
-    const unsigned long long kj = p.skey[j];
-    const long long cj = kj ? p.scount[j] : 0;
-    all += cj;
-    before += kj > key ? cj : 0;
-  }
   long long off, total;
-  block_excl_scan<kEmitThreads>(before, &off);
-  block_excl_scan<kEmitThreads>(all, &total);
+  if (p.S > kEmitScanMax) {      // placed by k_rank_prefix
+    off = key ? p.sbefore[sid] : 0;
+    total = p.ctl[C_RANK_TOTAL];
+  } else {
+    long long before = 0, all = 0;
+    for (int32_t j = threadIdx.x; j < p.S; j += kEmitThreads) {
+      const unsigned long long kj = p.skey[j];
+      const long long cj = kj ? p.scount[j] : 0;
+      all += cj;
+      before += kj > key ? cj : 0;
+    }
+    block_excl_scan<kEmitThreads>(before, &off);
+    block_excl_scan<kEmitThreads>(all, &total);
+  }
   const long long n_out = k < total ? k : total;
   if (sid == 0 && threadIdx.x == 0) {
     p.ctl[C_SEL_COUNT] = n_out;
@@ -1098,93 +1158,115 @@ __global__ void k_selftest_wait(long long* ctl, long long limit_ns) {
 }
 
 // ---------------------------------------------------------------- commit
+// lv_remap runs in two passes.  Pass 1 (k_remap_tag) tags, for every entry i, its
+// block and its new location with i by non-returning minimum reductions, so a block
+// or location named by several entries of the call ends up tagged with the first
+// of them in list order.  Pass 2 (k_remap_commit) reads the tags back with every
+// other independent read of the entry: only the entry whose index a tag holds may
+// use that block or location (the others are double maps), and that entry puts the
+// tag back to kTagFree, so the tags are free again once the call has run.  Nothing
+// in either pass waits for a returning atomic.
 constexpr int kRemapThreads = 256;
+constexpr uint32_t kTagFree = 0xFFFFFFFFu;
 
-// The reads of one entry that do not depend on a check.
-struct RemapRead {
+// The entry's block and new location, with the range checks both passes share.
+struct RemapSlots {
   lv_remap_entry x;
-  size_t ti;            // table index (0 when out of range)
-  int32_t old;          // the block's current location
-  int32_t g;            // its clean-copy slot (inclusive tiers), or -1
-  int32_t nb;           // blocks of its session
-  uint32_t old_owner;   // owner word of the current location
-  bool in_range;
+  size_t ti;            // table index (valid when blk_ok)
+  uint32_t* ltag;       // the new location's tag word, or nullptr when loc is out of range
+  uint32_t* lown;       // its owner word
+  bool blk_ok;          // sid and blk inside the table
 };
+
+__device__ __forceinline__ RemapSlots remap_slots(const DevPool& p, const lv_remap_entry& x) {
+  RemapSlots r;
+  r.x = x;
+  r.blk_ok = x.sid >= 0 && x.sid < p.S && x.blk >= 0 && x.blk < p.maxB;
+  r.ti = r.blk_ok ? (size_t)x.sid * p.maxB + x.blk : 0;
+  r.ltag = nullptr;
+  r.lown = nullptr;
+  if (x.loc >= 0 && x.loc < p.hbm_pages) {
+    r.ltag = p.rtag_hbm + x.loc;
+    r.lown = p.own_hbm + x.loc;
+  } else if (x.loc <= -2 && -(long long)x.loc - 2 < p.host_pages) {
+    r.ltag = p.rtag_host + (-(long long)x.loc - 2);
+    r.lown = p.own_host + (-(long long)x.loc - 2);
+  }
+  return r;
+}
+
+__global__ void __launch_bounds__(kRemapThreads)
+k_remap_tag(DevPool p, const lv_remap_entry* __restrict__ e, long long n) {
+  pdl_entry();
+  const long long stride = (long long)gridDim.x * kRemapThreads;
+  for (long long i = blockIdx.x * (long long)kRemapThreads + threadIdx.x; i < n; i += stride) {
+    const RemapSlots r = remap_slots(p, e[i]);
+    if (r.blk_ok) atomicMin(&p.rtag_blk[r.ti], (uint32_t)i);
+    if (r.ltag) atomicMin(r.ltag, (uint32_t)i);
+  }
+}
 
 struct RemapCounts {
   int ok, hbm, host, clean;
 };
 
-__device__ __forceinline__ void remap_read_entry(const DevPool& p, const lv_remap_entry* e, long long i,
-                                                 long long n, RemapRead& r) {
-  r.x = i < n ? e[i] : lv_remap_entry{-1, -1, -1};
-  r.in_range = i < n && r.x.sid >= 0 && r.x.sid < p.S && r.x.blk >= 0 && r.x.blk < p.maxB;
-  r.ti = r.in_range ? (size_t)r.x.sid * p.maxB + r.x.blk : 0;
+// The reads of one entry in pass 2 that depend on nothing but the entry.
+struct RemapRead {
+  RemapSlots r;
+  uint32_t btag, ltag;  // the tags of its block and of its new location
+  uint32_t got;         // owner word of the new location
+  int32_t old;          // the block's current location
+  int32_t g;            // its clean-copy slot (inclusive tiers), or -1
+  int32_t nb;           // blocks of its session
+};
+
+__device__ __forceinline__ void remap_read(const DevPool& p, const lv_remap_entry* e, long long i,
+                                           long long n, RemapRead& q) {
+  q.r = remap_slots(p, i < n ? e[i] : lv_remap_entry{-1, -1, -1});
+  const bool b = i < n && q.r.blk_ok;
+  const bool l = i < n && q.r.ltag != nullptr;
+  q.btag = b ? p.rtag_blk[q.r.ti] : kTagFree;
+  q.old = b ? p.table[q.r.ti] : -1;
+  q.g = (b && p.incl) ? p.shadow[q.r.ti] : -1;
+  q.nb = b ? nblocks_of(p, q.r.x.sid) : 0;
+  q.ltag = l ? *q.r.ltag : kTagFree;
+  q.got = l ? *q.r.lown : kOwnerNone;
 }
 
-__device__ __forceinline__ void remap_read_table(const DevPool& p, RemapRead& r) {
-  r.old = r.in_range ? p.table[r.ti] : -1;
-  r.g = (r.in_range && p.incl) ? p.shadow[r.ti] : -1;
-  r.nb = r.in_range ? nblocks_of(p, r.x.sid) : 0;
-}
-
-__device__ __forceinline__ void remap_read_owner(const DevPool& p, RemapRead& r) {
-  const long long old_slot = -(long long)r.old - 2;
-  r.old_owner = kOwnerNone;
-  if (r.old >= 0 && r.old < p.hbm_pages) r.old_owner = p.own_hbm[r.old];
-  else if (r.old <= -2 && old_slot < p.host_pages) r.old_owner = p.own_host[old_slot];
-}
-
-// The block's epoch mark: one accepted entry per block per call.  Returns the
-// entry's error so far (a returning atomic; the caller issues every entry's
-// mark before it looks at any result).
-__device__ __forceinline__ int remap_mark(const DevPool& p, const RemapRead& r, int32_t epoch,
-                                          int32_t& seen) {
-  if (!r.in_range || r.x.blk >= r.nb) return LV_ERR_BOUNDS;
-  seen = atomicExch(&p.mark[r.ti], epoch);
-  return 0;
-}
-
-// The new location must be a reservation nobody owns yet: one CAS checks and
-// takes it.  Issued for every entry that passed its mark, before any result is read.
-__device__ __forceinline__ int remap_claim(const DevPool& p, const RemapRead& r, int err,
-                                           uint32_t& got) {
-  if (err) return err;
-  const lv_remap_entry& x = r.x;
-  const uint32_t key = owner_key(x.sid, x.blk);
-  if (x.loc >= 0) {
-    if (x.loc >= p.hbm_pages) return LV_ERR_BOUNDS;
-    got = atomicCAS(&p.own_hbm[x.loc], kOwnerReserved, key);
-  } else if (x.loc <= -2) {
-    if (-(long long)x.loc - 2 >= p.host_pages) return LV_ERR_BOUNDS;
-    got = atomicCAS(&p.own_host[-(long long)x.loc - 2], kOwnerReserved, key);
-  } else {
-    return LV_ERR_BOUNDS;
+// Releases the tags this entry holds and judges it: 0, or the status to report.
+__device__ __forceinline__ int remap_judge(const DevPool& p, const RemapRead& q, long long i) {
+  const uint32_t me = (uint32_t)i;
+  const bool own_b = q.r.blk_ok && q.btag == me;
+  const bool own_l = q.r.ltag != nullptr && q.ltag == me;
+  if (own_b) p.rtag_blk[q.r.ti] = kTagFree;
+  if (own_l) *q.r.ltag = kTagFree;
+  const lv_remap_entry& x = q.r.x;
+  if (!q.r.blk_ok || x.blk >= q.nb || q.r.ltag == nullptr) return LV_ERR_BOUNDS;
+  if (!own_b || !own_l) return LV_ERR_DOUBLE_MAP;   // the block or the location twice in the call
+  if (q.got != kOwnerReserved) {
+    // a host location already owned by this block is fine only as its own clean copy
+    const long long h = -(long long)x.loc - 2;
+    if (!(x.loc <= -2 && p.incl && (long long)q.g == h && q.got == owner_key(x.sid, x.blk)))
+      return LV_ERR_DOUBLE_MAP;
   }
   return 0;
 }
 
-// Judges the claim and applies the entry: table, clean copy, old location.
-__device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& r, int err,
-                                            uint32_t got, long long i, RemapCounts& c) {
-  const lv_remap_entry& x = r.x;
-  const int32_t old = r.old, g = r.g;
+// Applies an accepted entry: table, new owner, clean copy, old location.  The old
+// location's owner word, read after the table, only checks consistency.
+__device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& q, uint32_t old_owner,
+                                            long long i, RemapCounts& c) {
+  const lv_remap_entry& x = q.r.x;
+  const int32_t old = q.old, g = q.g;
   const long long old_slot = -(long long)old - 2;
   const bool old_hbm = old >= 0 && old < p.hbm_pages;
   const bool old_host = old <= -2 && old_slot < p.host_pages;
   const long long h = -(long long)x.loc - 2;
   const uint32_t key = owner_key(x.sid, x.blk);
-  if (!err && got != kOwnerReserved) {
-    // a host location already owned by this block is fine only as its own clean copy
-    if (!(x.loc <= -2 && p.incl && (long long)g == h && got == key)) err = LV_ERR_DOUBLE_MAP;
-  }
-  if (err) {
-    set_error(p.ctl, err, i);
-    return;
-  }
-  p.table[r.ti] = x.loc;
+  p.table[q.r.ti] = x.loc;
+  *q.r.lown = key;
   if (x.loc <= -2 && g >= 0) {          // the copy becomes the location, or goes
-    p.shadow[r.ti] = -1;
+    p.shadow[q.r.ti] = -1;
     c.clean -= 1;
     if ((long long)g != h) {
       p.own_host[g] = kOwnerNone;
@@ -1194,13 +1276,13 @@ __device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& r
   }
   // the old location belongs to this block alone (one entry per block per call)
   if (old_hbm || old_host) {
-    if (r.old_owner != key) set_error(p.ctl, LV_ERR_STATE, i);
+    if (old_owner != key) set_error(p.ctl, LV_ERR_STATE, i);
     if (old_hbm) {
       p.own_hbm[old] = kOwnerNone;
       atomicAnd(&p.bits_hbm[old >> 5], ~(1u << (old & 31)));
       c.hbm += 1;
     } else if (p.incl && x.loc >= 0) {   // back in HBM: the host slot stays as its clean copy
-      p.shadow[r.ti] = (int32_t)old_slot;
+      p.shadow[q.r.ti] = (int32_t)old_slot;
       c.clean += 1;
     } else {
       p.own_host[old_slot] = kOwnerNone;
@@ -1211,55 +1293,46 @@ __device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& r
   c.ok += 1;
 }
 
-// Each thread commits E entries, i0, i0 + stride, ... (stride = the grid's
-// threads, so a warp's entries stay contiguous).  The allocation counts and the
-// commit counter change by block totals (one atomic per block and counter).
-// Inclusive tiers: a host location may be the block's own clean copy; a block
-// committed to HBM from the host tier keeps its slot as its clean copy; a
-// block committed to another host slot loses its copy.
-//
-// The kernel is bound by the latency of dependent scattered accesses (entry ->
-// table entry -> owner of the old location -> epoch mark -> claim of the new
-// location), so each step is issued for all E entries of the thread before any
-// of its results is used: every read that does not depend on a check, then
-// every mark, then every claim, then the stores.  E chains then wait together.  The early
-// reads are race-free within one call: a block has at most one accepted entry
-// (the epoch mark), a location freed by one entry is never the new location of
-// another (new locations are reservations), and another entry can take an
-// owned location only through a CAS, which then fails.  A thread's own
-// entries apply in order, so a duplicate among them meets the epoch mark too.
+// Pass 2.  Each thread commits E entries, i0, i0 + stride, ... (stride = the grid's
+// threads, so a warp's entries stay contiguous).  All E entries' independent reads
+// are issued before any result is used, then the old locations' owner words, then
+// the stores: two dependent rounds of reads per entry.  The reads are race-free
+// within one call: an accepted entry is the only one on its block and on its new
+// location, a location freed by one entry is never the new location of another
+// (new locations are reservations, old ones are owned), and a rejected entry
+// writes nothing but its own tags.  The allocation counts and the commit counter
+// change by block totals (one atomic per block and counter).  Inclusive tiers: a
+// host location may be the block's own clean copy; a block committed to HBM from
+// the host tier keeps its slot as its clean copy; a block committed to another
+// host slot loses its copy.
 template <int E>
 __global__ void __launch_bounds__(kRemapThreads)
-k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t epoch) {
+k_remap_commit(DevPool p, const lv_remap_entry* __restrict__ e, long long n) {
+  pdl_entry();   // every tag of pass 1 is in place
   const long long stride = (long long)gridDim.x * kRemapThreads;
   const long long i0 = blockIdx.x * (long long)kRemapThreads + threadIdx.x;
-  RemapRead r[E];
+  RemapRead q[E];
 #pragma unroll
-  for (int j = 0; j < E; ++j) remap_read_entry(p, e, i0 + j * stride, n, r[j]);
-#pragma unroll
-  for (int j = 0; j < E; ++j) remap_read_table(p, r[j]);
-#pragma unroll
-  for (int j = 0; j < E; ++j) remap_read_owner(p, r[j]);
-  // the atomics of all E entries: every mark, then every claim, each group in flight
-  // together; a thread's own duplicate meets the mark of its earlier entry
+  for (int j = 0; j < E; ++j) remap_read(p, e, i0 + j * stride, n, q[j]);
   int err[E];
-  int32_t seen[E];
-  uint32_t got[E];
+  uint32_t old_owner[E];
 #pragma unroll
   for (int j = 0; j < E; ++j) {
-    seen[j] = 0;
-    err[j] = i0 + j * stride < n ? remap_mark(p, r[j], epoch, seen[j]) : -1;
-  }
-#pragma unroll
-  for (int j = 0; j < E; ++j) {
-    if (err[j] == 0 && seen[j] == epoch) err[j] = LV_ERR_DOUBLE_MAP;   // same block twice
-    got[j] = kOwnerReserved;
-    if (err[j] >= 0) err[j] = remap_claim(p, r[j], err[j], got[j]);
+    const long long i = i0 + j * stride;
+    err[j] = i < n ? remap_judge(p, q[j], i) : -1;
+    old_owner[j] = kOwnerNone;
+    if (err[j] == 0) {
+      const int32_t old = q[j].old;
+      if (old >= 0 && old < p.hbm_pages) old_owner[j] = p.own_hbm[old];
+      else if (old <= -2 && -(long long)old - 2 < p.host_pages) old_owner[j] = p.own_host[-(long long)old - 2];
+    }
   }
   RemapCounts c{0, 0, 0, 0};
 #pragma unroll
-  for (int j = 0; j < E; ++j)
-    if (err[j] >= 0) remap_apply(p, r[j], err[j], got[j], i0 + j * stride, c);
+  for (int j = 0; j < E; ++j) {
+    if (err[j] > 0) set_error(p.ctl, err[j], i0 + j * stride);
+    else if (err[j] == 0) remap_apply(p, q[j], old_owner[j], i0 + j * stride, c);
+  }
   // block totals: warp sums, one shared atomic per warp, one global atomic per block
   __shared__ int tot[4];
   if (threadIdx.x < 4) tot[threadIdx.x] = 0;
@@ -1704,10 +1777,10 @@ cudaError_t launch_session_set(const DevPool& p, const lv_session_state* in, int
 // A launch that lets the kernel be scheduled while the previous kernel on `s`
 // still runs; the kernel must begin with pdl_entry().
 template <typename... KArgs, typename... Args>
-cudaError_t launch_pdl(void (*kernel)(KArgs...), unsigned grid, unsigned block, size_t smem,
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, unsigned block, size_t smem,
                        cudaStream_t s, Args&&... args) {
   cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(grid);
+  cfg.gridDim = grid;
   cfg.blockDim = dim3(block);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
@@ -1730,6 +1803,12 @@ cudaError_t launch_select(const DevPool& p, int64_t now_us, int64_t k, bool fall
   cudaError_t e = launch_pdl(k_rank_census, (unsigned)p.S, kCensusThreads, 0, s, p, (long long)now_us,
                              fallback);
   if (e != cudaSuccess) return e;
+  if (p.S > kEmitScanMax) {
+    const dim3 grid((unsigned)((p.S + kPrefixTile - 1) / kPrefixTile),
+                    (unsigned)((p.S + kPrefixChunk - 1) / kPrefixChunk));
+    e = launch_pdl(k_rank_prefix, grid, kPrefixTile, 0, s, p);
+    if (e != cudaSuccess) return e;
+  }
   e = launch_pdl(k_rank_emit, (unsigned)p.S, kEmitThreads, 0, s, p, (long long)k, k_dev, fallback,
                  count_dev, out);
   if (e != cudaSuccess) return e;
@@ -1965,18 +2044,22 @@ cudaError_t launch_exchange_plan(const DevPool& p, const lv_victim* v, int64_t n
   return cudaGetLastError();
 }
 
-cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, int32_t epoch,
-                         cudaStream_t s, int num_sms, int per_thread) {
+cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, cudaStream_t s,
+                         int num_sms, int per_thread) {
   if (n <= 0) return cudaSuccess;
+  const long long resident = (long long)(num_sms > 0 ? num_sms : 1) * 2048;
+  cudaError_t err = launch_pdl(k_remap_tag, blocks_for(n, kRemapThreads, resident / kRemapThreads),
+                               kRemapThreads, 0, s, p, e, (long long)n);
+  if (err != cudaSuccess) return err;
   // one entry per thread while the GPU holds every thread at once; beyond that, up
   // to four entries per thread so that their reads overlap
-  const long long resident = (long long)(num_sms > 0 ? num_sms : 1) * 2048;
   int E = per_thread;
   if (E != 1 && E != 2 && E != 4) E = n <= resident ? 1 : (n <= 2 * resident ? 2 : 4);
   const unsigned grid = blocks_for((n + E - 1) / E, kRemapThreads, 1ll << 30);
-  if (E == 1) k_remap<1><<<grid, kRemapThreads, 0, s>>>(p, e, n, epoch);
-  else if (E == 2) k_remap<2><<<grid, kRemapThreads, 0, s>>>(p, e, n, epoch);
-  else k_remap<4><<<grid, kRemapThreads, 0, s>>>(p, e, n, epoch);
+  if (E == 1) err = launch_pdl(k_remap_commit<1>, grid, kRemapThreads, 0, s, p, e, (long long)n);
+  else if (E == 2) err = launch_pdl(k_remap_commit<2>, grid, kRemapThreads, 0, s, p, e, (long long)n);
+  else err = launch_pdl(k_remap_commit<4>, grid, kRemapThreads, 0, s, p, e, (long long)n);
+  if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
 

@@ -31,7 +31,7 @@ LV_SELECT_FALLBACK = 1
 LV_POLICY_NEXT_USE, LV_POLICY_LRU = 0, 1
 LV_TIERS_EXCLUSIVE, LV_TIERS_INCLUSIVE = 0, 1
 LV_RESIDENT_ASYNC_COPY = 2
-LV_VERSION = 2                     # include/lv.h
+LV_VERSION = 3                     # include/lv.h
 LV_MODE_ASYNC = 16
 LV_RUNNING, LV_IMMEDIATE, LV_RESP_OPEN, LV_DONE_VALID = 1, 2, 4, 8
 (LV_EV_TURN_BEGIN, LV_EV_TURN_END, LV_EV_PLAYBACK, LV_EV_SPEECH_START, LV_EV_BARGE_IN,
@@ -70,10 +70,6 @@ class lv_controller_desc(ctypes.Structure):
                 ("cap_pages", ctypes.c_int64), ("mode", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
-class lv_probe_mix(ctypes.Structure):
-    _fields_ = [(n, ctypes.c_int32) for n in ("loads", "atomics", "stores", "reductions")]
-
-
 class lv_controller_counters(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int64) for n in ("admitted", "completed", "waited", "given_up",
                                                "cancelled", "hits", "victims", "pages_in")]
@@ -108,7 +104,8 @@ class lv_rank_params(ctypes.Structure):
     _fields_ = [("num_sessions", ctypes.c_int32), ("max_blocks", ctypes.c_int32),
                 ("page_tokens", ctypes.c_int32), ("within_order", ctypes.c_int32),
                 ("t_play_mode", ctypes.c_int32), ("flags", ctypes.c_uint32),
-                ("reply_prior_us", ctypes.c_int64), ("unit_us", ctypes.c_int64)]
+                ("reply_prior_us", ctypes.c_int64), ("unit_us", ctypes.c_int64),
+                ("policy", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
 class lv_sched_params(ctypes.Structure):
@@ -164,7 +161,6 @@ def _load():
         "lv_join": [vp, vp],
         "lv_evict": [vp, i64, i64, u32, vp, vp, vp, vp],
         "lv_page_checksums": [vp, vp, i64, vp, vp],
-        "lv_probe_scattered": [ctypes.POINTER(lv_probe_mix), vp, i64, i64, vp, vp],
         "lv_controller_create": [vp, ctypes.POINTER(lv_controller_desc), ctypes.POINTER(vp)],
         "lv_controller_destroy": [vp, vp],
         "lv_controller_tick": [vp, i64, vp],
@@ -219,7 +215,7 @@ EXPORTED = ("lv_pool_create", "lv_pool_destroy", "lv_pool_host_ptr", "lv_pool_im
             "lv_get_stats", "lv_clear_error", "lv_status_str", "lv_version",
             "lv_select_victims_noalloc", "lv_timing_enable", "lv_timing_read", "lv_pack_pages",
             "lv_unpack_pages", "lv_pool_host_device_ptr", "lv_schedule", "lv_inject_fault",
-            "lv_selftest_wait", "lv_turn", "lv_evict", "lv_join", "lv_page_checksums", "lv_probe_scattered",
+            "lv_selftest_wait", "lv_turn", "lv_evict", "lv_join", "lv_page_checksums",
             "lv_controller_create", "lv_controller_destroy", "lv_controller_tick",
             "lv_controller_speech", "lv_controller_turn_begin", "lv_controller_turn_loaded",
             "lv_controller_records", "lv_controller_counters_get")
@@ -357,13 +353,6 @@ def lv_evict(pool, now_us, k, flags=0, victims_out=None, slots_out=None, result_
 def lv_page_checksums(pool, pages, n, sums_out, stream=None):
     _check(_lib.lv_page_checksums(pool, ptr(pages), n, ptr(sums_out), stream_handle(stream)),
            "lv_page_checksums")
-
-
-def lv_probe_scattered(mix, array, words, threads, sink=None, stream=None):
-    """mix = (loads, atomics, stores, reductions) per thread."""
-    m = lv_probe_mix(*(int(x) for x in mix))
-    _check(_lib.lv_probe_scattered(ctypes.byref(m), ptr(array), words, threads, ptr(sink),
-                                   stream_handle(stream)), "lv_probe_scattered")
 
 
 def lv_controller_create(pool, link_bytes_per_us, lead_prior_us, cap_pages=None, mode=LV_MODE_AUTO):

@@ -73,8 +73,9 @@ int main(void) {
   printf("sizeof lv_controller_desc %zu\n", sizeof(lv_controller_desc));
   printf("sizeof lv_controller_counters %zu\n", sizeof(lv_controller_counters));
   printf("sizeof lv_controller_record %zu\n", sizeof(lv_controller_record));
-  printf("sizeof lv_probe_mix %zu\n", sizeof(lv_probe_mix));
-  F(lv_probe_mix, loads); F(lv_probe_mix, atomics); F(lv_probe_mix, stores); F(lv_probe_mix, reductions);
+  printf("sizeof lv_rank_params %zu\n", sizeof(lv_rank_params));
+  F(lv_rank_params, num_sessions); F(lv_rank_params, flags); F(lv_rank_params, reply_prior_us);
+  F(lv_rank_params, unit_us); F(lv_rank_params, policy); F(lv_rank_params, reserved);
   F(lv_controller_record, kind); F(lv_controller_record, sid); F(lv_controller_record, start_us);
   F(lv_controller_record, finish_us); F(lv_controller_record, deadline_us); F(lv_controller_record, n);
   F(lv_controller_record, data_offset);
@@ -116,9 +117,9 @@ int main(void) {
     assert got["lv_controller_desc"] == ctypes.sizeof(lv.lv_controller_desc)
     assert got["lv_controller_counters"] == ctypes.sizeof(lv.lv_controller_counters)
     assert got["lv_controller_record"] == lv.CTL_RECORD_DTYPE.itemsize
-    assert got["lv_probe_mix"] == ctypes.sizeof(lv.lv_probe_mix)
-    for name, _ in lv.lv_probe_mix._fields_:
-        assert getattr(lv.lv_probe_mix, name).offset == got[f"lv_probe_mix.{name}"][0], name
+    assert got["lv_rank_params"] == ctypes.sizeof(lv.lv_rank_params) == 48
+    for name in ("num_sessions", "flags", "reply_prior_us", "unit_us", "policy", "reserved"):
+        assert getattr(lv.lv_rank_params, name).offset == got[f"lv_rank_params.{name}"][0], name
     for name in lv.CTL_RECORD_DTYPE.names:
         assert lv.CTL_RECORD_DTYPE.fields[name][1] == got[f"lv_controller_record.{name}"][0], name
     for name, _ in lv.lv_turn_desc._fields_:
@@ -144,7 +145,7 @@ def test_status_strings_and_argument_checks(lib):
     from paper_2606_22983_gb300 import lv
     for code, name in lv.STATUS_NAMES.items():
         assert lv.lv_status_str(code) == name
-    assert lv.lv_version() == lv.LV_VERSION == 2
+    assert lv.lv_version() == lv.LV_VERSION == 3
     # argument checks that need no device: a NULL descriptor / NULL out pointer
     L = lv.lib()
     h = ctypes.c_void_p()

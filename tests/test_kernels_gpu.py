@@ -362,40 +362,6 @@ def test_largest_pool_shape_and_ids():
         pool.close()
 
 
-def test_scattered_access_probe():
-    """lv_probe_scattered does what its mix says on a small array, and refuses bad
-    arguments: loads change nothing, stores and atomics write thread indices,
-    reductions clear the low four bits of the words they touch."""
-    import torch
-    from paper_2606_22983_gb300 import lv
-    words, threads = 1 << 12, 300
-    a = torch.full((words,), -1, dtype=torch.int32, device="cuda")
-    lv.lv_probe_scattered((8, 0, 0, 0), a, words, threads)
-    torch.cuda.synchronize()
-    assert bool((a == -1).all())
-    lv.lv_probe_scattered((0, 0, 0, 8), a, words, threads)
-    torch.cuda.synchronize()
-    v = a.cpu().numpy().view(np.uint32)
-    assert set(np.unique(v).tolist()) == {0xFFFFFFF0, 0xFFFFFFFF}
-    touched = int((v == 0xFFFFFFF0).sum())
-    assert 0.5 * threads * 8 < touched <= threads * 8     # spread over the array
-    lv.lv_probe_scattered((0, 8, 0, 0), a, words, threads)
-    lv.lv_probe_scattered((0, 0, 8, 0), a, words, threads)
-    torch.cuda.synchronize()
-    v = a.cpu().numpy().view(np.uint32)
-    assert int((v < threads).sum()) == touched and int((v == 0xFFFFFFFF).sum()) == words - touched
-    # a mixed launch touches as many words as its requests allow
-    b = torch.full((words,), -1, dtype=torch.int32, device="cuda")
-    lv.lv_probe_scattered((2, 2, 2, 1), b, words, threads)
-    torch.cuda.synchronize()
-    changed = int((b != -1).sum())
-    assert 0.5 * threads * 5 < changed <= threads * 5
-    for mix, w, n in (((65, 0, 0, 0), words, threads), ((-1, 0, 0, 0), words, threads),
-                      ((8, 0, 0, 0), 3000, threads), ((8, 0, 0, 0), words, 0)):
-        with pytest.raises(Exception):
-            lv.lv_probe_scattered(mix, a, w, n)
-
-
 def test_turn_picks_the_first_candidate_with_host_blocks():
     """lv_turn with sid = -1: the first listed session that has a block in the host
     tier (else the first listed), then turn begin, make resident, turn end -- the
