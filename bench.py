@@ -171,16 +171,19 @@ def ours(args, torch):
         dev_events.append(torch.from_numpy(ev.view(np.uint8).copy()).to(pool.device))
     torch.cuda.synchronize()
 
+    # the clock sampler starts before the warm-up, so that its start-up (NVML
+    # initialisation) is over before the timed region; it samples throughout it
+    clocks = ClockSampler(local)
+    clocks.start()
     run_turns(gm, wl, 0, W, dev_events)                         # warm-up
     pool.sync()
+    time.sleep(0.5)
     p0, o0, i0 = _moved_pages(pool)
     lv.lv_timing_read(pool.handle, reset=True)
     lv.lv_timing_enable(pool.handle, True)
-    clocks = ClockSampler(local)
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
-    clocks.start()
     l0 = pool.launches
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
@@ -321,69 +324,166 @@ def ours(args, torch):
         }
     if line is not None and KO:
         line["overlap"] = overlap_measure(torch, pool, wl, W + 2 * K, KO)
+    if line is not None and args.directions:
+        line["directions"] = direction_legs(torch, pool, int(wl.t_us[-1]) + 1_000_000)
     if line is not None and args.micro:
         micro = kernel_micro(torch, pool, args.seed)
         line["ranker"] = micro.pop("ranker")
         line["scheduler"] = micro.pop("scheduler")
         line["hbm_kernels"] = micro
     pool.close()
+    if line is not None and args.five:
+        line["workloads"] = five_workloads(torch, args.seed)
     if line is not None and args.cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(args.cpu_seconds, args.seed)
+        line["cpu_baseline"] = cpu_baseline(args, args.cpu_seconds, args.seed)
     if dist:
         dist.destroy_process_group()
     return line
 
 
 OVERLAP_TURNS = 40
-REMAP_BYTES_PER_ENTRY = 52   # entry 12; read+write of: table 4+4, epoch 4+4, new owner 4+4, old owner 4+4, old bitmap 4+4
-# The scattered requests one k_remap entry makes when the micro commits every page to
-# the host tier: the old location's owner is loaded and cleared and its bitmap bit
-# reduced at a random position (pages are a random permutation); the epoch mark
-# (exchange) and the new slot's owner (CAS) are returning atomics, at consecutive
-# positions here (entries follow the victim order, slots ascend).  The entry, the
-# table word and the session's length are coalesced or cached loads and are left out.
-REMAP_REQUESTS = {"load": 1, "store": 1, "reduce": 1, "atomic": 2}
+# The commit's algorithmic bytes per entry: the entry 12; read and write of the table
+# word 4+4 and of the new location's owner word 4+4; write of the old location's owner
+# word 4; read and write of the old location's bitmap word 4+4.  The per-block epoch
+# mark (duplicate detection) and the read of the old location's owner word (a
+# consistency check) are the implementation's own and are not counted.
+REMAP_BYTES_PER_ENTRY = 40
+
+
+class ChecksumConsumer:
+    """Stands in for the engine's attention reads of resident KV: lv_page_checksums
+    over n resident pages (HBM-bound, every byte read once) issued on its own stream
+    through a second liblv pool over the same KV arrays, so that its reads never wait
+    for the first pool's copies.  ``top_up`` keeps a few calls queued, so it runs
+    without gaps while the other work is issued."""
+
+    def __init__(self, torch, pool, n_pages=4096, seed=0, depth=3):
+        from paper_2606_22983_gb300.pool import KVPool
+        self.torch = torch
+        self.stream = torch.cuda.Stream(device=pool.device)
+        elems = pool.P // 2                       # bf16 elements of one sub-page
+        self.cp = KVPool(layers=pool.L, kv_heads=1, head_dim=elems // pool.T, page_tokens=pool.T,
+                         max_sessions=1, max_blocks=1, hbm_pages=pool.hbm_pages, hbm_budget_pages=1,
+                         host_pages=0, device=pool.device, stream=self.stream, kv=pool.kv)
+        g = torch.Generator(device=pool.device).manual_seed(seed)
+        n = min(n_pages, pool.hbm_pages)
+        self.pages = torch.randperm(pool.hbm_pages, generator=g, device=pool.device)[:n].to(torch.int32)
+        self.n = n
+        self.sums = torch.empty(n, dtype=torch.int64, device=pool.device)
+        self.bytes_per_call = n * pool.J * pool.P
+        self.depth = depth
+        self.pending = []
+        self.ends = []
+        self.calls = 0
+        self.call_ms = 1.0
+
+    def issue(self):
+        from paper_2606_22983_gb300 import lv
+        lv.lv_page_checksums(self.cp.handle, self.pages, self.n, self.sums, self.stream)
+        ev = self.torch.cuda.Event(enable_timing=True)
+        ev.record(self.stream)
+        self.pending.append(ev)
+        self.ends.append(ev)
+        self.calls += 1
+
+    def start(self):
+        """Starts a window: the consumer's calls from now on are counted."""
+        self.ends = []
+        self.top_up()
+
+    def keep_busy_until(self, ev):
+        """Keeps calls queued until event ``ev`` (recorded on another stream) has
+        completed, then returns the end events of the window's calls."""
+        while not ev.query():
+            self.top_up()
+            time.sleep(0.0002)
+        self.top_up()
+        return list(self.ends)
+
+    def rate_within(self, ends, t0, t1):
+        """The consumer's GB/s within the window [t0, t1] of another stream (after a
+        synchronize): calls completed in it, the call running at t1 counted by the
+        part of it inside the window; and whether the consumer ran past t1."""
+        T = t0.elapsed_time(t1)
+        x = [t0.elapsed_time(e) for e in ends]
+        done = sum(1 for v in x if 0 < v <= T)
+        later = [v for v in x if v > T]
+        if later:
+            prev = max([v for v in x if v <= T], default=0.0)
+            span = later[0] - prev
+            if span > 0:
+                done += (T - prev) / span
+        return done * self.bytes_per_call / (T / 1e3) / 1e9, bool(later)
+
+    def top_up(self, *_):
+        self.pending = [e for e in self.pending if not e.query()]
+        while len(self.pending) < self.depth:
+            self.issue()
+
+    def alone_gbs(self, reps=10):
+        torch = self.torch
+        for _ in range(2):
+            self.issue()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(self.stream)
+        for _ in range(reps):
+            self.issue()
+        b.record(self.stream)
+        torch.cuda.synchronize()
+        self.call_ms = a.elapsed_time(b) / reps
+        return self.bytes_per_call * reps / (a.elapsed_time(b) / 1e3) / 1e9
+
+    def window(self):
+        """Starts counting: returns a closure that, after a synchronize, gives the
+        consumer's GB/s over the window."""
+        torch = self.torch
+        a = torch.cuda.Event(enable_timing=True)
+        a.record(self.stream)
+        c0 = self.calls
+
+        def done():
+            b = torch.cuda.Event(enable_timing=True)
+            b.record(self.stream)
+            torch.cuda.synchronize()
+            return (self.calls - c0) * self.bytes_per_call / (a.elapsed_time(b) / 1e3) / 1e9
+        return done
+
+    def close(self):
+        self.torch.cuda.synchronize()
+        self.cp.close()
 
 
 def overlap_measure(torch, pool, wl, first_turn, n_turns):
-    """Config 3's overlap of KV movement with serving work: a consumer standing in
-    for the engine's attention reads (a torch sum over 4096 resident pages, 6.4 GB,
-    on its own stream; not part of liblv) runs alone, then throughout n_turns
-    thinker turns moved by the zero-copy device-driven path (SM copies, async) and
-    then by the staged path (copy engines).  The consumer's pages may change under
+    """Config 3's overlap of KV movement with serving work: a consumer reading resident
+    KV at HBM speed (lv_page_checksums over 4096 resident pages, 6.4 GB per call, on
+    its own stream) runs alone, then throughout n_turns thinker turns moved by the
+    zero-copy device-driven path (SM copies, async) and then by the staged path (copy
+    engines).  The turns' calls are issued on a high-priority stream (the KV manager's
+    work gates the turns; the exchange copy's own stream has the highest priority), the
+    consumer's on a stream of normal priority.  The consumer's pages may change under
     it; its sums are not used."""
+    torch.cuda.synchronize()
+    with torch.cuda.stream(torch.cuda.Stream(device=pool.device, priority=-1)):
+        return _overlap_measure(torch, pool, wl, first_turn, n_turns)
+
+
+def _overlap_measure(torch, pool, wl, first_turn, n_turns):
     from paper_2606_22983_gb300 import lv
     from paper_2606_22983_gb300.manager import KVManager
-    n_pages = min(4096, pool.hbm_pages)
-    view = pool.kv[:, :n_pages, :].view(torch.int64)
-    read_bytes = view.numel() * 8
-    cs = torch.cuda.Stream(device=pool.device)
-
-    def consume(k):
-        with torch.cuda.stream(cs):
-            for _ in range(k):
-                view.sum(dtype=torch.int64)
-
-    ev = lambda: torch.cuda.Event(enable_timing=True)
-    consume(3)
-    torch.cuda.synchronize()
-    a0, a1 = ev(), ev()
-    a0.record(cs)
-    consume(20)
-    a1.record(cs)
-    torch.cuda.synchronize()
-    alone_ms = a0.elapsed_time(a1) / 20
-    out = {"consumer": "torch sum over 4096 resident pages (6.4 GB read), its own stream",
-           "consumer_alone_gbs": round(read_bytes / alone_ms / 1e6, 1)}
+    cons = ChecksumConsumer(torch, pool)
+    alone = cons.alone_gbs()
+    out = {"consumer": "lv_page_checksums over 4096 resident pages (6.4 GB read per call), "
+                       "its own stream and pool over the same KV arrays",
+           "consumer_alone_gbs": round(alone, 1), "consumer_alone_hbm_frac": round(alone / HBM_PEAK, 3)}
     page_bytes = pool.J * pool.P
-    per_turn = 3          # consumer reads queued per turn: it never runs dry
+    ev = lambda: torch.cuda.Event(enable_timing=True)
     turn = first_turn
     for label, driver, mode, async_copy in (("zero_copy_sm", "device", 0, True),
                                             ("staged_copy_engine", "exchange", 2, True)):
         gm = KVManager(pool, perms=wl.perms, rank_on="none", mode=mode, record=False,
                        driver=driver, async_copy=async_copy)
-        # warm-up of this driver (the staged path's stream-ordered staging pool grows
-        # during its first calls)
+        # warm-up of this driver (the staged path's staging runs grow during its first calls)
         run_turns(gm, wl, turn, turn + 10, None)
         turn += 10
         lv.lv_join(pool.handle, pool.stream)
@@ -396,30 +496,220 @@ def overlap_measure(torch, pool, wl, first_turn, n_turns):
         lv.lv_join(pool.handle, pool.stream)
         t1.record()
         torch.cuda.synchronize()
-        alone_gbs = (_moved_pages(pool)[0] - p0) * page_bytes / (t0.elapsed_time(t1) / 1e3) / 1e9
+        alone_ms = t0.elapsed_time(t1)
+        alone_gbs = (_moved_pages(pool)[0] - p0) * page_bytes / (alone_ms / 1e3) / 1e9
         turn += n_turns
-        # the turns with the consumer running throughout
+        # the turns with the consumer running throughout (kept topped up from the host
+        # until the turns are done)
         p0 = _moved_pages(pool)[0]
-        c0, c1 = ev(), ev()
-        c0.record(cs)
+        cons.start()
         t0.record()
-        calls = 0
         for i in range(turn, turn + n_turns):
-            consume(per_turn)
-            calls += per_turn
+            cons.top_up()
             run_turns(gm, wl, i, i + 1, None)
         lv.lv_join(pool.handle, pool.stream)
         t1.record()
-        c1.record(cs)
+        ends = cons.keep_busy_until(t1)
         torch.cuda.synchronize()
+        cons_gbs, covered = cons.rate_within(ends, t0, t1)
         turn += n_turns
         both_gbs = (_moved_pages(pool)[0] - p0) * page_bytes / (t0.elapsed_time(t1) / 1e3) / 1e9
-        cons_gbs = calls * read_bytes / (c0.elapsed_time(c1) / 1e3) / 1e9
         out[label] = {"turns": n_turns, "turns_alone_gbs": round(alone_gbs, 1),
                       "turns_with_consumer_gbs": round(both_gbs, 1),
                       "consumer_with_turns_gbs": round(cons_gbs, 1),
-                      "consumer_frac_kept": round(cons_gbs / out["consumer_alone_gbs"], 3)}
+                      "consumer_frac_kept": round(cons_gbs / alone, 3),
+                      "consumer_ran_throughout": covered}
+    cons.close()
     assert pool.sync(raise_on_error=False) == 0, "device error during the overlap turns"
+    return out
+
+
+def direction_legs(torch, pool, now_us, rounds=8, k_pages=1100):
+    """Each link direction on its own, device-driven: lv_evict of up to k_pages pages
+    (the ranking's first k, as many as the host tier has room for; offload only), then
+    preloads (lv_make_resident with LV_RESIDENT_PRELOAD) of the sessions with the most
+    host-tier blocks that fit in the free HBM pages, one after the other while one fits
+    (reload only, no eviction).  Copies run on the caller's stream; each call is timed
+    with CUDA events on it.  The peaks are same-run contiguous page-locked copies of the
+    mean call's byte count, D2H and H2D."""
+    from paper_2606_22983_gb300 import lv
+    from paper_2606_22983_gb300.harness import link_peaks
+    res = torch.zeros(lv.RESIDENT_DTYPE.itemsize, dtype=torch.uint8, device=pool.device)
+    page = pool.J * pool.P
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    off_ms, off_pages, in_ms, in_pages = [], [], [], []
+    t = now_us
+    for r in range(rounds):
+        t += 100_000
+        st0 = pool.stats()
+        k = min(k_pages, pool.host_pages - st0["host_allocated"] - 64)
+        if k < 64:
+            break
+        a, b = ev(), ev()
+        a.record()
+        lv.lv_evict(pool.handle, t, k, 0, None, None, res, pool.stream)
+        b.record()
+        b.synchronize()
+        st1 = pool.stats()
+        assert st1["bytes_in"] == st0["bytes_in"]
+        off_ms.append(a.elapsed_time(b))
+        off_pages.append((st1["bytes_out"] - st0["bytes_out"]) // page)
+        for _ in range(8):
+            free = pool.budget - st1["hbm_allocated"]
+            _, host = pool.counts()
+            fits = np.where(host <= free, host, -1)
+            sid = int(np.argmax(fits))
+            if fits[sid] <= 0:
+                break
+            a.record()
+            lv.lv_make_resident(pool.handle, sid, t, 0, lv.LV_RESIDENT_PRELOAD, -1, None, None, None,
+                                None, None, res, pool.stream)
+            b.record()
+            b.synchronize()
+            st2 = pool.stats()
+            assert st2["bytes_out"] == st1["bytes_out"]
+            in_ms.append(a.elapsed_time(b))
+            in_pages.append((st2["bytes_in"] - st1["bytes_in"]) // page)
+            st1 = st2
+    assert pool.sync(raise_on_error=False) == 0, "device error during the direction legs"
+    out_b, in_b = sum(off_pages) * page, sum(in_pages) * page
+    mean = int(min(max((out_b + in_b) / max(len(off_ms) + len(in_ms), 1), 1 << 26), 1 << 30))
+    peaks = link_peaks(pool, mean // 4096 * 4096)
+    res = {}
+    for name, nb, ms, peak in (("offload_only", out_b, off_ms, peaks["d2h"]),
+                               ("reload_only", in_b, in_ms, peaks["h2d"])):
+        if not ms:
+            continue
+        gbs = nb / (sum(ms) / 1e3) / 1e9
+        res[name] = {"calls": len(ms), "gb": round(nb / 1e9, 2), "gbs": round(gbs, 1),
+                     "blocks_per_s": round(nb / page / (sum(ms) / 1e3), 1),
+                     "peak_gbs": round(peak, 1), "frac": round(gbs / peak, 3),
+                     "ms_p50": round(float(np.median(ms)), 3)}
+    if "offload_only" in res:
+        res["offload_only"]["call"] = "lv_evict (rank, plan, out-only exchange copy)"
+    if "reload_only" in res:
+        res["reload_only"]["call"] = "lv_make_resident with LV_RESIDENT_PRELOAD (no eviction)"
+    res["peak_source"] = (f"same-run contiguous page-locked cudaMemcpyAsync of {mean // 4096 * 4096} B "
+                          "per direction")
+    return res
+
+
+def _restart(pool, wl):
+    """Puts a pool back in the workload's initial state (placement and sessions)."""
+    from paper_2606_22983_gb300.harness import initial_sessions
+    init = wl.init
+    pool.import_placement(init.placement, init.ctx_tokens)
+    pool.set_sessions(initial_sessions(wl))
+    pool.sync()
+
+
+def _streamed_with_consumer(torch, pool, wl, moves, seed):
+    """The whole script issued without a host wait between events (turns and preloads
+    with their copies on the pool's copy stream, each event's decisions overlapping the
+    copies before it), from the initial state, alone and then with the checksum consumer
+    kept running throughout on a stream of normal priority (the manager's calls on a
+    high-priority one).  Link fraction: the link's best time for every moving
+    event's own mix (from the event-by-event pass of the same script) over the elapsed
+    device time."""
+    from paper_2606_22983_gb300 import lv
+    from paper_2606_22983_gb300.manager import KVManager
+    from workloads import scatter_order
+    best_s = moves["link_best_s"]
+    out = {}
+    cons = None
+    for label in ("alone", "with_consumer"):
+        _restart(pool, wl)
+        st0 = pool.stats()
+        with torch.cuda.stream(torch.cuda.Stream(device=pool.device, priority=-1)):
+            gm = KVManager(pool, perms=wl.perms, rank_on="none", record=False, driver="device",
+                           order_fn=scatter_order, async_copy=True)
+            ends = None
+            if label == "with_consumer":
+                cons = ChecksumConsumer(torch, pool, seed=seed)
+                cons_alone = cons.alone_gbs()
+                cons.start()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            for i in range(wl.n_events):
+                if cons is not None:
+                    cons.top_up()
+                gm.step(wl.event(i), i)
+            lv.lv_join(pool.handle, pool.stream)
+            b.record()
+            if cons is not None:
+                ends = cons.keep_busy_until(b)
+            torch.cuda.synchronize()
+        assert pool.sync(raise_on_error=False) == 0
+        st1 = pool.stats()
+        moved = st1["bytes_out"] + st1["bytes_in"] - st0["bytes_out"] - st0["bytes_in"]
+        ms = a.elapsed_time(b)
+        out[label] = {"ms": round(ms, 2), "gb": round(moved / 1e9, 2),
+                      "gbs": round(moved / (ms / 1e3) / 1e9, 1),
+                      "link_frac": round(best_s / (ms / 1e3), 3)}
+        if ends is not None:
+            got, covered = cons.rate_within(ends, a, b)
+            out[label].update({"consumer_alone_gbs": round(cons_alone, 1),
+                               "consumer_with_events_gbs": round(got, 1),
+                               "consumer_frac_kept": round(got / cons_alone, 3),
+                               "consumer_ran_throughout": covered})
+            cons.close()
+    return out
+
+
+def five_workloads(torch, seed, consumer_on="mixed"):
+    """All five seeded workloads through the device driver, one event at a time
+    (paper_2606_22983_gb300.runner): GB/s and link fraction overall, by event kind and
+    by direction.  Mixed and frag run at their stated session counts (256, 1024) where
+    the host can page-lock their host tier within min(400 GB, 0.8 * MemAvailable), else
+    scaled to it (``sizing``).  The mixed script runs a second time from the same initial
+    state with the checksum consumer reading resident KV throughout (its calls on a stream
+    of normal priority, the manager's on a high-priority one), so that its speech start
+    and barge-in preloads are measured next to serving work."""
+    from paper_2606_22983_gb300.harness import fill_random, link_peaks, pool_for
+    from paper_2606_22983_gb300.manager import KVManager
+    from paper_2606_22983_gb300.runner import link_summary, peak_bytes, quantiles, run_events
+    from workloads import CONFIG_NAMES, EVENT_NAMES, host_tier_limit, make_workload, mem_available_bytes, scatter_order
+    out = {"mem_available_bytes": mem_available_bytes()}
+    for name in CONFIG_NAMES:
+        wl = make_workload(name, seed, host_limit=host_tier_limit())
+        pool = pool_for(wl)
+        try:
+            fill_random(pool, seed)
+            gm = KVManager(pool, perms=wl.perms, rank_on="none", record=False, driver="device",
+                           order_fn=scatter_order)
+            copies = {}
+            moves, turn_ms, _, wall = run_events(torch, pool, gm, wl, wl.n_events, copy_times=copies)
+            nbytes = peak_bytes(pool, moves)
+            peaks = link_peaks(pool, nbytes)
+            r = {"sessions": wl.spec.n_sessions, "events": wl.n_events,
+                 "host_pages": wl.spec.host_pages, "sizing": wl.meta.get("sizing"),
+                 "turn_ms": quantiles(turn_ms), "wall_s": round(wall, 1),
+                 "moves": link_summary(moves, peaks, EVENT_NAMES),
+                 "copy_kernels": copies}
+            if name == consumer_on:
+                r["streamed"] = _streamed_with_consumer(torch, pool, wl, r["moves"], seed)
+                _restart(pool, wl)
+                cons = ChecksumConsumer(torch, pool, seed=seed)
+                alone = cons.alone_gbs()
+                gm2 = KVManager(pool, perms=wl.perms, rank_on="none", record=False, driver="device",
+                                order_fn=scatter_order)
+                with torch.cuda.stream(torch.cuda.Stream(device=pool.device, priority=-1)):
+                    cons.top_up()
+                    done = cons.window()
+                    moves2, turn2, _, _ = run_events(torch, pool, gm2, wl, wl.n_events,
+                                                     before_event=cons.top_up)
+                    got = done()
+                cons.close()
+                r["with_consumer"] = {"consumer_alone_gbs": round(alone, 1),
+                                      "consumer_with_events_gbs": round(got, 1),
+                                      "consumer_frac_kept": round(got / alone, 3),
+                                      "turn_ms": quantiles(turn2),
+                                      "moves": link_summary(moves2, peaks, EVENT_NAMES)}
+            out[name] = r
+        finally:
+            torch.cuda.synchronize()
+            pool.close()
+            torch.cuda.empty_cache()
     return out
 
 
@@ -434,12 +724,13 @@ def ab_measure(torch, seed, n_events):
     from paper_2606_22983_gb300.controller import ControlledKVManager
     from paper_2606_22983_gb300.harness import pool_for
     from paper_2606_22983_gb300.manager import KVManager
-    from workloads import make_workload, pool_spec, scatter_order
-    out = {"workload": f"mixed (128 sessions, 60 GB HBM budget), {n_events} events, seed {seed}"}
+    from workloads import host_tier_limit, make_workload, pool_spec, scatter_order
+    out = {"workload": f"mixed (256 sessions or as the host allows, 60 GB HBM budget), "
+                       f"{n_events} events, seed {seed}"}
     turn_kinds = (1, 2, 7)
     for label in ("next_use_controller", "next_use_preload", "lru"):
         spec = pool_spec("mixed").with_(policy=1 if label == "lru" else 0)
-        wl = make_workload("mixed", seed, spec=spec, n_events=n_events)
+        wl = make_workload("mixed", seed, spec=spec, n_events=n_events, host_limit=host_tier_limit())
         pool = pool_for(wl)
         try:
             if label == "next_use_controller":
@@ -595,6 +886,7 @@ def kernel_micro(torch, pool, seed=0):
         torch.cuda.synchronize()
         out["ranker"] = {"resident_pages": N, "sessions": S, "k": 256,
                          "us_per_decision": round(a.elapsed_time(b) * 1e3 / 50, 2)}
+        out["ranker"]["sessions_4096"] = _ranker_4096(torch, pool, seed)
         # remap: the commit of all 2^20 pages to the host tier.  Each repetition
         # re-imports the placement, swaps everything out, flushes L2 (a 256 MB
         # write) and times one k_remap launch; the first repetition is untimed.
@@ -621,30 +913,6 @@ def kernel_micro(torch, pool, seed=0):
                            "entries_per_s": round(N / (ms / 1e3)), "achieved_gbs": round(gbs, 1),
                            "peak_gbs": HBM_PEAK, "frac": round(gbs / HBM_PEAK, 3),
                            "l2": "flushed before each launch"}
-        # The ceiling for remap's own traffic: the rate of each kind of scattered 4-byte
-        # request alone (lv_probe_scattered over a 16 MB array, timed like the remap, L2
-        # flushed first), each request of an entry taking its kind's share of time.
-        arr = torch.zeros(1 << 22, dtype=torch.int32, device=pool.device)
-        rates = {}
-        for i, kind in enumerate(("load", "atomic", "store", "reduce")):
-            mix = [0, 0, 0, 0]
-            mix[i] = 8
-            t = []
-            for rep in range(4):
-                flush.fill_(rep)
-                a.record()
-                lv.lv_probe_scattered(mix, arr, arr.numel(), N, None, mp.stream)
-                b.record()
-                torch.cuda.synchronize()
-                if rep:
-                    t.append(a.elapsed_time(b))
-            rates[kind] = N * 8 / (float(np.mean(t)) / 1e3)
-        model_ms = N * sum(c / rates[k] for k, c in REMAP_REQUESTS.items()) * 1e3
-        out["remap_1m"]["scattered_ceiling"] = {
-            "requests_per_entry": REMAP_REQUESTS,
-            "g_requests_per_s": {k: round(v / 1e9, 1) for k, v in rates.items()},
-            "model_ms": round(model_ms, 4), "frac": round(model_ms / ms, 3)}
-        del arr
         # and at a turn's size: 1024 entries (one whole thinker session), latency
         mp.import_placement(placement, ctx)
         lat = []
@@ -667,6 +935,40 @@ def kernel_micro(torch, pool, seed=0):
     finally:
         mp.close()
     return out
+
+
+def _ranker_4096(torch, pool, seed):
+    """One top-256 decision over 4096 sessions x 256 resident blocks (2^20 pages, the
+    most sessions a pool takes), 50 back to back, CUDA events."""
+    from paper_2606_22983_gb300 import lv
+    from paper_2606_22983_gb300.pool import KVPool
+    S, B = 4096, 256
+    N = S * B
+    mp = KVPool(layers=1, kv_heads=1, head_dim=8, max_sessions=S, max_blocks=B, hbm_pages=N,
+                hbm_budget_pages=N, host_pages=0, device=pool.device, stream=pool.stream)
+    try:
+        rng = np.random.default_rng(seed)
+        mp.import_placement(rng.permutation(N).astype(np.int32).reshape(S, B), np.full(S, B * 16, np.int32))
+        st = np.zeros(S, dtype=lv.SESSION_DTYPE)
+        st["gen_us"] = rng.integers(0, 10_000_000, S)
+        mp.set_sessions(st)
+        mp.sync()
+        o = torch.empty((256, 3), dtype=torch.int32, device=pool.device)
+        c = torch.zeros(1, dtype=torch.int64, device=pool.device)
+        for _ in range(5):
+            lv.lv_select_victims(mp.handle, 0, 256, 0, o, 256, c, mp.stream)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(50):
+            lv.lv_select_victims(mp.handle, 0, 256, 0, o, 256, c, mp.stream)
+        b.record()
+        torch.cuda.synchronize()
+        assert mp.sync(raise_on_error=False) == 0 and int(c.item()) == 256
+        return {"resident_pages": N, "sessions": S, "k": 256,
+                "us_per_decision": round(a.elapsed_time(b) * 1e3 / 50, 2)}
+    finally:
+        mp.close()
 
 
 def micro_only(args, torch):
@@ -712,41 +1014,80 @@ def _profiled_traffic(kernel, bytes_per_launch):
 
 
 # ----------------------------------------------------------- the oracle arm
-def _oracle_sample(seed, n_turns=400):
-    from workloads import make_workload, pool_spec
-    spec = pool_spec(WORKLOAD).with_(n_sessions=8, hbm_pages=1500, hbm_budget_pages=1500)
-    return make_workload(WORKLOAD, seed, spec=spec, n_turns=max(400, int(n_turns)))
-
-
-def cpu_baseline(seconds, seed, steps=None):
-    """The oracle (single thread, numpy memcpy per sub-page) on a bounded sample:
-    thinker-shaped pages, 8 sessions, a 1500-page HBM image, turns until about
-    ``seconds`` of CPU time (or ``steps`` turns)."""
+def _oracle_for(wl):
+    """The oracle over the whole workload, with full byte images (a 40 GB HBM image and
+    the host tier for the thinker pool), touched once so that no timed turn pays for
+    first-touch page faults."""
     from oracle import OracleManager
-    wl = _oracle_sample(seed)
     om = OracleManager(wl, with_bytes=True, content=None, rank_on="none")
-    om.pool.hbm.fill(1)        # touch the images so that timing excludes first-touch faults
+    om.pool.hbm.fill(1)
     om.pool.host.fill(1)
+    return om
+
+
+def _oracle_turn(om, S, i):
+    """Turn i of a turn-driven script on the oracle (its playback batch, then the
+    turn); returns the bytes it moved."""
+    b0 = om.pool.bytes_out + om.pool.bytes_in
+    for j in range(i * (S + 1), (i + 1) * (S + 1)):
+        om.step(j)
+    return om.pool.bytes_out + om.pool.bytes_in - b0
+
+
+def cpu_baseline(args, seconds, seed):
+    """The oracle (single thread, numpy memcpy per sub-page) on a bounded sample of the
+    benchmark's own workload: the same pool and script, its first turns until about
+    ``seconds`` of CPU time."""
+    wl = _arm_spec(args, seed)
+    om = _oracle_for(wl)
     S = wl.spec.n_sessions
     moved, turns = 0, 0
     t0 = time.perf_counter()
-    i = 0
-    per_turn = S + 1
-    while i + per_turn <= wl.n_events:
-        b0 = om.pool.bytes_out + om.pool.bytes_in
-        for j in range(i, i + per_turn):
-            om.step(j)
-        moved += om.pool.bytes_out + om.pool.bytes_in - b0
+    el = 0.0
+    while (turns + 1) * (S + 1) <= wl.n_events and el < seconds:
+        moved += _oracle_turn(om, S, turns)
         turns += 1
-        i += per_turn
         el = time.perf_counter() - t0
-        if (steps is not None and turns >= steps) or (steps is None and el >= seconds):
-            break
-    el = time.perf_counter() - t0
     return {"value": round(moved / el / 1e9, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{turns} turns of a thinker-shaped pool (8 sessions, 1500-page HBM image, "
+            "sample": f"the first {turns} turns of the benchmark's workload (the same "
+                      f"{S}-session pool with a {wl.spec.hbm_budget_pages}-page HBM image and "
                       f"{wl.spec.host_pages} host slots), {moved / 1e9:.2f} GB moved in {el:.1f} s",
             "seconds": round(el, 2), "ranker": _oracle_ranker(seed)}
+
+
+def oracle_configs(seed, seconds=8.0):
+    """The oracle as it stands (one host core, byte images) on a bounded sample of each
+    of the five workloads at the sizes the GPU runs them: events in script order until
+    about ``seconds`` of CPU time.  The tiny and thinker images are touched before
+    timing; the larger ones (mixed 60 + ~134 GB, long 40 + ~50 GB, frag 100 + ~148 GB)
+    are left untouched, so their timed events include first-touch page faults, and
+    only the pages the sample writes take host memory."""
+    from oracle import OracleManager
+    from workloads import CONFIG_NAMES, host_tier_limit, make_workload
+    out = {}
+    for name in CONFIG_NAMES:
+        wl = make_workload(name, seed, host_limit=host_tier_limit())
+        om = OracleManager(wl, with_bytes=True, content=None, rank_on="none")
+        touched = name in ("tiny", "thinker")
+        if touched:
+            om.pool.hbm.fill(1)
+            om.pool.host.fill(1)
+        b0 = om.pool.bytes_out + om.pool.bytes_in
+        t0 = time.perf_counter()
+        i = 0
+        el = 0.0
+        while i < wl.n_events and el < seconds:
+            om.step(i)
+            i += 1
+            el = time.perf_counter() - t0
+        moved = om.pool.bytes_out + om.pool.bytes_in - b0
+        page = wl.spec.shape.page_bytes
+        out[name] = {"sessions": wl.spec.n_sessions, "events": i, "of_events": wl.n_events,
+                     "gb_moved": round(moved / 1e9, 3), "seconds": round(el, 2),
+                     "gbs": round(moved / el / 1e9, 4), "blocks_per_s": round(moved / page / el, 1),
+                     "images_touched_first": touched, "cores": 1}
+        del om
+    return out
 
 
 def _oracle_ranker(seed):
@@ -801,40 +1142,31 @@ def _arm_spec(args, seed):
 
 
 def reference(args):
+    """The oracle as it stands, on the host cores, over the benchmark's own workload: W
+    warm-up turns, then K timed turns of the same script, pool and sizes as our arm."""
     ws, rank, _ = _dist()
     if rank != 0:
         return None
     K, W = args.steps, args.warmup
-    from oracle import OracleManager
-    wl = _oracle_sample(args.seed, n_turns=W + K + 1)
-    om = OracleManager(wl, with_bytes=True, content=None, rank_on="none")
-    om.pool.hbm.fill(1)
-    om.pool.host.fill(1)
+    wl = _arm_spec(args, args.seed)
+    om = _oracle_for(wl)
     S = wl.spec.n_sessions
-    per_turn = S + 1
-    assert (W + K) * per_turn <= wl.n_events
-
-    def turn(i):
-        b0 = om.pool.bytes_out + om.pool.bytes_in
-        for j in range(i * per_turn, (i + 1) * per_turn):
-            om.step(j)
-        return om.pool.bytes_out + om.pool.bytes_in - b0
-
+    assert (W + K) * (S + 1) <= wl.n_events
     for i in range(W):
-        turn(i)
+        _oracle_turn(om, S, i)
     t0 = time.perf_counter()
-    moved = sum(turn(i) for i in range(W, W + K))
+    moved = sum(_oracle_turn(om, S, i) for i in range(W, W + K))
     el = time.perf_counter() - t0
     v = moved / el / 1e9
     return {"impl": "reference", "metric": METRIC, "value": round(v, 4), "unit": UNIT,
             "n_gpus": ws, "steps": K, "warmup": W, "ms_per_step": round(el * 1e3 / K, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
             "data": "synthetic",
-            "config": arm_config(args, _arm_spec(args, args.seed).spec, ws),
+            "config": arm_config(args, wl.spec, ws),
             "cpu_baseline": {"value": round(v, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
-                             "sample": f"{K} turns of the oracle's bounded sample of this workload "
-                                       f"(thinker-shaped pages, 8 sessions, 1500-page HBM image) "
-                                       f"after {W} warm-up, {moved / 1e9:.2f} GB moved"},
+                             "sample": f"{K} turns of this workload after {W} warm-up turns, "
+                                       f"{moved / 1e9:.2f} GB moved (the whole workload: "
+                                       f"{S} sessions, {wl.spec.hbm_budget_pages}-page HBM image)"},
             "e2e": {"value": round(v, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
 
@@ -860,11 +1192,17 @@ def main():
                     help="smaller case for profiling: number of sessions")
     ap.add_argument("--budget-pages", type=int, default=0,
                     help="smaller case for profiling: HBM budget in pages")
+    ap.add_argument("--oracle-configs", action="store_true",
+                    help="only the oracle's bounded samples of all five workloads (host cores)")
     ap.add_argument("--ab", action="store_true",
                     help="only the policy A/B on the mixed workload (NEXT rows f1 and f3)")
     ap.add_argument("--ab-events", type=int, default=3000)
     ap.add_argument("--no-overlap", dest="overlap", action="store_false",
                     help="skip the consumer-overlap measurement")
+    ap.add_argument("--no-directions", dest="directions", action="store_false",
+                    help="skip the offload-only and reload-only legs")
+    ap.add_argument("--no-five", dest="five", action="store_false",
+                    help="skip the five workloads run event by event")
     ap.add_argument("--no-async-copy", dest="async_copy", action="store_false",
                     help="device driver: copy on the caller's stream (no overlap of the next "
                          "turn's decisions with this turn's copy)")
@@ -875,6 +1213,8 @@ def main():
         ap.error("--warmup must be at least 3")
     if args.impl == "reference":
         line = reference(args)
+    elif args.oracle_configs:
+        line = {"oracle_configs": oracle_configs(args.seed, args.cpu_seconds)}
     elif args.micro_only:
         import torch
         line = micro_only(args, torch)

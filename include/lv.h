@@ -216,7 +216,7 @@ typedef struct lv_stats {
    out of range, P not a multiple of 16, a misaligned or non-device KV pointer,
    a host_kv that is not page-locked), LV_ERR_OOM or LV_ERR_CUDA.
    Launch shapes can be overridden through the environment at creation time (for
-   tuning sweeps): LV_EXCHANGE_CTAS (the exchange copy's grid, default a fifth of
+   tuning sweeps): LV_EXCHANGE_CTAS (the exchange copy's grid, default 3/10 of
    the SMs) or LV_EXCHANGE_CTAS_PER_SM; LV_STAGE_STAGES and LV_STAGE_CTAS_PER_SM
    (the TMA pack/unpack kernel, default about 48 KiB of stages per CTA and two
    CTAs per SM); LV_STAGE_KERNEL=lsu (16-byte copies instead of TMA);

@@ -216,14 +216,6 @@ lv_status dev_alloc(lv_pool* pool, T** ptr, size_t count) {
   return LV_OK;
 }
 
-// lv_remap's tags start free (every entry of a call then finds only its own call's tags).
-cudaError_t reset_remap_tags(const lv::DevPool& d, cudaStream_t s) {
-  cudaError_t e = cudaMemsetAsync(d.rtag_blk, 0xff, (size_t)d.S * d.maxB * 4, s);
-  if (e == cudaSuccess) e = cudaMemsetAsync(d.rtag_hbm, 0xff, (size_t)d.hbm_pages * 4, s);
-  if (e == cudaSuccess) e = cudaMemsetAsync(d.rtag_host, 0xff, (size_t)(d.host_pages ? d.host_pages : 1) * 4, s);
-  return e;
-}
-
 // The event pair for the next launch of kind `kind`, or nullptr when timing is off.
 const lv::EventPair* timing_pair(lv_pool* pool, int kind) {
   if (!pool->timing) return nullptr;
@@ -616,10 +608,7 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       (st = dev_alloc(pool, &d.skey, d.S)) != LV_OK ||
       (st = dev_alloc(pool, &d.scount, d.S)) != LV_OK ||
       (st = dev_alloc(pool, &d.sbefore, d.S)) != LV_OK ||
-      (st = dev_alloc(pool, &d.page_tag, (size_t)d.hbm_pages)) != LV_OK ||
-      (st = dev_alloc(pool, &d.rtag_blk, tb)) != LV_OK ||
-      (st = dev_alloc(pool, &d.rtag_hbm, (size_t)d.hbm_pages)) != LV_OK ||
-      (st = dev_alloc(pool, &d.rtag_host, (size_t)(d.host_pages ? d.host_pages : 1))) != LV_OK)
+      (st = dev_alloc(pool, &d.page_tag, (size_t)d.hbm_pages)) != LV_OK)
     return fail(st);
   lv::ResidentScratch& rs = pool->rs;
   if ((st = dev_alloc(pool, &rs.victims, (size_t)d.budget)) != LV_OK ||
@@ -658,15 +647,16 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
       cudaMemsetAsync(d.bits_hbm, 0, wh * 4, s) != cudaSuccess ||
       cudaMemsetAsync(d.bits_host, 0, (wo ? wo : 1) * 4, s) != cudaSuccess ||
       cudaMemsetAsync(d.ctl, 0, lv::C_N * sizeof(long long), s) != cudaSuccess ||
-      cudaMemsetAsync(d.page_tag, 0, (size_t)d.hbm_pages * 8, s) != cudaSuccess ||
-      reset_remap_tags(d, s) != cudaSuccess)
+      cudaMemsetAsync(d.page_tag, 0, (size_t)d.hbm_pages * 8, s) != cudaSuccess)
     return fail(LV_ERR_CUDA);
   // A fifth of the SMs (30 CTAs on GB300) keeps both link directions saturated (338 GB/s,
   // the same as 50 CTAs or one per SM; 25 CTAs fall to 326) and leaves the rest of the
   // GPU to the serving work that runs meanwhile: next to a consumer reading resident KV
   // at HBM speed, 30 CTAs moved 211 GB/s and left it 0.88 of its rate, against 197 GB/s
   // and 0.835 for 50 CTAs and 167 GB/s and 0.67 for 152.
-  pool->exchange_ctas = pool->num_sms / 5 > 0 ? pool->num_sms / 5 : 1;
+  // 3/10 of the SMs (45 on GB300): the fewest CTAs that keep both link directions busy
+  // alone, and most of the link next to a kernel that reads HBM on every SM
+  pool->exchange_ctas = pool->num_sms * 3 / 10 > 0 ? pool->num_sms * 3 / 10 : 1;
   if (const char* env = std::getenv("LV_EXCHANGE_CTAS_PER_SM")) {
     const int per = std::atoi(env);
     if (per >= 1 && per <= 16) pool->exchange_ctas = pool->num_sms * per;
@@ -792,7 +782,6 @@ lv_status lv_pool_import(lv_pool* pool, const int32_t* placement, const int32_t*
     if (d.host_pages) LV_TRY(cudaMemsetAsync(d.bits_host, 0, (size_t)((d.host_pages + 31) / 32) * 4, s));
     LV_TRY(cudaMemsetAsync(d.ctl, 0, 2 * sizeof(long long), s));   // allocation counts
     LV_TRY(cudaMemsetAsync(d.ctl + lv::C_CLEAN, 0, sizeof(long long), s));   // no clean copies
-    LV_TRY(reset_remap_tags(d, s));
     LV_TRY(lv::launch_import(d, static_cast<const int32_t*>(pl), static_cast<const int32_t*>(cx), s));
     LV_TRY(lv::launch_check_budget(d, s));
     return st.finish();
@@ -982,7 +971,8 @@ lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_ou
     if ((r = st.out(slots_out, (size_t)n_out * 4, &sdev, true)) != LV_OK) return r;
     if ((r = st.out(pages_out, (size_t)n_in * 4, &pdev, true)) != LV_OK) return r;
     if ((r = st.out(nullptr, (size_t)(n_out + n_in) * sizeof(int4), &tdev, true)) != LV_OK) return r;
-    if ((r = st.out(nullptr, sizeof(long long), &ndev, true)) != LV_OK) return r;
+    // the task count, and the copy kernel's cursor
+    if ((r = st.out(nullptr, 2 * sizeof(long long), &ndev, true)) != LV_OK) return r;
     if (++pool->epoch <= 0) pool->epoch = 1;
     if (mode == LV_MODE_STAGED) {
       LV_TRY(lv::launch_exchange_plan(pool->d, static_cast<const lv_victim*>(vin), n_out, sid,
@@ -999,7 +989,8 @@ lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_ou
                                static_cast<const int32_t*>(bin), n_in, static_cast<int32_t*>(sdev),
                                static_cast<int32_t*>(pdev), static_cast<int4*>(tdev),
                                static_cast<long long*>(ndev), pool->epoch, pool->d.page_tag, s,
-                               pool->exchange_ctas, nullptr, 0, timing_pair(pool, LV_TIMING_EXCHANGE)));
+                               pool->exchange_ctas, nullptr, 0, timing_pair(pool, LV_TIMING_EXCHANGE),
+                               nullptr, nullptr, 0, static_cast<long long*>(ndev) + 1));
     return st.finish();
   } catch (const std::bad_alloc&) {
     return LV_ERR_OOM;
@@ -1259,8 +1250,7 @@ lv_status lv_schedule(lv_pool* pool, const lv_sched_params* q, const lv_request*
 
 lv_status lv_remap(lv_pool* pool, const lv_remap_entry* entries, int64_t n, lv_stream stream) {
   NvtxRange nvtx_range("lv_remap");
-  // entry indices are 32-bit tags; more entries than blocks cannot all be accepted anyway
-  if (!pool || n < 0 || n > 0xFFFFFFFEll || (n > 0 && !entries)) return LV_ERR_INVALID;
+  if (!pool || n < 0 || (n > 0 && !entries)) return LV_ERR_INVALID;
   if (n == 0) return LV_OK;
   DeviceGuard g(pool->device);
   cudaStream_t s = as_stream(stream);
@@ -1269,8 +1259,9 @@ lv_status lv_remap(lv_pool* pool, const lv_remap_entry* entries, int64_t n, lv_s
     const void* in = nullptr;
     lv_status r = st.in(entries, (size_t)n * sizeof(lv_remap_entry), &in);
     if (r != LV_OK) return r;
-    LV_TRY(lv::launch_remap(pool->d, static_cast<const lv_remap_entry*>(in), n, s, pool->num_sms,
-                            pool->remap_per_thread));
+    if (++pool->epoch <= 0) pool->epoch = 1;
+    LV_TRY(lv::launch_remap(pool->d, static_cast<const lv_remap_entry*>(in), n, pool->epoch, s,
+                            pool->num_sms, pool->remap_per_thread));
     return st.finish();
   } catch (const std::bad_alloc&) {
     return LV_ERR_OOM;

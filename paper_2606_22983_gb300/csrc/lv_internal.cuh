@@ -71,11 +71,6 @@ struct DevPool {
   long long* sbefore;        // [S] resident blocks of the candidates ranked ahead of it
   // exchange scratch
   unsigned long long* page_tag;  // [hbm_pages] epoch << 32 | victim index (| paired bit)
-  // lv_remap's tags (0xFFFFFFFF between calls): the first entry of a call naming a
-  // block or a location
-  uint32_t* rtag_blk;     // [S][maxB]
-  uint32_t* rtag_hbm;     // [hbm_pages]
-  uint32_t* rtag_host;    // [host_pages]
 };
 
 __host__ __device__ inline uint32_t owner_key(int32_t sid, int32_t blk) {
@@ -129,10 +124,10 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
                             unsigned long long* page_tag, cudaStream_t s, int copy_ctas,
                             const long long* counts_dev = nullptr, long long max_units = 0,
                             const EventPair* ev = nullptr, const long long* sid_dev = nullptr,
-                            const CopyOffload* off = nullptr, int gate = 0);
-// n <= 2^32 - 2 (entry indices are the 32-bit tags of the two passes)
-cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, cudaStream_t s,
-                         int num_sms, int per_thread);
+                            const CopyOffload* off = nullptr, int gate = 0,
+                            long long* cursor = nullptr, const struct StepFinish* fin = nullptr);
+cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, int32_t epoch,
+                         cudaStream_t s, int num_sms, int per_thread);
 cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cudaStream_t s);
 cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32_t* pages,
                           int32_t* count, cudaStream_t s, const long long* gate = nullptr,
@@ -150,13 +145,35 @@ struct ResidentScratch {
   long long* words;     // [16]
   int32_t* hits;        // [S] lv_turn's pick
 };
+// The end of a device-driven step (lv_make_resident, lv_turn, lv_evict): the turn's
+// LV_EV_TURN_END, a completed preload's protection, and the result record.
+struct StepFinish {
+  bool on;
+  int32_t sid;                    // the session, or read from sid_dev when that is set
+  const long long* sid_dev;
+  long long now_us;
+  bool preload;
+  bool turn_end;
+  long long audio_us, units;      // LV_EV_TURN_END's a and b
+  lv_resident_result* out;        // may be null
+};
+// lv_turn's start, done by the first kernel of the make-resident chain: pick the
+// session when sid < 0 (the first of cand[0..n_cand) with hit set), then TURN_BEGIN.
+struct TurnStart {
+  bool on;
+  const int32_t* cand;
+  int32_t n_cand;
+  const int32_t* hit;
+  long long now_us;
+};
 cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, int32_t sid,
                                  int64_t now_us, int32_t append_tokens, bool preload,
                                  int64_t max_load, int32_t epoch, cudaStream_t s, int copy_ctas,
                                  lv_resident_result* result, const EventPair* ev = nullptr,
                                  const long long* sid_dev = nullptr, const CopyOffload* off = nullptr,
                                  const unsigned long long* load_keys = nullptr, bool turn_end = false,
-                                 int64_t audio_us = 0, int64_t units = 0);
+                                 int64_t audio_us = 0, int64_t units = 0,
+                                 const TurnStart* ts = nullptr);
 // lv_turn: pick (sid < 0), LV_EV_TURN_BEGIN, make resident, LV_EV_TURN_END
 // lv_evict: rank, evict up to k victims (no loads), finish
 cudaError_t launch_evict(const DevPool& p, const ResidentScratch& rs, int64_t now_us, int64_t k,

@@ -7,7 +7,7 @@
 //             k_stage_tasks (TMA) / k_stage_tasks_lsu         (staged copy-engine path)
 //   commit    k_remap, k_cancel, k_append                    (Section 6 side tables)
 //   monitor   k_events                                       (Section 3, Sections 5.1-5.2)
-//   turn      k_resident_*, k_pick_scan, k_turn_begin,        (a whole turn on the device;
+//   turn      k_resident_*, k_pick_scan,                      (a whole turn on the device;
 //             k_order_loads, k_evict_prepare                 the gate runs in the plan)
 //   verify    k_checksum                                     (page checksums)
 //
@@ -41,6 +41,15 @@ __device__ __forceinline__ void set_error(long long* ctl, int code, long long de
 // ordinary way both instructions have no effect.
 __device__ __forceinline__ void pdl_entry() {
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// The same two steps apart, for a kernel with a large grid: it waits at its start and
+// lets the next kernel be scheduled only when its own work is done, so that the next
+// kernel's CTAs do not sit on SMs, waiting, while this grid still needs them.  A CTA
+// that returns early counts as having let it.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
@@ -358,14 +367,18 @@ __device__ __forceinline__ unsigned long long session_key(const DevPool& p, int3
 
 constexpr int kCensusThreads = 256;
 // Up to this many sessions every emit CTA finds its session's place by reading all
-// S keys itself; above it, k_rank_prefix computes every place once, between the
-// census and the emission (S^2 key comparisons, but S^2 / 256 key reads).
-constexpr int kEmitScanMax = 256;
+// S keys itself (S^2 key reads, from L2); above it, k_rank_prefix computes every place
+// once, between the census and the emission (S^2 key comparisons, but S^2 / 256 key
+// reads), at the cost of one more launch in the chain.
+#ifndef LV_EMIT_SCAN_MAX
+#define LV_EMIT_SCAN_MAX 1024
+#endif
+constexpr int kEmitScanMax = LV_EMIT_SCAN_MAX;
 
 // One CTA per session: its key and its count of HBM-resident blocks.
 __global__ void __launch_bounds__(kCensusThreads)
 k_rank_census(DevPool p, long long now_us, bool fallback) {
-  pdl_entry();
+  pdl_wait();
   const int32_t s = blockIdx.x;
   __shared__ unsigned long long key;
   if (threadIdx.x == 0) {
@@ -390,6 +403,7 @@ k_rank_census(DevPool p, long long now_us, bool fallback) {
     p.skey[s] = key;
     p.scount[s] = (int32_t)total;
   }
+  pdl_trigger();
 }
 
 constexpr int kPrefixTile = 128;    // sessions placed by one CTA (one per thread)
@@ -403,7 +417,7 @@ constexpr int kPrefixChunk = 256;   // keys staged by one CTA in shared memory
 // all candidates' blocks into C_RANK_TOTAL.  The census zeroed both.
 __global__ void __launch_bounds__(kPrefixTile)
 k_rank_prefix(DevPool p) {
-  pdl_entry();   // the census is complete and visible
+  pdl_wait();   // the census is complete and visible
   __shared__ unsigned long long kc[kPrefixChunk];
   __shared__ int32_t cc[kPrefixChunk];
   __shared__ long long part[kPrefixTile / 32];
@@ -435,6 +449,7 @@ k_rank_prefix(DevPool p) {
       if (all) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_RANK_TOTAL]), (unsigned long long)all);
     }
   }
+  pdl_trigger();
 }
 
 constexpr int kEmitThreads = 256;
@@ -449,7 +464,7 @@ constexpr int kEmitThreads = 256;
 __global__ void __launch_bounds__(kEmitThreads)
 k_rank_emit(DevPool p, long long k, const long long* k_dev, bool fallback, long long* count_dev,
             lv_victim* __restrict__ out) {
-  pdl_entry();   // the census is complete and visible
+  pdl_wait();   // the census (and the places) are complete and visible
   const int32_t sid = blockIdx.x;
   const unsigned long long key = p.skey[sid];
   if (key == 0ull && sid != 0) return;
@@ -496,6 +511,7 @@ k_rank_emit(DevPool p, long long k, const long long* k_dev, bool fallback, long 
     if (flag && pos < n_out) out[pos] = lv_victim{sid, b, e};
     run += chunk;
   }
+  pdl_trigger();
 }
 
 // ------------------------------------------------------------ allocation
@@ -668,7 +684,8 @@ enum ResWord : int {
   R_N_TASKS = 6,
   R_APPENDED = 7,   // int32 count of appended pages, in the low half
   R_FOUND = 8,      // victims the ranking found
-  R_SID = 9         // lv_turn: the turn's session (-1 when the pick failed)
+  R_SID = 9,        // lv_turn: the turn's session (-1 when the pick failed)
+  R_CURSOR = 10     // the exchange copy's next unit (zeroed by the plan)
 };
 
 // The gate after a device-driven step's ranking, run by the exchange plan's first
@@ -705,17 +722,20 @@ __device__ __forceinline__ void step_gate(const DevPool& p, long long* __restric
   }
 }
 
+__device__ void finish_step(const DevPool& p, const StepFinish& f, const long long* __restrict__ R);
+
 __global__ void __launch_bounds__(kPlanThreads)
 k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int32_t sid,
                 const int32_t* __restrict__ blks, long long n_in, int32_t* __restrict__ slots,
                 int32_t* __restrict__ pages, int4* __restrict__ tasks, long long* n_tasks,
                 int32_t epoch, unsigned long long* __restrict__ page_tag,
                 const long long* counts_dev, const long long* __restrict__ sid_dev,
-                long long* R, int gate) {
+                long long* R, int gate, long long* __restrict__ cursor, StepFinish fin) {
   pdl_entry();
   __shared__ int bad;
   if (threadIdx.x == 0) {
     bad = 0;
+    if (cursor) *cursor = 0;
     if (gate != GATE_NONE) step_gate(p, R, gate);   // a device-driven step: may set the counts
   }
   __syncthreads();
@@ -773,7 +793,10 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
   if (bad) {
     for (long long i = threadIdx.x; i < n_out; i += kPlanThreads) slots[i] = -1;
     for (long long i = threadIdx.x; i < n_in; i += kPlanThreads) pages[i] = -1;
-    if (threadIdx.x == 0) *n_tasks = 0;
+    if (threadIdx.x == 0) {
+      *n_tasks = 0;
+      if (fin.on) finish_step(p, fin, R);
+    }
     return;
   }
   // host slots for the victims: a clean copy, or the lowest free slots in victim order
@@ -852,18 +875,28 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PAGES_OUT]), (unsigned long long)n_out);
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PAGES_IN]), (unsigned long long)n_in);
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_REMAP]), (unsigned long long)(n_out + n_in));
+    if (fin.on) finish_step(p, fin, R);   // the step's end when nothing follows the plan
   }
 }
 
 // Unit u = (task t, sub-page j): the out half copies hbm_kv[j][page] to host[slot][j],
 // the in half host[slot'][j] to hbm_kv[j][page']; each thread loads both before it
-// stores either, so a paired task reads the old page before overwriting it.
+// stores either, so a paired task reads the old page before overwriting it.  CTAs take
+// units in order from a shared cursor (zeroed by the plan), the next one fetched while
+// the current one is copied: a CTA that starts late, or runs on an SM crowded by other
+// work, simply takes fewer units.
 __global__ void __launch_bounds__(kCopyThreads)
-k_exchange_copy(DevPool p, const int4* __restrict__ tasks, const long long* __restrict__ n_tasks) {
+k_exchange_copy(DevPool p, const int4* __restrict__ tasks, const long long* __restrict__ n_tasks,
+                long long* __restrict__ cursor) {
   pdl_entry();
   const long long units = *n_tasks * p.J;
   const int nvec = (int)(p.P >> 4);
-  for (long long u = blockIdx.x; u < units; u += gridDim.x) {
+  __shared__ long long next;
+  if (threadIdx.x == 0) next = (long long)atomicAdd(reinterpret_cast<unsigned long long*>(cursor), 1ull);
+  __syncthreads();
+  for (long long u = next; u < units; u = next) {
+    __syncthreads();   // every thread holds u before `next` is replaced
+    if (threadIdx.x == 0) next = (long long)atomicAdd(reinterpret_cast<unsigned long long*>(cursor), 1ull);
     const int4 t = tasks[u / p.J];
     const int j = (int)(u % p.J);
     const bool has_out = t.x >= 0, has_in = t.z >= 0;
@@ -890,6 +923,7 @@ k_exchange_copy(DevPool p, const int4* __restrict__ tasks, const long long* __re
         }
       }
     }
+    __syncthreads();   // thread 0's fetch of the next unit is visible
   }
 }
 
@@ -1158,115 +1192,93 @@ __global__ void k_selftest_wait(long long* ctl, long long limit_ns) {
 }
 
 // ---------------------------------------------------------------- commit
-// lv_remap runs in two passes.  Pass 1 (k_remap_tag) tags, for every entry i, its
-// block and its new location with i by non-returning minimum reductions, so a block
-// or location named by several entries of the call ends up tagged with the first
-// of them in list order.  Pass 2 (k_remap_commit) reads the tags back with every
-// other independent read of the entry: only the entry whose index a tag holds may
-// use that block or location (the others are double maps), and that entry puts the
-// tag back to kTagFree, so the tags are free again once the call has run.  Nothing
-// in either pass waits for a returning atomic.
 constexpr int kRemapThreads = 256;
-constexpr uint32_t kTagFree = 0xFFFFFFFFu;
 
-// The entry's block and new location, with the range checks both passes share.
-struct RemapSlots {
+// The reads of one entry that do not depend on a check.
+struct RemapRead {
   lv_remap_entry x;
-  size_t ti;            // table index (valid when blk_ok)
-  uint32_t* ltag;       // the new location's tag word, or nullptr when loc is out of range
-  uint32_t* lown;       // its owner word
-  bool blk_ok;          // sid and blk inside the table
+  size_t ti;            // table index (0 when out of range)
+  int32_t old;          // the block's current location
+  int32_t g;            // its clean-copy slot (inclusive tiers), or -1
+  int32_t nb;           // blocks of its session
+  uint32_t old_owner;   // owner word of the current location
+  bool in_range;
 };
-
-__device__ __forceinline__ RemapSlots remap_slots(const DevPool& p, const lv_remap_entry& x) {
-  RemapSlots r;
-  r.x = x;
-  r.blk_ok = x.sid >= 0 && x.sid < p.S && x.blk >= 0 && x.blk < p.maxB;
-  r.ti = r.blk_ok ? (size_t)x.sid * p.maxB + x.blk : 0;
-  r.ltag = nullptr;
-  r.lown = nullptr;
-  if (x.loc >= 0 && x.loc < p.hbm_pages) {
-    r.ltag = p.rtag_hbm + x.loc;
-    r.lown = p.own_hbm + x.loc;
-  } else if (x.loc <= -2 && -(long long)x.loc - 2 < p.host_pages) {
-    r.ltag = p.rtag_host + (-(long long)x.loc - 2);
-    r.lown = p.own_host + (-(long long)x.loc - 2);
-  }
-  return r;
-}
-
-__global__ void __launch_bounds__(kRemapThreads)
-k_remap_tag(DevPool p, const lv_remap_entry* __restrict__ e, long long n) {
-  pdl_entry();
-  const long long stride = (long long)gridDim.x * kRemapThreads;
-  for (long long i = blockIdx.x * (long long)kRemapThreads + threadIdx.x; i < n; i += stride) {
-    const RemapSlots r = remap_slots(p, e[i]);
-    if (r.blk_ok) atomicMin(&p.rtag_blk[r.ti], (uint32_t)i);
-    if (r.ltag) atomicMin(r.ltag, (uint32_t)i);
-  }
-}
 
 struct RemapCounts {
   int ok, hbm, host, clean;
 };
 
-// The reads of one entry in pass 2 that depend on nothing but the entry.
-struct RemapRead {
-  RemapSlots r;
-  uint32_t btag, ltag;  // the tags of its block and of its new location
-  uint32_t got;         // owner word of the new location
-  int32_t old;          // the block's current location
-  int32_t g;            // its clean-copy slot (inclusive tiers), or -1
-  int32_t nb;           // blocks of its session
-};
-
-__device__ __forceinline__ void remap_read(const DevPool& p, const lv_remap_entry* e, long long i,
-                                           long long n, RemapRead& q) {
-  q.r = remap_slots(p, i < n ? e[i] : lv_remap_entry{-1, -1, -1});
-  const bool b = i < n && q.r.blk_ok;
-  const bool l = i < n && q.r.ltag != nullptr;
-  q.btag = b ? p.rtag_blk[q.r.ti] : kTagFree;
-  q.old = b ? p.table[q.r.ti] : -1;
-  q.g = (b && p.incl) ? p.shadow[q.r.ti] : -1;
-  q.nb = b ? nblocks_of(p, q.r.x.sid) : 0;
-  q.ltag = l ? *q.r.ltag : kTagFree;
-  q.got = l ? *q.r.lown : kOwnerNone;
+__device__ __forceinline__ void remap_read_entry(const DevPool& p, const lv_remap_entry* e, long long i,
+                                                 long long n, RemapRead& r) {
+  r.x = i < n ? e[i] : lv_remap_entry{-1, -1, -1};
+  r.in_range = i < n && r.x.sid >= 0 && r.x.sid < p.S && r.x.blk >= 0 && r.x.blk < p.maxB;
+  r.ti = r.in_range ? (size_t)r.x.sid * p.maxB + r.x.blk : 0;
 }
 
-// Releases the tags this entry holds and judges it: 0, or the status to report.
-__device__ __forceinline__ int remap_judge(const DevPool& p, const RemapRead& q, long long i) {
-  const uint32_t me = (uint32_t)i;
-  const bool own_b = q.r.blk_ok && q.btag == me;
-  const bool own_l = q.r.ltag != nullptr && q.ltag == me;
-  if (own_b) p.rtag_blk[q.r.ti] = kTagFree;
-  if (own_l) *q.r.ltag = kTagFree;
-  const lv_remap_entry& x = q.r.x;
-  if (!q.r.blk_ok || x.blk >= q.nb || q.r.ltag == nullptr) return LV_ERR_BOUNDS;
-  if (!own_b || !own_l) return LV_ERR_DOUBLE_MAP;   // the block or the location twice in the call
-  if (q.got != kOwnerReserved) {
-    // a host location already owned by this block is fine only as its own clean copy
-    const long long h = -(long long)x.loc - 2;
-    if (!(x.loc <= -2 && p.incl && (long long)q.g == h && q.got == owner_key(x.sid, x.blk)))
-      return LV_ERR_DOUBLE_MAP;
+__device__ __forceinline__ void remap_read_table(const DevPool& p, RemapRead& r) {
+  r.old = r.in_range ? p.table[r.ti] : -1;
+  r.g = (r.in_range && p.incl) ? p.shadow[r.ti] : -1;
+  r.nb = r.in_range ? nblocks_of(p, r.x.sid) : 0;
+}
+
+__device__ __forceinline__ void remap_read_owner(const DevPool& p, RemapRead& r) {
+  const long long old_slot = -(long long)r.old - 2;
+  r.old_owner = kOwnerNone;
+  if (r.old >= 0 && r.old < p.hbm_pages) r.old_owner = p.own_hbm[r.old];
+  else if (r.old <= -2 && old_slot < p.host_pages) r.old_owner = p.own_host[old_slot];
+}
+
+// The block's epoch mark: one accepted entry per block per call.  Returns the
+// entry's error so far (a returning atomic; the caller issues every entry's
+// mark before it looks at any result).
+__device__ __forceinline__ int remap_mark(const DevPool& p, const RemapRead& r, int32_t epoch,
+                                          int32_t& seen) {
+  if (!r.in_range || r.x.blk >= r.nb) return LV_ERR_BOUNDS;
+  seen = atomicExch(&p.mark[r.ti], epoch);
+  return 0;
+}
+
+// The new location must be a reservation nobody owns yet: one CAS checks and
+// takes it.  Issued for every entry that passed its mark, before any result is read.
+__device__ __forceinline__ int remap_claim(const DevPool& p, const RemapRead& r, int err,
+                                           uint32_t& got) {
+  if (err) return err;
+  const lv_remap_entry& x = r.x;
+  const uint32_t key = owner_key(x.sid, x.blk);
+  if (x.loc >= 0) {
+    if (x.loc >= p.hbm_pages) return LV_ERR_BOUNDS;
+    got = atomicCAS(&p.own_hbm[x.loc], kOwnerReserved, key);
+  } else if (x.loc <= -2) {
+    if (-(long long)x.loc - 2 >= p.host_pages) return LV_ERR_BOUNDS;
+    got = atomicCAS(&p.own_host[-(long long)x.loc - 2], kOwnerReserved, key);
+  } else {
+    return LV_ERR_BOUNDS;
   }
   return 0;
 }
 
-// Applies an accepted entry: table, new owner, clean copy, old location.  The old
-// location's owner word, read after the table, only checks consistency.
-__device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& q, uint32_t old_owner,
-                                            long long i, RemapCounts& c) {
-  const lv_remap_entry& x = q.r.x;
-  const int32_t old = q.old, g = q.g;
+// Judges the claim and applies the entry: table, clean copy, old location.
+__device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& r, int err,
+                                            uint32_t got, long long i, RemapCounts& c) {
+  const lv_remap_entry& x = r.x;
+  const int32_t old = r.old, g = r.g;
   const long long old_slot = -(long long)old - 2;
   const bool old_hbm = old >= 0 && old < p.hbm_pages;
   const bool old_host = old <= -2 && old_slot < p.host_pages;
   const long long h = -(long long)x.loc - 2;
   const uint32_t key = owner_key(x.sid, x.blk);
-  p.table[q.r.ti] = x.loc;
-  *q.r.lown = key;
+  if (!err && got != kOwnerReserved) {
+    // a host location already owned by this block is fine only as its own clean copy
+    if (!(x.loc <= -2 && p.incl && (long long)g == h && got == key)) err = LV_ERR_DOUBLE_MAP;
+  }
+  if (err) {
+    set_error(p.ctl, err, i);
+    return;
+  }
+  p.table[r.ti] = x.loc;
   if (x.loc <= -2 && g >= 0) {          // the copy becomes the location, or goes
-    p.shadow[q.r.ti] = -1;
+    p.shadow[r.ti] = -1;
     c.clean -= 1;
     if ((long long)g != h) {
       p.own_host[g] = kOwnerNone;
@@ -1276,13 +1288,13 @@ __device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& q
   }
   // the old location belongs to this block alone (one entry per block per call)
   if (old_hbm || old_host) {
-    if (old_owner != key) set_error(p.ctl, LV_ERR_STATE, i);
+    if (r.old_owner != key) set_error(p.ctl, LV_ERR_STATE, i);
     if (old_hbm) {
       p.own_hbm[old] = kOwnerNone;
       atomicAnd(&p.bits_hbm[old >> 5], ~(1u << (old & 31)));
       c.hbm += 1;
     } else if (p.incl && x.loc >= 0) {   // back in HBM: the host slot stays as its clean copy
-      p.shadow[q.r.ti] = (int32_t)old_slot;
+      p.shadow[r.ti] = (int32_t)old_slot;
       c.clean += 1;
     } else {
       p.own_host[old_slot] = kOwnerNone;
@@ -1293,46 +1305,55 @@ __device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& q
   c.ok += 1;
 }
 
-// Pass 2.  Each thread commits E entries, i0, i0 + stride, ... (stride = the grid's
-// threads, so a warp's entries stay contiguous).  All E entries' independent reads
-// are issued before any result is used, then the old locations' owner words, then
-// the stores: two dependent rounds of reads per entry.  The reads are race-free
-// within one call: an accepted entry is the only one on its block and on its new
-// location, a location freed by one entry is never the new location of another
-// (new locations are reservations, old ones are owned), and a rejected entry
-// writes nothing but its own tags.  The allocation counts and the commit counter
-// change by block totals (one atomic per block and counter).  Inclusive tiers: a
-// host location may be the block's own clean copy; a block committed to HBM from
-// the host tier keeps its slot as its clean copy; a block committed to another
-// host slot loses its copy.
+// Each thread commits E entries, i0, i0 + stride, ... (stride = the grid's
+// threads, so a warp's entries stay contiguous).  The allocation counts and the
+// commit counter change by block totals (one atomic per block and counter).
+// Inclusive tiers: a host location may be the block's own clean copy; a block
+// committed to HBM from the host tier keeps its slot as its clean copy; a
+// block committed to another host slot loses its copy.
+//
+// The kernel is bound by the latency of dependent scattered accesses (entry ->
+// table entry -> owner of the old location -> epoch mark -> claim of the new
+// location), so each step is issued for all E entries of the thread before any
+// of its results is used: every read that does not depend on a check, then
+// every mark, then every claim, then the stores.  E chains then wait together.  The early
+// reads are race-free within one call: a block has at most one accepted entry
+// (the epoch mark), a location freed by one entry is never the new location of
+// another (new locations are reservations), and another entry can take an
+// owned location only through a CAS, which then fails.  A thread's own
+// entries apply in order, so a duplicate among them meets the epoch mark too.
 template <int E>
 __global__ void __launch_bounds__(kRemapThreads)
-k_remap_commit(DevPool p, const lv_remap_entry* __restrict__ e, long long n) {
-  pdl_entry();   // every tag of pass 1 is in place
+k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t epoch) {
   const long long stride = (long long)gridDim.x * kRemapThreads;
   const long long i0 = blockIdx.x * (long long)kRemapThreads + threadIdx.x;
-  RemapRead q[E];
+  RemapRead r[E];
 #pragma unroll
-  for (int j = 0; j < E; ++j) remap_read(p, e, i0 + j * stride, n, q[j]);
+  for (int j = 0; j < E; ++j) remap_read_entry(p, e, i0 + j * stride, n, r[j]);
+#pragma unroll
+  for (int j = 0; j < E; ++j) remap_read_table(p, r[j]);
+#pragma unroll
+  for (int j = 0; j < E; ++j) remap_read_owner(p, r[j]);
+  // the atomics of all E entries: every mark, then every claim, each group in flight
+  // together; a thread's own duplicate meets the mark of its earlier entry
   int err[E];
-  uint32_t old_owner[E];
+  int32_t seen[E];
+  uint32_t got[E];
 #pragma unroll
   for (int j = 0; j < E; ++j) {
-    const long long i = i0 + j * stride;
-    err[j] = i < n ? remap_judge(p, q[j], i) : -1;
-    old_owner[j] = kOwnerNone;
-    if (err[j] == 0) {
-      const int32_t old = q[j].old;
-      if (old >= 0 && old < p.hbm_pages) old_owner[j] = p.own_hbm[old];
-      else if (old <= -2 && -(long long)old - 2 < p.host_pages) old_owner[j] = p.own_host[-(long long)old - 2];
-    }
+    seen[j] = 0;
+    err[j] = i0 + j * stride < n ? remap_mark(p, r[j], epoch, seen[j]) : -1;
+  }
+#pragma unroll
+  for (int j = 0; j < E; ++j) {
+    if (err[j] == 0 && seen[j] == epoch) err[j] = LV_ERR_DOUBLE_MAP;   // same block twice
+    got[j] = kOwnerReserved;
+    if (err[j] >= 0) err[j] = remap_claim(p, r[j], err[j], got[j]);
   }
   RemapCounts c{0, 0, 0, 0};
 #pragma unroll
-  for (int j = 0; j < E; ++j) {
-    if (err[j] > 0) set_error(p.ctl, err[j], i0 + j * stride);
-    else if (err[j] == 0) remap_apply(p, q[j], old_owner[j], i0 + j * stride, c);
-  }
+  for (int j = 0; j < E; ++j)
+    if (err[j] >= 0) remap_apply(p, r[j], err[j], got[j], i0 + j * stride, c);
   // block totals: warp sums, one shared atomic per warp, one global atomic per block
   __shared__ int tot[4];
   if (threadIdx.x < 4) tot[threadIdx.x] = 0;
@@ -1462,13 +1483,57 @@ k_append(DevPool p, int32_t sid, int32_t n_tokens, int32_t* __restrict__ pages,
 
 // -------------------------------------------------------- make_resident
 
-// One CTA: sid's host-tier blocks (ascending), the deficit k and the admission.
+// lv_turn's start, run first by k_resident_prepare: the turn's session (sid, or the
+// first candidate with a hit, else the first candidate) into R[R_SID], then
+// LV_EV_TURN_BEGIN for it.  Returns the session, -1 when the pick failed.
+__device__ int32_t turn_begin(const DevPool& p, int32_t sid, const TurnStart& ts, long long* R) {
+  __shared__ int first;
+  __shared__ int32_t picked;
+  if (threadIdx.x == 0) first = ts.n_cand;
+  __syncthreads();
+  if (sid < 0) {
+    int mine = ts.n_cand;
+    for (int c = threadIdx.x; c < ts.n_cand; c += blockDim.x)
+      if (ts.hit[c]) { mine = c; break; }
+    if (mine < ts.n_cand) atomicMin(&first, mine);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int32_t s = sid;
+    if (s < 0) {
+      const int c = first < ts.n_cand ? first : 0;
+      s = ts.cand[c];
+      if (s < 0 || s >= p.S) {
+        set_error(p.ctl, LV_ERR_BOUNDS, c);
+        s = -1;
+      }
+    }
+    R[R_SID] = s;
+    if (s >= 0) {
+      lv_session_state st = p.sess[s];
+      lv_event x{};
+      x.kind = LV_EV_TURN_BEGIN;
+      x.sid = s;
+      x.t_us = ts.now_us;
+      apply_event(p, st, x);
+      p.sess[s] = st;
+      atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_EVENTS]), 1ull);
+    }
+    picked = s;
+  }
+  __syncthreads();
+  return picked;
+}
+
+// One CTA: sid's host-tier blocks (ascending), the deficit k and the admission; for
+// lv_turn (ts.on) the turn's start first.
 __global__ void __launch_bounds__(kCensusThreads)
 k_resident_prepare(DevPool p, int32_t sid, int32_t append_tokens, bool preload,
                    long long max_load, int32_t* __restrict__ blocks, long long* __restrict__ R,
-                   const long long* __restrict__ sid_dev) {
+                   const long long* __restrict__ sid_dev, TurnStart ts) {
   pdl_entry();
-  if (sid_dev) sid = (int32_t)*sid_dev;
+  if (ts.on) sid = turn_begin(p, sid, ts, R);
+  else if (sid_dev) sid = (int32_t)*sid_dev;
   if (sid < 0 || sid >= p.S) {        // lv_turn's pick failed (already reported)
     if (threadIdx.x == 0) {
       R[R_K_SELECT] = 0; R[R_N_OUT] = 0; R[R_N_IN] = 0; R[R_STATUS] = LV_RESIDENT_FAILED;
@@ -1547,31 +1612,26 @@ k_order_loads(const long long* __restrict__ R, const int32_t* __restrict__ block
 
 // The step's result and, for lv_turn (turn_end), LV_EV_TURN_END for the turn's session
 // unless its KV could not be made resident.
-__global__ void k_resident_finish(DevPool p, int32_t sid, long long now_us, bool preload,
-                                  long long* __restrict__ R, lv_resident_result* __restrict__ out,
-                                  const long long* __restrict__ sid_dev, bool turn_end,
-                                  long long audio_us, long long units) {
-  pdl_entry();
-  if (threadIdx.x != 0) return;
-  if (sid_dev) sid = (int32_t)*sid_dev;
+__device__ void finish_step(const DevPool& p, const StepFinish& f, const long long* __restrict__ R) {
+  int32_t sid = f.sid_dev ? (int32_t)*f.sid_dev : f.sid;
   const int status = (int)R[R_STATUS];
-  if (turn_end && sid >= 0 && sid < p.S && status != LV_RESIDENT_FAILED) {
+  if (f.turn_end && sid >= 0 && sid < p.S && status != LV_RESIDENT_FAILED) {
     lv_session_state st = p.sess[sid];
     lv_event x{};
     x.kind = LV_EV_TURN_END;
     x.sid = sid;
-    x.t_us = now_us;
-    x.a = audio_us;
-    x.b = units;
+    x.t_us = f.now_us;
+    x.a = f.audio_us;
+    x.b = f.units;
     apply_event(p, st, x);
     p.sess[sid] = st;
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_EVENTS]), 1ull);
   }
-  if (preload && status == LV_RESIDENT_DONE) {
-    p.sess[sid].protect_until_us = now_us + p.protect_us;   // warmed KV (Section 5.2)
+  if (f.preload && status == LV_RESIDENT_DONE) {
+    p.sess[sid].protect_until_us = f.now_us + p.protect_us;   // warmed KV (Section 5.2)
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_PRELOADS]), 1ull);
   }
-  if (out) {
+  if (f.out) {
     lv_resident_result r;
     r.k = R[R_K];
     r.n_found = R[R_FOUND];
@@ -1580,8 +1640,13 @@ __global__ void k_resident_finish(DevPool p, int32_t sid, long long now_us, bool
     r.n_appended = (int32_t)R[R_APPENDED];
     r.status = status;
     r.sid = sid;
-    *out = r;
+    *f.out = r;
   }
+}
+
+__global__ void k_resident_finish(DevPool p, StepFinish f, const long long* __restrict__ R) {
+  pdl_entry();
+  if (threadIdx.x == 0) finish_step(p, f, R);
 }
 
 // ----------------------------------------------------------------- evict
@@ -1617,43 +1682,6 @@ k_pick_scan(DevPool p, const int32_t* __restrict__ cand, int32_t* __restrict__ h
   any = __syncthreads_or(any);
   if (threadIdx.x == 0) hit[blockIdx.x] = any;
 }
-
-// The turn's session (sid, or the first candidate with a hit, else the first
-// candidate) into R[R_SID], then LV_EV_TURN_BEGIN for it.
-__global__ void __launch_bounds__(1024)
-k_turn_begin(DevPool p, int32_t sid, const int32_t* __restrict__ cand, int32_t n,
-             const int32_t* __restrict__ hit, long long now_us, long long* __restrict__ R) {
-  pdl_entry();
-  __shared__ int first;
-  if (threadIdx.x == 0) first = n;
-  __syncthreads();
-  if (sid < 0) {
-    int mine = n;
-    for (int c = threadIdx.x; c < n; c += blockDim.x)
-      if (hit[c]) { mine = c; break; }
-    if (mine < n) atomicMin(&first, mine);
-  }
-  __syncthreads();
-  if (threadIdx.x != 0) return;
-  if (sid < 0) {
-    sid = cand[first < n ? first : 0];
-    if (sid < 0 || sid >= p.S) {
-      set_error(p.ctl, LV_ERR_BOUNDS, first < n ? first : 0);
-      R[R_SID] = -1;
-      return;
-    }
-  }
-  R[R_SID] = sid;
-  lv_session_state st = p.sess[sid];
-  lv_event x{};
-  x.kind = LV_EV_TURN_BEGIN;
-  x.sid = sid;
-  x.t_us = now_us;
-  apply_event(p, st, x);
-  p.sess[sid] = st;
-  atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_EVENTS]), 1ull);
-}
-
 
 // ------------------------------------------------------------- checksums
 constexpr int kSumThreads = 256;
@@ -1855,11 +1883,14 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
                             int4* tasks, long long* n_tasks, int32_t epoch,
                             unsigned long long* page_tag, cudaStream_t s, int copy_ctas,
                             const long long* counts_dev, long long max_units, const EventPair* ev,
-                            const long long* sid_dev, const CopyOffload* off, int gate) {
+                            const long long* sid_dev, const CopyOffload* off, int gate,
+                            long long* cursor, const StepFinish* fin) {
   long long* R = gate != GATE_NONE ? const_cast<long long*>(counts_dev) - R_N_OUT : nullptr;
+  if (R) cursor = R + R_CURSOR;
+  const StepFinish no_fin{};
   cudaError_t le = launch_pdl(k_exchange_plan, 1, kPlanThreads, 0, s, p, v, (long long)n_out, sid,
                               blks, (long long)n_in, slots, pages, tasks, n_tasks, epoch, page_tag,
-                              counts_dev, sid_dev, R, gate);
+                              counts_dev, sid_dev, R, gate, cursor, fin && R ? *fin : no_fin);
   if (le != cudaSuccess) return le;
   const long long units = counts_dev ? max_units : (n_out + n_in) * (long long)p.J;
   cudaStream_t cs = s;
@@ -1872,10 +1903,10 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
   if (ev) cudaEventRecord(ev->start, cs);
   else if (off && off->started) cudaEventRecord(off->started, cs);
   if (off || ev) {   // after an event wait or record: an ordinary launch
-    k_exchange_copy<<<blocks_for(units, 1, copy_ctas), kCopyThreads, 0, cs>>>(p, tasks, n_tasks);
+    k_exchange_copy<<<blocks_for(units, 1, copy_ctas), kCopyThreads, 0, cs>>>(p, tasks, n_tasks, cursor);
   } else {
     le = launch_pdl(k_exchange_copy, blocks_for(units, 1, copy_ctas), kCopyThreads, 0, cs, p,
-                    (const int4*)tasks, (const long long*)n_tasks);
+                    (const int4*)tasks, (const long long*)n_tasks, cursor);
     if (le != cudaSuccess) return le;
   }
   if (ev) cudaEventRecord(ev->end, cs);
@@ -1893,10 +1924,11 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
                                  lv_resident_result* result, const EventPair* ev,
                                  const long long* sid_dev, const CopyOffload* off,
                                  const unsigned long long* load_keys, bool turn_end,
-                                 int64_t audio_us, int64_t units) {
+                                 int64_t audio_us, int64_t units, const TurnStart* ts) {
   long long* R = rs.words;
+  const TurnStart none{};
   cudaError_t e = launch_pdl(k_resident_prepare, 1, kCensusThreads, 0, s, p, sid, append_tokens,
-                             preload, (long long)max_load, rs.blocks, R, sid_dev);
+                             preload, (long long)max_load, rs.blocks, R, sid_dev, ts ? *ts : none);
   if (e != cudaSuccess) return e;
   if (load_keys) {
     e = launch_pdl(k_order_loads, blocks_for(p.maxB, kOrderThreads / 32, 1ll << 30), kOrderThreads, 0,
@@ -1906,18 +1938,22 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
   e = launch_select(p, now_us, 0, !preload, rs.victims, nullptr, s, 0, R + R_K_SELECT);
   if (e != cudaSuccess) return e;
   const long long max_units = ((long long)p.budget + p.maxB) * p.J;
+  // the step's end (turn end, preload protection, result): in the plan kernel when no
+  // append follows it, else in a kernel of its own after the append
+  const StepFinish fin{true, sid, sid_dev, (long long)now_us, preload, turn_end, (long long)audio_us,
+                       (long long)units, result};
   e = launch_exchange(p, rs.victims, 0, sid, load_keys ? rs.loads : rs.blocks, 0, rs.slots, rs.pages,
                       rs.tasks, R + R_N_TASKS, epoch, p.page_tag, s, copy_ctas, R + R_N_OUT, max_units,
-                      ev, sid_dev, off, preload ? GATE_PRELOAD : GATE_RESIDENT);
+                      ev, sid_dev, off, preload ? GATE_PRELOAD : GATE_RESIDENT, nullptr,
+                      append_tokens > 0 ? nullptr : &fin);
   if (e != cudaSuccess) return e;
   if (append_tokens > 0) {
     e = launch_append(p, sid, append_tokens, rs.append, reinterpret_cast<int32_t*>(R + R_APPENDED), s,
                       R + R_GATE, sid_dev);
     if (e != cudaSuccess) return e;
+    e = launch_pdl(k_resident_finish, 1, 32, 0, s, p, fin, (const long long*)R);
+    if (e != cudaSuccess) return e;
   }
-  e = launch_pdl(k_resident_finish, 1, 32, 0, s, p, sid, (long long)now_us, preload, R, result,
-                 sid_dev, turn_end, (long long)audio_us, (long long)units);
-  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
@@ -1930,12 +1966,10 @@ cudaError_t launch_evict(const DevPool& p, const ResidentScratch& rs, int64_t no
   e = launch_select(p, now_us, 0, false, rs.victims, nullptr, s, 0, R + R_K_SELECT);
   if (e != cudaSuccess) return e;
   const long long max_units = (long long)p.budget * p.J;
+  const StepFinish fin{true, -1, nullptr, (long long)now_us, false, false, 0, 0, result};
   e = launch_exchange(p, rs.victims, 0, -1, rs.blocks, 0, rs.slots, rs.pages, rs.tasks,
                       R + R_N_TASKS, epoch, p.page_tag, s, copy_ctas, R + R_N_OUT, max_units, ev,
-                      nullptr, off, GATE_EVICT);
-  if (e != cudaSuccess) return e;
-  e = launch_pdl(k_resident_finish, 1, 32, 0, s, p, (int32_t)-1, (long long)now_us, false, R, result,
-                 (const long long*)nullptr, false, 0ll, 0ll);
+                      nullptr, off, GATE_EVICT, nullptr, &fin);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
@@ -1951,13 +1985,12 @@ cudaError_t launch_turn(const DevPool& p, const ResidentScratch& rs, int32_t sid
     e0 = launch_pdl(k_pick_scan, (unsigned)n_cand, kCensusThreads, 0, s, p, cand, rs.hits);
     if (e0 != cudaSuccess) return e0;
   }
-  e0 = launch_pdl(k_turn_begin, 1, 1024, 0, s, p, sid, cand, n_cand, (const int32_t*)rs.hits,
-                  (long long)now_us, R);
-  if (e0 != cudaSuccess) return e0;
-  // make resident, then (in its finish kernel) LV_EV_TURN_END
+  // turn start (in the prepare kernel), make resident, then (in its finish kernel)
+  // LV_EV_TURN_END
+  const TurnStart ts{true, cand, n_cand, rs.hits, (long long)now_us};
   cudaError_t e = launch_make_resident(p, rs, sid, now_us, append_tokens, false, -1, epoch, s,
                                        copy_ctas, result, ev, R + R_SID, off, load_keys, true,
-                                       audio_us, units);
+                                       audio_us, units, &ts);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
@@ -2040,26 +2073,22 @@ cudaError_t launch_exchange_plan(const DevPool& p, const lv_victim* v, int64_t n
                                  unsigned long long* page_tag, cudaStream_t s) {
   k_exchange_plan<<<1, kPlanThreads, 0, s>>>(p, v, n_out, sid, blks, n_in, slots, pages, tasks,
                                              n_tasks, epoch, page_tag, nullptr, nullptr, nullptr,
-                                             (int)GATE_NONE);
+                                             (int)GATE_NONE, nullptr, StepFinish{});
   return cudaGetLastError();
 }
 
-cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, cudaStream_t s,
-                         int num_sms, int per_thread) {
+cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, int32_t epoch,
+                         cudaStream_t s, int num_sms, int per_thread) {
   if (n <= 0) return cudaSuccess;
-  const long long resident = (long long)(num_sms > 0 ? num_sms : 1) * 2048;
-  cudaError_t err = launch_pdl(k_remap_tag, blocks_for(n, kRemapThreads, resident / kRemapThreads),
-                               kRemapThreads, 0, s, p, e, (long long)n);
-  if (err != cudaSuccess) return err;
   // one entry per thread while the GPU holds every thread at once; beyond that, up
   // to four entries per thread so that their reads overlap
+  const long long resident = (long long)(num_sms > 0 ? num_sms : 1) * 2048;
   int E = per_thread;
   if (E != 1 && E != 2 && E != 4) E = n <= resident ? 1 : (n <= 2 * resident ? 2 : 4);
   const unsigned grid = blocks_for((n + E - 1) / E, kRemapThreads, 1ll << 30);
-  if (E == 1) err = launch_pdl(k_remap_commit<1>, grid, kRemapThreads, 0, s, p, e, (long long)n);
-  else if (E == 2) err = launch_pdl(k_remap_commit<2>, grid, kRemapThreads, 0, s, p, e, (long long)n);
-  else err = launch_pdl(k_remap_commit<4>, grid, kRemapThreads, 0, s, p, e, (long long)n);
-  if (err != cudaSuccess) return err;
+  if (E == 1) k_remap<1><<<grid, kRemapThreads, 0, s>>>(p, e, n, epoch);
+  else if (E == 2) k_remap<2><<<grid, kRemapThreads, 0, s>>>(p, e, n, epoch);
+  else k_remap<4><<<grid, kRemapThreads, 0, s>>>(p, e, n, epoch);
   return cudaGetLastError();
 }
 

@@ -35,14 +35,20 @@ def pool_for(workload, device=None, stream=None, kv=None) -> KVPool:
                   device=device, stream=stream, kv=kv, policy=spec.policy, tiers=spec.tiers)
     init = workload.init
     pool.import_placement(init.placement, init.ctx_tokens)
-    st = np.zeros(spec.n_sessions, dtype=lv.SESSION_DTYPE)
+    pool.set_sessions(initial_sessions(workload))
+    pool.sync()
+    return pool
+
+
+def initial_sessions(workload) -> np.ndarray:
+    """The session table a workload starts from (lv_session_state [S])."""
+    init = workload.init
+    st = np.zeros(workload.spec.n_sessions, dtype=lv.SESSION_DTYPE)
     st["flags"] = np.where(init.resp_open != 0, lv.LV_RESP_OPEN, 0)
     st["gen_us"] = init.gen_us
     st["play_us"] = init.play_us
     st["reply_tokens"] = init.reply_tokens
-    pool.set_sessions(st)
-    pool.sync()
-    return pool
+    return st
 
 
 class ContentWriter:

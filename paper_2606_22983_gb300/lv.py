@@ -32,6 +32,7 @@ LV_POLICY_NEXT_USE, LV_POLICY_LRU = 0, 1
 LV_TIERS_EXCLUSIVE, LV_TIERS_INCLUSIVE = 0, 1
 LV_RESIDENT_ASYNC_COPY = 2
 LV_VERSION = 3                     # include/lv.h
+EMIT_SCAN_MAX = 1024               # above this many sessions a ranking runs one more kernel
 LV_MODE_ASYNC = 16
 LV_RUNNING, LV_IMMEDIATE, LV_RESP_OPEN, LV_DONE_VALID = 1, 2, 4, 8
 (LV_EV_TURN_BEGIN, LV_EV_TURN_END, LV_EV_PLAYBACK, LV_EV_SPEECH_START, LV_EV_BARGE_IN,

@@ -119,7 +119,8 @@ class KVManager:
             self.timer.start("resident")
         lv.lv_make_resident(pool.handle, sid, now_us, append_tokens, flags, -1, *outs,
                             self.res_h, pool.stream)
-        pool.launches += 6 + (1 if append_tokens else 0)
+        # prepare, census, emit, plan (with the step's end), copy; append and end after it
+        pool.launches += 5 + pool.rank_extra + (2 if append_tokens else 0)
         if self.timer:
             self.timer.stop("resident", None)
         if not rec_bufs:
@@ -170,7 +171,7 @@ class KVManager:
                    cand, int(cand.numel()) if cand is not None else 0, pool.stream,
                    lv.LV_RESIDENT_ASYNC_COPY if self.async_copy else 0, load_keys)
         pool.launches += 1 if load_keys is not None else 0
-        pool.launches += 7 + (1 if sid < 0 else 0) + (1 if append_tokens else 0)
+        pool.launches += 5 + pool.rank_extra + (1 if sid < 0 else 0) + (2 if append_tokens else 0)
         if not rec_bufs:
             return sid
         pool.sync(raise_on_error=False)
@@ -381,7 +382,7 @@ class KVManager:
         outs = (pool.victims, pool.slots) if self.record else (None, None)
         lv.lv_evict(pool.handle, now_us, int(k), lv.LV_RESIDENT_ASYNC_COPY if self.async_copy else 0,
                     *outs, self.res_h, pool.stream)
-        pool.launches += 6
+        pool.launches += 5 + pool.rank_extra
         rec["k"] = int(k)
         if not self.record:
             return

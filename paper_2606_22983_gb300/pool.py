@@ -39,6 +39,8 @@ class KVPool:
         self.S, self.max_blocks = max_sessions, max_blocks
         self.hbm_pages, self.budget, self.host_pages = hbm_pages, hbm_budget_pages, host_pages
         self.launches = 0      # liblv kernels launched through this object
+        # a ranking is two kernels, three above 1024 sessions (liblv's k_rank_prefix)
+        self.rank_extra = 1 if max_sessions > lv.EMIT_SCAN_MAX else 0
         self.policy = policy
         self.tiers = tiers
         with torch.cuda.device(self.device):
@@ -135,7 +137,7 @@ class KVPool:
                                                                 device=self.device)
         lv.lv_select_victims(self.handle, now_us, min(k, lv.LV_ALL), flags, out, cap,
                              self.count_h[0:1], self.stream)
-        self.launches += 2
+        self.launches += 2 + self.rank_extra
         self.sync()
         n = int(self.count_h[0])
         return out[:n], n
