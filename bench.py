@@ -889,7 +889,8 @@ def kernel_micro(torch, pool, seed=0):
         out["ranker"]["sessions_4096"] = _ranker_4096(torch, pool, seed)
         # remap: the commit of all 2^20 pages to the host tier.  Each repetition
         # re-imports the placement, swaps everything out, flushes L2 (a 256 MB
-        # write) and times one k_remap launch; the first repetition is untimed.
+        # write) and times one lv_remap call (its commit and release passes); the first
+        # repetition is untimed.
         placement = rng.permutation(N).astype(np.int32).reshape(S, B)
         ctx = np.full(S, B * 16, np.int32)
         flush = torch.empty(256 << 20, dtype=torch.uint8, device=pool.device)

@@ -11,6 +11,9 @@ namespace lv {
 // Owner words: the (sid << 16 | blk) that owns a page or slot, or one of two states.
 constexpr uint32_t kOwnerNone = 0xFFFFFFFFu;       // free
 constexpr uint32_t kOwnerReserved = 0xFFFFFFFEu;   // reserved by a swap, not yet committed
+// freed by lv_remap's commit pass; its release pass makes it kOwnerNone and clears
+// the bitmap bit (no key reaches this value: sid < 4096)
+constexpr uint32_t kOwnerFreeing = 0xFFFFFFFDu;
 constexpr long long kKeyMax = 0xFFFFFFFFll;   // T_next is clamped to 32 bits (microseconds)
 
 // Layout of the per-pool int64 control block in device memory.

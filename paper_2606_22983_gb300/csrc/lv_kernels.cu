@@ -1193,6 +1193,7 @@ __global__ void k_selftest_wait(long long* ctl, long long limit_ns) {
 
 // ---------------------------------------------------------------- commit
 constexpr int kRemapThreads = 256;
+constexpr int kReleaseThreads = 256;
 
 // The reads of one entry that do not depend on a check.
 struct RemapRead {
@@ -1201,7 +1202,6 @@ struct RemapRead {
   int32_t old;          // the block's current location
   int32_t g;            // its clean-copy slot (inclusive tiers), or -1
   int32_t nb;           // blocks of its session
-  uint32_t old_owner;   // owner word of the current location
   bool in_range;
 };
 
@@ -1222,20 +1222,21 @@ __device__ __forceinline__ void remap_read_table(const DevPool& p, RemapRead& r)
   r.nb = r.in_range ? nblocks_of(p, r.x.sid) : 0;
 }
 
-__device__ __forceinline__ void remap_read_owner(const DevPool& p, RemapRead& r) {
-  const long long old_slot = -(long long)r.old - 2;
-  r.old_owner = kOwnerNone;
-  if (r.old >= 0 && r.old < p.hbm_pages) r.old_owner = p.own_hbm[r.old];
-  else if (r.old <= -2 && old_slot < p.host_pages) r.old_owner = p.own_host[old_slot];
+// The block's epoch mark: one accepted entry per block per call.  It depends on
+// the entry alone, so it is issued with the entry's table reads; a mark made for
+// a block past its session's context is harmless (every entry naming that block
+// fails the same range check).  A returning atomic: the caller issues every
+// entry's mark before it looks at any result.
+__device__ __forceinline__ void remap_mark(const DevPool& p, const RemapRead& r, int32_t epoch,
+                                           int32_t& seen) {
+  seen = r.in_range ? atomicExch(&p.mark[r.ti], epoch) : 0;
 }
 
-// The block's epoch mark: one accepted entry per block per call.  Returns the
-// entry's error so far (a returning atomic; the caller issues every entry's
-// mark before it looks at any result).
-__device__ __forceinline__ int remap_mark(const DevPool& p, const RemapRead& r, int32_t epoch,
-                                          int32_t& seen) {
+// The entry's error once its table reads and mark are back: range first, then
+// a second entry for the same block.
+__device__ __forceinline__ int remap_judge(const RemapRead& r, int32_t epoch, int32_t seen) {
   if (!r.in_range || r.x.blk >= r.nb) return LV_ERR_BOUNDS;
-  seen = atomicExch(&p.mark[r.ti], epoch);
+  if (seen == epoch) return LV_ERR_DOUBLE_MAP;
   return 0;
 }
 
@@ -1258,9 +1259,14 @@ __device__ __forceinline__ int remap_claim(const DevPool& p, const RemapRead& r,
   return 0;
 }
 
-// Judges the claim and applies the entry: table, clean copy, old location.
+// Judges the claim and applies the entry: table, clean copy, old location.  A
+// location that the entry frees is exchanged to kOwnerFreeing (the release pass
+// after the commit makes it free and clears its bitmap bit); the exchange returns
+// the old location's owner word into `was` (kOwnerNone when nothing was freed), for
+// the consistency check the caller makes once every entry has been applied.
 __device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& r, int err,
-                                            uint32_t got, long long i, RemapCounts& c) {
+                                            uint32_t got, long long i, RemapCounts& c,
+                                            uint32_t& was) {
   const lv_remap_entry& x = r.x;
   const int32_t old = r.old, g = r.g;
   const long long old_slot = -(long long)old - 2;
@@ -1268,6 +1274,7 @@ __device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& r
   const bool old_host = old <= -2 && old_slot < p.host_pages;
   const long long h = -(long long)x.loc - 2;
   const uint32_t key = owner_key(x.sid, x.blk);
+  was = key;
   if (!err && got != kOwnerReserved) {
     // a host location already owned by this block is fine only as its own clean copy
     if (!(x.loc <= -2 && p.incl && (long long)g == h && got == key)) err = LV_ERR_DOUBLE_MAP;
@@ -1281,24 +1288,21 @@ __device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& r
     p.shadow[r.ti] = -1;
     c.clean -= 1;
     if ((long long)g != h) {
-      p.own_host[g] = kOwnerNone;
-      atomicAnd(&p.bits_host[g >> 5], ~(1u << (g & 31)));
+      atomicExch(&p.own_host[g], kOwnerFreeing);
       c.host += 1;
     }
   }
   // the old location belongs to this block alone (one entry per block per call)
-  if (old_hbm || old_host) {
-    if (r.old_owner != key) set_error(p.ctl, LV_ERR_STATE, i);
-    if (old_hbm) {
-      p.own_hbm[old] = kOwnerNone;
-      atomicAnd(&p.bits_hbm[old >> 5], ~(1u << (old & 31)));
-      c.hbm += 1;
-    } else if (p.incl && x.loc >= 0) {   // back in HBM: the host slot stays as its clean copy
+  if (old_hbm) {
+    was = atomicExch(&p.own_hbm[old], kOwnerFreeing);
+    c.hbm += 1;
+  } else if (old_host) {
+    if (p.incl && x.loc >= 0) {         // back in HBM: the host slot stays as its clean copy
+      was = p.own_host[old_slot];
       p.shadow[r.ti] = (int32_t)old_slot;
       c.clean += 1;
     } else {
-      p.own_host[old_slot] = kOwnerNone;
-      atomicAnd(&p.bits_host[old_slot >> 5], ~(1u << (old_slot & 31)));
+      was = atomicExch(&p.own_host[old_slot], kOwnerFreeing);
       c.host += 1;
     }
   }
@@ -1312,48 +1316,52 @@ __device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& r
 // committed to HBM from the host tier keeps its slot as its clean copy; a
 // block committed to another host slot loses its copy.
 //
-// The kernel is bound by the latency of dependent scattered accesses (entry ->
-// table entry -> owner of the old location -> epoch mark -> claim of the new
-// location), so each step is issued for all E entries of the thread before any
-// of its results is used: every read that does not depend on a check, then
-// every mark, then every claim, then the stores.  E chains then wait together.  The early
+// The kernel is bound by the latency of dependent scattered accesses, so each
+// round of requests is issued for all E entries of the thread before any of its
+// results is used, and requests that do not depend on one another share a
+// round: (1) the entries; (2) the block's table word, its session's block count
+// and the block's epoch mark; (3) the claim of the new location (only for an
+// entry that passed its range check and its mark) together with the owner word
+// of the old location; (4) the stores.  E chains then wait together.  The early
 // reads are race-free within one call: a block has at most one accepted entry
 // (the epoch mark), a location freed by one entry is never the new location of
 // another (new locations are reservations), and another entry can take an
 // owned location only through a CAS, which then fails.  A thread's own
 // entries apply in order, so a duplicate among them meets the epoch mark too.
 template <int E>
-__global__ void __launch_bounds__(kRemapThreads)
+__global__ void __launch_bounds__(kRemapThreads, 4)
 k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t epoch) {
   const long long stride = (long long)gridDim.x * kRemapThreads;
   const long long i0 = blockIdx.x * (long long)kRemapThreads + threadIdx.x;
   RemapRead r[E];
+  int32_t seen[E];
 #pragma unroll
   for (int j = 0; j < E; ++j) remap_read_entry(p, e, i0 + j * stride, n, r[j]);
 #pragma unroll
-  for (int j = 0; j < E; ++j) remap_read_table(p, r[j]);
-#pragma unroll
-  for (int j = 0; j < E; ++j) remap_read_owner(p, r[j]);
-  // the atomics of all E entries: every mark, then every claim, each group in flight
-  // together; a thread's own duplicate meets the mark of its earlier entry
+  for (int j = 0; j < E; ++j) {
+    remap_read_table(p, r[j]);
+    remap_mark(p, r[j], epoch, seen[j]);
+  }
   int err[E];
-  int32_t seen[E];
   uint32_t got[E];
 #pragma unroll
   for (int j = 0; j < E; ++j) {
-    seen[j] = 0;
-    err[j] = i0 + j * stride < n ? remap_mark(p, r[j], epoch, seen[j]) : -1;
-  }
-#pragma unroll
-  for (int j = 0; j < E; ++j) {
-    if (err[j] == 0 && seen[j] == epoch) err[j] = LV_ERR_DOUBLE_MAP;   // same block twice
     got[j] = kOwnerReserved;
+    err[j] = i0 + j * stride < n ? remap_judge(r[j], epoch, seen[j]) : -1;
     if (err[j] >= 0) err[j] = remap_claim(p, r[j], err[j], got[j]);
   }
   RemapCounts c{0, 0, 0, 0};
+  uint32_t was[E];
+#pragma unroll
+  for (int j = 0; j < E; ++j) {
+    was[j] = kOwnerNone;
+    if (err[j] >= 0) remap_apply(p, r[j], err[j], got[j], i0 + j * stride, c, was[j]);
+  }
+  // a freed location that this block did not own means the tables were inconsistent
 #pragma unroll
   for (int j = 0; j < E; ++j)
-    if (err[j] >= 0) remap_apply(p, r[j], err[j], got[j], i0 + j * stride, c);
+    if (was[j] != kOwnerNone && was[j] != owner_key(r[j].x.sid, r[j].x.blk))
+      set_error(p.ctl, LV_ERR_STATE, i0 + j * stride);
   // block totals: warp sums, one shared atomic per warp, one global atomic per block
   __shared__ int tot[4];
   if (threadIdx.x < 4) tot[threadIdx.x] = 0;
@@ -1372,6 +1380,47 @@ k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t ep
     if (tot[2]) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HOST_ALLOC]), (unsigned long long)-(long long)tot[2]);
     if (tot[0]) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_REMAP]), (unsigned long long)tot[0]);
     if (tot[3]) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_CLEAN]), (unsigned long long)(long long)tot[3]);
+  }
+}
+
+// The commit's second pass: every owner word that the commit exchanged to
+// kOwnerFreeing becomes kOwnerNone, and its bit is cleared in the allocation
+// bitmap with one reduction per bitmap word (the commit itself would issue one
+// reduction per freed page, 32 to a word when a whole run of pages is freed).
+// Thread q reads owner words 4q..4q+3 of its tier with one 16-byte load; the 8
+// threads of a bitmap word combine their bits with shuffles.  Quads [0, qh) are
+// the HBM pages and [qh, qh + qo) the host slots; qh and qo are multiples of 8,
+// so the 8 threads of a word are always 8 aligned lanes of one tier.  Only the
+// freed words are written, so concurrent work on other pages is left alone.
+__global__ void __launch_bounds__(kReleaseThreads)
+k_release(DevPool p, long long qh, long long qo) {
+  pdl_wait();   // the commit is complete and visible
+  const long long total = qh + qo;
+  const int lane8 = threadIdx.x & 7;
+  for (long long q0 = (long long)blockIdx.x * kReleaseThreads; q0 < total;
+       q0 += (long long)gridDim.x * kReleaseThreads) {
+    const long long q = q0 + threadIdx.x;
+    const bool hbm = q < qh;
+    uint32_t* own = hbm ? p.own_hbm : p.own_host;
+    const long long n = hbm ? p.hbm_pages : p.host_pages;
+    const long long base = (hbm ? q : q - qh) * 4;
+    uint32_t m = 0;
+    if (q < total && base < n) {
+      if (base + 3 < n) {
+        const uint4 v = *reinterpret_cast<const uint4*>(own + base);
+        m = (uint32_t)(v.x == kOwnerFreeing) | (uint32_t)(v.y == kOwnerFreeing) << 1 |
+            (uint32_t)(v.z == kOwnerFreeing) << 2 | (uint32_t)(v.w == kOwnerFreeing) << 3;
+      } else {
+        for (int k = 0; base + k < n; ++k) m |= (uint32_t)(own[base + k] == kOwnerFreeing) << k;
+      }
+      for (int k = 0; k < 4; ++k)
+        if (m >> k & 1u) own[base + k] = kOwnerNone;
+    }
+    uint32_t w = m << (4 * lane8);
+    w |= __shfl_xor_sync(0xffffffffu, w, 1);
+    w |= __shfl_xor_sync(0xffffffffu, w, 2);
+    w |= __shfl_xor_sync(0xffffffffu, w, 4);
+    if (lane8 == 0 && w) atomicAnd(&(hbm ? p.bits_hbm : p.bits_host)[base >> 5], ~w);
   }
 }
 
@@ -2089,6 +2138,16 @@ cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, i
   if (E == 1) k_remap<1><<<grid, kRemapThreads, 0, s>>>(p, e, n, epoch);
   else if (E == 2) k_remap<2><<<grid, kRemapThreads, 0, s>>>(p, e, n, epoch);
   else k_remap<4><<<grid, kRemapThreads, 0, s>>>(p, e, n, epoch);
+  cudaError_t err = cudaGetLastError();
+  if (err != cudaSuccess) return err;
+  // the release pass over both tiers' owner words (8 quads of 4 per bitmap word)
+  const long long qh = (long long)((p.hbm_pages + 31) / 32) * 8;
+  const long long qo = (long long)((p.host_pages + 31) / 32) * 8;
+  const long long cap = (long long)(num_sms > 0 ? num_sms : 1) * 8;
+  long long rg = (qh + qo + kReleaseThreads - 1) / kReleaseThreads;
+  if (rg > cap) rg = cap;
+  err = launch_pdl(k_release, dim3((unsigned)rg), kReleaseThreads, 0, s, p, qh, qo);
+  if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
 

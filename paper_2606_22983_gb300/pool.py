@@ -161,7 +161,7 @@ class KVPool:
 
     def remap(self, entries, n: int):
         lv.lv_remap(self.handle, entries, n, self.stream)
-        self.launches += 1
+        self.launches += 2 if n > 0 else 0
 
     def cancel(self, locs, n: int):
         lv.lv_cancel(self.handle, locs, n, self.stream)
