@@ -1240,33 +1240,51 @@ __device__ __forceinline__ int remap_judge(const RemapRead& r, int32_t epoch, in
   return 0;
 }
 
-// The new location must be a reservation nobody owns yet: one CAS checks and
-// takes it.  Issued for every entry that passed its mark, before any result is read.
+// Round 3 of an entry that passed its range check and its mark.  The claim of the
+// new location (one CAS checks that it is a reservation nobody owns and takes it)
+// goes out together with the entry's own writes, made before the claim's result
+// is known: the table word, and the old location exchanged to kOwnerFreeing
+// (which returns its owner word into `was`, for the consistency check).  The
+// release pass after the commit makes a kOwnerFreeing word free and clears its
+// bitmap bit.  A claim that fails undoes the writes in remap_settle; until then
+// no other entry of the call can see them, since only an entry for the same
+// block reads its table word (and the mark turned it away), and every claim of
+// an owned location fails, kOwnerFreeing or not.
 __device__ __forceinline__ int remap_claim(const DevPool& p, const RemapRead& r, int err,
-                                           uint32_t& got) {
+                                           uint32_t& got, uint32_t& was) {
   if (err) return err;
   const lv_remap_entry& x = r.x;
   const uint32_t key = owner_key(x.sid, x.blk);
+  uint32_t* own;
   if (x.loc >= 0) {
     if (x.loc >= p.hbm_pages) return LV_ERR_BOUNDS;
-    got = atomicCAS(&p.own_hbm[x.loc], kOwnerReserved, key);
+    own = &p.own_hbm[x.loc];
   } else if (x.loc <= -2) {
     if (-(long long)x.loc - 2 >= p.host_pages) return LV_ERR_BOUNDS;
-    got = atomicCAS(&p.own_host[-(long long)x.loc - 2], kOwnerReserved, key);
+    own = &p.own_host[-(long long)x.loc - 2];
   } else {
     return LV_ERR_BOUNDS;
   }
+  got = atomicCAS(own, kOwnerReserved, key);
+  const int32_t old = r.old;
+  const long long old_slot = -(long long)old - 2;
+  if (old >= 0 && old < p.hbm_pages) {
+    was = atomicExch(&p.own_hbm[old], kOwnerFreeing);
+  } else if (old <= -2 && old_slot < p.host_pages) {
+    if (p.incl && x.loc >= 0) was = p.own_host[old_slot];   // back in HBM: the slot stays as its clean copy
+    else was = atomicExch(&p.own_host[old_slot], kOwnerFreeing);
+  }
+  p.table[r.ti] = x.loc;
   return 0;
 }
 
-// Judges the claim and applies the entry: table, clean copy, old location.  A
-// location that the entry frees is exchanged to kOwnerFreeing (the release pass
-// after the commit makes it free and clears its bitmap bit); the exchange returns
-// the old location's owner word into `was` (kOwnerNone when nothing was freed), for
-// the consistency check the caller makes once every entry has been applied.
-__device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& r, int err,
-                                            uint32_t got, long long i, RemapCounts& c,
-                                            uint32_t& was) {
+// Judges the claim once its result is back.  A failed claim is a double map and
+// its entry's writes are put back; an accepted entry settles its clean copy
+// (inclusive tiers) and is counted, and a freed location that this block did not
+// own means the tables were inconsistent.
+__device__ __forceinline__ void remap_settle(const DevPool& p, const RemapRead& r, int err,
+                                             uint32_t got, uint32_t was, long long i,
+                                             RemapCounts& c) {
   const lv_remap_entry& x = r.x;
   const int32_t old = r.old, g = r.g;
   const long long old_slot = -(long long)old - 2;
@@ -1274,16 +1292,19 @@ __device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& r
   const bool old_host = old <= -2 && old_slot < p.host_pages;
   const long long h = -(long long)x.loc - 2;
   const uint32_t key = owner_key(x.sid, x.blk);
-  was = key;
   if (!err && got != kOwnerReserved) {
     // a host location already owned by this block is fine only as its own clean copy
-    if (!(x.loc <= -2 && p.incl && (long long)g == h && got == key)) err = LV_ERR_DOUBLE_MAP;
+    if (!(x.loc <= -2 && p.incl && (long long)g == h && got == key)) {
+      err = LV_ERR_DOUBLE_MAP;
+      p.table[r.ti] = old;
+      if (old_hbm) p.own_hbm[old] = was;
+      else if (old_host && !(p.incl && x.loc >= 0)) p.own_host[old_slot] = was;
+    }
   }
   if (err) {
     set_error(p.ctl, err, i);
     return;
   }
-  p.table[r.ti] = x.loc;
   if (x.loc <= -2 && g >= 0) {          // the copy becomes the location, or goes
     p.shadow[r.ti] = -1;
     c.clean -= 1;
@@ -1292,20 +1313,17 @@ __device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& r
       c.host += 1;
     }
   }
-  // the old location belongs to this block alone (one entry per block per call)
   if (old_hbm) {
-    was = atomicExch(&p.own_hbm[old], kOwnerFreeing);
     c.hbm += 1;
   } else if (old_host) {
-    if (p.incl && x.loc >= 0) {         // back in HBM: the host slot stays as its clean copy
-      was = p.own_host[old_slot];
+    if (p.incl && x.loc >= 0) {
       p.shadow[r.ti] = (int32_t)old_slot;
       c.clean += 1;
     } else {
-      was = atomicExch(&p.own_host[old_slot], kOwnerFreeing);
       c.host += 1;
     }
   }
+  if (was != kOwnerNone && was != key) set_error(p.ctl, LV_ERR_STATE, i);
   c.ok += 1;
 }
 
@@ -1320,14 +1338,15 @@ __device__ __forceinline__ void remap_apply(const DevPool& p, const RemapRead& r
 // round of requests is issued for all E entries of the thread before any of its
 // results is used, and requests that do not depend on one another share a
 // round: (1) the entries; (2) the block's table word, its session's block count
-// and the block's epoch mark; (3) the claim of the new location (only for an
-// entry that passed its range check and its mark) together with the owner word
-// of the old location; (4) the stores.  E chains then wait together.  The early
-// reads are race-free within one call: a block has at most one accepted entry
-// (the epoch mark), a location freed by one entry is never the new location of
-// another (new locations are reservations), and another entry can take an
-// owned location only through a CAS, which then fails.  A thread's own
-// entries apply in order, so a duplicate among them meets the epoch mark too.
+// and the block's epoch mark; (3) the claim of the new location, the table word
+// and the exchange of the old location's owner word (only for an entry that
+// passed its range check and its mark; the writes are undone if the claim
+// fails).  E chains then wait together.  The early reads are race-free within
+// one call: a block has at most one accepted entry (the epoch mark), a location
+// freed by one entry is never the new location of another (new locations are
+// reservations), and another entry can take an owned location only through a
+// CAS, which then fails.  A thread's own entries are issued in order, so a
+// duplicate among them meets the epoch mark too.
 template <int E>
 __global__ void __launch_bounds__(kRemapThreads, 4)
 k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t epoch) {
@@ -1343,25 +1362,18 @@ k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t ep
     remap_mark(p, r[j], epoch, seen[j]);
   }
   int err[E];
-  uint32_t got[E];
+  uint32_t got[E], was[E];
 #pragma unroll
   for (int j = 0; j < E; ++j) {
     got[j] = kOwnerReserved;
+    was[j] = kOwnerNone;
     err[j] = i0 + j * stride < n ? remap_judge(r[j], epoch, seen[j]) : -1;
-    if (err[j] >= 0) err[j] = remap_claim(p, r[j], err[j], got[j]);
+    if (err[j] >= 0) err[j] = remap_claim(p, r[j], err[j], got[j], was[j]);
   }
   RemapCounts c{0, 0, 0, 0};
-  uint32_t was[E];
-#pragma unroll
-  for (int j = 0; j < E; ++j) {
-    was[j] = kOwnerNone;
-    if (err[j] >= 0) remap_apply(p, r[j], err[j], got[j], i0 + j * stride, c, was[j]);
-  }
-  // a freed location that this block did not own means the tables were inconsistent
 #pragma unroll
   for (int j = 0; j < E; ++j)
-    if (was[j] != kOwnerNone && was[j] != owner_key(r[j].x.sid, r[j].x.blk))
-      set_error(p.ctl, LV_ERR_STATE, i0 + j * stride);
+    if (err[j] >= 0) remap_settle(p, r[j], err[j], got[j], was[j], i0 + j * stride, c);
   // block totals: warp sums, one shared atomic per warp, one global atomic per block
   __shared__ int tot[4];
   if (threadIdx.x < 4) tot[threadIdx.x] = 0;
@@ -1390,37 +1402,62 @@ k_remap(DevPool p, const lv_remap_entry* __restrict__ e, long long n, int32_t ep
 // Thread q reads owner words 4q..4q+3 of its tier with one 16-byte load; the 8
 // threads of a bitmap word combine their bits with shuffles.  Quads [0, qh) are
 // the HBM pages and [qh, qh + qo) the host slots; qh and qo are multiples of 8,
-// so the 8 threads of a word are always 8 aligned lanes of one tier.  Only the
-// freed words are written, so concurrent work on other pages is left alone.
+// so the 8 threads of a word are always 8 aligned lanes of one tier.  Each thread
+// issues the loads of kReleaseUnroll quads, a grid's width apart, before it looks
+// at any of them.  Only the freed words are written, so concurrent work on other
+// pages is left alone.
+constexpr int kReleaseUnroll = 2;
+
+__device__ __forceinline__ uint4 release_load(const DevPool& p, long long q, long long qh,
+                                              long long total) {
+  uint4 v = make_uint4(kOwnerNone, kOwnerNone, kOwnerNone, kOwnerNone);
+  if (q >= total) return v;
+  const bool hbm = q < qh;
+  const uint32_t* own = hbm ? p.own_hbm : p.own_host;
+  const long long n = hbm ? p.hbm_pages : p.host_pages;
+  const long long base = (hbm ? q : q - qh) * 4;
+  if (base + 3 < n) {
+    v = *reinterpret_cast<const uint4*>(own + base);
+  } else {
+    if (base < n) v.x = own[base];
+    if (base + 1 < n) v.y = own[base + 1];
+    if (base + 2 < n) v.z = own[base + 2];
+  }
+  return v;
+}
+
+__device__ __forceinline__ void release_apply(const DevPool& p, long long q, long long qh,
+                                              long long total, uint4 v, int lane8) {
+  const bool hbm = q < qh;
+  uint32_t* own = hbm ? p.own_hbm : p.own_host;
+  const long long base = (hbm ? q : q - qh) * 4;
+  uint32_t m = 0;
+  if (q < total) {
+    m = (uint32_t)(v.x == kOwnerFreeing) | (uint32_t)(v.y == kOwnerFreeing) << 1 |
+        (uint32_t)(v.z == kOwnerFreeing) << 2 | (uint32_t)(v.w == kOwnerFreeing) << 3;
+    for (int k = 0; k < 4; ++k)
+      if (m >> k & 1u) own[base + k] = kOwnerNone;
+  }
+  uint32_t w = m << (4 * lane8);
+  w |= __shfl_xor_sync(0xffffffffu, w, 1);
+  w |= __shfl_xor_sync(0xffffffffu, w, 2);
+  w |= __shfl_xor_sync(0xffffffffu, w, 4);
+  if (lane8 == 0 && w) atomicAnd(&(hbm ? p.bits_hbm : p.bits_host)[base >> 5], ~w);
+}
+
 __global__ void __launch_bounds__(kReleaseThreads)
 k_release(DevPool p, long long qh, long long qo) {
   pdl_wait();   // the commit is complete and visible
   const long long total = qh + qo;
+  const long long step = (long long)gridDim.x * kReleaseThreads;
   const int lane8 = threadIdx.x & 7;
-  for (long long q0 = (long long)blockIdx.x * kReleaseThreads; q0 < total;
-       q0 += (long long)gridDim.x * kReleaseThreads) {
-    const long long q = q0 + threadIdx.x;
-    const bool hbm = q < qh;
-    uint32_t* own = hbm ? p.own_hbm : p.own_host;
-    const long long n = hbm ? p.hbm_pages : p.host_pages;
-    const long long base = (hbm ? q : q - qh) * 4;
-    uint32_t m = 0;
-    if (q < total && base < n) {
-      if (base + 3 < n) {
-        const uint4 v = *reinterpret_cast<const uint4*>(own + base);
-        m = (uint32_t)(v.x == kOwnerFreeing) | (uint32_t)(v.y == kOwnerFreeing) << 1 |
-            (uint32_t)(v.z == kOwnerFreeing) << 2 | (uint32_t)(v.w == kOwnerFreeing) << 3;
-      } else {
-        for (int k = 0; base + k < n; ++k) m |= (uint32_t)(own[base + k] == kOwnerFreeing) << k;
-      }
-      for (int k = 0; k < 4; ++k)
-        if (m >> k & 1u) own[base + k] = kOwnerNone;
-    }
-    uint32_t w = m << (4 * lane8);
-    w |= __shfl_xor_sync(0xffffffffu, w, 1);
-    w |= __shfl_xor_sync(0xffffffffu, w, 2);
-    w |= __shfl_xor_sync(0xffffffffu, w, 4);
-    if (lane8 == 0 && w) atomicAnd(&(hbm ? p.bits_hbm : p.bits_host)[base >> 5], ~w);
+  for (long long q0 = (long long)blockIdx.x * kReleaseThreads + threadIdx.x;
+       q0 - threadIdx.x < total; q0 += kReleaseUnroll * step) {
+    uint4 v[kReleaseUnroll];
+#pragma unroll
+    for (int u = 0; u < kReleaseUnroll; ++u) v[u] = release_load(p, q0 + u * step, qh, total);
+#pragma unroll
+    for (int u = 0; u < kReleaseUnroll; ++u) release_apply(p, q0 + u * step, qh, total, v[u], lane8);
   }
 }
 
@@ -2144,7 +2181,8 @@ cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, i
   const long long qh = (long long)((p.hbm_pages + 31) / 32) * 8;
   const long long qo = (long long)((p.host_pages + 31) / 32) * 8;
   const long long cap = (long long)(num_sms > 0 ? num_sms : 1) * 8;
-  long long rg = (qh + qo + kReleaseThreads - 1) / kReleaseThreads;
+  const long long per_cta = (long long)kReleaseThreads * kReleaseUnroll;
+  long long rg = (qh + qo + per_cta - 1) / per_cta;
   if (rg > cap) rg = cap;
   err = launch_pdl(k_release, dim3((unsigned)rg), kReleaseThreads, 0, s, p, qh, qo);
   if (err != cudaSuccess) return err;
