@@ -24,6 +24,7 @@ import argparse
 import json
 import os
 import statistics
+import select
 import subprocess
 import sys
 import time
@@ -72,16 +73,23 @@ class ClockSampler:
     def __init__(self, gpu_index):
         self.gpu = gpu_index
         self.proc = None
-        self.lines = []
+        self.first = ""
 
-    def start(self):
+    def start(self, wait_s=10.0):
+        """Starts sampling and returns once the first sample is in (or after wait_s), so
+        that nvidia-smi's start-up (NVML initialisation) is over before the caller's
+        timed region begins."""
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except (OSError, ValueError):
             self.proc = None
+            return
+        ready, _, _ = select.select([self.proc.stdout], [], [], wait_s)
+        if ready:
+            self.first = self.proc.stdout.readline()
 
     def stop(self):
         if not self.proc:
@@ -92,6 +100,8 @@ class ClockSampler:
         except subprocess.TimeoutExpired:
             self.proc.kill()
             out, _ = self.proc.communicate()
+        if not out.strip():       # nothing after the start-up sample: report that one
+            out = self.first
         sm, mx, reasons = [], [], set()
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
         for line in out.strip().splitlines():
@@ -171,13 +181,12 @@ def ours(args, torch):
         dev_events.append(torch.from_numpy(ev.view(np.uint8).copy()).to(pool.device))
     torch.cuda.synchronize()
 
-    # the clock sampler starts before the warm-up, so that its start-up (NVML
-    # initialisation) is over before the timed region; it samples throughout it
+    # the clock sampler's start-up (NVML initialisation) is over before the warm-up, and
+    # it samples throughout the timed region
     clocks = ClockSampler(local)
     clocks.start()
     run_turns(gm, wl, 0, W, dev_events)                         # warm-up
     pool.sync()
-    time.sleep(0.5)
     p0, o0, i0 = _moved_pages(pool)
     lv.lv_timing_read(pool.handle, reset=True)
     lv.lv_timing_enable(pool.handle, True)
@@ -622,7 +631,7 @@ def _streamed_with_consumer(torch, pool, wl, moves, seed):
         st0 = pool.stats()
         with torch.cuda.stream(torch.cuda.Stream(device=pool.device, priority=-1)):
             gm = KVManager(pool, perms=wl.perms, rank_on="none", record=False, driver="device",
-                           order_fn=scatter_order, async_copy=True)
+                           order_fn=scatter_order, async_copy=True, script=wl)
             ends = None
             if label == "with_consumer":
                 cons = ChecksumConsumer(torch, pool, seed=seed)
@@ -676,7 +685,7 @@ def five_workloads(torch, seed, consumer_on="mixed"):
         try:
             fill_random(pool, seed)
             gm = KVManager(pool, perms=wl.perms, rank_on="none", record=False, driver="device",
-                           order_fn=scatter_order)
+                           order_fn=scatter_order, script=wl)
             copies = {}
             moves, turn_ms, _, wall = run_events(torch, pool, gm, wl, wl.n_events, copy_times=copies)
             nbytes = peak_bytes(pool, moves)
@@ -692,7 +701,7 @@ def five_workloads(torch, seed, consumer_on="mixed"):
                 cons = ChecksumConsumer(torch, pool, seed=seed)
                 alone = cons.alone_gbs()
                 gm2 = KVManager(pool, perms=wl.perms, rank_on="none", record=False, driver="device",
-                                order_fn=scatter_order)
+                                order_fn=scatter_order, script=wl)
                 with torch.cuda.stream(torch.cuda.Stream(device=pool.device, priority=-1)):
                     cons.top_up()
                     done = cons.window()

@@ -55,7 +55,7 @@ def main(argv=None) -> int:
                                      perms=wl.perms, mode=args.mode, order_fn=scatter_order)
         else:
             gm = KVManager(pool, perms=wl.perms, rank_on="none", record=args.record, driver=args.driver,
-                           mode=args.mode, order_fn=scatter_order)
+                           mode=args.mode, order_fn=scatter_order, script=wl)
         n = wl.n_events if args.events <= 0 else min(args.events, wl.n_events)
         copies = {}
         moves, turn_ms, load_ms, wall = run_events(torch, pool, gm, wl, n, copy_times=copies)

@@ -66,7 +66,7 @@ def load_keys(order_fn, order_key, n_blocks):
 class KVManager:
     def __init__(self, pool: KVPool, perms=None, on_append=None, rank_on="none", admit=None,
                  mode=lv.LV_MODE_AUTO, record=True, driver="device", order_fn=None,
-                 async_copy=False):
+                 async_copy=False, script=None):
         self.pool = pool
         # device driver: turns' page copies on the pool's copy stream, overlapping the
         # next turn's decisions (LV_RESIDENT_ASYNC_COPY); exchange driver, staged mode:
@@ -94,6 +94,22 @@ class KVManager:
         self.bytes_moved = 0
         self.timer = None               # optional start(name) / stop(name, bytes) hooks
         self.last_readback_bytes = 0    # bytes of lists read back to the host by the last step
+        # the load keys of a script's scattered-reload turns, resident on the device
+        self._keys_dev, self._keys_row = None, {}
+        if script is not None and order_fn is not None:
+            self.stage_load_keys(script)
+
+    def stage_load_keys(self, wl):
+        """Uploads once the per-block load keys of every scattered-reload turn of the
+        script ``wl``.  They are script input, like the events: a turn then passes a
+        device pointer to its row instead of computing its keys and staging them."""
+        sel = np.nonzero(np.asarray(wl.kind) == EV_TURN_SCATTER)[0]
+        order_keys = sorted({int(k) for k in np.asarray(wl.a)[sel]})
+        if not order_keys:
+            return
+        rows = np.stack([self._load_keys(k) for k in order_keys])
+        self._keys_dev = torch.from_numpy(rows.view(np.int64)).to(self.pool.device)
+        self._keys_row = {k: i for i, k in enumerate(order_keys)}
 
     # ------------------------------------------------------------- queries
     def free_budget(self) -> int:
@@ -418,7 +434,9 @@ class KVManager:
             self.counters["turns"] += 1
         elif kind == EV_TURN_SCATTER and self.driver == "device" and self.order_fn is not None:
             # the reload order is the script's scatter order, given as per-block keys
-            sid = self._device_turn(-1, d, t, 0, b, c, rec, load_keys=self._load_keys(a))
+            row = self._keys_row.get(a)
+            keys = self._keys_dev[row] if row is not None else self._load_keys(a)
+            sid = self._device_turn(-1, d, t, 0, b, c, rec, load_keys=keys)
             self.counters["turns"] += 1
         elif kind in (EV_TURN, EV_TURN_ANY, EV_TURN_SCATTER):
             order_key = None

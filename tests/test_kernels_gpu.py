@@ -250,6 +250,80 @@ def test_remap_cancel_and_allocation_errors():
         pool.close()
 
 
+def _owner_words(owner, used):
+    """The oracle's owners as the library's owner words (sid << 16 | blk, reserved, free)."""
+    w = np.where(used, -2, -1).astype(np.int64)
+    own = owner[:, 0] >= 0
+    w[own] = (owner[own, 0] << 16) | owner[own, 1]
+    return w.astype(np.int32)
+
+
+@pytest.mark.parametrize("per_thread", [1, 2, 4])
+def test_remap_batch_with_refused_entries(per_thread, monkeypatch):
+    """A 32 768-entry commit (every page of a pool to the host tier) in which 600
+    entries are refused -- 400 name another block's HBM page as their new location (a
+    double map), 200 name a block past its session's context -- at 1, 2 and 4 entries
+    per thread.  A refused entry changes nothing (its block stays on its page, its
+    reserved slot stays reserved) and every other entry is committed: tables, owner
+    words and allocation counts equal the oracle's after it commits the accepted
+    entries alone, and the allocation bitmaps agree with it on the next reservations."""
+    import torch
+    from oracle.pool import OraclePool
+    from paper_2606_22983_gb300 import lv
+    from paper_2606_22983_gb300.pool import KVPool
+    monkeypatch.setenv("LV_REMAP_ENTRIES_PER_THREAD", str(per_thread))
+    rng = np.random.default_rng(per_thread)
+    S, B = 64, 512
+    N = S * B
+    pool = KVPool(layers=1, kv_heads=1, head_dim=8, max_sessions=S, max_blocks=B, hbm_pages=N,
+                  hbm_budget_pages=N, host_pages=N)
+    om = OraclePool(1, 1, 8, 16, 2, S, B, N, N, N, with_bytes=False)
+    try:
+        placement = rng.permutation(N).astype(np.int32).reshape(S, B)
+        ctx = np.full(S, B * 16, np.int32)
+        ctx[-1] = (B - 8) * 16          # the last session's last 8 blocks lie past its context
+        placement[-1, B - 8:] = -1
+        pool.import_placement(placement, ctx)
+        om.import_placement(placement, ctx)
+        victims, nv = pool.select(0, lv.LV_ALL, 0)
+        v = victims.cpu().numpy().astype(np.int64)
+        slots, commit = pool.swap_out(victims, nv)
+        assert np.array_equal(slots.cpu().numpy(), om.swap_out(v[:, 0], v[:, 1], v[:, 2]))
+        reserved = commit.cpu().numpy().copy()
+        e = reserved.copy()
+        bad = rng.choice(nv, 600, replace=False)
+        owned, past = bad[:400], bad[400:]
+        good = np.setdiff1d(np.arange(nv), bad)
+        e[owned, 2] = v[rng.choice(good, owned.size), 2]
+        e[past, 0] = S - 1
+        e[past, 1] = B - 1 - rng.integers(0, 8, past.size)
+        pool.remap(torch.from_numpy(e).to(pool.device), nv)
+        assert pool.sync(raise_on_error=False) in (lv.LV_ERR_DOUBLE_MAP, lv.LV_ERR_BOUNDS)
+        pool.clear_error()
+        om.remap(e[good, 0], e[good, 1], e[good, 2])
+        t, oh, oo = pool.tables()
+        assert np.array_equal(t, om.tables.astype(np.int32))
+        assert np.array_equal(oh, _owner_words(om.owner_hbm, om.hbm_used))
+        assert np.array_equal(oo, _owner_words(om.owner_host, om.host_used))
+        st = pool.stats()
+        assert st["hbm_allocated"] == int(om.hbm_used.sum()) == 600
+        assert st["host_allocated"] == int(om.host_used.sum()) == nv
+        # the refused entries' slots are still reservations: releasing them works
+        refused_slots = reserved[bad, 2]
+        pool.cancel(torch.from_numpy(refused_slots.astype(np.int32)).to(pool.device), bad.size)
+        assert pool.sync(raise_on_error=False) == 0
+        om.cancel(refused_slots)
+        # and the next reservations take the same lowest free slots as the oracle's
+        victims2, n2 = pool.select(0, 50, 0)
+        v2 = victims2.cpu().numpy().astype(np.int64)
+        slots2, _ = pool.swap_out(victims2, n2)
+        assert np.array_equal(slots2.cpu().numpy(), om.swap_out(v2[:, 0], v2[:, 1], v2[:, 2]))
+        assert pool.sync(raise_on_error=False) == 0
+        assert pool.stats()["host_allocated"] == int(om.host_used.sum())
+    finally:
+        pool.close()
+
+
 def test_degenerate_sizes_and_host_pointer_arguments():
     import torch
     from paper_2606_22983_gb300 import lv

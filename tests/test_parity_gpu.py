@@ -95,7 +95,9 @@ def _sampled_full_size(wl, driver, mode, n_sample=48, rank_on="turns", record=Tr
         writer.write_initial(wl)
         gm = KVManager(pool, perms=wl.perms, rank_on=rank_on if record else "none", driver=driver,
                        mode=mode, order_fn=scatter_order, on_append=writer.write_appended,
-                       record=record, async_copy=async_copy)
+                       record=record, async_copy=async_copy,
+                       # unrecorded runs take the script's load keys from the device
+                       script=None if record else wl)
         touched = []
         for i in range(wl.n_events):
             ro, rg = om.step(i), gm.step(wl.event(i), i)
