@@ -666,6 +666,20 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
     if (n >= 1 && n <= pool->num_sms * 16) pool->exchange_ctas = n;
   }
 
+  // the exchange copy: 16-byte SM loads and stores by default; LV_EXCHANGE_KERNEL=tma
+  // moves it with TMA bulk copies through LV_EXCHANGE_STAGES (default 4) stages of 2P
+  // bytes per CTA, where two stages fit in a CTA's shared memory
+  d.xstages = 0;
+  if (const char* env = std::getenv("LV_EXCHANGE_KERNEL")) {
+    if (std::strcmp(env, "tma") == 0) {
+      int st = 4;
+      if (const char* e2 = std::getenv("LV_EXCHANGE_STAGES")) st = std::atoi(e2);
+      const int lim = lv::exchange_stage_limit(d.P);
+      if (st > lim) st = lim;
+      d.xstages = st >= 2 ? st : 0;
+    }
+  }
+  if (lv::configure_exchange_tma(d) != cudaSuccess) return fail(LV_ERR_CUDA);
   if (const char* env = std::getenv("LV_STAGE_STAGES")) {   // TMA pack/unpack stages per CTA
     const int st = std::atoi(env);
     if (st >= 2 && st <= 16) d.stages = st;

@@ -57,6 +57,7 @@ struct DevPool {
   int32_t policy;         // LV_POLICY_NEXT_USE / LV_POLICY_LRU
   int32_t incl;           // 1: LV_TIERS_INCLUSIVE
   int32_t stages;         // shared-memory stages of the TMA pack/unpack kernel (0: from P)
+  int32_t xstages;        // stages of the TMA exchange copy (0: the 16-byte LSU copy kernel)
   uint8_t* const* kv;     // [J] device pointers, sub-page j of page p at kv[j] + p*P
   uint8_t* host;          // device view of the host pool [host_pages][J][P]
   lv_session_state* sess; // [S]
@@ -210,6 +211,10 @@ cudaError_t launch_stage(const DevPool& p, bool pack, const int4* tasks, int64_t
 cudaError_t launch_tasks_pages(const DevPool& p, const int32_t* pages, int64_t n, bool pack,
                                int4* tasks, cudaStream_t s);
 cudaError_t configure_stage_kernels(const DevPool& p);
+// The largest number of exchange-copy TMA stages (2P bytes each) for sub-pages of P
+// bytes (0 when two do not fit in a CTA's shared memory), and the kernel's set-up.
+int exchange_stage_limit(long long P);
+cudaError_t configure_exchange_tma(const DevPool& p);
 cudaError_t launch_selftest_wait(const DevPool& p, long long limit_ns, cudaStream_t s);
 // lv_sched.cu
 // scratch: device memory of 32 * LV_SCHED_MAX_REQUESTS bytes (keys and costs)

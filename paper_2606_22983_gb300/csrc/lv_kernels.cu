@@ -1142,6 +1142,102 @@ k_stage_tasks(DevPool p, const int4* __restrict__ tasks, long long t_begin, long
   bulk_wait_all();
 }
 
+// The exchange's copies with TMA bulk copies instead of the SMs' loads and stores:
+// one thread per CTA moves units u = (task, sub-page j) through `stages`
+// shared-memory stages of 2P bytes.  A unit's out half (old HBM page -> its new host
+// slot) and in half (host slot -> its new HBM page) are loaded into one stage
+// together and stored from it once both have arrived, so a paired task's page is
+// read before it is overwritten.  Units come from the shared cursor (zeroed by the
+// plan) kXBatch at a time; a CTA refills the stage of unit k-1 while unit k's stores
+// still run.  The CTA issues a few instructions per 2P bytes, so its SM stays free
+// for other work; every barrier wait is bounded (LV_ERR_TIMEOUT).
+constexpr int kXStageMax = 8;
+constexpr int kXBatch = 8;
+
+__global__ void __launch_bounds__(kStageThreads)
+k_exchange_copy_tma(DevPool p, const int4* __restrict__ tasks, const long long* __restrict__ n_tasks,
+                    long long* __restrict__ cursor) {
+  extern __shared__ __align__(128) unsigned char xmem[];
+  __shared__ __align__(8) uint64_t bars[kXStageMax];
+  pdl_entry();
+  if (threadIdx.x != 0) return;
+  const int stages = p.xstages;
+  const uint32_t P = (uint32_t)p.P;
+  const long long units = *n_tasks * p.J;
+  for (int s = 0; s < stages; ++s) mbar_init(&bars[s], 1);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  uint8_t* dout[kXStageMax];
+  uint8_t* din[kXStageMax];
+  bool pending[kXStageMax];
+  uint32_t phase[kXStageMax];
+  for (int s = 0; s < stages; ++s) {
+    dout[s] = din[s] = nullptr;
+    pending[s] = false;
+    phase[s] = 0;
+  }
+  long long ub = 0, ue = 0, taken = 0;
+  bool exhausted = false;
+  // takes the CTA's unit number k (its k-th, in order) into stage k % stages
+  auto take = [&](long long k) {
+    if (exhausted) return;
+    if (ub == ue) {
+      ub = (long long)atomicAdd(reinterpret_cast<unsigned long long*>(cursor), (unsigned long long)kXBatch);
+      ue = ub + kXBatch < units ? ub + kXBatch : units;
+      if (ub >= units) {
+        exhausted = true;
+        return;
+      }
+    }
+    const long long u = ub++;
+    const int s = (int)(k % stages);
+    const int4 t = tasks[u / p.J];
+    const int j = (int)(u % p.J);
+    unsigned char* so = xmem + (size_t)s * 2 * P;
+    dout[s] = t.x >= 0 ? p.host + ((size_t)t.y * p.J + j) * P : nullptr;
+    din[s] = t.z >= 0 ? p.kv[j] + (size_t)t.w * P : nullptr;
+    const uint32_t bytes = (t.x >= 0 ? P : 0u) + (t.z >= 0 ? P : 0u);
+    pending[s] = bytes > 0;
+    if (bytes) {
+      mbar_expect_tx(&bars[s], bytes);
+      if (t.x >= 0) bulk_load(so, p.kv[j] + (size_t)t.x * P, P, &bars[s]);
+      if (t.z >= 0) bulk_load(so + P, p.host + ((size_t)t.z * p.J + j) * P, P, &bars[s]);
+    }
+    taken = k + 1;
+  };
+  for (long long k = 0; k < stages; ++k) take(k);
+  bool failed = false;
+  for (long long k = 0; k < taken; ++k) {
+    const int s = (int)(k % stages);
+    bool stored = false;
+    if (pending[s]) {
+      if (!mbar_wait_bounded(&bars[s], phase[s], kWaitLimitNs)) {
+        failed = true;
+        break;
+      }
+      pending[s] = false;
+      phase[s] ^= 1u;
+      unsigned char* so = xmem + (size_t)s * 2 * P;
+      if (dout[s]) bulk_store(dout[s], so, P);
+      if (din[s]) bulk_store(din[s], so + P, P);
+      bulk_commit();
+      stored = true;
+    }
+    // refill the stage of unit k-1 once its stores have read it; unit k's may still run
+    if (k >= 1 && !exhausted) {
+      if (stored) bulk_wait_read_1();
+      else bulk_wait_read_all();
+      take(k - 1 + stages);
+    }
+  }
+  if (failed) {
+    set_error(p.ctl, LV_ERR_TIMEOUT, blockIdx.x);
+    // let every load still in flight land before the shared memory is released
+    for (int s = 0; s < stages; ++s)
+      if (pending[s]) mbar_wait_bounded(&bars[s], phase[s], kWaitLimitNs);
+  }
+  bulk_wait_all();
+}
+
 // The same moves with plain 16-byte loads and stores (256 threads per CTA).
 template <bool kPack>
 __global__ void __launch_bounds__(kCopyThreads)
@@ -1988,11 +2084,21 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
   }
   if (ev) cudaEventRecord(ev->start, cs);
   else if (off && off->started) cudaEventRecord(off->started, cs);
-  if (off || ev) {   // after an event wait or record: an ordinary launch
-    k_exchange_copy<<<blocks_for(units, 1, copy_ctas), kCopyThreads, 0, cs>>>(p, tasks, n_tasks, cursor);
+  const unsigned grid = blocks_for(units, 1, copy_ctas);
+  if (p.xstages > 0) {
+    const size_t smem = (size_t)p.xstages * 2 * p.P;
+    if (off || ev) {
+      k_exchange_copy_tma<<<grid, kStageThreads, smem, cs>>>(p, tasks, n_tasks, cursor);
+    } else {
+      le = launch_pdl(k_exchange_copy_tma, grid, kStageThreads, smem, cs, p, (const int4*)tasks,
+                      (const long long*)n_tasks, cursor);
+      if (le != cudaSuccess) return le;
+    }
+  } else if (off || ev) {   // after an event wait or record: an ordinary launch
+    k_exchange_copy<<<grid, kCopyThreads, 0, cs>>>(p, tasks, n_tasks, cursor);
   } else {
-    le = launch_pdl(k_exchange_copy, blocks_for(units, 1, copy_ctas), kCopyThreads, 0, cs, p,
-                    (const int4*)tasks, (const long long*)n_tasks, cursor);
+    le = launch_pdl(k_exchange_copy, grid, kCopyThreads, 0, cs, p, (const int4*)tasks,
+                    (const long long*)n_tasks, cursor);
     if (le != cudaSuccess) return le;
   }
   if (ev) cudaEventRecord(ev->end, cs);
@@ -2121,6 +2227,19 @@ cudaError_t configure_stage_kernels(const DevPool& p) {
   cudaError_t e = cudaFuncSetAttribute(k_stage_tasks<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   return cudaFuncSetAttribute(k_stage_tasks<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+}
+
+int exchange_stage_limit(long long P) {
+  const long long per = 2 * P;
+  long long n = (227ll * 1024) / per;
+  if (n > kXStageMax) n = kXStageMax;
+  return n >= 2 ? (int)n : 0;
+}
+
+cudaError_t configure_exchange_tma(const DevPool& p) {
+  if (p.xstages <= 0) return cudaSuccess;
+  return cudaFuncSetAttribute(k_exchange_copy_tma, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)((size_t)p.xstages * 2 * p.P));
 }
 
 cudaError_t launch_stage(const DevPool& p, bool pack, const int4* tasks, int64_t t_begin, int64_t t_end,

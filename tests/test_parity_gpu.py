@@ -36,6 +36,17 @@ def test_tiny_workload_address_tagged_bytes(driver, mode):
     assert om.counters == gm.counters and gm.counters["pages_out"] > 300
 
 
+@pytest.mark.parametrize("driver", ["device", "exchange"])
+def test_tiny_workload_tma_exchange_copy(driver, monkeypatch):
+    """The exchange's copies moved by TMA bulk copies (LV_EXCHANGE_KERNEL=tma) instead of
+    16-byte loads and stores: the tiny script with address-tagged contents, every
+    decision and full byte images after every 25 events."""
+    monkeypatch.setenv("LV_EXCHANGE_KERNEL", "tma")
+    wl = make_workload("tiny", 6)
+    om, gm = run_lockstep(wl, with_bytes=True, check_every=25, driver=driver, mode=0, tagged=True)
+    assert om.counters == gm.counters and gm.counters["pages_out"] > 300
+
+
 @pytest.mark.parametrize("driver,mode", [("device", 0), ("exchange", 0), ("exchange", 2),
                                          ("sequential", 0)])
 def test_hand_worked_turns(driver, mode):
@@ -141,6 +152,14 @@ def test_thinker_full_size_async_copies():
     round trip between turns (the next turn ranks and plans while the previous
     turn's pages still move): the end state and sampled bytes equal the oracle's."""
     _sampled_full_size(make_workload("thinker", 1, n_turns=30), "device", 0, record=False,
+                       async_copy=True)
+
+
+def test_thinker_full_size_tma_exchange_copy(monkeypatch):
+    """Thinker turns at full size with the TMA exchange copy and asynchronous copies
+    (nothing read back between turns): end state and sampled bytes equal the oracle's."""
+    monkeypatch.setenv("LV_EXCHANGE_KERNEL", "tma")
+    _sampled_full_size(make_workload("thinker", 2, n_turns=30), "device", 0, record=False,
                        async_copy=True)
 
 
