@@ -31,11 +31,13 @@
  * needs memory that cannot be had, and LV_ERR_CUDA when a CUDA runtime call
  * fails; the comments below name the other statuses.
  *
- * Pointers.  Array arguments may point to device memory or to host memory.  A
- * host input is copied to the device in stream order before use (pageable host
- * memory: before the call returns; page-locked host memory: the caller keeps
- * it unchanged until the stream reaches the call).  A host output is written
- * by a copy queued on the stream: read it after the stream has completed.
+ * Pointers.  Array arguments may point to device memory or to host memory.
+ * Mapped page-locked host memory (any page-locked allocation under unified
+ * addressing) is read and written by the kernels in place, over the host link;
+ * the caller keeps such an input unchanged until the stream reaches the call.
+ * A pageable host input is copied to the device before the call returns, and a
+ * pageable host output is written by a copy queued on the stream.  Read any host
+ * output after the stream has completed.
  * Calls that allocate from the same tier (swap-out: host slots; swap-in and
  * append: HBM pages) must be ordered with respect to each other.
  *

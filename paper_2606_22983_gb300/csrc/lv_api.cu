@@ -139,8 +139,23 @@ bool is_device_ptr(const void* p) {
   return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
 }
 
-// Per-call staging: host-pointer inputs are copied in, host-pointer (or absent)
-// outputs get stream-ordered device buffers that are copied back at the end.
+// The address the GPU uses for p: p itself for device or managed memory, the
+// device alias of mapped page-locked host memory, else nullptr (pageable memory).
+const void* gpu_view(const void* p) {
+  cudaPointerAttributes a{};
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return p;
+  if (a.type == cudaMemoryTypeHost) return a.devicePointer;
+  return nullptr;
+}
+
+// Per-call staging.  Device, managed and mapped page-locked host arguments are
+// used in place (the kernels read and write page-locked host memory over the host
+// link, in stream order); pageable host inputs are copied in, and pageable (or
+// absent) outputs get stream-ordered device buffers that are copied back at the end.
 class Staging {
  public:
   Staging(lv_pool* pool, cudaStream_t s) : pool_(pool), s_(s) {}
@@ -152,8 +167,8 @@ class Staging {
     *dev = nullptr;
     if (bytes == 0) return LV_OK;
     if (user == nullptr) return LV_ERR_INVALID;
-    if (is_device_ptr(user)) {
-      *dev = user;
+    if (const void* v = gpu_view(user)) {
+      *dev = v;
       return LV_OK;
     }
     void* t = nullptr;
@@ -168,9 +183,11 @@ class Staging {
   lv_status out(void* user, size_t bytes, void** dev, bool required) {
     *dev = nullptr;
     if (bytes == 0) return LV_OK;
-    if (user != nullptr && is_device_ptr(user)) {
-      *dev = user;
-      return LV_OK;
+    if (user != nullptr) {
+      if (const void* v = gpu_view(user)) {
+        *dev = const_cast<void*>(v);
+        return LV_OK;
+      }
     }
     if (user == nullptr && !required) return LV_OK;
     void* t = nullptr;

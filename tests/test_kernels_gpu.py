@@ -356,6 +356,18 @@ def test_degenerate_sizes_and_host_pointer_arguments():
         assert slots_d.cpu().tolist() == [0, 1]
         assert np.array_equal(commit_d.cpu().numpy(), commit_h)
         assert np.array_equal(pool.host[0], pool.kv[:, 7].cpu().numpy())
+        # page-locked host arguments are used in place: the commit's entries are read and
+        # a victim list is written over the host link, in stream order
+        commit_p = torch.from_numpy(commit_h).pin_memory()
+        pool.remap(commit_p, 2)
+        cnt_p = torch.full((1,), -7, dtype=torch.int64).pin_memory()
+        out_p = torch.full((4, 3), -7, dtype=torch.int32).pin_memory()
+        lv.lv_select_victims(pool.handle, 0, lv.LV_ALL, 0, out_p, 4, cnt_p, pool.stream)
+        assert pool.sync(raise_on_error=False) == 0
+        t, _, _ = pool.tables()
+        assert t[0, :3].tolist() == [5, -3, -2]
+        assert int(cnt_p[0]) == 1
+        assert out_p[0].tolist() == [0, 0, 5] and out_p[1].tolist() == [-7, -7, -7]
     finally:
         pool.close()
 
