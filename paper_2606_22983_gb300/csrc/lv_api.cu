@@ -1237,9 +1237,13 @@ lv_status lv_page_checksums(lv_pool* pool, const int32_t* pages, int64_t n, uint
     lv_status r;
     if ((r = st.in(pages, (size_t)n * 4, &pin)) != LV_OK) return r;
     if ((r = st.out(sums_out, (size_t)n * 8, &sdev, true)) != LV_OK) return r;
-    LV_TRY(cudaMemsetAsync(sdev, 0, (size_t)n * 8, s));
+    void* cdev = nullptr;   // the kernel's unit cursor
+    if ((r = st.out(nullptr, sizeof(unsigned long long), &cdev, true)) != LV_OK) return r;
+    LV_TRY(cudaMemsetAsync(cdev, 0, sizeof(unsigned long long), s));
+    LV_TRY(lv::launch_zero(sdev, n * 8, s));
     LV_TRY(lv::launch_checksums(pool->d, static_cast<const int32_t*>(pin), n,
-                                static_cast<unsigned long long*>(sdev), s, pool->num_sms * 8));
+                                static_cast<unsigned long long*>(sdev),
+                                static_cast<unsigned long long*>(cdev), s, pool->num_sms * 8));
     return st.finish();
   } catch (const std::bad_alloc&) {
     return LV_ERR_OOM;
@@ -1268,7 +1272,7 @@ lv_status lv_schedule(lv_pool* pool, const lv_sched_params* q, const lv_request*
     if ((r = st.out(order_out, (size_t)n * 4, &odev, true)) != LV_OK) return r;
     if ((r = st.out(batch_out, 4, &bdev, true)) != LV_OK) return r;
     if (n == 0) {
-      LV_TRY(cudaMemsetAsync(bdev, 0, 4, s));
+      LV_TRY(lv::launch_zero(bdev, 4, s));
       return st.finish();
     }
     LV_TRY(lv::launch_schedule(*q, static_cast<const lv_request*>(rin), n, static_cast<int32_t*>(odev),

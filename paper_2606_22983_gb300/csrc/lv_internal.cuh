@@ -133,6 +133,8 @@ cudaError_t launch_exchange(const DevPool& p, const lv_victim* v, int64_t n_out,
 cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, int32_t epoch,
                          cudaStream_t s, int num_sms, int per_thread);
 cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cudaStream_t s);
+// Zeroes bytes (a multiple of 4) at q: device memory or mapped page-locked host memory.
+cudaError_t launch_zero(void* q, int64_t bytes, cudaStream_t s);
 cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32_t* pages,
                           int32_t* count, cudaStream_t s, const long long* gate = nullptr,
                           const long long* sid_dev = nullptr);
@@ -191,7 +193,8 @@ cudaError_t launch_turn(const DevPool& p, const ResidentScratch& rs, int32_t sid
 cudaError_t launch_counts(const DevPool& p, int32_t* hbm, int32_t* host, cudaStream_t s);
 // sums[i] = position-weighted 64-bit sum of page pages[i] (sums zeroed by the caller)
 cudaError_t launch_checksums(const DevPool& p, const int32_t* pages, int64_t n,
-                             unsigned long long* sums, cudaStream_t s, int ctas);
+                             unsigned long long* sums, unsigned long long* cursor, cudaStream_t s,
+                             int ctas);
 cudaError_t launch_blocks(const DevPool& p, int32_t sid, int32_t where, int32_t* out,
                           long long* count, cudaStream_t s);
 cudaError_t launch_check_budget(const DevPool& p, cudaStream_t s);

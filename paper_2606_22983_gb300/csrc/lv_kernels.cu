@@ -895,8 +895,10 @@ k_exchange_copy(DevPool p, const int4* __restrict__ tasks, const long long* __re
   if (threadIdx.x == 0) next = (long long)atomicAdd(reinterpret_cast<unsigned long long*>(cursor), 1ull);
   __syncthreads();
   for (long long u = next; u < units; u = next) {
-    __syncthreads();   // every thread holds u before `next` is replaced
-    if (threadIdx.x == 0) next = (long long)atomicAdd(reinterpret_cast<unsigned long long*>(cursor), 1ull);
+    // thread 0 fetches the next unit now and publishes it after the copy, so that its
+    // warp does not wait for the atomic's result meanwhile
+    unsigned long long fetched = 0;
+    if (threadIdx.x == 0) fetched = atomicAdd(reinterpret_cast<unsigned long long*>(cursor), 1ull);
     const int4 t = tasks[u / p.J];
     const int j = (int)(u % p.J);
     const bool has_out = t.x >= 0, has_in = t.z >= 0;
@@ -923,7 +925,9 @@ k_exchange_copy(DevPool p, const int4* __restrict__ tasks, const long long* __re
         }
       }
     }
-    __syncthreads();   // thread 0's fetch of the next unit is visible
+    __syncthreads();   // every thread holds u before `next` is replaced
+    if (threadIdx.x == 0) next = (long long)fetched;
+    __syncthreads();
   }
 }
 
@@ -1868,53 +1872,70 @@ k_pick_scan(DevPool p, const int32_t* __restrict__ cand, int32_t* __restrict__ h
 // ------------------------------------------------------------- checksums
 constexpr int kSumThreads = 256;
 constexpr int kSumUnroll = 4;
+constexpr int kSumBatch = 4;      // sub-pages taken from the cursor at a time
 
 // Unit u = (page i, sub-page j); the sub-page's words are q0 + k (q0 = j*P/8).
 // Each thread keeps kSumUnroll 16-byte loads in flight; the per-unit partial sum
 // goes to sums[i] with one atomic add (addition mod 2^64 is order-free).
 __global__ void __launch_bounds__(kSumThreads)
-k_checksum(DevPool p, const int32_t* __restrict__ pages, long long n, unsigned long long* __restrict__ sums) {
+k_checksum(DevPool p, const int32_t* __restrict__ pages, long long n, unsigned long long* __restrict__ sums,
+           unsigned long long* __restrict__ cursor) {
   __shared__ unsigned long long warp_part[kSumThreads / 32];
+  __shared__ long long s_next;
   const long long units = n * p.J;
   const int nvec = (int)(p.P >> 4);                   // 16-byte vectors per sub-page
-  for (long long u = blockIdx.x; u < units; u += gridDim.x) {
-    const long long i = u / p.J;
-    const int j = (int)(u % p.J);
-    const int32_t pg = pages[i];
-    const bool ok = pg >= 0 && pg < p.hbm_pages;
-    unsigned long long acc = 0;
-    if (ok) {
-      const ulonglong2* src = reinterpret_cast<const ulonglong2*>(p.kv[j] + (size_t)pg * p.P);
-      const unsigned long long q0 = (unsigned long long)j * (unsigned long long)(p.P >> 3);
-      for (int base = threadIdx.x; base < nvec; base += kSumThreads * kSumUnroll) {
-        ulonglong2 r[kSumUnroll];
+  // units come from a shared cursor, kSumBatch at a time, the next batch fetched while
+  // the current one is read: a CTA that starts late (its SM held by other work) takes
+  // fewer units instead of holding up the end of the call
+  // (thread 0 keeps the fetched index in a register and publishes it only at the end
+  // of the batch, so that its warp does not wait for the atomic's result meanwhile)
+  if (threadIdx.x == 0) s_next = (long long)atomicAdd(cursor, (unsigned long long)kSumBatch);
+  __syncthreads();
+  for (long long b = s_next; b < units; b = s_next) {
+    unsigned long long fetched = 0;
+    if (threadIdx.x == 0) fetched = atomicAdd(cursor, (unsigned long long)kSumBatch);
+    const long long b_end = b + kSumBatch < units ? b + kSumBatch : units;
+    for (long long u = b; u < b_end; ++u) {
+      const long long i = u / p.J;
+      const int j = (int)(u % p.J);
+      const int32_t pg = pages[i];
+      const bool ok = pg >= 0 && pg < p.hbm_pages;
+      unsigned long long acc = 0;
+      if (ok) {
+        const ulonglong2* src = reinterpret_cast<const ulonglong2*>(p.kv[j] + (size_t)pg * p.P);
+        const unsigned long long q0 = (unsigned long long)j * (unsigned long long)(p.P >> 3);
+        for (int base = threadIdx.x; base < nvec; base += kSumThreads * kSumUnroll) {
+          ulonglong2 r[kSumUnroll];
 #pragma unroll
-        for (int k = 0; k < kSumUnroll; ++k) {
-          const int v = base + k * kSumThreads;
-          if (v < nvec) r[k] = src[v];
-        }
+          for (int k = 0; k < kSumUnroll; ++k) {
+            const int v = base + k * kSumThreads;
+            if (v < nvec) r[k] = src[v];
+          }
 #pragma unroll
-        for (int k = 0; k < kSumUnroll; ++k) {
-          const int v = base + k * kSumThreads;
-          if (v < nvec) {
-            const unsigned long long q = q0 + 2ull * (unsigned long long)v;   // word index of r.x
-            acc += r[k].x * (2ull * q + 1ull) + r[k].y * (2ull * q + 3ull);
+          for (int k = 0; k < kSumUnroll; ++k) {
+            const int v = base + k * kSumThreads;
+            if (v < nvec) {
+              const unsigned long long q = q0 + 2ull * (unsigned long long)v;   // word index of r.x
+              acc += r[k].x * (2ull * q + 1ull) + r[k].y * (2ull * q + 3ull);
+            }
           }
         }
+      } else if (j == 0 && threadIdx.x == 0) {
+        set_error(p.ctl, LV_ERR_BOUNDS, i);
       }
-    } else if (j == 0 && threadIdx.x == 0) {
-      set_error(p.ctl, LV_ERR_BOUNDS, i);
-    }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) acc += __shfl_down_sync(0xffffffffu, acc, o);
-    if ((threadIdx.x & 31) == 0) warp_part[threadIdx.x >> 5] = acc;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      unsigned long long t = 0;
+      for (int o = 16; o > 0; o >>= 1) acc += __shfl_down_sync(0xffffffffu, acc, o);
+      if ((threadIdx.x & 31) == 0) warp_part[threadIdx.x >> 5] = acc;
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        unsigned long long t = 0;
 #pragma unroll
-      for (int w = 0; w < kSumThreads / 32; ++w) t += warp_part[w];
-      if (ok) atomicAdd(&sums[i], t);
+        for (int w = 0; w < kSumThreads / 32; ++w) t += warp_part[w];
+        if (ok) atomicAdd(&sums[i], t);
+      }
+      __syncthreads();
     }
+    if (threadIdx.x == 0) s_next = (long long)fetched;   // every thread has read b
     __syncthreads();
   }
 }
@@ -2187,10 +2208,26 @@ cudaError_t launch_turn(const DevPool& p, const ResidentScratch& rs, int32_t sid
   return cudaGetLastError();
 }
 
+// Zeroes `words` 32-bit words at p, which may be device memory or the device alias of
+// mapped page-locked host memory (a kernel, so that either works).
+__global__ void k_zero(uint32_t* __restrict__ q, long long words) {
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < words;
+       i += (long long)gridDim.x * blockDim.x)
+    q[i] = 0u;
+}
+
+cudaError_t launch_zero(void* q, int64_t bytes, cudaStream_t s) {
+  const long long words = (long long)(bytes / 4);
+  if (words <= 0) return cudaSuccess;
+  k_zero<<<blocks_for(words, 256, 1024), 256, 0, s>>>(static_cast<uint32_t*>(q), words);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_checksums(const DevPool& p, const int32_t* pages, int64_t n,
-                             unsigned long long* sums, cudaStream_t s, int ctas) {
+                             unsigned long long* sums, unsigned long long* cursor, cudaStream_t s,
+                             int ctas) {
   if (n <= 0) return cudaSuccess;
-  k_checksum<<<blocks_for(n * p.J, 1, ctas), kSumThreads, 0, s>>>(p, pages, n, sums);
+  k_checksum<<<blocks_for(n * p.J, kSumBatch, ctas), kSumThreads, 0, s>>>(p, pages, n, sums, cursor);
   return cudaGetLastError();
 }
 
