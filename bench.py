@@ -363,10 +363,12 @@ class ChecksumConsumer:
     """Stands in for the engine's attention reads of resident KV: lv_page_checksums
     over n resident pages (HBM-bound, every byte read once) issued on its own stream
     through a second liblv pool over the same KV arrays, so that its reads never wait
-    for the first pool's copies.  ``top_up`` keeps a few calls queued, so it runs
-    without gaps while the other work is issued."""
+    for the first pool's copies.  A call reads 512 pages (0.8 GB, about 0.11 ms alone),
+    the length of a serving step's larger kernels, so that its SMs are handed back as
+    often as a serving engine's would be; ``top_up`` keeps ``depth`` calls queued, so it
+    runs without gaps while the other work is issued."""
 
-    def __init__(self, torch, pool, n_pages=4096, seed=0, depth=3):
+    def __init__(self, torch, pool, n_pages=512, seed=0, depth=24):
         from paper_2606_22983_gb300.pool import KVPool
         self.torch = torch
         self.stream = torch.cuda.Stream(device=pool.device)
@@ -385,6 +387,11 @@ class ChecksumConsumer:
         self.ends = []
         self.calls = 0
         self.call_ms = 1.0
+
+    def describe(self):
+        return (f"lv_page_checksums over {self.n} resident pages ({self.bytes_per_call / 1e9:.1f} GB "
+                f"read per call, {self.depth} calls kept queued), its own stream and pool over the "
+                "same KV arrays")
 
     def issue(self):
         from paper_2606_22983_gb300 import lv
@@ -482,8 +489,7 @@ def _overlap_measure(torch, pool, wl, first_turn, n_turns):
     from paper_2606_22983_gb300.manager import KVManager
     cons = ChecksumConsumer(torch, pool)
     alone = cons.alone_gbs()
-    out = {"consumer": "lv_page_checksums over 4096 resident pages (6.4 GB read per call), "
-                       "its own stream and pool over the same KV arrays",
+    out = {"consumer": cons.describe(),
            "consumer_alone_gbs": round(alone, 1), "consumer_alone_hbm_frac": round(alone / HBM_PEAK, 3)}
     page_bytes = pool.J * pool.P
     ev = lambda: torch.cuda.Event(enable_timing=True)
@@ -709,7 +715,8 @@ def five_workloads(torch, seed, consumer_on="mixed"):
                                                      before_event=cons.top_up)
                     got = done()
                 cons.close()
-                r["with_consumer"] = {"consumer_alone_gbs": round(alone, 1),
+                r["with_consumer"] = {"consumer": cons.describe(),
+                                      "consumer_alone_gbs": round(alone, 1),
                                       "consumer_with_events_gbs": round(got, 1),
                                       "consumer_frac_kept": round(got / alone, 3),
                                       "turn_ms": quantiles(turn2),
