@@ -89,6 +89,9 @@ class KVManager:
         self.perms_dev = None
         if perms is not None and len(perms):
             self.perms_dev = torch.from_numpy(np.ascontiguousarray(perms, dtype=np.int32)).to(pool.device)
+            # a row's device address, without building a tensor view per turn
+            self._perm_row = (self.perms_dev.data_ptr(), self.perms_dev.shape[1] * 4,
+                              int(self.perms_dev.shape[1]))
         self.counters = dict(victims=0, pages_out=0, pages_in=0, preloads=0,
                              preload_skipped=0, turns=0, sync_loads=0, appended=0)
         self.bytes_moved = 0
@@ -109,7 +112,8 @@ class KVManager:
             return
         rows = np.stack([self._load_keys(k) for k in order_keys])
         self._keys_dev = torch.from_numpy(rows.view(np.int64)).to(self.pool.device)
-        self._keys_row = {k: i for i, k in enumerate(order_keys)}
+        base, stride = self._keys_dev.data_ptr(), rows.shape[1] * 8
+        self._keys_row = {k: base + i * stride for i, k in enumerate(order_keys)}
 
     # ------------------------------------------------------------- queries
     def free_budget(self) -> int:
@@ -180,12 +184,15 @@ class KVManager:
         """One lv_turn: (pick,) turn begin, make resident, turn end -- no host round trip
         unless the decisions are recorded.  Returns the session id (-1 when not read back)."""
         pool = self.pool
-        cand = self.perms_dev[row] if sid < 0 else None
+        cand, n_cand = None, 0
+        if sid < 0:
+            base, stride, n_cand = self._perm_row
+            cand = base + row * stride
         rec_bufs = self.record or (self.on_append is not None and append_tokens > 0)
         outs = (pool.victims, pool.slots, pool.blks, pool.pages, pool.app) if self.record else (None,) * 5
         lv.lv_turn(pool.handle, sid, now_us, append_tokens, reply_us, reply_units, outs, self.res_h,
-                   cand, int(cand.numel()) if cand is not None else 0, pool.stream,
-                   lv.LV_RESIDENT_ASYNC_COPY if self.async_copy else 0, load_keys)
+                   cand, n_cand, pool.stream, lv.LV_RESIDENT_ASYNC_COPY if self.async_copy else 0,
+                   load_keys)
         pool.launches += 1 if load_keys is not None else 0
         pool.launches += 5 + pool.rank_extra + (1 if sid < 0 else 0) + (2 if append_tokens else 0)
         if not rec_bufs:
@@ -434,8 +441,9 @@ class KVManager:
             self.counters["turns"] += 1
         elif kind == EV_TURN_SCATTER and self.driver == "device" and self.order_fn is not None:
             # the reload order is the script's scatter order, given as per-block keys
-            row = self._keys_row.get(a)
-            keys = self._keys_dev[row] if row is not None else self._load_keys(a)
+            keys = self._keys_row.get(a)        # the row's device address, if staged
+            if keys is None:
+                keys = self._load_keys(a)
             sid = self._device_turn(-1, d, t, 0, b, c, rec, load_keys=keys)
             self.counters["turns"] += 1
         elif kind in (EV_TURN, EV_TURN_ANY, EV_TURN_SCATTER):
