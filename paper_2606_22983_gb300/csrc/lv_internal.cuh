@@ -135,9 +135,12 @@ cudaError_t launch_remap(const DevPool& p, const lv_remap_entry* e, int64_t n, i
 cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cudaStream_t s);
 // Zeroes bytes (a multiple of 4) at q: device memory or mapped page-locked host memory.
 cudaError_t launch_zero(void* q, int64_t bytes, cudaStream_t s);
+// fin (with R, the step's control words): a device-driven step's end, done by the
+// append kernel after the growth
 cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32_t* pages,
                           int32_t* count, cudaStream_t s, const long long* gate = nullptr,
-                          const long long* sid_dev = nullptr);
+                          const long long* sid_dev = nullptr, const struct StepFinish* fin = nullptr,
+                          const long long* R = nullptr);
 
 // Device buffers of lv_make_resident, owned by the pool.
 struct ResidentScratch {

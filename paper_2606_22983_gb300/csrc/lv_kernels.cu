@@ -1595,11 +1595,14 @@ __global__ void k_cancel(DevPool p, const int32_t* __restrict__ locs, long long 
 __global__ void __launch_bounds__(kAllocThreads)
 k_append(DevPool p, int32_t sid, int32_t n_tokens, int32_t* __restrict__ pages,
          int32_t* __restrict__ count, const long long* __restrict__ gate,
-         const long long* __restrict__ sid_dev) {
+         const long long* __restrict__ sid_dev, StepFinish fin, const long long* __restrict__ R) {
   pdl_entry();
   __shared__ long long m_s, nb_s, ctx_s;
   if (gate && *gate != 0) {   // an earlier step of lv_make_resident did not complete
-    if (threadIdx.x == 0 && count) *count = 0;
+    if (threadIdx.x == 0) {
+      if (count) *count = 0;
+      if (fin.on) finish_step(p, fin, R);
+    }
     return;
   }
   if (sid_dev) sid = (int32_t)*sid_dev;
@@ -1635,7 +1638,10 @@ k_append(DevPool p, int32_t sid, int32_t n_tokens, int32_t* __restrict__ pages,
   __syncthreads();
   const long long m = m_s;
   if (m < 0) {
-    if (threadIdx.x == 0 && count) *count = 0;
+    if (threadIdx.x == 0) {
+      if (count) *count = 0;
+      if (fin.on) finish_step(p, fin, R);
+    }
     return;
   }
   if (m > 0) block_alloc_lowest<kAllocThreads>(p.bits_hbm, p.hbm_pages, m, pages);
@@ -1664,6 +1670,7 @@ k_append(DevPool p, int32_t sid, int32_t n_tokens, int32_t* __restrict__ pages,
     p.sess[sid].ctx_tokens = (int32_t)ctx_s;
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_APPENDED]), (unsigned long long)m);
     if (count) *count = (int32_t)m;
+    if (fin.on) finish_step(p, fin, R);   // a device-driven step's end, after its growth
   }
 }
 
@@ -1828,11 +1835,6 @@ __device__ void finish_step(const DevPool& p, const StepFinish& f, const long lo
     r.sid = sid;
     *f.out = r;
   }
-}
-
-__global__ void k_resident_finish(DevPool p, StepFinish f, const long long* __restrict__ R) {
-  pdl_entry();
-  if (threadIdx.x == 0) finish_step(p, f, R);
 }
 
 // ----------------------------------------------------------------- evict
@@ -2160,11 +2162,9 @@ cudaError_t launch_make_resident(const DevPool& p, const ResidentScratch& rs, in
                       ev, sid_dev, off, preload ? GATE_PRELOAD : GATE_RESIDENT, nullptr,
                       append_tokens > 0 ? nullptr : &fin);
   if (e != cudaSuccess) return e;
-  if (append_tokens > 0) {
+  if (append_tokens > 0) {   // the growth, then the step's end in the same kernel
     e = launch_append(p, sid, append_tokens, rs.append, reinterpret_cast<int32_t*>(R + R_APPENDED), s,
-                      R + R_GATE, sid_dev);
-    if (e != cudaSuccess) return e;
-    e = launch_pdl(k_resident_finish, 1, 32, 0, s, p, fin, (const long long*)R);
+                      R + R_GATE, sid_dev, &fin, R);
     if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();
@@ -2352,9 +2352,10 @@ cudaError_t launch_cancel(const DevPool& p, const int32_t* locs, int64_t n, cuda
 
 cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32_t* pages,
                           int32_t* count, cudaStream_t s, const long long* gate,
-                          const long long* sid_dev) {
+                          const long long* sid_dev, const StepFinish* fin, const long long* R) {
+  const StepFinish none{};
   const cudaError_t e = launch_pdl(k_append, 1, kAllocThreads, 0, s, p, sid, n_tokens, pages, count,
-                                   gate, sid_dev);
+                                   gate, sid_dev, fin ? *fin : none, R);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

@@ -139,8 +139,8 @@ class KVManager:
             self.timer.start("resident")
         lv.lv_make_resident(pool.handle, sid, now_us, append_tokens, flags, -1, *outs,
                             self.res_h, pool.stream)
-        # prepare, census, emit, plan (with the step's end), copy; append and end after it
-        pool.launches += 5 + pool.rank_extra + (2 if append_tokens else 0)
+        # prepare, census, emit, plan (with the step's end), copy; or the append with the end
+        pool.launches += 5 + pool.rank_extra + (1 if append_tokens else 0)
         if self.timer:
             self.timer.stop("resident", None)
         if not rec_bufs:
@@ -194,7 +194,7 @@ class KVManager:
                    cand, n_cand, pool.stream, lv.LV_RESIDENT_ASYNC_COPY if self.async_copy else 0,
                    load_keys)
         pool.launches += 1 if load_keys is not None else 0
-        pool.launches += 5 + pool.rank_extra + (1 if sid < 0 else 0) + (2 if append_tokens else 0)
+        pool.launches += 5 + pool.rank_extra + (1 if sid < 0 else 0) + (1 if append_tokens else 0)
         if not rec_bufs:
             return sid
         pool.sync(raise_on_error=False)
