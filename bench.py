@@ -223,9 +223,10 @@ def ours(args, torch):
                           "gbs": nb / 1e9 / (t["total_ms"] / 1e3)}
 
     # e2e: K further turns through the public API from host buffers, timed on the host
-    # clock: every step copies its event batch from page-locked host memory to the
-    # device and reads the turn's result (lv_resident_result) back into page-locked
-    # host memory, in stream order; the results are checked after the final join
+    # clock: every step moves its event batch from page-locked host memory to the device
+    # and the turn's result (lv_resident_result) back into page-locked host memory, in
+    # stream order (the library's kernels read and write page-locked arguments in place,
+    # over the host link); the results are checked after the final join
     gm.record = False
     ev_h = torch.empty((K, S * lv.EVENT_DTYPE.itemsize), dtype=torch.uint8).pin_memory()
     for j, i in enumerate(range(W + K, W + 2 * K)):
