@@ -93,6 +93,20 @@ struct lv_pool {
   void* host_base = nullptr;       // host-visible address of the host pool
   std::vector<void*> dev_allocs;
   cudaMemPool_t mp = nullptr;      // stream-ordered staging memory
+  // device-driven steps whose kernels all run on the caller's stream go out as one
+  // CUDA graph launch: one instantiated graph per shape of the launch sequence, its
+  // kernel nodes' arguments replaced for every step
+  struct StepGraph {
+    std::vector<const void*> funcs;
+    std::vector<dim3> grids, blocks;
+    std::vector<size_t> smems;
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    std::vector<cudaGraphNode_t> nodes;   // kernel nodes in launch order
+  };
+  std::vector<StepGraph> step_graphs;
+  bool step_graphs_on = true;
+  cudaStream_t s_capture = nullptr;
 };
 
 namespace {
@@ -489,6 +503,12 @@ cudaError_t next_scratch(lv_pool* pool, cudaStream_t s, bool async, const lv::Re
 }
 
 void free_pool(lv_pool* pool) {
+  for (auto& g : pool->step_graphs) {
+    if (g.exec) cudaGraphExecDestroy(g.exec);
+    if (g.graph) cudaGraphDestroy(g.graph);
+  }
+  pool->step_graphs.clear();
+  if (pool->s_capture) cudaStreamDestroy(pool->s_capture);
   if (pool->s_unpack) cudaStreamSynchronize(pool->s_unpack);
   if (pool->s_unpack) cudaStreamDestroy(pool->s_unpack);
   for (cudaEvent_t e : {pool->ev_st_d2h, pool->ev_st_h2d, pool->ev_st_unpack, pool->ev_st_packed,
@@ -731,6 +751,9 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
     if (per >= 1 && per <= 4) pool->stage_ctas = pool->num_sms * per;
   }
   if (const char* env = std::getenv("LV_STAGE_KERNEL")) pool->stage_tma = std::strcmp(env, "lsu") != 0;
+  // device-driven steps on the caller's stream as graph launches (LV_STEP_GRAPHS=0: one
+  // kernel launch at a time)
+  if (const char* env = std::getenv("LV_STEP_GRAPHS")) pool->step_graphs_on = std::strcmp(env, "0") != 0;
   if (const char* env = std::getenv("LV_REMAP_ENTRIES_PER_THREAD")) {   // 1, 2 or 4
     const int e = std::atoi(env);
     if (e == 1 || e == 2 || e == 4) pool->remap_per_thread = e;
@@ -753,6 +776,112 @@ lv_status create_impl(const lv_pool_desc* desc, cudaStream_t s, lv_pool** out) {
   if (cudaStreamSynchronize(s) != cudaSuccess) return fail(LV_ERR_CUDA);
   *out = pool;
   return LV_OK;
+}
+
+// The kernel nodes of a captured launch chain, in launch order (each node depends on
+// the one before it); false unless the graph is exactly such a chain of n nodes.
+bool chain_nodes(cudaGraph_t graph, size_t n, std::vector<cudaGraphNode_t>* order) {
+  size_t count = 0;
+  if (cudaGraphGetNodes(graph, nullptr, &count) != cudaSuccess || count != n) return false;
+  std::vector<cudaGraphNode_t> nodes(count);
+  if (cudaGraphGetNodes(graph, nodes.data(), &count) != cudaSuccess) return false;
+  std::vector<cudaGraphNode_t> prev(count, nullptr);
+  cudaGraphNode_t root = nullptr;
+  for (size_t i = 0; i < count; ++i) {
+    // with room for two, so that a node with more than one dependency is seen; the edge
+    // data is asked for too (programmatic edges are not default edges)
+    cudaGraphNode_t deps[2] = {nullptr, nullptr};
+    cudaGraphEdgeData edge[2] = {};
+    size_t nd = 2;
+    if (cudaGraphNodeGetDependencies(nodes[i], deps, edge, &nd) != cudaSuccess || nd > 1) return false;
+    if (nd == 1) {
+      prev[i] = deps[0];
+    } else if (root) {
+      return false;
+    } else {
+      root = nodes[i];
+    }
+  }
+  order->clear();
+  for (cudaGraphNode_t cur = root; cur && order->size() < count;) {
+    order->push_back(cur);
+    cudaGraphNode_t next = nullptr;
+    for (size_t i = 0; i < count; ++i)
+      if (prev[i] == cur) next = nodes[i];
+    cur = next;
+  }
+  for (cudaGraphNode_t nd : *order) {
+    cudaGraphNodeType t;
+    if (cudaGraphNodeGetType(nd, &t) != cudaSuccess || t != cudaGraphNodeTypeKernel) return false;
+  }
+  return order->size() == count;
+}
+
+// Issues a device-driven step whose kernels all run on `s` (`launch(stream)` makes its
+// launches): the launches are recorded, and the instantiated graph of the same shape
+// (built by stream capture on first use) is launched with every kernel node's arguments
+// replaced by this step's.  A shape that cannot be captured as a chain turns the graphs
+// off for the pool, and the recorded launches are issued one by one.
+template <typename F>
+cudaError_t run_step(lv_pool* pool, cudaStream_t s, F&& launch) {
+  if (!pool->step_graphs_on) return launch(s);
+  std::vector<lv::LaunchRecord> recs;
+  lv::set_launch_recorder(&recs);
+  cudaError_t e = launch(s);
+  lv::set_launch_recorder(nullptr);
+  if (e != cudaSuccess || recs.empty()) return e;
+  lv_pool::StepGraph* g = nullptr;
+  for (auto& c : pool->step_graphs) {
+    if (c.funcs.size() != recs.size()) continue;
+    bool same = true;
+    for (size_t i = 0; i < recs.size() && same; ++i)
+      same = c.funcs[i] == recs[i].func && c.grids[i].x == recs[i].grid.x && c.grids[i].y == recs[i].grid.y &&
+             c.blocks[i].x == recs[i].block.x && c.smems[i] == recs[i].smem;
+    if (same) {
+      g = &c;
+      break;
+    }
+  }
+  if (g) {
+    for (size_t i = 0; i < recs.size(); ++i) {
+      cudaKernelNodeParams kp{};
+      kp.func = const_cast<void*>(recs[i].func);
+      kp.gridDim = recs[i].grid;
+      kp.blockDim = recs[i].block;
+      kp.sharedMemBytes = (unsigned)recs[i].smem;
+      kp.kernelParams = const_cast<void**>(recs[i].args.data());
+      e = cudaGraphExecKernelNodeSetParams(g->exec, g->nodes[i], &kp);
+      if (e != cudaSuccess) return e;
+    }
+    return cudaGraphLaunch(g->exec, s);
+  }
+  // a new shape: capture the launches on the pool's capture stream
+  lv_pool::StepGraph c;
+  bool ok = pool->step_graphs.size() < 32;
+  if (ok && !pool->s_capture) ok = cudaStreamCreateWithFlags(&pool->s_capture, cudaStreamNonBlocking) == cudaSuccess;
+  if (ok) ok = cudaStreamBeginCapture(pool->s_capture, cudaStreamCaptureModeThreadLocal) == cudaSuccess;
+  if (ok) {
+    const cudaError_t le = lv::replay_launches(recs, pool->s_capture);
+    const cudaError_t ce = cudaStreamEndCapture(pool->s_capture, &c.graph);
+    ok = le == cudaSuccess && ce == cudaSuccess && c.graph;
+  }
+  if (ok) ok = chain_nodes(c.graph, recs.size(), &c.nodes);
+  if (ok) ok = cudaGraphInstantiate(&c.exec, c.graph, 0) == cudaSuccess;
+  if (!ok) {
+    cudaGetLastError();
+    if (c.exec) cudaGraphExecDestroy(c.exec);
+    if (c.graph) cudaGraphDestroy(c.graph);
+    pool->step_graphs_on = false;
+    return lv::replay_launches(recs, s);
+  }
+  for (const auto& r : recs) {
+    c.funcs.push_back(r.func);
+    c.grids.push_back(r.grid);
+    c.blocks.push_back(r.block);
+    c.smems.push_back(r.smem);
+  }
+  pool->step_graphs.push_back(std::move(c));
+  return cudaGraphLaunch(pool->step_graphs.back().exec, s);
 }
 
 }  // namespace
@@ -1073,11 +1202,14 @@ lv_status lv_make_resident(lv_pool* pool, int32_t sid, int64_t now_us, int32_t a
     const lv::ResidentScratch* rs = nullptr;
     lv::CopyOffload off{};
     LV_TRY(next_scratch(pool, s, async, &rs, &off));
-    LV_TRY(lv::launch_make_resident(d, *rs, sid, now_us, append_tokens, preload, max_load_pages,
-                                    pool->epoch, s, pool->exchange_ctas,
-                                    static_cast<lv_resident_result*>(rdev),
-                                    timing_pair(pool, LV_TIMING_EXCHANGE), nullptr,
-                                    async ? &off : nullptr));
+    const lv::EventPair* ev = timing_pair(pool, LV_TIMING_EXCHANGE);
+    auto launch = [&](cudaStream_t cs) {
+      return lv::launch_make_resident(d, *rs, sid, now_us, append_tokens, preload, max_load_pages,
+                                      pool->epoch, cs, pool->exchange_ctas,
+                                      static_cast<lv_resident_result*>(rdev), ev, nullptr,
+                                      async ? &off : nullptr);
+    };
+    LV_TRY(async || ev ? launch(s) : run_step(pool, s, launch));
     LV_TRY(copy_resident_outputs(pool, append_tokens, victims_out, slots_out, blocks_out, pages_out,
                                  append_out, s));
     return st.finish();
@@ -1104,9 +1236,12 @@ lv_status lv_evict(lv_pool* pool, int64_t now_us, int64_t k, uint32_t flags, lv_
     lv::CopyOffload off{};
     LV_TRY(next_scratch(pool, s, async, &rs, &off));
     const int64_t kk = k < (int64_t)pool->d.budget ? k : (int64_t)pool->d.budget;
-    LV_TRY(lv::launch_evict(pool->d, *rs, now_us, kk, pool->epoch, s, pool->exchange_ctas,
-                            static_cast<lv_resident_result*>(rdev),
-                            timing_pair(pool, LV_TIMING_EXCHANGE), async ? &off : nullptr));
+    const lv::EventPair* ev = timing_pair(pool, LV_TIMING_EXCHANGE);
+    auto launch = [&](cudaStream_t cs) {
+      return lv::launch_evict(pool->d, *rs, now_us, kk, pool->epoch, cs, pool->exchange_ctas,
+                              static_cast<lv_resident_result*>(rdev), ev, async ? &off : nullptr);
+    };
+    LV_TRY(async || ev ? launch(s) : run_step(pool, s, launch));
     LV_TRY(copy_resident_outputs(pool, 0, victims_out, slots_out, nullptr, nullptr, nullptr, s));
     return st.finish();
   } catch (const std::bad_alloc&) {
@@ -1152,11 +1287,15 @@ lv_status lv_turn(lv_pool* pool, const lv_turn_desc* d, lv_victim* victims_out, 
     const lv::ResidentScratch* rs = nullptr;
     lv::CopyOffload off{};
     LV_TRY(next_scratch(pool, s, async, &rs, &off));
-    LV_TRY(lv::launch_turn(pool->d, *rs, d->sid, static_cast<const int32_t*>(cdev),
-                           d->sid == -1 ? d->num_candidates : 0, d->now_us, d->append_tokens,
-                           d->reply_audio_us, d->reply_units, pool->epoch, s, pool->exchange_ctas,
-                           static_cast<lv_resident_result*>(rdev), timing_pair(pool, LV_TIMING_EXCHANGE),
-                           async ? &off : nullptr, static_cast<const unsigned long long*>(kdev)));
+    const lv::EventPair* ev = timing_pair(pool, LV_TIMING_EXCHANGE);
+    auto launch = [&](cudaStream_t cs) {
+      return lv::launch_turn(pool->d, *rs, d->sid, static_cast<const int32_t*>(cdev),
+                             d->sid == -1 ? d->num_candidates : 0, d->now_us, d->append_tokens,
+                             d->reply_audio_us, d->reply_units, pool->epoch, cs, pool->exchange_ctas,
+                             static_cast<lv_resident_result*>(rdev), ev, async ? &off : nullptr,
+                             static_cast<const unsigned long long*>(kdev));
+    };
+    LV_TRY(async || ev ? launch(s) : run_step(pool, s, launch));
     LV_TRY(copy_resident_outputs(pool, d->append_tokens, victims_out, slots_out, blocks_out, pages_out,
                                  append_out, s, d->load_keys != nullptr));
     return st.finish();

@@ -2,6 +2,8 @@
 #pragma once
 
 #include <cstdint>
+#include <memory>
+#include <vector>
 #include <cuda_runtime.h>
 
 #include "lv.h"
@@ -141,6 +143,23 @@ cudaError_t launch_append(const DevPool& p, int32_t sid, int32_t n_tokens, int32
                           int32_t* count, cudaStream_t s, const long long* gate = nullptr,
                           const long long* sid_dev = nullptr, const struct StepFinish* fin = nullptr,
                           const long long* R = nullptr);
+
+// One kernel launch of a device-driven step, recorded instead of issued (for replay
+// through a CUDA graph): the kernel, its launch shape, whether it is a programmatic
+// dependent launch, and its argument values (`args` points into `holder`).
+struct LaunchRecord {
+  const void* func;
+  dim3 grid, block;
+  size_t smem;
+  bool pdl;
+  std::shared_ptr<void> holder;
+  std::vector<void*> args;
+};
+// While a recorder is set on the calling host thread, the step launchers append their
+// programmatic dependent launches to it instead of issuing them.
+void set_launch_recorder(std::vector<LaunchRecord>* rec);
+// Issues recorded launches on s (the same launches the launchers would have made).
+cudaError_t replay_launches(const std::vector<LaunchRecord>& recs, cudaStream_t s);
 
 // Device buffers of lv_make_resident, owned by the pool.
 struct ResidentScratch {

@@ -17,6 +17,8 @@
 // index read from memory is range-checked and a bad item is skipped with the
 // sticky error set.
 #include <cstdint>
+#include <memory>
+#include <tuple>
 #include <utility>
 
 #include "lv_internal.cuh"
@@ -2007,11 +2009,43 @@ cudaError_t launch_session_set(const DevPool& p, const lv_session_state* in, int
   return cudaGetLastError();
 }
 
+thread_local std::vector<LaunchRecord>* t_recorder = nullptr;
+
+void set_launch_recorder(std::vector<LaunchRecord>* rec) { t_recorder = rec; }
+
+cudaError_t replay_launches(const std::vector<LaunchRecord>& recs, cudaStream_t s) {
+  for (const LaunchRecord& r : recs) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = r.grid;
+    cfg.blockDim = r.block;
+    cfg.dynamicSmemBytes = r.smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = r.pdl ? 1 : 0;
+    const cudaError_t e = cudaLaunchKernelExC(&cfg, r.func, const_cast<void**>(r.args.data()));
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
 // A launch that lets the kernel be scheduled while the previous kernel on `s`
-// still runs; the kernel must begin with pdl_entry().
+// still runs; the kernel must begin with pdl_entry().  With a recorder set on this
+// thread the launch is recorded (its arguments converted to the kernel's parameter
+// types and kept) instead of issued.
 template <typename... KArgs, typename... Args>
 cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, unsigned block, size_t smem,
                        cudaStream_t s, Args&&... args) {
+  if (t_recorder) {
+    using Values = std::tuple<std::decay_t<KArgs>...>;
+    auto values = std::make_shared<Values>(std::forward<Args>(args)...);
+    LaunchRecord r{reinterpret_cast<const void*>(kernel), grid, dim3(block), smem, true, values, {}};
+    std::apply([&r](auto&... x) { (r.args.push_back(static_cast<void*>(&x)), ...); }, *values);
+    t_recorder->push_back(std::move(r));
+    return cudaSuccess;
+  }
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = grid;
   cfg.blockDim = dim3(block);
