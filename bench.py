@@ -619,21 +619,21 @@ def _restart(pool, wl):
     pool.sync()
 
 
-def _streamed_with_consumer(torch, pool, wl, moves, seed):
+def _streamed(torch, pool, wl, moves, seed, with_consumer=True):
     """The whole script issued without a host wait between events (turns and preloads
     with their copies on the pool's copy stream, each event's decisions overlapping the
-    copies before it), from the initial state, alone and then with the checksum consumer
-    kept running throughout on a stream of normal priority (the manager's calls on a
-    high-priority one).  Link fraction: the link's best time for every moving
-    event's own mix (from the event-by-event pass of the same script) over the elapsed
-    device time."""
+    copies before it), from the initial state, alone and then (``with_consumer``) with the
+    checksum consumer kept running throughout on a stream of normal priority (the
+    manager's calls on a high-priority one).  Link fraction: the link's best time for
+    every moving event's own mix (from the event-by-event pass of the same script) over
+    the elapsed device time."""
     from paper_2606_22983_gb300 import lv
     from paper_2606_22983_gb300.manager import KVManager
     from workloads import scatter_order
     best_s = moves["link_best_s"]
     out = {}
     cons = None
-    for label in ("alone", "with_consumer"):
+    for label in ("alone", "with_consumer") if with_consumer else ("alone",):
         _restart(pool, wl)
         st0 = pool.stats()
         with torch.cuda.stream(torch.cuda.Stream(device=pool.device, priority=-1)):
@@ -672,15 +672,16 @@ def _streamed_with_consumer(torch, pool, wl, moves, seed):
     return out
 
 
-def five_workloads(torch, seed, consumer_on="mixed"):
+def five_workloads(torch, seed, consumer_on="mixed", streamed=("mixed", "long", "frag")):
     """All five seeded workloads through the device driver, one event at a time
     (paper_2606_22983_gb300.runner): GB/s and link fraction overall, by event kind and
     by direction.  Mixed and frag run at their stated session counts (256, 1024) where
     the host can page-lock their host tier within min(400 GB, 0.8 * MemAvailable), else
-    scaled to it (``sizing``).  The mixed script runs a second time from the same initial
-    state with the checksum consumer reading resident KV throughout (its calls on a stream
-    of normal priority, the manager's on a high-priority one), so that its speech start
-    and barge-in preloads are measured next to serving work."""
+    scaled to it (``sizing``).  The ``streamed`` workloads run a second time from the same
+    initial state without a host wait between events (``_streamed``).  The mixed script
+    also runs with the checksum consumer reading resident KV throughout (its calls on a
+    stream of normal priority, the manager's on a high-priority one), so that its speech
+    start and barge-in preloads are measured next to serving work."""
     from paper_2606_22983_gb300.harness import fill_random, link_peaks, pool_for
     from paper_2606_22983_gb300.manager import KVManager
     from paper_2606_22983_gb300.runner import link_summary, peak_bytes, quantiles, run_events
@@ -702,8 +703,10 @@ def five_workloads(torch, seed, consumer_on="mixed"):
                  "turn_ms": quantiles(turn_ms), "wall_s": round(wall, 1),
                  "moves": link_summary(moves, peaks, EVENT_NAMES),
                  "copy_kernels": copies}
+            if name in streamed:
+                r["streamed"] = _streamed(torch, pool, wl, r["moves"], seed,
+                                          with_consumer=name == consumer_on)
             if name == consumer_on:
-                r["streamed"] = _streamed_with_consumer(torch, pool, wl, r["moves"], seed)
                 _restart(pool, wl)
                 cons = ChecksumConsumer(torch, pool, seed=seed)
                 alone = cons.alone_gbs()
