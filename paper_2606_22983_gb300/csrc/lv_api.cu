@@ -855,10 +855,12 @@ cudaError_t run_step(lv_pool* pool, cudaStream_t s, F&& launch) {
     }
     return cudaGraphLaunch(g->exec, s);
   }
-  // a new shape: capture the launches on the pool's capture stream
+  // a new shape: capture the launches on the pool's capture stream (past 32 shapes,
+  // further shapes are issued launch by launch)
+  if (pool->step_graphs.size() >= 32) return lv::replay_launches(recs, s);
   lv_pool::StepGraph c;
-  bool ok = pool->step_graphs.size() < 32;
-  if (ok && !pool->s_capture) ok = cudaStreamCreateWithFlags(&pool->s_capture, cudaStreamNonBlocking) == cudaSuccess;
+  bool ok = true;
+  if (!pool->s_capture) ok = cudaStreamCreateWithFlags(&pool->s_capture, cudaStreamNonBlocking) == cudaSuccess;
   if (ok) ok = cudaStreamBeginCapture(pool->s_capture, cudaStreamCaptureModeThreadLocal) == cudaSuccess;
   if (ok) {
     const cudaError_t le = lv::replay_launches(recs, pool->s_capture);
