@@ -900,9 +900,9 @@ __device__ __forceinline__ long long merged_task(long long k, long long n, long 
 // Unit u = (task t, sub-page j): the out half copies hbm_kv[j][page] to host[slot][j],
 // the in half host[slot'][j] to hbm_kv[j][page']; each thread loads both before it
 // stores either, so a paired task reads the old page before overwriting it.  CTAs take
-// units in order from a shared cursor (zeroed by the plan), the next one fetched while
-// the current one is copied: a CTA that starts late, or runs on an SM crowded by other
-// work, simply takes fewer units.
+// units in order from a shared cursor (zeroed by the plan; tasks in the merged order of
+// merged_task), the next one fetched while the current one is copied: a CTA that starts
+// late, or runs on an SM crowded by other work, simply takes fewer units.
 __global__ void __launch_bounds__(kCopyThreads)
 k_exchange_copy(DevPool p, const int4* __restrict__ tasks, const long long* __restrict__ n_tasks,
                 long long* __restrict__ cursor) {
