@@ -1133,8 +1133,8 @@ lv_status lv_swap_exchange(lv_pool* pool, const lv_victim* victims, int64_t n_ou
     if ((r = st.out(slots_out, (size_t)n_out * 4, &sdev, true)) != LV_OK) return r;
     if ((r = st.out(pages_out, (size_t)n_in * 4, &pdev, true)) != LV_OK) return r;
     if ((r = st.out(nullptr, (size_t)(n_out + n_in) * sizeof(int4), &tdev, true)) != LV_OK) return r;
-    // the task count, the copy kernel's cursor and the plan's count of loading tasks
-    if ((r = st.out(nullptr, 3 * sizeof(long long), &ndev, true)) != LV_OK) return r;
+    // the task count, and the copy kernel's cursor
+    if ((r = st.out(nullptr, 2 * sizeof(long long), &ndev, true)) != LV_OK) return r;
     if (++pool->epoch <= 0) pool->epoch = 1;
     if (mode == LV_MODE_STAGED) {
       LV_TRY(lv::launch_exchange_plan(pool->d, static_cast<const lv_victim*>(vin), n_out, sid,

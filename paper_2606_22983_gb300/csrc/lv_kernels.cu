@@ -687,8 +687,7 @@ enum ResWord : int {
   R_APPENDED = 7,   // int32 count of appended pages, in the low half
   R_FOUND = 8,      // victims the ranking found
   R_SID = 9,        // lv_turn: the turn's session (-1 when the pick failed)
-  R_CURSOR = 10,    // the exchange copy's next unit (zeroed by the plan)
-  R_N_IN_TASKS = 11 // the word after the cursor: the plan's number of tasks that load
+  R_CURSOR = 10     // the exchange copy's next unit (zeroed by the plan)
 };
 
 // The gate after a device-driven step's ranking, run by the exchange plan's first
@@ -867,7 +866,6 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
   }
   if (threadIdx.x == 0) {
     *n_tasks = n_in + run;
-    if (cursor) cursor[1] = n_in;   // tasks [0, n_in) load, [n_in, n_tasks) only evict
     const long long n_clean = n_out - n_dirty;
     const long long host_delta = p.incl ? n_dirty : n_dirty - n_in;
     atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_HOST_ALLOC]), (unsigned long long)host_delta);
@@ -883,32 +881,17 @@ k_exchange_plan(DevPool p, const lv_victim* __restrict__ v, long long n_out, int
   }
 }
 
-// The order in which the copy kernels take the tasks.  The plan lists the n_in tasks
-// that load (each paired with an eviction when its page was a victim's) before the tasks
-// that only evict; a step that loads and evicts unequal amounts would then run both link
-// directions for a while and one alone at the end.  The k-th task taken is instead the
-// k-th of a proportional merge of the two lists, each kept in its own order: position k
-// holds a loading task when floor((k + 1) n_in / n) steps up at k, else the next evicting
-// one.  Any order is correct (a task's two halves stay in one unit, and tasks are
-// independent).
-__device__ __forceinline__ long long merged_task(long long k, long long n, long long n_in) {
-  if (n_in <= 0 || n_in >= n) return k;
-  const long long c = (k + 1) * n_in / n, c0 = k * n_in / n;
-  return c > c0 ? c - 1 : n_in + (k - c);
-}
-
 // Unit u = (task t, sub-page j): the out half copies hbm_kv[j][page] to host[slot][j],
 // the in half host[slot'][j] to hbm_kv[j][page']; each thread loads both before it
 // stores either, so a paired task reads the old page before overwriting it.  CTAs take
-// units in order from a shared cursor (zeroed by the plan; tasks in the merged order of
-// merged_task), the next one fetched while the current one is copied: a CTA that starts
-// late, or runs on an SM crowded by other work, simply takes fewer units.
+// units in order from a shared cursor (zeroed by the plan), the next one fetched while
+// the current one is copied: a CTA that starts late, or runs on an SM crowded by other
+// work, simply takes fewer units.
 __global__ void __launch_bounds__(kCopyThreads)
 k_exchange_copy(DevPool p, const int4* __restrict__ tasks, const long long* __restrict__ n_tasks,
                 long long* __restrict__ cursor) {
   pdl_entry();
-  const long long ntask = *n_tasks, n_load = cursor[1];
-  const long long units = ntask * p.J;
+  const long long units = *n_tasks * p.J;
   const int nvec = (int)(p.P >> 4);
   __shared__ long long next;
   if (threadIdx.x == 0) next = (long long)atomicAdd(reinterpret_cast<unsigned long long*>(cursor), 1ull);
@@ -918,7 +901,7 @@ k_exchange_copy(DevPool p, const int4* __restrict__ tasks, const long long* __re
     // warp does not wait for the atomic's result meanwhile
     unsigned long long fetched = 0;
     if (threadIdx.x == 0) fetched = atomicAdd(reinterpret_cast<unsigned long long*>(cursor), 1ull);
-    const int4 t = tasks[merged_task(u / p.J, ntask, n_load)];
+    const int4 t = tasks[u / p.J];
     const int j = (int)(u % p.J);
     const bool has_out = t.x >= 0, has_in = t.z >= 0;
     const int4* so = has_out ? reinterpret_cast<const int4*>(p.kv[j] + (size_t)t.x * p.P) : nullptr;
@@ -1186,8 +1169,7 @@ k_exchange_copy_tma(DevPool p, const int4* __restrict__ tasks, const long long* 
   if (threadIdx.x != 0) return;
   const int stages = p.xstages;
   const uint32_t P = (uint32_t)p.P;
-  const long long ntask = *n_tasks, n_load = cursor[1];
-  const long long units = ntask * p.J;
+  const long long units = *n_tasks * p.J;
   for (int s = 0; s < stages; ++s) mbar_init(&bars[s], 1);
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   uint8_t* dout[kXStageMax];
@@ -1214,7 +1196,7 @@ k_exchange_copy_tma(DevPool p, const int4* __restrict__ tasks, const long long* 
     }
     const long long u = ub++;
     const int s = (int)(k % stages);
-    const int4 t = tasks[merged_task(u / p.J, ntask, n_load)];
+    const int4 t = tasks[u / p.J];
     const int j = (int)(u % p.J);
     unsigned char* so = xmem + (size_t)s * 2 * P;
     dout[s] = t.x >= 0 ? p.host + ((size_t)t.y * p.J + j) * P : nullptr;
