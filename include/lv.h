@@ -196,8 +196,10 @@ typedef struct lv_stats {
   int64_t host_pages;
   int64_t error;               /* sticky lv_status of the first device-detected error */
   int64_t error_detail;        /* index of the offending item */
-  int64_t last_select_count;   /* victims written by the last lv_select_victims */
-  int64_t last_select_total;   /* candidates it saw */
+  int64_t last_select_count;   /* victims selected by the last ranking (lv_select_victims or a
+                                  device-driven step's; 0 for a step with no deficit) */
+  int64_t last_select_total;   /* candidate blocks the last ranking that ran saw (a device-driven
+                                  step with no deficit ranks nothing and leaves it as it was) */
   /* counters of policy fallbacks and of preload outcomes (Section 6) */
   int64_t selects, victims, shortfalls, pages_out, pages_in, bytes_out, bytes_in;
   int64_t remap_entries, appended_pages, cancels, events, fallback_selects;

@@ -379,8 +379,9 @@ constexpr int kEmitScanMax = LV_EMIT_SCAN_MAX;
 
 // One CTA per session: its key and its count of HBM-resident blocks.
 __global__ void __launch_bounds__(kCensusThreads)
-k_rank_census(DevPool p, long long now_us, bool fallback) {
+k_rank_census(DevPool p, long long now_us, bool fallback, const long long* __restrict__ k_dev) {
   pdl_wait();
+  if (k_dev && *k_dev == 0) return;   // a device-driven step with no deficit ranks nothing
   const int32_t s = blockIdx.x;
   __shared__ unsigned long long key;
   if (threadIdx.x == 0) {
@@ -418,8 +419,9 @@ constexpr int kPrefixChunk = 256;   // keys staged by one CTA in shared memory
 // once: a broadcast), and adds its partial sums; the CTAs of tile 0 also add up
 // all candidates' blocks into C_RANK_TOTAL.  The census zeroed both.
 __global__ void __launch_bounds__(kPrefixTile)
-k_rank_prefix(DevPool p) {
+k_rank_prefix(DevPool p, const long long* __restrict__ k_dev) {
   pdl_wait();   // the census is complete and visible
+  if (k_dev && *k_dev == 0) return;
   __shared__ unsigned long long kc[kPrefixChunk];
   __shared__ int32_t cc[kPrefixChunk];
   __shared__ long long part[kPrefixTile / 32];
@@ -468,9 +470,20 @@ k_rank_emit(DevPool p, long long k, const long long* k_dev, bool fallback, long 
             lv_victim* __restrict__ out) {
   pdl_wait();   // the census (and the places) are complete and visible
   const int32_t sid = blockIdx.x;
+  if (k_dev) {            // k decided on the device (lv_make_resident, lv_evict)
+    k = *k_dev;
+    if (k == 0) {         // no deficit: the census did not run, nothing is selected
+      if (sid == 0 && threadIdx.x == 0) {
+        p.ctl[C_SEL_COUNT] = 0;
+        atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_SELECTS]), 1ull);
+        if (fallback) atomicAdd(reinterpret_cast<unsigned long long*>(&p.ctl[C_FALLBACK]), 1ull);
+        if (count_dev) *count_dev = 0;
+      }
+      return;
+    }
+  }
   const unsigned long long key = p.skey[sid];
   if (key == 0ull && sid != 0) return;
-  if (k_dev) k = *k_dev;   // k decided on the device (lv_make_resident)
   long long off, total;
   if (p.S > kEmitScanMax) {      // placed by k_rank_prefix
     off = key ? p.sbefore[sid] : 0;
@@ -2068,12 +2081,12 @@ cudaError_t launch_select(const DevPool& p, int64_t now_us, int64_t k, bool fall
                           lv_victim* out, long long* count_dev, cudaStream_t s, int /*num_sms*/,
                           const long long* k_dev) {
   cudaError_t e = launch_pdl(k_rank_census, (unsigned)p.S, kCensusThreads, 0, s, p, (long long)now_us,
-                             fallback);
+                             fallback, k_dev);
   if (e != cudaSuccess) return e;
   if (p.S > kEmitScanMax) {
     const dim3 grid((unsigned)((p.S + kPrefixTile - 1) / kPrefixTile),
                     (unsigned)((p.S + kPrefixChunk - 1) / kPrefixChunk));
-    e = launch_pdl(k_rank_prefix, grid, kPrefixTile, 0, s, p);
+    e = launch_pdl(k_rank_prefix, grid, kPrefixTile, 0, s, p, k_dev);
     if (e != cudaSuccess) return e;
   }
   e = launch_pdl(k_rank_emit, (unsigned)p.S, kEmitThreads, 0, s, p, (long long)k, k_dev, fallback,
