@@ -225,7 +225,12 @@ typedef struct lv_stats {
    (the TMA pack/unpack kernel, default about 48 KiB of stages per CTA and two
    CTAs per SM); LV_STAGE_KERNEL=lsu (16-byte copies instead of TMA);
    LV_REMAP_ENTRIES_PER_THREAD = 1, 2 or 4 (lv_remap's entries per thread,
-   default 1 while the GPU holds one thread per entry at once, else 2 or 4). */
+   default 1 while the GPU holds one thread per entry at once, else 2 or 4);
+   LV_EXCHANGE_KERNEL=tma (the exchange copy by TMA bulk copies, one issuing
+   thread per CTA, with LV_EXCHANGE_STAGES stages of 2P bytes, default 4);
+   LV_STEP_GRAPHS=0 (a device-driven step whose kernels all run on the caller's
+   stream is issued kernel by kernel instead of as one CUDA graph launch; the
+   results are the same). */
 lv_status lv_pool_create(const lv_pool_desc* desc, lv_stream stream, lv_pool** out);
 
 /* Waits for the pool's outstanding work on `stream`, then frees everything the
