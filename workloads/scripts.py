@@ -283,8 +283,8 @@ def _turns(spec: PoolSpec, seed: int, n_turns: int, ctx_lo: int, ctx_hi: int,
     rng = np.random.default_rng(seed)
     S, T = spec.n_sessions, spec.shape.page_tokens
     need = spec.hbm_budget_pages + spec.max_blocks
-    # Contexts are log-uniform (or uniform); draws whose total KV would fit the budget
-    # with less than one largest session to spare are redrawn, so every turn must evict.
+    # Contexts are log-uniform (or uniform); draws whose total KV exceeds the budget by
+    # less than one largest possible session are redrawn, so every turn must evict.
     for _ in range(1000):
         if ctx_dist == "log":
             raw = _log_uniform_tokens(rng, ctx_lo, ctx_hi, S)
